@@ -1,0 +1,162 @@
+"""ctypes front end of the float64 Gauss-sum oracle (test infrastructure only).
+
+``gauss_oracle.c`` is compiled with the host C compiler into
+``oracle/_build/libgauss_oracle.so`` on first use (or by ``build_oracle()``).
+Inputs are converted to contiguous float64 arrays here; all arithmetic
+happens in the C file.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import subprocess
+import threading
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_SRC = os.path.join(_HERE, "gauss_oracle.c")
+_BUILD_DIR = os.path.join(_HERE, "_build")
+_LIB_PATH = os.path.join(_BUILD_DIR, "libgauss_oracle.so")
+
+_lock = threading.Lock()
+_lib = None
+
+
+def oracle_library_path() -> str:
+    return _LIB_PATH
+
+
+def build_oracle(src: str | None = None, out: str | None = None, force: bool = False) -> str:
+    """Compile the oracle C source into a shared library and return its path.
+
+    ``src``/``out`` default to the committed oracle; tests that plant a
+    mistake in a copy of the source pass their own paths.
+    """
+    src = src or _SRC
+    out = out or _LIB_PATH
+    os.makedirs(os.path.dirname(out), exist_ok=True)
+    if (not force and os.path.exists(out)
+            and os.path.getmtime(out) >= os.path.getmtime(src)):
+        return out
+    cc = os.environ.get("CC", "gcc")
+    tmp = out + f".tmp{os.getpid()}"
+    cmd = [cc, "-O2", "-fopenmp", "-fPIC", "-shared", "-std=c11", "-o", tmp, src, "-lm"]
+    subprocess.run(cmd, check=True)
+    os.replace(tmp, out)
+    return out
+
+
+def _load(path: str | None = None):
+    global _lib
+    if path is not None:
+        lib = ctypes.CDLL(path)
+        _declare(lib)
+        return lib
+    with _lock:
+        if _lib is None:
+            lib = ctypes.CDLL(build_oracle())
+            _declare(lib)
+            _lib = lib
+    return _lib
+
+
+def _declare(lib):
+    dp = ctypes.POINTER(ctypes.c_double)
+    ip = ctypes.POINTER(ctypes.c_int64)
+    i64 = ctypes.c_int64
+    lib.gs_oracle_sum.argtypes = [dp, dp, dp, ctypes.c_double, i64, i64, i64, i64,
+                                  ip, i64, dp, dp, ctypes.c_int]
+    lib.gs_oracle_sum.restype = ctypes.c_int
+    lib.gs_oracle_grad_q.argtypes = [dp, dp, dp, ctypes.c_double, i64, i64, i64,
+                                     ip, i64, dp, dp, dp, dp, ctypes.c_int]
+    lib.gs_oracle_grad_q.restype = ctypes.c_int
+    lib.gs_oracle_max_threads.argtypes = []
+    lib.gs_oracle_max_threads.restype = ctypes.c_int
+
+
+def _f64(a, shape):
+    a = np.ascontiguousarray(np.asarray(a, dtype=np.float64)).reshape(shape)
+    return a
+
+
+def _ptr(a):
+    if a is None:
+        return None
+    ctype = ctypes.c_int64 if a.dtype == np.int64 else ctypes.c_double
+    return a.ctypes.data_as(ctypes.POINTER(ctype))
+
+
+def _threads(nthreads):
+    if nthreads is None:
+        return max(1, len(os.sched_getaffinity(0)))
+    return int(nthreads)
+
+
+def oracle_max_threads(lib_path: str | None = None) -> int:
+    return int(_load(lib_path).gs_oracle_max_threads())
+
+
+def oracle_sum(q, k, v, tau, rows=None, nthreads=None, lib_path=None):
+    """Eq. 1 in float64.  Returns (s, den) with s, den of shape (R, C).
+
+    q: (M, D), k: (N, D), v: (N, C) -- any real dtype, upcast to float64.
+    rows: optional sequence of row indices (default: all M rows).
+    den[r, c] = sum_n Phi |v[n, c]| is the scale used for relative errors.
+    """
+    q = np.asarray(q)
+    k = np.asarray(k)
+    v = np.asarray(v)
+    M, D = q.shape
+    N = k.shape[0]
+    if v.ndim == 1:
+        v = v.reshape(N, 1)
+    C = v.shape[1]
+    q64 = _f64(q, (M, D))
+    k64 = _f64(k, (N, D))
+    v64 = _f64(v, (N, C))
+    if rows is None:
+        R = M
+        rows_a = None
+    else:
+        rows_a = np.ascontiguousarray(np.asarray(rows, dtype=np.int64))
+        R = rows_a.shape[0]
+    s = np.empty((R, C), dtype=np.float64)
+    den = np.empty((R, C), dtype=np.float64)
+    rc = _load(lib_path).gs_oracle_sum(_ptr(q64), _ptr(k64), _ptr(v64), float(tau), M, N, D, C,
+                                       _ptr(rows_a), R, _ptr(s), _ptr(den), _threads(nthreads))
+    if rc != 0:
+        raise ValueError("gs_oracle_sum rejected its arguments")
+    return s, den
+
+
+def oracle_grad_q(q, k, v, tau, rows=None, nthreads=None, lib_path=None):
+    """Sec. 3 q-gradient in float64 for scalar weights.
+
+    Returns (g, s, den, den_shift): g, den, den_shift of shape (R, D), s of
+    shape (R,).
+    """
+    q = np.asarray(q)
+    k = np.asarray(k)
+    v = np.asarray(v).reshape(-1)
+    M, D = q.shape
+    N = k.shape[0]
+    q64 = _f64(q, (M, D))
+    k64 = _f64(k, (N, D))
+    v64 = _f64(v, (N,))
+    if rows is None:
+        R = M
+        rows_a = None
+    else:
+        rows_a = np.ascontiguousarray(np.asarray(rows, dtype=np.int64))
+        R = rows_a.shape[0]
+    g = np.empty((R, D), dtype=np.float64)
+    s = np.empty((R,), dtype=np.float64)
+    den = np.empty((R, D), dtype=np.float64)
+    dsh = np.empty((R, D), dtype=np.float64)
+    rc = _load(lib_path).gs_oracle_grad_q(_ptr(q64), _ptr(k64), _ptr(v64), float(tau), M, N, D,
+                                          _ptr(rows_a), R, _ptr(g), _ptr(s), _ptr(den), _ptr(dsh),
+                                          _threads(nthreads))
+    if rc != 0:
+        raise ValueError("gs_oracle_grad_q rejected its arguments")
+    return g, s, den, dsh

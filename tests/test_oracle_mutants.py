@@ -1,0 +1,90 @@
+"""The oracle's pins are strong enough to catch plausible mistakes.
+
+Each case plants one mistake in a temporary copy of ``oracle/gauss_oracle.c``
+(a dropped factor, a flipped sign, a dropped term, a wrong index or stride),
+compiles it on the CPU, and checks that at least one pin rejects it.  The
+committed oracle is never modified.
+"""
+import math
+import os
+
+import numpy as np
+import pytest
+
+from oracle import build_oracle, oracle_grad_q, oracle_sum
+from tests.paper_forms import prescale
+
+SRC = os.path.join(os.path.dirname(os.path.dirname(os.path.abspath(__file__))), "oracle",
+                   "gauss_oracle.c")
+
+MUTANTS = {
+    "dropped_half": ("exp(-0.5 * tau * sq_dist(a, b, D))", "exp(-tau * sq_dist(a, b, D))"),
+    "sign_of_difference": ("double t = a[d] - b[d];", "double t = a[d] + b[d];"),
+    "dropped_coordinate": ("for (int64_t d = 0; d < D; ++d) {\n        double t",
+                           "for (int64_t d = 0; d < D - 1; ++d) {\n        double t"),
+    "channel_index": ("sr[c] += phi * vn[c];", "sr[c] += phi * vn[0];"),
+    "value_stride": ("const double* vn = v + n * C;", "const double* vn = v + n;"),
+    "row_index": ("const double* qm = q + m * D;\n        double* sr",
+                  "const double* qm = q + r * D;\n        double* sr"),
+    "grad_sign": ("gr[d] += w * (kn[d] - qm[d]);", "gr[d] += w * (qm[d] - kn[d]);"),
+    "grad_factor": ("gr[d] *= tau;", "gr[d] *= 0.5 * tau;"),
+    "transposed_key": ("double phi = gauss_kernel(qm, k + n * D, D, tau);",
+                       "double phi = gauss_kernel(qm, k + n, D, tau);"),
+}
+
+
+def _pin_failures(lib):
+    """Run a fast subset of the pins against the library at ``lib``."""
+    fails = []
+    rng = np.random.default_rng(0)
+    # single key closed form, D=3, C=2
+    q = rng.standard_normal((3, 3))
+    k = rng.standard_normal((1, 3))
+    v = rng.standard_normal((1, 2))
+    s, _ = oracle_sum(q, k, v, 0.7, lib_path=lib)
+    for m in range(3):
+        want = math.exp(-0.35 * math.fsum((q[m] - k[0]) ** 2)) * v[0]
+        if not np.allclose(s[m], want, rtol=1e-12, atol=0):
+            fails.append("single_key")
+            break
+    # Alg. 1 route, multi-channel
+    q = rng.standard_normal((6, 4))
+    k = rng.standard_normal((9, 4))
+    v = rng.standard_normal((9, 3))
+    s, den = oracle_sum(q, k, v, 0.5, lib_path=lib)
+    if np.max(np.abs(prescale(q, k, v, 0.5) - s) / den) > 1e-10:
+        fails.append("alg1")
+    # row subset equals full evaluation
+    sub, _ = oracle_sum(q, k, v, 0.5, rows=[5, 1], lib_path=lib)
+    if not np.array_equal(sub, s[[5, 1]]):
+        fails.append("row_subset")
+    # gradient vs finite differences
+    q = rng.standard_normal((2, 3))
+    k = rng.standard_normal((8, 3))
+    v = rng.standard_normal(8)
+    g, _, _, _ = oracle_grad_q(q, k, v, 0.9, lib_path=lib)
+    h = 1e-6
+    for d in range(3):
+        qp = q[:1].copy(); qp[0, d] += h
+        qm = q[:1].copy(); qm[0, d] -= h
+        fd = (oracle_sum(qp, k, v[:, None], 0.9, lib_path=lib)[0][0, 0]
+              - oracle_sum(qm, k, v[:, None], 0.9, lib_path=lib)[0][0, 0]) / (2 * h)
+        if abs(fd - g[0, d]) > 1e-6 * (1 + abs(fd)):
+            fails.append("grad_fd")
+            break
+    return fails
+
+
+def test_committed_oracle_passes_fast_pins():
+    assert _pin_failures(None) == []
+
+
+@pytest.mark.parametrize("name", sorted(MUTANTS))
+def test_planted_mistake_is_caught(name, tmp_path):
+    old, new = MUTANTS[name]
+    src = open(SRC).read()
+    assert src.count(old) == 1, f"mutation anchor for {name} not unique"
+    mutated = tmp_path / "mutant.c"
+    mutated.write_text(src.replace(old, new))
+    lib = build_oracle(src=str(mutated), out=str(tmp_path / "libmutant.so"), force=True)
+    assert _pin_failures(lib), f"no pin caught the planted mistake {name}"

@@ -1,0 +1,302 @@
+"""Pins of the float64 oracle against facts fixed by the paper and by mathematics.
+
+None of these checks re-evaluates the oracle's own formula: each compares it
+with a closed form, a symmetry, an independent algebraic route (Alg. 1,
+Alg. 2), finite differences, a Monte-Carlo expectation or brute force.
+"""
+import json
+import math
+import os
+
+import numpy as np
+import pytest
+
+from oracle import oracle_grad_q, oracle_sum
+from tests.paper_forms import prescale, reweight
+
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden")
+
+
+def _rel(a, b, den):
+    return float(np.max(np.abs(a - b) / (den + 1e-300)))
+
+
+# ---------------------------------------------------------------- closed forms
+def test_worked_example_d1():
+    """D=1, q=0, k=1, tau=2: Phi = exp(-1) (Sec. 1 definition)."""
+    s, den = oracle_sum(np.zeros((1, 1)), np.ones((1, 1)), np.ones((1, 1)), 2.0)
+    assert s[0, 0] == pytest.approx(math.exp(-1.0), rel=1e-15)
+    assert den[0, 0] == pytest.approx(math.exp(-1.0), rel=1e-15)
+
+
+def test_single_key_closed_form():
+    """N=1: s_m = exp(-tau/2 ||q_m - k||^2) v (Eq. 1 with one term)."""
+    rng = np.random.default_rng(3)
+    q = rng.standard_normal((5, 7))
+    k = rng.standard_normal((1, 7))
+    v = rng.standard_normal((1, 3))
+    tau = 0.37
+    s, _ = oracle_sum(q, k, v, tau)
+    for m in range(5):
+        d2 = math.fsum((q[m, d] - k[0, d]) ** 2 for d in range(7))
+        want = math.exp(-tau * d2 / 2.0) * v[0]
+        np.testing.assert_allclose(s[m], want, rtol=1e-14, atol=0)
+
+
+def test_tau_to_zero_gives_plain_sum():
+    """tau -> 0: Phi -> 1, so s_m = sum_n v_n for every m."""
+    rng = np.random.default_rng(4)
+    q = rng.standard_normal((6, 4))
+    k = rng.standard_normal((50, 4))
+    v = rng.standard_normal((50, 2))
+    s, den = oracle_sum(q, k, v, 1e-30)
+    want = np.array([math.fsum(v[:, c]) for c in range(2)])
+    np.testing.assert_allclose(s, np.broadcast_to(want, s.shape), rtol=1e-13, atol=1e-14)
+    np.testing.assert_allclose(den, np.broadcast_to(np.abs(v).sum(0), den.shape), rtol=1e-13)
+
+
+def test_identical_keys():
+    """k_n = k for all n: s_m = Phi(q_m, k) sum_n v_n."""
+    rng = np.random.default_rng(5)
+    q = rng.standard_normal((4, 3))
+    k1 = rng.standard_normal(3)
+    k = np.tile(k1, (9, 1))
+    v = rng.standard_normal((9, 1))
+    tau = 1.3
+    s, _ = oracle_sum(q, k, v, tau)
+    for m in range(4):
+        phi = math.exp(-tau / 2 * math.fsum((q[m] - k1) ** 2))
+        assert s[m, 0] == pytest.approx(phi * math.fsum(v[:, 0]), rel=1e-13)
+
+
+def test_separable_lattice_factorises():
+    """Keys on a product grid G^D with unit weights: the Gauss kernel
+    factorises over coordinates, so s(q) = prod_d sum_{g in G} exp(-tau/2 (q_d - g)^2).
+    A dropped coordinate, a wrong index or a wrong factor breaks the product."""
+    G = np.array([-1.5, -0.2, 0.4, 1.1])
+    D = 3
+    grid = np.array(np.meshgrid(*([G] * D), indexing="ij")).reshape(D, -1).T
+    rng = np.random.default_rng(6)
+    q = rng.standard_normal((5, D))
+    tau = 0.8
+    s, _ = oracle_sum(q, grid, np.ones((grid.shape[0], 1)), tau)
+    for m in range(5):
+        want = 1.0
+        for d in range(D):
+            want *= math.fsum(math.exp(-tau / 2 * (q[m, d] - g) ** 2) for g in G)
+        assert s[m, 0] == pytest.approx(want, rel=1e-13)
+
+
+# ---------------------------------------------------------------- symmetry
+def test_kernel_matrix_symmetry():
+    """Phi(q,k) = Phi(k,q): with one-hot values the oracle returns the kernel
+    matrix, and swapping the roles of q and k transposes it."""
+    rng = np.random.default_rng(7)
+    q = rng.standard_normal((6, 4))
+    k = rng.standard_normal((9, 4))
+    Kqk, _ = oracle_sum(q, k, np.eye(9), 0.6)
+    Kkq, _ = oracle_sum(k, q, np.eye(6), 0.6)
+    np.testing.assert_allclose(Kqk, Kkq.T, rtol=1e-14, atol=0)
+    assert np.all(Kqk > 0) and np.all(Kqk <= 1.0)
+
+
+def test_unit_weight_total_symmetry():
+    """M = N, C = 1, unit weights: 1^T s(q,k) = 1^T s(k,q)."""
+    rng = np.random.default_rng(8)
+    q = rng.standard_normal((40, 5))
+    k = rng.standard_normal((40, 5))
+    a, _ = oracle_sum(q, k, np.ones((40, 1)), 0.9)
+    b, _ = oracle_sum(k, q, np.ones((40, 1)), 0.9)
+    assert math.fsum(a[:, 0]) == pytest.approx(math.fsum(b[:, 0]), rel=1e-13)
+
+
+# ---------------------------------------------------------------- algebraic routes
+@pytest.mark.parametrize("M,N,D,C,tau", [(7, 11, 3, 1, 1.0), (16, 40, 8, 5, 0.25),
+                                         (5, 64, 32, 3, 1.0 / 32), (9, 13, 1, 2, 3.0)])
+def test_alg1_prescale_matches(M, N, D, C, tau):
+    """Alg. 1: Att(q,k,v~) exp(lse) exp(-tau/2||q||^2) with v~ = v exp(-tau/2||k||^2)."""
+    rng = np.random.default_rng(M * 1000 + N)
+    q = rng.standard_normal((M, D))
+    k = rng.standard_normal((N, D))
+    v = rng.standard_normal((N, C))
+    s, den = oracle_sum(q, k, v, tau)
+    assert _rel(prescale(q, k, v, tau), s, den) < 1e-10
+
+
+@pytest.mark.parametrize("M,N,D,C,tau", [(7, 11, 3, 1, 1.0), (16, 40, 8, 5, 0.25),
+                                         (5, 64, 32, 3, 1.0 / 32), (9, 13, 1, 2, 3.0)])
+def test_alg2_reweight_and_prop1(M, N, D, C, tau):
+    """Alg. 2 reproduces the sum, and Prop. 1's bounds hold:
+    kappa/(N+1) <= beta_m <= kappa and ||alpha_m||_inf <= max_n ||v_n||_inf."""
+    rng = np.random.default_rng(M * 7 + N)
+    q = rng.standard_normal((M, D))
+    k = rng.standard_normal((N, D))
+    v = rng.standard_normal((N, C))
+    s_rw, alpha, beta, kappa = reweight(q, k, v, tau, return_parts=True)
+    s, den = oracle_sum(q, k, v, tau)
+    assert _rel(s_rw, s, den) < 1e-10
+    assert np.all(beta <= kappa * (1 + 1e-14))
+    assert np.all(beta >= kappa / (N + 1) * (1 - 1e-14))
+    assert np.max(np.abs(alpha)) <= np.max(np.abs(v)) * (1 + 1e-14)
+    # The proof's closed form: beta_m = kappa / (1 + sum_n Phi(q_m, k_n)).
+    ones, _ = oracle_sum(q, k, np.ones((N, 1)), tau)
+    np.testing.assert_allclose(beta, kappa / (1.0 + ones[:, 0]), rtol=1e-12)
+
+
+# ---------------------------------------------------------------- gradient
+def test_gradient_matches_finite_differences():
+    """Sec. 3 q-gradient vs central differences of the oracle's own s."""
+    rng = np.random.default_rng(9)
+    M, N, D = 4, 30, 5
+    q = rng.standard_normal((M, D))
+    k = rng.standard_normal((N, D))
+    v = rng.standard_normal((N, 1))
+    tau = 0.7
+    g, s, den, dsh = oracle_grad_q(q, k, v, tau)
+    s_ref, _ = oracle_sum(q, k, v, tau)
+    np.testing.assert_allclose(s, s_ref[:, 0], rtol=1e-14)
+    h = 1e-6
+    for m in range(M):
+        for d in range(D):
+            qp = q.copy(); qp[m, d] += h
+            qm = q.copy(); qm[m, d] -= h
+            sp, _ = oracle_sum(qp[m:m + 1], k, v, tau)
+            sm, _ = oracle_sum(qm[m:m + 1], k, v, tau)
+            fd = (sp[0, 0] - sm[0, 0]) / (2 * h)
+            assert abs(fd - g[m, d]) <= 1e-7 * (1 + abs(g[m, d]))
+    assert np.all(dsh >= np.abs(g) * (1 - 1e-12))
+
+
+def test_gradient_error_scale_definition():
+    """den of the gradient is tau(sum Phi|v||k_d-mu_d| + |q_d-mu_d| sum Phi|v|)
+    with mu the mean of all points; checked by brute force."""
+    rng = np.random.default_rng(10)
+    q = rng.standard_normal((3, 2)) + 2.0
+    k = rng.standard_normal((4, 2)) - 1.0
+    v = rng.standard_normal(4)
+    tau = 0.5
+    g, s, den, dsh = oracle_grad_q(q, k, v, tau)
+    mu = np.concatenate([q, k]).mean(0)
+    for m in range(3):
+        phi = [math.exp(-tau / 2 * math.fsum((q[m] - k[n]) ** 2)) for n in range(4)]
+        absw = math.fsum(phi[n] * abs(v[n]) for n in range(4))
+        for d in range(2):
+            want = tau * (math.fsum(phi[n] * abs(v[n]) * abs(k[n, d] - mu[d]) for n in range(4))
+                          + abs(q[m, d] - mu[d]) * absw)
+            assert den[m, d] == pytest.approx(want, rel=1e-13)
+            gw = tau * math.fsum(phi[n] * v[n] * (k[n, d] - q[m, d]) for n in range(4))
+            assert g[m, d] == pytest.approx(gw, rel=1e-12, abs=1e-15)
+
+
+def test_gradient_as_augmented_gauss_sum():
+    """Sec. 3: the gradient is one Gauss sum with values (v_n k_n, v_n):
+    g = tau (S[:D] - q_m S[D])."""
+    rng = np.random.default_rng(11)
+    q = rng.standard_normal((5, 3))
+    k = rng.standard_normal((20, 3))
+    v = rng.standard_normal(20)
+    tau = 1.1
+    g, s, _, _ = oracle_grad_q(q, k, v, tau)
+    aug = np.concatenate([v[:, None] * k, v[:, None]], axis=1)
+    S, _ = oracle_sum(q, k, aug, tau)
+    want = tau * (S[:, :3] - q * S[:, 3:4])
+    np.testing.assert_allclose(g, want, rtol=1e-10, atol=1e-13)
+
+
+# ---------------------------------------------------------------- MMD invariants
+def test_mmd_nonnegative_and_zero_for_equal_samples():
+    """Sec. 3: MMD^2 = sum_m v_m s_m with q = k is >= 0 (positive-definite
+    kernel) and is 0 when the two signed halves sit on the same points."""
+    rng = np.random.default_rng(12)
+    X = rng.standard_normal((30, 4))
+    v = np.concatenate([np.full(15, 1 / 15), np.full(15, -1 / 15)])[:, None]
+    s, _ = oracle_sum(X, X, v, 0.5)
+    assert float(v[:, 0] @ s[:, 0]) > 0
+    Y = np.concatenate([X[:15], X[:15]])
+    s2, den2 = oracle_sum(Y, Y, v, 0.5)
+    assert abs(float(v[:, 0] @ s2[:, 0])) < 1e-15
+    assert np.max(np.abs(s2)) < 1e-15
+
+
+# ---------------------------------------------------------------- statistics
+def test_gaussian_expectation_monte_carlo():
+    """For k ~ N(0, sigma^2 I_D): E Phi(q, k) = (1+tau sigma^2)^(-D/2)
+    exp(-tau ||q||^2 / (2 (1 + tau sigma^2))).  The oracle's mean over many
+    keys must agree within Monte-Carlo error."""
+    rng = np.random.default_rng(13)
+    D, N, sigma, tau = 3, 200000, 0.8, 1.2
+    q = np.array([[0.3, -0.5, 0.9], [0.0, 0.0, 0.0]])
+    k = sigma * rng.standard_normal((N, D))
+    ones = np.ones((N, 1))
+    s, _ = oracle_sum(q, k, ones, tau, nthreads=2)
+    a = 1.0 + tau * sigma ** 2
+    for m in range(2):
+        want = a ** (-D / 2) * math.exp(-tau * float(q[m] @ q[m]) / (2 * a))
+        # Phi in (0, 1]; its standard deviation is below 0.5.
+        assert abs(s[m, 0] / N - want) < 5 * 0.5 / math.sqrt(N)
+
+
+# ---------------------------------------------------------------- brute force
+def test_brute_force_tiny():
+    """Tiny inputs expanded by hand with math.exp / math.fsum."""
+    rng = np.random.default_rng(14)
+    for M, N, D, C in [(1, 1, 1, 1), (2, 3, 2, 1), (4, 4, 3, 2), (3, 2, 1, 3)]:
+        q = rng.standard_normal((M, D))
+        k = rng.standard_normal((N, D))
+        v = rng.standard_normal((N, C))
+        tau = float(rng.uniform(0.1, 2.0))
+        s, den = oracle_sum(q, k, v, tau)
+        for m in range(M):
+            for c in range(C):
+                terms = []
+                absterms = []
+                for n in range(N):
+                    if D == 1:
+                        d2 = (q[m, 0] - k[n, 0]) ** 2
+                    elif D == 2:
+                        d2 = (q[m, 0] - k[n, 0]) ** 2 + (q[m, 1] - k[n, 1]) ** 2
+                    else:
+                        d2 = ((q[m, 0] - k[n, 0]) ** 2 + (q[m, 1] - k[n, 1]) ** 2
+                              + (q[m, 2] - k[n, 2]) ** 2)
+                    terms.append(math.exp(-0.5 * tau * d2) * v[n, c])
+                    absterms.append(math.exp(-0.5 * tau * d2) * abs(v[n, c]))
+                assert abs(s[m, c] - math.fsum(terms)) <= 1e-14 * (1 + math.fsum(absterms))
+                assert den[m, c] == pytest.approx(math.fsum(absterms), rel=1e-14)
+
+
+# ---------------------------------------------------------------- golden values
+def test_golden_fixtures():
+    """Small hand-checkable fixtures stored under tests/golden/, each with the
+    passage it follows; expected values are closed forms written out there."""
+    with open(os.path.join(GOLDEN, "closed_forms.json")) as f:
+        cases = json.load(f)
+    assert len(cases) >= 3
+    for case in cases:
+        q = np.array(case["q"], dtype=np.float64)
+        k = np.array(case["k"], dtype=np.float64)
+        v = np.array(case["v"], dtype=np.float64)
+        s, _ = oracle_sum(q, k, v, case["tau"])
+        np.testing.assert_allclose(s, np.array(case["s"]), rtol=1e-13, atol=1e-300,
+                                   err_msg=case["cite"])
+
+
+# ---------------------------------------------------------------- plumbing
+def test_row_subset_and_thread_count_invariance():
+    rng = np.random.default_rng(15)
+    q = rng.standard_normal((50, 6))
+    k = rng.standard_normal((70, 6))
+    v = rng.standard_normal((70, 2))
+    full, fden = oracle_sum(q, k, v, 0.4, nthreads=1)
+    rows = np.array([49, 0, 17, 17, 3])
+    sub, sden = oracle_sum(q, k, v, 0.4, rows=rows, nthreads=3)
+    np.testing.assert_array_equal(sub, full[rows])
+    np.testing.assert_array_equal(sden, fden[rows])
+    full4, _ = oracle_sum(q, k, v, 0.4, nthreads=4)
+    np.testing.assert_array_equal(full4, full)
+
+
+def test_empty_and_rejected_inputs():
+    s, den = oracle_sum(np.zeros((3, 2)), np.zeros((0, 2)), np.zeros((0, 1)), 1.0)
+    assert np.all(s == 0) and s.shape == (3, 1)
+    with pytest.raises(ValueError):
+        oracle_sum(np.zeros((3, 2)), np.zeros((4, 2)), np.zeros((4, 1)), 1.0, rows=[3])
