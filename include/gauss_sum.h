@@ -1,0 +1,148 @@
+/*
+ * gauss_sum.h -- C ABI of the GB300 (sm_103a) Gauss kernel sum library.
+ *
+ * The library evaluates the Gauss kernel sum of arXiv 2609.04910, Sec. 1,
+ * Eq. 1:
+ *
+ *     s_m = sum_{n=1..N} exp(-tau/2 * ||q_m - k_n||^2) * v_n  in R^C,
+ *                                                      m = 1..M,
+ *
+ * for query points q (M x D), key points k (N x D), signed values v (N x C)
+ * and bandwidth tau > 0, and the gradient of s_m with respect to q_m for
+ * scalar weights (Sec. 3, MMD flows and SVGD):
+ *
+ *     grad_m = tau * ( sum_n Phi(q_m,k_n) v_n k_n  -  q_m sum_n Phi(q_m,k_n) v_n ),
+ *
+ * which the library evaluates as one Gauss sum with the augmented values
+ * (v_n k_n, v_n) in R^{D+1}.
+ *
+ * Conventions shared by every entry point:
+ *  - Array arguments are DEVICE pointers to contiguous row-major arrays,
+ *    owned by the caller and not retained after the call returns.  q, k and
+ *    v share one element type (gs_dtype); q may alias k (the MMD form q = k
+ *    of Sec. 3).  Outputs are float32 and are overwritten, not accumulated.
+ *  - Base pointers must be 16-byte aligned.
+ *  - `stream` is a cudaStream_t passed as void* (NULL: the legacy default
+ *    stream).  Calls are asynchronous and stream ordered; the status return
+ *    covers argument checks, allocation and launch errors.  A device-side
+ *    wait that runs out of time is reported by gauss_sum_device_status().
+ *  - Without a caller workspace the library allocates its workspace with
+ *    cudaMallocAsync on `stream` and frees it with cudaFreeAsync on the same
+ *    stream.
+ *  - M = 0 is a no-op; N = 0 writes zeros.
+ *  - fp16/bf16 inputs run on the tensor-core kernel (tcgen05, sm_103a) and
+ *    need D <= 256 and C <= 256 (grad: D + 1 <= 256).  fp32 inputs run on
+ *    the fp32 SIMT kernel (D <= 128 forward, D <= 64 gradient, any C).
+ *  - On a non-OK return gauss_sum_last_error() describes the failure.
+ */
+#ifndef GAUSS_SUM_H
+#define GAUSS_SUM_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* Element type of q, k and v. */
+typedef enum { GS_FP32 = 0, GS_FP16 = 1, GS_BF16 = 2 } gs_dtype;
+
+typedef enum {
+    GS_OK = 0,
+    GS_ERR_INVALID_ARGUMENT = 1, /* null pointer, negative size, bad tau, misalignment */
+    GS_ERR_UNSUPPORTED = 2,      /* shape or dtype outside the supported range, or no sm_103 GPU */
+    GS_ERR_OUT_OF_MEMORY = 3,    /* workspace allocation failed / caller workspace too small */
+    GS_ERR_CUDA = 4,             /* a CUDA runtime call or a kernel launch failed */
+    GS_ERR_DEVICE_TIMEOUT = 5    /* a bounded device-side wait ran out (see device_status) */
+} gs_status;
+
+/* Which kernel family evaluates the sum. */
+typedef enum { GS_PATH_AUTO = 0, GS_PATH_TENSOR = 1, GS_PATH_SIMT = 2 } gs_path;
+
+/*
+ * Options of the _ex entry points.  Initialise with gauss_sum_default_options.
+ *  center          1: shift q and k by their common mean before rounding to
+ *                     the MMA type (the overflow/cancellation safeguard of
+ *                     Remark 3, Sec. 2); 0: use the raw points.
+ *  split_n         number of key splits per row tile (0: chosen from the
+ *                  SM count); partial sums over splits are added in a fixed
+ *                  order, so results are deterministic for a fixed split.
+ *  workspace       caller-owned device buffer of workspace_bytes bytes
+ *                  (256-byte aligned) used instead of an allocation; its
+ *                  required size is gauss_sum_workspace_size().
+ *  path            GS_PATH_AUTO picks the tensor-core kernel for fp16/bf16
+ *                  and the SIMT kernel for fp32; GS_PATH_TENSOR rejects fp32,
+ *                  GS_PATH_SIMT rejects fp16/bf16.
+ */
+typedef struct gs_options {
+    int center;
+    int split_n;
+    void* workspace;
+    size_t workspace_bytes;
+    int path;
+} gs_options;
+
+/* Fill *opt with the defaults (center = 1, split_n = 0, no workspace, auto path). */
+void gauss_sum_default_options(gs_options* opt);
+
+/*
+ * Eq. 1.  q: M x D, k: N x D, v: N x C (all `dtype`); out: M x C float32.
+ */
+gs_status gauss_sum(const void* q, const void* k, const void* v, double tau, int64_t M,
+                    int64_t N, int64_t D, int64_t C, gs_dtype dtype, float* out, void* stream);
+
+/* Eq. 1 with options (opt may be NULL for the defaults). */
+gs_status gauss_sum_ex(const void* q, const void* k, const void* v, double tau, int64_t M,
+                       int64_t N, int64_t D, int64_t C, gs_dtype dtype, float* out,
+                       void* stream, const gs_options* opt);
+
+/*
+ * q-gradient of Sec. 3 for scalar weights: v is N x 1.
+ * grad: M x D float32, grad[m] = d/dq_m sum_n Phi(q_m, k_n) v_n.
+ * s_out: M x 1 float32 forward sum s_m, or NULL.
+ */
+gs_status gauss_sum_grad_q(const void* q, const void* k, const void* v, double tau, int64_t M,
+                           int64_t N, int64_t D, gs_dtype dtype, float* grad, float* s_out,
+                           void* stream);
+
+gs_status gauss_sum_grad_q_ex(const void* q, const void* k, const void* v, double tau,
+                              int64_t M, int64_t N, int64_t D, gs_dtype dtype, float* grad,
+                              float* s_out, void* stream, const gs_options* opt);
+
+/*
+ * Workspace bytes that gauss_sum_ex (grad = 0, C channels) or
+ * gauss_sum_grad_q_ex (grad = 1, C ignored) needs for these sizes and
+ * options (opt may be NULL).  Returns 0 for a no-op call and (size_t)-1 for
+ * arguments the call would reject.
+ */
+size_t gauss_sum_workspace_size(int64_t M, int64_t N, int64_t D, int64_t C, gs_dtype dtype,
+                                int grad, const gs_options* opt);
+
+/*
+ * Synchronise `stream`, then return and clear the device status word of the
+ * current device: GS_OK, or GS_ERR_DEVICE_TIMEOUT if a kernel gave up a
+ * bounded wait since the last call (its outputs are then invalid), or
+ * GS_ERR_CUDA if the synchronisation itself failed.
+ */
+gs_status gauss_sum_device_status(void* stream);
+
+/* Description of the last non-OK status returned on this host thread. */
+const char* gauss_sum_last_error(void);
+
+/* Static name of a status code. */
+const char* gauss_sum_status_string(gs_status status);
+
+/*
+ * Measurement helper (not part of Eq. 1): sustained MUFU exp2 throughput of
+ * the current device in exponentials per second, measured with CUDA events
+ * by a kernel of independent ex2.approx chains on every SM.  Synchronises
+ * `stream`.  Used as the SFU roofline of the fused kernel.
+ */
+gs_status gauss_sum_probe_ex2_rate(void* stream, double* exp2_per_second);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* GAUSS_SUM_H */

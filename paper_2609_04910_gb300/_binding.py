@@ -1,0 +1,207 @@
+"""Thin ctypes binding of the C ABI in ``include/gauss_sum.h``.
+
+Only argument marshalling happens here: torch tensors are reduced to device
+pointers, sizes, a dtype code and the current CUDA stream, and every step of
+the computation runs in the library's CUDA kernels.  There is no fallback:
+if ``libgauss_sum.so`` has not been built, every call raises.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import threading
+
+from .build import LIB_PATH
+
+GS_FP32, GS_FP16, GS_BF16 = 0, 1, 2
+GS_PATH_AUTO, GS_PATH_TENSOR, GS_PATH_SIMT = 0, 1, 2
+STATUS_NAMES = {
+    0: "GS_OK", 1: "GS_ERR_INVALID_ARGUMENT", 2: "GS_ERR_UNSUPPORTED",
+    3: "GS_ERR_OUT_OF_MEMORY", 4: "GS_ERR_CUDA", 5: "GS_ERR_DEVICE_TIMEOUT",
+}
+
+# Every symbol include/gauss_sum.h declares.
+EXPORTS = (
+    "gauss_sum_default_options", "gauss_sum", "gauss_sum_ex", "gauss_sum_grad_q",
+    "gauss_sum_grad_q_ex", "gauss_sum_workspace_size", "gauss_sum_device_status",
+    "gauss_sum_last_error", "gauss_sum_status_string", "gauss_sum_probe_ex2_rate",
+)
+
+
+class GaussSumError(RuntimeError):
+    def __init__(self, status: int, message: str):
+        super().__init__(f"{STATUS_NAMES.get(status, status)}: {message}")
+        self.status = status
+        self.message = message
+
+
+class GsOptions(ctypes.Structure):
+    _fields_ = [("center", ctypes.c_int), ("split_n", ctypes.c_int),
+                ("workspace", ctypes.c_void_p), ("workspace_bytes", ctypes.c_size_t),
+                ("path", ctypes.c_int)]
+
+
+_lock = threading.Lock()
+_lib = None
+
+
+def library_path() -> str:
+    return LIB_PATH
+
+
+def load_library(path: str | None = None):
+    """Load (once) and return the ctypes handle of libgauss_sum.so."""
+    global _lib
+    with _lock:
+        if _lib is not None and path is None:
+            return _lib
+        p = path or LIB_PATH
+        if not os.path.exists(p):
+            raise RuntimeError(
+                f"{p} is missing: build the CUDA library first "
+                "(python -m paper_2609_04910_gb300.build or __graft_entry__.build())")
+        lib = ctypes.CDLL(p)
+        _declare(lib)
+        if path is None:
+            _lib = lib
+        return lib
+
+
+def _declare(lib):
+    vp, i64, f = ctypes.c_void_p, ctypes.c_int64, ctypes.c_int
+    d = ctypes.c_double
+    lib.gauss_sum_default_options.argtypes = [ctypes.POINTER(GsOptions)]
+    lib.gauss_sum_default_options.restype = None
+    lib.gauss_sum.argtypes = [vp, vp, vp, d, i64, i64, i64, i64, f, vp, vp]
+    lib.gauss_sum.restype = f
+    lib.gauss_sum_ex.argtypes = [vp, vp, vp, d, i64, i64, i64, i64, f, vp, vp,
+                                 ctypes.POINTER(GsOptions)]
+    lib.gauss_sum_ex.restype = f
+    lib.gauss_sum_grad_q.argtypes = [vp, vp, vp, d, i64, i64, i64, f, vp, vp, vp]
+    lib.gauss_sum_grad_q.restype = f
+    lib.gauss_sum_grad_q_ex.argtypes = [vp, vp, vp, d, i64, i64, i64, f, vp, vp, vp,
+                                        ctypes.POINTER(GsOptions)]
+    lib.gauss_sum_grad_q_ex.restype = f
+    lib.gauss_sum_workspace_size.argtypes = [i64, i64, i64, i64, f, f, ctypes.POINTER(GsOptions)]
+    lib.gauss_sum_workspace_size.restype = ctypes.c_size_t
+    lib.gauss_sum_device_status.argtypes = [vp]
+    lib.gauss_sum_device_status.restype = f
+    lib.gauss_sum_last_error.argtypes = []
+    lib.gauss_sum_last_error.restype = ctypes.c_char_p
+    lib.gauss_sum_status_string.argtypes = [f]
+    lib.gauss_sum_status_string.restype = ctypes.c_char_p
+    lib.gauss_sum_probe_ex2_rate.argtypes = [vp, ctypes.POINTER(ctypes.c_double)]
+    lib.gauss_sum_probe_ex2_rate.restype = f
+
+
+def _check(lib, status: int):
+    if status != 0:
+        raise GaussSumError(status, lib.gauss_sum_last_error().decode())
+
+
+def options(center=True, split_n=0, workspace=None, workspace_bytes=0, path=GS_PATH_AUTO):
+    o = GsOptions()
+    load_library().gauss_sum_default_options(ctypes.byref(o))
+    o.center = 1 if center else 0
+    o.split_n = int(split_n)
+    o.workspace = workspace
+    o.workspace_bytes = int(workspace_bytes)
+    o.path = int(path)
+    return o
+
+
+def _dtype_code(t):
+    import torch
+    if t.dtype == torch.float32:
+        return GS_FP32
+    if t.dtype == torch.float16:
+        return GS_FP16
+    if t.dtype == torch.bfloat16:
+        return GS_BF16
+    raise TypeError(f"unsupported dtype {t.dtype}")
+
+
+def _stream_ptr(stream):
+    import torch
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return ctypes.c_void_p(stream.cuda_stream)
+
+
+def _ptr(t):
+    return None if t is None else ctypes.c_void_p(t.data_ptr())
+
+
+def _check_tensor(t, name):
+    if not t.is_cuda:
+        raise ValueError(f"{name} must be a CUDA tensor")
+    if not t.is_contiguous():
+        raise ValueError(f"{name} must be contiguous")
+
+
+def gauss_sum(q, k, v, tau, out=None, stream=None, center=True, split_n=0, workspace=None):
+    """Eq. 1: s[m] = sum_n exp(-tau/2 ||q_m - k_n||^2) v[n] as an (M, C) fp32 tensor.
+
+    q: (M, D), k: (N, D), v: (N, C) or (N,) CUDA tensors of one dtype
+    (fp32, fp16 or bf16).  ``q`` may be the same tensor as ``k``.
+    """
+    import torch
+    lib = load_library()
+    for t, n in ((q, "q"), (k, "k"), (v, "v")):
+        _check_tensor(t, n)
+    M, D = q.shape
+    N = k.shape[0]
+    C = 1 if v.dim() == 1 else v.shape[1]
+    if out is None:
+        out = torch.empty((M, C), dtype=torch.float32, device=q.device)
+    opt = options(center=center, split_n=split_n,
+                  workspace=None if workspace is None else workspace.data_ptr(),
+                  workspace_bytes=0 if workspace is None else workspace.numel() * workspace.element_size())
+    st = lib.gauss_sum_ex(_ptr(q), _ptr(k), _ptr(v), float(tau), M, N, D, C, _dtype_code(q),
+                          _ptr(out), _stream_ptr(stream), ctypes.byref(opt))
+    _check(lib, st)
+    return out
+
+
+def gauss_sum_grad_q(q, k, v, tau, grad=None, s_out=None, want_s=True, stream=None,
+                     center=True, split_n=0, workspace=None):
+    """Sec. 3 q-gradient for scalar weights.  Returns (grad (M, D), s (M,) or None)."""
+    import torch
+    lib = load_library()
+    for t, n in ((q, "q"), (k, "k"), (v, "v")):
+        _check_tensor(t, n)
+    M, D = q.shape
+    N = k.shape[0]
+    if grad is None:
+        grad = torch.empty((M, D), dtype=torch.float32, device=q.device)
+    if s_out is None and want_s:
+        s_out = torch.empty((M,), dtype=torch.float32, device=q.device)
+    opt = options(center=center, split_n=split_n,
+                  workspace=None if workspace is None else workspace.data_ptr(),
+                  workspace_bytes=0 if workspace is None else workspace.numel() * workspace.element_size())
+    st = lib.gauss_sum_grad_q_ex(_ptr(q), _ptr(k), _ptr(v), float(tau), M, N, D, _dtype_code(q),
+                                 _ptr(grad), _ptr(s_out), _stream_ptr(stream), ctypes.byref(opt))
+    _check(lib, st)
+    return grad, s_out
+
+
+def gauss_sum_workspace_size(M, N, D, C, dtype_code, grad=False, center=True, split_n=0):
+    lib = load_library()
+    opt = options(center=center, split_n=split_n)
+    return int(lib.gauss_sum_workspace_size(M, N, D, C, dtype_code, 1 if grad else 0,
+                                            ctypes.byref(opt)))
+
+
+def gauss_sum_device_status(stream=None):
+    """Synchronise and return (and clear) the device status; raises on a timeout."""
+    lib = load_library()
+    st = lib.gauss_sum_device_status(_stream_ptr(stream))
+    _check(lib, st)
+    return st
+
+
+def gauss_sum_probe_ex2_rate(stream=None) -> float:
+    lib = load_library()
+    r = ctypes.c_double(0.0)
+    _check(lib, lib.gauss_sum_probe_ex2_rate(_stream_ptr(stream), ctypes.byref(r)))
+    return r.value

@@ -1,0 +1,418 @@
+// C ABI of the Gauss-sum library: argument checks, workspace handling,
+// kernel sequencing and error reporting.  See include/gauss_sum.h.
+#include <cuda_runtime.h>
+
+#include <cmath>
+#include <cstdio>
+#include <cstdlib>
+#include <cstring>
+#include <mutex>
+
+#include "gauss_sum.h"
+#include "internal.h"
+#include "ptx.cuh"
+
+namespace {
+
+thread_local char g_last_error[512] = "no error";
+
+gs_status fail(gs_status st, const char* fmt, const char* detail = nullptr) {
+    if (detail)
+        std::snprintf(g_last_error, sizeof(g_last_error), fmt, detail);
+    else
+        std::snprintf(g_last_error, sizeof(g_last_error), "%s", fmt);
+    return st;
+}
+
+gs_status cuda_fail(cudaError_t e, const char* where) {
+    char buf[256];
+    std::snprintf(buf, sizeof(buf), "%s: %s", where, cudaGetErrorString(e));
+    return fail(e == cudaErrorMemoryAllocation ? GS_ERR_OUT_OF_MEMORY : GS_ERR_CUDA, "%s", buf);
+}
+
+// Device status word: a kernel that gives up a bounded wait records the
+// reason here; gauss_sum_device_status() reads and clears it.
+__device__ unsigned g_device_status = 0;
+
+constexpr int kMaxDevices = 64;
+std::mutex g_dev_mu;
+unsigned* g_status_ptr[kMaxDevices] = {};
+int g_sm_count[kMaxDevices] = {};
+int g_is_sm103[kMaxDevices] = {};  // 0 unknown, 1 yes, 2 no
+
+cudaError_t device_info(int* dev, unsigned** status) {
+    cudaError_t e = cudaGetDevice(dev);
+    if (e != cudaSuccess) return e;
+    if (*dev < 0 || *dev >= kMaxDevices) return cudaErrorInvalidDevice;
+    std::lock_guard<std::mutex> lk(g_dev_mu);
+    if (!g_status_ptr[*dev]) {
+        void* p = nullptr;
+        e = cudaGetSymbolAddress(&p, g_device_status);
+        if (e != cudaSuccess) return e;
+        int sms = 0, major = 0, minor = 0;
+        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, *dev);
+        cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, *dev);
+        cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, *dev);
+        g_sm_count[*dev] = sms > 0 ? sms : 1;
+        g_is_sm103[*dev] = (major == 10 && minor == 3) ? 1 : 2;
+        g_status_ptr[*dev] = static_cast<unsigned*>(p);
+    }
+    *status = g_status_ptr[*dev];
+    return cudaSuccess;
+}
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+struct Call {
+    const void* q;
+    const void* k;
+    const void* v;
+    double tau;
+    int64_t M, N, D, C;
+    gs_dtype dtype;
+    bool grad;
+    float* out;    // M x C (forward) or M x D (grad)
+    float* s_out;  // grad only, nullable
+    cudaStream_t stream;
+    gs_options opt;
+};
+
+gs_status validate(const Call& c) {
+    if (c.dtype != GS_FP32 && c.dtype != GS_FP16 && c.dtype != GS_BF16)
+        return fail(GS_ERR_INVALID_ARGUMENT, "unknown dtype");
+    if (c.M < 0 || c.N < 0 || c.D < 0 || c.C < 0)
+        return fail(GS_ERR_INVALID_ARGUMENT, "negative size");
+    if (!(std::isfinite(c.tau) && c.tau > 0.0))
+        return fail(GS_ERR_INVALID_ARGUMENT, "tau must be finite and > 0");
+    if (c.grad && c.C != 1) return fail(GS_ERR_INVALID_ARGUMENT, "the q-gradient needs C = 1");
+    const int64_t out_w = c.grad ? c.D : c.C;
+    if (c.M > 0 && out_w > 0 && !c.out) return fail(GS_ERR_INVALID_ARGUMENT, "null output pointer");
+    if (c.M > 0 && c.D > 0 && !c.q) return fail(GS_ERR_INVALID_ARGUMENT, "null q pointer");
+    if (c.N > 0 && c.D > 0 && !c.k) return fail(GS_ERR_INVALID_ARGUMENT, "null k pointer");
+    if (c.N > 0 && c.C > 0 && !c.v) return fail(GS_ERR_INVALID_ARGUMENT, "null v pointer");
+    if (!aligned16(c.q) || !aligned16(c.k) || !aligned16(c.v) || !aligned16(c.out) ||
+        !aligned16(c.s_out))
+        return fail(GS_ERR_INVALID_ARGUMENT, "base pointers must be 16-byte aligned");
+    if (c.opt.path == GS_PATH_TENSOR && c.dtype == GS_FP32)
+        return fail(GS_ERR_UNSUPPORTED, "the tensor-core path takes fp16/bf16 inputs");
+    if (c.opt.path == GS_PATH_SIMT && c.dtype != GS_FP32)
+        return fail(GS_ERR_UNSUPPORTED, "the SIMT path takes fp32 inputs");
+    if (c.opt.path < 0 || c.opt.path > 2) return fail(GS_ERR_INVALID_ARGUMENT, "unknown path");
+    if (c.opt.split_n < 0) return fail(GS_ERR_INVALID_ARGUMENT, "split_n must be >= 0");
+    if (c.opt.workspace && (reinterpret_cast<uintptr_t>(c.opt.workspace) & 255u))
+        return fail(GS_ERR_INVALID_ARGUMENT, "caller workspace must be 256-byte aligned");
+    return GS_OK;
+}
+
+gs::InType in_type(gs_dtype d) {
+    return d == GS_FP16 ? gs::InType::F16 : d == GS_BF16 ? gs::InType::BF16 : gs::InType::F32;
+}
+
+// Plans the call; returns GS_OK and the workspace size, or an error.
+gs_status plan(const Call& c, int sms, bool* tensor, gs::TcPlan* tp, gs::SimtPlan* sp,
+               size_t* bytes) {
+    const char* why = "unsupported shape";
+    *tensor = c.dtype != GS_FP32;
+    if (*tensor) {
+        const bool alias = c.q == c.k && c.M == c.N && c.q != nullptr;
+        if (!gs::plan_tensor(c.M, c.N, c.D, c.C, c.grad, c.opt.center != 0, alias, c.opt.split_n,
+                             sms, tp, &why))
+            return fail(GS_ERR_UNSUPPORTED, "%s", why);
+        *bytes = tp->total;
+    } else {
+        if (!gs::plan_simt(c.M, c.N, c.D, c.C, c.grad, c.opt.split_n, sms, sp, &why))
+            return fail(GS_ERR_UNSUPPORTED, "%s", why);
+        *bytes = sp->total;
+    }
+    return GS_OK;
+}
+
+// Test hook: GS_TEST_FAIL_ALLOC=1 makes the workspace allocation fail.
+bool forced_alloc_failure() {
+    const char* s = std::getenv("GS_TEST_FAIL_ALLOC");
+    return s && s[0] == '1';
+}
+
+gs_status run(Call c) {
+    gs_status st = validate(c);
+    if (st != GS_OK) return st;
+    if (c.M == 0) return GS_OK;
+    if (c.grad && c.D == 0) {
+        // No coordinates: the gradient is empty and s is the plain forward sum.
+        if (!c.s_out) return GS_OK;
+        c.grad = false;
+        c.out = c.s_out;
+        c.s_out = nullptr;
+    }
+    const int64_t out_w = c.grad ? c.D : c.C;
+    if (out_w == 0 && !(c.grad && c.s_out)) return GS_OK;
+
+    if (c.N == 0) {
+        cudaError_t e = cudaSuccess;
+        if (out_w > 0) e = cudaMemsetAsync(c.out, 0, sizeof(float) * c.M * out_w, c.stream);
+        if (e == cudaSuccess && c.grad && c.s_out)
+            e = cudaMemsetAsync(c.s_out, 0, sizeof(float) * c.M, c.stream);
+        return e == cudaSuccess ? GS_OK : cuda_fail(e, "cudaMemsetAsync");
+    }
+
+    int dev = 0;
+    unsigned* status = nullptr;
+    cudaError_t e = device_info(&dev, &status);
+    if (e != cudaSuccess) return cuda_fail(e, "device query");
+    const bool tensor_path = c.dtype != GS_FP32;
+    if (tensor_path && g_is_sm103[dev] != 1)
+        return fail(GS_ERR_UNSUPPORTED, "the tensor-core kernel needs an sm_103 (GB300) GPU");
+
+    bool tensor = false;
+    gs::TcPlan tp{};
+    gs::SimtPlan sp{};
+    size_t bytes = 0;
+    st = plan(c, g_sm_count[dev], &tensor, &tp, &sp, &bytes);
+    if (st != GS_OK) return st;
+
+    char* ws = static_cast<char*>(c.opt.workspace);
+    bool owned = false;
+    if (ws) {
+        if (c.opt.workspace_bytes < bytes)
+            return fail(GS_ERR_OUT_OF_MEMORY, "caller workspace is smaller than gauss_sum_workspace_size()");
+    } else if (bytes > 0) {
+        if (forced_alloc_failure()) return fail(GS_ERR_OUT_OF_MEMORY, "workspace allocation failed (test hook)");
+        e = cudaMallocAsync(reinterpret_cast<void**>(&ws), bytes, c.stream);
+        if (e != cudaSuccess) return cuda_fail(e, "workspace cudaMallocAsync");
+        owned = true;
+    }
+
+    const double log2e = 1.4426950408889634;
+    const float cexp = static_cast<float>(c.tau * log2e);
+    const float half_c = static_cast<float>(0.5 * c.tau * log2e);
+    const char* why = "";
+    const char* where = "kernel launch";
+    if (tensor) {
+        const gs::InType t = in_type(c.dtype);
+        float* mu = nullptr;
+        if (tp.center && c.D > 0) {
+            mu = reinterpret_cast<float*>(ws + tp.off_mu);
+            e = gs::launch_mean(t, c.q, c.k, c.M, c.N, static_cast<int>(c.D), tp.mean_blocks,
+                                reinterpret_cast<float*>(ws + tp.off_mean_part), mu, c.stream);
+            where = "mean kernel";
+        }
+        const float ninf = -INFINITY;
+        if (e == cudaSuccess) {
+            e = gs::launch_center_cast_norm(t, c.q, c.M, tp.Mpad, static_cast<int>(c.D), tp.Dp, mu,
+                                            half_c, ws + tp.off_qh,
+                                            reinterpret_cast<float*>(ws + tp.off_A), ninf, c.stream);
+            where = "centre/cast kernel (q)";
+        }
+        if (e == cudaSuccess && !tp.alias) {
+            e = gs::launch_center_cast_norm(t, c.k, c.N, tp.Npad, static_cast<int>(c.D), tp.Dp, mu,
+                                            half_c, ws + tp.off_kh,
+                                            reinterpret_cast<float*>(ws + tp.off_B), ninf, c.stream);
+            where = "centre/cast kernel (k)";
+        }
+        if (e == cudaSuccess) {
+            e = gs::launch_value_prep(t, c.grad, c.v, c.k, mu, c.N, tp.Npad, static_cast<int>(c.D),
+                                      static_cast<int>(tp.Cv), tp.Cp,
+                                      reinterpret_cast<unsigned*>(ws + tp.off_vmax), ws + tp.off_vt,
+                                      reinterpret_cast<float*>(ws + tp.off_inv), c.stream);
+            where = "value kernel";
+        }
+        if (e == cudaSuccess) {
+            e = gs::launch_tc(tp, t, cexp, ws, status, c.stream, &why);
+            where = "fused tensor-core kernel";
+        }
+        if (e == cudaSuccess) {
+            e = gs::launch_finalize(c.grad ? 1 : 0, t, reinterpret_cast<float*>(ws + tp.off_part),
+                                    tp.splits, tp.Mpad, c.M, static_cast<int>(tp.Cv), tp.Cp,
+                                    reinterpret_cast<float*>(ws + tp.off_inv), c.q, mu,
+                                    static_cast<float>(c.tau), static_cast<int>(c.D), c.out,
+                                    c.s_out, c.stream);
+            where = "finalise kernel";
+        }
+    } else {
+        float* part = reinterpret_cast<float*>(ws + sp.off_part);
+        e = gs::launch_simt(sp, c.grad, static_cast<const float*>(c.q),
+                            static_cast<const float*>(c.k), static_cast<const float*>(c.v), half_c,
+                            part, c.stream);
+        where = "fp32 kernel";
+        if (e == cudaSuccess) {
+            e = gs::launch_finalize(c.grad ? 2 : 0, gs::InType::F32, part, sp.splits, c.M, c.M,
+                                    static_cast<int>(sp.Cv), static_cast<int>(sp.Cv), nullptr,
+                                    nullptr, nullptr, static_cast<float>(c.tau),
+                                    static_cast<int>(c.D), c.out, c.s_out, c.stream);
+            where = "finalise kernel";
+        }
+    }
+    if (owned) {
+        cudaError_t ef = cudaFreeAsync(ws, c.stream);
+        if (e == cudaSuccess && ef != cudaSuccess) return cuda_fail(ef, "workspace cudaFreeAsync");
+    }
+    if (e != cudaSuccess) {
+        if (why && why[0]) return fail(GS_ERR_CUDA, "%s", why);
+        return cuda_fail(e, where);
+    }
+    return GS_OK;
+}
+
+gs_options defaults() {
+    gs_options o;
+    o.center = 1;
+    o.split_n = 0;
+    o.workspace = nullptr;
+    o.workspace_bytes = 0;
+    o.path = GS_PATH_AUTO;
+    return o;
+}
+
+// ---------------------------------------------------------------- ex2 probe
+template <int CH>
+__global__ void ex2_probe_kernel(float* out, int iters) {
+    float x[CH];
+#pragma unroll
+    for (int i = 0; i < CH; ++i) x[i] = -0.001f * static_cast<float>(threadIdx.x + i);
+    for (int it = 0; it < iters; ++it) {
+#pragma unroll
+        for (int i = 0; i < CH; ++i) x[i] = gs::ex2_approx(x[i]) - 1.0f;
+    }
+    float s = 0.f;
+#pragma unroll
+    for (int i = 0; i < CH; ++i) s += x[i];
+    out[blockIdx.x * blockDim.x + threadIdx.x] = s;
+}
+
+}  // namespace
+
+namespace gs {
+cudaError_t run_ex2_probe(cudaStream_t s, double* rate) {
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    int sms = 1;
+    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    const int blocks = sms * 4, threads = 512, iters = 4096;
+    float* out = nullptr;
+    e = cudaMallocAsync(reinterpret_cast<void**>(&out), sizeof(float) * blocks * threads, s);
+    if (e != cudaSuccess) return e;
+    cudaEvent_t e0, e1;
+    cudaEventCreate(&e0);
+    cudaEventCreate(&e1);
+    double best = 0.0;
+    for (int rep = 0; rep < 4; ++rep) {
+        cudaEventRecord(e0, s);
+        ex2_probe_kernel<8><<<blocks, threads, 0, s>>>(out, iters);
+        cudaEventRecord(e1, s);
+        e = cudaEventSynchronize(e1);
+        if (e != cudaSuccess) break;
+        float ms = 0.f;
+        cudaEventElapsedTime(&ms, e0, e1);
+        const double n = static_cast<double>(blocks) * threads * iters * 8;
+        if (rep > 0 && ms > 0.f) best = std::max(best, n / (ms * 1e-3));
+    }
+    cudaEventDestroy(e0);
+    cudaEventDestroy(e1);
+    cudaFreeAsync(out, s);
+    cudaError_t e2 = cudaStreamSynchronize(s);
+    *rate = best;
+    return e != cudaSuccess ? e : e2;
+}
+}  // namespace gs
+
+extern "C" {
+
+void gauss_sum_default_options(gs_options* opt) {
+    if (opt) *opt = defaults();
+}
+
+gs_status gauss_sum_ex(const void* q, const void* k, const void* v, double tau, int64_t M,
+                       int64_t N, int64_t D, int64_t C, gs_dtype dtype, float* out, void* stream,
+                       const gs_options* opt) {
+    Call c{q, k, v, tau, M, N, D, C, dtype, false, out, nullptr,
+           static_cast<cudaStream_t>(stream), opt ? *opt : defaults()};
+    return run(c);
+}
+
+gs_status gauss_sum(const void* q, const void* k, const void* v, double tau, int64_t M,
+                    int64_t N, int64_t D, int64_t C, gs_dtype dtype, float* out, void* stream) {
+    return gauss_sum_ex(q, k, v, tau, M, N, D, C, dtype, out, stream, nullptr);
+}
+
+gs_status gauss_sum_grad_q_ex(const void* q, const void* k, const void* v, double tau,
+                              int64_t M, int64_t N, int64_t D, gs_dtype dtype, float* grad,
+                              float* s_out, void* stream, const gs_options* opt) {
+    Call c{q, k, v, tau, M, N, D, 1, dtype, true, grad, s_out,
+           static_cast<cudaStream_t>(stream), opt ? *opt : defaults()};
+    return run(c);
+}
+
+gs_status gauss_sum_grad_q(const void* q, const void* k, const void* v, double tau, int64_t M,
+                           int64_t N, int64_t D, gs_dtype dtype, float* grad, float* s_out,
+                           void* stream) {
+    return gauss_sum_grad_q_ex(q, k, v, tau, M, N, D, dtype, grad, s_out, stream, nullptr);
+}
+
+size_t gauss_sum_workspace_size(int64_t M, int64_t N, int64_t D, int64_t C, gs_dtype dtype,
+                                int grad, const gs_options* opt) {
+    const gs_options o = opt ? *opt : defaults();
+    // Distinct stand-in pointers: the size returned covers q and k being
+    // different arrays (an aliased call needs less).
+    static const char dummy[64] __attribute__((aligned(16))) = {0};
+    Call c{dummy, dummy + 16, dummy + 32, 1.0, M, N, D, grad ? 1 : C, dtype, grad != 0,
+           reinterpret_cast<float*>(const_cast<char*>(dummy + 48)), nullptr, nullptr, o};
+    c.opt.workspace = nullptr;
+    if (validate(c) != GS_OK) return static_cast<size_t>(-1);
+    if (M == 0 || N == 0) return 0;
+    int sms = 152;
+    int dev = 0;
+    if (cudaGetDevice(&dev) == cudaSuccess) {
+        int s = 0;
+        if (cudaDeviceGetAttribute(&s, cudaDevAttrMultiProcessorCount, dev) == cudaSuccess && s > 0) sms = s;
+    } else {
+        cudaGetLastError();
+    }
+    bool tensor = false;
+    gs::TcPlan tp{};
+    gs::SimtPlan sp{};
+    size_t bytes = 0;
+    if (plan(c, sms, &tensor, &tp, &sp, &bytes) != GS_OK) return static_cast<size_t>(-1);
+    return bytes;
+}
+
+gs_status gauss_sum_device_status(void* stream) {
+    int dev = 0;
+    unsigned* status = nullptr;
+    cudaError_t e = cudaStreamSynchronize(static_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_fail(e, "cudaStreamSynchronize");
+    e = device_info(&dev, &status);
+    if (e != cudaSuccess) return cuda_fail(e, "device query");
+    unsigned v = 0;
+    e = cudaMemcpy(&v, status, sizeof(unsigned), cudaMemcpyDeviceToHost);
+    if (e != cudaSuccess) return cuda_fail(e, "status read");
+    const unsigned zero = 0;
+    e = cudaMemcpy(status, &zero, sizeof(unsigned), cudaMemcpyHostToDevice);
+    if (e != cudaSuccess) return cuda_fail(e, "status clear");
+    if (v == gs::kDevTimeout)
+        return fail(GS_ERR_DEVICE_TIMEOUT, "a device-side wait ran out of time");
+    return GS_OK;
+}
+
+const char* gauss_sum_last_error(void) { return g_last_error; }
+
+const char* gauss_sum_status_string(gs_status s) {
+    switch (s) {
+        case GS_OK: return "GS_OK";
+        case GS_ERR_INVALID_ARGUMENT: return "GS_ERR_INVALID_ARGUMENT";
+        case GS_ERR_UNSUPPORTED: return "GS_ERR_UNSUPPORTED";
+        case GS_ERR_OUT_OF_MEMORY: return "GS_ERR_OUT_OF_MEMORY";
+        case GS_ERR_CUDA: return "GS_ERR_CUDA";
+        case GS_ERR_DEVICE_TIMEOUT: return "GS_ERR_DEVICE_TIMEOUT";
+    }
+    return "unknown status";
+}
+
+gs_status gauss_sum_probe_ex2_rate(void* stream, double* exp2_per_second) {
+    if (!exp2_per_second) return fail(GS_ERR_INVALID_ARGUMENT, "null output pointer");
+    cudaError_t e = gs::run_ex2_probe(static_cast<cudaStream_t>(stream), exp2_per_second);
+    if (e != cudaSuccess) return cuda_fail(e, "ex2 probe");
+    return GS_OK;
+}
+
+}  // extern "C"

@@ -1,0 +1,74 @@
+// Internal interfaces between the C ABI (api.cu) and the kernel files.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <cstddef>
+#include <cstdint>
+
+namespace gs {
+
+enum class InType { F32 = 0, F16 = 1, BF16 = 2 };
+
+// Workspace plan of the tensor-core path.  All offsets are bytes from the
+// workspace base and are 1024-byte aligned.
+struct TcPlan {
+    int64_t M, N, D, Cv;     // Cv: value channels (C, or D + 1 for the gradient)
+    int64_t Mpad, Npad;      // rows padded to the row tile / key tile
+    int Dp, Cp;              // D and Cv rounded up to 16
+    int BN;                  // key tile width (128, or 64 when Cp > 128)
+    int splits;              // key splits per row tile
+    int stages;              // shared-memory pipeline depth
+    size_t smem_bytes;       // dynamic shared memory of the fused kernel
+    int mean_blocks;
+    bool alias;              // q and k are the same array (M == N): prep once
+    bool center;
+    size_t off_mean_part, off_mu, off_qh, off_kh, off_A, off_B, off_vt, off_vmax, off_inv,
+        off_part, total;
+};
+
+struct SimtPlan {
+    int64_t M, N, D, Cv;
+    int dmax;          // register tile of the query row (16, 32, 64 or 128)
+    int cblk;          // channels per launch slice
+    int splits;
+    int64_t keys_per_split;
+    size_t off_part, total;
+};
+
+int device_sm_count(int device);
+bool device_is_sm103(int device);
+
+bool plan_tensor(int64_t M, int64_t N, int64_t D, int64_t C, bool grad, bool center,
+                 bool alias, int split_override, int sms, TcPlan* p, const char** why);
+bool plan_simt(int64_t M, int64_t N, int64_t D, int64_t C, bool grad, int split_override,
+               int sms, SimtPlan* p, const char** why);
+
+// prep.cu --------------------------------------------------------------
+cudaError_t launch_mean(InType t, const void* q, const void* k, int64_t M, int64_t N, int D,
+                        int blocks, float* partial, float* mu, cudaStream_t s);
+cudaError_t launch_center_cast_norm(InType t, const void* x, int64_t rows, int64_t rows_pad,
+                                    int D, int Dp, const float* mu, float half_c, void* xh,
+                                    float* nrm, float pad_value, cudaStream_t s);
+cudaError_t launch_value_prep(InType t, bool grad, const void* v, const void* k,
+                              const float* mu, int64_t N, int64_t Npad, int D, int Cv, int Cp,
+                              unsigned* vmax_bits, void* vt, float* inv_scale, cudaStream_t s);
+// mode 0: forward (out M x Cv, scaled by inv_scale when given)
+// mode 1: gradient from augmented values (tensor path): needs q, mu, tau
+// mode 2: gradient from direct partials (SIMT path): Cv = D + 1
+cudaError_t launch_finalize(int mode, InType t, const float* part, int splits,
+                            int64_t split_stride_rows, int64_t M, int Cv, int part_ld,
+                            const float* inv_scale, const void* q, const float* mu, float tau,
+                            int D, float* out, float* s_out, cudaStream_t s);
+
+// simt_fp32.cu ---------------------------------------------------------
+cudaError_t launch_simt(const SimtPlan& p, bool grad, const float* q, const float* k,
+                        const float* v, float half_c, float* part, cudaStream_t s);
+
+// tc_gauss.cu ----------------------------------------------------------
+cudaError_t launch_tc(const TcPlan& p, InType t, float c, char* ws, unsigned* status,
+                      cudaStream_t s, const char** why);
+
+// probe
+cudaError_t run_ex2_probe(cudaStream_t s, double* rate);
+
+}  // namespace gs

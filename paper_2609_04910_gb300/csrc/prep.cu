@@ -1,0 +1,351 @@
+// Preparation and finalisation kernels of the Gauss-sum path.
+//
+//  * common mean of all query and key points (the shift safeguard of
+//    Remark 3, Sec. 2: the kernel depends on q - k only, so any common shift
+//    is exact and only changes rounding);
+//  * centring, rounding to the MMA operand type and the scaled squared norms
+//    A_m = -(c/2)||q^_m||^2, B_n = -(c/2)||k^_n||^2 (c = tau log2 e) taken
+//    from the ROUNDED points, so that c q^.k^ + A_m + B_n is exactly
+//    -(c/2)||q^_m - k^_n||^2 up to fp32 rounding (the norm factors of Alg. 1,
+//    folded into one exponent);
+//  * the value operand: per-channel power-of-two scaling of v (or of the
+//    gradient values (v_n k_n, v_n) of Sec. 3) rounded to fp16 and stored
+//    transposed (channel-major) so that both MMAs read K-major operands;
+//  * the fixed-order sum of key-split partials and the final scaling, or
+//    the gradient tau (S[:D] - q_m S[D]) of Sec. 3.
+#include <cuda_bf16.h>
+#include <cuda_fp16.h>
+#include <math_constants.h>
+
+#include "internal.h"
+
+namespace gs {
+namespace {
+
+template <typename T> __device__ __forceinline__ float to_f(T x);
+template <> __device__ __forceinline__ float to_f<float>(float x) { return x; }
+template <> __device__ __forceinline__ float to_f<__half>(__half x) { return __half2float(x); }
+template <> __device__ __forceinline__ float to_f<__nv_bfloat16>(__nv_bfloat16 x) {
+    return __bfloat162float(x);
+}
+
+template <typename H> __device__ __forceinline__ H from_f(float x);
+template <> __device__ __forceinline__ __half from_f<__half>(float x) { return __float2half_rn(x); }
+template <> __device__ __forceinline__ __nv_bfloat16 from_f<__nv_bfloat16>(float x) {
+    return __float2bfloat16_rn(x);
+}
+
+// ---------------------------------------------------------------- mean
+// Block (32, 8): 32 consecutive coordinates x 8 row lanes; each block sums
+// a contiguous chunk of the stacked rows [q; k] and writes D partial sums.
+template <typename T>
+__global__ void mean_partial_kernel(const T* __restrict__ q, const T* __restrict__ k, int64_t M,
+                                    int64_t N, int D, int64_t rows_per_block,
+                                    float* __restrict__ partial) {
+    __shared__ float red[8][33];
+    const int64_t r0 = static_cast<int64_t>(blockIdx.x) * rows_per_block;
+    const int64_t r1 = min(r0 + rows_per_block, M + N);
+    for (int d0 = 0; d0 < D; d0 += 32) {
+        const int d = d0 + threadIdx.x;
+        float acc = 0.f;
+        if (d < D) {
+            for (int64_t r = r0 + threadIdx.y; r < r1; r += 8) {
+                const T x = r < M ? q[r * D + d] : k[(r - M) * D + d];
+                acc += to_f(x);
+            }
+        }
+        red[threadIdx.y][threadIdx.x] = acc;
+        __syncthreads();
+        if (threadIdx.y == 0 && d < D) {
+            float s = 0.f;
+#pragma unroll
+            for (int y = 0; y < 8; ++y) s += red[y][threadIdx.x];
+            partial[static_cast<int64_t>(blockIdx.x) * D + d] = s;
+        }
+        __syncthreads();
+    }
+}
+
+__global__ void mean_final_kernel(const float* __restrict__ partial, int G, int D, double total,
+                                  float* __restrict__ mu) {
+    const int d = blockIdx.x * blockDim.x + threadIdx.x;
+    if (d >= D) return;
+    double s = 0.0;
+    for (int g = 0; g < G; ++g) s += static_cast<double>(partial[static_cast<int64_t>(g) * D + d]);
+    mu[d] = static_cast<float>(s / total);
+}
+
+// ---------------------------------------------------------------- centre / cast / norm
+// One warp per row.  Rows in [rows, rows_pad) become zero rows with norm
+// term `pad_value` (-inf for padded keys, so their kernel value is 0).
+template <typename T, typename H>
+__global__ void center_cast_norm_kernel(const T* __restrict__ x, int64_t rows, int64_t rows_pad,
+                                        int D, int Dp, const float* __restrict__ mu,
+                                        float half_c, H* __restrict__ xh,
+                                        float* __restrict__ nrm, float pad_value) {
+    const int lane = threadIdx.x & 31;
+    const int64_t row = static_cast<int64_t>(blockIdx.x) * (blockDim.x >> 5) + (threadIdx.x >> 5);
+    if (row >= rows_pad) return;
+    H* out = xh + row * Dp;
+    if (row >= rows) {
+        for (int d = lane; d < Dp; d += 32) out[d] = from_f<H>(0.f);
+        if (lane == 0) nrm[row] = pad_value;
+        return;
+    }
+    const T* in = x + row * D;
+    float acc = 0.f;
+    for (int d = lane; d < Dp; d += 32) {
+        float val = 0.f;
+        if (d < D) val = to_f(in[d]) - (mu ? mu[d] : 0.f);
+        const H h = from_f<H>(val);
+        out[d] = h;
+        const float hf = to_f(h);
+        acc = fmaf(hf, hf, acc);
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
+    if (lane == 0) nrm[row] = -half_c * acc;
+}
+
+// ---------------------------------------------------------------- values
+// Value of channel c of key n: v[n, c] (forward) or, for the gradient of
+// Sec. 3, v_n (k[n, c] - mu_c) for c < D and v_n for c = D.
+template <typename T, bool GRAD>
+__device__ __forceinline__ float value_at(const T* __restrict__ v, const T* __restrict__ k,
+                                          const float* __restrict__ mu, int64_t n, int c, int D,
+                                          int Cv) {
+    if (GRAD) {
+        const float vn = to_f(v[n]);
+        if (c < D) return vn * (to_f(k[n * D + c]) - (mu ? mu[c] : 0.f));
+        return vn;
+    }
+    return to_f(v[n * Cv + c]);
+}
+
+// Per-channel max |value| over the keys; block (32, 8) as in the mean.
+template <typename T, bool GRAD>
+__global__ void value_max_kernel(const T* __restrict__ v, const T* __restrict__ k,
+                                 const float* __restrict__ mu, int64_t N, int D, int Cv,
+                                 int64_t rows_per_block, unsigned* __restrict__ vmax_bits) {
+    __shared__ float red[8][33];
+    const int64_t r0 = static_cast<int64_t>(blockIdx.x) * rows_per_block;
+    const int64_t r1 = min(r0 + rows_per_block, N);
+    for (int c0 = 0; c0 < Cv; c0 += 32) {
+        const int c = c0 + threadIdx.x;
+        float mx = 0.f;
+        if (c < Cv)
+            for (int64_t n = r0 + threadIdx.y; n < r1; n += 8)
+                mx = fmaxf(mx, fabsf(value_at<T, GRAD>(v, k, mu, n, c, D, Cv)));
+        red[threadIdx.y][threadIdx.x] = mx;
+        __syncthreads();
+        if (threadIdx.y == 0 && c < Cv) {
+            float m = 0.f;
+#pragma unroll
+            for (int y = 0; y < 8; ++y) m = fmaxf(m, red[y][threadIdx.x]);
+            // Non-negative floats order like their bit patterns.
+            atomicMax(&vmax_bits[c], __float_as_uint(m));
+        }
+        __syncthreads();
+    }
+}
+
+// Power-of-two channel scale 2^e with e = -floor(log2 max|value|), so that
+// the scaled channel's largest magnitude lies in [1, 2); e is clamped to
+// [-126, 126] and is 0 for an all-zero channel.  Exact bit construction.
+__device__ __forceinline__ int channel_exponent(unsigned max_bits) {
+    if (max_bits == 0u) return 0;
+    int E = static_cast<int>((max_bits >> 23) & 0xffu);
+    if (E == 0) E = 1;             // subnormal maximum: clamp
+    if (E == 0xff) return 0;       // inf / nan: leave unscaled
+    int e = 127 - E;               // -floor(log2 max)
+    return max(-126, min(126, e));
+}
+
+__device__ __forceinline__ float pow2f(int e) { return __uint_as_float(static_cast<unsigned>(e + 127) << 23); }
+
+// Transposed, scaled fp16 value operand vt[c][n] (Cp x Npad, zero padded),
+// through a 32 x 32 shared-memory tile; block (32, 8).
+template <typename T, bool GRAD>
+__global__ void value_prep_kernel(const T* __restrict__ v, const T* __restrict__ k,
+                                  const float* __restrict__ mu, int64_t N, int64_t Npad, int D,
+                                  int Cv, int Cp, const unsigned* __restrict__ vmax_bits,
+                                  __half* __restrict__ vt, float* __restrict__ inv_scale) {
+    __shared__ float tile[32][33];
+    const int64_t n0 = static_cast<int64_t>(blockIdx.x) * 32;
+    const int c0 = blockIdx.y * 32;
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        const int64_t n = n0 + threadIdx.y + 8 * i;
+        const int c = c0 + threadIdx.x;
+        float val = 0.f;
+        if (n < N && c < Cv) val = value_at<T, GRAD>(v, k, mu, n, c, D, Cv);
+        tile[threadIdx.y + 8 * i][threadIdx.x] = val;
+    }
+    __syncthreads();
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        const int c = c0 + threadIdx.y + 8 * i;
+        const int64_t n = n0 + threadIdx.x;
+        if (c < Cp && n < Npad) {
+            const float sc = c < Cv ? pow2f(channel_exponent(vmax_bits[c])) : 0.f;
+            vt[static_cast<int64_t>(c) * Npad + n] = __float2half_rn(tile[threadIdx.x][threadIdx.y + 8 * i] * sc);
+        }
+    }
+    if (blockIdx.x == 0 && threadIdx.y == 0) {
+        const int c = c0 + threadIdx.x;
+        if (c < Cp) inv_scale[c] = c < Cv ? pow2f(-channel_exponent(vmax_bits[c])) : 0.f;
+    }
+}
+
+// ---------------------------------------------------------------- finalise
+// part: splits blocks of split_stride_rows rows x part_ld floats.
+template <int MODE, typename T>
+__global__ void finalize_kernel(const float* __restrict__ part, int splits,
+                                int64_t split_stride_rows, int64_t M, int Cv, int part_ld,
+                                const float* __restrict__ inv_scale, const T* __restrict__ q,
+                                const float* __restrict__ mu, float tau, int D,
+                                float* __restrict__ out, float* __restrict__ s_out) {
+    const int64_t width = MODE == 0 ? Cv : D;
+    const int64_t idx = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
+    if (idx >= M * width) return;
+    const int64_t m = idx / width;
+    const int c = static_cast<int>(idx - m * width);
+    auto sum_channel = [&](int ch) {
+        float acc = 0.f;
+        for (int s = 0; s < splits; ++s)
+            acc += part[(static_cast<int64_t>(s) * split_stride_rows + m) * part_ld + ch];
+        return acc;
+    };
+    if (MODE == 0) {
+        const float sc = inv_scale ? inv_scale[c] : 1.f;
+        out[idx] = sum_channel(c) * sc;
+    } else if (MODE == 1) {
+        const float sd = sum_channel(c) * inv_scale[c];
+        const float s0 = sum_channel(D) * inv_scale[D];
+        const float qc = to_f(q[m * D + c]) - (mu ? mu[c] : 0.f);
+        out[idx] = tau * (sd - qc * s0);
+        if (c == 0 && s_out) s_out[m] = s0;
+    } else {
+        out[idx] = tau * sum_channel(c);
+        if (c == 0 && s_out) s_out[m] = sum_channel(D);
+    }
+}
+
+template <typename T, typename H>
+cudaError_t ccn_typed(const void* x, int64_t rows, int64_t rows_pad, int D, int Dp,
+                      const float* mu, float half_c, void* xh, float* nrm, float pad_value,
+                      cudaStream_t s) {
+    const int warps = 8;
+    const int64_t blocks = (rows_pad + warps - 1) / warps;
+    center_cast_norm_kernel<T, H><<<static_cast<unsigned>(blocks), warps * 32, 0, s>>>(
+        static_cast<const T*>(x), rows, rows_pad, D, Dp, mu, half_c, static_cast<H*>(xh), nrm,
+        pad_value);
+    return cudaGetLastError();
+}
+
+template <typename T, bool GRAD>
+cudaError_t value_prep_typed(const void* v, const void* k, const float* mu, int64_t N,
+                             int64_t Npad, int D, int Cv, int Cp, unsigned* vmax_bits, void* vt,
+                             float* inv_scale, cudaStream_t s) {
+    cudaError_t e = cudaMemsetAsync(vmax_bits, 0, sizeof(unsigned) * Cp, s);
+    if (e != cudaSuccess) return e;
+    const int64_t rows_per_block = 512;
+    const int64_t blocks = N > 0 ? (N + rows_per_block - 1) / rows_per_block : 0;
+    if (blocks > 0) {
+        value_max_kernel<T, GRAD><<<static_cast<unsigned>(blocks), dim3(32, 8), 0, s>>>(
+            static_cast<const T*>(v), static_cast<const T*>(k), mu, N, D, Cv, rows_per_block,
+            vmax_bits);
+        e = cudaGetLastError();
+        if (e != cudaSuccess) return e;
+    }
+    dim3 grid(static_cast<unsigned>((Npad + 31) / 32), static_cast<unsigned>((Cp + 31) / 32));
+    value_prep_kernel<T, GRAD><<<grid, dim3(32, 8), 0, s>>>(
+        static_cast<const T*>(v), static_cast<const T*>(k), mu, N, Npad, D, Cv, Cp, vmax_bits,
+        static_cast<__half*>(vt), inv_scale);
+    return cudaGetLastError();
+}
+
+template <int MODE, typename T>
+cudaError_t finalize_typed(const float* part, int splits, int64_t stride_rows, int64_t M, int Cv,
+                           int part_ld, const float* inv_scale, const void* q, const float* mu,
+                           float tau, int D, float* out, float* s_out, cudaStream_t s) {
+    const int64_t width = MODE == 0 ? Cv : D;
+    const int64_t total = M * width;
+    if (total == 0) return cudaSuccess;
+    const int threads = 256;
+    const int64_t blocks = (total + threads - 1) / threads;
+    finalize_kernel<MODE, T><<<static_cast<unsigned>(blocks), threads, 0, s>>>(
+        part, splits, stride_rows, M, Cv, part_ld, inv_scale, static_cast<const T*>(q), mu, tau,
+        D, out, s_out);
+    return cudaGetLastError();
+}
+
+}  // namespace
+
+cudaError_t launch_mean(InType t, const void* q, const void* k, int64_t M, int64_t N, int D,
+                        int blocks, float* partial, float* mu, cudaStream_t s) {
+    const int64_t total = M + N;
+    const int64_t rpb = (total + blocks - 1) / blocks;
+    const int G = static_cast<int>((total + rpb - 1) / rpb);
+    switch (t) {
+        case InType::F16:
+            mean_partial_kernel<__half><<<G, dim3(32, 8), 0, s>>>(
+                static_cast<const __half*>(q), static_cast<const __half*>(k), M, N, D, rpb, partial);
+            break;
+        case InType::BF16:
+            mean_partial_kernel<__nv_bfloat16><<<G, dim3(32, 8), 0, s>>>(
+                static_cast<const __nv_bfloat16*>(q), static_cast<const __nv_bfloat16*>(k), M, N,
+                D, rpb, partial);
+            break;
+        default:
+            mean_partial_kernel<float><<<G, dim3(32, 8), 0, s>>>(
+                static_cast<const float*>(q), static_cast<const float*>(k), M, N, D, rpb, partial);
+    }
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    mean_final_kernel<<<(D + 127) / 128, 128, 0, s>>>(partial, G, D, static_cast<double>(total), mu);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_center_cast_norm(InType t, const void* x, int64_t rows, int64_t rows_pad,
+                                    int D, int Dp, const float* mu, float half_c, void* xh,
+                                    float* nrm, float pad_value, cudaStream_t s) {
+    if (t == InType::BF16)
+        return ccn_typed<__nv_bfloat16, __nv_bfloat16>(x, rows, rows_pad, D, Dp, mu, half_c, xh,
+                                                       nrm, pad_value, s);
+    return ccn_typed<__half, __half>(x, rows, rows_pad, D, Dp, mu, half_c, xh, nrm, pad_value, s);
+}
+
+cudaError_t launch_value_prep(InType t, bool grad, const void* v, const void* k,
+                              const float* mu, int64_t N, int64_t Npad, int D, int Cv, int Cp,
+                              unsigned* vmax_bits, void* vt, float* inv_scale, cudaStream_t s) {
+    if (t == InType::BF16) {
+        return grad ? value_prep_typed<__nv_bfloat16, true>(v, k, mu, N, Npad, D, Cv, Cp,
+                                                            vmax_bits, vt, inv_scale, s)
+                    : value_prep_typed<__nv_bfloat16, false>(v, k, mu, N, Npad, D, Cv, Cp,
+                                                             vmax_bits, vt, inv_scale, s);
+    }
+    return grad ? value_prep_typed<__half, true>(v, k, mu, N, Npad, D, Cv, Cp, vmax_bits, vt,
+                                                 inv_scale, s)
+                : value_prep_typed<__half, false>(v, k, mu, N, Npad, D, Cv, Cp, vmax_bits, vt,
+                                                  inv_scale, s);
+}
+
+cudaError_t launch_finalize(int mode, InType t, const float* part, int splits,
+                            int64_t split_stride_rows, int64_t M, int Cv, int part_ld,
+                            const float* inv_scale, const void* q, const float* mu, float tau,
+                            int D, float* out, float* s_out, cudaStream_t s) {
+    if (mode == 0)
+        return finalize_typed<0, float>(part, splits, split_stride_rows, M, Cv, part_ld,
+                                        inv_scale, nullptr, nullptr, tau, D, out, s_out, s);
+    if (mode == 2)
+        return finalize_typed<2, float>(part, splits, split_stride_rows, M, Cv, part_ld,
+                                        inv_scale, nullptr, nullptr, tau, D, out, s_out, s);
+    if (t == InType::BF16)
+        return finalize_typed<1, __nv_bfloat16>(part, splits, split_stride_rows, M, Cv, part_ld,
+                                                inv_scale, q, mu, tau, D, out, s_out, s);
+    return finalize_typed<1, __half>(part, splits, split_stride_rows, M, Cv, part_ld, inv_scale,
+                                     q, mu, tau, D, out, s_out, s);
+}
+
+}  // namespace gs

@@ -1,0 +1,169 @@
+// fp32 SIMT Gauss-sum kernel (the single-precision regime of the paper's
+// appendix, where tensor-core attention is not available).
+//
+// Each thread owns one query row, held in registers and zero padded to
+// DMAX coordinates.  Keys stream through shared memory in tiles of KT keys
+// (zero padded to DMAX, so padded coordinates add (0 - 0)^2 = 0).  For each
+// pair the squared distance is formed in the direct-difference form
+// sum_d (q_d - k_d)^2 (no Gram identity, hence no cancellation), the kernel
+// value is 2^(-(c/2) d^2) with c = tau log2 e, and the values are
+// accumulated with fp32 FMAs:
+//   forward (Eq. 1):     acc[j] += Phi v[n, c0 + j]       for CBLK channels
+//   gradient (Sec. 3):   acc[d] += Phi v_n (k_d - q_d),   acc[D] += Phi v_n
+// The key range is split over gridDim.y; partial sums go to a workspace and
+// are added in a fixed order by the finalise kernel.
+#include <algorithm>
+
+#include "internal.h"
+#include "ptx.cuh"
+
+namespace gs {
+namespace {
+
+constexpr int KT = 64;       // keys per shared-memory tile
+constexpr int THREADS = 128; // query rows per block
+
+template <int DMAX, int CBLK, bool GRAD>
+__global__ void __launch_bounds__(THREADS)
+simt_gauss_kernel(const float* __restrict__ q, const float* __restrict__ k,
+                  const float* __restrict__ v, int64_t M, int64_t N, int D, int Cv,
+                  float half_c, int64_t keys_per_split, float* __restrict__ part) {
+    constexpr int NACC = GRAD ? DMAX + 1 : CBLK;
+    __shared__ __align__(16) float ks[KT][DMAX];
+    __shared__ float vs[KT][GRAD ? 1 : CBLK];
+
+    const int64_t m = static_cast<int64_t>(blockIdx.x) * THREADS + threadIdx.x;
+    const int split = blockIdx.y;
+    const int c0 = GRAD ? 0 : blockIdx.z * CBLK;
+    const int64_t n_begin = static_cast<int64_t>(split) * keys_per_split;
+    const int64_t n_end = min(N, n_begin + keys_per_split);
+
+    float qr[DMAX];
+#pragma unroll
+    for (int d = 0; d < DMAX; ++d) qr[d] = (m < M && d < D) ? q[m * D + d] : 0.f;
+    float acc[NACC];
+#pragma unroll
+    for (int j = 0; j < NACC; ++j) acc[j] = 0.f;
+
+    for (int64_t t0 = n_begin; t0 < n_end; t0 += KT) {
+        const int cnt = static_cast<int>(min(static_cast<int64_t>(KT), n_end - t0));
+        __syncthreads();
+        for (int i = threadIdx.x; i < KT * DMAX; i += THREADS) {
+            const int kk = i / DMAX, d = i - kk * DMAX;
+            ks[kk][d] = (kk < cnt && d < D) ? k[(t0 + kk) * D + d] : 0.f;
+        }
+        if (GRAD) {
+            for (int i = threadIdx.x; i < KT; i += THREADS) vs[i][0] = i < cnt ? v[t0 + i] : 0.f;
+        } else {
+            for (int i = threadIdx.x; i < KT * CBLK; i += THREADS) {
+                const int kk = i / CBLK, j = i - kk * CBLK;
+                vs[kk][j] = (kk < cnt && c0 + j < Cv) ? v[(t0 + kk) * Cv + c0 + j] : 0.f;
+            }
+        }
+        __syncthreads();
+        for (int kk = 0; kk < cnt; ++kk) {
+            float d2 = 0.f;
+#pragma unroll
+            for (int d = 0; d < DMAX; d += 4) {
+                const float4 kv = *reinterpret_cast<const float4*>(&ks[kk][d]);
+                float t;
+                t = qr[d + 0] - kv.x; d2 = fmaf(t, t, d2);
+                t = qr[d + 1] - kv.y; d2 = fmaf(t, t, d2);
+                t = qr[d + 2] - kv.z; d2 = fmaf(t, t, d2);
+                t = qr[d + 3] - kv.w; d2 = fmaf(t, t, d2);
+            }
+            const float phi = ex2_approx(-half_c * d2);
+            if (GRAD) {
+                const float w = phi * vs[kk][0];
+#pragma unroll
+                for (int d = 0; d < DMAX; d += 4) {
+                    const float4 kv = *reinterpret_cast<const float4*>(&ks[kk][d]);
+                    acc[d + 0] = fmaf(w, kv.x - qr[d + 0], acc[d + 0]);
+                    acc[d + 1] = fmaf(w, kv.y - qr[d + 1], acc[d + 1]);
+                    acc[d + 2] = fmaf(w, kv.z - qr[d + 2], acc[d + 2]);
+                    acc[d + 3] = fmaf(w, kv.w - qr[d + 3], acc[d + 3]);
+                }
+                acc[DMAX] += w;
+            } else {
+#pragma unroll
+                for (int j = 0; j < CBLK; ++j) acc[j] = fmaf(phi, vs[kk][j], acc[j]);
+            }
+        }
+    }
+    if (m >= M) return;
+    if (GRAD) {
+        float* out = part + (static_cast<int64_t>(split) * M + m) * (D + 1);
+#pragma unroll
+        for (int d = 0; d < DMAX; ++d)
+            if (d < D) out[d] = acc[d];
+        out[D] = acc[DMAX];
+    } else {
+        float* out = part + (static_cast<int64_t>(split) * M + m) * Cv + c0;
+#pragma unroll
+        for (int j = 0; j < CBLK; ++j)
+            if (c0 + j < Cv) out[j] = acc[j];
+    }
+}
+
+template <int DMAX, bool GRAD>
+cudaError_t launch_dmax(const SimtPlan& p, const float* q, const float* k, const float* v,
+                        float half_c, float* part, cudaStream_t s) {
+    constexpr int CBLK = 4;
+    dim3 grid(static_cast<unsigned>((p.M + THREADS - 1) / THREADS), p.splits,
+              GRAD ? 1u : static_cast<unsigned>((p.Cv + CBLK - 1) / CBLK));
+    simt_gauss_kernel<DMAX, CBLK, GRAD><<<grid, THREADS, 0, s>>>(
+        q, k, v, p.M, p.N, static_cast<int>(p.D), static_cast<int>(p.Cv), half_c,
+        p.keys_per_split, part);
+    return cudaGetLastError();
+}
+
+}  // namespace
+
+bool plan_simt(int64_t M, int64_t N, int64_t D, int64_t C, bool grad, int split_override,
+               int sms, SimtPlan* p, const char** why) {
+    p->M = M;
+    p->N = N;
+    p->D = D;
+    p->Cv = grad ? D + 1 : C;
+    const int64_t dlimit = grad ? 64 : 128;
+    if (D > dlimit) {
+        *why = grad ? "fp32 gradient supports D <= 64" : "fp32 path supports D <= 128";
+        return false;
+    }
+    p->dmax = D <= 16 ? 16 : D <= 32 ? 32 : D <= 64 ? 64 : 128;
+    p->cblk = 4;
+    const int64_t rowblocks = (M + THREADS - 1) / THREADS;
+    const int64_t chunks = grad ? 1 : (p->Cv + 3) / 4;
+    const int64_t key_tiles = (N + KT - 1) / KT;
+    int64_t splits = split_override > 0 ? split_override
+                                        : (4LL * sms + rowblocks * chunks - 1) / (rowblocks * chunks);
+    splits = std::max<int64_t>(1, std::min<int64_t>(splits, std::max<int64_t>(1, key_tiles)));
+    splits = std::min<int64_t>(splits, 65535);
+    const int64_t tiles_per_split = (key_tiles + splits - 1) / splits;
+    p->keys_per_split = std::max<int64_t>(KT, tiles_per_split * KT);
+    p->splits = static_cast<int>((N + p->keys_per_split - 1) / p->keys_per_split);
+    if (p->splits < 1) p->splits = 1;
+    p->off_part = 0;
+    p->total = static_cast<size_t>(p->splits) * M * p->Cv * sizeof(float);
+    p->total = (p->total + 1023) & ~static_cast<size_t>(1023);
+    return true;
+}
+
+cudaError_t launch_simt(const SimtPlan& p, bool grad, const float* q, const float* k,
+                        const float* v, float half_c, float* part, cudaStream_t s) {
+    if (grad) {
+        switch (p.dmax) {
+            case 16: return launch_dmax<16, true>(p, q, k, v, half_c, part, s);
+            case 32: return launch_dmax<32, true>(p, q, k, v, half_c, part, s);
+            default: return launch_dmax<64, true>(p, q, k, v, half_c, part, s);
+        }
+    }
+    switch (p.dmax) {
+        case 16: return launch_dmax<16, false>(p, q, k, v, half_c, part, s);
+        case 32: return launch_dmax<32, false>(p, q, k, v, half_c, part, s);
+        case 64: return launch_dmax<64, false>(p, q, k, v, half_c, part, s);
+        default: return launch_dmax<128, false>(p, q, k, v, half_c, part, s);
+    }
+}
+
+}  // namespace gs

@@ -1,0 +1,218 @@
+"""GPU parity: the CUDA path against the float64 oracle, element by element.
+
+Tolerance (per output): rel = |s_gpu - s_oracle| / (sum_n Phi |v_n| + 1e-30)
+must stay <= 2e-3 for fp16/bf16 inputs (fp16/bf16 MMA operands, fp32
+accumulation) and <= 1e-5 for the fp32 SIMT path.  Shapes span several row
+and key tiles with ragged tails; all calls go through the C ABI.
+"""
+import numpy as np
+import pytest
+
+from tests.gpu_helpers import TOL, case, device_inputs, forward_check, grad_check, rel_err
+
+pytestmark = pytest.mark.gpu
+
+torch = pytest.importorskip("torch")
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _gpu():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    from paper_2609_04910_gb300.build import build_library
+    build_library()
+    torch.cuda.set_device(0)
+
+
+FWD_CASES = [
+    # M, N, D, C, dtype
+    (1, 1, 1, 1, "fp16"), (7, 130, 3, 1, "fp16"), (128, 128, 16, 16, "fp16"),
+    (129, 257, 17, 2, "fp16"), (300, 1000, 64, 1, "fp16"), (257, 300, 100, 33, "fp16"),
+    (130, 200, 128, 64, "fp16"), (64, 300, 255, 4, "fp16"), (200, 150, 256, 200, "fp16"),
+    (100, 129, 32, 15, "fp16"), (513, 700, 8, 17, "fp16"), (90, 2000, 64, 128, "fp16"),
+    (1, 1, 1, 1, "bf16"), (129, 257, 17, 2, "bf16"), (300, 500, 128, 64, "bf16"),
+    (77, 260, 256, 1, "bf16"),
+    (1, 1, 1, 1, "fp32"), (7, 130, 3, 1, "fp32"), (129, 257, 17, 2, "fp32"),
+    (300, 1000, 64, 5, "fp32"), (100, 200, 128, 3, "fp32"), (50, 70, 32, 9, "fp32"),
+]
+
+
+@pytest.mark.parametrize("M,N,D,C,dtype", FWD_CASES)
+def test_forward_parity(M, N, D, C, dtype):
+    forward_check(case(M, N, D, C, dtype))
+
+
+@pytest.mark.parametrize("dtype", ["fp16", "bf16", "fp32"])
+def test_forward_q_aliases_k(dtype):
+    forward_check(case(300, 300, 64, 1, dtype, kind="mmd", q_is_k=True))
+
+
+@pytest.mark.parametrize("split_n", [1, 2, 3, 7])
+def test_key_splits(split_n):
+    forward_check(case(260, 1500, 64, 3, "fp16"), split_n=split_n)
+
+
+@pytest.mark.parametrize("dtype", ["fp16", "bf16"])
+def test_centering_off(dtype):
+    forward_check(case(200, 400, 32, 2, dtype), center=False)
+
+
+GRAD_CASES = [
+    (300, 300, 32, "fp16", True), (129, 200, 17, "fp16", False), (150, 150, 64, "bf16", True),
+    (64, 500, 100, "fp16", False), (40, 90, 255, "fp16", False),
+    (100, 130, 16, "fp32", False), (64, 64, 64, "fp32", True), (33, 80, 5, "fp32", False),
+]
+
+
+@pytest.mark.parametrize("M,N,D,dtype,alias", GRAD_CASES)
+def test_grad_parity(M, N, D, dtype, alias):
+    grad_check(case(M, N, D, 1, dtype, kind="mmd" if alias else "normal", q_is_k=alias))
+
+
+# ---------------------------------------------------------------- edge values
+def _call(q, k, v, tau, **kw):
+    import paper_2609_04910_gb300 as gs
+    s = gs.gauss_sum(q, k, v, tau, **kw)
+    gs.gauss_sum_device_status()
+    return s
+
+
+@pytest.mark.parametrize("dtype", ["fp16", "fp32"])
+def test_zero_values_give_zero(dtype):
+    tdt = {"fp16": torch.float16, "fp32": torch.float32}[dtype]
+    q = torch.randn(200, 20, device="cuda", dtype=tdt)
+    k = torch.randn(300, 20, device="cuda", dtype=tdt)
+    v = torch.zeros(300, 3, device="cuda", dtype=tdt)
+    assert torch.count_nonzero(_call(q, k, v, 0.5)).item() == 0
+
+
+@pytest.mark.parametrize("dtype", ["fp16", "bf16", "fp32"])
+def test_tiny_tau_gives_plain_sum(dtype):
+    forward_check(case(150, 400, 24, 2, dtype, tau=1e-6))
+
+
+@pytest.mark.parametrize("dtype", ["fp16", "fp32"])
+def test_large_tau_coincident_points(dtype):
+    # q = k, tau large: the self pair (exponent exactly 0) dominates.
+    forward_check(case(260, 260, 16, 1, dtype, tau=40.0, kind="mmd", q_is_k=True))
+
+
+def test_far_points_underflow_to_zero():
+    q = torch.zeros(130, 8, device="cuda", dtype=torch.float16)
+    k = torch.full((140, 8), 60.0, device="cuda", dtype=torch.float16)
+    v = torch.ones(140, 2, device="cuda", dtype=torch.float16)
+    s = _call(q, k, v, 1.0)
+    assert torch.count_nonzero(s).item() == 0
+
+
+def test_fp16_kernel_value_floor():
+    """Kernel values below 2^-29 may be flushed (fp16 P stored with a +15
+    exponent shift); the error stays below tol * den + sum of flushed terms."""
+    from oracle import oracle_sum
+    rng = np.random.default_rng(5)
+    M, N, D = 64, 300, 4
+    q = rng.standard_normal((M, D)).astype(np.float16)
+    k = (rng.standard_normal((N, D)) * 3.0).astype(np.float16)
+    v = rng.standard_normal((N, 1)).astype(np.float16)
+    tau = 3.0
+    s = _call(torch.from_numpy(q).cuda(), torch.from_numpy(k).cuda(), torch.from_numpy(v).cuda(), tau)
+    ref, den = oracle_sum(q, k, v, tau)
+    d2 = ((q.astype(np.float64)[:, None, :] - k.astype(np.float64)[None]) ** 2).sum(-1)
+    phi = np.exp(-tau / 2 * d2)
+    flushed = (phi * (phi < 2.0 ** -28) * np.abs(v.astype(np.float64)[:, 0])[None]).sum(1)
+    err = np.abs(s.cpu().numpy()[:, 0] - ref[:, 0])
+    assert np.all(err <= 2e-3 * den[:, 0] + flushed + 1e-30)
+
+
+def test_deterministic_bitwise():
+    import paper_2609_04910_gb300 as gs
+    from paper_2609_04910_gb300.workloads import generate
+    w = case(300, 900, 64, 4, "fp16")
+    q, k, v = device_inputs(generate(w))
+    a = gs.gauss_sum(q, k, v, w.tau)
+    b = gs.gauss_sum(q, k, v, w.tau)
+    torch.cuda.synchronize()
+    assert torch.equal(a, b)
+
+
+def test_output_guards_and_prefill():
+    import paper_2609_04910_gb300 as gs
+    from paper_2609_04910_gb300.workloads import generate
+    w = case(130, 260, 32, 3, "fp16")
+    q, k, v = device_inputs(generate(w))
+    guard = 1024
+    buf = torch.full((guard + 130 * 3 + guard,), float("nan"), device="cuda")
+    sentinel = 12345.5
+    buf[:guard] = sentinel
+    buf[-guard:] = sentinel
+    out = buf[guard:guard + 130 * 3].view(130, 3)
+    gs.gauss_sum(q, k, v, w.tau, out=out)
+    gs.gauss_sum_device_status()
+    assert torch.all(buf[:guard] == sentinel) and torch.all(buf[-guard:] == sentinel)
+    assert not torch.isnan(out).any()
+
+
+def test_empty_inputs():
+    import paper_2609_04910_gb300 as gs
+    q = torch.randn(5, 4, device="cuda", dtype=torch.float16)
+    k = torch.randn(0, 4, device="cuda", dtype=torch.float16)
+    v = torch.randn(0, 2, device="cuda", dtype=torch.float16)
+    out = torch.full((5, 2), 7.0, device="cuda")
+    gs.gauss_sum(q, k, v, 1.0, out=out)
+    torch.cuda.synchronize()
+    assert torch.count_nonzero(out).item() == 0
+    q0 = torch.randn(0, 4, device="cuda", dtype=torch.float16)
+    assert gs.gauss_sum(q0, q, torch.ones(5, 1, device="cuda", dtype=torch.float16), 1.0).shape == (0, 1)
+
+
+def test_caller_workspace_matches_allocated():
+    import paper_2609_04910_gb300 as gs
+    from paper_2609_04910_gb300.workloads import generate
+    w = case(200, 700, 48, 5, "fp16")
+    q, k, v = device_inputs(generate(w))
+    a = gs.gauss_sum(q, k, v, w.tau)
+    n = gs.gauss_sum_workspace_size(200, 700, 48, 5, gs.GS_FP16)
+    ws = torch.empty(n, dtype=torch.uint8, device="cuda")
+    b = gs.gauss_sum(q, k, v, w.tau, workspace=ws)
+    torch.cuda.synchronize()
+    assert torch.equal(a, b)
+    small = torch.empty(max(n // 2, 256), dtype=torch.uint8, device="cuda")
+    with pytest.raises(gs.GaussSumError) as ei:
+        gs.gauss_sum(q, k, v, w.tau, workspace=small)
+    assert ei.value.status == 3
+
+
+def test_unsupported_shapes_raise():
+    import paper_2609_04910_gb300 as gs
+    q = torch.randn(4, 300, device="cuda", dtype=torch.float16)
+    v = torch.ones(4, 1, device="cuda", dtype=torch.float16)
+    with pytest.raises(gs.GaussSumError) as ei:
+        gs.gauss_sum(q, q, v, 1.0)
+    assert ei.value.status == 2
+
+
+def test_forced_allocation_failure(monkeypatch):
+    import paper_2609_04910_gb300 as gs
+    q = torch.randn(4, 8, device="cuda", dtype=torch.float16)
+    v = torch.ones(4, 1, device="cuda", dtype=torch.float16)
+    monkeypatch.setenv("GS_TEST_FAIL_ALLOC", "1")
+    with pytest.raises(gs.GaussSumError) as ei:
+        gs.gauss_sum(q, q, v, 1.0)
+    assert ei.value.status == 3
+    monkeypatch.delenv("GS_TEST_FAIL_ALLOC")
+    gs.gauss_sum(q, q, v, 1.0)
+    torch.cuda.synchronize()
+
+
+def test_stream_ordering_on_side_stream():
+    import paper_2609_04910_gb300 as gs
+    from paper_2609_04910_gb300.workloads import generate
+    w = case(257, 600, 64, 2, "fp16")
+    q, k, v = device_inputs(generate(w))
+    ref = gs.gauss_sum(q, k, v, w.tau)
+    s = torch.cuda.Stream()
+    s.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.stream(s):
+        out = gs.gauss_sum(q, k, v, w.tau)
+    s.synchronize()
+    assert torch.equal(out, ref)
