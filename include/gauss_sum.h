@@ -74,6 +74,11 @@ typedef enum { GS_PATH_AUTO = 0, GS_PATH_TENSOR = 1, GS_PATH_SIMT = 2 } gs_path;
  *  path            GS_PATH_AUTO picks the tensor-core kernel for fp16/bf16
  *                  and the SIMT kernel for fp32; GS_PATH_TENSOR rejects fp32,
  *                  GS_PATH_SIMT rejects fp16/bf16.
+ *  main_events     measurement hook: two cudaEvent_t handles (or NULL) that
+ *                  the call records on `stream` immediately before and after
+ *                  the launch of its main kernel (the fused tensor-core
+ *                  kernel, or the fp32 SIMT kernel), so a caller can time
+ *                  that kernel alone.  The caller owns the events.
  */
 typedef struct gs_options {
     int center;
@@ -81,6 +86,7 @@ typedef struct gs_options {
     void* workspace;
     size_t workspace_bytes;
     int path;
+    void* main_events[2];
 } gs_options;
 
 /* Fill *opt with the defaults (center = 1, split_n = 0, no workspace, auto path). */

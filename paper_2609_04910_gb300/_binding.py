@@ -38,7 +38,7 @@ class GaussSumError(RuntimeError):
 class GsOptions(ctypes.Structure):
     _fields_ = [("center", ctypes.c_int), ("split_n", ctypes.c_int),
                 ("workspace", ctypes.c_void_p), ("workspace_bytes", ctypes.c_size_t),
-                ("path", ctypes.c_int)]
+                ("path", ctypes.c_int), ("main_events", ctypes.c_void_p * 2)]
 
 
 _lock = threading.Lock()
@@ -99,7 +99,11 @@ def _check(lib, status: int):
         raise GaussSumError(status, lib.gauss_sum_last_error().decode())
 
 
-def options(center=True, split_n=0, workspace=None, workspace_bytes=0, path=GS_PATH_AUTO):
+def options(center=True, split_n=0, workspace=None, workspace_bytes=0, path=GS_PATH_AUTO,
+            main_events=None):
+    """gs_options; ``main_events`` is an optional pair of torch.cuda.Event
+    (already recorded once, so that their CUDA events exist) that the call
+    records around its main kernel."""
     o = GsOptions()
     load_library().gauss_sum_default_options(ctypes.byref(o))
     o.center = 1 if center else 0
@@ -107,6 +111,9 @@ def options(center=True, split_n=0, workspace=None, workspace_bytes=0, path=GS_P
     o.workspace = workspace
     o.workspace_bytes = int(workspace_bytes)
     o.path = int(path)
+    if main_events is not None:
+        o.main_events[0] = main_events[0].cuda_event
+        o.main_events[1] = main_events[1].cuda_event
     return o
 
 
@@ -139,7 +146,8 @@ def _check_tensor(t, name):
         raise ValueError(f"{name} must be contiguous")
 
 
-def gauss_sum(q, k, v, tau, out=None, stream=None, center=True, split_n=0, workspace=None):
+def gauss_sum(q, k, v, tau, out=None, stream=None, center=True, split_n=0, workspace=None,
+              main_events=None):
     """Eq. 1: s[m] = sum_n exp(-tau/2 ||q_m - k_n||^2) v[n] as an (M, C) fp32 tensor.
 
     q: (M, D), k: (N, D), v: (N, C) or (N,) CUDA tensors of one dtype
@@ -156,7 +164,8 @@ def gauss_sum(q, k, v, tau, out=None, stream=None, center=True, split_n=0, works
         out = torch.empty((M, C), dtype=torch.float32, device=q.device)
     opt = options(center=center, split_n=split_n,
                   workspace=None if workspace is None else workspace.data_ptr(),
-                  workspace_bytes=0 if workspace is None else workspace.numel() * workspace.element_size())
+                  workspace_bytes=0 if workspace is None else workspace.numel() * workspace.element_size(),
+                  main_events=main_events)
     st = lib.gauss_sum_ex(_ptr(q), _ptr(k), _ptr(v), float(tau), M, N, D, C, _dtype_code(q),
                           _ptr(out), _stream_ptr(stream), ctypes.byref(opt))
     _check(lib, st)
@@ -164,7 +173,7 @@ def gauss_sum(q, k, v, tau, out=None, stream=None, center=True, split_n=0, works
 
 
 def gauss_sum_grad_q(q, k, v, tau, grad=None, s_out=None, want_s=True, stream=None,
-                     center=True, split_n=0, workspace=None):
+                     center=True, split_n=0, workspace=None, main_events=None):
     """Sec. 3 q-gradient for scalar weights.  Returns (grad (M, D), s (M,) or None)."""
     import torch
     lib = load_library()
@@ -178,7 +187,8 @@ def gauss_sum_grad_q(q, k, v, tau, grad=None, s_out=None, want_s=True, stream=No
         s_out = torch.empty((M,), dtype=torch.float32, device=q.device)
     opt = options(center=center, split_n=split_n,
                   workspace=None if workspace is None else workspace.data_ptr(),
-                  workspace_bytes=0 if workspace is None else workspace.numel() * workspace.element_size())
+                  workspace_bytes=0 if workspace is None else workspace.numel() * workspace.element_size(),
+                  main_events=main_events)
     st = lib.gauss_sum_grad_q_ex(_ptr(q), _ptr(k), _ptr(v), float(tau), M, N, D, _dtype_code(q),
                                  _ptr(grad), _ptr(s_out), _stream_ptr(stream), ctypes.byref(opt))
     _check(lib, st)

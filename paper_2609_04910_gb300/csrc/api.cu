@@ -127,6 +127,10 @@ gs_status plan(const Call& c, int sms, bool* tensor, gs::TcPlan* tp, gs::SimtPla
     return GS_OK;
 }
 
+cudaError_t record_event(void* ev, cudaStream_t s) {
+    return ev ? cudaEventRecord(static_cast<cudaEvent_t>(ev), s) : cudaSuccess;
+}
+
 // Test hook: GS_TEST_FAIL_ALLOC=1 makes the workspace allocation fail.
 bool forced_alloc_failure() {
     const char* s = std::getenv("GS_TEST_FAIL_ALLOC");
@@ -217,7 +221,9 @@ gs_status run(Call c) {
             where = "value kernel";
         }
         if (e == cudaSuccess) {
-            e = gs::launch_tc(tp, t, cexp, ws, status, c.stream, &why);
+            e = record_event(c.opt.main_events[0], c.stream);
+            if (e == cudaSuccess) e = gs::launch_tc(tp, t, cexp, ws, status, c.stream, &why);
+            if (e == cudaSuccess) e = record_event(c.opt.main_events[1], c.stream);
             where = "fused tensor-core kernel";
         }
         if (e == cudaSuccess) {
@@ -230,9 +236,12 @@ gs_status run(Call c) {
         }
     } else {
         float* part = reinterpret_cast<float*>(ws + sp.off_part);
-        e = gs::launch_simt(sp, c.grad, static_cast<const float*>(c.q),
-                            static_cast<const float*>(c.k), static_cast<const float*>(c.v), half_c,
-                            part, c.stream);
+        e = record_event(c.opt.main_events[0], c.stream);
+        if (e == cudaSuccess)
+            e = gs::launch_simt(sp, c.grad, static_cast<const float*>(c.q),
+                                static_cast<const float*>(c.k), static_cast<const float*>(c.v),
+                                half_c, part, c.stream);
+        if (e == cudaSuccess) e = record_event(c.opt.main_events[1], c.stream);
         where = "fp32 kernel";
         if (e == cudaSuccess) {
             e = gs::launch_finalize(c.grad ? 2 : 0, gs::InType::F32, part, sp.splits, c.M, c.M,
@@ -260,6 +269,8 @@ gs_options defaults() {
     o.workspace = nullptr;
     o.workspace_bytes = 0;
     o.path = GS_PATH_AUTO;
+    o.main_events[0] = nullptr;
+    o.main_events[1] = nullptr;
     return o;
 }
 

@@ -178,6 +178,23 @@ def generate(w: Workload, seed: int = 0) -> dict:
     }
 
 
+def to_device(a: np.ndarray, dtype: str, dev="cuda:0"):
+    """Copy a ``round_to`` array to a torch device tensor of the storage dtype."""
+    import torch
+    if dtype == "bf16":
+        return torch.from_numpy(np.ascontiguousarray(a).view(np.int16)).to(dev).view(torch.bfloat16)
+    return torch.from_numpy(np.ascontiguousarray(a)).to(dev)
+
+
+def device_inputs(inp: dict, dev="cuda:0"):
+    """(q, k, v) device tensors of a ``generate`` result; q is k when aliased."""
+    w = inp["workload"]
+    k = to_device(inp["k"], w.dtype, dev)
+    q = k if inp["q"] is inp["k"] else to_device(inp["q"], w.dtype, dev)
+    v = to_device(inp["v"], w.dtype, dev)
+    return q, k, v
+
+
 def sample_rows(M: int, count: int, seed: int = 1) -> np.ndarray:
     """Seeded, sorted subset of row indices for checks on large M."""
     if count >= M:

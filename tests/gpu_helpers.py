@@ -3,24 +3,9 @@ call the library through its C ABI, and compare with the float64 oracle."""
 import numpy as np
 
 from oracle import oracle_grad_q, oracle_sum
-from paper_2609_04910_gb300.workloads import Workload, generate
+from paper_2609_04910_gb300.workloads import Workload, device_inputs, generate, to_device  # noqa: F401
 
 TOL = {"fp32": 1e-5, "fp16": 2e-3, "bf16": 2e-3}
-
-
-def to_device(a, dtype, dev="cuda:0"):
-    import torch
-    if dtype == "bf16":
-        return torch.from_numpy(np.ascontiguousarray(a).view(np.int16)).to(dev).view(torch.bfloat16)
-    return torch.from_numpy(np.ascontiguousarray(a)).to(dev)
-
-
-def device_inputs(inp, dev="cuda:0"):
-    w = inp["workload"]
-    k = to_device(inp["k"], w.dtype, dev)
-    q = k if inp["q"] is inp["k"] else to_device(inp["q"], w.dtype, dev)
-    v = to_device(inp["v"], w.dtype, dev)
-    return q, k, v
 
 
 def rel_err(got, ref, den):

@@ -45,6 +45,7 @@ def test_default_options(lib):
     o.center = 7
     lib.gauss_sum_default_options(ctypes.byref(o))
     assert (o.center, o.split_n, o.workspace, o.workspace_bytes, o.path) == (1, 0, None, 0, 0)
+    assert list(o.main_events) == [None, None]
 
 
 ALIGNED = 4096  # a fake 16-byte-aligned address; never dereferenced
