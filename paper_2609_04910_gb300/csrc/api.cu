@@ -213,7 +213,12 @@ gs_status run(Call c) {
                                             reinterpret_cast<float*>(ws + tp.off_B), ninf, c.stream);
             where = "centre/cast kernel (k)";
         }
-        if (e == cudaSuccess) {
+        if (e == cudaSuccess && tp.fma) {
+            e = gs::launch_key_records(t, c.v, reinterpret_cast<const float*>(ws + tp.off_B), c.N,
+                                       tp.Npad, static_cast<int>(tp.Cv),
+                                       reinterpret_cast<float*>(ws + tp.off_rec), c.stream);
+            where = "key-record kernel";
+        } else if (e == cudaSuccess) {
             e = gs::launch_value_prep(t, c.grad, c.v, c.k, mu, c.N, tp.Npad, static_cast<int>(c.D),
                                       static_cast<int>(tp.Cv), tp.Cp,
                                       reinterpret_cast<unsigned*>(ws + tp.off_vmax), ws + tp.off_vt,
@@ -222,16 +227,26 @@ gs_status run(Call c) {
         }
         if (e == cudaSuccess) {
             e = record_event(c.opt.main_events[0], c.stream);
-            if (e == cudaSuccess) e = gs::launch_tc(tp, t, cexp, ws, status, c.stream, &why);
+            if (e == cudaSuccess)
+                e = tp.fma ? gs::launch_tc_fma(tp, t, cexp, ws, status, c.stream, &why)
+                           : gs::launch_tc(tp, t, cexp, ws, status, c.stream, &why);
             if (e == cudaSuccess) e = record_event(c.opt.main_events[1], c.stream);
             where = "fused tensor-core kernel";
         }
         if (e == cudaSuccess) {
-            e = gs::launch_finalize(c.grad ? 1 : 0, t, reinterpret_cast<float*>(ws + tp.off_part),
-                                    tp.splits, tp.Mpad, c.M, static_cast<int>(tp.Cv), tp.Cp,
-                                    reinterpret_cast<float*>(ws + tp.off_inv), c.q, mu,
-                                    static_cast<float>(c.tau), static_cast<int>(c.D), c.out,
-                                    c.s_out, c.stream);
+            if (tp.fma)
+                e = gs::launch_finalize(0, t, reinterpret_cast<float*>(ws + tp.off_part), tp.splits,
+                                        tp.Mpad, c.M, static_cast<int>(tp.Cv),
+                                        static_cast<int>(tp.Cv), nullptr, nullptr, nullptr,
+                                        static_cast<float>(c.tau), static_cast<int>(c.D), c.out,
+                                        nullptr, c.stream);
+            else
+                e = gs::launch_finalize(c.grad ? 1 : 0, t,
+                                        reinterpret_cast<float*>(ws + tp.off_part), tp.splits,
+                                        tp.Mpad, c.M, static_cast<int>(tp.Cv), tp.Cp,
+                                        reinterpret_cast<float*>(ws + tp.off_inv), c.q, mu,
+                                        static_cast<float>(c.tau), static_cast<int>(c.D), c.out,
+                                        c.s_out, c.stream);
             where = "finalise kernel";
         }
     } else {

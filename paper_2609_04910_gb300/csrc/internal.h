@@ -9,6 +9,10 @@ namespace gs {
 
 enum class InType { F32 = 0, F16 = 1, BF16 = 2 };
 
+// Largest value-channel count evaluated on the FMA pipe (the P.v product of
+// tc_gauss_fma.cu); more channels use the two-MMA kernel of tc_gauss.cu.
+constexpr int kFmaMaxChannels = 4;
+
 // Workspace plan of the tensor-core path.  All offsets are bytes from the
 // workspace base and are 1024-byte aligned.
 struct TcPlan {
@@ -22,8 +26,10 @@ struct TcPlan {
     int mean_blocks;
     bool alias;              // q and k are the same array (M == N): prep once
     bool center;
+    bool fma;                // kernel of tc_gauss_fma.cu (C <= kFmaMaxChannels, forward)
+    int nq;                  // query tiles of 128 rows per CTA (FMA kernel)
     size_t off_mean_part, off_mu, off_qh, off_kh, off_A, off_B, off_vt, off_vmax, off_inv,
-        off_part, total;
+        off_rec, off_part, total;
 };
 
 struct SimtPlan {
@@ -64,9 +70,19 @@ cudaError_t launch_finalize(int mode, InType t, const float* part, int splits,
 cudaError_t launch_simt(const SimtPlan& p, bool grad, const float* q, const float* k,
                         const float* v, float half_c, float* part, cudaStream_t s);
 
+// Key records of the FMA kernel: per key pair (2t, 2t+1) the floats
+// B_2t, B_2t+1, v_2t[0], v_2t+1[0], ..., v_2t[C-1], v_2t+1[C-1].
+cudaError_t launch_key_records(InType t, const void* v, const float* B, int64_t N, int64_t Npad,
+                               int C, float* rec, cudaStream_t s);
+
 // tc_gauss.cu ----------------------------------------------------------
 cudaError_t launch_tc(const TcPlan& p, InType t, float c, char* ws, unsigned* status,
                       cudaStream_t s, const char** why);
+
+// tc_gauss_fma.cu ------------------------------------------------------
+bool plan_fma_kernel(int Dp, int C, int* nq, int* stages, size_t* smem);
+cudaError_t launch_tc_fma(const TcPlan& p, InType t, float c, char* ws, unsigned* status,
+                          cudaStream_t s, const char** why);
 
 // probe
 cudaError_t run_ex2_probe(cudaStream_t s, double* rate);

@@ -197,6 +197,24 @@ __global__ void value_prep_kernel(const T* __restrict__ v, const T* __restrict__
     }
 }
 
+// ---------------------------------------------------------------- key records
+// One thread per key pair t: B_2t, B_2t+1, then the values of both keys
+// channel by channel, in fp32 (zero for padded keys).
+template <typename T>
+__global__ void key_record_kernel(const T* __restrict__ v, const float* __restrict__ B, int64_t N,
+                                  int64_t pairs, int C, float* __restrict__ rec) {
+    const int64_t t = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
+    if (t >= pairs) return;
+    const int64_t n0 = 2 * t, n1 = 2 * t + 1;
+    float* out = rec + t * (2 + 2 * C);
+    out[0] = B[n0];
+    out[1] = B[n1];
+    for (int c = 0; c < C; ++c) {
+        out[2 + 2 * c] = n0 < N ? to_f(v[n0 * C + c]) : 0.f;
+        out[3 + 2 * c] = n1 < N ? to_f(v[n1 * C + c]) : 0.f;
+    }
+}
+
 // ---------------------------------------------------------------- finalise
 // part: splits blocks of split_stride_rows rows x part_ld floats.
 template <int MODE, typename T>
@@ -329,6 +347,21 @@ cudaError_t launch_value_prep(InType t, bool grad, const void* v, const void* k,
                                                  inv_scale, s)
                 : value_prep_typed<__half, false>(v, k, mu, N, Npad, D, Cv, Cp, vmax_bits, vt,
                                                   inv_scale, s);
+}
+
+cudaError_t launch_key_records(InType t, const void* v, const float* B, int64_t N, int64_t Npad,
+                               int C, float* rec, cudaStream_t s) {
+    const int64_t pairs = Npad / 2;
+    if (pairs == 0) return cudaSuccess;
+    const int threads = 256;
+    const unsigned blocks = static_cast<unsigned>((pairs + threads - 1) / threads);
+    if (t == InType::BF16)
+        key_record_kernel<__nv_bfloat16><<<blocks, threads, 0, s>>>(
+            static_cast<const __nv_bfloat16*>(v), B, N, pairs, C, rec);
+    else
+        key_record_kernel<__half><<<blocks, threads, 0, s>>>(static_cast<const __half*>(v), B, N,
+                                                             pairs, C, rec);
+    return cudaGetLastError();
 }
 
 cudaError_t launch_finalize(int mode, InType t, const float* part, int splits,

@@ -12,44 +12,45 @@
 //
 //   MMA1  S   = q^ k^T          tcgen05.mma kind::f16, A,B from shared memory,
 //                               fp32 accumulator in TMEM (128 x BN)
-//   exp   P   = fp16(2^min(c S + A_m + B_n + 15, 15)) TMEM -> registers -> TMEM
+//   exp   P   = fp16(2^(c S + A_m + B_n + 15))   TMEM -> registers -> TMEM
 //   MMA2  O  += P v~            tcgen05.mma kind::f16, A = P from TMEM,
 //                               B = value tile from shared memory, fp32 TMEM
 //
-// Warp roles (320 threads):
-//   warps 0-7  exponent warps; warp w owns TMEM lanes 32 (w % 4) .. +31 (its
-//              hardware lane quarter) and half (w / 4) of the key columns;
-//              they also run the epilogue (TMEM O -> fp32 partial sums).
-//   warp 8     TMA producer: q^ tile once, then k^ / v~ / B tiles into a
+// Warp roles ((NEXP + 2) x 32 threads; NEXP = 16 for BN = 128, 8 for BN = 64):
+//   warps 0 .. NEXP-1  exponent warps in two groups of NEXP/2; group g
+//              handles the key tiles j = g (mod 2).  Warp w owns TMEM lanes
+//              32 (w % 4) .. +31 (its hardware lane quarter) and a share of
+//              the key columns; all of them run the epilogue (TMEM O -> fp32
+//              partial sums).
+//   warp NEXP  TMA producer: q^ tile once, then k^ / v~ / B tiles into a
 //              ring of `stages` shared-memory stages.
-//   warp 9     TMEM allocator and single-thread MMA issuer.
+//   warp NEXP+1  TMEM allocator and single-thread MMA issuer.
 // TMEM columns: S double buffer [0, 2 BN), P double buffer [2 BN, 3 BN)
 // (fp16 pairs packed in 32-bit columns), O accumulator [3 BN, 3 BN + Cp).
-// MMA1 of tile j overlaps the exponent work of tile j - 1; MMA2 of tile
-// j - 1 is issued after MMA1 of tile j.
+// MMA1 of tile j + 1 and the exponent work of tile j (one group) overlap the
+// exponent work of tile j - 1 (the other group); MMA2 of tile j - 1 is
+// issued after MMA1 of tile j.
 #include <cuda.h>
-#include <cudaTypedefs.h>
 #include <cuda_runtime.h>
 
 #include <algorithm>
-#include <mutex>
 
 #include "internal.h"
 #include "ptx.cuh"
+#include "tensor_map.h"
 
 namespace gs {
 namespace {
 
 constexpr int BM = 128;           // query rows per CTA (MMA M)
 constexpr int KB = 64;            // 16-bit elements per 128-byte swizzled row
-constexpr int NUM_EXP_WARPS = 8;
-constexpr int PRODUCER_WARP = 8;
-constexpr int MMA_WARP = 9;
-constexpr int THREADS = 320;
 constexpr uint32_t TMEM_COLS = 512;
 // P is stored as fp16(2^(x + P_SHIFT)): since x <= 0 the stored value is at
 // most 2^15 < 65504, and kernel values down to 2^-29 stay normal fp16
 // numbers (instead of 2^-14).  The epilogue multiplies O by 2^-P_SHIFT.
+// x is not clamped: a rounding-positive exponent (x slightly above 0) is
+// kept as is, and the saturating fp16 conversion bounds P by 65504, i.e.
+// the kernel value by 65504 / 2^15 < 2, so that no inf can reach the MMA.
 constexpr float P_SHIFT = 15.f;
 constexpr float P_UNSHIFT = 1.f / 32768.f;
 
@@ -91,10 +92,26 @@ __device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity, volati
     return __all_sync(0xffffffffu, ok);
 }
 
-template <int BN>
-__global__ void __launch_bounds__(THREADS, 1)
+// Threads of a CTA with NEXP exponent warps plus the producer and MMA warps.
+template <int NEXP>
+constexpr int cta_threads() { return (NEXP + 2) * 32; }
+
+template <int BN, int NEXP>
+__global__ void __launch_bounds__(cta_threads<NEXP>(), 1)
 tc_gauss_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
                 const __grid_constant__ CUtensorMap tm_v, const TcParams p) {
+    static_assert(NEXP % 4 == 0, "exponent warps cover the four TMEM lane quarters");
+    constexpr int PRODUCER_WARP = NEXP;
+    constexpr int MMA_WARP = NEXP + 1;
+    // The exponent warps form two groups; group g handles the key tiles
+    // j = g (mod 2), i.e. S/P buffer g, so that one group's TMEM and MMA
+    // latency overlaps the other group's exp2 work.
+    constexpr int GROUP_WARPS = NEXP / 2;
+    constexpr int COLS = BN * 4 / GROUP_WARPS;  // key columns per exponent warp and tile
+    constexpr int NCH = COLS / 32;              // 32-column TMEM loads per warp and tile
+    static_assert(GROUP_WARPS % 4 == 0, "each group covers the four TMEM lane quarters");
+    static_assert(COLS % 32 == 0, "exponent warps load whole 32-column chunks");
+
     extern __shared__ uint8_t smem_raw[];
     // 1024-byte aligned base for the 128-byte swizzle atoms.
     const uint32_t raw_addr = smem_u32(smem_raw);
@@ -119,7 +136,7 @@ tc_gauss_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant_
         mbar_init(&bars->drain, 1);
         for (int b = 0; b < 2; ++b) {
             mbar_init(&bars->s_full[b], 1);
-            mbar_init(&bars->p_full[b], NUM_EXP_WARPS * 32);
+            mbar_init(&bars->p_full[b], GROUP_WARPS);  // one arrival per warp
         }
         for (int s = 0; s < p.stages; ++s) {
             mbar_init(&bars->kv_full[s], 1);
@@ -153,10 +170,10 @@ tc_gauss_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant_
             for (int kb = 0; kb < p.nkb; ++kb)
                 tma_load_2d(q_smem + kb * (BM * 128), &tm_q, &bars->q_full, kb * KB, tile_m * BM);
             int issued = 0;
-            for (int j = 0; j < T; ++j) {
-                const int s = j % p.stages;
-                const uint32_t ph = static_cast<uint32_t>(j / p.stages) & 1u;
-                if (!mbar_wait_bounded(&bars->kv_empty[s], ph ^ 1u, abort_flag, p.status)) break;
+            RingPos st;
+            for (int j = 0; j < T; ++j, st.advance(p.stages)) {
+                const int s = st.idx;
+                if (!mbar_wait_bounded(&bars->kv_empty[s], st.phase ^ 1u, abort_flag, p.status)) break;
                 mbar_arrive_expect_tx(&bars->kv_full[s], p.tx_bytes);
                 const int n0 = (kt0 + j) * BN;
                 for (int kb = 0; kb < p.nkb; ++kb)
@@ -176,12 +193,12 @@ tc_gauss_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant_
         if (lane == 0 && T > 0) {
             const uint32_t q_base = smem_u32(q_smem);
             bool ok = mbar_wait_bounded(&bars->q_full, 0, abort_flag, p.status);
+            RingPos st, stp;   // stage of tile j (MMA1) and of tile j - 1 (MMA2)
             for (int j = 0; ok && j <= T; ++j) {
                 if (j < T) {
-                    const int s = j % p.stages;
+                    const int s = st.idx;
                     const int b = j & 1;
-                    ok = mbar_wait_bounded(&bars->kv_full[s], static_cast<uint32_t>(j / p.stages) & 1u,
-                                           abort_flag, p.status);
+                    ok = mbar_wait_bounded(&bars->kv_full[s], st.phase, abort_flag, p.status);
                     if (!ok) break;
                     tc_fence_after();
                     const uint32_t kh_base = smem_u32(kh_smem(s));
@@ -192,11 +209,12 @@ tc_gauss_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant_
                         mma_ss_f16(tmem + S_col0 + b * BN, ad, bd, p.idesc1, kk > 0 ? 1u : 0u);
                     }
                     mma_commit(&bars->s_full[b]);
+                    st.advance(p.stages);
                 }
                 if (j >= 1) {
                     const int jp = j - 1;
                     const int bp = jp & 1;
-                    const int sp = jp % p.stages;
+                    const int sp = stp.idx;
                     ok = mbar_wait_bounded(&bars->p_full[bp], static_cast<uint32_t>(jp >> 1) & 1u,
                                            abort_flag, p.status);
                     if (!ok) break;
@@ -208,6 +226,7 @@ tc_gauss_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant_
                                    (jp > 0 || kk > 0) ? 1u : 0u);
                     }
                     mma_commit(&bars->kv_empty[sp]);
+                    stp.advance(p.stages);
                 }
             }
             if (ok) mma_commit(&bars->o_full);
@@ -217,57 +236,68 @@ tc_gauss_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant_
         }
     } else {
         // ------------------------------------------------ exponent warps
+        // Warp w of group g = w / GROUP_WARPS reads TMEM lanes 32 (w % 4) ..
+        // +31 (rows of the tile) and key columns [COLS part, COLS (part + 1))
+        // of S buffer g, part = (w % GROUP_WARPS) / 4.
+        const int group = warp / GROUP_WARPS;
         const int quarter = warp & 3;
-        const int half = warp >> 2;
+        const int part = (warp % GROUP_WARPS) >> 2;
+        const int col0 = part * COLS;
         const int row_local = quarter * 32 + lane;
         const int64_t row = static_cast<int64_t>(tile_m) * BM + row_local;
         const float a_m = p.A[row] + P_SHIFT;
-        const float c = p.c;
+        const uint64_t a2 = f32x2_pack(a_m, a_m);
+        const uint64_t c2 = f32x2_pack(p.c, p.c);
         const uint32_t lane_base = static_cast<uint32_t>(quarter * 32) << 16;
-        constexpr int COLS = BN / 2;  // key columns per warp
         bool ok = true;
-        for (int j = 0; j < T; ++j) {
-            const int b = j & 1;
-            const int s = j % p.stages;
-            ok = warp_wait(&bars->kv_full[s], static_cast<uint32_t>(j / p.stages) & 1u, abort_flag,
-                           p.status);
+        RingPos st;   // stage of key tile j
+        if (group) st.advance(p.stages);
+        for (int j = group; j < T; j += 2, st.advance(p.stages), st.advance(p.stages)) {
+            const int b = group;
+            const int s = st.idx;
+            ok = warp_wait(&bars->kv_full[s], st.phase, abort_flag, p.status);
             if (ok) ok = warp_wait(&bars->s_full[b], static_cast<uint32_t>(j >> 1) & 1u, abort_flag,
                                    p.status);
             if (!ok) break;
             tc_fence_after();
-            const float* Bs = b_smem(s);
+            uint32_t r[NCH][32];
 #pragma unroll
-            for (int ch = 0; ch < COLS / 32; ++ch) {
-                const int col = half * COLS + ch * 32;
-                uint32_t r[32];
-                tmem_ld_32x32b_x32(tmem + lane_base + S_col0 + b * BN + col, r);
-                tmem_wait_ld();
+            for (int ch = 0; ch < NCH; ++ch)
+                tmem_ld_32x32b_x32(tmem + lane_base + S_col0 + b * BN + col0 + ch * 32, r[ch]);
+            tmem_wait_ld();
+            const float* Bs = b_smem(s) + col0;
+#pragma unroll
+            for (int ch = 0; ch < NCH; ++ch) {
                 uint32_t pk[16];
 #pragma unroll
                 for (int i = 0; i < 8; ++i) {
-                    const float4 bb = *reinterpret_cast<const float4*>(Bs + col + 4 * i);
-                    const float x0 = fmaf(c, __uint_as_float(r[4 * i + 0]), a_m + bb.x);
-                    const float x1 = fmaf(c, __uint_as_float(r[4 * i + 1]), a_m + bb.y);
-                    const float x2 = fmaf(c, __uint_as_float(r[4 * i + 2]), a_m + bb.z);
-                    const float x3 = fmaf(c, __uint_as_float(r[4 * i + 3]), a_m + bb.w);
-                    const float p0 = ex2_approx(fminf(x0, P_SHIFT));
-                    const float p1 = ex2_approx(fminf(x1, P_SHIFT));
-                    const float p2 = ex2_approx(fminf(x2, P_SHIFT));
-                    const float p3 = ex2_approx(fminf(x3, P_SHIFT));
-                    pk[2 * i + 0] = pack_half2(p0, p1);
-                    pk[2 * i + 1] = pack_half2(p2, p3);
+                    // x = c S + (A_m + 15) + B_n for four keys, two per f32x2 op.
+                    const float4 bb = *reinterpret_cast<const float4*>(Bs + ch * 32 + 4 * i);
+                    const uint64_t t01 = f32x2_add(f32x2_pack(bb.x, bb.y), a2);
+                    const uint64_t t23 = f32x2_add(f32x2_pack(bb.z, bb.w), a2);
+                    const uint64_t s01 = f32x2_pack(__uint_as_float(r[ch][4 * i + 0]),
+                                                    __uint_as_float(r[ch][4 * i + 1]));
+                    const uint64_t s23 = f32x2_pack(__uint_as_float(r[ch][4 * i + 2]),
+                                                    __uint_as_float(r[ch][4 * i + 3]));
+                    float x0, x1, x2, x3;
+                    f32x2_unpack(f32x2_fma(s01, c2, t01), x0, x1);
+                    f32x2_unpack(f32x2_fma(s23, c2, t23), x2, x3);
+                    pk[2 * i + 0] = pack_half2_satfinite(ex2_approx(x0), ex2_approx(x1));
+                    pk[2 * i + 1] = pack_half2_satfinite(ex2_approx(x2), ex2_approx(x3));
                 }
-                tmem_st_32x32b_x16(tmem + lane_base + P_col0 + b * (BN / 2) + col / 2, pk);
+                tmem_st_32x32b_x16(tmem + lane_base + P_col0 + b * (BN / 2) + (col0 + ch * 32) / 2, pk);
             }
             tmem_wait_st();
             tc_fence_before();
-            mbar_arrive(&bars->p_full[b]);
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&bars->p_full[b]);
         }
         if (ok && T > 0 && warp_wait(&bars->o_full, 0, abort_flag, p.status)) {
             tc_fence_after();
-            const int cols = p.Cp / 2;
             float* out = p.part + (static_cast<int64_t>(split) * p.Mpad + row) * p.Cp;
-            for (int c8 = half * cols; c8 < (half + 1) * cols; c8 += 8) {
+            constexpr int PARTS = NEXP / 4;
+            const int epart = warp >> 2;
+            for (int c8 = epart * 8; c8 < p.Cp; c8 += 8 * PARTS) {
                 uint32_t r[8];
                 tmem_ld_32x32b_x8(tmem + lane_base + O_col + c8, r);
                 tmem_wait_ld();
@@ -290,46 +320,18 @@ tc_gauss_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant_
 }
 
 // ---------------------------------------------------------------- host side
-PFN_cuTensorMapEncodeTiled_v12000 get_encode_fn() {
-    static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
-    static std::once_flag once;
-    std::call_once(once, [] {
-        void* ptr = nullptr;
-        cudaDriverEntryPointQueryResult q;
-        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault,
-                                             &q) == cudaSuccess &&
-            q == cudaDriverEntryPointSuccess)
-            fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(ptr);
-    });
-    return fn;
-}
-
-bool encode_2d(CUtensorMap* map, CUtensorMapDataType dt, const void* base, uint64_t inner,
-               uint64_t outer, uint64_t row_bytes, uint32_t box_inner, uint32_t box_outer) {
-    auto fn = get_encode_fn();
-    if (!fn) return false;
-    cuuint64_t dims[2] = {inner, outer};
-    cuuint64_t strides[1] = {row_bytes};
-    cuuint32_t box[2] = {box_inner, box_outer};
-    cuuint32_t estr[2] = {1, 1};
-    CUresult r = fn(map, dt, 2, const_cast<void*>(base), dims, strides, box, estr,
-                    CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
-                    CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
-    return r == CUDA_SUCCESS;
-}
-
 size_t align1k(size_t x) { return (x + 1023) & ~static_cast<size_t>(1023); }
 
-template <int BN>
+template <int BN, int NEXP>
 cudaError_t launch_bn(const TcPlan& pl, InType t, float c, char* ws, unsigned* status,
                       cudaStream_t s, const char** why) {
     const CUtensorMapDataType hdt =
         t == InType::BF16 ? CU_TENSOR_MAP_DATA_TYPE_BFLOAT16 : CU_TENSOR_MAP_DATA_TYPE_FLOAT16;
     CUtensorMap tm_q, tm_k, tm_v;
-    if (!encode_2d(&tm_q, hdt, ws + pl.off_qh, pl.Dp, pl.Mpad, pl.Dp * 2ull, KB, BM) ||
-        !encode_2d(&tm_k, hdt, ws + pl.off_kh, pl.Dp, pl.Npad, pl.Dp * 2ull, KB, BN) ||
-        !encode_2d(&tm_v, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, ws + pl.off_vt, pl.Npad, pl.Cp,
-                   pl.Npad * 2ull, KB, pl.Cp)) {
+    if (!encode_tile_map_2d(&tm_q, hdt, ws + pl.off_qh, pl.Dp, pl.Mpad, pl.Dp * 2ull, KB, BM) ||
+        !encode_tile_map_2d(&tm_k, hdt, ws + pl.off_kh, pl.Dp, pl.Npad, pl.Dp * 2ull, KB, BN) ||
+        !encode_tile_map_2d(&tm_v, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, ws + pl.off_vt, pl.Npad,
+                            pl.Cp, pl.Npad * 2ull, KB, pl.Cp)) {
         *why = "cuTensorMapEncodeTiled failed or is unavailable";
         return cudaErrorInvalidValue;
     }
@@ -355,12 +357,12 @@ cudaError_t launch_bn(const TcPlan& pl, InType t, float c, char* ws, unsigned* s
     p.idesc2 = idesc_f16(BM, static_cast<uint32_t>(pl.Cp), 0u, 0u);
 
     // Per-device function attribute; cheap enough to set on every launch.
-    cudaError_t e = cudaFuncSetAttribute(tc_gauss_kernel<BN>,
+    cudaError_t e = cudaFuncSetAttribute(tc_gauss_kernel<BN, NEXP>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          static_cast<int>(pl.smem_bytes));
     if (e != cudaSuccess) return e;
     dim3 grid(static_cast<unsigned>(pl.Mpad / BM), static_cast<unsigned>(pl.splits));
-    tc_gauss_kernel<BN><<<grid, THREADS, pl.smem_bytes, s>>>(tm_q, tm_k, tm_v, p);
+    tc_gauss_kernel<BN, NEXP><<<grid, cta_threads<NEXP>(), pl.smem_bytes, s>>>(tm_q, tm_k, tm_v, p);
     return cudaGetLastError();
 }
 
@@ -376,25 +378,38 @@ bool plan_tensor(int64_t M, int64_t N, int64_t D, int64_t C, bool grad, bool cen
     p->Cp = static_cast<int>((p->Cv + 15) / 16 * 16);
     if (D > 256) { *why = "tensor-core path supports D <= 256"; return false; }
     if (p->Cp > 256) { *why = grad ? "gradient needs D + 1 <= 256" : "tensor-core path supports C <= 256"; return false; }
-    p->BN = p->Cp <= 128 ? 128 : 64;
     p->alias = alias;
     p->center = center;
-    p->Mpad = (M + BM - 1) / BM * BM;
-    p->Npad = alias ? p->Mpad : (N + 127) / 128 * 128;
     const int nkb = (p->Dp + KB - 1) / KB;
-    const size_t stage = align1k(static_cast<size_t>(nkb) * p->BN * 128 +
-                                 static_cast<size_t>(p->BN / KB) * p->Cp * 128 + p->BN * 4);
-    const size_t qbytes = static_cast<size_t>(nkb) * BM * 128;
-    const size_t fixed = 1024 /*alignment slack*/ + qbytes + sizeof(Barriers) + 64;
-    const size_t budget = 232448;
-    int stages = static_cast<int>(std::min<size_t>(6, (budget - fixed) / stage));
-    if (stages < 2) { *why = "shared-memory budget exceeded"; return false; }
-    p->stages = stages;
-    // At least ~116 KB so that one CTA (which owns all 512 TMEM columns)
-    // runs per SM.
-    p->smem_bytes = std::max<size_t>(fixed + stages * stage, 118 * 1024);
+    size_t fma_smem = 0;
+    int fma_stages = 0, nq = 1;
+    p->fma = !grad && p->Cv <= kFmaMaxChannels &&
+             plan_fma_kernel(p->Dp, static_cast<int>(p->Cv), &nq, &fma_stages, &fma_smem);
+    if (p->fma) {
+        p->BN = 128;
+        p->nq = nq;
+        p->stages = fma_stages;
+        p->smem_bytes = fma_smem;
+    } else {
+        p->BN = p->Cp <= 128 ? 128 : 64;
+        p->nq = 1;
+        const size_t stage = align1k(static_cast<size_t>(nkb) * p->BN * 128 +
+                                     static_cast<size_t>(p->BN / KB) * p->Cp * 128 + p->BN * 4);
+        const size_t qbytes = static_cast<size_t>(nkb) * BM * 128;
+        const size_t fixed = 1024 /*alignment slack*/ + qbytes + sizeof(Barriers) + 64;
+        const size_t budget = 232448;
+        int stages = static_cast<int>(std::min<size_t>(6, (budget - fixed) / stage));
+        if (stages < 2) { *why = "shared-memory budget exceeded"; return false; }
+        p->stages = stages;
+        // At least ~116 KB so that one CTA (which owns all 512 TMEM columns)
+        // runs per SM.
+        p->smem_bytes = std::max<size_t>(fixed + stages * stage, 118 * 1024);
+    }
+    const int64_t rows_per_cta = static_cast<int64_t>(BM) * p->nq;
+    p->Mpad = (M + rows_per_cta - 1) / rows_per_cta * rows_per_cta;
+    p->Npad = alias ? p->Mpad : (N + 127) / 128 * 128;
 
-    const int64_t tiles = p->Mpad / BM;
+    const int64_t tiles = p->Mpad / rows_per_cta;
     const int64_t key_tiles = p->Npad / p->BN;
     int best_s = 1;
     if (split_override > 0) {
@@ -414,7 +429,8 @@ bool plan_tensor(int64_t M, int64_t N, int64_t D, int64_t C, bool grad, bool cen
         best_s = static_cast<int>((key_tiles + tps - 1) / tps);
     }
     p->splits = std::max(1, best_s);
-    p->mean_blocks = static_cast<int>(std::max<int64_t>(1, std::min<int64_t>(1024, (M + N + 2047) / 2048)));
+    // ~256 rows per block of the mean kernel, so that every SM has work.
+    p->mean_blocks = static_cast<int>(std::max<int64_t>(1, std::min<int64_t>(4096, (M + N + 255) / 256)));
 
     size_t off = 0;
     auto take = [&](size_t bytes) { size_t o = off; off = align1k(off + bytes); return o; };
@@ -424,18 +440,25 @@ bool plan_tensor(int64_t M, int64_t N, int64_t D, int64_t C, bool grad, bool cen
     p->off_kh = alias ? p->off_qh : take(static_cast<size_t>(p->Npad) * p->Dp * 2);
     p->off_A = take(static_cast<size_t>(p->Mpad) * 4);
     p->off_B = alias ? p->off_A : take(static_cast<size_t>(p->Npad) * 4);
-    p->off_vt = take(static_cast<size_t>(p->Cp) * p->Npad * 2);
-    p->off_vmax = take(static_cast<size_t>(p->Cp) * 4);
-    p->off_inv = take(static_cast<size_t>(p->Cp) * 4);
-    p->off_part = take(static_cast<size_t>(p->splits) * p->Mpad * p->Cp * 4);
+    if (p->fma) {
+        p->off_vt = p->off_vmax = p->off_inv = 0;
+        p->off_rec = take(static_cast<size_t>(p->Npad / 2) * (2 + 2 * p->Cv) * 4);
+        p->off_part = take(static_cast<size_t>(p->splits) * p->Mpad * p->Cv * 4);
+    } else {
+        p->off_rec = 0;
+        p->off_vt = take(static_cast<size_t>(p->Cp) * p->Npad * 2);
+        p->off_vmax = take(static_cast<size_t>(p->Cp) * 4);
+        p->off_inv = take(static_cast<size_t>(p->Cp) * 4);
+        p->off_part = take(static_cast<size_t>(p->splits) * p->Mpad * p->Cp * 4);
+    }
     p->total = off;
     return true;
 }
 
 cudaError_t launch_tc(const TcPlan& p, InType t, float c, char* ws, unsigned* status,
                       cudaStream_t s, const char** why) {
-    if (p.BN == 128) return launch_bn<128>(p, t, c, ws, status, s, why);
-    return launch_bn<64>(p, t, c, ws, status, s, why);
+    if (p.BN == 128) return launch_bn<128, 16>(p, t, c, ws, status, s, why);
+    return launch_bn<64, 8>(p, t, c, ws, status, s, why);
 }
 
 }  // namespace gs

@@ -1,0 +1,415 @@
+// Fused Gauss-sum kernel for few value channels (C <= 4), sm_103a.
+//
+// Only the dense contraction runs on the tensor cores: tcgen05 MMAs form
+// S = q^ k^T (fp16/bf16 operands, fp32 accumulator in TMEM) for 128 x 128
+// tiles.  The exponent warps turn each S tile into kernel values
+// 2^(c S + A_m + B_n) = Phi(q_m, k_n) (the exponent is <= 0, so no running
+// maximum is needed; see tc_gauss.cu) and accumulate sum_n Phi v_n in fp32
+// on the FMA pipe.  For C <= 4 this costs fewer issue slots than a second
+// MMA with N = 16, and it keeps kernel values and values in fp32.
+//
+// Shared-memory bandwidth (128 B/clk/SM) is the resource this layout is
+// built around: an M=128, N=128, K=16 MMA with both operands in shared
+// memory alone would use all of it.  So
+//   * the query operand q^ lives in TMEM (A operand of tcgen05.mma), and
+//     only the key tile k^ is read from shared memory by the MMAs;
+//   * a CTA owns two query tiles (256 rows), which halves the L2 -> shared
+//     memory traffic of the key tiles, and every exponent warp handles the
+//     same key columns of both query tiles, so one broadcast load of a key
+//     record serves two kernel values;
+//   * S buffers are handed back to the MMA warp as soon as they are in
+//     registers.
+//
+// Warp roles (18 warps):
+//   warps 0-15  exponent warps.  Warp w reads TMEM lanes 32 (w % 4) .. +31
+//               (rows of both query tiles) and key columns 32 (w / 4) .. +31
+//               of the two S buffers of each key tile; at the start it
+//               copies its share of q^ from global memory into TMEM.
+//   warp 16     TMA producer: per key tile the k^ rows and the key records.
+//   warp 17     TMEM allocator and single-thread MMA issuer.
+// TMEM columns: NB S buffers of 128 columns, then the two q^ tiles
+// (Dp / 2 columns each, fp16/bf16 pairs packed in 32-bit columns).
+// Work items i = 2 j + h (key tile j, query tile h) use S buffer i % NB.
+// Key records: for each pair of keys (2t, 2t + 1) the floats
+//   B_2t, B_2t+1, v_2t[0], v_2t+1[0], ..., v_2t[C-1], v_2t+1[C-1].
+#include <cuda.h>
+#include <cuda_runtime.h>
+
+#include <algorithm>
+
+#include "internal.h"
+#include "ptx.cuh"
+#include "tensor_map.h"
+
+namespace gs {
+namespace {
+
+constexpr int BM = 128;            // rows per query tile (MMA M)
+constexpr int NQ = 2;              // query tiles per CTA
+constexpr int BN = 128;            // keys per key tile (MMA N)
+constexpr int KB = 64;             // 16-bit elements per 128-byte swizzled row
+constexpr int NEXP = 16;
+constexpr int PRODUCER_WARP = 16;
+constexpr int MMA_WARP = 17;
+constexpr int THREADS = 18 * 32;
+constexpr int NPART = 4;           // column groups (partial sums) per row
+constexpr int MAX_NB = 3;
+constexpr uint32_t TMEM_COLS = 512;
+constexpr int MAX_STAGES = 8;
+
+struct FmaParams {
+    const uint32_t* qh;  // Mpad x Dp/2 packed 16-bit pairs (centred, rounded q)
+    const float* A;      // Mpad: -(c/2)||q^_m||^2
+    const float* rec;    // key records, Npad / 2 pairs
+    float* part;         // splits x Mpad x C partial sums
+    unsigned* status;
+    int64_t Mpad;
+    int key_tiles;
+    int tiles_per_split;
+    int Dp;
+    int nkb;             // 64-element K blocks of k^
+    int nb;              // S buffers in TMEM
+    int stages;
+    uint32_t stage_bytes;
+    uint32_t kh_bytes;
+    uint32_t rec_bytes;  // key-record bytes of one key tile
+    uint32_t red_offset; // byte offset of the reduction area
+    float c;
+    uint32_t idesc;
+};
+
+struct __align__(8) FmaBarriers {
+    uint64_t qa_ready;
+    uint64_t drain;
+    uint64_t s_full[MAX_NB];
+    uint64_t s_free[MAX_NB];
+    uint64_t kv_full[MAX_STAGES];
+    uint64_t kv_empty[MAX_STAGES];
+    uint32_t tmem_base;
+    int abort_flag;
+};
+
+__device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity, volatile int* abort_flag,
+                                          unsigned* status) {
+    const bool ok = mbar_wait_bounded(bar, parity, abort_flag, status);
+    return __all_sync(0xffffffffu, ok);
+}
+
+__device__ __forceinline__ void exp_warps_sync() {
+    asm volatile("bar.sync 1, %0;" ::"r"(NEXP * 32) : "memory");
+}
+
+template <int C>
+__global__ void __launch_bounds__(THREADS, 1)
+tc_gauss_fma_kernel(const __grid_constant__ CUtensorMap tm_k, const FmaParams p) {
+    constexpr int REC_PAIR = 2 + 2 * C;               // floats per key pair
+    extern __shared__ uint8_t smem_raw[];
+    const uint32_t raw_addr = smem_u32(smem_raw);
+    uint8_t* smem = smem_raw + (((raw_addr + 1023u) & ~1023u) - raw_addr);
+    uint8_t* stage0 = smem;
+    float* red = reinterpret_cast<float*>(smem + p.red_offset);    // NPART x 256 x C
+    FmaBarriers* bars = reinterpret_cast<FmaBarriers*>(smem + p.red_offset + NPART * NQ * BM * C * 4);
+
+    const int tid = threadIdx.x;
+    const int warp = tid >> 5;
+    const int lane = tid & 31;
+    const int tile_m = blockIdx.x;   // query tiles 2 tile_m and 2 tile_m + 1
+    const int split = blockIdx.y;
+    const int kt0 = split * p.tiles_per_split;
+    const int T = min(p.key_tiles, kt0 + p.tiles_per_split) - kt0;
+    const int items = T * NQ;
+    const int NB = p.nb;
+    volatile int* abort_flag = &bars->abort_flag;
+
+    if (tid == 0) {
+        mbar_init(&bars->qa_ready, NEXP);
+        mbar_init(&bars->drain, 1);
+        for (int b = 0; b < NB; ++b) {
+            mbar_init(&bars->s_full[b], 1);
+            mbar_init(&bars->s_free[b], NEXP);       // one arrival per exponent warp
+        }
+        for (int s = 0; s < p.stages; ++s) {
+            mbar_init(&bars->kv_full[s], 1);
+            mbar_init(&bars->kv_empty[s], 1 + NEXP);  // MMA commit + exponent warps
+        }
+        bars->abort_flag = 0;
+        fence_mbar_init();
+    }
+    if (warp == MMA_WARP) {
+        tmem_alloc(&bars->tmem_base, TMEM_COLS);
+        tmem_relinquish();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = bars->tmem_base;
+    const uint32_t qa_col = static_cast<uint32_t>(NB * BN);   // q^ tile h at qa_col + h Dp/2
+
+    auto kh_smem = [&](int s) { return stage0 + s * p.stage_bytes; };
+    auto rec_smem = [&](int s) {
+        return reinterpret_cast<const float*>(stage0 + s * p.stage_bytes + p.kh_bytes);
+    };
+
+    if (warp == PRODUCER_WARP) {
+        if (lane == 0 && T > 0) {
+            tma_prefetch_desc(&tm_k);
+            int issued = 0;
+            RingPos st;
+            for (int j = 0; j < T; ++j, st.advance(p.stages)) {
+                const int s = st.idx;
+                if (!mbar_wait_bounded(&bars->kv_empty[s], st.phase ^ 1u, abort_flag, p.status)) break;
+                mbar_arrive_expect_tx(&bars->kv_full[s], p.kh_bytes + p.rec_bytes);
+                const int n0 = (kt0 + j) * BN;
+                for (int kb = 0; kb < p.nkb; ++kb)
+                    tma_load_2d(kh_smem(s) + kb * (BN * 128), &tm_k, &bars->kv_full[s], kb * KB, n0);
+                bulk_load(const_cast<float*>(rec_smem(s)), p.rec + static_cast<int64_t>(n0 / 2) * REC_PAIR,
+                          p.rec_bytes, &bars->kv_full[s]);
+                issued = j + 1;
+            }
+            // Every copy this CTA started must land before it exits.
+            for (int j = max(0, issued - p.stages); j < issued; ++j)
+                mbar_wait_bounded(&bars->kv_full[j % p.stages],
+                                  static_cast<uint32_t>(j / p.stages) & 1u, nullptr, p.status);
+        }
+    } else if (warp == MMA_WARP) {
+        if (lane == 0 && T > 0) {
+            bool ok = mbar_wait_bounded(&bars->qa_ready, 0, abort_flag, p.status);
+            const int ksteps = p.Dp / 16;
+            RingPos buf, st;   // S buffer of item i, stage of key tile i / 2
+            for (int i = 0; ok && i < items; ++i) {
+                const int h = i & 1;
+                const int b = buf.idx;
+                const int s = st.idx;
+                if (i >= NB) {
+                    // Wait for the release of this buffer's previous item.
+                    ok = mbar_wait_bounded(&bars->s_free[b], buf.phase ^ 1u, abort_flag, p.status);
+                    if (!ok) break;
+                }
+                if (h == 0) {
+                    ok = mbar_wait_bounded(&bars->kv_full[s], st.phase, abort_flag, p.status);
+                    if (!ok) break;
+                }
+                tc_fence_after();
+                const uint32_t a_tmem = tmem + qa_col + h * (p.Dp / 2);
+                const uint32_t b_base = smem_u32(kh_smem(s));
+                for (int kk = 0; kk < ksteps; ++kk) {
+                    const uint64_t bd = smem_desc_kmajor_sw128(b_base + (kk >> 2) * (BN * 128) + (kk & 3) * 32);
+                    mma_ts_f16(tmem + b * BN, a_tmem + kk * 8, bd, p.idesc, kk > 0 ? 1u : 0u);
+                }
+                mma_commit(&bars->s_full[b]);
+                if (h == NQ - 1) {
+                    mma_commit(&bars->kv_empty[s]);
+                    st.advance(p.stages);
+                }
+                buf.advance(NB);
+            }
+            mma_commit(&bars->drain);
+            mbar_wait_bounded(&bars->drain, 0, nullptr, p.status);
+        }
+    } else {
+        // ------------------------------------------------ exponent warps
+        const int quarter = warp & 3;
+        const int cg = warp >> 2;                  // column group: keys 32 cg .. 32 cg + 31
+        const uint32_t lane_base = static_cast<uint32_t>(quarter * 32) << 16;
+        const int row_t = quarter * 32 + lane;     // row inside each query tile
+        const int64_t row0 = static_cast<int64_t>(tile_m) * NQ * BM + row_t;
+        const int64_t row1 = row0 + BM;
+
+        // q^ rows -> TMEM (A operand).  Column group cg copies query tile
+        // cg / 2, 8-column chunks ck = cg % 2 (mod 2) of its Dp / 2 columns.
+        {
+            const int h = cg >> 1;
+            const uint32_t* src = p.qh + (row0 + h * BM) * (p.Dp / 2);
+            for (int ck = cg & 1; ck < p.Dp / 16; ck += 2) {
+                const uint4 lo = *reinterpret_cast<const uint4*>(src + ck * 8);
+                const uint4 hi = *reinterpret_cast<const uint4*>(src + ck * 8 + 4);
+                const uint32_t r[8] = {lo.x, lo.y, lo.z, lo.w, hi.x, hi.y, hi.z, hi.w};
+                tmem_st_32x32b_x8(tmem + lane_base + qa_col + h * (p.Dp / 2) + ck * 8, r);
+            }
+            tmem_wait_st();
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&bars->qa_ready);
+        }
+
+        const uint64_t a2_0 = f32x2_pack(p.A[row0], p.A[row0]);
+        const uint64_t a2_1 = f32x2_pack(p.A[row1], p.A[row1]);
+        const uint64_t c2 = f32x2_pack(p.c, p.c);
+        uint64_t acc0[C], acc1[C];
+#pragma unroll
+        for (int cc = 0; cc < C; ++cc) acc0[cc] = acc1[cc] = 0ull;
+        bool ok = true;
+        RingPos buf, st;   // S buffer of the next item, stage of key tile j
+        for (int j = 0; j < T; ++j, st.advance(p.stages)) {
+            const int s = st.idx;
+            const int b0 = buf.idx;
+            const uint32_t ph0 = buf.phase;
+            buf.advance(NB);
+            const int b1 = buf.idx;
+            const uint32_t ph1 = buf.phase;
+            buf.advance(NB);
+            ok = warp_wait(&bars->kv_full[s], st.phase, abort_flag, p.status);
+            if (ok) ok = warp_wait(&bars->s_full[b0], ph0, abort_flag, p.status);
+            if (ok) ok = warp_wait(&bars->s_full[b1], ph1, abort_flag, p.status);
+            if (!ok) break;
+            tc_fence_after();
+            uint32_t r0[32], r1[32];
+            tmem_ld_32x32b_x32(tmem + lane_base + b0 * BN + cg * 32, r0);
+            tmem_ld_32x32b_x32(tmem + lane_base + b1 * BN + cg * 32, r1);
+            tmem_wait_ld();
+            // Both S slices are in registers: hand the buffers back.
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) {
+                mbar_arrive(&bars->s_free[b0]);
+                mbar_arrive(&bars->s_free[b1]);
+            }
+            const float* rec = rec_smem(s) + (cg * 16) * REC_PAIR;
+#pragma unroll
+            for (int t = 0; t < 16; ++t) {
+                // Keys 32 cg + 2t and + 1, rows row0 (S0) and row1 (S1).
+                const float* pr = rec + t * REC_PAIR;
+                float2 bb, v0;
+                if (C == 1) {
+                    const float4 bv = *reinterpret_cast<const float4*>(pr);
+                    bb = make_float2(bv.x, bv.y);
+                    v0 = make_float2(bv.z, bv.w);
+                } else {
+                    bb = *reinterpret_cast<const float2*>(pr);
+                    v0 = *reinterpret_cast<const float2*>(pr + 2);
+                }
+                const uint64_t b2 = f32x2_pack(bb.x, bb.y);
+                const uint64_t x01 = f32x2_fma(f32x2_pack(__uint_as_float(r0[2 * t]), __uint_as_float(r0[2 * t + 1])),
+                                               c2, f32x2_add(b2, a2_0));
+                const uint64_t y01 = f32x2_fma(f32x2_pack(__uint_as_float(r1[2 * t]), __uint_as_float(r1[2 * t + 1])),
+                                               c2, f32x2_add(b2, a2_1));
+                float x0, x1, y0, y1;
+                f32x2_unpack(x01, x0, x1);
+                f32x2_unpack(y01, y0, y1);
+                const uint64_t px = f32x2_pack(ex2_approx(x0), ex2_approx(x1));
+                const uint64_t py = f32x2_pack(ex2_approx(y0), ex2_approx(y1));
+                const uint64_t vv0 = f32x2_pack(v0.x, v0.y);
+                acc0[0] = f32x2_fma(px, vv0, acc0[0]);
+                acc1[0] = f32x2_fma(py, vv0, acc1[0]);
+#pragma unroll
+                for (int cc = 1; cc < C; ++cc) {
+                    const float2 vc = *reinterpret_cast<const float2*>(pr + 2 + 2 * cc);
+                    const uint64_t vv = f32x2_pack(vc.x, vc.y);
+                    acc0[cc] = f32x2_fma(px, vv, acc0[cc]);
+                    acc1[cc] = f32x2_fma(py, vv, acc1[cc]);
+                }
+            }
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&bars->kv_empty[s]);
+        }
+        // Fixed-order reduction of the NPART column-group partial sums.
+#pragma unroll
+        for (int cc = 0; cc < C; ++cc) {
+            float lo, hi;
+            f32x2_unpack(acc0[cc], lo, hi);
+            red[(cg * NQ * BM + row_t) * C + cc] = lo + hi;
+            f32x2_unpack(acc1[cc], lo, hi);
+            red[(cg * NQ * BM + BM + row_t) * C + cc] = lo + hi;
+        }
+        exp_warps_sync();
+        if (cg < NQ && T > 0 && *abort_flag == 0) {
+            // Column group cg writes the rows of query tile cg.
+            const int rt = cg * BM + row_t;
+            float* out = p.part + (static_cast<int64_t>(split) * p.Mpad + row0 + cg * BM) * C;
+#pragma unroll
+            for (int cc = 0; cc < C; ++cc) {
+                float sum = 0.f;
+#pragma unroll
+                for (int q = 0; q < NPART; ++q) sum += red[(q * NQ * BM + rt) * C + cc];
+                out[cc] = sum;
+            }
+        }
+    }
+
+    tc_fence_before();
+    __syncthreads();
+    if (warp == MMA_WARP) {
+        tc_fence_after();
+        tmem_dealloc(tmem, TMEM_COLS);
+    }
+}
+
+size_t align1k(size_t x) { return (x + 1023) & ~static_cast<size_t>(1023); }
+
+size_t stage_bytes_for(int nkb, int C) {
+    return align1k(static_cast<size_t>(nkb) * BN * 128 + static_cast<size_t>(BN / 2) * (2 + 2 * C) * 4);
+}
+
+size_t fixed_bytes_for(int C) {
+    return 1024 /*alignment slack*/ + static_cast<size_t>(NPART) * NQ * BM * C * 4 +
+           sizeof(FmaBarriers) + 64;
+}
+
+int buffers_for(int Dp) { return std::min(MAX_NB, (static_cast<int>(TMEM_COLS) - Dp) / BN); }
+
+template <int C>
+cudaError_t launch_typed(const TcPlan& pl, InType t, float c, char* ws, unsigned* status,
+                         cudaStream_t s, const char** why) {
+    const CUtensorMapDataType hdt =
+        t == InType::BF16 ? CU_TENSOR_MAP_DATA_TYPE_BFLOAT16 : CU_TENSOR_MAP_DATA_TYPE_FLOAT16;
+    CUtensorMap tm_k;
+    if (!encode_tile_map_2d(&tm_k, hdt, ws + pl.off_kh, pl.Dp, pl.Npad, pl.Dp * 2ull, KB, BN)) {
+        *why = "cuTensorMapEncodeTiled failed or is unavailable";
+        return cudaErrorInvalidValue;
+    }
+    FmaParams p;
+    p.qh = reinterpret_cast<const uint32_t*>(ws + pl.off_qh);
+    p.A = reinterpret_cast<const float*>(ws + pl.off_A);
+    p.rec = reinterpret_cast<const float*>(ws + pl.off_rec);
+    p.part = reinterpret_cast<float*>(ws + pl.off_part);
+    p.status = status;
+    p.Mpad = pl.Mpad;
+    p.key_tiles = static_cast<int>(pl.Npad / BN);
+    p.tiles_per_split = (p.key_tiles + pl.splits - 1) / pl.splits;
+    p.Dp = pl.Dp;
+    p.nkb = (pl.Dp + KB - 1) / KB;
+    p.nb = buffers_for(pl.Dp);
+    p.stages = pl.stages;
+    p.kh_bytes = static_cast<uint32_t>(p.nkb * BN * 128);
+    p.rec_bytes = static_cast<uint32_t>((BN / 2) * (2 + 2 * C) * 4);
+    p.stage_bytes = static_cast<uint32_t>(stage_bytes_for(p.nkb, C));
+    p.red_offset = static_cast<uint32_t>(pl.stages * p.stage_bytes);
+    p.c = c;
+    const uint32_t hb = t == InType::BF16 ? 1u : 0u;
+    p.idesc = idesc_f16(BM, BN, hb, hb);
+    cudaError_t e = cudaFuncSetAttribute(tc_gauss_fma_kernel<C>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         static_cast<int>(pl.smem_bytes));
+    if (e != cudaSuccess) return e;
+    dim3 grid(static_cast<unsigned>(pl.Mpad / (NQ * BM)), static_cast<unsigned>(pl.splits));
+    tc_gauss_fma_kernel<C><<<grid, THREADS, pl.smem_bytes, s>>>(tm_k, p);
+    return cudaGetLastError();
+}
+
+}  // namespace
+
+bool plan_fma_kernel(int Dp, int C, int* nq, int* stages, size_t* smem) {
+    if (C < 1 || C > kFmaMaxChannels || Dp > 256 || buffers_for(Dp) < 2) return false;
+    const int nkb = (Dp + KB - 1) / KB;
+    const size_t budget = 232448;
+    const size_t stage = stage_bytes_for(nkb, C);
+    const size_t fixed = fixed_bytes_for(C);
+    const int st = static_cast<int>(std::min<size_t>(MAX_STAGES, (budget - fixed) / stage));
+    if (st < 2) return false;
+    *nq = NQ;
+    *stages = st;
+    *smem = std::max<size_t>(fixed + st * stage, 118 * 1024);
+    return true;
+}
+
+cudaError_t launch_tc_fma(const TcPlan& p, InType t, float c, char* ws, unsigned* status,
+                          cudaStream_t s, const char** why) {
+    switch (p.Cv) {
+        case 1: return launch_typed<1>(p, t, c, ws, status, s, why);
+        case 2: return launch_typed<2>(p, t, c, ws, status, s, why);
+        case 3: return launch_typed<3>(p, t, c, ws, status, s, why);
+        default: return launch_typed<4>(p, t, c, ws, status, s, why);
+    }
+}
+
+}  // namespace gs
