@@ -139,6 +139,34 @@ const char* gauss_sum_last_error(void);
 /* Static name of a status code. */
 const char* gauss_sum_status_string(gs_status status);
 
+/* Size of the static scratch array used by gauss_sum_noalloc: 16 MiB. */
+#define GS_NOALLOC_SCRATCH_BYTES (16u * 1024u * 1024u)
+
+/*
+ * Eq. 1 like gauss_sum (default options), but without allocating device
+ * memory.  The paper has no counterpart: this is for callers that cannot
+ * allocate at the point of the call, e.g. code inside a framework that owns
+ * every device allocation through its own pool, or code that has reserved
+ * all free device memory up front.  The scratch memory is a static device
+ * array of GS_NOALLOC_SCRATCH_BYTES bytes inside the library, held by every
+ * GPU that loads the library until the process exits.
+ *  - Arguments, layouts and ownership are those of gauss_sum.
+ *  - Calls that need more scratch than the array holds return
+ *    GS_ERR_UNSUPPORTED (see gauss_sum_last_error) without any GPU work;
+ *    the M = N = 65536, D = 64, C = 1 fp16 MMD workload fits.
+ *  - The first call on a device looks up the array's device address
+ *    (cudaGetSymbolAddress with that device current); make that first call
+ *    before any stream capture.
+ *  - All calls on a device share the array and leave their data in it:
+ *    calls whose GPU work can overlap (unordered streams, several host
+ *    threads) race and must be ordered by the caller.
+ *  - No cudaMalloc, cudaMallocAsync, cudaFree or allocating library call is
+ *    made.
+ */
+gs_status gauss_sum_noalloc(const void* q, const void* k, const void* v, double tau, int64_t M,
+                            int64_t N, int64_t D, int64_t C, gs_dtype dtype, float* out,
+                            void* stream);
+
 /*
  * Measurement helper (not part of Eq. 1): sustained MUFU exp2 throughput of
  * the current device in exponentials per second, measured with CUDA events

@@ -25,7 +25,12 @@ EXPORTS = (
     "gauss_sum_default_options", "gauss_sum", "gauss_sum_ex", "gauss_sum_grad_q",
     "gauss_sum_grad_q_ex", "gauss_sum_workspace_size", "gauss_sum_device_status",
     "gauss_sum_last_error", "gauss_sum_status_string", "gauss_sum_probe_ex2_rate",
+    "gauss_sum_noalloc",
 )
+
+# Bytes of the static scratch array behind gauss_sum_noalloc
+# (GS_NOALLOC_SCRATCH_BYTES in include/gauss_sum.h).
+NOALLOC_SCRATCH_BYTES = 16 * 1024 * 1024
 
 
 class GaussSumError(RuntimeError):
@@ -92,6 +97,8 @@ def _declare(lib):
     lib.gauss_sum_status_string.restype = ctypes.c_char_p
     lib.gauss_sum_probe_ex2_rate.argtypes = [vp, ctypes.POINTER(ctypes.c_double)]
     lib.gauss_sum_probe_ex2_rate.restype = f
+    lib.gauss_sum_noalloc.argtypes = [vp, vp, vp, d, i64, i64, i64, i64, f, vp, vp]
+    lib.gauss_sum_noalloc.restype = f
 
 
 def _check(lib, status: int):
@@ -168,6 +175,26 @@ def gauss_sum(q, k, v, tau, out=None, stream=None, center=True, split_n=0, works
                   main_events=main_events)
     st = lib.gauss_sum_ex(_ptr(q), _ptr(k), _ptr(v), float(tau), M, N, D, C, _dtype_code(q),
                           _ptr(out), _stream_ptr(stream), ctypes.byref(opt))
+    _check(lib, st)
+    return out
+
+
+def gauss_sum_noalloc(q, k, v, tau, out=None, stream=None):
+    """Eq. 1 like ``gauss_sum`` but without any device allocation by the
+    library: its scratch lives in a static 16 MiB device array (see
+    ``gauss_sum_noalloc`` in include/gauss_sum.h for the rules of use).
+    ``out`` should be passed by callers that must not allocate at all."""
+    import torch
+    lib = load_library()
+    for t, n in ((q, "q"), (k, "k"), (v, "v")):
+        _check_tensor(t, n)
+    M, D = q.shape
+    N = k.shape[0]
+    C = 1 if v.dim() == 1 else v.shape[1]
+    if out is None:
+        out = torch.empty((M, C), dtype=torch.float32, device=q.device)
+    st = lib.gauss_sum_noalloc(_ptr(q), _ptr(k), _ptr(v), float(tau), M, N, D, C, _dtype_code(q),
+                               _ptr(out), _stream_ptr(stream))
     _check(lib, st)
     return out
 

@@ -18,7 +18,7 @@ CSRC = os.path.join(PKG_DIR, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 BUILD_DIR = os.path.join(PKG_DIR, "_build")
 LIB_PATH = os.path.join(PKG_DIR, "libgauss_sum.so")
-SOURCES = ["api.cu", "prep.cu", "simt_fp32.cu", "tc_gauss.cu", "tc_gauss_fma.cu"]
+SOURCES = ["api.cu", "prep.cu", "simt_fp32.cu", "tc_gauss.cu", "tc_gauss_fma.cu", "noalloc.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 

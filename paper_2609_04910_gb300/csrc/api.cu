@@ -308,6 +308,27 @@ __global__ void ex2_probe_kernel(float* out, int iters) {
 }  // namespace
 
 namespace gs {
+
+gs_status forward_workspace_bytes(const void* q, const void* k, const void* v, double tau,
+                                  int64_t M, int64_t N, int64_t D, int64_t C, gs_dtype dtype,
+                                  float* out, size_t* bytes) {
+    Call c{q, k, v, tau, M, N, D, C, dtype, false, out, nullptr, nullptr, defaults()};
+    *bytes = 0;
+    gs_status st = validate(c);
+    if (st != GS_OK) return st;
+    if (M == 0 || N == 0 || C == 0) return GS_OK;
+    int dev = 0;
+    unsigned* status = nullptr;
+    cudaError_t e = device_info(&dev, &status);
+    if (e != cudaSuccess) return cuda_fail(e, "device query");
+    bool tensor = false;
+    TcPlan tp{};
+    SimtPlan sp{};
+    return plan(c, g_sm_count[dev], &tensor, &tp, &sp, bytes);
+}
+
+gs_status set_last_error(gs_status st, const char* msg) { return fail(st, "%s", msg); }
+
 cudaError_t run_ex2_probe(cudaStream_t s, double* rate) {
     int dev = 0;
     cudaError_t e = cudaGetDevice(&dev);

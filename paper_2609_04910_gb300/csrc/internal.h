@@ -5,6 +5,8 @@
 #include <cstddef>
 #include <cstdint>
 
+#include "gauss_sum.h"
+
 namespace gs {
 
 enum class InType { F32 = 0, F16 = 1, BF16 = 2 };
@@ -86,5 +88,13 @@ cudaError_t launch_tc_fma(const TcPlan& p, InType t, float c, char* ws, unsigned
 
 // probe
 cudaError_t run_ex2_probe(cudaStream_t s, double* rate);
+
+// api.cu: workspace bytes that a forward call with exactly these arguments
+// and default options needs (through *bytes), or the status the call
+// would fail with; and recording a message for gauss_sum_last_error().
+gs_status forward_workspace_bytes(const void* q, const void* k, const void* v, double tau,
+                                  int64_t M, int64_t N, int64_t D, int64_t C, gs_dtype dtype,
+                                  float* out, size_t* bytes);
+gs_status set_last_error(gs_status st, const char* msg);
 
 }  // namespace gs
