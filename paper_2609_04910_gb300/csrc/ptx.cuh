@@ -67,6 +67,38 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
     return ok != 0;
 }
 
+// Non-blocking test of the phase with the given parity.  A barrier query
+// takes on the order of a hundred cycles to answer, so hot loops issue it
+// early and branch on the answer only after other work has been issued.
+__device__ __forceinline__ bool mbar_test_wait(uint64_t* bar, uint32_t parity) {
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok)
+        : "r"(smem_u32(bar)), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+
+// Non-blocking test of two barriers at once: both queries are in flight
+// together, so their latencies overlap.  True if both phases are complete.
+__device__ __forceinline__ bool mbar_test_wait2(uint64_t* bar1, uint32_t parity1, uint64_t* bar2,
+                                                uint32_t parity2) {
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p1, p2;\n\t"
+        "mbarrier.test_wait.parity.shared::cta.b64 p1, [%1], %2;\n\t"
+        "mbarrier.test_wait.parity.shared::cta.b64 p2, [%3], %4;\n\t"
+        "and.pred p1, p1, p2;\n\t"
+        "selp.u32 %0, 1, 0, p1;\n\t}"
+        : "=r"(ok)
+        : "r"(smem_u32(bar1)), "r"(parity1), "r"(smem_u32(bar2)), "r"(parity2)
+        : "memory");
+    return ok != 0;
+}
+
 // Wait for the phase of `bar` with the given parity to complete.  Returns
 // false (without waiting any longer) if the CTA abort flag is raised or the
 // global-time limit runs out; in the latter case the status word receives

@@ -8,16 +8,21 @@
 // on the FMA pipe.  For C <= 4 this costs fewer issue slots than a second
 // MMA with N = 16, and it keeps kernel values and values in fp32.
 //
-// Shared-memory bandwidth (128 B/clk/SM) is the resource this layout is
-// built around: an M=128, N=128, K=16 MMA with both operands in shared
-// memory alone would use all of it.  So
-//   * the query operand q^ lives in TMEM (A operand of tcgen05.mma), and
-//     only the key tile k^ is read from shared memory by the MMAs;
-//   * a CTA owns two query tiles (256 rows), which halves the L2 -> shared
-//     memory traffic of the key tiles, and every exponent warp handles the
-//     same key columns of both query tiles, so one broadcast load of a key
-//     record serves two kernel values;
-//   * S buffers are handed back to the MMA warp as soon as they are in
+// Layout choices:
+//   * Shared-memory bandwidth (128 B/clk/SM): an M=128, N=128, K=16 MMA
+//     with both operands in shared memory would use all of it, and such
+//     MMAs also slow down while other warps read TMEM.  So the query
+//     operand q^ lives in TMEM (A operand of tcgen05.mma) and only the key
+//     tile k^ is read from shared memory.
+//   * A CTA owns two query tiles (256 rows), which halves the L2 -> shared
+//     memory traffic of the key tiles; every exponent warp handles the same
+//     key columns of both query tiles, so one broadcast load of a key
+//     record serves two kernel values.
+//   * Barrier handshakes cost the single issuing thread one to two hundred
+//     cycles each, so there is one handshake per key tile (not per MMA
+//     tile): the MMA thread issues the 2 x (Dp / 16) MMAs of a key tile back
+//     to back and commits once; the exponent warps release both S buffers
+//     of the key tile with one arrival per warp, as soon as they are in
 //     registers.
 //
 // Warp roles (18 warps):
@@ -28,8 +33,9 @@
 //   warp 16     TMA producer: per key tile the k^ rows and the key records.
 //   warp 17     TMEM allocator and single-thread MMA issuer.
 // TMEM columns: NB S buffers of 128 columns, then the two q^ tiles
-// (Dp / 2 columns each, fp16/bf16 pairs packed in 32-bit columns).
-// Work items i = 2 j + h (key tile j, query tile h) use S buffer i % NB.
+// (Dp / 2 columns each, fp16/bf16 pairs packed in 32-bit columns).  Key
+// tile j uses S buffers (2j) % NB and (2j + 1) % NB, so with NB = 2 or 3 the
+// MMAs of key tile j may start once key tile j - 1 has been released.
 // Key records: for each pair of keys (2t, 2t + 1) the floats
 //   B_2t, B_2t+1, v_2t[0], v_2t+1[0], ..., v_2t[C-1], v_2t+1[C-1].
 #include <cuda.h>
@@ -79,10 +85,10 @@ struct FmaParams {
 };
 
 struct __align__(8) FmaBarriers {
-    uint64_t qa_ready;
+    uint64_t qa_ready;   // q^ copied into TMEM (16 warp arrivals)
     uint64_t drain;
-    uint64_t s_full[MAX_NB];
-    uint64_t s_free[MAX_NB];
+    uint64_t s_full;     // phase j: both S tiles of key tile j computed
+    uint64_t s_free;     // phase j: both S tiles of key tile j in registers
     uint64_t kv_full[MAX_STAGES];
     uint64_t kv_empty[MAX_STAGES];
     uint32_t tmem_base;
@@ -117,17 +123,14 @@ tc_gauss_fma_kernel(const __grid_constant__ CUtensorMap tm_k, const FmaParams p)
     const int split = blockIdx.y;
     const int kt0 = split * p.tiles_per_split;
     const int T = min(p.key_tiles, kt0 + p.tiles_per_split) - kt0;
-    const int items = T * NQ;
     const int NB = p.nb;
     volatile int* abort_flag = &bars->abort_flag;
 
     if (tid == 0) {
         mbar_init(&bars->qa_ready, NEXP);
         mbar_init(&bars->drain, 1);
-        for (int b = 0; b < NB; ++b) {
-            mbar_init(&bars->s_full[b], 1);
-            mbar_init(&bars->s_free[b], NEXP);       // one arrival per exponent warp
-        }
+        mbar_init(&bars->s_full, 1);
+        mbar_init(&bars->s_free, NEXP);                // one arrival per exponent warp
         for (int s = 0; s < p.stages; ++s) {
             mbar_init(&bars->kv_full[s], 1);
             mbar_init(&bars->kv_empty[s], 1 + NEXP);  // MMA commit + exponent warps
@@ -175,33 +178,44 @@ tc_gauss_fma_kernel(const __grid_constant__ CUtensorMap tm_k, const FmaParams p)
         if (lane == 0 && T > 0) {
             bool ok = mbar_wait_bounded(&bars->qa_ready, 0, abort_flag, p.status);
             const int ksteps = p.Dp / 16;
-            RingPos buf, st;   // S buffer of item i, stage of key tile i / 2
-            for (int i = 0; ok && i < items; ++i) {
-                const int h = i & 1;
-                const int b = buf.idx;
+            // Shared-memory descriptor of k^ stage 0; stage s and K step kk
+            // add (s stage_bytes + (kk / 4) BN 128 + (kk % 4) 32) / 16 to the
+            // start-address field.
+            const uint64_t desc0 = smem_desc_kmajor_sw128(smem_u32(stage0));
+            const uint32_t a0 = tmem + qa_col, a1 = a0 + (p.Dp / 2);
+            RingPos st, buf;
+            for (int j = 0; ok && j < T; ++j, st.advance(p.stages)) {
                 const int s = st.idx;
-                if (i >= NB) {
-                    // Wait for the release of this buffer's previous item.
-                    ok = mbar_wait_bounded(&bars->s_free[b], buf.phase ^ 1u, abort_flag, p.status);
-                    if (!ok) break;
-                }
-                if (h == 0) {
+                // Key tile j - 1 released (which also frees the buffers of
+                // earlier tiles) and stage s loaded; both queried at once.
+                const uint32_t free_parity = static_cast<uint32_t>(j - 1) & 1u;
+                const bool ready = j == 0 ? mbar_test_wait(&bars->kv_full[s], st.phase)
+                                          : mbar_test_wait2(&bars->s_free, free_parity,
+                                                            &bars->kv_full[s], st.phase);
+                if (!ready) {
+                    if (j > 0) {
+                        ok = mbar_wait_bounded(&bars->s_free, free_parity, abort_flag, p.status);
+                        if (!ok) break;
+                    }
                     ok = mbar_wait_bounded(&bars->kv_full[s], st.phase, abort_flag, p.status);
                     if (!ok) break;
                 }
                 tc_fence_after();
-                const uint32_t a_tmem = tmem + qa_col + h * (p.Dp / 2);
-                const uint32_t b_base = smem_u32(kh_smem(s));
-                for (int kk = 0; kk < ksteps; ++kk) {
-                    const uint64_t bd = smem_desc_kmajor_sw128(b_base + (kk >> 2) * (BN * 128) + (kk & 3) * 32);
-                    mma_ts_f16(tmem + b * BN, a_tmem + kk * 8, bd, p.idesc, kk > 0 ? 1u : 0u);
-                }
-                mma_commit(&bars->s_full[b]);
-                if (h == NQ - 1) {
-                    mma_commit(&bars->kv_empty[s]);
-                    st.advance(p.stages);
-                }
+                const uint32_t d0 = tmem + buf.idx * BN;
                 buf.advance(NB);
+                const uint32_t d1 = tmem + buf.idx * BN;
+                buf.advance(NB);
+                const uint64_t bdesc = desc0 + ((static_cast<uint64_t>(s) * p.stage_bytes) >> 4);
+                for (int kk = 0; kk < ksteps; ++kk) {
+                    const uint64_t bd = bdesc + static_cast<uint64_t>((kk >> 2) * (BN * 128 / 16) + (kk & 3) * 2);
+                    mma_ts_f16(d0, a0 + kk * 8, bd, p.idesc, kk > 0 ? 1u : 0u);
+                }
+                for (int kk = 0; kk < ksteps; ++kk) {
+                    const uint64_t bd = bdesc + static_cast<uint64_t>((kk >> 2) * (BN * 128 / 16) + (kk & 3) * 2);
+                    mma_ts_f16(d1, a1 + kk * 8, bd, p.idesc, kk > 0 ? 1u : 0u);
+                }
+                mma_commit(&bars->s_full);
+                mma_commit(&bars->kv_empty[s]);
             }
             mma_commit(&bars->drain);
             mbar_wait_bounded(&bars->drain, 0, nullptr, p.status);
@@ -239,31 +253,29 @@ tc_gauss_fma_kernel(const __grid_constant__ CUtensorMap tm_k, const FmaParams p)
 #pragma unroll
         for (int cc = 0; cc < C; ++cc) acc0[cc] = acc1[cc] = 0ull;
         bool ok = true;
-        RingPos buf, st;   // S buffer of the next item, stage of key tile j
+        RingPos st, buf;   // stage of key tile j; S buffer of its first tile
         for (int j = 0; j < T; ++j, st.advance(p.stages)) {
             const int s = st.idx;
-            const int b0 = buf.idx;
-            const uint32_t ph0 = buf.phase;
+            const uint32_t col0 = static_cast<uint32_t>(buf.idx * BN);
             buf.advance(NB);
-            const int b1 = buf.idx;
-            const uint32_t ph1 = buf.phase;
+            const uint32_t col1 = static_cast<uint32_t>(buf.idx * BN);
             buf.advance(NB);
-            ok = warp_wait(&bars->kv_full[s], st.phase, abort_flag, p.status);
-            if (ok) ok = warp_wait(&bars->s_full[b0], ph0, abort_flag, p.status);
-            if (ok) ok = warp_wait(&bars->s_full[b1], ph1, abort_flag, p.status);
-            if (!ok) break;
+            const uint32_t full_parity = static_cast<uint32_t>(j) & 1u;
+            if (!__all_sync(0xffffffffu, mbar_test_wait2(&bars->kv_full[s], st.phase, &bars->s_full,
+                                                         full_parity))) {
+                ok = warp_wait(&bars->kv_full[s], st.phase, abort_flag, p.status);
+                if (ok) ok = warp_wait(&bars->s_full, full_parity, abort_flag, p.status);
+                if (!ok) break;
+            }
             tc_fence_after();
             uint32_t r0[32], r1[32];
-            tmem_ld_32x32b_x32(tmem + lane_base + b0 * BN + cg * 32, r0);
-            tmem_ld_32x32b_x32(tmem + lane_base + b1 * BN + cg * 32, r1);
+            tmem_ld_32x32b_x32(tmem + lane_base + col0 + cg * 32, r0);
+            tmem_ld_32x32b_x32(tmem + lane_base + col1 + cg * 32, r1);
             tmem_wait_ld();
             // Both S slices are in registers: hand the buffers back.
             tc_fence_before();
             __syncwarp();
-            if (lane == 0) {
-                mbar_arrive(&bars->s_free[b0]);
-                mbar_arrive(&bars->s_free[b1]);
-            }
+            if (lane == 0) mbar_arrive(&bars->s_free);
             const float* rec = rec_smem(s) + (cg * 16) * REC_PAIR;
 #pragma unroll
             for (int t = 0; t < 16; ++t) {
