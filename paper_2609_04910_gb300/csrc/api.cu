@@ -115,8 +115,8 @@ gs_status plan(const Call& c, int sms, bool* tensor, gs::TcPlan* tp, gs::SimtPla
     *tensor = c.dtype != GS_FP32;
     if (*tensor) {
         const bool alias = c.q == c.k && c.M == c.N && c.q != nullptr;
-        if (!gs::plan_tensor(c.M, c.N, c.D, c.C, c.grad, c.opt.center != 0, alias, c.opt.split_n,
-                             sms, tp, &why))
+        if (!gs::plan_tensor(in_type(c.dtype), c.M, c.N, c.D, c.C, c.grad, c.opt.center != 0,
+                             alias, c.opt.split_n, sms, tp, &why))
             return fail(GS_ERR_UNSUPPORTED, "%s", why);
         *bytes = tp->total;
     } else {
@@ -201,22 +201,37 @@ gs_status run(Call c) {
             where = "mean kernel";
         }
         const float ninf = -INFINITY;
-        if (e == cudaSuccess) {
-            e = gs::launch_center_cast_norm(t, c.q, c.M, tp.Mpad, static_cast<int>(c.D), tp.Dp, mu,
-                                            half_c, ws + tp.off_qh,
-                                            reinterpret_cast<float*>(ws + tp.off_A), ninf, c.stream);
-            where = "centre/cast kernel (q)";
-        }
-        if (e == cudaSuccess && !tp.alias) {
-            e = gs::launch_center_cast_norm(t, c.k, c.N, tp.Npad, static_cast<int>(c.D), tp.Dp, mu,
-                                            half_c, ws + tp.off_kh,
-                                            reinterpret_cast<float*>(ws + tp.off_B), ninf, c.stream);
-            where = "centre/cast kernel (k)";
+        if (e == cudaSuccess && tp.aug) {
+            // Augmented operands: centred points with the norms folded in.
+            e = gs::launch_aug_prep(t, c.q, c.M, tp.Mpad, static_cast<int>(c.D), tp.Dp, mu,
+                                    ws + tp.off_qh, tp.alias ? ws + tp.off_kh : nullptr, c.stream);
+            where = "augmented-operand kernel (q)";
+            if (e == cudaSuccess && !tp.alias) {
+                e = gs::launch_aug_prep(t, c.k, c.N, tp.Npad, static_cast<int>(c.D), tp.Dp, mu,
+                                        nullptr, ws + tp.off_kh, c.stream);
+                where = "augmented-operand kernel (k)";
+            }
+        } else {
+            if (e == cudaSuccess) {
+                e = gs::launch_center_cast_norm(t, c.q, c.M, tp.Mpad, static_cast<int>(c.D), tp.Dp,
+                                                mu, half_c, ws + tp.off_qh,
+                                                reinterpret_cast<float*>(ws + tp.off_A), ninf,
+                                                c.stream);
+                where = "centre/cast kernel (q)";
+            }
+            if (e == cudaSuccess && !tp.alias) {
+                e = gs::launch_center_cast_norm(t, c.k, c.N, tp.Npad, static_cast<int>(c.D), tp.Dp,
+                                                mu, half_c, ws + tp.off_kh,
+                                                reinterpret_cast<float*>(ws + tp.off_B), ninf,
+                                                c.stream);
+                where = "centre/cast kernel (k)";
+            }
         }
         if (e == cudaSuccess && tp.fma) {
-            e = gs::launch_key_records(t, c.v, reinterpret_cast<const float*>(ws + tp.off_B), c.N,
-                                       tp.Npad, static_cast<int>(tp.Cv),
-                                       reinterpret_cast<float*>(ws + tp.off_rec), c.stream);
+            e = gs::launch_key_records(
+                t, c.v, tp.aug ? nullptr : reinterpret_cast<const float*>(ws + tp.off_B), c.N,
+                tp.Npad, static_cast<int>(tp.Cv), reinterpret_cast<float*>(ws + tp.off_rec),
+                c.stream);
             where = "key-record kernel";
         } else if (e == cudaSuccess) {
             e = gs::launch_value_prep(t, c.grad, c.v, c.k, mu, c.N, tp.Npad, static_cast<int>(c.D),

@@ -29,6 +29,8 @@ struct TcPlan {
     bool alias;              // q and k are the same array (M == N): prep once
     bool center;
     bool fma;                // kernel of tc_gauss_fma.cu (C <= kFmaMaxChannels, forward)
+    bool aug;                // FMA kernel with augmented operands (Dp = D + 2 aug_norm_terms
+                             // rounded to 16)
     int nq;                  // query tiles of 128 rows per CTA (FMA kernel)
     size_t off_mean_part, off_mu, off_qh, off_kh, off_A, off_B, off_vt, off_vmax, off_inv,
         off_rec, off_part, total;
@@ -46,7 +48,7 @@ struct SimtPlan {
 int device_sm_count(int device);
 bool device_is_sm103(int device);
 
-bool plan_tensor(int64_t M, int64_t N, int64_t D, int64_t C, bool grad, bool center,
+bool plan_tensor(InType t, int64_t M, int64_t N, int64_t D, int64_t C, bool grad, bool center,
                  bool alias, int split_override, int sms, TcPlan* p, const char** why);
 bool plan_simt(int64_t M, int64_t N, int64_t D, int64_t C, bool grad, int split_override,
                int sms, SimtPlan* p, const char** why);
@@ -73,16 +75,26 @@ cudaError_t launch_simt(const SimtPlan& p, bool grad, const float* q, const floa
                         const float* v, float half_c, float* part, cudaStream_t s);
 
 // Key records of the FMA kernel: per key pair (2t, 2t+1) the floats
-// B_2t, B_2t+1, v_2t[0], v_2t+1[0], ..., v_2t[C-1], v_2t+1[C-1].
+// B_2t, B_2t+1 (omitted when B is null), v_2t[0], v_2t+1[0], ...,
+// v_2t[C-1], v_2t+1[C-1].
 cudaError_t launch_key_records(InType t, const void* v, const float* B, int64_t N, int64_t Npad,
                                int C, float* rec, cudaStream_t s);
+// Augmented MMA operands (see prep.cu): query layout into out_q, key layout
+// into out_k (either may be null), Dpa >= D + 2 aug_norm_terms(t) columns
+// per row.
+constexpr int aug_norm_terms(InType t) { return t == InType::BF16 ? 3 : 2; }
+cudaError_t launch_aug_prep(InType t, const void* x, int64_t rows, int64_t rows_pad, int D,
+                            int Dpa, const float* mu, void* out_q, void* out_k, cudaStream_t s);
 
 // tc_gauss.cu ----------------------------------------------------------
 cudaError_t launch_tc(const TcPlan& p, InType t, float c, char* ws, unsigned* status,
                       cudaStream_t s, const char** why);
 
 // tc_gauss_fma.cu ------------------------------------------------------
-bool plan_fma_kernel(int Dp, int C, int* nq, int* stages, size_t* smem);
+// Largest (augmented) Dp for which the FMA kernel keeps q^ in shared memory
+// and folds the norms into the MMA.
+constexpr int kAugMaxDp = 128;
+bool plan_fma_kernel(int Dp, int C, bool aug, int* nq, int* stages, size_t* smem);
 cudaError_t launch_tc_fma(const TcPlan& p, InType t, float c, char* ws, unsigned* status,
                           cudaStream_t s, const char** why);
 

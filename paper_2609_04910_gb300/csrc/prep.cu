@@ -2,7 +2,8 @@
 //
 //  * common mean of all query and key points (the shift safeguard of
 //    Remark 3, Sec. 2: the kernel depends on q - k only, so any common shift
-//    is exact and only changes rounding);
+//    is exact and only changes rounding), rounded to the input format's
+//    grid so that the shift itself adds no rounding near the mean;
 //  * centring, rounding to the MMA operand type and the scaled squared norms
 //    A_m = -(c/2)||q^_m||^2, B_n = -(c/2)||k^_n||^2 (c = tau log2 e) taken
 //    from the ROUNDED points, so that c q^.k^ + A_m + B_n is exactly
@@ -37,42 +38,70 @@ template <> __device__ __forceinline__ __nv_bfloat16 from_f<__nv_bfloat16>(float
 
 // ---------------------------------------------------------------- mean
 // Block (32, 8): 32 consecutive coordinates x 8 row lanes; each block sums
-// a contiguous chunk of the stacked rows [q; k] and writes D partial sums.
+// a contiguous chunk of the stacked rows [q; k] and writes, per coordinate,
+// its partial sum (partial[block][d]) and largest magnitude
+// (partial[G + block][d]).
 template <typename T>
 __global__ void mean_partial_kernel(const T* __restrict__ q, const T* __restrict__ k, int64_t M,
                                     int64_t N, int D, int64_t rows_per_block,
                                     float* __restrict__ partial) {
     __shared__ float red[8][33];
+    __shared__ float big[8][33];
     const int64_t r0 = static_cast<int64_t>(blockIdx.x) * rows_per_block;
     const int64_t r1 = min(r0 + rows_per_block, M + N);
     for (int d0 = 0; d0 < D; d0 += 32) {
         const int d = d0 + threadIdx.x;
-        float acc = 0.f;
+        float acc = 0.f, mx = 0.f;
         if (d < D) {
             for (int64_t r = r0 + threadIdx.y; r < r1; r += 8) {
-                const T x = r < M ? q[r * D + d] : k[(r - M) * D + d];
-                acc += to_f(x);
+                const float x = to_f(r < M ? q[r * D + d] : k[(r - M) * D + d]);
+                acc += x;
+                mx = fmaxf(mx, fabsf(x));
             }
         }
         red[threadIdx.y][threadIdx.x] = acc;
+        big[threadIdx.y][threadIdx.x] = mx;
         __syncthreads();
         if (threadIdx.y == 0 && d < D) {
-            float s = 0.f;
+            float sum = 0.f, m = 0.f;
 #pragma unroll
-            for (int y = 0; y < 8; ++y) s += red[y][threadIdx.x];
-            partial[static_cast<int64_t>(blockIdx.x) * D + d] = s;
+            for (int y = 0; y < 8; ++y) {
+                sum += red[y][threadIdx.x];
+                m = fmaxf(m, big[y][threadIdx.x]);
+            }
+            partial[static_cast<int64_t>(blockIdx.x) * D + d] = sum;
+            partial[static_cast<int64_t>(gridDim.x + blockIdx.x) * D + d] = m;
         }
         __syncthreads();
     }
 }
 
+// mu_d = the mean of coordinate d rounded to a multiple of g_d, the spacing
+// of the input format at max |x_d| (2^(e - mant_bits) for max |x_d| in
+// [2^e, 2^(e+1)), at least the subnormal spacing 2^min_exp).  Every input
+// x_d is a multiple of its own spacing, which divides g_d, so x_d - mu_d is
+// a multiple of the spacing of x_d: it is exact in the input format
+// whenever |x_d - mu_d| stays below 2^(e_x + 1) (x_d in [2^e_x, 2^(e_x+1))),
+// i.e. the shift adds no rounding for points near the mean.  Any common
+// shift leaves the Gauss sum unchanged.
 __global__ void mean_final_kernel(const float* __restrict__ partial, int G, int D, double total,
-                                  float* __restrict__ mu) {
+                                  int mant_bits, int min_exp, float* __restrict__ mu) {
     const int d = blockIdx.x * blockDim.x + threadIdx.x;
     if (d >= D) return;
     double s = 0.0;
-    for (int g = 0; g < G; ++g) s += static_cast<double>(partial[static_cast<int64_t>(g) * D + d]);
-    mu[d] = static_cast<float>(s / total);
+    float mx = 0.f;
+    for (int g = 0; g < G; ++g) {
+        s += static_cast<double>(partial[static_cast<int64_t>(g) * D + d]);
+        mx = fmaxf(mx, partial[static_cast<int64_t>(G + g) * D + d]);
+    }
+    double m = s / total;
+    if (mx > 0.f) {
+        int e;
+        frexp(static_cast<double>(mx), &e);              // mx in [2^(e-1), 2^e)
+        const double g = ldexp(1.0, max(e - 1 - mant_bits, min_exp));
+        m = rint(m / g) * g;
+    }
+    mu[d] = static_cast<float>(m);
 }
 
 // ---------------------------------------------------------------- centre / cast / norm
@@ -198,21 +227,105 @@ __global__ void value_prep_kernel(const T* __restrict__ v, const T* __restrict__
 }
 
 // ---------------------------------------------------------------- key records
-// One thread per key pair t: B_2t, B_2t+1, then the values of both keys
-// channel by channel, in fp32 (zero for padded keys).
+// One thread per key pair t: B_2t, B_2t+1 (only when B is given), then the
+// values of both keys channel by channel, in fp32 (zero for padded keys).
 template <typename T>
 __global__ void key_record_kernel(const T* __restrict__ v, const float* __restrict__ B, int64_t N,
                                   int64_t pairs, int C, float* __restrict__ rec) {
     const int64_t t = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
     if (t >= pairs) return;
     const int64_t n0 = 2 * t, n1 = 2 * t + 1;
-    float* out = rec + t * (2 + 2 * C);
-    out[0] = B[n0];
-    out[1] = B[n1];
-    for (int c = 0; c < C; ++c) {
-        out[2 + 2 * c] = n0 < N ? to_f(v[n0 * C + c]) : 0.f;
-        out[3 + 2 * c] = n1 < N ? to_f(v[n1 * C + c]) : 0.f;
+    const int head = B ? 2 : 0;
+    float* out = rec + t * (head + 2 * C);
+    if (B) {
+        out[0] = B[n0];
+        out[1] = B[n1];
     }
+    for (int c = 0; c < C; ++c) {
+        out[head + 2 * c] = n0 < N ? to_f(v[n0 * C + c]) : 0.f;
+        out[head + 1 + 2 * c] = n1 < N ? to_f(v[n1 * C + c]) : 0.f;
+    }
+}
+
+// ---------------------------------------------------------------- augmented operands
+// Centred points rounded to the MMA type, x^ = rn(x - mu) (as for the
+// plain operands, so that fp16/bf16 inputs near the mean stay exact),
+// followed by 2 NT columns that make the MMA produce the whole exponent up
+// to the factor c = tau log2 e:
+//   query rows  [q^, F, 1, .., 1, a_0, a_1, .., a_NT-1, 0 ...]
+//   key rows    [k^, b_0, b_1, .., b_NT-1, F, 1, .., 1, 0 ...]
+// with a = -||q^||^2 / 2 and b = -||k^||^2 / 2 taken from the rounded
+// points in fp32 and written as F t_0 + t_1 + ... + t_NT-1, each t_i a
+// rounded remainder, so that
+//   q^_aug . k^_aug = q^.k^ + a + b = -||q^ - k^||^2 / 2
+// up to the split error (|a| 2^-22 for two fp16 terms, |a| 2^-24 for three
+// bf16 terms) and the fp32 accumulation; the kernel value is 2^(c S).  The
+// power of two F (1024 for fp16) keeps norms up to 6.7e7 inside the fp16
+// range.  Padded key rows get b_0 = -30000 / F (their values are zero as
+// well); padded query rows are zero.  One warp per row; `out_q` and/or
+// `out_k` may be given (both for q = k).
+template <typename T, typename H>
+__global__ void aug_prep_kernel(const T* __restrict__ x, int64_t rows, int64_t rows_pad, int D,
+                                int Dpa, int nt, float F, const float* __restrict__ mu,
+                                H* __restrict__ out_q, H* __restrict__ out_k) {
+    const int lane = threadIdx.x & 31;
+    const int64_t row = static_cast<int64_t>(blockIdx.x) * (blockDim.x >> 5) + (threadIdx.x >> 5);
+    if (row >= rows_pad) return;
+    H* oq = out_q ? out_q + row * Dpa : nullptr;
+    H* ok = out_k ? out_k + row * Dpa : nullptr;
+    const H zero = from_f<H>(0.f);
+    if (row >= rows) {
+        for (int d = lane; d < Dpa; d += 32) {
+            if (oq) oq[d] = zero;
+            if (ok) ok[d] = d == D ? from_f<H>(-30000.f / F) : zero;
+        }
+        return;
+    }
+    const T* in = x + row * D;
+    float acc = 0.f;
+    for (int d = lane; d < D; d += 32) {
+        const H h = from_f<H>(to_f(in[d]) - (mu ? mu[d] : 0.f));
+        if (oq) oq[d] = h;
+        if (ok) ok[d] = h;
+        const float hf = to_f(h);
+        acc = fmaf(hf, hf, acc);
+    }
+    for (int d = D + 2 * nt + lane; d < Dpa; d += 32) {
+        if (oq) oq[d] = zero;
+        if (ok) ok[d] = zero;
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
+    if (lane < nt) {
+        // Lane i writes term i of the split and its partner column.
+        float r = -0.5f * acc;
+        H t = from_f<H>(r / F);
+        r -= F * to_f(t);
+        for (int i = 1; i <= lane; ++i) {
+            t = from_f<H>(r);
+            r -= to_f(t);
+        }
+        const H one = from_f<H>(lane == 0 ? F : 1.f);
+        if (oq) {
+            oq[D + lane] = one;
+            oq[D + nt + lane] = t;
+        }
+        if (ok) {
+            ok[D + lane] = t;
+            ok[D + nt + lane] = one;
+        }
+    }
+}
+
+template <typename T, typename H>
+cudaError_t aug_typed(const void* x, int64_t rows, int64_t rows_pad, int D, int Dpa, int nt,
+                      float F, const float* mu, void* out_q, void* out_k, cudaStream_t s) {
+    const int warps = 8;
+    const int64_t blocks = (rows_pad + warps - 1) / warps;
+    aug_prep_kernel<T, H><<<static_cast<unsigned>(blocks), warps * 32, 0, s>>>(
+        static_cast<const T*>(x), rows, rows_pad, D, Dpa, nt, F, mu, static_cast<H*>(out_q),
+        static_cast<H*>(out_k));
+    return cudaGetLastError();
 }
 
 // ---------------------------------------------------------------- finalise
@@ -321,7 +434,10 @@ cudaError_t launch_mean(InType t, const void* q, const void* k, int64_t M, int64
     }
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
-    mean_final_kernel<<<(D + 127) / 128, 128, 0, s>>>(partial, G, D, static_cast<double>(total), mu);
+    const int mant_bits = t == InType::F16 ? 10 : t == InType::BF16 ? 7 : 23;
+    const int min_exp = t == InType::F16 ? -24 : t == InType::BF16 ? -133 : -149;
+    mean_final_kernel<<<(D + 127) / 128, 128, 0, s>>>(partial, G, D, static_cast<double>(total),
+                                                      mant_bits, min_exp, mu);
     return cudaGetLastError();
 }
 
@@ -347,6 +463,15 @@ cudaError_t launch_value_prep(InType t, bool grad, const void* v, const void* k,
                                                  inv_scale, s)
                 : value_prep_typed<__half, false>(v, k, mu, N, Npad, D, Cv, Cp, vmax_bits, vt,
                                                   inv_scale, s);
+}
+
+cudaError_t launch_aug_prep(InType t, const void* x, int64_t rows, int64_t rows_pad, int D,
+                            int Dpa, const float* mu, void* out_q, void* out_k, cudaStream_t s) {
+    const int nt = aug_norm_terms(t);
+    if (t == InType::BF16)
+        return aug_typed<__nv_bfloat16, __nv_bfloat16>(x, rows, rows_pad, D, Dpa, nt, 1.f, mu,
+                                                       out_q, out_k, s);
+    return aug_typed<__half, __half>(x, rows, rows_pad, D, Dpa, nt, 1024.f, mu, out_q, out_k, s);
 }
 
 cudaError_t launch_key_records(InType t, const void* v, const float* B, int64_t N, int64_t Npad,

@@ -368,8 +368,8 @@ cudaError_t launch_bn(const TcPlan& pl, InType t, float c, char* ws, unsigned* s
 
 }  // namespace
 
-bool plan_tensor(int64_t M, int64_t N, int64_t D, int64_t C, bool grad, bool center, bool alias,
-                 int split_override, int sms, TcPlan* p, const char** why) {
+bool plan_tensor(InType t, int64_t M, int64_t N, int64_t D, int64_t C, bool grad, bool center,
+                 bool alias, int split_override, int sms, TcPlan* p, const char** why) {
     p->M = M;
     p->N = N;
     p->D = D;
@@ -383,9 +383,17 @@ bool plan_tensor(int64_t M, int64_t N, int64_t D, int64_t C, bool grad, bool cen
     const int nkb = (p->Dp + KB - 1) / KB;
     size_t fma_smem = 0;
     int fma_stages = 0, nq = 1;
+    // Few channels: FMA-pipe kernel.  When the augmented rows fit in 128
+    // columns it takes the augmented operands (q^ in shared memory, norms
+    // folded into the MMA).
+    const int dp_aug = static_cast<int>((D + 2 * aug_norm_terms(t) + 15) / 16 * 16);
+    p->aug = !grad && p->Cv <= kFmaMaxChannels && dp_aug <= kAugMaxDp;
+    const int dp_fma = p->aug ? dp_aug : p->Dp;
     p->fma = !grad && p->Cv <= kFmaMaxChannels &&
-             plan_fma_kernel(p->Dp, static_cast<int>(p->Cv), &nq, &fma_stages, &fma_smem);
+             plan_fma_kernel(dp_fma, static_cast<int>(p->Cv), p->aug, &nq, &fma_stages, &fma_smem);
+    if (!p->fma) p->aug = false;
     if (p->fma) {
+        p->Dp = dp_fma;
         p->BN = 128;
         p->nq = nq;
         p->stages = fma_stages;
@@ -434,15 +442,21 @@ bool plan_tensor(int64_t M, int64_t N, int64_t D, int64_t C, bool grad, bool cen
 
     size_t off = 0;
     auto take = [&](size_t bytes) { size_t o = off; off = align1k(off + bytes); return o; };
-    p->off_mean_part = take(static_cast<size_t>(p->mean_blocks) * D * 4);
+    p->off_mean_part = take(static_cast<size_t>(p->mean_blocks) * D * 2 * 4);
     p->off_mu = take(static_cast<size_t>(D) * 4);
     p->off_qh = take(static_cast<size_t>(p->Mpad) * p->Dp * 2);
-    p->off_kh = alias ? p->off_qh : take(static_cast<size_t>(p->Npad) * p->Dp * 2);
-    p->off_A = take(static_cast<size_t>(p->Mpad) * 4);
-    p->off_B = alias ? p->off_A : take(static_cast<size_t>(p->Npad) * 4);
+    // Augmented query and key operands differ in their extra columns, so
+    // they are separate arrays even when q and k are the same points.
+    p->off_kh = (alias && !p->aug) ? p->off_qh : take(static_cast<size_t>(p->Npad) * p->Dp * 2);
+    if (p->aug) {
+        p->off_A = p->off_B = 0;   // the norms live in the augmented columns
+    } else {
+        p->off_A = take(static_cast<size_t>(p->Mpad) * 4);
+        p->off_B = alias ? p->off_A : take(static_cast<size_t>(p->Npad) * 4);
+    }
     if (p->fma) {
         p->off_vt = p->off_vmax = p->off_inv = 0;
-        p->off_rec = take(static_cast<size_t>(p->Npad / 2) * (2 + 2 * p->Cv) * 4);
+        p->off_rec = take(static_cast<size_t>(p->Npad / 2) * ((p->aug ? 0 : 2) + 2 * p->Cv) * 4);
         p->off_part = take(static_cast<size_t>(p->splits) * p->Mpad * p->Cv * 4);
     } else {
         p->off_rec = 0;

@@ -3,39 +3,36 @@
 // Only the dense contraction runs on the tensor cores: tcgen05 MMAs form
 // S = q^ k^T (fp16/bf16 operands, fp32 accumulator in TMEM) for 128 x 128
 // tiles.  The exponent warps turn each S tile into kernel values
-// 2^(c S + A_m + B_n) = Phi(q_m, k_n) (the exponent is <= 0, so no running
+// Phi(q_m, k_n) = 2^(c S + A_m + B_n) (the exponent is <= 0, so no running
 // maximum is needed; see tc_gauss.cu) and accumulate sum_n Phi v_n in fp32
-// on the FMA pipe.  For C <= 4 this costs fewer issue slots than a second
+// on the FMA pipe.  With augmented operands (prep.cu) the MMA already adds
+// the norm terms, S = -||q^ - k^||^2 / 2, and Phi = 2^(c S).  For C <= 4 this costs fewer issue slots than a second
 // MMA with N = 16, and it keeps kernel values and values in fp32.
 //
 // Layout choices:
-//   * Shared-memory bandwidth (128 B/clk/SM): an M=128, N=128, K=16 MMA
-//     with both operands in shared memory would use all of it, and such
-//     MMAs also slow down while other warps read TMEM.  So the query
-//     operand q^ lives in TMEM (A operand of tcgen05.mma) and only the key
-//     tile k^ is read from shared memory.
 //   * A CTA owns two query tiles (256 rows), which halves the L2 -> shared
 //     memory traffic of the key tiles; every exponent warp handles the same
 //     key columns of both query tiles, so one broadcast load of a key
 //     record serves two kernel values.
-//   * Barrier handshakes cost the single issuing thread one to two hundred
-//     cycles each, so there is one handshake per key tile (not per MMA
-//     tile): the MMA thread issues the 2 x (Dp / 16) MMAs of a key tile back
-//     to back and commits once; the exponent warps release both S buffers
-//     of the key tile with one arrival per warp, as soon as they are in
-//     registers.
+//   * Barrier handshakes cost the single MMA-issuing thread one to two
+//     hundred cycles each, so there is one handshake per key tile: the MMA
+//     thread issues the 2 x (Dp / 16) MMAs of a key tile back to back and
+//     commits once; the exponent warps release both S buffers of the key
+//     tile with one arrival per warp, as soon as they are in registers.
+//   * TMEM holds SL slots of two 128-column S buffers (one per query
+//     tile); key tile j uses slot j % SL, so the MMAs of key tile j only
+//     wait for the release of key tile j - SL.  With Dp <= 128 the query
+//     tiles q^ stay in shared memory (A operand read by the MMA from shared
+//     memory) and SL = 2; with larger Dp they would not fit next to the key
+//     stages, so q^ is copied into TMEM (A operand from TMEM) and SL = 1.
 //
 // Warp roles (18 warps):
 //   warps 0-15  exponent warps.  Warp w reads TMEM lanes 32 (w % 4) .. +31
 //               (rows of both query tiles) and key columns 32 (w / 4) .. +31
-//               of the two S buffers of each key tile; at the start it
-//               copies its share of q^ from global memory into TMEM.
-//   warp 16     TMA producer: per key tile the k^ rows and the key records.
+//               of the two S buffers of each key tile.
+//   warp 16     TMA producer: the q^ tiles (shared-memory variant), then per
+//               key tile the k^ rows and the key records.
 //   warp 17     TMEM allocator and single-thread MMA issuer.
-// TMEM columns: NB S buffers of 128 columns, then the two q^ tiles
-// (Dp / 2 columns each, fp16/bf16 pairs packed in 32-bit columns).  Key
-// tile j uses S buffers (2j) % NB and (2j + 1) % NB, so with NB = 2 or 3 the
-// MMAs of key tile j may start once key tile j - 1 has been released.
 // Key records: for each pair of keys (2t, 2t + 1) the floats
 //   B_2t, B_2t+1, v_2t[0], v_2t+1[0], ..., v_2t[C-1], v_2t+1[C-1].
 #include <cuda.h>
@@ -59,7 +56,7 @@ constexpr int PRODUCER_WARP = 16;
 constexpr int MMA_WARP = 17;
 constexpr int THREADS = 18 * 32;
 constexpr int NPART = 4;           // column groups (partial sums) per row
-constexpr int MAX_NB = 3;
+constexpr int MAX_SL = 2;          // TMEM slots of two S buffers
 constexpr uint32_t TMEM_COLS = 512;
 constexpr int MAX_STAGES = 8;
 
@@ -73,9 +70,9 @@ struct FmaParams {
     int key_tiles;
     int tiles_per_split;
     int Dp;
-    int nkb;             // 64-element K blocks of k^
-    int nb;              // S buffers in TMEM
+    int nkb;             // 64-element K blocks of q^ / k^
     int stages;
+    uint32_t q_bytes;    // shared-memory q^ tiles (0 when q^ is in TMEM)
     uint32_t stage_bytes;
     uint32_t kh_bytes;
     uint32_t rec_bytes;  // key-record bytes of one key tile
@@ -85,10 +82,10 @@ struct FmaParams {
 };
 
 struct __align__(8) FmaBarriers {
-    uint64_t qa_ready;   // q^ copied into TMEM (16 warp arrivals)
+    uint64_t qa_ready;          // q^ available to the MMAs
     uint64_t drain;
-    uint64_t s_full;     // phase j: both S tiles of key tile j computed
-    uint64_t s_free;     // phase j: both S tiles of key tile j in registers
+    uint64_t s_full[MAX_SL];    // slot phase: both S tiles of a key tile computed
+    uint64_t s_free[MAX_SL];    // slot phase: both S tiles of a key tile in registers
     uint64_t kv_full[MAX_STAGES];
     uint64_t kv_empty[MAX_STAGES];
     uint32_t tmem_base;
@@ -105,14 +102,19 @@ __device__ __forceinline__ void exp_warps_sync() {
     asm volatile("bar.sync 1, %0;" ::"r"(NEXP * 32) : "memory");
 }
 
-template <int C>
+// QS: q^ tiles in shared memory (A operand from shared memory, SL = 2);
+// otherwise q^ in TMEM (A operand from TMEM, SL = 1).
+template <int C, bool QS>
 __global__ void __launch_bounds__(THREADS, 1)
-tc_gauss_fma_kernel(const __grid_constant__ CUtensorMap tm_k, const FmaParams p) {
-    constexpr int REC_PAIR = 2 + 2 * C;               // floats per key pair
+tc_gauss_fma_kernel(const __grid_constant__ CUtensorMap tm_q,
+                    const __grid_constant__ CUtensorMap tm_k, const FmaParams p) {
+    constexpr int REC_PAIR = (QS ? 0 : 2) + 2 * C;    // floats per key pair
+    constexpr int SL = QS ? 2 : 1;
     extern __shared__ uint8_t smem_raw[];
     const uint32_t raw_addr = smem_u32(smem_raw);
     uint8_t* smem = smem_raw + (((raw_addr + 1023u) & ~1023u) - raw_addr);
-    uint8_t* stage0 = smem;
+    uint8_t* q_smem = smem;                            // QS: NQ x nkb x 16 KB
+    uint8_t* stage0 = smem + p.q_bytes;
     float* red = reinterpret_cast<float*>(smem + p.red_offset);    // NPART x 256 x C
     FmaBarriers* bars = reinterpret_cast<FmaBarriers*>(smem + p.red_offset + NPART * NQ * BM * C * 4);
 
@@ -123,14 +125,15 @@ tc_gauss_fma_kernel(const __grid_constant__ CUtensorMap tm_k, const FmaParams p)
     const int split = blockIdx.y;
     const int kt0 = split * p.tiles_per_split;
     const int T = min(p.key_tiles, kt0 + p.tiles_per_split) - kt0;
-    const int NB = p.nb;
     volatile int* abort_flag = &bars->abort_flag;
 
     if (tid == 0) {
-        mbar_init(&bars->qa_ready, NEXP);
+        mbar_init(&bars->qa_ready, QS ? 1 : NEXP);
         mbar_init(&bars->drain, 1);
-        mbar_init(&bars->s_full, 1);
-        mbar_init(&bars->s_free, NEXP);                // one arrival per exponent warp
+        for (int sl = 0; sl < SL; ++sl) {
+            mbar_init(&bars->s_full[sl], 1);
+            mbar_init(&bars->s_free[sl], NEXP);        // one arrival per exponent warp
+        }
         for (int s = 0; s < p.stages; ++s) {
             mbar_init(&bars->kv_full[s], 1);
             mbar_init(&bars->kv_empty[s], 1 + NEXP);  // MMA commit + exponent warps
@@ -146,7 +149,7 @@ tc_gauss_fma_kernel(const __grid_constant__ CUtensorMap tm_k, const FmaParams p)
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = bars->tmem_base;
-    const uint32_t qa_col = static_cast<uint32_t>(NB * BN);   // q^ tile h at qa_col + h Dp/2
+    const uint32_t qa_col = static_cast<uint32_t>(2 * SL * BN);   // TMEM q^ (not QS)
 
     auto kh_smem = [&](int s) { return stage0 + s * p.stage_bytes; };
     auto rec_smem = [&](int s) {
@@ -154,70 +157,100 @@ tc_gauss_fma_kernel(const __grid_constant__ CUtensorMap tm_k, const FmaParams p)
     };
 
     if (warp == PRODUCER_WARP) {
-        if (lane == 0 && T > 0) {
-            tma_prefetch_desc(&tm_k);
+        // The whole warp runs the loop (warp-uniform operands); the elected
+        // lane issues the copies.
+        if (T > 0) {
+            const bool leader = elect_one();
+            if (leader) {
+                tma_prefetch_desc(&tm_k);
+                if (QS) {
+                    tma_prefetch_desc(&tm_q);
+                    mbar_arrive_expect_tx(&bars->qa_ready, p.q_bytes);
+                    for (int h = 0; h < NQ; ++h)
+                        for (int kb = 0; kb < p.nkb; ++kb)
+                            tma_load_2d(q_smem + (h * p.nkb + kb) * (BM * 128), &tm_q, &bars->qa_ready,
+                                        kb * KB, (tile_m * NQ + h) * BM);
+                }
+            }
+            __syncwarp();
             int issued = 0;
             RingPos st;
             for (int j = 0; j < T; ++j, st.advance(p.stages)) {
                 const int s = st.idx;
-                if (!mbar_wait_bounded(&bars->kv_empty[s], st.phase ^ 1u, abort_flag, p.status)) break;
-                mbar_arrive_expect_tx(&bars->kv_full[s], p.kh_bytes + p.rec_bytes);
-                const int n0 = (kt0 + j) * BN;
-                for (int kb = 0; kb < p.nkb; ++kb)
-                    tma_load_2d(kh_smem(s) + kb * (BN * 128), &tm_k, &bars->kv_full[s], kb * KB, n0);
-                bulk_load(const_cast<float*>(rec_smem(s)), p.rec + static_cast<int64_t>(n0 / 2) * REC_PAIR,
-                          p.rec_bytes, &bars->kv_full[s]);
+                if (!warp_wait(&bars->kv_empty[s], st.phase ^ 1u, abort_flag, p.status)) break;
+                if (leader) {
+                    mbar_arrive_expect_tx(&bars->kv_full[s], p.kh_bytes + p.rec_bytes);
+                    const int n0 = (kt0 + j) * BN;
+                    for (int kb = 0; kb < p.nkb; ++kb)
+                        tma_load_2d(kh_smem(s) + kb * (BN * 128), &tm_k, &bars->kv_full[s], kb * KB, n0);
+                    bulk_load(const_cast<float*>(rec_smem(s)),
+                              p.rec + static_cast<int64_t>(n0 / 2) * REC_PAIR, p.rec_bytes,
+                              &bars->kv_full[s]);
+                }
+                __syncwarp();
                 issued = j + 1;
             }
             // Every copy this CTA started must land before it exits.
+            if (QS) mbar_wait_bounded(&bars->qa_ready, 0, nullptr, p.status);
             for (int j = max(0, issued - p.stages); j < issued; ++j)
                 mbar_wait_bounded(&bars->kv_full[j % p.stages],
                                   static_cast<uint32_t>(j / p.stages) & 1u, nullptr, p.status);
         }
     } else if (warp == MMA_WARP) {
-        if (lane == 0 && T > 0) {
-            bool ok = mbar_wait_bounded(&bars->qa_ready, 0, abort_flag, p.status);
+        // The whole warp runs the loop (warp-uniform descriptors and TMEM
+        // addresses); the elected lane issues the MMAs and commits.
+        if (T > 0) {
+            const bool leader = elect_one();
+            bool ok = warp_wait(&bars->qa_ready, 0, abort_flag, p.status);
             const int ksteps = p.Dp / 16;
-            // Shared-memory descriptor of k^ stage 0; stage s and K step kk
-            // add (s stage_bytes + (kk / 4) BN 128 + (kk % 4) 32) / 16 to the
+            // Shared-memory descriptors of k^ stage 0 and of q^ tile 0; stage
+            // s, query tile h and K step kk add byte offsets / 16 to the
             // start-address field.
-            const uint64_t desc0 = smem_desc_kmajor_sw128(smem_u32(stage0));
+            const uint64_t kdesc0 = smem_desc_kmajor_sw128(smem_u32(stage0));
+            const uint64_t qdesc0 = smem_desc_kmajor_sw128(smem_u32(q_smem));
+            const uint32_t qdesc_h = static_cast<uint32_t>((p.nkb * BM * 128) >> 4);
             const uint32_t a0 = tmem + qa_col, a1 = a0 + (p.Dp / 2);
-            RingPos st, buf;
-            for (int j = 0; ok && j < T; ++j, st.advance(p.stages)) {
+            RingPos st, sl;
+            for (int j = 0; ok && j < T; ++j, st.advance(p.stages), sl.advance(SL)) {
                 const int s = st.idx;
-                // Key tile j - 1 released (which also frees the buffers of
-                // earlier tiles) and stage s loaded; both queried at once.
-                const uint32_t free_parity = static_cast<uint32_t>(j - 1) & 1u;
-                const bool ready = j == 0 ? mbar_test_wait(&bars->kv_full[s], st.phase)
-                                          : mbar_test_wait2(&bars->s_free, free_parity,
-                                                            &bars->kv_full[s], st.phase);
+                // Key tile j - SL released its slot and stage s is loaded;
+                // both queried at once.
+                const uint32_t free_parity = sl.phase ^ 1u;
+                const bool ready = __all_sync(
+                    0xffffffffu, j < SL ? mbar_test_wait(&bars->kv_full[s], st.phase)
+                                        : mbar_test_wait2(&bars->s_free[sl.idx], free_parity,
+                                                          &bars->kv_full[s], st.phase));
                 if (!ready) {
-                    if (j > 0) {
-                        ok = mbar_wait_bounded(&bars->s_free, free_parity, abort_flag, p.status);
+                    if (j >= SL) {
+                        ok = warp_wait(&bars->s_free[sl.idx], free_parity, abort_flag, p.status);
                         if (!ok) break;
                     }
-                    ok = mbar_wait_bounded(&bars->kv_full[s], st.phase, abort_flag, p.status);
+                    ok = warp_wait(&bars->kv_full[s], st.phase, abort_flag, p.status);
                     if (!ok) break;
                 }
                 tc_fence_after();
-                const uint32_t d0 = tmem + buf.idx * BN;
-                buf.advance(NB);
-                const uint32_t d1 = tmem + buf.idx * BN;
-                buf.advance(NB);
-                const uint64_t bdesc = desc0 + ((static_cast<uint64_t>(s) * p.stage_bytes) >> 4);
-                for (int kk = 0; kk < ksteps; ++kk) {
-                    const uint64_t bd = bdesc + static_cast<uint64_t>((kk >> 2) * (BN * 128 / 16) + (kk & 3) * 2);
-                    mma_ts_f16(d0, a0 + kk * 8, bd, p.idesc, kk > 0 ? 1u : 0u);
+                const uint32_t d0 = tmem + sl.idx * (2 * BN), d1 = d0 + BN;
+                const uint64_t kdesc = kdesc0 + ((static_cast<uint64_t>(s) * p.stage_bytes) >> 4);
+                if (leader) {
+                for (int h = 0; h < NQ; ++h) {
+                    for (int kk = 0; kk < ksteps; ++kk) {
+                        const uint32_t koff = static_cast<uint32_t>((kk >> 2) * (BN * 128 / 16) + (kk & 3) * 2);
+                        if (QS) {
+                            const uint32_t qoff = h * qdesc_h + static_cast<uint32_t>((kk >> 2) * (BM * 128 / 16) + (kk & 3) * 2);
+                            mma_ss_f16(h ? d1 : d0, qdesc0 + qoff, kdesc + koff, p.idesc, kk > 0 ? 1u : 0u);
+                        } else {
+                            mma_ts_f16(h ? d1 : d0, (h ? a1 : a0) + kk * 8, kdesc + koff, p.idesc,
+                                       kk > 0 ? 1u : 0u);
+                        }
+                    }
                 }
-                for (int kk = 0; kk < ksteps; ++kk) {
-                    const uint64_t bd = bdesc + static_cast<uint64_t>((kk >> 2) * (BN * 128 / 16) + (kk & 3) * 2);
-                    mma_ts_f16(d1, a1 + kk * 8, bd, p.idesc, kk > 0 ? 1u : 0u);
-                }
-                mma_commit(&bars->s_full);
+                mma_commit(&bars->s_full[sl.idx]);
                 mma_commit(&bars->kv_empty[s]);
+                }
+                __syncwarp();
             }
-            mma_commit(&bars->drain);
+            if (leader) mma_commit(&bars->drain);
+            __syncwarp();
             mbar_wait_bounded(&bars->drain, 0, nullptr, p.status);
         }
     } else {
@@ -229,9 +262,9 @@ tc_gauss_fma_kernel(const __grid_constant__ CUtensorMap tm_k, const FmaParams p)
         const int64_t row0 = static_cast<int64_t>(tile_m) * NQ * BM + row_t;
         const int64_t row1 = row0 + BM;
 
-        // q^ rows -> TMEM (A operand).  Column group cg copies query tile
-        // cg / 2, 8-column chunks ck = cg % 2 (mod 2) of its Dp / 2 columns.
-        {
+        if (!QS) {
+            // q^ rows -> TMEM (A operand).  Column group cg copies query tile
+            // cg / 2, 8-column chunks ck = cg % 2 (mod 2) of its Dp / 2 columns.
             const int h = cg >> 1;
             const uint32_t* src = p.qh + (row0 + h * BM) * (p.Dp / 2);
             for (int ck = cg & 1; ck < p.Dp / 16; ck += 2) {
@@ -246,37 +279,56 @@ tc_gauss_fma_kernel(const __grid_constant__ CUtensorMap tm_k, const FmaParams p)
             if (lane == 0) mbar_arrive(&bars->qa_ready);
         }
 
-        const uint64_t a2_0 = f32x2_pack(p.A[row0], p.A[row0]);
-        const uint64_t a2_1 = f32x2_pack(p.A[row1], p.A[row1]);
+        // Row terms of the exponent (only without augmented operands).
+        const float am0 = QS ? 0.f : p.A[row0];
+        const float am1 = QS ? 0.f : p.A[row1];
+        const uint64_t a2_0 = f32x2_pack(am0, am0);
+        const uint64_t a2_1 = f32x2_pack(am1, am1);
         const uint64_t c2 = f32x2_pack(p.c, p.c);
         uint64_t acc0[C], acc1[C];
 #pragma unroll
         for (int cc = 0; cc < C; ++cc) acc0[cc] = acc1[cc] = 0ull;
         bool ok = true;
-        RingPos st, buf;   // stage of key tile j; S buffer of its first tile
-        for (int j = 0; j < T; ++j, st.advance(p.stages)) {
+        RingPos st, sl;   // stage and TMEM slot of key tile j
+        for (int j = 0; j < T; ++j, st.advance(p.stages), sl.advance(SL)) {
             const int s = st.idx;
-            const uint32_t col0 = static_cast<uint32_t>(buf.idx * BN);
-            buf.advance(NB);
-            const uint32_t col1 = static_cast<uint32_t>(buf.idx * BN);
-            buf.advance(NB);
-            const uint32_t full_parity = static_cast<uint32_t>(j) & 1u;
-            if (!__all_sync(0xffffffffu, mbar_test_wait2(&bars->kv_full[s], st.phase, &bars->s_full,
-                                                         full_parity))) {
+            const uint32_t col0 = static_cast<uint32_t>(sl.idx * 2 * BN);
+            if (!__all_sync(0xffffffffu, mbar_test_wait2(&bars->kv_full[s], st.phase,
+                                                         &bars->s_full[sl.idx], sl.phase))) {
                 ok = warp_wait(&bars->kv_full[s], st.phase, abort_flag, p.status);
-                if (ok) ok = warp_wait(&bars->s_full, full_parity, abort_flag, p.status);
+                if (ok) ok = warp_wait(&bars->s_full[sl.idx], sl.phase, abort_flag, p.status);
                 if (!ok) break;
             }
             tc_fence_after();
             uint32_t r0[32], r1[32];
             tmem_ld_32x32b_x32(tmem + lane_base + col0 + cg * 32, r0);
-            tmem_ld_32x32b_x32(tmem + lane_base + col1 + cg * 32, r1);
+            tmem_ld_32x32b_x32(tmem + lane_base + col0 + BN + cg * 32, r1);
             tmem_wait_ld();
-            // Both S slices are in registers: hand the buffers back.
+            // Both S slices are in registers: hand the slot back.
             tc_fence_before();
             __syncwarp();
-            if (lane == 0) mbar_arrive(&bars->s_free);
+            if (lane == 0) mbar_arrive(&bars->s_free[sl.idx]);
             const float* rec = rec_smem(s) + (cg * 16) * REC_PAIR;
+            if (QS) {
+                // Augmented operands: S = -||q^ - k^||^2 / 2, so Phi = 2^(c S).
+                // Keys 32 cg + 2t and + 1, rows row0 (S0) and row1 (S1).
+#pragma unroll
+                for (int t = 0; t < 16; ++t) {
+                    const float* pr = rec + t * REC_PAIR;
+                    float x0, x1, y0, y1;
+                    f32x2_unpack(f32x2_mul(f32x2_pack(__uint_as_float(r0[2 * t]), __uint_as_float(r0[2 * t + 1])), c2), x0, x1);
+                    f32x2_unpack(f32x2_mul(f32x2_pack(__uint_as_float(r1[2 * t]), __uint_as_float(r1[2 * t + 1])), c2), y0, y1);
+                    const uint64_t px = f32x2_pack(ex2_approx(x0), ex2_approx(x1));
+                    const uint64_t py = f32x2_pack(ex2_approx(y0), ex2_approx(y1));
+#pragma unroll
+                    for (int cc = 0; cc < C; ++cc) {
+                        const float2 vc = *reinterpret_cast<const float2*>(pr + 2 * cc);
+                        const uint64_t vv = f32x2_pack(vc.x, vc.y);
+                        acc0[cc] = f32x2_fma(px, vv, acc0[cc]);
+                        acc1[cc] = f32x2_fma(py, vv, acc1[cc]);
+                    }
+                }
+            } else {
 #pragma unroll
             for (int t = 0; t < 16; ++t) {
                 // Keys 32 cg + 2t and + 1, rows row0 (S0) and row1 (S1).
@@ -310,6 +362,7 @@ tc_gauss_fma_kernel(const __grid_constant__ CUtensorMap tm_k, const FmaParams p)
                     acc0[cc] = f32x2_fma(px, vv, acc0[cc]);
                     acc1[cc] = f32x2_fma(py, vv, acc1[cc]);
                 }
+            }
             }
             __syncwarp();
             if (lane == 0) mbar_arrive(&bars->kv_empty[s]);
@@ -348,30 +401,39 @@ tc_gauss_fma_kernel(const __grid_constant__ CUtensorMap tm_k, const FmaParams p)
 
 size_t align1k(size_t x) { return (x + 1023) & ~static_cast<size_t>(1023); }
 
-size_t stage_bytes_for(int nkb, int C) {
-    return align1k(static_cast<size_t>(nkb) * BN * 128 + static_cast<size_t>(BN / 2) * (2 + 2 * C) * 4);
+// Floats per key pair in the key records: (B_2t, B_2t+1 unless the norms
+// are folded into augmented operands) + both keys' values.
+int rec_pair_floats(int C, bool aug) { return (aug ? 0 : 2) + 2 * C; }
+
+size_t stage_bytes_for(int nkb, int C, bool aug) {
+    return align1k(static_cast<size_t>(nkb) * BN * 128 +
+                   static_cast<size_t>(BN / 2) * rec_pair_floats(C, aug) * 4);
 }
 
-size_t fixed_bytes_for(int C) {
-    return 1024 /*alignment slack*/ + static_cast<size_t>(NPART) * NQ * BM * C * 4 +
+size_t fixed_bytes_for(int C, size_t q_bytes) {
+    return 1024 /*alignment slack*/ + q_bytes + static_cast<size_t>(NPART) * NQ * BM * C * 4 +
            sizeof(FmaBarriers) + 64;
 }
 
-int buffers_for(int Dp) { return std::min(MAX_NB, (static_cast<int>(TMEM_COLS) - Dp) / BN); }
+// q^ tiles in shared memory (augmented variant only).
+size_t q_bytes_for(int Dp, bool aug) {
+    return aug ? static_cast<size_t>(NQ) * ((Dp + KB - 1) / KB) * BM * 128 : 0;
+}
 
-template <int C>
+template <int C, bool QS>
 cudaError_t launch_typed(const TcPlan& pl, InType t, float c, char* ws, unsigned* status,
                          cudaStream_t s, const char** why) {
     const CUtensorMapDataType hdt =
         t == InType::BF16 ? CU_TENSOR_MAP_DATA_TYPE_BFLOAT16 : CU_TENSOR_MAP_DATA_TYPE_FLOAT16;
-    CUtensorMap tm_k;
-    if (!encode_tile_map_2d(&tm_k, hdt, ws + pl.off_kh, pl.Dp, pl.Npad, pl.Dp * 2ull, KB, BN)) {
+    CUtensorMap tm_q, tm_k;
+    if (!encode_tile_map_2d(&tm_k, hdt, ws + pl.off_kh, pl.Dp, pl.Npad, pl.Dp * 2ull, KB, BN) ||
+        !encode_tile_map_2d(&tm_q, hdt, ws + pl.off_qh, pl.Dp, pl.Mpad, pl.Dp * 2ull, KB, BM)) {
         *why = "cuTensorMapEncodeTiled failed or is unavailable";
         return cudaErrorInvalidValue;
     }
     FmaParams p;
     p.qh = reinterpret_cast<const uint32_t*>(ws + pl.off_qh);
-    p.A = reinterpret_cast<const float*>(ws + pl.off_A);
+    p.A = QS ? nullptr : reinterpret_cast<const float*>(ws + pl.off_A);
     p.rec = reinterpret_cast<const float*>(ws + pl.off_rec);
     p.part = reinterpret_cast<float*>(ws + pl.off_part);
     p.status = status;
@@ -380,32 +442,43 @@ cudaError_t launch_typed(const TcPlan& pl, InType t, float c, char* ws, unsigned
     p.tiles_per_split = (p.key_tiles + pl.splits - 1) / pl.splits;
     p.Dp = pl.Dp;
     p.nkb = (pl.Dp + KB - 1) / KB;
-    p.nb = buffers_for(pl.Dp);
     p.stages = pl.stages;
+    p.q_bytes = static_cast<uint32_t>(q_bytes_for(pl.Dp, QS));
     p.kh_bytes = static_cast<uint32_t>(p.nkb * BN * 128);
-    p.rec_bytes = static_cast<uint32_t>((BN / 2) * (2 + 2 * C) * 4);
-    p.stage_bytes = static_cast<uint32_t>(stage_bytes_for(p.nkb, C));
-    p.red_offset = static_cast<uint32_t>(pl.stages * p.stage_bytes);
+    p.rec_bytes = static_cast<uint32_t>((BN / 2) * rec_pair_floats(C, QS) * 4);
+    p.stage_bytes = static_cast<uint32_t>(stage_bytes_for(p.nkb, C, QS));
+    p.red_offset = p.q_bytes + static_cast<uint32_t>(pl.stages * p.stage_bytes);
     p.c = c;
     const uint32_t hb = t == InType::BF16 ? 1u : 0u;
     p.idesc = idesc_f16(BM, BN, hb, hb);
-    cudaError_t e = cudaFuncSetAttribute(tc_gauss_fma_kernel<C>,
+    cudaError_t e = cudaFuncSetAttribute(tc_gauss_fma_kernel<C, QS>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          static_cast<int>(pl.smem_bytes));
     if (e != cudaSuccess) return e;
     dim3 grid(static_cast<unsigned>(pl.Mpad / (NQ * BM)), static_cast<unsigned>(pl.splits));
-    tc_gauss_fma_kernel<C><<<grid, THREADS, pl.smem_bytes, s>>>(tm_k, p);
+    tc_gauss_fma_kernel<C, QS><<<grid, THREADS, pl.smem_bytes, s>>>(tm_q, tm_k, p);
     return cudaGetLastError();
+}
+
+template <int C>
+cudaError_t launch_c(const TcPlan& pl, InType t, float c, char* ws, unsigned* status,
+                     cudaStream_t s, const char** why) {
+    if (pl.aug) return launch_typed<C, true>(pl, t, c, ws, status, s, why);
+    return launch_typed<C, false>(pl, t, c, ws, status, s, why);
 }
 
 }  // namespace
 
-bool plan_fma_kernel(int Dp, int C, int* nq, int* stages, size_t* smem) {
-    if (C < 1 || C > kFmaMaxChannels || Dp > 256 || buffers_for(Dp) < 2) return false;
+bool plan_fma_kernel(int Dp, int C, bool aug, int* nq, int* stages, size_t* smem) {
+    if (C < 1 || C > kFmaMaxChannels || Dp > 256) return false;
+    if (aug && Dp > kAugMaxDp) return false;
+    // TMEM: q^ in TMEM needs Dp columns beside one slot of two S buffers.
+    if (!aug && static_cast<int>(TMEM_COLS) - 2 * BN < Dp) return false;
     const int nkb = (Dp + KB - 1) / KB;
     const size_t budget = 232448;
-    const size_t stage = stage_bytes_for(nkb, C);
-    const size_t fixed = fixed_bytes_for(C);
+    const size_t stage = stage_bytes_for(nkb, C, aug);
+    const size_t fixed = fixed_bytes_for(C, q_bytes_for(Dp, aug));
+    if (fixed >= budget) return false;
     const int st = static_cast<int>(std::min<size_t>(MAX_STAGES, (budget - fixed) / stage));
     if (st < 2) return false;
     *nq = NQ;
@@ -417,10 +490,10 @@ bool plan_fma_kernel(int Dp, int C, int* nq, int* stages, size_t* smem) {
 cudaError_t launch_tc_fma(const TcPlan& p, InType t, float c, char* ws, unsigned* status,
                           cudaStream_t s, const char** why) {
     switch (p.Cv) {
-        case 1: return launch_typed<1>(p, t, c, ws, status, s, why);
-        case 2: return launch_typed<2>(p, t, c, ws, status, s, why);
-        case 3: return launch_typed<3>(p, t, c, ws, status, s, why);
-        default: return launch_typed<4>(p, t, c, ws, status, s, why);
+        case 1: return launch_c<1>(p, t, c, ws, status, s, why);
+        case 2: return launch_c<2>(p, t, c, ws, status, s, why);
+        case 3: return launch_c<3>(p, t, c, ws, status, s, why);
+        default: return launch_c<4>(p, t, c, ws, status, s, why);
     }
 }
 

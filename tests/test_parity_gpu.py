@@ -124,6 +124,25 @@ def test_fp16_kernel_value_floor():
     assert np.all(err <= 2e-3 * den[:, 0] + flushed + 1e-30)
 
 
+@pytest.mark.parametrize("dtype", ["fp16", "bf16"])
+def test_norms_beyond_fp16_range(dtype):
+    """Two clusters at +-40 per coordinate (D = 64): ||x - mu||^2 ~ 1e5 is
+    above the fp16 range, so the folded norm terms need their range factor."""
+    from oracle import oracle_sum
+    rng = np.random.default_rng(11)
+    M, N, D, C = 200, 333, 64, 2
+    tdt = {"fp16": torch.float16, "bf16": torch.bfloat16}[dtype]
+    def pts(n):
+        x = rng.standard_normal((n, D)) + np.where(rng.random((n, 1)) < 0.5, -40.0, 40.0)
+        return torch.from_numpy(x).to(tdt)
+    q, k = pts(M), pts(N)
+    v = torch.from_numpy(rng.standard_normal((N, C))).to(tdt)
+    tau = 1.0 / 16
+    s = _call(q.cuda(), k.cuda(), v.cuda(), tau).cpu().numpy()
+    ref, den = oracle_sum(q.double().numpy(), k.double().numpy(), v.double().numpy(), tau)
+    assert rel_err(s, ref, den) <= TOL[dtype]
+
+
 def test_deterministic_bitwise():
     import paper_2609_04910_gb300 as gs
     from paper_2609_04910_gb300.workloads import generate
