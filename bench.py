@@ -206,36 +206,36 @@ def measured_peaks():
 
 
 def kernel_source_hash():
+    """Hash of every library source file: a profile taken on other sources
+    no longer describes the kernel."""
     h = hashlib.sha256()
-    for name in ("tc_gauss.cu", "ptx.cuh"):
-        with open(os.path.join(ROOT, "paper_2609_04910_gb300", "csrc", name), "rb") as f:
-            h.update(f.read())
+    csrc = os.path.join(ROOT, "paper_2609_04910_gb300", "csrc")
+    for name in sorted(os.listdir(csrc)):
+        if name.endswith((".cu", ".cuh", ".h")):
+            with open(os.path.join(csrc, name), "rb") as f:
+                h.update(name.encode())
+                h.update(f.read())
     return h.hexdigest()[:16]
 
 
-def profiled_traffic(workload):
+def main_kernel_name(w):
+    """Fused kernel the library picks for this workload (plan in csrc)."""
+    if w.dtype == "fp32":
+        return "simt_gauss_kernel"
+    return "tc_gauss_fma_kernel" if (not w.grad and w.C <= 4) else "tc_gauss_kernel"
+
+
+def profiled_traffic(w):
     """DRAM bytes per launch of the fused kernel from the committed ncu
-    summary, if it was taken on the current kernel source."""
+    summary, if it was taken on the current library sources."""
     src = kernel_source_hash()
-    for path in glob.glob(os.path.join(ROOT, "profiles", f"tc_gauss_kernel*{workload}*.md")):
+    for path in glob.glob(os.path.join(ROOT, "profiles", f"{main_kernel_name(w)}_{w.name}*.md")):
         text = open(path).read()
         m_h = re.search(r"source_sha256_16:\s*([0-9a-f]+)", text)
         m_t = re.search(r"dram_bytes_per_launch:\s*([0-9.eE+]+)", text)
         if m_h and m_t and m_h.group(1) == src:
             return float(m_t.group(1)), os.path.relpath(path, ROOT)
     return None, None
-
-
-def launches_per_step(w, center=True):
-    """Kernels of this library one call launches (plan in csrc/api.cu)."""
-    if w.dtype == "fp32":
-        return 2  # SIMT kernel + finalise
-    n = 5  # centre/cast/norm of q, value max, value prep, fused kernel, finalise
-    if not w.q_is_k:
-        n += 1  # centre/cast/norm of k
-    if center and w.D > 0:
-        n += 2  # mean partial sums + final mean
-    return n
 
 
 # ---------------------------------------------------------------- own arm
@@ -300,11 +300,13 @@ def run_own(args):
     barrier()
     torch.cuda.synchronize()
     wall0 = time.perf_counter()
+    launches0 = gs.gauss_sum_kernel_launches()
     for i in range(K):
         flush.zero_()
         ev[i][0].record(stream)
         step(main_events=mev[i])
         ev[i][1].record(stream)
+    launches = gs.gauss_sum_kernel_launches() - launches0
     torch.cuda.synchronize()
     barrier()
     wall = time.perf_counter() - wall0
@@ -377,28 +379,33 @@ def run_own(args):
     t_tensor = flops / r_t
     t_sfu = exps / r_x
     t_main = main_mean * 1e-3
-    traffic, traffic_src = profiled_traffic(w.name)
+    traffic, traffic_src = profiled_traffic(w)
     if w.dtype == "fp32":
         roof = None
     elif t_sfu >= t_tensor:
-        roof = {"bound": "sfu", "achieved": exps / t_main / 1e12, "peak": r_x / 1e12,
-                "unit": "Texp/s", "frac": (t_sfu / t_main)}
+        # Bound by the MUFU exp2 issue rate: peak from unit count x SMs x
+        # maximum SM clock (32 ex2 per clock per SM, the rate the probe
+        # reaches at the maximum clock).
+        roof = {"bound": "alu", "achieved": exps / t_main / 1e12, "peak": r_x_nominal / 1e12,
+                "unit": "Texp/s", "frac": exps / r_x_nominal / t_main}
     else:
         roof = {"bound": "tensor", "achieved": flops / t_main / 1e12, "peak": r_t / 1e12,
                 "unit": "TFLOP/s", "frac": (t_tensor / t_main)}
     if roof is not None:
         roof.update({
             "traffic": traffic, "traffic_source": traffic_src,
-            "kernel": "tc_gauss_kernel", "kernel_ms": main_mean,
-            "t_roof_ms": max(t_tensor, t_sfu) * 1e3,
-            "peak_note": ("SFU peak = ex2.approx throughput measured live by the library's probe "
-                          f"({r_x:.4g}/s; nominal 32/clk/SM x {sms} SMs x {sm_max_mhz:.0f} MHz = "
-                          f"{r_x_nominal:.4g}/s); tensor peak = {peak_src} bf16 dense "
-                          f"{r_t/1e12:.1f} TFLOP/s (fp16 runs at the bf16 rate)"),
+            "kernel": main_kernel_name(w), "kernel_ms": main_mean,
+            "t_roof_ms": max(t_tensor, exps / r_x_nominal) * 1e3,
+            "peak_note": ("alu = MUFU ex2.approx: 32/clk/SM x "
+                          f"{sms} SMs x {sm_max_mhz:.0f} MHz = {r_x_nominal:.4g}/s "
+                          f"(the library's probe measured {r_x:.4g}/s live); tensor peak = "
+                          f"{peak_src} bf16 dense {r_t/1e12:.1f} TFLOP/s (fp16 runs at the bf16 "
+                          "rate)"),
             "tensor": {"achieved": flops / t_main / 1e12, "peak": r_t / 1e12, "unit": "TFLOP/s",
                        "frac": t_tensor / t_main},
-            "sfu": {"achieved": exps / t_main / 1e12, "peak": r_x / 1e12, "unit": "Texp/s",
-                    "frac": t_sfu / t_main},
+            "sfu": {"achieved": exps / t_main / 1e12, "peak": r_x_nominal / 1e12,
+                    "unit": "Texp/s", "frac": exps / r_x_nominal / t_main,
+                    "probe_ex2_per_s": r_x},
         })
 
     cpu = None
@@ -418,7 +425,7 @@ def run_own(args):
             "dtype": "fp16" if w.dtype == "fp16" else w.dtype, "data": "synthetic",
             "config": workload_config(w),
             "roofline": roof, "cpu_baseline": cpu, "e2e": e2e,
-            "gpu_launches": launches_per_step(w) * K,
+            "gpu_launches": launches,
             "clocks": clocks, "wall_s_timed": wall,
             "main_kernel_ms": main_mean,
             "main_kernel_ms_min": min(main_ms),

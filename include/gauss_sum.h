@@ -175,6 +175,13 @@ gs_status gauss_sum_noalloc(const void* q, const void* k, const void* v, double 
  */
 gs_status gauss_sum_probe_ex2_rate(void* stream, double* exp2_per_second);
 
+/*
+ * Accounting helper (not part of Eq. 1): number of CUDA kernels this
+ * library has launched in this process, over all devices and streams,
+ * counted on the host at each launch.  Never fails.
+ */
+uint64_t gauss_sum_kernel_launches(void);
+
 #ifdef __cplusplus
 }
 #endif

@@ -25,7 +25,7 @@ EXPORTS = (
     "gauss_sum_default_options", "gauss_sum", "gauss_sum_ex", "gauss_sum_grad_q",
     "gauss_sum_grad_q_ex", "gauss_sum_workspace_size", "gauss_sum_device_status",
     "gauss_sum_last_error", "gauss_sum_status_string", "gauss_sum_probe_ex2_rate",
-    "gauss_sum_noalloc",
+    "gauss_sum_noalloc", "gauss_sum_kernel_launches",
 )
 
 # Bytes of the static scratch array behind gauss_sum_noalloc
@@ -99,6 +99,8 @@ def _declare(lib):
     lib.gauss_sum_probe_ex2_rate.restype = f
     lib.gauss_sum_noalloc.argtypes = [vp, vp, vp, d, i64, i64, i64, i64, f, vp, vp]
     lib.gauss_sum_noalloc.restype = f
+    lib.gauss_sum_kernel_launches.argtypes = []
+    lib.gauss_sum_kernel_launches.restype = ctypes.c_uint64
 
 
 def _check(lib, status: int):
@@ -242,3 +244,8 @@ def gauss_sum_probe_ex2_rate(stream=None) -> float:
     r = ctypes.c_double(0.0)
     _check(lib, lib.gauss_sum_probe_ex2_rate(_stream_ptr(stream), ctypes.byref(r)))
     return r.value
+
+
+def gauss_sum_kernel_launches() -> int:
+    """Kernels the library has launched in this process (all devices)."""
+    return int(load_library().gauss_sum_kernel_launches())

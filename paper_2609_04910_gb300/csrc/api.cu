@@ -6,6 +6,7 @@
 #include <cstdio>
 #include <cstdlib>
 #include <cstring>
+#include <atomic>
 #include <mutex>
 
 #include "gauss_sum.h"
@@ -15,6 +16,7 @@
 namespace {
 
 thread_local char g_last_error[512] = "no error";
+std::atomic<uint64_t> g_launches{0};
 
 gs_status fail(gs_status st, const char* fmt, const char* detail = nullptr) {
     if (detail)
@@ -344,6 +346,8 @@ gs_status forward_workspace_bytes(const void* q, const void* k, const void* v, d
 
 gs_status set_last_error(gs_status st, const char* msg) { return fail(st, "%s", msg); }
 
+void note_launches(int n) { g_launches.fetch_add(static_cast<uint64_t>(n), std::memory_order_relaxed); }
+
 cudaError_t run_ex2_probe(cudaStream_t s, double* rate) {
     int dev = 0;
     cudaError_t e = cudaGetDevice(&dev);
@@ -361,6 +365,7 @@ cudaError_t run_ex2_probe(cudaStream_t s, double* rate) {
     for (int rep = 0; rep < 4; ++rep) {
         cudaEventRecord(e0, s);
         ex2_probe_kernel<8><<<blocks, threads, 0, s>>>(out, iters);
+        note_launches(1);
         cudaEventRecord(e1, s);
         e = cudaEventSynchronize(e1);
         if (e != cudaSuccess) break;
@@ -469,6 +474,8 @@ const char* gauss_sum_status_string(gs_status s) {
     }
     return "unknown status";
 }
+
+uint64_t gauss_sum_kernel_launches(void) { return g_launches.load(std::memory_order_relaxed); }
 
 gs_status gauss_sum_probe_ex2_rate(void* stream, double* exp2_per_second) {
     if (!exp2_per_second) return fail(GS_ERR_INVALID_ARGUMENT, "null output pointer");

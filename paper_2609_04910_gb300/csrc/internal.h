@@ -108,5 +108,8 @@ gs_status forward_workspace_bytes(const void* q, const void* k, const void* v, d
                                   int64_t M, int64_t N, int64_t D, int64_t C, gs_dtype dtype,
                                   float* out, size_t* bytes);
 gs_status set_last_error(gs_status st, const char* msg);
+// Adds n to the count behind gauss_sum_kernel_launches(); called right
+// after each kernel launch of the library.
+void note_launches(int n);
 
 }  // namespace gs

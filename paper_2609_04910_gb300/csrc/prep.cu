@@ -84,17 +84,36 @@ __global__ void mean_partial_kernel(const T* __restrict__ q, const T* __restrict
 // whenever |x_d - mu_d| stays below 2^(e_x + 1) (x_d in [2^e_x, 2^(e_x+1))),
 // i.e. the shift adds no rounding for points near the mean.  Any common
 // shift leaves the Gauss sum unchanged.
-__global__ void mean_final_kernel(const float* __restrict__ partial, int G, int D, double total,
-                                  int mant_bits, int min_exp, float* __restrict__ mu) {
-    const int d = blockIdx.x * blockDim.x + threadIdx.x;
-    if (d >= D) return;
+constexpr int kMeanFinalThreads = 256;
+
+__global__ void __launch_bounds__(kMeanFinalThreads)
+mean_final_kernel(const float* __restrict__ partial, int G, int D, double total, int mant_bits,
+                  int min_exp, float* __restrict__ mu) {
+    // Block d: thread t folds partials t, t + 256, ... in order, then a
+    // fixed tree combines the threads (deterministic).
+    __shared__ double red_s[kMeanFinalThreads];
+    __shared__ float red_m[kMeanFinalThreads];
+    const int d = blockIdx.x;
+    const int t = threadIdx.x;
     double s = 0.0;
     float mx = 0.f;
-    for (int g = 0; g < G; ++g) {
+    for (int g = t; g < G; g += kMeanFinalThreads) {
         s += static_cast<double>(partial[static_cast<int64_t>(g) * D + d]);
         mx = fmaxf(mx, partial[static_cast<int64_t>(G + g) * D + d]);
     }
-    double m = s / total;
+    red_s[t] = s;
+    red_m[t] = mx;
+    __syncthreads();
+    for (int w = kMeanFinalThreads / 2; w > 0; w >>= 1) {
+        if (t < w) {
+            red_s[t] += red_s[t + w];
+            red_m[t] = fmaxf(red_m[t], red_m[t + w]);
+        }
+        __syncthreads();
+    }
+    if (t != 0) return;
+    double m = red_s[0] / total;
+    mx = red_m[0];
     if (mx > 0.f) {
         int e;
         frexp(static_cast<double>(mx), &e);              // mx in [2^(e-1), 2^e)
@@ -104,36 +123,145 @@ __global__ void mean_final_kernel(const float* __restrict__ partial, int G, int 
     mu[d] = static_cast<float>(m);
 }
 
-// ---------------------------------------------------------------- centre / cast / norm
-// One warp per row.  Rows in [rows, rows_pad) become zero rows with norm
-// term `pad_value` (-inf for padded keys, so their kernel value is 0).
-template <typename T, typename H>
-__global__ void center_cast_norm_kernel(const T* __restrict__ x, int64_t rows, int64_t rows_pad,
-                                        int D, int Dp, const float* __restrict__ mu,
-                                        float half_c, H* __restrict__ xh,
-                                        float* __restrict__ nrm, float pad_value) {
-    const int lane = threadIdx.x & 31;
-    const int64_t row = static_cast<int64_t>(blockIdx.x) * (blockDim.x >> 5) + (threadIdx.x >> 5);
-    if (row >= rows_pad) return;
-    H* out = xh + row * Dp;
-    if (row >= rows) {
-        for (int d = lane; d < Dp; d += 32) out[d] = from_f<H>(0.f);
-        if (lane == 0) nrm[row] = pad_value;
-        return;
+// ---------------------------------------------------------------- MMA operands
+// Both operand layouts are written by one kernel that stages kRowsPerBlock
+// rows through shared memory: the block's input rows are one contiguous
+// run of rows x D elements (16-byte vector loads), and its output rows one
+// contiguous run of rows x Dp elements (16-byte vector stores).  One warp
+// per row inside the block.
+//
+// Plain layout (AUG = false): centred points rounded to the MMA type,
+// x^ = rn(x - mu), zero padded to Dp columns, and the scaled squared norm
+// nrm = -(c/2)||x^||^2 (c = tau log2 e) taken from the ROUNDED point, so that
+// c q^.k^ + A_m + B_n is exactly -(c/2)||q^_m - k^_n||^2 up to fp32
+// rounding (the norm factors of Alg. 1 folded into one exponent).  Rows in
+// [rows, rows_pad) become zero rows with norm `pad_value` (-inf for padded
+// keys, so their kernel value is 0).
+//
+// Augmented layout (AUG = true): x^ followed by 2 NT columns that make the
+// MMA produce the whole exponent up to the factor c:
+//   query rows  [q^, F, 1, .., 1, a_0, a_1, .., a_NT-1, 0 ...]
+//   key rows    [k^, b_0, b_1, .., b_NT-1, F, 1, .., 1, 0 ...]
+// with a = -||q^||^2 / 2 and b = -||k^||^2 / 2 taken from the rounded
+// points in fp32 and written as F t_0 + t_1 + ... + t_NT-1, each t_i a
+// rounded remainder, so that
+//   q^_aug . k^_aug = q^.k^ + a + b = -||q^ - k^||^2 / 2
+// up to the split error (|a| 2^-22 for two fp16 terms, |a| 2^-24 for three
+// bf16 terms) and the fp32 accumulation; the kernel value is 2^(c S).  The
+// power of two F (1024 for fp16) keeps norms up to 6.7e7 inside the fp16
+// range.  Padded key rows get b_0 = -30000 / F (their values are zero as
+// well); padded query rows are zero.  `out_q` and/or `out_k` may be given
+// (both for q = k).
+constexpr int kRowsPerBlock = 32;
+constexpr int kOperandThreads = 128;
+constexpr int kOperandMaxCols = 256;
+
+template <typename T, bool AUG>
+__global__ void __launch_bounds__(kOperandThreads)
+operand_kernel(const T* __restrict__ x, int64_t rows, int D, int Dp, int nt, float F,
+               const float* __restrict__ mu, float half_c, float pad_value,
+               T* __restrict__ out_q, T* __restrict__ out_k, float* __restrict__ nrm) {
+    constexpr int R = kRowsPerBlock;
+    __shared__ __align__(16) T s_in[R * kOperandMaxCols];
+    __shared__ __align__(16) T s_out[R * kOperandMaxCols];   // AUG: q rows, then k rows
+    __shared__ float s_mu[kOperandMaxCols];
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int64_t r0 = static_cast<int64_t>(blockIdx.x) * R;
+    for (int d = tid; d < D; d += kOperandThreads) s_mu[d] = mu ? mu[d] : 0.f;
+    const int64_t left = rows - r0;
+    const int rin = left <= 0 ? 0 : left >= R ? R : static_cast<int>(left);
+    {
+        // r0 D sizeof(T) is a multiple of 16 (R = 32) and x is 16-byte aligned.
+        const int n_el = rin * D;
+        constexpr int PER_VEC = 16 / static_cast<int>(sizeof(T));
+        const int nvec = n_el / PER_VEC;
+        const T* src = x + r0 * D;
+        for (int i = tid; i < nvec; i += kOperandThreads)
+            reinterpret_cast<uint4*>(s_in)[i] = reinterpret_cast<const uint4*>(src)[i];
+        for (int i = nvec * PER_VEC + tid; i < n_el; i += kOperandThreads) s_in[i] = src[i];
     }
-    const T* in = x + row * D;
-    float acc = 0.f;
-    for (int d = lane; d < Dp; d += 32) {
-        float val = 0.f;
-        if (d < D) val = to_f(in[d]) - (mu ? mu[d] : 0.f);
-        const H h = from_f<H>(val);
-        out[d] = h;
-        const float hf = to_f(h);
-        acc = fmaf(hf, hf, acc);
-    }
+    __syncthreads();
+    const bool wq = AUG ? out_q != nullptr : true;
+    const bool wk = AUG && out_k != nullptr;
+    T* sq = s_out;
+    T* sk = s_out + (wq ? R * Dp : 0);
+    const T zero = from_f<T>(0.f);
+    for (int row = warp; row < R; row += kOperandThreads / 32) {
+        const bool valid = row < rin;
+        T* oq = sq + row * Dp;
+        T* ok = sk + row * Dp;
+        float acc = 0.f;
+        const int dend = AUG ? D : Dp;
+        for (int d = lane; d < dend; d += 32) {
+            const float val = (valid && d < D) ? to_f(s_in[row * D + d]) - s_mu[d] : 0.f;
+            const T h = from_f<T>(val);
+            if (wq) oq[d] = h;
+            if (wk) ok[d] = h;
+            const float hf = to_f(h);
+            acc = fmaf(hf, hf, acc);
+        }
 #pragma unroll
-    for (int o = 16; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
-    if (lane == 0) nrm[row] = -half_c * acc;
+        for (int o = 16; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
+        if (!AUG) {
+            if (lane == 0) nrm[r0 + row] = valid ? -half_c * acc : pad_value;
+            continue;
+        }
+        for (int d = D + 2 * nt + lane; d < Dp; d += 32) {
+            if (wq) oq[d] = zero;
+            if (wk) ok[d] = zero;
+        }
+        if (lane < nt) {
+            // Lane i writes term i of the split and its partner column.
+            T t = zero, one = zero;
+            if (valid) {
+                float r = -0.5f * acc;
+                t = from_f<T>(r / F);
+                r -= F * to_f(t);
+                for (int i = 1; i <= lane; ++i) {
+                    t = from_f<T>(r);
+                    r -= to_f(t);
+                }
+                one = from_f<T>(lane == 0 ? F : 1.f);
+            } else if (lane == 0) {
+                t = from_f<T>(-30000.f / F);
+            }
+            if (wq) {
+                oq[D + lane] = valid ? one : zero;
+                oq[D + nt + lane] = valid ? t : zero;
+            }
+            if (wk) {
+                ok[D + lane] = t;
+                ok[D + nt + lane] = one;
+            }
+        }
+    }
+    __syncthreads();
+    // r0 Dp sizeof(T) is a multiple of 16 (Dp is a multiple of 16).
+    const int nvec = R * Dp * static_cast<int>(sizeof(T)) / 16;
+    if (wq) {
+        uint4* dst = reinterpret_cast<uint4*>(out_q + r0 * Dp);
+        for (int i = tid; i < nvec; i += kOperandThreads) dst[i] = reinterpret_cast<const uint4*>(sq)[i];
+    }
+    if (wk) {
+        uint4* dst = reinterpret_cast<uint4*>(out_k + r0 * Dp);
+        for (int i = tid; i < nvec; i += kOperandThreads) dst[i] = reinterpret_cast<const uint4*>(sk)[i];
+    }
+}
+
+template <typename T, bool AUG>
+cudaError_t operand_typed(const void* x, int64_t rows, int64_t rows_pad, int D, int Dp, int nt,
+                          float F, const float* mu, float half_c, float pad_value, void* out_q,
+                          void* out_k, float* nrm, cudaStream_t s) {
+    if (rows_pad % kRowsPerBlock != 0 || Dp % 16 != 0 || Dp > kOperandMaxCols ||
+        (AUG && 2 * Dp > kOperandMaxCols))
+        return cudaErrorInvalidValue;
+    const int64_t blocks = rows_pad / kRowsPerBlock;
+    if (blocks == 0) return cudaSuccess;
+    operand_kernel<T, AUG><<<static_cast<unsigned>(blocks), kOperandThreads, 0, s>>>(
+        static_cast<const T*>(x), rows, D, Dp, nt, F, mu, half_c, pad_value,
+        static_cast<T*>(out_q), static_cast<T*>(out_k), nrm);
+    note_launches(1);
+    return cudaGetLastError();
 }
 
 // ---------------------------------------------------------------- values
@@ -247,87 +375,6 @@ __global__ void key_record_kernel(const T* __restrict__ v, const float* __restri
     }
 }
 
-// ---------------------------------------------------------------- augmented operands
-// Centred points rounded to the MMA type, x^ = rn(x - mu) (as for the
-// plain operands, so that fp16/bf16 inputs near the mean stay exact),
-// followed by 2 NT columns that make the MMA produce the whole exponent up
-// to the factor c = tau log2 e:
-//   query rows  [q^, F, 1, .., 1, a_0, a_1, .., a_NT-1, 0 ...]
-//   key rows    [k^, b_0, b_1, .., b_NT-1, F, 1, .., 1, 0 ...]
-// with a = -||q^||^2 / 2 and b = -||k^||^2 / 2 taken from the rounded
-// points in fp32 and written as F t_0 + t_1 + ... + t_NT-1, each t_i a
-// rounded remainder, so that
-//   q^_aug . k^_aug = q^.k^ + a + b = -||q^ - k^||^2 / 2
-// up to the split error (|a| 2^-22 for two fp16 terms, |a| 2^-24 for three
-// bf16 terms) and the fp32 accumulation; the kernel value is 2^(c S).  The
-// power of two F (1024 for fp16) keeps norms up to 6.7e7 inside the fp16
-// range.  Padded key rows get b_0 = -30000 / F (their values are zero as
-// well); padded query rows are zero.  One warp per row; `out_q` and/or
-// `out_k` may be given (both for q = k).
-template <typename T, typename H>
-__global__ void aug_prep_kernel(const T* __restrict__ x, int64_t rows, int64_t rows_pad, int D,
-                                int Dpa, int nt, float F, const float* __restrict__ mu,
-                                H* __restrict__ out_q, H* __restrict__ out_k) {
-    const int lane = threadIdx.x & 31;
-    const int64_t row = static_cast<int64_t>(blockIdx.x) * (blockDim.x >> 5) + (threadIdx.x >> 5);
-    if (row >= rows_pad) return;
-    H* oq = out_q ? out_q + row * Dpa : nullptr;
-    H* ok = out_k ? out_k + row * Dpa : nullptr;
-    const H zero = from_f<H>(0.f);
-    if (row >= rows) {
-        for (int d = lane; d < Dpa; d += 32) {
-            if (oq) oq[d] = zero;
-            if (ok) ok[d] = d == D ? from_f<H>(-30000.f / F) : zero;
-        }
-        return;
-    }
-    const T* in = x + row * D;
-    float acc = 0.f;
-    for (int d = lane; d < D; d += 32) {
-        const H h = from_f<H>(to_f(in[d]) - (mu ? mu[d] : 0.f));
-        if (oq) oq[d] = h;
-        if (ok) ok[d] = h;
-        const float hf = to_f(h);
-        acc = fmaf(hf, hf, acc);
-    }
-    for (int d = D + 2 * nt + lane; d < Dpa; d += 32) {
-        if (oq) oq[d] = zero;
-        if (ok) ok[d] = zero;
-    }
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
-    if (lane < nt) {
-        // Lane i writes term i of the split and its partner column.
-        float r = -0.5f * acc;
-        H t = from_f<H>(r / F);
-        r -= F * to_f(t);
-        for (int i = 1; i <= lane; ++i) {
-            t = from_f<H>(r);
-            r -= to_f(t);
-        }
-        const H one = from_f<H>(lane == 0 ? F : 1.f);
-        if (oq) {
-            oq[D + lane] = one;
-            oq[D + nt + lane] = t;
-        }
-        if (ok) {
-            ok[D + lane] = t;
-            ok[D + nt + lane] = one;
-        }
-    }
-}
-
-template <typename T, typename H>
-cudaError_t aug_typed(const void* x, int64_t rows, int64_t rows_pad, int D, int Dpa, int nt,
-                      float F, const float* mu, void* out_q, void* out_k, cudaStream_t s) {
-    const int warps = 8;
-    const int64_t blocks = (rows_pad + warps - 1) / warps;
-    aug_prep_kernel<T, H><<<static_cast<unsigned>(blocks), warps * 32, 0, s>>>(
-        static_cast<const T*>(x), rows, rows_pad, D, Dpa, nt, F, mu, static_cast<H*>(out_q),
-        static_cast<H*>(out_k));
-    return cudaGetLastError();
-}
-
 // ---------------------------------------------------------------- finalise
 // part: splits blocks of split_stride_rows rows x part_ld floats.
 template <int MODE, typename T>
@@ -362,18 +409,6 @@ __global__ void finalize_kernel(const float* __restrict__ part, int splits,
     }
 }
 
-template <typename T, typename H>
-cudaError_t ccn_typed(const void* x, int64_t rows, int64_t rows_pad, int D, int Dp,
-                      const float* mu, float half_c, void* xh, float* nrm, float pad_value,
-                      cudaStream_t s) {
-    const int warps = 8;
-    const int64_t blocks = (rows_pad + warps - 1) / warps;
-    center_cast_norm_kernel<T, H><<<static_cast<unsigned>(blocks), warps * 32, 0, s>>>(
-        static_cast<const T*>(x), rows, rows_pad, D, Dp, mu, half_c, static_cast<H*>(xh), nrm,
-        pad_value);
-    return cudaGetLastError();
-}
-
 template <typename T, bool GRAD>
 cudaError_t value_prep_typed(const void* v, const void* k, const float* mu, int64_t N,
                              int64_t Npad, int D, int Cv, int Cp, unsigned* vmax_bits, void* vt,
@@ -386,6 +421,7 @@ cudaError_t value_prep_typed(const void* v, const void* k, const float* mu, int6
         value_max_kernel<T, GRAD><<<static_cast<unsigned>(blocks), dim3(32, 8), 0, s>>>(
             static_cast<const T*>(v), static_cast<const T*>(k), mu, N, D, Cv, rows_per_block,
             vmax_bits);
+        note_launches(1);
         e = cudaGetLastError();
         if (e != cudaSuccess) return e;
     }
@@ -393,6 +429,7 @@ cudaError_t value_prep_typed(const void* v, const void* k, const float* mu, int6
     value_prep_kernel<T, GRAD><<<grid, dim3(32, 8), 0, s>>>(
         static_cast<const T*>(v), static_cast<const T*>(k), mu, N, Npad, D, Cv, Cp, vmax_bits,
         static_cast<__half*>(vt), inv_scale);
+    note_launches(1);
     return cudaGetLastError();
 }
 
@@ -408,6 +445,7 @@ cudaError_t finalize_typed(const float* part, int splits, int64_t stride_rows, i
     finalize_kernel<MODE, T><<<static_cast<unsigned>(blocks), threads, 0, s>>>(
         part, splits, stride_rows, M, Cv, part_ld, inv_scale, static_cast<const T*>(q), mu, tau,
         D, out, s_out);
+    note_launches(1);
     return cudaGetLastError();
 }
 
@@ -422,22 +460,26 @@ cudaError_t launch_mean(InType t, const void* q, const void* k, int64_t M, int64
         case InType::F16:
             mean_partial_kernel<__half><<<G, dim3(32, 8), 0, s>>>(
                 static_cast<const __half*>(q), static_cast<const __half*>(k), M, N, D, rpb, partial);
+            note_launches(1);
             break;
         case InType::BF16:
             mean_partial_kernel<__nv_bfloat16><<<G, dim3(32, 8), 0, s>>>(
                 static_cast<const __nv_bfloat16*>(q), static_cast<const __nv_bfloat16*>(k), M, N,
                 D, rpb, partial);
+            note_launches(1);
             break;
         default:
             mean_partial_kernel<float><<<G, dim3(32, 8), 0, s>>>(
                 static_cast<const float*>(q), static_cast<const float*>(k), M, N, D, rpb, partial);
+            note_launches(1);
     }
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
     const int mant_bits = t == InType::F16 ? 10 : t == InType::BF16 ? 7 : 23;
     const int min_exp = t == InType::F16 ? -24 : t == InType::BF16 ? -133 : -149;
-    mean_final_kernel<<<(D + 127) / 128, 128, 0, s>>>(partial, G, D, static_cast<double>(total),
-                                                      mant_bits, min_exp, mu);
+    mean_final_kernel<<<D, kMeanFinalThreads, 0, s>>>(partial, G, D, static_cast<double>(total),
+                                                     mant_bits, min_exp, mu);
+    note_launches(1);
     return cudaGetLastError();
 }
 
@@ -445,9 +487,10 @@ cudaError_t launch_center_cast_norm(InType t, const void* x, int64_t rows, int64
                                     int D, int Dp, const float* mu, float half_c, void* xh,
                                     float* nrm, float pad_value, cudaStream_t s) {
     if (t == InType::BF16)
-        return ccn_typed<__nv_bfloat16, __nv_bfloat16>(x, rows, rows_pad, D, Dp, mu, half_c, xh,
-                                                       nrm, pad_value, s);
-    return ccn_typed<__half, __half>(x, rows, rows_pad, D, Dp, mu, half_c, xh, nrm, pad_value, s);
+        return operand_typed<__nv_bfloat16, false>(x, rows, rows_pad, D, Dp, 0, 1.f, mu, half_c,
+                                                   pad_value, xh, nullptr, nrm, s);
+    return operand_typed<__half, false>(x, rows, rows_pad, D, Dp, 0, 1.f, mu, half_c, pad_value,
+                                        xh, nullptr, nrm, s);
 }
 
 cudaError_t launch_value_prep(InType t, bool grad, const void* v, const void* k,
@@ -469,9 +512,10 @@ cudaError_t launch_aug_prep(InType t, const void* x, int64_t rows, int64_t rows_
                             int Dpa, const float* mu, void* out_q, void* out_k, cudaStream_t s) {
     const int nt = aug_norm_terms(t);
     if (t == InType::BF16)
-        return aug_typed<__nv_bfloat16, __nv_bfloat16>(x, rows, rows_pad, D, Dpa, nt, 1.f, mu,
-                                                       out_q, out_k, s);
-    return aug_typed<__half, __half>(x, rows, rows_pad, D, Dpa, nt, 1024.f, mu, out_q, out_k, s);
+        return operand_typed<__nv_bfloat16, true>(x, rows, rows_pad, D, Dpa, nt, 1.f, mu, 0.f, 0.f,
+                                                  out_q, out_k, nullptr, s);
+    return operand_typed<__half, true>(x, rows, rows_pad, D, Dpa, nt, 1024.f, mu, 0.f, 0.f, out_q,
+                                       out_k, nullptr, s);
 }
 
 cudaError_t launch_key_records(InType t, const void* v, const float* B, int64_t N, int64_t Npad,
@@ -486,6 +530,7 @@ cudaError_t launch_key_records(InType t, const void* v, const float* B, int64_t 
     else
         key_record_kernel<__half><<<blocks, threads, 0, s>>>(static_cast<const __half*>(v), B, N,
                                                              pairs, C, rec);
+    note_launches(1);
     return cudaGetLastError();
 }
 

@@ -114,6 +114,7 @@ cudaError_t launch_dmax(const SimtPlan& p, const float* q, const float* k, const
     simt_gauss_kernel<DMAX, CBLK, GRAD><<<grid, THREADS, 0, s>>>(
         q, k, v, p.M, p.N, static_cast<int>(p.D), static_cast<int>(p.Cv), half_c,
         p.keys_per_split, part);
+    note_launches(1);
     return cudaGetLastError();
 }
 

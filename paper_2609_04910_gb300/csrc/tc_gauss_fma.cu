@@ -457,6 +457,7 @@ cudaError_t launch_typed(const TcPlan& pl, InType t, float c, char* ws, unsigned
     if (e != cudaSuccess) return e;
     dim3 grid(static_cast<unsigned>(pl.Mpad / (NQ * BM)), static_cast<unsigned>(pl.splits));
     tc_gauss_fma_kernel<C, QS><<<grid, THREADS, pl.smem_bytes, s>>>(tm_q, tm_k, p);
+    note_launches(1);
     return cudaGetLastError();
 }
 

@@ -28,10 +28,18 @@ def _declared_functions():
 def test_every_declared_symbol_is_exported(lib):
     from paper_2609_04910_gb300._binding import EXPORTS
     declared = _declared_functions()
-    assert len(declared) == 11
+    assert len(declared) == 12
     assert sorted(EXPORTS) == declared
     for name in declared:
         assert hasattr(lib, name), name
+
+
+def test_launch_counter_starts_without_gpu_work(lib):
+    # Argument errors return before any launch, so the count does not move.
+    n0 = lib.gauss_sum_kernel_launches()
+    st = lib.gauss_sum(None, None, None, 1.0, 1, 1, 1, 1, 1, None, None)
+    assert st == 1
+    assert lib.gauss_sum_kernel_launches() == n0
 
 
 def test_status_strings(lib):
