@@ -64,7 +64,7 @@ typedef enum { GS_PATH_AUTO = 0, GS_PATH_TENSOR = 1, GS_PATH_SIMT = 2 } gs_path;
  * Options of the _ex entry points.  Initialise with gauss_sum_default_options.
  *  center          1: shift q and k by their common mean before rounding to
  *                     the MMA type (the overflow/cancellation safeguard of
- *                     Remark 3, Sec. 2); 0: use the raw points.
+ *                     Remark 2, Sec. 2); 0: use the raw points.
  *  split_n         number of key splits per row tile (0: chosen from the
  *                  SM count); partial sums over splits are added in a fixed
  *                  order, so results are deterministic for a fixed split.

@@ -1,7 +1,7 @@
 // Preparation and finalisation kernels of the Gauss-sum path.
 //
 //  * common mean of all query and key points (the shift safeguard of
-//    Remark 3, Sec. 2: the kernel depends on q - k only, so any common shift
+//    Remark 2, Sec. 2: the kernel depends on q - k only, so any common shift
 //    is exact and only changes rounding), rounded to the input format's
 //    grid so that the shift itself adds no rounding near the mean;
 //  * centring, rounding to the MMA operand type and the scaled squared norms
