@@ -6,35 +6,43 @@
 // Phi(q_m, k_n) = 2^(c S + A_m + B_n) (the exponent is <= 0, so no running
 // maximum is needed; see tc_gauss.cu) and accumulate sum_n Phi v_n in fp32
 // on the FMA pipe.  With augmented operands (prep.cu) the MMA already adds
-// the norm terms, S = -||q^ - k^||^2 / 2, and Phi = 2^(c S).  For C <= 4 this costs fewer issue slots than a second
-// MMA with N = 16, and it keeps kernel values and values in fp32.
+// the norm terms, S = -||q^ - k^||^2 / 2, and Phi = 2^(c S).  For C <= 4
+// this costs fewer issue slots than a second MMA with N = 16, and it keeps
+// kernel values and values in fp32.
 //
 // Layout choices:
 //   * A CTA owns two query tiles (256 rows), which halves the L2 -> shared
 //     memory traffic of the key tiles; every exponent warp handles the same
 //     key columns of both query tiles, so one broadcast load of a key
 //     record serves two kernel values.
-//   * Barrier handshakes cost the single MMA-issuing thread one to two
-//     hundred cycles each, so there is one handshake per key tile: the MMA
-//     thread issues the 2 x (Dp / 16) MMAs of a key tile back to back and
-//     commits once; the exponent warps release both S buffers of the key
-//     tile with one arrival per warp, as soon as they are in registers.
+//   * One barrier handshake per key tile: the 2 x (Dp / 16) MMAs of a key
+//     tile are issued back to back and committed once; the exponent warps
+//     release both S buffers of the key tile with one arrival per warp, as
+//     soon as they are in registers, and query the next key tile's
+//     barriers before exponentiating the current one.
 //   * TMEM holds SL slots of two 128-column S buffers (one per query
 //     tile); key tile j uses slot j % SL, so the MMAs of key tile j only
 //     wait for the release of key tile j - SL.  With Dp <= 128 the query
 //     tiles q^ stay in shared memory (A operand read by the MMA from shared
 //     memory) and SL = 2; with larger Dp they would not fit next to the key
 //     stages, so q^ is copied into TMEM (A operand from TMEM) and SL = 1.
+//   * The kernel is bound by instruction dispatch next to the MUFU pipe,
+//     and TMEM lane quarters tie every row to one SMSP, so each SMSP must
+//     carry the same extra work: the MMA issue and key loads are split over
+//     one control warp per SMSP (round robin over key tiles) rather than
+//     given to one MMA warp, whose SMSP would otherwise pace all others.
 //
-// Warp roles (18 warps):
-//   warps 0-15  exponent warps.  Warp w reads TMEM lanes 32 (w % 4) .. +31
-//               (rows of both query tiles) and key columns 32 (w / 4) .. +31
-//               of the two S buffers of each key tile.
-//   warp 16     TMA producer: the q^ tiles (shared-memory variant), then per
-//               key tile the k^ rows and the key records.
-//   warp 17     TMEM allocator and single-thread MMA issuer.
+// Warp roles (20 warps):
+//   warps 0-15   exponent warps.  Warp w reads TMEM lanes 32 (w % 4) .. +31
+//                (rows of both query tiles) and key columns 32 (w / 4) .. +31
+//                of the two S buffers of each key tile.
+//   warps 16-19  control warps, one per SMSP.  Control warp k owns shared-
+//                memory stage k and key tiles j = k (mod stages): it loads
+//                their k^ rows and key records (TMA) and issues and commits
+//                their MMAs.  Warp 16 also allocates TMEM and loads q^.
 // Key records: for each pair of keys (2t, 2t + 1) the floats
-//   B_2t, B_2t+1, v_2t[0], v_2t+1[0], ..., v_2t[C-1], v_2t+1[C-1].
+//   [B_2t, B_2t+1,] v_2t[0], v_2t+1[0], ..., v_2t[C-1], v_2t+1[C-1]
+// (B only without augmented operands).
 #include <cuda.h>
 #include <cuda_runtime.h>
 
@@ -52,13 +60,15 @@ constexpr int NQ = 2;              // query tiles per CTA
 constexpr int BN = 128;            // keys per key tile (MMA N)
 constexpr int KB = 64;             // 16-bit elements per 128-byte swizzled row
 constexpr int NEXP = 16;
-constexpr int PRODUCER_WARP = 16;
-constexpr int MMA_WARP = 17;
-constexpr int THREADS = 18 * 32;
+constexpr int CTRL_WARP0 = 16;     // control warps 16..19, one per SMSP
+constexpr int NCTRL_MAX = 4;
+constexpr int THREADS = (NEXP + NCTRL_MAX) * 32;
 constexpr int NPART = 4;           // column groups (partial sums) per row
 constexpr int MAX_SL = 2;          // TMEM slots of two S buffers
 constexpr uint32_t TMEM_COLS = 512;
-constexpr int MAX_STAGES = 8;
+constexpr int MAX_STAGES = NCTRL_MAX;   // one stage per control warp
+// Augmented operands keep q^ in shared memory (two TMEM slots of S).
+constexpr bool kAugQsm = true;
 
 struct FmaParams {
     const uint32_t* qh;  // Mpad x Dp/2 packed 16-bit pairs (centred, rounded q)
@@ -102,18 +112,19 @@ __device__ __forceinline__ void exp_warps_sync() {
     asm volatile("bar.sync 1, %0;" ::"r"(NEXP * 32) : "memory");
 }
 
-// QS: q^ tiles in shared memory (A operand from shared memory, SL = 2);
-// otherwise q^ in TMEM (A operand from TMEM, SL = 1).
-template <int C, bool QS>
+// AUG: augmented operands (S = -||q^ - k^||^2 / 2; no norm terms in the
+// key records).  QSM: q^ tiles in shared memory (A operand from shared
+// memory, SL = 2); otherwise q^ in TMEM (A operand from TMEM, SL = 1).
+template <int C, bool AUG, bool QSM>
 __global__ void __launch_bounds__(THREADS, 1)
 tc_gauss_fma_kernel(const __grid_constant__ CUtensorMap tm_q,
                     const __grid_constant__ CUtensorMap tm_k, const FmaParams p) {
-    constexpr int REC_PAIR = (QS ? 0 : 2) + 2 * C;    // floats per key pair
-    constexpr int SL = QS ? 2 : 1;
+    constexpr int REC_PAIR = (AUG ? 0 : 2) + 2 * C;   // floats per key pair
+    constexpr int SL = QSM ? 2 : 1;
     extern __shared__ uint8_t smem_raw[];
     const uint32_t raw_addr = smem_u32(smem_raw);
     uint8_t* smem = smem_raw + (((raw_addr + 1023u) & ~1023u) - raw_addr);
-    uint8_t* q_smem = smem;                            // QS: NQ x nkb x 16 KB
+    uint8_t* q_smem = smem;                            // QSM: NQ x nkb x 16 KB
     uint8_t* stage0 = smem + p.q_bytes;
     float* red = reinterpret_cast<float*>(smem + p.red_offset);    // NPART x 256 x C
     FmaBarriers* bars = reinterpret_cast<FmaBarriers*>(smem + p.red_offset + NPART * NQ * BM * C * 4);
@@ -128,8 +139,9 @@ tc_gauss_fma_kernel(const __grid_constant__ CUtensorMap tm_q,
     volatile int* abort_flag = &bars->abort_flag;
 
     if (tid == 0) {
-        mbar_init(&bars->qa_ready, QS ? 1 : NEXP);
-        mbar_init(&bars->drain, 1);
+        mbar_init(&bars->qa_ready, QSM ? 1 : NEXP);
+        // One drain commit per control warp that has key tiles.
+        mbar_init(&bars->drain, max(1, min(T, p.stages)));
         for (int sl = 0; sl < SL; ++sl) {
             mbar_init(&bars->s_full[sl], 1);
             mbar_init(&bars->s_free[sl], NEXP);        // one arrival per exponent warp
@@ -141,7 +153,7 @@ tc_gauss_fma_kernel(const __grid_constant__ CUtensorMap tm_q,
         bars->abort_flag = 0;
         fence_mbar_init();
     }
-    if (warp == MMA_WARP) {
+    if (warp == CTRL_WARP0) {
         tmem_alloc(&bars->tmem_base, TMEM_COLS);
         tmem_relinquish();
     }
@@ -149,21 +161,37 @@ tc_gauss_fma_kernel(const __grid_constant__ CUtensorMap tm_q,
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = bars->tmem_base;
-    const uint32_t qa_col = static_cast<uint32_t>(2 * SL * BN);   // TMEM q^ (not QS)
+    const uint32_t qa_col = static_cast<uint32_t>(2 * SL * BN);   // TMEM q^ (not QSM)
 
     auto kh_smem = [&](int s) { return stage0 + s * p.stage_bytes; };
     auto rec_smem = [&](int s) {
         return reinterpret_cast<const float*>(stage0 + s * p.stage_bytes + p.kh_bytes);
     };
 
-    if (warp == PRODUCER_WARP) {
-        // The whole warp runs the loop (warp-uniform operands); the elected
-        // lane issues the copies.
-        if (T > 0) {
+    if (warp >= CTRL_WARP0) {
+        // ------------------------------------------------ control warps
+        // Control warp k (on SMSP k) owns shared-memory stage k and key
+        // tiles j = k, k + nctrl, ...: it loads their keys and records and
+        // issues their MMAs, so that the MMA issue work is spread over the
+        // SMSPs instead of slowing the exponent warps of one of them.  The
+        // whole warp runs the loop (warp-uniform operands); the elected lane
+        // issues copies, MMAs and commits.
+        const int k = warp - CTRL_WARP0;
+        const int nctrl = p.stages;
+        if (k < nctrl && k < T) {
             const bool leader = elect_one();
+            auto load_keys = [&](int j) {
+                mbar_arrive_expect_tx(&bars->kv_full[k], p.kh_bytes + p.rec_bytes);
+                const int n0 = (kt0 + j) * BN;
+                for (int kb = 0; kb < p.nkb; ++kb)
+                    tma_load_2d(kh_smem(k) + kb * (BN * 128), &tm_k, &bars->kv_full[k], kb * KB, n0);
+                bulk_load(const_cast<float*>(rec_smem(k)),
+                          p.rec + static_cast<int64_t>(n0 / 2) * REC_PAIR, p.rec_bytes,
+                          &bars->kv_full[k]);
+            };
             if (leader) {
                 tma_prefetch_desc(&tm_k);
-                if (QS) {
+                if (QSM && k == 0) {
                     tma_prefetch_desc(&tm_q);
                     mbar_arrive_expect_tx(&bars->qa_ready, p.q_bytes);
                     for (int h = 0; h < NQ; ++h)
@@ -171,84 +199,74 @@ tc_gauss_fma_kernel(const __grid_constant__ CUtensorMap tm_q,
                             tma_load_2d(q_smem + (h * p.nkb + kb) * (BM * 128), &tm_q, &bars->qa_ready,
                                         kb * KB, (tile_m * NQ + h) * BM);
                 }
+                load_keys(k);
             }
             __syncwarp();
-            int issued = 0;
-            RingPos st;
-            for (int j = 0; j < T; ++j, st.advance(p.stages)) {
-                const int s = st.idx;
-                if (!warp_wait(&bars->kv_empty[s], st.phase ^ 1u, abort_flag, p.status)) break;
-                if (leader) {
-                    mbar_arrive_expect_tx(&bars->kv_full[s], p.kh_bytes + p.rec_bytes);
-                    const int n0 = (kt0 + j) * BN;
-                    for (int kb = 0; kb < p.nkb; ++kb)
-                        tma_load_2d(kh_smem(s) + kb * (BN * 128), &tm_k, &bars->kv_full[s], kb * KB, n0);
-                    bulk_load(const_cast<float*>(rec_smem(s)),
-                              p.rec + static_cast<int64_t>(n0 / 2) * REC_PAIR, p.rec_bytes,
-                              &bars->kv_full[s]);
-                }
-                __syncwarp();
-                issued = j + 1;
-            }
-            // Every copy this CTA started must land before it exits.
-            if (QS) mbar_wait_bounded(&bars->qa_ready, 0, nullptr, p.status);
-            for (int j = max(0, issued - p.stages); j < issued; ++j)
-                mbar_wait_bounded(&bars->kv_full[j % p.stages],
-                                  static_cast<uint32_t>(j / p.stages) & 1u, nullptr, p.status);
-        }
-    } else if (warp == MMA_WARP) {
-        // The whole warp runs the loop (warp-uniform descriptors and TMEM
-        // addresses); the elected lane issues the MMAs and commits.
-        if (T > 0) {
-            const bool leader = elect_one();
             bool ok = warp_wait(&bars->qa_ready, 0, abort_flag, p.status);
             const int ksteps = p.Dp / 16;
-            // Shared-memory descriptors of k^ stage 0 and of q^ tile 0; stage
-            // s, query tile h and K step kk add byte offsets / 16 to the
-            // start-address field.
-            const uint64_t kdesc0 = smem_desc_kmajor_sw128(smem_u32(stage0));
+            // Shared-memory descriptors of stage k and of q^ tile 0; query
+            // tile h and K step kk add byte offsets / 16 to the start-address
+            // field.
+            const uint64_t kdesc = smem_desc_kmajor_sw128(smem_u32(kh_smem(k)));
             const uint64_t qdesc0 = smem_desc_kmajor_sw128(smem_u32(q_smem));
             const uint32_t qdesc_h = static_cast<uint32_t>((p.nkb * BM * 128) >> 4);
             const uint32_t a0 = tmem + qa_col, a1 = a0 + (p.Dp / 2);
-            RingPos st, sl;
-            for (int j = 0; ok && j < T; ++j, st.advance(p.stages), sl.advance(SL)) {
-                const int s = st.idx;
-                // Key tile j - SL released its slot and stage s is loaded;
-                // both queried at once.
-                const uint32_t free_parity = sl.phase ^ 1u;
+            bool pending = true;          // keys of tile j requested, not yet waited for
+            uint32_t ph = 0;              // parity of this warp's stage barriers for tile j
+            int j = k;
+            for (; ok && j < T; j += nctrl, ph ^= 1u) {
+                // S slot of tile j and the parities of its barriers: s_full
+                // completes once per tile of the slot, and tile j reuses the
+                // slot that tile j - SL released.
+                const int sl = SL == 2 ? (j & 1) : 0;
+                const uint32_t full_parity = static_cast<uint32_t>(SL == 2 ? (j >> 1) : j) & 1u;
+                const uint32_t free_parity = full_parity ^ 1u;
                 const bool ready = __all_sync(
-                    0xffffffffu, j < SL ? mbar_test_wait(&bars->kv_full[s], st.phase)
-                                        : mbar_test_wait2(&bars->s_free[sl.idx], free_parity,
-                                                          &bars->kv_full[s], st.phase));
+                    0xffffffffu, j < SL ? mbar_test_wait(&bars->kv_full[k], ph)
+                                        : mbar_test_wait2(&bars->s_free[sl], free_parity,
+                                                          &bars->kv_full[k], ph));
                 if (!ready) {
                     if (j >= SL) {
-                        ok = warp_wait(&bars->s_free[sl.idx], free_parity, abort_flag, p.status);
+                        ok = warp_wait(&bars->s_free[sl], free_parity, abort_flag, p.status);
                         if (!ok) break;
                     }
-                    ok = warp_wait(&bars->kv_full[s], st.phase, abort_flag, p.status);
+                    ok = warp_wait(&bars->kv_full[k], ph, abort_flag, p.status);
                     if (!ok) break;
                 }
+                pending = false;
                 tc_fence_after();
-                const uint32_t d0 = tmem + sl.idx * (2 * BN), d1 = d0 + BN;
-                const uint64_t kdesc = kdesc0 + ((static_cast<uint64_t>(s) * p.stage_bytes) >> 4);
+                const uint32_t d0 = tmem + sl * (2 * BN), d1 = d0 + BN;
                 if (leader) {
-                for (int h = 0; h < NQ; ++h) {
-                    for (int kk = 0; kk < ksteps; ++kk) {
-                        const uint32_t koff = static_cast<uint32_t>((kk >> 2) * (BN * 128 / 16) + (kk & 3) * 2);
-                        if (QS) {
-                            const uint32_t qoff = h * qdesc_h + static_cast<uint32_t>((kk >> 2) * (BM * 128 / 16) + (kk & 3) * 2);
-                            mma_ss_f16(h ? d1 : d0, qdesc0 + qoff, kdesc + koff, p.idesc, kk > 0 ? 1u : 0u);
-                        } else {
-                            mma_ts_f16(h ? d1 : d0, (h ? a1 : a0) + kk * 8, kdesc + koff, p.idesc,
-                                       kk > 0 ? 1u : 0u);
+                    for (int h = 0; h < NQ; ++h) {
+                        for (int kk = 0; kk < ksteps; ++kk) {
+                            const uint32_t koff = static_cast<uint32_t>((kk >> 2) * (BN * 128 / 16) + (kk & 3) * 2);
+                            if (QSM) {
+                                const uint32_t qoff = h * qdesc_h + static_cast<uint32_t>((kk >> 2) * (BM * 128 / 16) + (kk & 3) * 2);
+                                mma_ss_f16(h ? d1 : d0, qdesc0 + qoff, kdesc + koff, p.idesc, kk > 0 ? 1u : 0u);
+                            } else {
+                                mma_ts_f16(h ? d1 : d0, (h ? a1 : a0) + kk * 8, kdesc + koff, p.idesc,
+                                           kk > 0 ? 1u : 0u);
+                            }
                         }
                     }
-                }
-                mma_commit(&bars->s_full[sl.idx]);
-                mma_commit(&bars->kv_empty[s]);
+                    mma_commit(&bars->s_full[sl]);
+                    mma_commit(&bars->kv_empty[k]);
                 }
                 __syncwarp();
+                if (j + nctrl < T) {
+                    // Stage k is free again once these MMAs and the exponent
+                    // warps are done with tile j.
+                    ok = warp_wait(&bars->kv_empty[k], ph, abort_flag, p.status);
+                    if (!ok) break;
+                    if (leader) load_keys(j + nctrl);
+                    __syncwarp();
+                    pending = true;
+                }
             }
+            // Every copy and MMA this warp started must be complete before
+            // the CTA exits.
+            if (pending) mbar_wait_bounded(&bars->kv_full[k], ph, nullptr, p.status);
+            if (QSM && k == 0) mbar_wait_bounded(&bars->qa_ready, 0, nullptr, p.status);
             if (leader) mma_commit(&bars->drain);
             __syncwarp();
             mbar_wait_bounded(&bars->drain, 0, nullptr, p.status);
@@ -262,7 +280,7 @@ tc_gauss_fma_kernel(const __grid_constant__ CUtensorMap tm_q,
         const int64_t row0 = static_cast<int64_t>(tile_m) * NQ * BM + row_t;
         const int64_t row1 = row0 + BM;
 
-        if (!QS) {
+        if (!QSM) {
             // q^ rows -> TMEM (A operand).  Column group cg copies query tile
             // cg / 2, 8-column chunks ck = cg % 2 (mod 2) of its Dp / 2 columns.
             const int h = cg >> 1;
@@ -280,8 +298,8 @@ tc_gauss_fma_kernel(const __grid_constant__ CUtensorMap tm_q,
         }
 
         // Row terms of the exponent (only without augmented operands).
-        const float am0 = QS ? 0.f : p.A[row0];
-        const float am1 = QS ? 0.f : p.A[row1];
+        const float am0 = AUG ? 0.f : p.A[row0];
+        const float am1 = AUG ? 0.f : p.A[row1];
         const uint64_t a2_0 = f32x2_pack(am0, am0);
         const uint64_t a2_1 = f32x2_pack(am1, am1);
         const uint64_t c2 = f32x2_pack(p.c, p.c);
@@ -289,12 +307,13 @@ tc_gauss_fma_kernel(const __grid_constant__ CUtensorMap tm_q,
 #pragma unroll
         for (int cc = 0; cc < C; ++cc) acc0[cc] = acc1[cc] = 0ull;
         bool ok = true;
-        RingPos st, sl;   // stage and TMEM slot of key tile j
+        bool ready = false;   // both barriers of key tile j already seen complete
+        RingPos st, sl;       // stage and TMEM slot of key tile j
         for (int j = 0; j < T; ++j, st.advance(p.stages), sl.advance(SL)) {
             const int s = st.idx;
             const uint32_t col0 = static_cast<uint32_t>(sl.idx * 2 * BN);
-            if (!__all_sync(0xffffffffu, mbar_test_wait2(&bars->kv_full[s], st.phase,
-                                                         &bars->s_full[sl.idx], sl.phase))) {
+            if (!__all_sync(0xffffffffu, ready || mbar_test_wait2(&bars->kv_full[s], st.phase,
+                                                                  &bars->s_full[sl.idx], sl.phase))) {
                 ok = warp_wait(&bars->kv_full[s], st.phase, abort_flag, p.status);
                 if (ok) ok = warp_wait(&bars->s_full[sl.idx], sl.phase, abort_flag, p.status);
                 if (!ok) break;
@@ -308,8 +327,20 @@ tc_gauss_fma_kernel(const __grid_constant__ CUtensorMap tm_q,
             tc_fence_before();
             __syncwarp();
             if (lane == 0) mbar_arrive(&bars->s_free[sl.idx]);
+            // Query the barriers of key tile j + 1 now and read the answer
+            // after the exponent work of tile j: the query latency overlaps
+            // the arithmetic instead of stalling all exponent warps at once.
+            // A phase seen complete stays complete until this warp releases
+            // that stage and slot.
+            {
+                RingPos st2 = st, sl2 = sl;
+                st2.advance(p.stages);
+                sl2.advance(SL);
+                ready = j + 1 < T && mbar_test_wait2(&bars->kv_full[st2.idx], st2.phase,
+                                                     &bars->s_full[sl2.idx], sl2.phase);
+            }
             const float* rec = rec_smem(s) + (cg * 16) * REC_PAIR;
-            if (QS) {
+            if (AUG) {
                 // Augmented operands: S = -||q^ - k^||^2 / 2, so Phi = 2^(c S).
                 // Keys 32 cg + 2t and + 1, rows row0 (S0) and row1 (S1).
 #pragma unroll
@@ -393,7 +424,7 @@ tc_gauss_fma_kernel(const __grid_constant__ CUtensorMap tm_q,
 
     tc_fence_before();
     __syncthreads();
-    if (warp == MMA_WARP) {
+    if (warp == CTRL_WARP0) {
         tc_fence_after();
         tmem_dealloc(tmem, TMEM_COLS);
     }
@@ -415,12 +446,12 @@ size_t fixed_bytes_for(int C, size_t q_bytes) {
            sizeof(FmaBarriers) + 64;
 }
 
-// q^ tiles in shared memory (augmented variant only).
-size_t q_bytes_for(int Dp, bool aug) {
-    return aug ? static_cast<size_t>(NQ) * ((Dp + KB - 1) / KB) * BM * 128 : 0;
+// Shared-memory bytes of the q^ tiles when they live in shared memory.
+size_t q_bytes_for(int Dp, bool qsm) {
+    return qsm ? static_cast<size_t>(NQ) * ((Dp + KB - 1) / KB) * BM * 128 : 0;
 }
 
-template <int C, bool QS>
+template <int C, bool AUG, bool QSM>
 cudaError_t launch_typed(const TcPlan& pl, InType t, float c, char* ws, unsigned* status,
                          cudaStream_t s, const char** why) {
     const CUtensorMapDataType hdt =
@@ -433,7 +464,7 @@ cudaError_t launch_typed(const TcPlan& pl, InType t, float c, char* ws, unsigned
     }
     FmaParams p;
     p.qh = reinterpret_cast<const uint32_t*>(ws + pl.off_qh);
-    p.A = QS ? nullptr : reinterpret_cast<const float*>(ws + pl.off_A);
+    p.A = AUG ? nullptr : reinterpret_cast<const float*>(ws + pl.off_A);
     p.rec = reinterpret_cast<const float*>(ws + pl.off_rec);
     p.part = reinterpret_cast<float*>(ws + pl.off_part);
     p.status = status;
@@ -443,20 +474,20 @@ cudaError_t launch_typed(const TcPlan& pl, InType t, float c, char* ws, unsigned
     p.Dp = pl.Dp;
     p.nkb = (pl.Dp + KB - 1) / KB;
     p.stages = pl.stages;
-    p.q_bytes = static_cast<uint32_t>(q_bytes_for(pl.Dp, QS));
+    p.q_bytes = static_cast<uint32_t>(q_bytes_for(pl.Dp, QSM));
     p.kh_bytes = static_cast<uint32_t>(p.nkb * BN * 128);
-    p.rec_bytes = static_cast<uint32_t>((BN / 2) * rec_pair_floats(C, QS) * 4);
-    p.stage_bytes = static_cast<uint32_t>(stage_bytes_for(p.nkb, C, QS));
+    p.rec_bytes = static_cast<uint32_t>((BN / 2) * rec_pair_floats(C, AUG) * 4);
+    p.stage_bytes = static_cast<uint32_t>(stage_bytes_for(p.nkb, C, AUG));
     p.red_offset = p.q_bytes + static_cast<uint32_t>(pl.stages * p.stage_bytes);
     p.c = c;
     const uint32_t hb = t == InType::BF16 ? 1u : 0u;
     p.idesc = idesc_f16(BM, BN, hb, hb);
-    cudaError_t e = cudaFuncSetAttribute(tc_gauss_fma_kernel<C, QS>,
+    cudaError_t e = cudaFuncSetAttribute(tc_gauss_fma_kernel<C, AUG, QSM>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          static_cast<int>(pl.smem_bytes));
     if (e != cudaSuccess) return e;
     dim3 grid(static_cast<unsigned>(pl.Mpad / (NQ * BM)), static_cast<unsigned>(pl.splits));
-    tc_gauss_fma_kernel<C, QS><<<grid, THREADS, pl.smem_bytes, s>>>(tm_q, tm_k, p);
+    tc_gauss_fma_kernel<C, AUG, QSM><<<grid, THREADS, pl.smem_bytes, s>>>(tm_q, tm_k, p);
     note_launches(1);
     return cudaGetLastError();
 }
@@ -464,8 +495,8 @@ cudaError_t launch_typed(const TcPlan& pl, InType t, float c, char* ws, unsigned
 template <int C>
 cudaError_t launch_c(const TcPlan& pl, InType t, float c, char* ws, unsigned* status,
                      cudaStream_t s, const char** why) {
-    if (pl.aug) return launch_typed<C, true>(pl, t, c, ws, status, s, why);
-    return launch_typed<C, false>(pl, t, c, ws, status, s, why);
+    if (pl.aug) return launch_typed<C, true, kAugQsm>(pl, t, c, ws, status, s, why);
+    return launch_typed<C, false, false>(pl, t, c, ws, status, s, why);
 }
 
 }  // namespace
@@ -474,13 +505,22 @@ bool plan_fma_kernel(int Dp, int C, bool aug, int* nq, int* stages, size_t* smem
     if (C < 1 || C > kFmaMaxChannels || Dp > 256) return false;
     if (aug && Dp > kAugMaxDp) return false;
     // TMEM: q^ in TMEM needs Dp columns beside one slot of two S buffers.
-    if (!aug && static_cast<int>(TMEM_COLS) - 2 * BN < Dp) return false;
+    const bool qsm = aug && kAugQsm;
+    if (!qsm && static_cast<int>(TMEM_COLS) - 2 * BN < Dp) return false;
     const int nkb = (Dp + KB - 1) / KB;
     const size_t budget = 232448;
     const size_t stage = stage_bytes_for(nkb, C, aug);
-    const size_t fixed = fixed_bytes_for(C, q_bytes_for(Dp, aug));
+    const size_t fixed = fixed_bytes_for(C, q_bytes_for(Dp, qsm));
     if (fixed >= budget) return false;
-    const int st = static_cast<int>(std::min<size_t>(MAX_STAGES, (budget - fixed) / stage));
+    // Control warp k owns stage k (stages = control warps) and checks the
+    // S-slot release of key tile j - SL before the MMAs of tile j.  An
+    // mbarrier parity test is only unambiguous while the barrier is at most
+    // one phase behind the phase it asks about; the warp knows every key
+    // tile up to j - stages is done (its previous stage release), and the
+    // slot's previous phase is tile j - 2 SL, so stages <= 2 SL.
+    const int sl = qsm ? 2 : 1;
+    const int st = static_cast<int>(
+        std::min<size_t>(std::min(MAX_STAGES, 2 * sl), (budget - fixed) / stage));
     if (st < 2) return false;
     *nq = NQ;
     *stages = st;

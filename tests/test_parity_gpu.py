@@ -52,6 +52,14 @@ def test_key_splits(split_n):
     forward_check(case(260, 1500, 64, 3, "fp16"), split_n=split_n)
 
 
+@pytest.mark.parametrize("D,dtype", [(64, "fp16"), (200, "fp16"), (120, "bf16"), (250, "bf16")])
+def test_long_key_range_one_split(D, dtype):
+    # One key split: every CTA walks 64 key tiles, so all control warps
+    # cycle through their stages and S slots many times (q^ in shared
+    # memory for D + 4 <= 128, in TMEM otherwise).
+    forward_check(case(256, 8192, D, 3, dtype), split_n=1)
+
+
 @pytest.mark.parametrize("dtype", ["fp16", "bf16"])
 def test_centering_off(dtype):
     forward_check(case(200, 400, 32, 2, dtype), center=False)
