@@ -34,7 +34,8 @@ gs_status cuda_fail(cudaError_t e, const char* where) {
 
 // Device status word: a kernel that gives up a bounded wait records the
 // reason here; gauss_sum_device_status() reads and clears it.
-__device__ unsigned g_device_status = 0;
+// Device status word and, after a timeout, where the first wait gave up.
+__device__ unsigned g_device_status[8];
 
 constexpr int kMaxDevices = 64;
 std::mutex g_dev_mu;
@@ -252,11 +253,10 @@ gs_status run(Call c) {
         }
         if (e == cudaSuccess) {
             if (tp.fma)
-                e = gs::launch_finalize(0, t, reinterpret_cast<float*>(ws + tp.off_part), tp.splits,
-                                        tp.Mpad, c.M, static_cast<int>(tp.Cv),
-                                        static_cast<int>(tp.Cv), nullptr, nullptr, nullptr,
-                                        static_cast<float>(c.tau), static_cast<int>(c.D), c.out,
-                                        nullptr, c.stream);
+                e = gs::launch_finalize_slots(reinterpret_cast<float*>(ws + tp.off_part), tp.Mpad,
+                                              c.M, static_cast<int>(tp.Cv),
+                                              128 * tp.nq, tp.Npad / tp.BN, tp.unit_len, c.out,
+                                              c.stream);
             else
                 e = gs::launch_finalize(c.grad ? 1 : 0, t,
                                         reinterpret_cast<float*>(ws + tp.off_part), tp.splits,
@@ -450,14 +450,19 @@ gs_status gauss_sum_device_status(void* stream) {
     if (e != cudaSuccess) return cuda_fail(e, "cudaStreamSynchronize");
     e = device_info(&dev, &status);
     if (e != cudaSuccess) return cuda_fail(e, "device query");
-    unsigned v = 0;
-    e = cudaMemcpy(&v, status, sizeof(unsigned), cudaMemcpyDeviceToHost);
+    unsigned v[8] = {0};
+    e = cudaMemcpy(v, status, sizeof(v), cudaMemcpyDeviceToHost);
     if (e != cudaSuccess) return cuda_fail(e, "status read");
-    const unsigned zero = 0;
-    e = cudaMemcpy(status, &zero, sizeof(unsigned), cudaMemcpyHostToDevice);
+    const unsigned zero[8] = {0};
+    e = cudaMemcpy(status, zero, sizeof(zero), cudaMemcpyHostToDevice);
     if (e != cudaSuccess) return cuda_fail(e, "status clear");
-    if (v == gs::kDevTimeout)
-        return fail(GS_ERR_DEVICE_TIMEOUT, "a device-side wait ran out of time");
+    if (v[0] == gs::kDevTimeout) {
+        char where[160];
+        std::snprintf(where, sizeof(where),
+                      "block (%u, %u), warp %u, barrier at shared address %u, parity %u", v[1],
+                      v[2], v[3], v[4], v[5]);
+        return fail(GS_ERR_DEVICE_TIMEOUT, "a device-side wait ran out of time: %s", where);
+    }
     return GS_OK;
 }
 

@@ -32,6 +32,12 @@ struct TcPlan {
     bool aug;                // FMA kernel with augmented operands (Dp = D + 2 aug_norm_terms
                              // rounded to 16)
     int nq;                  // query tiles of 128 rows per CTA (FMA kernel)
+    // FMA kernel work split: units = (pairs of query tiles) x key tiles, in
+    // row-major order; CTA i takes units [i unit_len, (i + 1) unit_len); the
+    // partial sums of a pair of query tiles have one slot per contributing
+    // CTA (`splits` = the largest number of contributors).
+    int64_t units, unit_len;
+    int grid;
     size_t off_mean_part, off_mu, off_qh, off_kh, off_A, off_B, off_vt, off_vmax, off_inv,
         off_rec, off_part, total;
 };
@@ -65,6 +71,13 @@ cudaError_t launch_value_prep(InType t, bool grad, const void* v, const void* k,
 // mode 0: forward (out M x Cv, scaled by inv_scale when given)
 // mode 1: gradient from augmented values (tensor path): needs q, mu, tau
 // mode 2: gradient from direct partials (SIMT path): Cv = D + 1
+// Forward sum of the FMA kernel's contributor slots: rows of the pair of
+// query tiles r = m / rows_per_unit have slots 0 .. last(r) - first(r), with
+// first(r) = r key_tiles / unit_len and last(r) = ((r + 1) key_tiles - 1) /
+// unit_len, added in slot order.
+cudaError_t launch_finalize_slots(const float* part, int64_t Mpad, int64_t M, int C,
+                                  int rows_per_unit, int64_t key_tiles, int64_t unit_len,
+                                  float* out, cudaStream_t s);
 cudaError_t launch_finalize(int mode, InType t, const float* part, int splits,
                             int64_t split_stride_rows, int64_t M, int Cv, int part_ld,
                             const float* inv_scale, const void* q, const float* mu, float tau,

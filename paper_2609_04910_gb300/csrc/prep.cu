@@ -14,6 +14,8 @@
 //    transposed (channel-major) so that both MMAs read K-major operands;
 //  * the fixed-order sum of key-split partials and the final scaling, or
 //    the gradient tau (S[:D] - q_m S[D]) of Sec. 3.
+#include <algorithm>
+
 #include <cuda_bf16.h>
 #include <cuda_fp16.h>
 #include <math_constants.h>
@@ -73,6 +75,62 @@ __global__ void mean_partial_kernel(const T* __restrict__ q, const T* __restrict
             partial[static_cast<int64_t>(gridDim.x + blockIdx.x) * D + d] = m;
         }
         __syncthreads();
+    }
+}
+
+// Vectorised variant for 16-bit inputs with D a power of two in [8, 2048]:
+// 256 threads read 16-byte vectors (8 coordinates) of a contiguous run of
+// rows; a block advances by 2048 elements, a multiple of D, so every thread
+// always sees the same 8 coordinates and keeps their sums and maxima in
+// registers.  Blocks [0, Gq) cover rows of q, blocks [Gq, G) rows of k
+// (none when q and k are the same points).  Same partial layout as above.
+constexpr int kMeanVecThreads = 256;
+
+template <typename T>
+__global__ void __launch_bounds__(kMeanVecThreads)
+mean_partial_vec_kernel(const T* __restrict__ q, const T* __restrict__ k, int64_t M, int64_t N,
+                        int D, int64_t rows_per_block, int Gq, float* __restrict__ partial) {
+    __shared__ float s_sum[kMeanVecThreads][9];
+    __shared__ float s_max[kMeanVecThreads][9];
+    const int t = threadIdx.x;
+    const bool on_q = static_cast<int>(blockIdx.x) < Gq;
+    const int64_t b = on_q ? blockIdx.x : blockIdx.x - Gq;
+    const int64_t rows = on_q ? M : N;
+    const T* x = on_q ? q : k;
+    const int64_t r0 = b * rows_per_block;
+    const int64_t r1 = min(r0 + rows_per_block, rows);
+    const int64_t v0 = r0 * D / 8, v1 = r1 * D / 8;      // 8-element vectors
+    const uint4* xv = reinterpret_cast<const uint4*>(x);
+    float sum[8], mx[8];
+#pragma unroll
+    for (int e = 0; e < 8; ++e) sum[e] = mx[e] = 0.f;
+    for (int64_t v = v0 + t; v < v1; v += kMeanVecThreads) {
+        const uint4 u = xv[v];
+        const T* h = reinterpret_cast<const T*>(&u);
+#pragma unroll
+        for (int e = 0; e < 8; ++e) {
+            const float f = to_f(h[e]);
+            sum[e] += f;
+            mx[e] = fmaxf(mx[e], fabsf(f));
+        }
+    }
+#pragma unroll
+    for (int e = 0; e < 8; ++e) {
+        s_sum[t][e] = sum[e];
+        s_max[t][e] = mx[e];
+    }
+    __syncthreads();
+    // Thread t holds coordinates 8 (t mod NG) .. +7, NG = D / 8 groups.
+    const int NG = D / 8;
+    for (int d = t; d < D; d += kMeanVecThreads) {
+        const int g = d >> 3, e = d & 7;
+        float a = 0.f, m = 0.f;
+        for (int u = g; u < kMeanVecThreads; u += NG) {
+            a += s_sum[u][e];
+            m = fmaxf(m, s_max[u][e]);
+        }
+        partial[static_cast<int64_t>(blockIdx.x) * D + d] = a;
+        partial[static_cast<int64_t>(gridDim.x + blockIdx.x) * D + d] = m;
     }
 }
 
@@ -162,9 +220,17 @@ operand_kernel(const T* __restrict__ x, int64_t rows, int D, int Dp, int nt, flo
                const float* __restrict__ mu, float half_c, float pad_value,
                T* __restrict__ out_q, T* __restrict__ out_k, float* __restrict__ nrm) {
     constexpr int R = kRowsPerBlock;
-    __shared__ __align__(16) T s_in[R * kOperandMaxCols];
-    __shared__ __align__(16) T s_out[R * kOperandMaxCols];   // AUG: q rows, then k rows
-    __shared__ float s_mu[kOperandMaxCols];
+    // Dynamic shared memory sized to this call: s_out holds R x Dp
+    // elements per written layout (AUG: q rows, then k rows), s_in the R x D
+    // input elements (rounded up to 16 bytes), then D floats of mu.
+    extern __shared__ __align__(16) uint8_t operand_smem[];
+    const bool wq = AUG ? out_q != nullptr : true;
+    const bool wk = AUG && out_k != nullptr;
+    const int nout = (wq ? 1 : 0) + (wk ? 1 : 0);
+    T* s_out = reinterpret_cast<T*>(operand_smem);
+    T* s_in = s_out + nout * R * Dp;
+    float* s_mu = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(s_in) +
+                                           ((R * D * static_cast<int>(sizeof(T)) + 15) & ~15));
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int64_t r0 = static_cast<int64_t>(blockIdx.x) * R;
     for (int d = tid; d < D; d += kOperandThreads) s_mu[d] = mu ? mu[d] : 0.f;
@@ -181,8 +247,6 @@ operand_kernel(const T* __restrict__ x, int64_t rows, int D, int Dp, int nt, flo
         for (int i = nvec * PER_VEC + tid; i < n_el; i += kOperandThreads) s_in[i] = src[i];
     }
     __syncthreads();
-    const bool wq = AUG ? out_q != nullptr : true;
-    const bool wk = AUG && out_k != nullptr;
     T* sq = s_out;
     T* sk = s_out + (wq ? R * Dp : 0);
     const T zero = from_f<T>(0.f);
@@ -248,6 +312,21 @@ operand_kernel(const T* __restrict__ x, int64_t rows, int D, int Dp, int nt, flo
     }
 }
 
+__global__ void finalize_slots_kernel(const float* __restrict__ part, int64_t Mpad, int64_t M,
+                                      int C, int rows_per_unit, int64_t key_tiles,
+                                      int64_t unit_len, float* __restrict__ out) {
+    const int64_t idx = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
+    if (idx >= M * C) return;
+    const int64_t m = idx / C;
+    const int c = static_cast<int>(idx - m * C);
+    const int64_t r = m / rows_per_unit;
+    const int64_t first = r * key_tiles / unit_len;
+    const int64_t last = ((r + 1) * key_tiles - 1) / unit_len;
+    float acc = 0.f;
+    for (int64_t sl = 0; sl <= last - first; ++sl) acc += part[(sl * Mpad + m) * C + c];
+    out[idx] = acc;
+}
+
 template <typename T, bool AUG>
 cudaError_t operand_typed(const void* x, int64_t rows, int64_t rows_pad, int D, int Dp, int nt,
                           float F, const float* mu, float half_c, float pad_value, void* out_q,
@@ -257,7 +336,11 @@ cudaError_t operand_typed(const void* x, int64_t rows, int64_t rows_pad, int D, 
         return cudaErrorInvalidValue;
     const int64_t blocks = rows_pad / kRowsPerBlock;
     if (blocks == 0) return cudaSuccess;
-    operand_kernel<T, AUG><<<static_cast<unsigned>(blocks), kOperandThreads, 0, s>>>(
+    const int nout = AUG ? (out_q ? 1 : 0) + (out_k ? 1 : 0) : 1;
+    const size_t smem = static_cast<size_t>(nout) * kRowsPerBlock * Dp * sizeof(T) +
+                        ((static_cast<size_t>(kRowsPerBlock) * D * sizeof(T) + 15) & ~size_t(15)) +
+                        static_cast<size_t>(D) * sizeof(float);
+    operand_kernel<T, AUG><<<static_cast<unsigned>(blocks), kOperandThreads, smem, s>>>(
         static_cast<const T*>(x), rows, D, Dp, nt, F, mu, half_c, pad_value,
         static_cast<T*>(out_q), static_cast<T*>(out_k), nrm);
     note_launches(1);
@@ -453,25 +536,48 @@ cudaError_t finalize_typed(const float* part, int splits, int64_t stride_rows, i
 
 cudaError_t launch_mean(InType t, const void* q, const void* k, int64_t M, int64_t N, int D,
                         int blocks, float* partial, float* mu, cudaStream_t s) {
+    // q and k the same points: the mean of [q; q] is the mean of q.
+    if (q == k && M == N) N = 0;
     const int64_t total = M + N;
-    const int64_t rpb = (total + blocks - 1) / blocks;
-    const int G = static_cast<int>((total + rpb - 1) / rpb);
-    switch (t) {
-        case InType::F16:
-            mean_partial_kernel<__half><<<G, dim3(32, 8), 0, s>>>(
-                static_cast<const __half*>(q), static_cast<const __half*>(k), M, N, D, rpb, partial);
-            note_launches(1);
-            break;
-        case InType::BF16:
-            mean_partial_kernel<__nv_bfloat16><<<G, dim3(32, 8), 0, s>>>(
-                static_cast<const __nv_bfloat16*>(q), static_cast<const __nv_bfloat16*>(k), M, N,
-                D, rpb, partial);
-            note_launches(1);
-            break;
-        default:
-            mean_partial_kernel<float><<<G, dim3(32, 8), 0, s>>>(
-                static_cast<const float*>(q), static_cast<const float*>(k), M, N, D, rpb, partial);
-            note_launches(1);
+    int G = 0;
+    const bool vec = t != InType::F32 && D >= 8 && D <= 2048 && (D & (D - 1)) == 0 &&
+                     2048 % D == 0 && blocks >= 4;
+    if (vec) {
+        // At most `blocks` blocks over both arrays (the partial buffer holds
+        // `blocks` rows of 2 D floats).
+        const int64_t rpb = std::max<int64_t>(1, (total + blocks - 3) / (blocks - 2));
+        const int Gq = static_cast<int>((M + rpb - 1) / rpb);
+        const int Gk = static_cast<int>((N + rpb - 1) / rpb);
+        G = Gq + Gk;
+        if (t == InType::F16)
+            mean_partial_vec_kernel<__half><<<G, kMeanVecThreads, 0, s>>>(
+                static_cast<const __half*>(q), static_cast<const __half*>(k), M, N, D, rpb, Gq,
+                partial);
+        else
+            mean_partial_vec_kernel<__nv_bfloat16><<<G, kMeanVecThreads, 0, s>>>(
+                static_cast<const __nv_bfloat16*>(q), static_cast<const __nv_bfloat16*>(k), M, N, D,
+                rpb, Gq, partial);
+        note_launches(1);
+    } else {
+        const int64_t rpb = (total + blocks - 1) / blocks;
+        G = static_cast<int>((total + rpb - 1) / rpb);
+        switch (t) {
+            case InType::F16:
+                mean_partial_kernel<__half><<<G, dim3(32, 8), 0, s>>>(
+                    static_cast<const __half*>(q), static_cast<const __half*>(k), M, N, D, rpb,
+                    partial);
+                break;
+            case InType::BF16:
+                mean_partial_kernel<__nv_bfloat16><<<G, dim3(32, 8), 0, s>>>(
+                    static_cast<const __nv_bfloat16*>(q), static_cast<const __nv_bfloat16*>(k), M, N,
+                    D, rpb, partial);
+                break;
+            default:
+                mean_partial_kernel<float><<<G, dim3(32, 8), 0, s>>>(
+                    static_cast<const float*>(q), static_cast<const float*>(k), M, N, D, rpb,
+                    partial);
+        }
+        note_launches(1);
     }
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
@@ -479,6 +585,18 @@ cudaError_t launch_mean(InType t, const void* q, const void* k, int64_t M, int64
     const int min_exp = t == InType::F16 ? -24 : t == InType::BF16 ? -133 : -149;
     mean_final_kernel<<<D, kMeanFinalThreads, 0, s>>>(partial, G, D, static_cast<double>(total),
                                                      mant_bits, min_exp, mu);
+    note_launches(1);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_finalize_slots(const float* part, int64_t Mpad, int64_t M, int C,
+                                  int rows_per_unit, int64_t key_tiles, int64_t unit_len,
+                                  float* out, cudaStream_t s) {
+    const int64_t total = M * C;
+    if (total == 0) return cudaSuccess;
+    const int threads = 256;
+    finalize_slots_kernel<<<static_cast<unsigned>((total + threads - 1) / threads), threads, 0, s>>>(
+        part, Mpad, M, C, rows_per_unit, key_tiles, unit_len, out);
     note_launches(1);
     return cudaGetLastError();
 }

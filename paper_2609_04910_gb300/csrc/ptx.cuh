@@ -116,7 +116,9 @@ __device__ __forceinline__ bool mbar_test_wait2(uint64_t* bar1, uint32_t parity1
 // Wait for the phase of `bar` with the given parity to complete.  Returns
 // false (without waiting any longer) if the CTA abort flag is raised or the
 // global-time limit runs out; in the latter case the status word receives
-// kDevTimeout and the abort flag is raised for the other roles.  With a null
+// kDevTimeout (the first such wait also writes its block, warp, barrier
+// address and parity into status[1..5]) and the abort flag is raised for
+// the other roles.  With a null
 // abort flag only the time limit applies (used to drain copies in flight).
 __device__ __forceinline__ bool mbar_wait_bounded(uint64_t* bar, uint32_t parity,
                                                   volatile int* abort_flag,
@@ -128,7 +130,15 @@ __device__ __forceinline__ bool mbar_wait_bounded(uint64_t* bar, uint32_t parity
         if ((i & 15u) == 0u) {
             if (abort_flag != nullptr && *abort_flag) return false;
             if (global_timer_ns() - t0 > GS_WAIT_LIMIT_NS) {
-                atomicCAS(status, kDevOk, kDevTimeout);
+                // The first wait to run out records where it was.
+                if (atomicCAS(status, kDevOk, kDevTimeout) == kDevOk) {
+                    volatile unsigned* rec = status + 1;
+                    rec[0] = blockIdx.x;
+                    rec[1] = blockIdx.y;
+                    rec[2] = threadIdx.x >> 5;
+                    rec[3] = smem_u32(bar);
+                    rec[4] = parity;
+                }
                 if (abort_flag != nullptr) *abort_flag = 1;
                 return false;
             }
@@ -352,6 +362,17 @@ __device__ __forceinline__ uint32_t pack_half2_satfinite(float lo, float hi) {
     uint32_t r;
     asm("cvt.rn.satfinite.f16x2.f32 %0, %1, %2;" : "=r"(r) : "f"(hi), "f"(lo));
     return r;
+}
+
+// Per-warpgroup register budget change (all warps of a warpgroup execute
+// the same one).  inc blocks until the CTA's register pool can serve it.
+template <uint32_t N>
+__device__ __forceinline__ void reg_alloc() {
+    asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;" ::"n"(N));
+}
+template <uint32_t N>
+__device__ __forceinline__ void reg_dealloc() {
+    asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(N));
 }
 
 // Packed pairs of fp32 values (sm_100+ f32x2 arithmetic): one instruction

@@ -438,6 +438,30 @@ bool plan_tensor(InType t, int64_t M, int64_t N, int64_t D, int64_t C, bool grad
         best_s = static_cast<int>((key_tiles + tps - 1) / tps);
     }
     p->splits = std::max(1, best_s);
+    p->units = p->unit_len = 0;
+    p->grid = 0;
+    if (p->fma) {
+        // Persistent split: one CTA per SM, each taking an equal run of
+        // (pair of query tiles, key tile) units; with a forced split count
+        // each pair of query tiles is cut into that many runs instead.
+        const int64_t units = tiles * key_tiles;
+        if (units >= (int64_t(1) << 31)) {
+            *why = "too many query/key tile pairs for the FMA kernel";
+            return false;
+        }
+        int64_t len = split_override > 0
+                          ? (key_tiles + std::min<int64_t>(split_override, key_tiles) - 1) /
+                                std::min<int64_t>(split_override, key_tiles)
+                          : (units + sms - 1) / sms;
+        len = std::max<int64_t>(1, len);
+        p->units = units;
+        p->unit_len = len;
+        p->grid = static_cast<int>((units + len - 1) / len);
+        int64_t most = 1;
+        for (int64_t r = 0; r < tiles; ++r)
+            most = std::max(most, ((r + 1) * key_tiles - 1) / len - r * key_tiles / len + 1);
+        p->splits = static_cast<int>(most);
+    }
     // ~256 rows per block of the mean kernel, so that every SM has work.
     p->mean_blocks = static_cast<int>(std::max<int64_t>(1, std::min<int64_t>(4096, (M + N + 255) / 256)));
 

@@ -69,16 +69,22 @@ constexpr uint32_t TMEM_COLS = 512;
 constexpr int MAX_STAGES = NCTRL_MAX;   // one stage per control warp
 // Augmented operands keep q^ in shared memory (two TMEM slots of S).
 constexpr bool kAugQsm = true;
+// Register split between the roles (setmaxnreg); the sum stays within the
+// registers the CTA is launched with (THREADS x 96).
+constexpr uint32_t kExpRegs = 104;
+constexpr uint32_t kCtrlRegs = 40;
+static_assert(NEXP * 32 * kExpRegs + NCTRL_MAX * 32 * kCtrlRegs <= THREADS * 96, "register split");
 
 struct FmaParams {
     const uint32_t* qh;  // Mpad x Dp/2 packed 16-bit pairs (centred, rounded q)
     const float* A;      // Mpad: -(c/2)||q^_m||^2
     const float* rec;    // key records, Npad / 2 pairs
-    float* part;         // splits x Mpad x C partial sums
+    float* part;         // contributor slots x Mpad x C partial sums
     unsigned* status;
     int64_t Mpad;
+    int units;           // work units: (pair of query tiles, key tile), row major
+    int unit_len;        // units per CTA (CTA i: units [i unit_len, (i + 1) unit_len))
     int key_tiles;
-    int tiles_per_split;
     int Dp;
     int nkb;             // 64-element K blocks of q^ / k^
     int stages;
@@ -93,7 +99,6 @@ struct FmaParams {
 
 struct __align__(8) FmaBarriers {
     uint64_t qa_ready;          // q^ available to the MMAs
-    uint64_t drain;
     uint64_t s_full[MAX_SL];    // slot phase: both S tiles of a key tile computed
     uint64_t s_free[MAX_SL];    // slot phase: both S tiles of a key tile in registers
     uint64_t kv_full[MAX_STAGES];
@@ -132,27 +137,9 @@ tc_gauss_fma_kernel(const __grid_constant__ CUtensorMap tm_q,
     const int tid = threadIdx.x;
     const int warp = tid >> 5;
     const int lane = tid & 31;
-    const int tile_m = blockIdx.x;   // query tiles 2 tile_m and 2 tile_m + 1
-    const int split = blockIdx.y;
-    const int kt0 = split * p.tiles_per_split;
-    const int T = min(p.key_tiles, kt0 + p.tiles_per_split) - kt0;
     volatile int* abort_flag = &bars->abort_flag;
 
-    if (tid == 0) {
-        mbar_init(&bars->qa_ready, QSM ? 1 : NEXP);
-        // One drain commit per control warp that has key tiles.
-        mbar_init(&bars->drain, max(1, min(T, p.stages)));
-        for (int sl = 0; sl < SL; ++sl) {
-            mbar_init(&bars->s_full[sl], 1);
-            mbar_init(&bars->s_free[sl], NEXP);        // one arrival per exponent warp
-        }
-        for (int s = 0; s < p.stages; ++s) {
-            mbar_init(&bars->kv_full[s], 1);
-            mbar_init(&bars->kv_empty[s], 1 + NEXP);  // MMA commit + exponent warps
-        }
-        bars->abort_flag = 0;
-        fence_mbar_init();
-    }
+    if (tid == 0) bars->abort_flag = 0;
     if (warp == CTRL_WARP0) {
         tmem_alloc(&bars->tmem_base, TMEM_COLS);
         tmem_relinquish();
@@ -168,257 +155,344 @@ tc_gauss_fma_kernel(const __grid_constant__ CUtensorMap tm_q,
         return reinterpret_cast<const float*>(stage0 + s * p.stage_bytes + p.kh_bytes);
     };
 
+    // The CTA's units form segments of consecutive key tiles of one pair of
+    // query tiles.  The barriers are initialised once and keep running
+    // across segments: every stage, slot and phase follows the CTA-local
+    // running tile index g = u - u_begin, and qa_ready completes once per
+    // segment.  Each segment writes its partial sums to the slot of this
+    // CTA among the CTAs that contribute to that pair of query tiles.
+    if (tid == 0) {
+        mbar_init(&bars->qa_ready, QSM ? 1 : NEXP);
+        for (int sl = 0; sl < SL; ++sl) {
+            mbar_init(&bars->s_full[sl], 1);
+            mbar_init(&bars->s_free[sl], NEXP);        // one arrival per exponent warp
+        }
+        for (int s = 0; s < p.stages; ++s) {
+            mbar_init(&bars->kv_full[s], 1);
+            mbar_init(&bars->kv_empty[s], 1 + NEXP);  // MMA commit + exponent warps
+        }
+        fence_mbar_init();
+    }
+    __syncthreads();
+    // Unit indices fit in 32 bits (the plan checks units < 2^31).
+    const int u_begin = static_cast<int>(blockIdx.x) * p.unit_len;
+    const int u_end = p.units < u_begin + p.unit_len ? p.units : u_begin + p.unit_len;
+    // Segment barrier of both role loops (a non-aligned barrier, since the
+    // two roles reach it from different loops).
+    auto segment_sync = [&]() {
+        tc_fence_before();
+        asm volatile("barrier.sync 2, %0;" ::"r"(THREADS) : "memory");
+        tc_fence_after();
+    };
     if (warp >= CTRL_WARP0) {
-        // ------------------------------------------------ control warps
-        // Control warp k (on SMSP k) owns shared-memory stage k and key
-        // tiles j = k, k + nctrl, ...: it loads their keys and records and
-        // issues their MMAs, so that the MMA issue work is spread over the
-        // SMSPs instead of slowing the exponent warps of one of them.  The
-        // whole warp runs the loop (warp-uniform operands); the elected lane
-        // issues copies, MMAs and commits.
-        const int k = warp - CTRL_WARP0;
-        const int nctrl = p.stages;
-        if (k < nctrl && k < T) {
+        // Control warps need few registers; the exponent warps take them
+        // (16 x 32 x kExpRegs + 4 x 32 x kCtrlRegs <= 640 x 96 at launch).
+        reg_dealloc<kCtrlRegs>();
+        uint32_t seg_parity = 0;   // parity of the qa_ready phase of this segment
+        for (int u = u_begin; u < u_end; seg_parity ^= 1u) {
+        // Read by every thread after a CTA barrier: uniform.
+        if (*abort_flag) break;
+        const int tile_m = u / p.key_tiles;   // query tiles 2 tile_m, 2 tile_m + 1
+        const int kt0 = u - tile_m * p.key_tiles;
+        const int T = min(p.key_tiles - kt0, u_end - u);
+        const int g0 = u - u_begin;           // running index of the segment's first tile
+        const int slot = static_cast<int>(blockIdx.x) -
+                         static_cast<int>(static_cast<int64_t>(tile_m) * p.key_tiles / p.unit_len);
+
+            // ------------------------------------------------ control warps
+            // Control warp k (on SMSP k) owns shared-memory stage k and the key
+            // tiles with running index g = k (mod nctrl): it loads their keys and
+            // records and issues their MMAs, so that the MMA issue work is spread over the
+            // SMSPs instead of slowing the exponent warps of one of them.  The
+            // whole warp runs the loop (warp-uniform operands); the elected lane
+            // issues copies, MMAs and commits.
+            const int k = warp - CTRL_WARP0;
+            const int nctrl = p.stages;
+            // This warp's tiles: running index g = g0 + j with g = k (mod nctrl).
+            const int j_first = (k - g0 % nctrl + nctrl) % nctrl;
+            const bool has_tiles = k < nctrl && j_first < T;
             const bool leader = elect_one();
-            auto load_keys = [&](int j) {
-                mbar_arrive_expect_tx(&bars->kv_full[k], p.kh_bytes + p.rec_bytes);
-                const int n0 = (kt0 + j) * BN;
-                for (int kb = 0; kb < p.nkb; ++kb)
-                    tma_load_2d(kh_smem(k) + kb * (BN * 128), &tm_k, &bars->kv_full[k], kb * KB, n0);
-                bulk_load(const_cast<float*>(rec_smem(k)),
-                          p.rec + static_cast<int64_t>(n0 / 2) * REC_PAIR, p.rec_bytes,
-                          &bars->kv_full[k]);
-            };
-            if (leader) {
-                tma_prefetch_desc(&tm_k);
-                if (QSM && k == 0) {
-                    tma_prefetch_desc(&tm_q);
-                    mbar_arrive_expect_tx(&bars->qa_ready, p.q_bytes);
-                    for (int h = 0; h < NQ; ++h)
-                        for (int kb = 0; kb < p.nkb; ++kb)
-                            tma_load_2d(q_smem + (h * p.nkb + kb) * (BM * 128), &tm_q, &bars->qa_ready,
-                                        kb * KB, (tile_m * NQ + h) * BM);
-                }
-                load_keys(k);
+            if (QSM && k == 0 && leader) {
+                // q^ of this segment; the MMAs of earlier segments are complete.
+                tma_prefetch_desc(&tm_q);
+                mbar_arrive_expect_tx(&bars->qa_ready, p.q_bytes);
+                for (int h = 0; h < NQ; ++h)
+                    for (int kb = 0; kb < p.nkb; ++kb)
+                        tma_load_2d(q_smem + (h * p.nkb + kb) * (BM * 128), &tm_q, &bars->qa_ready,
+                                    kb * KB, (tile_m * NQ + h) * BM);
             }
             __syncwarp();
-            bool ok = warp_wait(&bars->qa_ready, 0, abort_flag, p.status);
-            const int ksteps = p.Dp / 16;
-            // Shared-memory descriptors of stage k and of q^ tile 0; query
-            // tile h and K step kk add byte offsets / 16 to the start-address
-            // field.
-            const uint64_t kdesc = smem_desc_kmajor_sw128(smem_u32(kh_smem(k)));
-            const uint64_t qdesc0 = smem_desc_kmajor_sw128(smem_u32(q_smem));
-            const uint32_t qdesc_h = static_cast<uint32_t>((p.nkb * BM * 128) >> 4);
-            const uint32_t a0 = tmem + qa_col, a1 = a0 + (p.Dp / 2);
-            bool pending = true;          // keys of tile j requested, not yet waited for
-            uint32_t ph = 0;              // parity of this warp's stage barriers for tile j
-            int j = k;
-            for (; ok && j < T; j += nctrl, ph ^= 1u) {
-                // S slot of tile j and the parities of its barriers: s_full
-                // completes once per tile of the slot, and tile j reuses the
-                // slot that tile j - SL released.
-                const int sl = SL == 2 ? (j & 1) : 0;
-                const uint32_t full_parity = static_cast<uint32_t>(SL == 2 ? (j >> 1) : j) & 1u;
-                const uint32_t free_parity = full_parity ^ 1u;
-                const bool ready = __all_sync(
-                    0xffffffffu, j < SL ? mbar_test_wait(&bars->kv_full[k], ph)
-                                        : mbar_test_wait2(&bars->s_free[sl], free_parity,
-                                                          &bars->kv_full[k], ph));
-                if (!ready) {
-                    if (j >= SL) {
-                        ok = warp_wait(&bars->s_free[sl], free_parity, abort_flag, p.status);
-                        if (!ok) break;
-                    }
-                    ok = warp_wait(&bars->kv_full[k], ph, abort_flag, p.status);
-                    if (!ok) break;
-                }
-                pending = false;
-                tc_fence_after();
-                const uint32_t d0 = tmem + sl * (2 * BN), d1 = d0 + BN;
+            if (has_tiles) {
+                auto load_keys = [&](int j) {
+                    mbar_arrive_expect_tx(&bars->kv_full[k], p.kh_bytes + p.rec_bytes);
+                    const int n0 = (kt0 + j) * BN;
+                    for (int kb = 0; kb < p.nkb; ++kb)
+                        tma_load_2d(kh_smem(k) + kb * (BN * 128), &tm_k, &bars->kv_full[k], kb * KB, n0);
+                    bulk_load(const_cast<float*>(rec_smem(k)),
+                              p.rec + static_cast<int64_t>(n0 / 2) * REC_PAIR, p.rec_bytes,
+                              &bars->kv_full[k]);
+                };
                 if (leader) {
-                    for (int h = 0; h < NQ; ++h) {
-                        for (int kk = 0; kk < ksteps; ++kk) {
-                            const uint32_t koff = static_cast<uint32_t>((kk >> 2) * (BN * 128 / 16) + (kk & 3) * 2);
-                            if (QSM) {
-                                const uint32_t qoff = h * qdesc_h + static_cast<uint32_t>((kk >> 2) * (BM * 128 / 16) + (kk & 3) * 2);
-                                mma_ss_f16(h ? d1 : d0, qdesc0 + qoff, kdesc + koff, p.idesc, kk > 0 ? 1u : 0u);
-                            } else {
-                                mma_ts_f16(h ? d1 : d0, (h ? a1 : a0) + kk * 8, kdesc + koff, p.idesc,
-                                           kk > 0 ? 1u : 0u);
-                            }
-                        }
-                    }
-                    mma_commit(&bars->s_full[sl]);
-                    mma_commit(&bars->kv_empty[k]);
+                    tma_prefetch_desc(&tm_k);
+                    load_keys(j_first);
                 }
                 __syncwarp();
-                if (j + nctrl < T) {
+                bool ok = warp_wait(&bars->qa_ready, seg_parity, abort_flag, p.status);
+                const int ksteps = p.Dp / 16;
+                // Shared-memory descriptors of stage k and of q^ tile 0; query
+                // tile h and K step kk add byte offsets / 16 to the start-address
+                // field.
+                const uint64_t kdesc = smem_desc_kmajor_sw128(smem_u32(kh_smem(k)));
+                const uint64_t qdesc0 = smem_desc_kmajor_sw128(smem_u32(q_smem));
+                const uint32_t qdesc_h = static_cast<uint32_t>((p.nkb * BM * 128) >> 4);
+                const uint32_t a0 = tmem + qa_col, a1 = a0 + (p.Dp / 2);
+                bool pending = true;          // keys of tile j requested, not yet waited for
+                // Parity of stage k's barriers for tile j: stage k completes once
+                // per tile g = k (mod nctrl).
+                uint32_t ph = static_cast<uint32_t>((g0 + j_first) / nctrl) & 1u;
+                int j = j_first;
+                for (; ok && j < T; j += nctrl, ph ^= 1u) {
+                    // S slot of tile j and the parities of its barriers: s_full
+                    // completes once per tile of the slot, and tile g reuses the
+                    // slot that tile g - SL released.
+                    const int g = g0 + j;
+                    const int sl = SL == 2 ? (g & 1) : 0;
+                    const uint32_t full_parity = static_cast<uint32_t>(SL == 2 ? (g >> 1) : g) & 1u;
+                    const uint32_t free_parity = full_parity ^ 1u;
+                    const bool ready = __all_sync(
+                        0xffffffffu, g < SL ? mbar_test_wait(&bars->kv_full[k], ph)
+                                            : mbar_test_wait2(&bars->s_free[sl], free_parity,
+                                                              &bars->kv_full[k], ph));
+                    if (!ready) {
+                        if (g >= SL) {
+                            ok = warp_wait(&bars->s_free[sl], free_parity, abort_flag, p.status);
+                            if (!ok) break;
+                        }
+                        ok = warp_wait(&bars->kv_full[k], ph, abort_flag, p.status);
+                        if (!ok) break;
+                    }
+                    pending = false;
+                    tc_fence_after();
+                    const uint32_t d0 = tmem + sl * (2 * BN), d1 = d0 + BN;
+                    if (leader) {
+                        for (int h = 0; h < NQ; ++h) {
+                            for (int kk = 0; kk < ksteps; ++kk) {
+                                const uint32_t koff = static_cast<uint32_t>((kk >> 2) * (BN * 128 / 16) + (kk & 3) * 2);
+                                if (QSM) {
+                                    const uint32_t qoff = h * qdesc_h + static_cast<uint32_t>((kk >> 2) * (BM * 128 / 16) + (kk & 3) * 2);
+                                    mma_ss_f16(h ? d1 : d0, qdesc0 + qoff, kdesc + koff, p.idesc, kk > 0 ? 1u : 0u);
+                                } else {
+                                    mma_ts_f16(h ? d1 : d0, (h ? a1 : a0) + kk * 8, kdesc + koff, p.idesc,
+                                               kk > 0 ? 1u : 0u);
+                                }
+                            }
+                        }
+                        mma_commit(&bars->s_full[sl]);
+                        mma_commit(&bars->kv_empty[k]);
+                    }
+                    __syncwarp();
                     // Stage k is free again once these MMAs and the exponent
-                    // warps are done with tile j.
+                    // warps are done with tile j; after the last tile this also
+                    // makes sure every arrival on the stage has landed before the
+                    // barriers are initialised for the next segment.
                     ok = warp_wait(&bars->kv_empty[k], ph, abort_flag, p.status);
                     if (!ok) break;
-                    if (leader) load_keys(j + nctrl);
-                    __syncwarp();
-                    pending = true;
+                    if (j + nctrl < T) {
+                        if (leader) load_keys(j + nctrl);
+                        __syncwarp();
+                        pending = true;
+                    }
                 }
+                // Every copy and MMA this warp started must be complete before
+                // the barriers are initialised again or the CTA exits.  The
+                // stage-release wait after the last tile already covers the MMAs
+                // (the commit on kv_empty arrives once all MMAs this thread
+                // issued are complete); copies still in flight after an abort
+                // are waited for here.  These waits poll per lane, so the warp
+                // reconverges after them.
+                if (pending) mbar_wait_bounded(&bars->kv_full[k], ph, nullptr, p.status);
+                __syncwarp();
             }
-            // Every copy and MMA this warp started must be complete before
-            // the CTA exits.
-            if (pending) mbar_wait_bounded(&bars->kv_full[k], ph, nullptr, p.status);
-            if (QSM && k == 0) mbar_wait_bounded(&bars->qa_ready, 0, nullptr, p.status);
-            if (leader) mma_commit(&bars->drain);
-            __syncwarp();
-            mbar_wait_bounded(&bars->drain, 0, nullptr, p.status);
+            if (QSM && k == 0) {
+                // The q^ copy of this segment must have landed before the CTA
+                // moves on (the next segment overwrites q^).
+                mbar_wait_bounded(&bars->qa_ready, seg_parity, nullptr, p.status);
+                __syncwarp();
+            }
+        // Segment end: every MMA, copy and TMEM read of this segment is done
+        // (control warps waited for their last stage release and copies).
+        segment_sync();
+        u += T;
         }
     } else {
-        // ------------------------------------------------ exponent warps
-        const int quarter = warp & 3;
-        const int cg = warp >> 2;                  // column group: keys 32 cg .. 32 cg + 31
-        const uint32_t lane_base = static_cast<uint32_t>(quarter * 32) << 16;
-        const int row_t = quarter * 32 + lane;     // row inside each query tile
-        const int64_t row0 = static_cast<int64_t>(tile_m) * NQ * BM + row_t;
-        const int64_t row1 = row0 + BM;
+        reg_alloc<kExpRegs>();
+        uint32_t seg_parity = 0;
+        for (int u = u_begin; u < u_end; seg_parity ^= 1u) {
+        // Read by every thread after a CTA barrier: uniform.
+        if (*abort_flag) break;
+        const int tile_m = u / p.key_tiles;   // query tiles 2 tile_m, 2 tile_m + 1
+        const int kt0 = u - tile_m * p.key_tiles;
+        const int T = min(p.key_tiles - kt0, u_end - u);
+        const int g0 = u - u_begin;           // running index of the segment's first tile
+        const int slot = static_cast<int>(blockIdx.x) -
+                         static_cast<int>(static_cast<int64_t>(tile_m) * p.key_tiles / p.unit_len);
 
-        if (!QSM) {
-            // q^ rows -> TMEM (A operand).  Column group cg copies query tile
-            // cg / 2, 8-column chunks ck = cg % 2 (mod 2) of its Dp / 2 columns.
-            const int h = cg >> 1;
-            const uint32_t* src = p.qh + (row0 + h * BM) * (p.Dp / 2);
-            for (int ck = cg & 1; ck < p.Dp / 16; ck += 2) {
-                const uint4 lo = *reinterpret_cast<const uint4*>(src + ck * 8);
-                const uint4 hi = *reinterpret_cast<const uint4*>(src + ck * 8 + 4);
-                const uint32_t r[8] = {lo.x, lo.y, lo.z, lo.w, hi.x, hi.y, hi.z, hi.w};
-                tmem_st_32x32b_x8(tmem + lane_base + qa_col + h * (p.Dp / 2) + ck * 8, r);
-            }
-            tmem_wait_st();
-            tc_fence_before();
-            __syncwarp();
-            if (lane == 0) mbar_arrive(&bars->qa_ready);
-        }
+            // ------------------------------------------------ exponent warps
+            const int quarter = warp & 3;
+            const int cg = warp >> 2;                  // column group: keys 32 cg .. 32 cg + 31
+            const uint32_t lane_base = static_cast<uint32_t>(quarter * 32) << 16;
+            const int row_t = quarter * 32 + lane;     // row inside each query tile
+            const int64_t row0 = static_cast<int64_t>(tile_m) * NQ * BM + row_t;
+            const int64_t row1 = row0 + BM;
 
-        // Row terms of the exponent (only without augmented operands).
-        const float am0 = AUG ? 0.f : p.A[row0];
-        const float am1 = AUG ? 0.f : p.A[row1];
-        const uint64_t a2_0 = f32x2_pack(am0, am0);
-        const uint64_t a2_1 = f32x2_pack(am1, am1);
-        const uint64_t c2 = f32x2_pack(p.c, p.c);
-        uint64_t acc0[C], acc1[C];
-#pragma unroll
-        for (int cc = 0; cc < C; ++cc) acc0[cc] = acc1[cc] = 0ull;
-        bool ok = true;
-        bool ready = false;   // both barriers of key tile j already seen complete
-        RingPos st, sl;       // stage and TMEM slot of key tile j
-        for (int j = 0; j < T; ++j, st.advance(p.stages), sl.advance(SL)) {
-            const int s = st.idx;
-            const uint32_t col0 = static_cast<uint32_t>(sl.idx * 2 * BN);
-            if (!__all_sync(0xffffffffu, ready || mbar_test_wait2(&bars->kv_full[s], st.phase,
-                                                                  &bars->s_full[sl.idx], sl.phase))) {
-                ok = warp_wait(&bars->kv_full[s], st.phase, abort_flag, p.status);
-                if (ok) ok = warp_wait(&bars->s_full[sl.idx], sl.phase, abort_flag, p.status);
-                if (!ok) break;
+            if (!QSM) {
+                // q^ rows -> TMEM (A operand).  Column group cg copies query tile
+                // cg / 2, 8-column chunks ck = cg % 2 (mod 2) of its Dp / 2 columns.
+                const int h = cg >> 1;
+                const uint32_t* src = p.qh + (row0 + h * BM) * (p.Dp / 2);
+                for (int ck = cg & 1; ck < p.Dp / 16; ck += 2) {
+                    const uint4 lo = *reinterpret_cast<const uint4*>(src + ck * 8);
+                    const uint4 hi = *reinterpret_cast<const uint4*>(src + ck * 8 + 4);
+                    const uint32_t r[8] = {lo.x, lo.y, lo.z, lo.w, hi.x, hi.y, hi.z, hi.w};
+                    tmem_st_32x32b_x8(tmem + lane_base + qa_col + h * (p.Dp / 2) + ck * 8, r);
+                }
+                tmem_wait_st();
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0) mbar_arrive(&bars->qa_ready);
             }
-            tc_fence_after();
-            uint32_t r0[32], r1[32];
-            tmem_ld_32x32b_x32(tmem + lane_base + col0 + cg * 32, r0);
-            tmem_ld_32x32b_x32(tmem + lane_base + col0 + BN + cg * 32, r1);
-            tmem_wait_ld();
-            // Both S slices are in registers: hand the slot back.
-            tc_fence_before();
-            __syncwarp();
-            if (lane == 0) mbar_arrive(&bars->s_free[sl.idx]);
-            // Query the barriers of key tile j + 1 now and read the answer
-            // after the exponent work of tile j: the query latency overlaps
-            // the arithmetic instead of stalling all exponent warps at once.
-            // A phase seen complete stays complete until this warp releases
-            // that stage and slot.
-            {
-                RingPos st2 = st, sl2 = sl;
-                st2.advance(p.stages);
-                sl2.advance(SL);
-                ready = j + 1 < T && mbar_test_wait2(&bars->kv_full[st2.idx], st2.phase,
-                                                     &bars->s_full[sl2.idx], sl2.phase);
-            }
-            const float* rec = rec_smem(s) + (cg * 16) * REC_PAIR;
-            if (AUG) {
-                // Augmented operands: S = -||q^ - k^||^2 / 2, so Phi = 2^(c S).
-                // Keys 32 cg + 2t and + 1, rows row0 (S0) and row1 (S1).
-#pragma unroll
+
+            // Row terms of the exponent (only without augmented operands).
+            const float am0 = AUG ? 0.f : p.A[row0];
+            const float am1 = AUG ? 0.f : p.A[row1];
+            const uint64_t a2_0 = f32x2_pack(am0, am0);
+            const uint64_t a2_1 = f32x2_pack(am1, am1);
+            const uint64_t c2 = f32x2_pack(p.c, p.c);
+            uint64_t acc0[C], acc1[C];
+    #pragma unroll
+            for (int cc = 0; cc < C; ++cc) acc0[cc] = acc1[cc] = 0ull;
+            bool ok = true;
+            bool ready = false;   // both barriers of key tile j already seen complete
+            RingPos st, sl;       // stage and TMEM slot of key tile j (running index g0 + j)
+            st.idx = g0 % p.stages;
+            st.phase = static_cast<uint32_t>(g0 / p.stages) & 1u;
+            sl.idx = g0 % SL;
+            sl.phase = static_cast<uint32_t>(g0 / SL) & 1u;
+            for (int j = 0; j < T; ++j, st.advance(p.stages), sl.advance(SL)) {
+                const int s = st.idx;
+                const uint32_t col0 = static_cast<uint32_t>(sl.idx * 2 * BN);
+                if (!__all_sync(0xffffffffu, ready || mbar_test_wait2(&bars->kv_full[s], st.phase,
+                                                                      &bars->s_full[sl.idx], sl.phase))) {
+                    ok = warp_wait(&bars->kv_full[s], st.phase, abort_flag, p.status);
+                    if (ok) ok = warp_wait(&bars->s_full[sl.idx], sl.phase, abort_flag, p.status);
+                    if (!ok) break;
+                }
+                tc_fence_after();
+                uint32_t r0[32], r1[32];
+                tmem_ld_32x32b_x32(tmem + lane_base + col0 + cg * 32, r0);
+                tmem_ld_32x32b_x32(tmem + lane_base + col0 + BN + cg * 32, r1);
+                tmem_wait_ld();
+                // Both S slices are in registers: hand the slot back.
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0) mbar_arrive(&bars->s_free[sl.idx]);
+                // Query the barriers of key tile j + 1 now and read the answer
+                // after the exponent work of tile j: the query latency overlaps
+                // the arithmetic instead of stalling all exponent warps at once.
+                // A phase seen complete stays complete until this warp releases
+                // that stage and slot.
+                {
+                    RingPos st2 = st, sl2 = sl;
+                    st2.advance(p.stages);
+                    sl2.advance(SL);
+                    ready = j + 1 < T && mbar_test_wait2(&bars->kv_full[st2.idx], st2.phase,
+                                                         &bars->s_full[sl2.idx], sl2.phase);
+                }
+                const float* rec = rec_smem(s) + (cg * 16) * REC_PAIR;
+                if (AUG) {
+                    // Augmented operands: S = -||q^ - k^||^2 / 2, so Phi = 2^(c S).
+                    // Keys 32 cg + 2t and + 1, rows row0 (S0) and row1 (S1).
+    #pragma unroll
+                    for (int t = 0; t < 16; ++t) {
+                        const float* pr = rec + t * REC_PAIR;
+                        float x0, x1, y0, y1;
+                        f32x2_unpack(f32x2_mul(f32x2_pack(__uint_as_float(r0[2 * t]), __uint_as_float(r0[2 * t + 1])), c2), x0, x1);
+                        f32x2_unpack(f32x2_mul(f32x2_pack(__uint_as_float(r1[2 * t]), __uint_as_float(r1[2 * t + 1])), c2), y0, y1);
+                        const uint64_t px = f32x2_pack(ex2_approx(x0), ex2_approx(x1));
+                        const uint64_t py = f32x2_pack(ex2_approx(y0), ex2_approx(y1));
+    #pragma unroll
+                        for (int cc = 0; cc < C; ++cc) {
+                            const float2 vc = *reinterpret_cast<const float2*>(pr + 2 * cc);
+                            const uint64_t vv = f32x2_pack(vc.x, vc.y);
+                            acc0[cc] = f32x2_fma(px, vv, acc0[cc]);
+                            acc1[cc] = f32x2_fma(py, vv, acc1[cc]);
+                        }
+                    }
+                } else {
+    #pragma unroll
                 for (int t = 0; t < 16; ++t) {
+                    // Keys 32 cg + 2t and + 1, rows row0 (S0) and row1 (S1).
                     const float* pr = rec + t * REC_PAIR;
+                    float2 bb, v0;
+                    if (C == 1) {
+                        const float4 bv = *reinterpret_cast<const float4*>(pr);
+                        bb = make_float2(bv.x, bv.y);
+                        v0 = make_float2(bv.z, bv.w);
+                    } else {
+                        bb = *reinterpret_cast<const float2*>(pr);
+                        v0 = *reinterpret_cast<const float2*>(pr + 2);
+                    }
+                    const uint64_t b2 = f32x2_pack(bb.x, bb.y);
+                    const uint64_t x01 = f32x2_fma(f32x2_pack(__uint_as_float(r0[2 * t]), __uint_as_float(r0[2 * t + 1])),
+                                                   c2, f32x2_add(b2, a2_0));
+                    const uint64_t y01 = f32x2_fma(f32x2_pack(__uint_as_float(r1[2 * t]), __uint_as_float(r1[2 * t + 1])),
+                                                   c2, f32x2_add(b2, a2_1));
                     float x0, x1, y0, y1;
-                    f32x2_unpack(f32x2_mul(f32x2_pack(__uint_as_float(r0[2 * t]), __uint_as_float(r0[2 * t + 1])), c2), x0, x1);
-                    f32x2_unpack(f32x2_mul(f32x2_pack(__uint_as_float(r1[2 * t]), __uint_as_float(r1[2 * t + 1])), c2), y0, y1);
+                    f32x2_unpack(x01, x0, x1);
+                    f32x2_unpack(y01, y0, y1);
                     const uint64_t px = f32x2_pack(ex2_approx(x0), ex2_approx(x1));
                     const uint64_t py = f32x2_pack(ex2_approx(y0), ex2_approx(y1));
-#pragma unroll
-                    for (int cc = 0; cc < C; ++cc) {
-                        const float2 vc = *reinterpret_cast<const float2*>(pr + 2 * cc);
+                    const uint64_t vv0 = f32x2_pack(v0.x, v0.y);
+                    acc0[0] = f32x2_fma(px, vv0, acc0[0]);
+                    acc1[0] = f32x2_fma(py, vv0, acc1[0]);
+    #pragma unroll
+                    for (int cc = 1; cc < C; ++cc) {
+                        const float2 vc = *reinterpret_cast<const float2*>(pr + 2 + 2 * cc);
                         const uint64_t vv = f32x2_pack(vc.x, vc.y);
                         acc0[cc] = f32x2_fma(px, vv, acc0[cc]);
                         acc1[cc] = f32x2_fma(py, vv, acc1[cc]);
                     }
                 }
-            } else {
-#pragma unroll
-            for (int t = 0; t < 16; ++t) {
-                // Keys 32 cg + 2t and + 1, rows row0 (S0) and row1 (S1).
-                const float* pr = rec + t * REC_PAIR;
-                float2 bb, v0;
-                if (C == 1) {
-                    const float4 bv = *reinterpret_cast<const float4*>(pr);
-                    bb = make_float2(bv.x, bv.y);
-                    v0 = make_float2(bv.z, bv.w);
-                } else {
-                    bb = *reinterpret_cast<const float2*>(pr);
-                    v0 = *reinterpret_cast<const float2*>(pr + 2);
                 }
-                const uint64_t b2 = f32x2_pack(bb.x, bb.y);
-                const uint64_t x01 = f32x2_fma(f32x2_pack(__uint_as_float(r0[2 * t]), __uint_as_float(r0[2 * t + 1])),
-                                               c2, f32x2_add(b2, a2_0));
-                const uint64_t y01 = f32x2_fma(f32x2_pack(__uint_as_float(r1[2 * t]), __uint_as_float(r1[2 * t + 1])),
-                                               c2, f32x2_add(b2, a2_1));
-                float x0, x1, y0, y1;
-                f32x2_unpack(x01, x0, x1);
-                f32x2_unpack(y01, y0, y1);
-                const uint64_t px = f32x2_pack(ex2_approx(x0), ex2_approx(x1));
-                const uint64_t py = f32x2_pack(ex2_approx(y0), ex2_approx(y1));
-                const uint64_t vv0 = f32x2_pack(v0.x, v0.y);
-                acc0[0] = f32x2_fma(px, vv0, acc0[0]);
-                acc1[0] = f32x2_fma(py, vv0, acc1[0]);
-#pragma unroll
-                for (int cc = 1; cc < C; ++cc) {
-                    const float2 vc = *reinterpret_cast<const float2*>(pr + 2 + 2 * cc);
-                    const uint64_t vv = f32x2_pack(vc.x, vc.y);
-                    acc0[cc] = f32x2_fma(px, vv, acc0[cc]);
-                    acc1[cc] = f32x2_fma(py, vv, acc1[cc]);
-                }
+                __syncwarp();
+                if (lane == 0) mbar_arrive(&bars->kv_empty[s]);
             }
-            }
-            __syncwarp();
-            if (lane == 0) mbar_arrive(&bars->kv_empty[s]);
-        }
-        // Fixed-order reduction of the NPART column-group partial sums.
-#pragma unroll
-        for (int cc = 0; cc < C; ++cc) {
-            float lo, hi;
-            f32x2_unpack(acc0[cc], lo, hi);
-            red[(cg * NQ * BM + row_t) * C + cc] = lo + hi;
-            f32x2_unpack(acc1[cc], lo, hi);
-            red[(cg * NQ * BM + BM + row_t) * C + cc] = lo + hi;
-        }
-        exp_warps_sync();
-        if (cg < NQ && T > 0 && *abort_flag == 0) {
-            // Column group cg writes the rows of query tile cg.
-            const int rt = cg * BM + row_t;
-            float* out = p.part + (static_cast<int64_t>(split) * p.Mpad + row0 + cg * BM) * C;
-#pragma unroll
+            // Fixed-order reduction of the NPART column-group partial sums.
+    #pragma unroll
             for (int cc = 0; cc < C; ++cc) {
-                float sum = 0.f;
-#pragma unroll
-                for (int q = 0; q < NPART; ++q) sum += red[(q * NQ * BM + rt) * C + cc];
-                out[cc] = sum;
+                float lo, hi;
+                f32x2_unpack(acc0[cc], lo, hi);
+                red[(cg * NQ * BM + row_t) * C + cc] = lo + hi;
+                f32x2_unpack(acc1[cc], lo, hi);
+                red[(cg * NQ * BM + BM + row_t) * C + cc] = lo + hi;
             }
+            exp_warps_sync();
+            if (cg < NQ && T > 0 && *abort_flag == 0) {
+                // Column group cg writes the rows of query tile cg.
+                const int rt = cg * BM + row_t;
+                float* out = p.part + (static_cast<int64_t>(slot) * p.Mpad + row0 + cg * BM) * C;
+    #pragma unroll
+                for (int cc = 0; cc < C; ++cc) {
+                    float sum = 0.f;
+    #pragma unroll
+                    for (int q = 0; q < NPART; ++q) sum += red[(q * NQ * BM + rt) * C + cc];
+                    out[cc] = sum;
+                }
+            }
+        // Segment end: every MMA, copy and TMEM read of this segment is done
+        // (control warps waited for their last stage release and copies).
+        segment_sync();
+        u += T;
         }
     }
 
@@ -470,7 +544,8 @@ cudaError_t launch_typed(const TcPlan& pl, InType t, float c, char* ws, unsigned
     p.status = status;
     p.Mpad = pl.Mpad;
     p.key_tiles = static_cast<int>(pl.Npad / BN);
-    p.tiles_per_split = (p.key_tiles + pl.splits - 1) / pl.splits;
+    p.units = static_cast<int>(pl.units);
+    p.unit_len = static_cast<int>(pl.unit_len);
     p.Dp = pl.Dp;
     p.nkb = (pl.Dp + KB - 1) / KB;
     p.stages = pl.stages;
@@ -486,7 +561,7 @@ cudaError_t launch_typed(const TcPlan& pl, InType t, float c, char* ws, unsigned
                                          cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          static_cast<int>(pl.smem_bytes));
     if (e != cudaSuccess) return e;
-    dim3 grid(static_cast<unsigned>(pl.Mpad / (NQ * BM)), static_cast<unsigned>(pl.splits));
+    dim3 grid(static_cast<unsigned>(pl.grid));
     tc_gauss_fma_kernel<C, AUG, QSM><<<grid, THREADS, pl.smem_bytes, s>>>(tm_q, tm_k, p);
     note_launches(1);
     return cudaGetLastError();
