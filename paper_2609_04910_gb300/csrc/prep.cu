@@ -327,6 +327,110 @@ __global__ void finalize_slots_kernel(const float* __restrict__ part, int64_t Mp
     out[idx] = acc;
 }
 
+// Vectorised variant of operand_kernel for D a multiple of 8: G lanes
+// (G = the power of two >= D / 8) share a row, each converting one 16-byte
+// vector of 8 coordinates straight from global memory to global memory;
+// the squared norm is reduced over the G lanes and the group's first lane
+// writes the columns past D (norm terms or zeros).  Same outputs as
+// operand_kernel.
+constexpr int kOperandVecThreads = 256;
+
+template <typename T> __device__ __forceinline__ T bits_to(unsigned short b);
+template <> __device__ __forceinline__ __half bits_to<__half>(unsigned short b) {
+    return __ushort_as_half(b);
+}
+template <> __device__ __forceinline__ __nv_bfloat16 bits_to<__nv_bfloat16>(unsigned short b) {
+    return __ushort_as_bfloat16(b);
+}
+template <typename T> __device__ __forceinline__ unsigned short to_bits(T h);
+template <> __device__ __forceinline__ unsigned short to_bits<__half>(__half h) {
+    return __half_as_ushort(h);
+}
+template <> __device__ __forceinline__ unsigned short to_bits<__nv_bfloat16>(__nv_bfloat16 h) {
+    return __bfloat16_as_ushort(h);
+}
+
+template <typename T, bool AUG, int G>
+__global__ void __launch_bounds__(kOperandVecThreads)
+operand_vec_kernel(const T* __restrict__ x, int64_t rows, int64_t rows_pad, int D, int Dp, int nt,
+                   float F, const float* __restrict__ mu, float half_c, float pad_value,
+                   T* __restrict__ out_q, T* __restrict__ out_k, float* __restrict__ nrm) {
+    const int vi = threadIdx.x % G;                              // vector within the row
+    const int64_t row = (static_cast<int64_t>(blockIdx.x) * kOperandVecThreads + threadIdx.x) / G;
+    const bool in_pad = row < rows_pad;
+    const bool valid = row < rows;
+    const int V = D / 8;
+    const bool wq = AUG ? out_q != nullptr : true;
+    const bool wk = AUG && out_k != nullptr;
+    float acc = 0.f;
+    if (in_pad && vi < V) {
+        uint4 u = make_uint4(0u, 0u, 0u, 0u);
+        if (valid) {
+            const uint4 in = *reinterpret_cast<const uint4*>(x + row * D + 8 * vi);
+            const unsigned short* hb = reinterpret_cast<const unsigned short*>(&in);
+            float m[8];
+            if (mu) {
+                const float4 m0 = *reinterpret_cast<const float4*>(mu + 8 * vi);
+                const float4 m1 = *reinterpret_cast<const float4*>(mu + 8 * vi + 4);
+                m[0] = m0.x; m[1] = m0.y; m[2] = m0.z; m[3] = m0.w;
+                m[4] = m1.x; m[5] = m1.y; m[6] = m1.z; m[7] = m1.w;
+            } else {
+#pragma unroll
+                for (int e = 0; e < 8; ++e) m[e] = 0.f;
+            }
+            __align__(16) unsigned short ob[8];
+#pragma unroll
+            for (int e = 0; e < 8; ++e) {
+                const T h = from_f<T>(to_f(bits_to<T>(hb[e])) - m[e]);
+                const float hf = to_f(h);
+                acc = fmaf(hf, hf, acc);
+                ob[e] = to_bits(h);
+            }
+            u = *reinterpret_cast<const uint4*>(ob);
+        }
+        if (wq) *reinterpret_cast<uint4*>(out_q + row * Dp + 8 * vi) = u;
+        if (wk) *reinterpret_cast<uint4*>(out_k + row * Dp + 8 * vi) = u;
+    }
+#pragma unroll
+    for (int o = G / 2; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o, G);
+    if (!in_pad || vi != 0) return;
+    if (!AUG) {
+        nrm[row] = valid ? -half_c * acc : pad_value;
+        for (int c = D; c < Dp; c += 8)
+            *reinterpret_cast<uint4*>(out_q + row * Dp + c) = make_uint4(0u, 0u, 0u, 0u);
+        return;
+    }
+    // Norm terms: a (or b) = -||x^||^2 / 2 = F t_0 + t_1 + ... (rounded
+    // remainders), partners F, 1, 1 on the other side.
+    __align__(16) unsigned short tq[16];
+    __align__(16) unsigned short tk[16];
+#pragma unroll
+    for (int e = 0; e < 16; ++e) tq[e] = tk[e] = 0;
+    if (valid) {
+        float r = -0.5f * acc;
+        for (int i = 0; i < nt; ++i) {
+            const T t = from_f<T>(i == 0 ? r / F : r);
+            r -= (i == 0 ? F : 1.f) * to_f(t);
+            const unsigned short one = to_bits(from_f<T>(i == 0 ? F : 1.f));
+            tq[i] = one;
+            tq[nt + i] = to_bits(t);
+            tk[i] = to_bits(t);
+            tk[nt + i] = one;
+        }
+    } else {
+        tk[0] = to_bits(from_f<T>(-30000.f / F));
+    }
+    for (int c = D, e0 = 0; c < Dp; c += 8, e0 += 8) {
+        uint4 uq = make_uint4(0u, 0u, 0u, 0u), uk = make_uint4(0u, 0u, 0u, 0u);
+        if (e0 < 16) {
+            uq = *reinterpret_cast<const uint4*>(tq + e0);
+            uk = *reinterpret_cast<const uint4*>(tk + e0);
+        }
+        if (wq) *reinterpret_cast<uint4*>(out_q + row * Dp + c) = uq;
+        if (wk) *reinterpret_cast<uint4*>(out_k + row * Dp + c) = uk;
+    }
+}
+
 template <typename T, bool AUG>
 cudaError_t operand_typed(const void* x, int64_t rows, int64_t rows_pad, int D, int Dp, int nt,
                           float F, const float* mu, float half_c, float pad_value, void* out_q,
@@ -334,6 +438,29 @@ cudaError_t operand_typed(const void* x, int64_t rows, int64_t rows_pad, int D, 
     if (rows_pad % kRowsPerBlock != 0 || Dp % 16 != 0 || Dp > kOperandMaxCols ||
         (AUG && 2 * Dp > kOperandMaxCols))
         return cudaErrorInvalidValue;
+    if (D % 8 == 0 && D >= 8 && (!AUG || Dp - D >= 2 * nt)) {
+        // Vector path: G lanes per row.
+        const int V = D / 8;
+        const int G = V <= 1 ? 1 : V <= 2 ? 2 : V <= 4 ? 4 : V <= 8 ? 8 : V <= 16 ? 16 : 32;
+        const int64_t threads = rows_pad * G;
+        const unsigned blocks = static_cast<unsigned>((threads + kOperandVecThreads - 1) / kOperandVecThreads);
+        auto go = [&](auto kern) {
+            kern<<<blocks, kOperandVecThreads, 0, s>>>(static_cast<const T*>(x), rows, rows_pad, D,
+                                                     Dp, nt, F, mu, half_c, pad_value,
+                                                     static_cast<T*>(out_q), static_cast<T*>(out_k),
+                                                     nrm);
+        };
+        switch (G) {
+            case 1: go(operand_vec_kernel<T, AUG, 1>); break;
+            case 2: go(operand_vec_kernel<T, AUG, 2>); break;
+            case 4: go(operand_vec_kernel<T, AUG, 4>); break;
+            case 8: go(operand_vec_kernel<T, AUG, 8>); break;
+            case 16: go(operand_vec_kernel<T, AUG, 16>); break;
+            default: go(operand_vec_kernel<T, AUG, 32>); break;
+        }
+        note_launches(1);
+        return cudaGetLastError();
+    }
     const int64_t blocks = rows_pad / kRowsPerBlock;
     if (blocks == 0) return cudaSuccess;
     const int nout = AUG ? (out_q ? 1 : 0) + (out_k ? 1 : 0) : 1;

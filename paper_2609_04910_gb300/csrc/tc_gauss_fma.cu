@@ -71,8 +71,8 @@ constexpr int MAX_STAGES = NCTRL_MAX;   // one stage per control warp
 constexpr bool kAugQsm = true;
 // Register split between the roles (setmaxnreg); the sum stays within the
 // registers the CTA is launched with (THREADS x 96).
-constexpr uint32_t kExpRegs = 104;
-constexpr uint32_t kCtrlRegs = 40;
+constexpr uint32_t kExpRegs = 112;
+constexpr uint32_t kCtrlRegs = 32;
 static_assert(NEXP * 32 * kExpRegs + NCTRL_MAX * 32 * kCtrlRegs <= THREADS * 96, "register split");
 
 struct FmaParams {
