@@ -66,8 +66,10 @@ typedef enum { GS_PATH_AUTO = 0, GS_PATH_TENSOR = 1, GS_PATH_SIMT = 2 } gs_path;
  *                     the MMA type (the overflow/cancellation safeguard of
  *                     Remark 2, Sec. 2); 0: use the raw points.
  *  split_n         number of key splits per row tile (0: chosen from the
- *                  SM count); partial sums over splits are added in a fixed
- *                  order, so results are deterministic for a fixed split.
+ *                  SM count; for C <= 4 one persistent block per SM takes an
+ *                  equal run of (row tile, key tile) pairs); partial sums
+ *                  over splits are added in a fixed order, so results are
+ *                  deterministic for a fixed split and GPU.
  *  workspace       caller-owned device buffer of workspace_bytes bytes
  *                  (256-byte aligned) used instead of an allocation; its
  *                  required size is gauss_sum_workspace_size().
@@ -128,8 +130,9 @@ size_t gauss_sum_workspace_size(int64_t M, int64_t N, int64_t D, int64_t C, gs_d
 /*
  * Synchronise `stream`, then return and clear the device status word of the
  * current device: GS_OK, or GS_ERR_DEVICE_TIMEOUT if a kernel gave up a
- * bounded wait since the last call (its outputs are then invalid), or
- * GS_ERR_CUDA if the synchronisation itself failed.
+ * bounded wait since the last call (its outputs are then invalid;
+ * gauss_sum_last_error() names the block, warp and barrier of the first
+ * wait that gave up), or GS_ERR_CUDA if the synchronisation itself failed.
  */
 gs_status gauss_sum_device_status(void* stream);
 
