@@ -92,11 +92,19 @@ __device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity, volati
     return __all_sync(0xffffffffu, ok);
 }
 
-// Threads of a CTA with NEXP exponent warps plus the producer and MMA warps.
+// Threads of a CTA with NEXP exponent warps plus one warpgroup holding the
+// producer and MMA warps (and two idle warps, so that the register split
+// below applies to whole warpgroups).
 template <int NEXP>
-constexpr int cta_threads() { return (NEXP + 2) * 32; }
+constexpr int cta_threads() { return (NEXP + 4) * 32; }
 
-template <int BN, int NEXP>
+// Register split for NEXP = 16 (launched with 640 x 96 registers).
+constexpr uint32_t kExpRegs2 = 112;
+constexpr uint32_t kCtrlRegs2 = 32;
+static_assert(16 * 32 * kExpRegs2 + 4 * 32 * kCtrlRegs2 <= 640 * 96, "register split");
+
+// AUG: augmented operands (S = -||q^ - k^||^2 / 2, no B records).
+template <int BN, int NEXP, bool AUG>
 __global__ void __launch_bounds__(cta_threads<NEXP>(), 1)
 tc_gauss_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
                 const __grid_constant__ CUtensorMap tm_v, const TcParams p) {
@@ -162,25 +170,35 @@ tc_gauss_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant_
     };
 
     if (warp == PRODUCER_WARP) {
-        if (lane == 0 && T > 0) {
-            tma_prefetch_desc(&tm_q);
-            tma_prefetch_desc(&tm_k);
-            tma_prefetch_desc(&tm_v);
-            mbar_arrive_expect_tx(&bars->q_full, static_cast<uint32_t>(p.nkb * BM * 128));
-            for (int kb = 0; kb < p.nkb; ++kb)
-                tma_load_2d(q_smem + kb * (BM * 128), &tm_q, &bars->q_full, kb * KB, tile_m * BM);
+        if (NEXP == 16) reg_dealloc<kCtrlRegs2>();
+        // The whole warp runs the loop (warp-uniform operands); the elected
+        // lane issues the copies.
+        if (T > 0) {
+            const bool leader = elect_one();
+            if (leader) {
+                tma_prefetch_desc(&tm_q);
+                tma_prefetch_desc(&tm_k);
+                tma_prefetch_desc(&tm_v);
+                mbar_arrive_expect_tx(&bars->q_full, static_cast<uint32_t>(p.nkb * BM * 128));
+                for (int kb = 0; kb < p.nkb; ++kb)
+                    tma_load_2d(q_smem + kb * (BM * 128), &tm_q, &bars->q_full, kb * KB, tile_m * BM);
+            }
+            __syncwarp();
             int issued = 0;
             RingPos st;
             for (int j = 0; j < T; ++j, st.advance(p.stages)) {
                 const int s = st.idx;
-                if (!mbar_wait_bounded(&bars->kv_empty[s], st.phase ^ 1u, abort_flag, p.status)) break;
-                mbar_arrive_expect_tx(&bars->kv_full[s], p.tx_bytes);
-                const int n0 = (kt0 + j) * BN;
-                for (int kb = 0; kb < p.nkb; ++kb)
-                    tma_load_2d(kh_smem(s) + kb * (BN * 128), &tm_k, &bars->kv_full[s], kb * KB, n0);
-                for (int h = 0; h < BN / KB; ++h)
-                    tma_load_2d(vt_smem(s) + h * (p.Cp * 128), &tm_v, &bars->kv_full[s], n0 + h * KB, 0);
-                bulk_load(const_cast<float*>(b_smem(s)), p.B + n0, BN * 4, &bars->kv_full[s]);
+                if (!warp_wait(&bars->kv_empty[s], st.phase ^ 1u, abort_flag, p.status)) break;
+                if (leader) {
+                    mbar_arrive_expect_tx(&bars->kv_full[s], p.tx_bytes);
+                    const int n0 = (kt0 + j) * BN;
+                    for (int kb = 0; kb < p.nkb; ++kb)
+                        tma_load_2d(kh_smem(s) + kb * (BN * 128), &tm_k, &bars->kv_full[s], kb * KB, n0);
+                    for (int h = 0; h < BN / KB; ++h)
+                        tma_load_2d(vt_smem(s) + h * (p.Cp * 128), &tm_v, &bars->kv_full[s], n0 + h * KB, 0);
+                    if (!AUG) bulk_load(const_cast<float*>(b_smem(s)), p.B + n0, BN * 4, &bars->kv_full[s]);
+                }
+                __syncwarp();
                 issued = j + 1;
             }
             // Let every copy this CTA started land before the CTA can exit.
@@ -188,53 +206,72 @@ tc_gauss_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant_
             for (int j = max(0, issued - p.stages); j < issued; ++j)
                 mbar_wait_bounded(&bars->kv_full[j % p.stages],
                                   static_cast<uint32_t>(j / p.stages) & 1u, nullptr, p.status);
+            __syncwarp();
         }
     } else if (warp == MMA_WARP) {
-        if (lane == 0 && T > 0) {
+        if (NEXP == 16) reg_dealloc<kCtrlRegs2>();
+        // The whole warp runs the loop (warp-uniform descriptors); the
+        // elected lane issues the MMAs and commits.
+        if (T > 0) {
+            const bool leader = elect_one();
             const uint32_t q_base = smem_u32(q_smem);
-            bool ok = mbar_wait_bounded(&bars->q_full, 0, abort_flag, p.status);
+            bool ok = warp_wait(&bars->q_full, 0, abort_flag, p.status);
             RingPos st, stp;   // stage of tile j (MMA1) and of tile j - 1 (MMA2)
             for (int j = 0; ok && j <= T; ++j) {
                 if (j < T) {
                     const int s = st.idx;
                     const int b = j & 1;
-                    ok = mbar_wait_bounded(&bars->kv_full[s], st.phase, abort_flag, p.status);
+                    ok = warp_wait(&bars->kv_full[s], st.phase, abort_flag, p.status);
                     if (!ok) break;
                     tc_fence_after();
                     const uint32_t kh_base = smem_u32(kh_smem(s));
-                    for (int kk = 0; kk < p.ksteps1; ++kk) {
-                        const uint32_t koff = static_cast<uint32_t>(kk & 3) * 32;
-                        const uint64_t ad = smem_desc_kmajor_sw128(q_base + (kk >> 2) * (BM * 128) + koff);
-                        const uint64_t bd = smem_desc_kmajor_sw128(kh_base + (kk >> 2) * (BN * 128) + koff);
-                        mma_ss_f16(tmem + S_col0 + b * BN, ad, bd, p.idesc1, kk > 0 ? 1u : 0u);
+                    if (leader) {
+                        for (int kk = 0; kk < p.ksteps1; ++kk) {
+                            const uint32_t koff = static_cast<uint32_t>(kk & 3) * 32;
+                            const uint64_t ad = smem_desc_kmajor_sw128(q_base + (kk >> 2) * (BM * 128) + koff);
+                            const uint64_t bd = smem_desc_kmajor_sw128(kh_base + (kk >> 2) * (BN * 128) + koff);
+                            mma_ss_f16(tmem + S_col0 + b * BN, ad, bd, p.idesc1, kk > 0 ? 1u : 0u);
+                        }
+                        mma_commit(&bars->s_full[b]);
                     }
-                    mma_commit(&bars->s_full[b]);
+                    __syncwarp();
                     st.advance(p.stages);
                 }
                 if (j >= 1) {
                     const int jp = j - 1;
                     const int bp = jp & 1;
                     const int sp = stp.idx;
-                    ok = mbar_wait_bounded(&bars->p_full[bp], static_cast<uint32_t>(jp >> 1) & 1u,
-                                           abort_flag, p.status);
+                    ok = warp_wait(&bars->p_full[bp], static_cast<uint32_t>(jp >> 1) & 1u,
+                                   abort_flag, p.status);
                     if (!ok) break;
                     tc_fence_after();
                     const uint32_t vt_base = smem_u32(vt_smem(sp));
-                    for (int kk = 0; kk < BN / 16; ++kk) {
-                        const uint64_t bd = smem_desc_kmajor_sw128(vt_base + (kk >> 2) * (p.Cp * 128) + (kk & 3) * 32);
-                        mma_ts_f16(tmem + O_col, tmem + P_col0 + bp * (BN / 2) + kk * 8, bd, p.idesc2,
-                                   (jp > 0 || kk > 0) ? 1u : 0u);
+                    if (leader) {
+                        for (int kk = 0; kk < BN / 16; ++kk) {
+                            const uint64_t bd = smem_desc_kmajor_sw128(vt_base + (kk >> 2) * (p.Cp * 128) + (kk & 3) * 32);
+                            mma_ts_f16(tmem + O_col, tmem + P_col0 + bp * (BN / 2) + kk * 8, bd, p.idesc2,
+                                       (jp > 0 || kk > 0) ? 1u : 0u);
+                        }
+                        mma_commit(&bars->kv_empty[sp]);
                     }
-                    mma_commit(&bars->kv_empty[sp]);
+                    __syncwarp();
                     stp.advance(p.stages);
                 }
             }
-            if (ok) mma_commit(&bars->o_full);
-            // No MMA may still be running when TMEM is released.
-            mma_commit(&bars->drain);
+            if (leader) {
+                if (ok) mma_commit(&bars->o_full);
+                // No MMA may still be running when TMEM is released.
+                mma_commit(&bars->drain);
+            }
+            __syncwarp();
             mbar_wait_bounded(&bars->drain, 0, nullptr, p.status);
+            __syncwarp();
         }
+    } else if (warp > MMA_WARP) {
+        // Idle warps completing the control warpgroup.
+        if (NEXP == 16) reg_dealloc<kCtrlRegs2>();
     } else {
+        if (NEXP == 16) reg_alloc<kExpRegs2>();
         // ------------------------------------------------ exponent warps
         // Warp w of group g = w / GROUP_WARPS reads TMEM lanes 32 (w % 4) ..
         // +31 (rows of the tile) and key columns [COLS part, COLS (part + 1))
@@ -245,7 +282,7 @@ tc_gauss_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant_
         const int col0 = part * COLS;
         const int row_local = quarter * 32 + lane;
         const int64_t row = static_cast<int64_t>(tile_m) * BM + row_local;
-        const float a_m = p.A[row] + P_SHIFT;
+        const float a_m = (AUG ? 0.f : p.A[row]) + P_SHIFT;
         const uint64_t a2 = f32x2_pack(a_m, a_m);
         const uint64_t c2 = f32x2_pack(p.c, p.c);
         const uint32_t lane_base = static_cast<uint32_t>(quarter * 32) << 16;
@@ -271,10 +308,15 @@ tc_gauss_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant_
                 uint32_t pk[16];
 #pragma unroll
                 for (int i = 0; i < 8; ++i) {
-                    // x = c S + (A_m + 15) + B_n for four keys, two per f32x2 op.
-                    const float4 bb = *reinterpret_cast<const float4*>(Bs + ch * 32 + 4 * i);
-                    const uint64_t t01 = f32x2_add(f32x2_pack(bb.x, bb.y), a2);
-                    const uint64_t t23 = f32x2_add(f32x2_pack(bb.z, bb.w), a2);
+                    // x = c S + (A_m + 15) + B_n for four keys, two per f32x2
+                    // op (with augmented operands S already holds the norm
+                    // terms: x = c S + 15).
+                    uint64_t t01 = a2, t23 = a2;
+                    if (!AUG) {
+                        const float4 bb = *reinterpret_cast<const float4*>(Bs + ch * 32 + 4 * i);
+                        t01 = f32x2_add(f32x2_pack(bb.x, bb.y), a2);
+                        t23 = f32x2_add(f32x2_pack(bb.z, bb.w), a2);
+                    }
                     const uint64_t s01 = f32x2_pack(__uint_as_float(r[ch][4 * i + 0]),
                                                     __uint_as_float(r[ch][4 * i + 1]));
                     const uint64_t s23 = f32x2_pack(__uint_as_float(r[ch][4 * i + 2]),
@@ -322,7 +364,7 @@ tc_gauss_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant_
 // ---------------------------------------------------------------- host side
 size_t align1k(size_t x) { return (x + 1023) & ~static_cast<size_t>(1023); }
 
-template <int BN, int NEXP>
+template <int BN, int NEXP, bool AUG>
 cudaError_t launch_bn(const TcPlan& pl, InType t, float c, char* ws, unsigned* status,
                       cudaStream_t s, const char** why) {
     const CUtensorMapDataType hdt =
@@ -336,8 +378,8 @@ cudaError_t launch_bn(const TcPlan& pl, InType t, float c, char* ws, unsigned* s
         return cudaErrorInvalidValue;
     }
     TcParams p;
-    p.A = reinterpret_cast<const float*>(ws + pl.off_A);
-    p.B = reinterpret_cast<const float*>(ws + pl.off_B);
+    p.A = AUG ? nullptr : reinterpret_cast<const float*>(ws + pl.off_A);
+    p.B = AUG ? nullptr : reinterpret_cast<const float*>(ws + pl.off_B);
     p.part = reinterpret_cast<float*>(ws + pl.off_part);
     p.status = status;
     p.Mpad = pl.Mpad;
@@ -349,20 +391,20 @@ cudaError_t launch_bn(const TcPlan& pl, InType t, float c, char* ws, unsigned* s
     p.stages = pl.stages;
     p.kh_bytes = static_cast<uint32_t>(p.nkb * BN * 128);
     p.vt_bytes = static_cast<uint32_t>((BN / KB) * pl.Cp * 128);
-    p.tx_bytes = p.kh_bytes + p.vt_bytes + BN * 4;
-    p.stage_bytes = static_cast<uint32_t>(align1k(p.tx_bytes));
+    p.tx_bytes = p.kh_bytes + p.vt_bytes + (AUG ? 0 : BN * 4);
+    p.stage_bytes = static_cast<uint32_t>(align1k(p.kh_bytes + p.vt_bytes + BN * 4));
     p.c = c;
     const uint32_t hb = t == InType::BF16 ? 1u : 0u;
     p.idesc1 = idesc_f16(BM, BN, hb, hb);
     p.idesc2 = idesc_f16(BM, static_cast<uint32_t>(pl.Cp), 0u, 0u);
 
     // Per-device function attribute; cheap enough to set on every launch.
-    cudaError_t e = cudaFuncSetAttribute(tc_gauss_kernel<BN, NEXP>,
+    cudaError_t e = cudaFuncSetAttribute(tc_gauss_kernel<BN, NEXP, AUG>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          static_cast<int>(pl.smem_bytes));
     if (e != cudaSuccess) return e;
     dim3 grid(static_cast<unsigned>(pl.Mpad / BM), static_cast<unsigned>(pl.splits));
-    tc_gauss_kernel<BN, NEXP><<<grid, cta_threads<NEXP>(), pl.smem_bytes, s>>>(tm_q, tm_k, tm_v, p);
+    tc_gauss_kernel<BN, NEXP, AUG><<<grid, cta_threads<NEXP>(), pl.smem_bytes, s>>>(tm_q, tm_k, tm_v, p);
     note_launches(1);
     return cudaGetLastError();
 }
@@ -400,6 +442,14 @@ bool plan_tensor(InType t, int64_t M, int64_t N, int64_t D, int64_t C, bool grad
         p->stages = fma_stages;
         p->smem_bytes = fma_smem;
     } else {
+        // Two-MMA kernel: augmented operands when the extra MMA work stays
+        // small next to the exponentials (the norm terms then cost the
+        // exponent warps nothing).
+        if (dp_aug + p->Cp <= 128) {
+            p->aug = true;
+            p->Dp = dp_aug;
+        }
+        const int nkb = (p->Dp + KB - 1) / KB;
         p->BN = p->Cp <= 128 ? 128 : 64;
         p->nq = 1;
         const size_t stage = align1k(static_cast<size_t>(nkb) * p->BN * 128 +
@@ -496,8 +546,12 @@ bool plan_tensor(InType t, int64_t M, int64_t N, int64_t D, int64_t C, bool grad
 
 cudaError_t launch_tc(const TcPlan& p, InType t, float c, char* ws, unsigned* status,
                       cudaStream_t s, const char** why) {
-    if (p.BN == 128) return launch_bn<128, 16>(p, t, c, ws, status, s, why);
-    return launch_bn<64, 8>(p, t, c, ws, status, s, why);
+    if (p.aug) {
+        if (p.BN == 128) return launch_bn<128, 16, true>(p, t, c, ws, status, s, why);
+        return launch_bn<64, 8, true>(p, t, c, ws, status, s, why);
+    }
+    if (p.BN == 128) return launch_bn<128, 16, false>(p, t, c, ws, status, s, why);
+    return launch_bn<64, 8, false>(p, t, c, ws, status, s, why);
 }
 
 }  // namespace gs
