@@ -292,9 +292,13 @@ tc_gauss_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant_
         for (int j = group; j < T; j += 2, st.advance(p.stages), st.advance(p.stages)) {
             const int b = group;
             const int s = st.idx;
-            ok = warp_wait(&bars->kv_full[s], st.phase, abort_flag, p.status);
-            if (ok) ok = warp_wait(&bars->s_full[b], static_cast<uint32_t>(j >> 1) & 1u, abort_flag,
-                                   p.status);
+            // The B records of the stage are only read without augmented
+            // operands; S itself is ordered by s_full.
+            if (!AUG) ok = warp_wait(&bars->kv_full[s], st.phase, abort_flag, p.status);
+            if (ok && !__all_sync(0xffffffffu, mbar_test_wait(&bars->s_full[b],
+                                                               static_cast<uint32_t>(j >> 1) & 1u)))
+                ok = warp_wait(&bars->s_full[b], static_cast<uint32_t>(j >> 1) & 1u, abort_flag,
+                               p.status);
             if (!ok) break;
             tc_fence_after();
             uint32_t r[NCH][32];
