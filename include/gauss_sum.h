@@ -128,6 +128,34 @@ size_t gauss_sum_workspace_size(int64_t M, int64_t N, int64_t D, int64_t C, gs_d
                                 int grad, const gs_options* opt);
 
 /*
+ * A batch of B independent problems of Eq. 1 with equal sizes (the paper
+ * benchmarks batches of independent point clouds, Sec. 4), stored
+ * contiguously: q is B x M x D, k is B x N x D, v is B x N x C and out is
+ * B x M x C (float32).  Problem b uses only its own points; centring (the
+ * shift of Remark 2) is per problem.  Default options.  For C <= 4 (fp16 /
+ * bf16) the whole batch runs in one launch of each kernel; otherwise the
+ * problems run one after another on `stream`, and every problem's q, k, v
+ * and out must then start 16-byte aligned (GS_ERR_INVALID_ARGUMENT
+ * otherwise).  B = 0 is a no-op.
+ */
+gs_status gauss_sum_batched(const void* q, const void* k, const void* v, double tau, int64_t B,
+                            int64_t M, int64_t N, int64_t D, int64_t C, gs_dtype dtype, float* out,
+                            void* stream);
+
+/*
+ * Squared maximum mean discrepancy of Sec. 3 for B problems: for points
+ * x (B x N x D) carrying the signed weights v (B x N) of the difference of
+ * two discrete measures,
+ *     mmd2[b] = sum_{m,n} v[b,m] Phi(x[b,m], x[b,n]) v[b,n] = v_b^T s_b,
+ * with s_b the Gauss sum of Eq. 1 for q = k = x_b and C = 1.  mmd2 is a
+ * device array of B floats (16-byte aligned); the final sum over m runs in
+ * float64 in a fixed order.  Allocates B x N floats on `stream`
+ * (cudaMallocAsync) besides the Gauss sum's workspace.
+ */
+gs_status gauss_sum_mmd2(const void* x, const void* v, double tau, int64_t B, int64_t N,
+                         int64_t D, gs_dtype dtype, float* mmd2, void* stream);
+
+/*
  * Synchronise `stream`, then return and clear the device status word of the
  * current device: GS_OK, or GS_ERR_DEVICE_TIMEOUT if a kernel gave up a
  * bounded wait since the last call (its outputs are then invalid;

@@ -160,3 +160,15 @@ def oracle_grad_q(q, k, v, tau, rows=None, nthreads=None, lib_path=None):
     if rc != 0:
         raise ValueError("gs_oracle_grad_q rejected its arguments")
     return g, s, den, dsh
+
+
+def oracle_mmd2(x, v, tau, nthreads=None, lib_path=None):
+    """Squared MMD of Sec. 3 (Maximum mean discrepancy) for the signed
+    measure sum_n v_n delta_{x_n}: sum_m v_m s_m with s the Gauss sum of
+    Eq. 1 for q = k = x and C = 1.  Returns (mmd2, den) with
+    den = sum_m |v_m| sum_n Phi(x_m, x_n) |v_n|, the error scale of a
+    computed s carried through the weighted sum.  x: (N, D), v: (N,)."""
+    x = np.asarray(x, dtype=np.float64)
+    v = np.asarray(v, dtype=np.float64).reshape(-1)
+    s, den = oracle_sum(x, x, v.reshape(-1, 1), tau, nthreads=nthreads, lib_path=lib_path)
+    return float(np.dot(v, s[:, 0])), float(np.dot(np.abs(v), den[:, 0]))

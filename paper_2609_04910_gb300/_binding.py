@@ -25,7 +25,7 @@ EXPORTS = (
     "gauss_sum_default_options", "gauss_sum", "gauss_sum_ex", "gauss_sum_grad_q",
     "gauss_sum_grad_q_ex", "gauss_sum_workspace_size", "gauss_sum_device_status",
     "gauss_sum_last_error", "gauss_sum_status_string", "gauss_sum_probe_ex2_rate",
-    "gauss_sum_noalloc", "gauss_sum_kernel_launches",
+    "gauss_sum_noalloc", "gauss_sum_kernel_launches", "gauss_sum_batched", "gauss_sum_mmd2",
 )
 
 # Bytes of the static scratch array behind gauss_sum_noalloc
@@ -101,6 +101,10 @@ def _declare(lib):
     lib.gauss_sum_noalloc.restype = f
     lib.gauss_sum_kernel_launches.argtypes = []
     lib.gauss_sum_kernel_launches.restype = ctypes.c_uint64
+    lib.gauss_sum_batched.argtypes = [vp, vp, vp, d, i64, i64, i64, i64, i64, f, vp, vp]
+    lib.gauss_sum_batched.restype = f
+    lib.gauss_sum_mmd2.argtypes = [vp, vp, d, i64, i64, i64, f, vp, vp]
+    lib.gauss_sum_mmd2.restype = f
 
 
 def _check(lib, status: int):
@@ -177,6 +181,45 @@ def gauss_sum(q, k, v, tau, out=None, stream=None, center=True, split_n=0, works
                   main_events=main_events)
     st = lib.gauss_sum_ex(_ptr(q), _ptr(k), _ptr(v), float(tau), M, N, D, C, _dtype_code(q),
                           _ptr(out), _stream_ptr(stream), ctypes.byref(opt))
+    _check(lib, st)
+    return out
+
+
+def gauss_sum_batched(q, k, v, tau, out=None, stream=None):
+    """A batch of independent problems of Eq. 1: q (B, M, D), k (B, N, D),
+    v (B, N, C) or (B, N) CUDA tensors of one dtype; returns (B, M, C)
+    fp32.  ``q`` may be the same tensor as ``k``."""
+    import torch
+    lib = load_library()
+    for t, n in ((q, "q"), (k, "k"), (v, "v")):
+        _check_tensor(t, n)
+    B, M, D = q.shape
+    N = k.shape[1]
+    C = 1 if v.dim() == 2 else v.shape[2]
+    if out is None:
+        out = torch.empty((B, M, C), dtype=torch.float32, device=q.device)
+    st = lib.gauss_sum_batched(_ptr(q), _ptr(k), _ptr(v), float(tau), B, M, N, D, C,
+                               _dtype_code(q), _ptr(out), _stream_ptr(stream))
+    _check(lib, st)
+    return out
+
+
+def gauss_sum_mmd2(x, v, tau, out=None, stream=None):
+    """Squared MMD of Sec. 3: x (B, N, D) or (N, D) points with signed
+    weights v (B, N) or (N,); returns (B,) fp32 (a 1-element tensor for
+    unbatched input) with mmd2[b] = v_b^T K(x_b, x_b) v_b."""
+    import torch
+    lib = load_library()
+    for t, n in ((x, "x"), (v, "v")):
+        _check_tensor(t, n)
+    if x.dim() == 2:
+        B, (N, D) = 1, x.shape
+    else:
+        B, N, D = x.shape
+    if out is None:
+        out = torch.empty((B,), dtype=torch.float32, device=x.device)
+    st = lib.gauss_sum_mmd2(_ptr(x), _ptr(v), float(tau), B, N, D, _dtype_code(x), _ptr(out),
+                            _stream_ptr(stream))
     _check(lib, st)
     return out
 

@@ -78,21 +78,23 @@ struct Call {
     float* s_out;  // grad only, nullable
     cudaStream_t stream;
     gs_options opt;
+    int64_t B = 1;  // problems of a batch: q B x M x D, k B x N x D, v B x N x C, out B x M x ..
 };
 
 gs_status validate(const Call& c) {
     if (c.dtype != GS_FP32 && c.dtype != GS_FP16 && c.dtype != GS_BF16)
         return fail(GS_ERR_INVALID_ARGUMENT, "unknown dtype");
-    if (c.M < 0 || c.N < 0 || c.D < 0 || c.C < 0)
+    if (c.M < 0 || c.N < 0 || c.D < 0 || c.C < 0 || c.B < 0)
         return fail(GS_ERR_INVALID_ARGUMENT, "negative size");
     if (!(std::isfinite(c.tau) && c.tau > 0.0))
         return fail(GS_ERR_INVALID_ARGUMENT, "tau must be finite and > 0");
     if (c.grad && c.C != 1) return fail(GS_ERR_INVALID_ARGUMENT, "the q-gradient needs C = 1");
     const int64_t out_w = c.grad ? c.D : c.C;
-    if (c.M > 0 && out_w > 0 && !c.out) return fail(GS_ERR_INVALID_ARGUMENT, "null output pointer");
-    if (c.M > 0 && c.D > 0 && !c.q) return fail(GS_ERR_INVALID_ARGUMENT, "null q pointer");
-    if (c.N > 0 && c.D > 0 && !c.k) return fail(GS_ERR_INVALID_ARGUMENT, "null k pointer");
-    if (c.N > 0 && c.C > 0 && !c.v) return fail(GS_ERR_INVALID_ARGUMENT, "null v pointer");
+    const bool any = c.B > 0;   // an empty batch reads and writes nothing
+    if (any && c.M > 0 && out_w > 0 && !c.out) return fail(GS_ERR_INVALID_ARGUMENT, "null output pointer");
+    if (any && c.M > 0 && c.D > 0 && !c.q) return fail(GS_ERR_INVALID_ARGUMENT, "null q pointer");
+    if (any && c.N > 0 && c.D > 0 && !c.k) return fail(GS_ERR_INVALID_ARGUMENT, "null k pointer");
+    if (any && c.N > 0 && c.C > 0 && !c.v) return fail(GS_ERR_INVALID_ARGUMENT, "null v pointer");
     if (!aligned16(c.q) || !aligned16(c.k) || !aligned16(c.v) || !aligned16(c.out) ||
         !aligned16(c.s_out))
         return fail(GS_ERR_INVALID_ARGUMENT, "base pointers must be 16-byte aligned");
@@ -119,7 +121,7 @@ gs_status plan(const Call& c, int sms, bool* tensor, gs::TcPlan* tp, gs::SimtPla
     if (*tensor) {
         const bool alias = c.q == c.k && c.M == c.N && c.q != nullptr;
         if (!gs::plan_tensor(in_type(c.dtype), c.M, c.N, c.D, c.C, c.grad, c.opt.center != 0,
-                             alias, c.opt.split_n, sms, tp, &why))
+                             alias, c.opt.split_n, sms, tp, &why, c.B))
             return fail(GS_ERR_UNSUPPORTED, "%s", why);
         *bytes = tp->total;
     } else {
@@ -143,7 +145,7 @@ bool forced_alloc_failure() {
 gs_status run(Call c) {
     gs_status st = validate(c);
     if (st != GS_OK) return st;
-    if (c.M == 0) return GS_OK;
+    if (c.M == 0 || c.B == 0) return GS_OK;
     if (c.grad && c.D == 0) {
         // No coordinates: the gradient is empty and s is the plain forward sum.
         if (!c.s_out) return GS_OK;
@@ -156,9 +158,9 @@ gs_status run(Call c) {
 
     if (c.N == 0) {
         cudaError_t e = cudaSuccess;
-        if (out_w > 0) e = cudaMemsetAsync(c.out, 0, sizeof(float) * c.M * out_w, c.stream);
+        if (out_w > 0) e = cudaMemsetAsync(c.out, 0, sizeof(float) * c.B * c.M * out_w, c.stream);
         if (e == cudaSuccess && c.grad && c.s_out)
-            e = cudaMemsetAsync(c.s_out, 0, sizeof(float) * c.M, c.stream);
+            e = cudaMemsetAsync(c.s_out, 0, sizeof(float) * c.B * c.M, c.stream);
         return e == cudaSuccess ? GS_OK : cuda_fail(e, "cudaMemsetAsync");
     }
 
@@ -176,6 +178,25 @@ gs_status run(Call c) {
     size_t bytes = 0;
     st = plan(c, g_sm_count[dev], &tensor, &tp, &sp, &bytes);
     if (st != GS_OK) return st;
+    if (c.B > 1 && !(tensor && tp.fma)) {
+        // Only the FMA kernel takes a batch in one launch: the problems of a
+        // batch run one after another on the stream.
+        const int64_t es = c.dtype == GS_FP32 ? 4 : 2;
+        const int64_t out_w1 = c.grad ? c.D : c.C;
+        for (int64_t b = 0; b < c.B; ++b) {
+            Call cb = c;
+            cb.B = 1;
+            cb.q = static_cast<const char*>(c.q) + b * c.M * c.D * es;
+            cb.k = static_cast<const char*>(c.k) + b * c.N * c.D * es;
+            cb.v = static_cast<const char*>(c.v) + b * c.N * c.C * es;
+            cb.out = c.out + b * c.M * out_w1;
+            if (c.s_out) cb.s_out = c.s_out + b * c.M;
+            st = run(cb);
+            if (st != GS_OK) return st;
+        }
+        return GS_OK;
+    }
+    const int batch = static_cast<int>(tp.batch > 0 ? tp.batch : 1);
 
     char* ws = static_cast<char*>(c.opt.workspace);
     bool owned = false;
@@ -200,18 +221,20 @@ gs_status run(Call c) {
         if (tp.center && c.D > 0) {
             mu = reinterpret_cast<float*>(ws + tp.off_mu);
             e = gs::launch_mean(t, c.q, c.k, c.M, c.N, static_cast<int>(c.D), tp.mean_blocks,
-                                reinterpret_cast<float*>(ws + tp.off_mean_part), mu, c.stream);
+                                reinterpret_cast<float*>(ws + tp.off_mean_part), mu, c.stream,
+                                batch);
             where = "mean kernel";
         }
         const float ninf = -INFINITY;
         if (e == cudaSuccess && tp.aug) {
             // Augmented operands: centred points with the norms folded in.
             e = gs::launch_aug_prep(t, c.q, c.M, tp.Mpad, static_cast<int>(c.D), tp.Dp, mu,
-                                    ws + tp.off_qh, tp.alias ? ws + tp.off_kh : nullptr, c.stream);
+                                    ws + tp.off_qh, tp.alias ? ws + tp.off_kh : nullptr, c.stream,
+                                    batch);
             where = "augmented-operand kernel (q)";
             if (e == cudaSuccess && !tp.alias) {
                 e = gs::launch_aug_prep(t, c.k, c.N, tp.Npad, static_cast<int>(c.D), tp.Dp, mu,
-                                        nullptr, ws + tp.off_kh, c.stream);
+                                        nullptr, ws + tp.off_kh, c.stream, batch);
                 where = "augmented-operand kernel (k)";
             }
         } else {
@@ -219,14 +242,14 @@ gs_status run(Call c) {
                 e = gs::launch_center_cast_norm(t, c.q, c.M, tp.Mpad, static_cast<int>(c.D), tp.Dp,
                                                 mu, half_c, ws + tp.off_qh,
                                                 reinterpret_cast<float*>(ws + tp.off_A), ninf,
-                                                c.stream);
+                                                c.stream, batch);
                 where = "centre/cast kernel (q)";
             }
             if (e == cudaSuccess && !tp.alias) {
                 e = gs::launch_center_cast_norm(t, c.k, c.N, tp.Npad, static_cast<int>(c.D), tp.Dp,
                                                 mu, half_c, ws + tp.off_kh,
                                                 reinterpret_cast<float*>(ws + tp.off_B), ninf,
-                                                c.stream);
+                                                c.stream, batch);
                 where = "centre/cast kernel (k)";
             }
         }
@@ -234,7 +257,7 @@ gs_status run(Call c) {
             e = gs::launch_key_records(
                 t, c.v, tp.aug ? nullptr : reinterpret_cast<const float*>(ws + tp.off_B), c.N,
                 tp.Npad, static_cast<int>(tp.Cv), reinterpret_cast<float*>(ws + tp.off_rec),
-                c.stream);
+                c.stream, batch);
             where = "key-record kernel";
         } else if (e == cudaSuccess) {
             e = gs::launch_value_prep(t, c.grad, c.v, c.k, mu, c.N, tp.Npad, static_cast<int>(c.D),
@@ -256,7 +279,7 @@ gs_status run(Call c) {
                 e = gs::launch_finalize_slots(reinterpret_cast<float*>(ws + tp.off_part), tp.Mpad,
                                               c.M, static_cast<int>(tp.Cv),
                                               128 * tp.nq, tp.Npad / tp.BN, tp.unit_len, c.out,
-                                              c.stream);
+                                              c.stream, batch);
             else
                 e = gs::launch_finalize(c.grad ? 1 : 0, t,
                                         reinterpret_cast<float*>(ws + tp.off_part), tp.splits,
@@ -400,6 +423,47 @@ gs_status gauss_sum_ex(const void* q, const void* k, const void* v, double tau, 
 gs_status gauss_sum(const void* q, const void* k, const void* v, double tau, int64_t M,
                     int64_t N, int64_t D, int64_t C, gs_dtype dtype, float* out, void* stream) {
     return gauss_sum_ex(q, k, v, tau, M, N, D, C, dtype, out, stream, nullptr);
+}
+
+gs_status gauss_sum_batched(const void* q, const void* k, const void* v, double tau, int64_t B,
+                            int64_t M, int64_t N, int64_t D, int64_t C, gs_dtype dtype, float* out,
+                            void* stream) {
+    Call c{q, k, v, tau, M, N, D, C, dtype, false, out, nullptr,
+           static_cast<cudaStream_t>(stream), defaults()};
+    c.B = B;
+    return run(c);
+}
+
+gs_status gauss_sum_mmd2(const void* x, const void* v, double tau, int64_t B, int64_t N,
+                         int64_t D, gs_dtype dtype, float* mmd2, void* stream) {
+    const cudaStream_t st = static_cast<cudaStream_t>(stream);
+    if (B < 0 || N < 0 || D < 0) return fail(GS_ERR_INVALID_ARGUMENT, "negative size");
+    if (B > 0 && !mmd2) return fail(GS_ERR_INVALID_ARGUMENT, "null output pointer");
+    if (!aligned16(mmd2)) return fail(GS_ERR_INVALID_ARGUMENT, "base pointers must be 16-byte aligned");
+    if (B == 0) return GS_OK;
+    if (N == 0) {
+        cudaError_t e = cudaMemsetAsync(mmd2, 0, sizeof(float) * B, st);
+        return e == cudaSuccess ? GS_OK : cuda_fail(e, "cudaMemsetAsync");
+    }
+    // s = K v for every problem (q = k = x), then v^T s.  The arguments are
+    // validated with mmd2 standing in for the s buffer allocated below.
+    Call c{x, x, v, tau, N, N, D, 1, dtype, false, mmd2, nullptr, st, defaults()};
+    c.B = B;
+    gs_status status = validate(c);
+    if (status != GS_OK) return status;
+    if (forced_alloc_failure()) return fail(GS_ERR_OUT_OF_MEMORY, "workspace allocation failed (test hook)");
+    float* s_buf = nullptr;
+    cudaError_t e = cudaMallocAsync(reinterpret_cast<void**>(&s_buf), sizeof(float) * B * N, st);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaMallocAsync");
+    c.out = s_buf;
+    status = run(c);
+    if (status == GS_OK) {
+        e = gs::launch_mmd2_reduce(in_type(dtype), s_buf, v, B, N, mmd2, st);
+        if (e != cudaSuccess) status = cuda_fail(e, "MMD reduction kernel");
+    }
+    cudaError_t ef = cudaFreeAsync(s_buf, st);
+    if (status == GS_OK && ef != cudaSuccess) return cuda_fail(ef, "cudaFreeAsync");
+    return status;
 }
 
 gs_status gauss_sum_grad_q_ex(const void* q, const void* k, const void* v, double tau,

@@ -38,6 +38,9 @@ struct TcPlan {
     // CTA (`splits` = the largest number of contributors).
     int64_t units, unit_len;
     int grid;
+    // Problems of a batch handled by one launch (the FMA kernel stacks them:
+    // q^ batch x Mpad rows, k^ batch x Npad rows); 1 for the other paths.
+    int64_t batch;
     size_t off_mean_part, off_mu, off_qh, off_kh, off_A, off_B, off_vt, off_vmax, off_inv,
         off_rec, off_part, total;
 };
@@ -55,29 +58,34 @@ int device_sm_count(int device);
 bool device_is_sm103(int device);
 
 bool plan_tensor(InType t, int64_t M, int64_t N, int64_t D, int64_t C, bool grad, bool center,
-                 bool alias, int split_override, int sms, TcPlan* p, const char** why);
+                 bool alias, int split_override, int sms, TcPlan* p, const char** why,
+                 int64_t batch = 1);
 bool plan_simt(int64_t M, int64_t N, int64_t D, int64_t C, bool grad, int split_override,
                int sms, SimtPlan* p, const char** why);
 
 // prep.cu --------------------------------------------------------------
 cudaError_t launch_mean(InType t, const void* q, const void* k, int64_t M, int64_t N, int D,
-                        int blocks, float* partial, float* mu, cudaStream_t s);
+                        int blocks, float* partial, float* mu, cudaStream_t s, int batch = 1);
 cudaError_t launch_center_cast_norm(InType t, const void* x, int64_t rows, int64_t rows_pad,
                                     int D, int Dp, const float* mu, float half_c, void* xh,
-                                    float* nrm, float pad_value, cudaStream_t s);
+                                    float* nrm, float pad_value, cudaStream_t s, int batch = 1);
 cudaError_t launch_value_prep(InType t, bool grad, const void* v, const void* k,
                               const float* mu, int64_t N, int64_t Npad, int D, int Cv, int Cp,
                               unsigned* vmax_bits, void* vt, float* inv_scale, cudaStream_t s);
 // mode 0: forward (out M x Cv, scaled by inv_scale when given)
 // mode 1: gradient from augmented values (tensor path): needs q, mu, tau
 // mode 2: gradient from direct partials (SIMT path): Cv = D + 1
+// MMD^2 of Sec. 3 per problem of a batch: out[b] = sum_n v[b, n] s[b, n]
+// (float64 accumulation, fixed order).
+cudaError_t launch_mmd2_reduce(InType t, const float* s, const void* v, int64_t B, int64_t N,
+                               float* out, cudaStream_t st);
 // Forward sum of the FMA kernel's contributor slots: rows of the pair of
 // query tiles r = m / rows_per_unit have slots 0 .. last(r) - first(r), with
 // first(r) = r key_tiles / unit_len and last(r) = ((r + 1) key_tiles - 1) /
 // unit_len, added in slot order.
 cudaError_t launch_finalize_slots(const float* part, int64_t Mpad, int64_t M, int C,
                                   int rows_per_unit, int64_t key_tiles, int64_t unit_len,
-                                  float* out, cudaStream_t s);
+                                  float* out, cudaStream_t s, int batch = 1);
 cudaError_t launch_finalize(int mode, InType t, const float* part, int splits,
                             int64_t split_stride_rows, int64_t M, int Cv, int part_ld,
                             const float* inv_scale, const void* q, const float* mu, float tau,
@@ -91,13 +99,14 @@ cudaError_t launch_simt(const SimtPlan& p, bool grad, const float* q, const floa
 // B_2t, B_2t+1 (omitted when B is null), v_2t[0], v_2t+1[0], ...,
 // v_2t[C-1], v_2t+1[C-1].
 cudaError_t launch_key_records(InType t, const void* v, const float* B, int64_t N, int64_t Npad,
-                               int C, float* rec, cudaStream_t s);
+                               int C, float* rec, cudaStream_t s, int batch = 1);
 // Augmented MMA operands (see prep.cu): query layout into out_q, key layout
 // into out_k (either may be null), Dpa >= D + 2 aug_norm_terms(t) columns
 // per row.
 constexpr int aug_norm_terms(InType t) { return t == InType::BF16 ? 3 : 2; }
 cudaError_t launch_aug_prep(InType t, const void* x, int64_t rows, int64_t rows_pad, int D,
-                            int Dpa, const float* mu, void* out_q, void* out_k, cudaStream_t s);
+                            int Dpa, const float* mu, void* out_q, void* out_k, cudaStream_t s,
+                            int batch = 1);
 
 // tc_gauss.cu ----------------------------------------------------------
 cudaError_t launch_tc(const TcPlan& p, InType t, float c, char* ws, unsigned* status,

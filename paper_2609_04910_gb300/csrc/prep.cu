@@ -49,6 +49,10 @@ __global__ void mean_partial_kernel(const T* __restrict__ q, const T* __restrict
                                     float* __restrict__ partial) {
     __shared__ float red[8][33];
     __shared__ float big[8][33];
+    // Problem blockIdx.y of a batch: its own points and partial rows.
+    q += static_cast<int64_t>(blockIdx.y) * M * D;
+    k += static_cast<int64_t>(blockIdx.y) * N * D;
+    partial += static_cast<int64_t>(blockIdx.y) * 2 * gridDim.x * D;
     const int64_t r0 = static_cast<int64_t>(blockIdx.x) * rows_per_block;
     const int64_t r1 = min(r0 + rows_per_block, M + N);
     for (int d0 = 0; d0 < D; d0 += 32) {
@@ -93,6 +97,10 @@ mean_partial_vec_kernel(const T* __restrict__ q, const T* __restrict__ k, int64_
     __shared__ float s_sum[kMeanVecThreads][9];
     __shared__ float s_max[kMeanVecThreads][9];
     const int t = threadIdx.x;
+    // Problem blockIdx.y of a batch: its own points and partial rows.
+    q += static_cast<int64_t>(blockIdx.y) * M * D;
+    k += static_cast<int64_t>(blockIdx.y) * N * D;
+    partial += static_cast<int64_t>(blockIdx.y) * 2 * gridDim.x * D;
     const bool on_q = static_cast<int>(blockIdx.x) < Gq;
     const int64_t b = on_q ? blockIdx.x : blockIdx.x - Gq;
     const int64_t rows = on_q ? M : N;
@@ -153,6 +161,8 @@ mean_final_kernel(const float* __restrict__ partial, int G, int D, double total,
     __shared__ float red_m[kMeanFinalThreads];
     const int d = blockIdx.x;
     const int t = threadIdx.x;
+    partial += static_cast<int64_t>(blockIdx.y) * 2 * G * D;   // problem blockIdx.y
+    mu += static_cast<int64_t>(blockIdx.y) * D;
     double s = 0.0;
     float mx = 0.f;
     for (int g = t; g < G; g += kMeanFinalThreads) {
@@ -216,7 +226,7 @@ constexpr int kOperandMaxCols = 256;
 
 template <typename T, bool AUG>
 __global__ void __launch_bounds__(kOperandThreads)
-operand_kernel(const T* __restrict__ x, int64_t rows, int D, int Dp, int nt, float F,
+operand_kernel(const T* __restrict__ x, int64_t rows, int64_t rows_pad, int D, int Dp, int nt, float F,
                const float* __restrict__ mu, float half_c, float pad_value,
                T* __restrict__ out_q, T* __restrict__ out_k, float* __restrict__ nrm) {
     constexpr int R = kRowsPerBlock;
@@ -232,16 +242,28 @@ operand_kernel(const T* __restrict__ x, int64_t rows, int D, int Dp, int nt, flo
     float* s_mu = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(s_in) +
                                            ((R * D * static_cast<int>(sizeof(T)) + 15) & ~15));
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    // Problem blockIdx.y of a batch: its own rows, mean and outputs.
+    {
+        const int64_t b = blockIdx.y;
+        x += b * rows * D;
+        if (mu) mu += b * D;
+        if (out_q) out_q += b * rows_pad * Dp;
+        if (out_k) out_k += b * rows_pad * Dp;
+        if (nrm) nrm += b * rows_pad;
+    }
     const int64_t r0 = static_cast<int64_t>(blockIdx.x) * R;
     for (int d = tid; d < D; d += kOperandThreads) s_mu[d] = mu ? mu[d] : 0.f;
     const int64_t left = rows - r0;
     const int rin = left <= 0 ? 0 : left >= R ? R : static_cast<int>(left);
     {
-        // r0 D sizeof(T) is a multiple of 16 (R = 32) and x is 16-byte aligned.
+        // The block's rows are one run of rin x D elements.  Within one
+        // problem its start (r0 D sizeof(T), r0 a multiple of 32) is 16-byte
+        // aligned; a later problem of a batch may start anywhere, so the
+        // vector loads are used only when the run is 16-byte aligned.
         const int n_el = rin * D;
         constexpr int PER_VEC = 16 / static_cast<int>(sizeof(T));
-        const int nvec = n_el / PER_VEC;
         const T* src = x + r0 * D;
+        const int nvec = (reinterpret_cast<uintptr_t>(src) & 15u) == 0 ? n_el / PER_VEC : 0;
         for (int i = tid; i < nvec; i += kOperandThreads)
             reinterpret_cast<uint4*>(s_in)[i] = reinterpret_cast<const uint4*>(src)[i];
         for (int i = nvec * PER_VEC + tid; i < n_el; i += kOperandThreads) s_in[i] = src[i];
@@ -314,16 +336,20 @@ operand_kernel(const T* __restrict__ x, int64_t rows, int D, int Dp, int nt, flo
 
 __global__ void finalize_slots_kernel(const float* __restrict__ part, int64_t Mpad, int64_t M,
                                       int C, int rows_per_unit, int64_t key_tiles,
-                                      int64_t unit_len, float* __restrict__ out) {
+                                      int64_t unit_len, int64_t batch, float* __restrict__ out) {
+    // out: batch x M x C; partial rows are batch-stacked with Mpad rows per
+    // problem and batch Mpad rows per slot.
     const int64_t idx = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
-    if (idx >= M * C) return;
-    const int64_t m = idx / C;
-    const int c = static_cast<int>(idx - m * C);
+    if (idx >= batch * M * C) return;
+    const int64_t bm = idx / C;
+    const int c = static_cast<int>(idx - bm * C);
+    const int64_t b = bm / M;
+    const int64_t m = (bm - b * M) + b * Mpad;
     const int64_t r = m / rows_per_unit;
     const int64_t first = r * key_tiles / unit_len;
     const int64_t last = ((r + 1) * key_tiles - 1) / unit_len;
     float acc = 0.f;
-    for (int64_t sl = 0; sl <= last - first; ++sl) acc += part[(sl * Mpad + m) * C + c];
+    for (int64_t sl = 0; sl <= last - first; ++sl) acc += part[(sl * batch * Mpad + m) * C + c];
     out[idx] = acc;
 }
 
@@ -352,13 +378,19 @@ template <> __device__ __forceinline__ unsigned short to_bits<__nv_bfloat16>(__n
 
 template <typename T, bool AUG, int G>
 __global__ void __launch_bounds__(kOperandVecThreads)
-operand_vec_kernel(const T* __restrict__ x, int64_t rows, int64_t rows_pad, int D, int Dp, int nt,
-                   float F, const float* __restrict__ mu, float half_c, float pad_value,
-                   T* __restrict__ out_q, T* __restrict__ out_k, float* __restrict__ nrm) {
+operand_vec_kernel(const T* __restrict__ x, int64_t rows, int64_t rows_pad, int64_t batch, int D,
+                   int Dp, int nt, float F, const float* __restrict__ mu, float half_c,
+                   float pad_value, T* __restrict__ out_q, T* __restrict__ out_k,
+                   float* __restrict__ nrm) {
     const int vi = threadIdx.x % G;                              // vector within the row
+    // Output row of the batch-stacked operand (batch rows_pad rows per
+    // problem); problem b reads rows b rows .. of x and its own mean.
     const int64_t row = (static_cast<int64_t>(blockIdx.x) * kOperandVecThreads + threadIdx.x) / G;
-    const bool in_pad = row < rows_pad;
-    const bool valid = row < rows;
+    const int64_t b = row / rows_pad;
+    const int64_t i = row - b * rows_pad;
+    const bool in_pad = b < batch;
+    const bool valid = in_pad && i < rows;
+    if (mu && in_pad) mu += b * D;
     const int V = D / 8;
     const bool wq = AUG ? out_q != nullptr : true;
     const bool wk = AUG && out_k != nullptr;
@@ -366,7 +398,7 @@ operand_vec_kernel(const T* __restrict__ x, int64_t rows, int64_t rows_pad, int 
     if (in_pad && vi < V) {
         uint4 u = make_uint4(0u, 0u, 0u, 0u);
         if (valid) {
-            const uint4 in = *reinterpret_cast<const uint4*>(x + row * D + 8 * vi);
+            const uint4 in = *reinterpret_cast<const uint4*>(x + (b * rows + i) * D + 8 * vi);
             const unsigned short* hb = reinterpret_cast<const unsigned short*>(&in);
             float m[8];
             if (mu) {
@@ -434,7 +466,7 @@ operand_vec_kernel(const T* __restrict__ x, int64_t rows, int64_t rows_pad, int 
 template <typename T, bool AUG>
 cudaError_t operand_typed(const void* x, int64_t rows, int64_t rows_pad, int D, int Dp, int nt,
                           float F, const float* mu, float half_c, float pad_value, void* out_q,
-                          void* out_k, float* nrm, cudaStream_t s) {
+                          void* out_k, float* nrm, cudaStream_t s, int batch) {
     if (rows_pad % kRowsPerBlock != 0 || Dp % 16 != 0 || Dp > kOperandMaxCols ||
         (AUG && 2 * Dp > kOperandMaxCols))
         return cudaErrorInvalidValue;
@@ -442,10 +474,11 @@ cudaError_t operand_typed(const void* x, int64_t rows, int64_t rows_pad, int D, 
         // Vector path: G lanes per row.
         const int V = D / 8;
         const int G = V <= 1 ? 1 : V <= 2 ? 2 : V <= 4 ? 4 : V <= 8 ? 8 : V <= 16 ? 16 : 32;
-        const int64_t threads = rows_pad * G;
+        const int64_t threads = rows_pad * batch * G;
         const unsigned blocks = static_cast<unsigned>((threads + kOperandVecThreads - 1) / kOperandVecThreads);
         auto go = [&](auto kern) {
-            kern<<<blocks, kOperandVecThreads, 0, s>>>(static_cast<const T*>(x), rows, rows_pad, D,
+            kern<<<blocks, kOperandVecThreads, 0, s>>>(static_cast<const T*>(x), rows, rows_pad,
+                                                     static_cast<int64_t>(batch), D,
                                                      Dp, nt, F, mu, half_c, pad_value,
                                                      static_cast<T*>(out_q), static_cast<T*>(out_k),
                                                      nrm);
@@ -467,8 +500,8 @@ cudaError_t operand_typed(const void* x, int64_t rows, int64_t rows_pad, int D, 
     const size_t smem = static_cast<size_t>(nout) * kRowsPerBlock * Dp * sizeof(T) +
                         ((static_cast<size_t>(kRowsPerBlock) * D * sizeof(T) + 15) & ~size_t(15)) +
                         static_cast<size_t>(D) * sizeof(float);
-    operand_kernel<T, AUG><<<static_cast<unsigned>(blocks), kOperandThreads, smem, s>>>(
-        static_cast<const T*>(x), rows, D, Dp, nt, F, mu, half_c, pad_value,
+    operand_kernel<T, AUG><<<dim3(static_cast<unsigned>(blocks), batch), kOperandThreads, smem, s>>>(
+        static_cast<const T*>(x), rows, rows_pad, D, Dp, nt, F, mu, half_c, pad_value,
         static_cast<T*>(out_q), static_cast<T*>(out_k), nrm);
     note_launches(1);
     return cudaGetLastError();
@@ -574,6 +607,10 @@ __global__ void key_record_kernel(const T* __restrict__ v, const float* __restri
     if (t >= pairs) return;
     const int64_t n0 = 2 * t, n1 = 2 * t + 1;
     const int head = B ? 2 : 0;
+    // Problem blockIdx.y of a batch (2 pairs keys per problem).
+    v += static_cast<int64_t>(blockIdx.y) * N * C;
+    if (B) B += static_cast<int64_t>(blockIdx.y) * 2 * pairs;
+    rec += static_cast<int64_t>(blockIdx.y) * pairs * (head + 2 * C);
     float* out = rec + t * (head + 2 * C);
     if (B) {
         out[0] = B[n0];
@@ -662,7 +699,7 @@ cudaError_t finalize_typed(const float* part, int splits, int64_t stride_rows, i
 }  // namespace
 
 cudaError_t launch_mean(InType t, const void* q, const void* k, int64_t M, int64_t N, int D,
-                        int blocks, float* partial, float* mu, cudaStream_t s) {
+                        int blocks, float* partial, float* mu, cudaStream_t s, int batch) {
     // q and k the same points: the mean of [q; q] is the mean of q.
     if (q == k && M == N) N = 0;
     const int64_t total = M + N;
@@ -677,11 +714,11 @@ cudaError_t launch_mean(InType t, const void* q, const void* k, int64_t M, int64
         const int Gk = static_cast<int>((N + rpb - 1) / rpb);
         G = Gq + Gk;
         if (t == InType::F16)
-            mean_partial_vec_kernel<__half><<<G, kMeanVecThreads, 0, s>>>(
+            mean_partial_vec_kernel<__half><<<dim3(G, batch), kMeanVecThreads, 0, s>>>(
                 static_cast<const __half*>(q), static_cast<const __half*>(k), M, N, D, rpb, Gq,
                 partial);
         else
-            mean_partial_vec_kernel<__nv_bfloat16><<<G, kMeanVecThreads, 0, s>>>(
+            mean_partial_vec_kernel<__nv_bfloat16><<<dim3(G, batch), kMeanVecThreads, 0, s>>>(
                 static_cast<const __nv_bfloat16*>(q), static_cast<const __nv_bfloat16*>(k), M, N, D,
                 rpb, Gq, partial);
         note_launches(1);
@@ -690,17 +727,17 @@ cudaError_t launch_mean(InType t, const void* q, const void* k, int64_t M, int64
         G = static_cast<int>((total + rpb - 1) / rpb);
         switch (t) {
             case InType::F16:
-                mean_partial_kernel<__half><<<G, dim3(32, 8), 0, s>>>(
+                mean_partial_kernel<__half><<<dim3(G, batch), dim3(32, 8), 0, s>>>(
                     static_cast<const __half*>(q), static_cast<const __half*>(k), M, N, D, rpb,
                     partial);
                 break;
             case InType::BF16:
-                mean_partial_kernel<__nv_bfloat16><<<G, dim3(32, 8), 0, s>>>(
+                mean_partial_kernel<__nv_bfloat16><<<dim3(G, batch), dim3(32, 8), 0, s>>>(
                     static_cast<const __nv_bfloat16*>(q), static_cast<const __nv_bfloat16*>(k), M, N,
                     D, rpb, partial);
                 break;
             default:
-                mean_partial_kernel<float><<<G, dim3(32, 8), 0, s>>>(
+                mean_partial_kernel<float><<<dim3(G, batch), dim3(32, 8), 0, s>>>(
                     static_cast<const float*>(q), static_cast<const float*>(k), M, N, D, rpb,
                     partial);
         }
@@ -710,32 +747,78 @@ cudaError_t launch_mean(InType t, const void* q, const void* k, int64_t M, int64
     if (e != cudaSuccess) return e;
     const int mant_bits = t == InType::F16 ? 10 : t == InType::BF16 ? 7 : 23;
     const int min_exp = t == InType::F16 ? -24 : t == InType::BF16 ? -133 : -149;
-    mean_final_kernel<<<D, kMeanFinalThreads, 0, s>>>(partial, G, D, static_cast<double>(total),
+    mean_final_kernel<<<dim3(D, batch), kMeanFinalThreads, 0, s>>>(partial, G, D, static_cast<double>(total),
                                                      mant_bits, min_exp, mu);
+    note_launches(1);
+    return cudaGetLastError();
+}
+
+namespace {
+
+// Sec. 3: MMD^2 = v^T s for s = K v (q = k).  One block per problem: each
+// thread folds the products v_n s_n of n = t, t + 256, ... in float64 and a
+// fixed tree adds the threads (deterministic).
+template <typename T>
+__global__ void __launch_bounds__(256)
+mmd2_reduce_kernel(const float* __restrict__ s, const T* __restrict__ v, int64_t N,
+                   float* __restrict__ out) {
+    __shared__ double red[256];
+    const int t = threadIdx.x;
+    const int64_t b = blockIdx.x;
+    double acc = 0.0;
+    for (int64_t n = t; n < N; n += 256)
+        acc += static_cast<double>(to_f(v[b * N + n])) * static_cast<double>(s[b * N + n]);
+    red[t] = acc;
+    __syncthreads();
+    for (int w = 128; w > 0; w >>= 1) {
+        if (t < w) red[t] += red[t + w];
+        __syncthreads();
+    }
+    if (t == 0) out[b] = static_cast<float>(red[0]);
+}
+
+}  // namespace
+
+cudaError_t launch_mmd2_reduce(InType t, const float* s, const void* v, int64_t B, int64_t N,
+                               float* out, cudaStream_t st) {
+    if (B == 0) return cudaSuccess;
+    switch (t) {
+        case InType::F16:
+            mmd2_reduce_kernel<__half><<<static_cast<unsigned>(B), 256, 0, st>>>(
+                s, static_cast<const __half*>(v), N, out);
+            break;
+        case InType::BF16:
+            mmd2_reduce_kernel<__nv_bfloat16><<<static_cast<unsigned>(B), 256, 0, st>>>(
+                s, static_cast<const __nv_bfloat16*>(v), N, out);
+            break;
+        default:
+            mmd2_reduce_kernel<float><<<static_cast<unsigned>(B), 256, 0, st>>>(
+                s, static_cast<const float*>(v), N, out);
+    }
     note_launches(1);
     return cudaGetLastError();
 }
 
 cudaError_t launch_finalize_slots(const float* part, int64_t Mpad, int64_t M, int C,
                                   int rows_per_unit, int64_t key_tiles, int64_t unit_len,
-                                  float* out, cudaStream_t s) {
-    const int64_t total = M * C;
+                                  float* out, cudaStream_t s, int batch) {
+    const int64_t total = static_cast<int64_t>(batch) * M * C;
     if (total == 0) return cudaSuccess;
     const int threads = 256;
     finalize_slots_kernel<<<static_cast<unsigned>((total + threads - 1) / threads), threads, 0, s>>>(
-        part, Mpad, M, C, rows_per_unit, key_tiles, unit_len, out);
+        part, Mpad, M, C, rows_per_unit, key_tiles, unit_len, static_cast<int64_t>(batch), out);
     note_launches(1);
     return cudaGetLastError();
 }
 
 cudaError_t launch_center_cast_norm(InType t, const void* x, int64_t rows, int64_t rows_pad,
                                     int D, int Dp, const float* mu, float half_c, void* xh,
-                                    float* nrm, float pad_value, cudaStream_t s) {
+                                    float* nrm, float pad_value, cudaStream_t s, int batch) {
     if (t == InType::BF16)
         return operand_typed<__nv_bfloat16, false>(x, rows, rows_pad, D, Dp, 0, 1.f, mu, half_c,
-                                                   pad_value, xh, nullptr, nrm, s);
+                                                   pad_value, xh, nullptr, nrm, s, batch);
     return operand_typed<__half, false>(x, rows, rows_pad, D, Dp, 0, 1.f, mu, half_c, pad_value,
-                                        xh, nullptr, nrm, s);
+                                        xh, nullptr, nrm, s, batch);
 }
 
 cudaError_t launch_value_prep(InType t, bool grad, const void* v, const void* k,
@@ -754,26 +837,27 @@ cudaError_t launch_value_prep(InType t, bool grad, const void* v, const void* k,
 }
 
 cudaError_t launch_aug_prep(InType t, const void* x, int64_t rows, int64_t rows_pad, int D,
-                            int Dpa, const float* mu, void* out_q, void* out_k, cudaStream_t s) {
+                            int Dpa, const float* mu, void* out_q, void* out_k, cudaStream_t s,
+                            int batch) {
     const int nt = aug_norm_terms(t);
     if (t == InType::BF16)
         return operand_typed<__nv_bfloat16, true>(x, rows, rows_pad, D, Dpa, nt, 1.f, mu, 0.f, 0.f,
-                                                  out_q, out_k, nullptr, s);
+                                                  out_q, out_k, nullptr, s, batch);
     return operand_typed<__half, true>(x, rows, rows_pad, D, Dpa, nt, 1024.f, mu, 0.f, 0.f, out_q,
-                                       out_k, nullptr, s);
+                                       out_k, nullptr, s, batch);
 }
 
 cudaError_t launch_key_records(InType t, const void* v, const float* B, int64_t N, int64_t Npad,
-                               int C, float* rec, cudaStream_t s) {
+                               int C, float* rec, cudaStream_t s, int batch) {
     const int64_t pairs = Npad / 2;
     if (pairs == 0) return cudaSuccess;
     const int threads = 256;
     const unsigned blocks = static_cast<unsigned>((pairs + threads - 1) / threads);
     if (t == InType::BF16)
-        key_record_kernel<__nv_bfloat16><<<blocks, threads, 0, s>>>(
+        key_record_kernel<__nv_bfloat16><<<dim3(blocks, batch), threads, 0, s>>>(
             static_cast<const __nv_bfloat16*>(v), B, N, pairs, C, rec);
     else
-        key_record_kernel<__half><<<blocks, threads, 0, s>>>(static_cast<const __half*>(v), B, N,
+        key_record_kernel<__half><<<dim3(blocks, batch), threads, 0, s>>>(static_cast<const __half*>(v), B, N,
                                                              pairs, C, rec);
     note_launches(1);
     return cudaGetLastError();

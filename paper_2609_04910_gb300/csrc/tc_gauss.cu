@@ -416,7 +416,8 @@ cudaError_t launch_bn(const TcPlan& pl, InType t, float c, char* ws, unsigned* s
 }  // namespace
 
 bool plan_tensor(InType t, int64_t M, int64_t N, int64_t D, int64_t C, bool grad, bool center,
-                 bool alias, int split_override, int sms, TcPlan* p, const char** why) {
+                 bool alias, int split_override, int sms, TcPlan* p, const char** why,
+                 int64_t batch) {
     p->M = M;
     p->N = N;
     p->D = D;
@@ -472,7 +473,11 @@ bool plan_tensor(InType t, int64_t M, int64_t N, int64_t D, int64_t C, bool grad
     p->Mpad = (M + rows_per_cta - 1) / rows_per_cta * rows_per_cta;
     p->Npad = alias ? p->Mpad : (N + 127) / 128 * 128;
 
-    const int64_t tiles = p->Mpad / rows_per_cta;
+    // Only the FMA kernel takes a batch in one launch; the caller loops over
+    // the problems of a batch for the other kernels.
+    p->batch = p->fma ? std::max<int64_t>(1, batch) : 1;
+    const int64_t B = p->batch;
+    const int64_t tiles = B * (p->Mpad / rows_per_cta);
     const int64_t key_tiles = p->Npad / p->BN;
     int best_s = 1;
     if (split_override > 0) {
@@ -521,22 +526,23 @@ bool plan_tensor(InType t, int64_t M, int64_t N, int64_t D, int64_t C, bool grad
 
     size_t off = 0;
     auto take = [&](size_t bytes) { size_t o = off; off = align1k(off + bytes); return o; };
-    p->off_mean_part = take(static_cast<size_t>(p->mean_blocks) * D * 2 * 4);
-    p->off_mu = take(static_cast<size_t>(D) * 4);
-    p->off_qh = take(static_cast<size_t>(p->Mpad) * p->Dp * 2);
+    p->off_mean_part = take(static_cast<size_t>(B) * p->mean_blocks * D * 2 * 4);
+    p->off_mu = take(static_cast<size_t>(B) * D * 4);
+    p->off_qh = take(static_cast<size_t>(B) * p->Mpad * p->Dp * 2);
     // Augmented query and key operands differ in their extra columns, so
     // they are separate arrays even when q and k are the same points.
-    p->off_kh = (alias && !p->aug) ? p->off_qh : take(static_cast<size_t>(p->Npad) * p->Dp * 2);
+    p->off_kh = (alias && !p->aug) ? p->off_qh
+                                   : take(static_cast<size_t>(B) * p->Npad * p->Dp * 2);
     if (p->aug) {
         p->off_A = p->off_B = 0;   // the norms live in the augmented columns
     } else {
-        p->off_A = take(static_cast<size_t>(p->Mpad) * 4);
-        p->off_B = alias ? p->off_A : take(static_cast<size_t>(p->Npad) * 4);
+        p->off_A = take(static_cast<size_t>(B) * p->Mpad * 4);
+        p->off_B = alias ? p->off_A : take(static_cast<size_t>(B) * p->Npad * 4);
     }
     if (p->fma) {
         p->off_vt = p->off_vmax = p->off_inv = 0;
-        p->off_rec = take(static_cast<size_t>(p->Npad / 2) * ((p->aug ? 0 : 2) + 2 * p->Cv) * 4);
-        p->off_part = take(static_cast<size_t>(p->splits) * p->Mpad * p->Cv * 4);
+        p->off_rec = take(static_cast<size_t>(B) * (p->Npad / 2) * ((p->aug ? 0 : 2) + 2 * p->Cv) * 4);
+        p->off_part = take(static_cast<size_t>(p->splits) * B * p->Mpad * p->Cv * 4);
     } else {
         p->off_rec = 0;
         p->off_vt = take(static_cast<size_t>(p->Cp) * p->Npad * 2);

@@ -84,7 +84,9 @@ struct FmaParams {
     int64_t Mpad;
     int units;           // work units: (pair of query tiles, key tile), row major
     int unit_len;        // units per CTA (CTA i: units [i unit_len, (i + 1) unit_len))
-    int key_tiles;
+    int key_tiles;       // key tiles per problem
+    int pairs_per_batch; // pairs of query tiles per problem of a batch
+    int npad;            // k^ rows per problem of a batch
     int Dp;
     int nkb;             // 64-element K blocks of q^ / k^
     int stages;
@@ -193,6 +195,9 @@ tc_gauss_fma_kernel(const __grid_constant__ CUtensorMap tm_q,
         // Read by every thread after a CTA barrier: uniform.
         if (*abort_flag) break;
         const int tile_m = u / p.key_tiles;   // query tiles 2 tile_m, 2 tile_m + 1
+        // First k^ row of this pair's problem (batch-stacked operands).
+        const int kbase = (tile_m / p.pairs_per_batch) * p.npad;
+        (void)kbase;
         const int kt0 = u - tile_m * p.key_tiles;
         const int T = min(p.key_tiles - kt0, u_end - u);
         const int g0 = u - u_begin;           // running index of the segment's first tile
@@ -225,7 +230,7 @@ tc_gauss_fma_kernel(const __grid_constant__ CUtensorMap tm_q,
             if (has_tiles) {
                 auto load_keys = [&](int j) {
                     mbar_arrive_expect_tx(&bars->kv_full[k], p.kh_bytes + p.rec_bytes);
-                    const int n0 = (kt0 + j) * BN;
+                    const int n0 = kbase + (kt0 + j) * BN;
                     for (int kb = 0; kb < p.nkb; ++kb)
                         tma_load_2d(kh_smem(k) + kb * (BN * 128), &tm_k, &bars->kv_full[k], kb * KB, n0);
                     bulk_load(const_cast<float*>(rec_smem(k)),
@@ -331,6 +336,9 @@ tc_gauss_fma_kernel(const __grid_constant__ CUtensorMap tm_q,
         // Read by every thread after a CTA barrier: uniform.
         if (*abort_flag) break;
         const int tile_m = u / p.key_tiles;   // query tiles 2 tile_m, 2 tile_m + 1
+        // First k^ row of this pair's problem (batch-stacked operands).
+        const int kbase = (tile_m / p.pairs_per_batch) * p.npad;
+        (void)kbase;
         const int kt0 = u - tile_m * p.key_tiles;
         const int T = min(p.key_tiles - kt0, u_end - u);
         const int g0 = u - u_begin;           // running index of the segment's first tile
@@ -531,8 +539,8 @@ cudaError_t launch_typed(const TcPlan& pl, InType t, float c, char* ws, unsigned
     const CUtensorMapDataType hdt =
         t == InType::BF16 ? CU_TENSOR_MAP_DATA_TYPE_BFLOAT16 : CU_TENSOR_MAP_DATA_TYPE_FLOAT16;
     CUtensorMap tm_q, tm_k;
-    if (!encode_tile_map_2d(&tm_k, hdt, ws + pl.off_kh, pl.Dp, pl.Npad, pl.Dp * 2ull, KB, BN) ||
-        !encode_tile_map_2d(&tm_q, hdt, ws + pl.off_qh, pl.Dp, pl.Mpad, pl.Dp * 2ull, KB, BM)) {
+    if (!encode_tile_map_2d(&tm_k, hdt, ws + pl.off_kh, pl.Dp, pl.Npad * pl.batch, pl.Dp * 2ull, KB, BN) ||
+        !encode_tile_map_2d(&tm_q, hdt, ws + pl.off_qh, pl.Dp, pl.Mpad * pl.batch, pl.Dp * 2ull, KB, BM)) {
         *why = "cuTensorMapEncodeTiled failed or is unavailable";
         return cudaErrorInvalidValue;
     }
@@ -542,8 +550,10 @@ cudaError_t launch_typed(const TcPlan& pl, InType t, float c, char* ws, unsigned
     p.rec = reinterpret_cast<const float*>(ws + pl.off_rec);
     p.part = reinterpret_cast<float*>(ws + pl.off_part);
     p.status = status;
-    p.Mpad = pl.Mpad;
+    p.Mpad = pl.Mpad * pl.batch;   // partial-sum rows per contributor slot
     p.key_tiles = static_cast<int>(pl.Npad / BN);
+    p.pairs_per_batch = static_cast<int>(pl.Mpad / (NQ * BM));
+    p.npad = static_cast<int>(pl.Npad);
     p.units = static_cast<int>(pl.units);
     p.unit_len = static_cast<int>(pl.unit_len);
     p.Dp = pl.Dp;

@@ -28,7 +28,7 @@ def _declared_functions():
 def test_every_declared_symbol_is_exported(lib):
     from paper_2609_04910_gb300._binding import EXPORTS
     declared = _declared_functions()
-    assert len(declared) == 12
+    assert len(declared) == 14
     assert sorted(EXPORTS) == declared
     for name in declared:
         assert hasattr(lib, name), name

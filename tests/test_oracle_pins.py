@@ -300,3 +300,36 @@ def test_empty_and_rejected_inputs():
     assert np.all(s == 0) and s.shape == (3, 1)
     with pytest.raises(ValueError):
         oracle_sum(np.zeros((3, 2)), np.zeros((4, 2)), np.zeros((4, 1)), 1.0, rows=[3])
+
+
+# ---------------------------------------------------------------- MMD^2 (Sec. 3)
+def test_mmd2_brute_force_double_sum():
+    """oracle_mmd2 equals sum_{m,n} v_m exp(-tau/2 ||x_m - x_n||^2) v_n
+    written out with math.exp and math.fsum on a tiny case."""
+    from oracle import oracle_mmd2
+    rng = np.random.default_rng(21)
+    x = rng.standard_normal((5, 3))
+    v = np.array([0.4, -0.1, 0.3, -0.35, -0.25])
+    tau = 0.7
+    terms = []
+    for m in range(5):
+        for n in range(5):
+            d2 = sum((x[m, d] - x[n, d]) ** 2 for d in range(3))
+            terms.append(v[m] * math.exp(-tau / 2 * d2) * v[n])
+    got, den = oracle_mmd2(x, v, tau)
+    assert got == pytest.approx(math.fsum(terms), rel=1e-13, abs=1e-15)
+    assert den >= abs(got)
+
+
+def test_mmd2_zero_for_equal_samples_and_positive_otherwise():
+    """MMD^2 of two equal samples (weights +1/n on one copy, -1/n on the
+    other) is 0; for different samples it is > 0 (positive definite kernel)."""
+    from oracle import oracle_mmd2
+    rng = np.random.default_rng(22)
+    a = rng.standard_normal((40, 4))
+    v = np.concatenate([np.full(40, 1 / 40), np.full(40, -1 / 40)])
+    same, den = oracle_mmd2(np.concatenate([a, a]), v, 0.5)
+    assert abs(same) <= 1e-14 * den
+    b = rng.standard_normal((40, 4)) + 0.5
+    diff, _ = oracle_mmd2(np.concatenate([a, b]), v, 0.5)
+    assert diff > 0
