@@ -71,6 +71,9 @@ def _declare(lib):
     lib.gs_oracle_grad_q.argtypes = [dp, dp, dp, ctypes.c_double, i64, i64, i64,
                                      ip, i64, dp, dp, dp, dp, ctypes.c_int]
     lib.gs_oracle_grad_q.restype = ctypes.c_int
+    lib.gs_oracle_vjp.argtypes = [dp, dp, dp, dp, ctypes.c_double, i64, i64, i64, i64,
+                                  ip, i64, ip, i64, dp, dp, dp, dp, dp, dp, ctypes.c_int]
+    lib.gs_oracle_vjp.restype = ctypes.c_int
     lib.gs_oracle_max_threads.argtypes = []
     lib.gs_oracle_max_threads.restype = ctypes.c_int
 
@@ -172,3 +175,44 @@ def oracle_mmd2(x, v, tau, nthreads=None, lib_path=None):
     v = np.asarray(v, dtype=np.float64).reshape(-1)
     s, den = oracle_sum(x, x, v.reshape(-1, 1), tau, nthreads=nthreads, lib_path=lib_path)
     return float(np.dot(v, s[:, 0])), float(np.dot(np.abs(v), den[:, 0]))
+
+
+def _rows(rows):
+    if rows is None:
+        return None
+    return np.ascontiguousarray(np.asarray(rows, dtype=np.int64))
+
+
+def oracle_vjp(q, k, v, g, tau, rows_q=None, rows_k=None, nthreads=None, lib_path=None):
+    """Vector-Jacobian product of Eq. 1 in float64: the gradients of
+    L = sum_m g_m . s_m with respect to q, k and v.
+
+    q: (M, D), k: (N, D), v: (N, C), g: (M, C).  rows_q / rows_k select the
+    rows of dL/dq and of dL/dk, dL/dv (default: all).  Returns a dict with
+    gq (Rq, D), gk (Rk, D), gv (Rk, C) and their error scales dq, dk, dv of
+    the same shapes (see gauss_oracle.c).
+    """
+    q = np.asarray(q)
+    k = np.asarray(k)
+    M, D = q.shape
+    N = k.shape[0]
+    v = np.asarray(v).reshape(N, -1)
+    C = v.shape[1]
+    g = np.asarray(g).reshape(M, C)
+    q64, k64 = _f64(q, (M, D)), _f64(k, (N, D))
+    v64, g64 = _f64(v, (N, C)), _f64(g, (M, C))
+    rq, rk = _rows(rows_q), _rows(rows_k)
+    Rq = M if rq is None else rq.shape[0]
+    Rk = N if rk is None else rk.shape[0]
+    out = {
+        "gq": np.empty((Rq, D)), "dq": np.empty((Rq, D)),
+        "gk": np.empty((Rk, D)), "dk": np.empty((Rk, D)),
+        "gv": np.empty((Rk, C)), "dv": np.empty((Rk, C)),
+    }
+    rc = _load(lib_path).gs_oracle_vjp(
+        _ptr(q64), _ptr(k64), _ptr(v64), _ptr(g64), float(tau), M, N, D, C,
+        _ptr(rq), Rq, _ptr(rk), Rk, _ptr(out["gq"]), _ptr(out["gk"]), _ptr(out["gv"]),
+        _ptr(out["dq"]), _ptr(out["dk"]), _ptr(out["dv"]), _threads(nthreads))
+    if rc != 0:
+        raise ValueError("gs_oracle_vjp rejected its arguments")
+    return out

@@ -333,3 +333,123 @@ def test_mmd2_zero_for_equal_samples_and_positive_otherwise():
     b = rng.standard_normal((40, 4)) + 0.5
     diff, _ = oracle_mmd2(np.concatenate([a, b]), v, 0.5)
     assert diff > 0
+
+
+# ---------------------------------------------------------------- VJP of Eq. 1
+def _loss(q, k, v, g, tau):
+    """L = sum_m g_m . s_m through the (separately pinned) forward oracle."""
+    s, _ = oracle_sum(q, k, v, tau)
+    return math.fsum((g * s).ravel())
+
+
+def test_vjp_matches_finite_differences():
+    """Central differences of L = sum_m g_m . s_m in every coordinate of q,
+    k and v (chain rule on Eq. 1): catches a dropped term, a wrong sign or a
+    transposed contraction in any of the three outputs."""
+    from oracle import oracle_vjp
+    rng = np.random.default_rng(21)
+    M, N, D, C, tau = 4, 5, 3, 2, 0.8
+    q = rng.standard_normal((M, D))
+    k = rng.standard_normal((N, D))
+    v = rng.standard_normal((N, C))
+    g = rng.standard_normal((M, C))
+    r = oracle_vjp(q, k, v, g, tau)
+    h = 1e-6
+
+    def fd(arr, idx):
+        a = arr.copy()
+        a[idx] += h
+        args_p = [a if x is arr else x for x in (q, k, v)]
+        a2 = arr.copy()
+        a2[idx] -= h
+        args_m = [a2 if x is arr else x for x in (q, k, v)]
+        return (_loss(*args_p, g, tau) - _loss(*args_m, g, tau)) / (2 * h)
+
+    for name, arr, got in (("q", q, r["gq"]), ("k", k, r["gk"]), ("v", v, r["gv"])):
+        want = np.array([[fd(arr, (i, j)) for j in range(arr.shape[1])]
+                         for i in range(arr.shape[0])])
+        np.testing.assert_allclose(got, want, rtol=1e-7, atol=1e-8, err_msg=name)
+
+
+def test_vjp_reduces_to_q_gradient_for_unit_upstream():
+    """C = 1, g = 1: dL/dq_m is the q-gradient of Sec. 3 (the other oracle
+    function, written separately)."""
+    from oracle import oracle_vjp
+    rng = np.random.default_rng(22)
+    q = rng.standard_normal((9, 6))
+    k = rng.standard_normal((13, 6))
+    v = rng.standard_normal((13, 1))
+    r = oracle_vjp(q, k, v, np.ones((9, 1)), 0.45)
+    gq, _, den, _ = oracle_grad_q(q, k, v, 0.45)
+    np.testing.assert_allclose(r["gq"], gq, rtol=1e-13, atol=1e-15)
+    np.testing.assert_allclose(r["dq"], den, rtol=1e-13, atol=1e-15)
+
+
+def test_vjp_pairwise_antisymmetry_and_translation():
+    """Each pair contributes opposite forces to q_m and k_n, so
+    sum_m dL/dq_m + sum_n dL/dk_n = 0 (L is invariant under moving every
+    point by the same vector); a common shift of all points changes no
+    output."""
+    from oracle import oracle_vjp
+    rng = np.random.default_rng(23)
+    M, N, D, C, tau = 11, 7, 4, 3, 0.3
+    q = rng.standard_normal((M, D))
+    k = rng.standard_normal((N, D))
+    v = rng.standard_normal((N, C))
+    g = rng.standard_normal((M, C))
+    r = oracle_vjp(q, k, v, g, tau)
+    total = r["gq"].sum(0) + r["gk"].sum(0)
+    scale = np.abs(r["gq"]).sum(0) + np.abs(r["gk"]).sum(0)
+    assert np.all(np.abs(total) <= 1e-13 * scale)
+    t = rng.standard_normal(D) * 3.0
+    r2 = oracle_vjp(q + t, k + t, v, g, tau)
+    for key in ("gq", "gk", "gv"):
+        np.testing.assert_allclose(r2[key], r[key], rtol=1e-9, atol=1e-12, err_msg=key)
+
+
+def test_vjp_brute_force_tiny():
+    """Pure-Python double loop over pairs on a 2 x 3 problem."""
+    from oracle import oracle_vjp
+    q = [[0.5, -1.0], [0.0, 0.25]]
+    k = [[1.0, 0.0], [-0.5, 0.5], [0.25, -0.75]]
+    v = [[1.0, -2.0], [0.5, 0.0], [-1.5, 1.0]]
+    g = [[2.0, 1.0], [-1.0, 0.5]]
+    tau = 1.3
+    gq = [[0.0, 0.0] for _ in q]
+    gk = [[0.0, 0.0] for _ in k]
+    gv = [[0.0, 0.0] for _ in k]
+    for m in range(2):
+        for n in range(3):
+            phi = math.exp(-tau / 2 * sum((q[m][d] - k[n][d]) ** 2 for d in range(2)))
+            w = sum(g[m][c] * v[n][c] for c in range(2))
+            for d in range(2):
+                gq[m][d] += tau * phi * w * (k[n][d] - q[m][d])
+                gk[n][d] += tau * phi * w * (q[m][d] - k[n][d])
+            for c in range(2):
+                gv[n][c] += phi * g[m][c]
+    r = oracle_vjp(np.array(q), np.array(k), np.array(v), np.array(g), tau)
+    np.testing.assert_allclose(r["gq"], gq, rtol=1e-14, atol=1e-15)
+    np.testing.assert_allclose(r["gk"], gk, rtol=1e-14, atol=1e-15)
+    np.testing.assert_allclose(r["gv"], gv, rtol=1e-14, atol=1e-15)
+
+
+def test_vjp_row_subsets_and_scales():
+    """Row subsets return the selected rows of the full result; the error
+    scales bound the outputs they belong to (|x| <= its scale, since both
+    are sums of the same terms before and after taking magnitudes)."""
+    from oracle import oracle_vjp
+    rng = np.random.default_rng(24)
+    M, N, D, C = 17, 12, 5, 2
+    q = rng.standard_normal((M, D))
+    k = rng.standard_normal((N, D))
+    v = rng.standard_normal((N, C))
+    g = rng.standard_normal((M, C))
+    full = oracle_vjp(q, k, v, g, 0.6)
+    rq, rk = [16, 0, 5], [3, 11]
+    sub = oracle_vjp(q, k, v, g, 0.6, rows_q=rq, rows_k=rk, nthreads=1)
+    for key, rows in (("gq", rq), ("dq", rq), ("gk", rk), ("dk", rk), ("gv", rk), ("dv", rk)):
+        np.testing.assert_array_equal(sub[key], full[key][rows], err_msg=key)
+    for key, den in (("gq", "dq"), ("gk", "dk"), ("gv", "dv")):
+        assert np.all(np.abs(full[key]) <= full[den] * (1 + 1e-12))
+    with pytest.raises(ValueError):
+        oracle_vjp(q, k, v, g, 0.6, rows_q=[M])
