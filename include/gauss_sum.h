@@ -14,7 +14,8 @@
  *     grad_m = tau * ( sum_n Phi(q_m,k_n) v_n k_n  -  q_m sum_n Phi(q_m,k_n) v_n ),
  *
  * which the library evaluates as one Gauss sum with the augmented values
- * (v_n k_n, v_n) in R^{D+1}.
+ * (v_n k_n, v_n) in R^{D+1}, and the vector-Jacobian product of Eq. 1
+ * (gauss_sum_vjp: the gradients of sum_m g_m . s_m in q, k and v).
  *
  * Conventions shared by every entry point:
  *  - Array arguments are DEVICE pointers to contiguous row-major arrays,
@@ -31,8 +32,9 @@
  *    stream.
  *  - M = 0 is a no-op; N = 0 writes zeros.
  *  - fp16/bf16 inputs run on the tensor-core kernel (tcgen05, sm_103a) and
- *    need D <= 256 and C <= 256 (grad: D + 1 <= 256).  fp32 inputs run on
- *    the fp32 SIMT kernel (D <= 128 forward, D <= 64 gradient, any C).
+ *    need D <= 256 and C <= 256 (gradients: D <= 256, any C).  fp32 inputs
+ *    run on the fp32 SIMT kernel (D <= 128 forward, D <= 64 gradients, any
+ *    C).
  *  - On a non-OK return gauss_sum_last_error() describes the failure.
  */
 #ifndef GAUSS_SUM_H
@@ -117,6 +119,31 @@ gs_status gauss_sum_grad_q(const void* q, const void* k, const void* v, double t
 gs_status gauss_sum_grad_q_ex(const void* q, const void* k, const void* v, double tau,
                               int64_t M, int64_t N, int64_t D, gs_dtype dtype, float* grad,
                               float* s_out, void* stream, const gs_options* opt);
+
+/*
+ * Vector-Jacobian product of Eq. 1 (reverse-mode derivative, as used by the
+ * gradient flows of Sec. 3): for an upstream gradient g (M x C, float32) of
+ * L = sum_m g_m . s_m,
+ *
+ *     grad_q[m] = tau sum_n Phi(q_m, k_n) (g_m . v_n) (k_n - q_m)   M x D
+ *     grad_k[n] = tau sum_m Phi(q_m, k_n) (g_m . v_n) (q_m - k_n)   N x D
+ *     grad_v[n] =     sum_m Phi(q_m, k_n) g_m                       N x C
+ *
+ * (all float32).  q, k, v as for gauss_sum (dtype); any of grad_q, grad_k,
+ * grad_v may be NULL to skip it.  Evaluation: grad_q is a Gauss sum over
+ * the keys with the C (D + 1) values (v_nc k^_n, v_nc) contracted with g_m;
+ * grad_k and grad_v are one Gauss sum over the queries with the values
+ * (g_mc q^_m, g_mc) contracted with v_n (its unweighted channels are
+ * grad_v), k^ and q^ shifted by the common mean.  On the tensor-core path
+ * the channels are evaluated in launches of at most 256 channels
+ * (ceil(C (D + 1) / 256) launches per sum, each recomputing the kernel
+ * values), with the values rounded to fp16 after a per-channel power-of-two
+ * scale; the fp32 path makes C launches per sum.  g must be 16-byte
+ * aligned.  Default options; the workspace is allocated on `stream`.
+ */
+gs_status gauss_sum_vjp(const void* q, const void* k, const void* v, const float* g, double tau,
+                        int64_t M, int64_t N, int64_t D, int64_t C, gs_dtype dtype,
+                        float* grad_q, float* grad_k, float* grad_v, void* stream);
 
 /*
  * Workspace bytes that gauss_sum_ex (grad = 0, C channels) or

@@ -303,7 +303,7 @@ int gs_oracle_vjp(const double* q, const double* k, const double* v, const doubl
                     const double* gm = g + m * C;
                     const double phi = gauss_kernel(qm, kn, D, tau);
                     double w = 0.0;
-                    for (int64_t c = 0; c < C; ++c) w += gm[c] * vn[c];
+                    for (int64_t c = 0; c < C; ++c) w += vn[c] * gm[c];
                     if (outk)
                         for (int64_t d = 0; d < D; ++d) outk[d] += phi * w * (qm[d] - kn[d]);
                     for (int64_t c = 0; c < C; ++c) {

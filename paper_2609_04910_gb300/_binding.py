@@ -26,6 +26,7 @@ EXPORTS = (
     "gauss_sum_grad_q_ex", "gauss_sum_workspace_size", "gauss_sum_device_status",
     "gauss_sum_last_error", "gauss_sum_status_string", "gauss_sum_probe_ex2_rate",
     "gauss_sum_noalloc", "gauss_sum_kernel_launches", "gauss_sum_batched", "gauss_sum_mmd2",
+    "gauss_sum_vjp",
 )
 
 # Bytes of the static scratch array behind gauss_sum_noalloc
@@ -105,6 +106,8 @@ def _declare(lib):
     lib.gauss_sum_batched.restype = f
     lib.gauss_sum_mmd2.argtypes = [vp, vp, d, i64, i64, i64, f, vp, vp]
     lib.gauss_sum_mmd2.restype = f
+    lib.gauss_sum_vjp.argtypes = [vp, vp, vp, vp, d, i64, i64, i64, i64, f, vp, vp, vp, vp]
+    lib.gauss_sum_vjp.restype = f
 
 
 def _check(lib, status: int):
@@ -222,6 +225,36 @@ def gauss_sum_mmd2(x, v, tau, out=None, stream=None):
                             _stream_ptr(stream))
     _check(lib, st)
     return out
+
+
+def gauss_sum_vjp(q, k, v, g, tau, want=("q", "k", "v"), grad_q=None, grad_k=None,
+                  grad_v=None, stream=None):
+    """Vector-Jacobian product of Eq. 1 for the upstream g (M, C) fp32:
+    returns (grad_q (M, D), grad_k (N, D), grad_v (N, C)) as fp32 tensors,
+    None for the outputs not named in ``want``."""
+    import torch
+    lib = load_library()
+    for t, n in ((q, "q"), (k, "k"), (v, "v"), (g, "g")):
+        _check_tensor(t, n)
+    if g.dtype != torch.float32:
+        raise ValueError("g must be float32")
+    M, D = q.shape
+    N = k.shape[0]
+    C = 1 if v.dim() == 1 else v.shape[1]
+
+    def out(given, name, shape):
+        if given is None and name in want:
+            given = torch.empty(shape, dtype=torch.float32, device=q.device)
+        return given
+
+    grad_q = out(grad_q, "q", (M, D))
+    grad_k = out(grad_k, "k", (N, D))
+    grad_v = out(grad_v, "v", (N, C))
+    st = lib.gauss_sum_vjp(_ptr(q), _ptr(k), _ptr(v), _ptr(g), float(tau), M, N, D, C,
+                           _dtype_code(q), _ptr(grad_q), _ptr(grad_k), _ptr(grad_v),
+                           _stream_ptr(stream))
+    _check(lib, st)
+    return grad_q, grad_k, grad_v
 
 
 def gauss_sum_noalloc(q, k, v, tau, out=None, stream=None):

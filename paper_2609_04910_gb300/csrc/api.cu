@@ -2,6 +2,7 @@
 // kernel sequencing and error reporting.  See include/gauss_sum.h.
 #include <cuda_runtime.h>
 
+#include <algorithm>
 #include <cmath>
 #include <cstdio>
 #include <cstdlib>
@@ -75,10 +76,17 @@ struct Call {
     gs_dtype dtype;
     bool grad;
     float* out;    // M x C (forward) or M x D (grad)
-    float* s_out;  // grad only, nullable
+    float* s_out;  // grad only, M x C, nullable
     cudaStream_t stream;
     gs_options opt;
     int64_t B = 1;  // problems of a batch: q B x M x D, k B x N x D, v B x N x C, out B x M x ..
+    // Gradient mode: v holds the key weights w (N x C; float32 when w_f32,
+    // else the input dtype) and u the weights of the query rows that the C
+    // channels are contracted with (M x C; float32 when u_f32; null: ones).
+    // out (M x D) may be null when only s_out is wanted.
+    bool w_f32 = false;
+    const void* u = nullptr;
+    bool u_f32 = false;
 };
 
 gs_status validate(const Call& c) {
@@ -88,15 +96,14 @@ gs_status validate(const Call& c) {
         return fail(GS_ERR_INVALID_ARGUMENT, "negative size");
     if (!(std::isfinite(c.tau) && c.tau > 0.0))
         return fail(GS_ERR_INVALID_ARGUMENT, "tau must be finite and > 0");
-    if (c.grad && c.C != 1) return fail(GS_ERR_INVALID_ARGUMENT, "the q-gradient needs C = 1");
-    const int64_t out_w = c.grad ? c.D : c.C;
     const bool any = c.B > 0;   // an empty batch reads and writes nothing
-    if (any && c.M > 0 && out_w > 0 && !c.out) return fail(GS_ERR_INVALID_ARGUMENT, "null output pointer");
+    if (!c.grad && any && c.M > 0 && c.C > 0 && !c.out)
+        return fail(GS_ERR_INVALID_ARGUMENT, "null output pointer");
     if (any && c.M > 0 && c.D > 0 && !c.q) return fail(GS_ERR_INVALID_ARGUMENT, "null q pointer");
     if (any && c.N > 0 && c.D > 0 && !c.k) return fail(GS_ERR_INVALID_ARGUMENT, "null k pointer");
     if (any && c.N > 0 && c.C > 0 && !c.v) return fail(GS_ERR_INVALID_ARGUMENT, "null v pointer");
     if (!aligned16(c.q) || !aligned16(c.k) || !aligned16(c.v) || !aligned16(c.out) ||
-        !aligned16(c.s_out))
+        !aligned16(c.s_out) || !aligned16(c.u))
         return fail(GS_ERR_INVALID_ARGUMENT, "base pointers must be 16-byte aligned");
     if (c.opt.path == GS_PATH_TENSOR && c.dtype == GS_FP32)
         return fail(GS_ERR_UNSUPPORTED, "the tensor-core path takes fp16/bf16 inputs");
@@ -107,6 +114,15 @@ gs_status validate(const Call& c) {
     if (c.opt.workspace && (reinterpret_cast<uintptr_t>(c.opt.workspace) & 255u))
         return fail(GS_ERR_INVALID_ARGUMENT, "caller workspace must be 256-byte aligned");
     return GS_OK;
+}
+
+// Gradient channels on the tensor-core path: the C (D + 1) channels of
+// value_prep are split into *n launches of equal width (at most 256, the
+// widest value operand of the two-MMA kernel); returns that width.
+int64_t grad_chunk(int64_t D, int64_t C, int64_t* n) {
+    const int64_t total = std::max<int64_t>(1, C * (D + 1));
+    *n = (total + 255) / 256;
+    return (total + *n - 1) / *n;
 }
 
 gs::InType in_type(gs_dtype d) {
@@ -120,7 +136,9 @@ gs_status plan(const Call& c, int sms, bool* tensor, gs::TcPlan* tp, gs::SimtPla
     *tensor = c.dtype != GS_FP32;
     if (*tensor) {
         const bool alias = c.q == c.k && c.M == c.N && c.q != nullptr;
-        if (!gs::plan_tensor(in_type(c.dtype), c.M, c.N, c.D, c.C, c.grad, c.opt.center != 0,
+        int64_t nch = 1;
+        const int64_t width = c.grad ? grad_chunk(c.D, c.C, &nch) : c.C;
+        if (!gs::plan_tensor(in_type(c.dtype), c.M, c.N, c.D, width, c.grad, c.opt.center != 0,
                              alias, c.opt.split_n, sms, tp, &why, c.B))
             return fail(GS_ERR_UNSUPPORTED, "%s", why);
         *bytes = tp->total;
@@ -146,21 +164,17 @@ gs_status run(Call c) {
     gs_status st = validate(c);
     if (st != GS_OK) return st;
     if (c.M == 0 || c.B == 0) return GS_OK;
-    if (c.grad && c.D == 0) {
-        // No coordinates: the gradient is empty and s is the plain forward sum.
-        if (!c.s_out) return GS_OK;
-        c.grad = false;
-        c.out = c.s_out;
-        c.s_out = nullptr;
-    }
-    const int64_t out_w = c.grad ? c.D : c.C;
-    if (out_w == 0 && !(c.grad && c.s_out)) return GS_OK;
+    if (c.grad && c.D == 0) c.out = nullptr;   // the gradient has no coordinates
+    if (c.grad ? !(c.out || c.s_out) : c.C == 0) return GS_OK;
 
-    if (c.N == 0) {
+    if (c.N == 0 || c.C == 0) {
+        // No keys, or no weight channels (gradient): every sum is empty.
         cudaError_t e = cudaSuccess;
-        if (out_w > 0) e = cudaMemsetAsync(c.out, 0, sizeof(float) * c.B * c.M * out_w, c.stream);
-        if (e == cudaSuccess && c.grad && c.s_out)
-            e = cudaMemsetAsync(c.s_out, 0, sizeof(float) * c.B * c.M, c.stream);
+        const int64_t out_w = c.grad ? c.D : c.C;
+        if (c.out && out_w > 0)
+            e = cudaMemsetAsync(c.out, 0, sizeof(float) * c.B * c.M * out_w, c.stream);
+        if (e == cudaSuccess && c.grad && c.s_out && c.C > 0)
+            e = cudaMemsetAsync(c.s_out, 0, sizeof(float) * c.B * c.M * c.C, c.stream);
         return e == cudaSuccess ? GS_OK : cuda_fail(e, "cudaMemsetAsync");
     }
 
@@ -182,15 +196,17 @@ gs_status run(Call c) {
         // Only the FMA kernel takes a batch in one launch: the problems of a
         // batch run one after another on the stream.
         const int64_t es = c.dtype == GS_FP32 ? 4 : 2;
+        const int64_t ws_ = c.w_f32 ? 4 : es, us = c.u_f32 ? 4 : es;
         const int64_t out_w1 = c.grad ? c.D : c.C;
         for (int64_t b = 0; b < c.B; ++b) {
             Call cb = c;
             cb.B = 1;
             cb.q = static_cast<const char*>(c.q) + b * c.M * c.D * es;
             cb.k = static_cast<const char*>(c.k) + b * c.N * c.D * es;
-            cb.v = static_cast<const char*>(c.v) + b * c.N * c.C * es;
-            cb.out = c.out + b * c.M * out_w1;
-            if (c.s_out) cb.s_out = c.s_out + b * c.M;
+            cb.v = static_cast<const char*>(c.v) + b * c.N * c.C * ws_;
+            if (c.u) cb.u = static_cast<const char*>(c.u) + b * c.M * c.C * us;
+            if (c.out) cb.out = c.out + b * c.M * out_w1;
+            if (c.s_out) cb.s_out = c.s_out + b * c.M * c.C;
             st = run(cb);
             if (st != GS_OK) return st;
         }
@@ -259,51 +275,83 @@ gs_status run(Call c) {
                 tp.Npad, static_cast<int>(tp.Cv), reinterpret_cast<float*>(ws + tp.off_rec),
                 c.stream, batch);
             where = "key-record kernel";
-        } else if (e == cudaSuccess) {
-            e = gs::launch_value_prep(t, c.grad, c.v, c.k, mu, c.N, tp.Npad, static_cast<int>(c.D),
-                                      static_cast<int>(tp.Cv), tp.Cp,
-                                      reinterpret_cast<unsigned*>(ws + tp.off_vmax), ws + tp.off_vt,
-                                      reinterpret_cast<float*>(ws + tp.off_inv), c.stream);
-            where = "value kernel";
-        }
-        if (e == cudaSuccess) {
-            e = record_event(c.opt.main_events[0], c.stream);
-            if (e == cudaSuccess)
-                e = tp.fma ? gs::launch_tc_fma(tp, t, cexp, ws, status, c.stream, &why)
-                           : gs::launch_tc(tp, t, cexp, ws, status, c.stream, &why);
+            if (e == cudaSuccess) e = record_event(c.opt.main_events[0], c.stream);
+            if (e == cudaSuccess) {
+                e = gs::launch_tc_fma(tp, t, cexp, ws, status, c.stream, &why);
+                where = "fused tensor-core kernel";
+            }
             if (e == cudaSuccess) e = record_event(c.opt.main_events[1], c.stream);
-            where = "fused tensor-core kernel";
-        }
-        if (e == cudaSuccess) {
-            if (tp.fma)
+            if (e == cudaSuccess) {
                 e = gs::launch_finalize_slots(reinterpret_cast<float*>(ws + tp.off_part), tp.Mpad,
-                                              c.M, static_cast<int>(tp.Cv),
-                                              128 * tp.nq, tp.Npad / tp.BN, tp.unit_len, c.out,
-                                              c.stream, batch);
-            else
-                e = gs::launch_finalize(c.grad ? 1 : 0, t,
-                                        reinterpret_cast<float*>(ws + tp.off_part), tp.splits,
-                                        tp.Mpad, c.M, static_cast<int>(tp.Cv), tp.Cp,
-                                        reinterpret_cast<float*>(ws + tp.off_inv), c.q, mu,
-                                        static_cast<float>(c.tau), static_cast<int>(c.D), c.out,
-                                        c.s_out, c.stream);
-            where = "finalise kernel";
+                                              c.M, static_cast<int>(tp.Cv), 128 * tp.nq,
+                                              tp.Npad / tp.BN, tp.unit_len, c.out, c.stream,
+                                              batch);
+                where = "finalise kernel";
+            }
+        } else if (e == cudaSuccess) {
+            // Two-MMA kernel, once per chunk of value channels (one chunk for
+            // the forward sum; C (D + 1) channels in chunks for gradients).
+            const int64_t total = c.grad ? c.C * (c.D + 1) : c.C;
+            const int64_t width = tp.Cv;
+            float* part = reinterpret_cast<float*>(ws + tp.off_part);
+            float* inv = reinterpret_cast<float*>(ws + tp.off_inv);
+            for (int64_t ch0 = 0; ch0 < total && e == cudaSuccess; ch0 += width) {
+                const int cc = static_cast<int>(std::min(width, total - ch0));
+                e = gs::launch_value_prep(t, c.grad, c.w_f32, c.v, c.k, mu, c.N, tp.Npad,
+                                          static_cast<int>(c.D), static_cast<int>(c.C),
+                                          static_cast<int>(ch0), cc, tp.Cp,
+                                          reinterpret_cast<unsigned*>(ws + tp.off_vmax),
+                                          ws + tp.off_vt, inv, c.stream);
+                where = "value kernel";
+                if (e == cudaSuccess && ch0 == 0) e = record_event(c.opt.main_events[0], c.stream);
+                if (e == cudaSuccess) {
+                    e = gs::launch_tc(tp, t, cexp, ws, status, c.stream, &why);
+                    where = "fused tensor-core kernel";
+                }
+                if (e == cudaSuccess && ch0 + width >= total)
+                    e = record_event(c.opt.main_events[1], c.stream);
+                if (e == cudaSuccess) {
+                    if (c.grad)
+                        e = gs::launch_finalize_points(
+                            false, t, c.u_f32, part, tp.splits, tp.Mpad, c.M, tp.Cp, inv, c.q, mu,
+                            static_cast<float>(c.tau), static_cast<int>(c.D),
+                            static_cast<int>(c.C), static_cast<int>(ch0), cc, c.u, ch0 > 0,
+                            c.out, c.s_out, c.stream);
+                    else
+                        e = gs::launch_finalize(part, tp.splits, tp.Mpad, c.M, cc, tp.Cp, inv,
+                                                c.out, c.stream);
+                    where = "finalise kernel";
+                }
+            }
         }
     } else {
         float* part = reinterpret_cast<float*>(ws + sp.off_part);
-        e = record_event(c.opt.main_events[0], c.stream);
-        if (e == cudaSuccess)
-            e = gs::launch_simt(sp, c.grad, static_cast<const float*>(c.q),
-                                static_cast<const float*>(c.k), static_cast<const float*>(c.v),
-                                half_c, part, c.stream);
-        if (e == cudaSuccess) e = record_event(c.opt.main_events[1], c.stream);
-        where = "fp32 kernel";
-        if (e == cudaSuccess) {
-            e = gs::launch_finalize(c.grad ? 2 : 0, gs::InType::F32, part, sp.splits, c.M, c.M,
-                                    static_cast<int>(sp.Cv), static_cast<int>(sp.Cv), nullptr,
-                                    nullptr, nullptr, static_cast<float>(c.tau),
-                                    static_cast<int>(c.D), c.out, c.s_out, c.stream);
-            where = "finalise kernel";
+        const float* qf = static_cast<const float*>(c.q);
+        const float* kf = static_cast<const float*>(c.k);
+        const float* vf = static_cast<const float*>(c.v);
+        // Forward: one launch over all channels.  Gradient: one launch per
+        // weight channel, contracted into out by the finalise kernel.
+        const int64_t passes = c.grad ? c.C : 1;
+        for (int64_t wc = 0; wc < passes && e == cudaSuccess; ++wc) {
+            if (wc == 0) e = record_event(c.opt.main_events[0], c.stream);
+            if (e == cudaSuccess)
+                e = gs::launch_simt(sp, c.grad, qf, kf, vf, static_cast<int>(c.C),
+                                    static_cast<int>(wc), half_c, part, c.stream);
+            where = "fp32 kernel";
+            if (e == cudaSuccess && wc + 1 == passes) e = record_event(c.opt.main_events[1], c.stream);
+            if (e == cudaSuccess) {
+                const int G = static_cast<int>(c.D + 1);
+                if (c.grad)
+                    e = gs::launch_finalize_points(
+                        true, gs::InType::F32, true, part, sp.splits, c.M, c.M, G, nullptr,
+                        nullptr, nullptr, static_cast<float>(c.tau), static_cast<int>(c.D),
+                        static_cast<int>(c.C), static_cast<int>(wc) * G, G, c.u, wc > 0, c.out,
+                        c.s_out, c.stream);
+                else
+                    e = gs::launch_finalize(part, sp.splits, c.M, c.M, static_cast<int>(sp.Cv),
+                                            static_cast<int>(sp.Cv), nullptr, c.out, c.stream);
+                where = "finalise kernel";
+            }
         }
     }
     if (owned) {
@@ -471,7 +519,31 @@ gs_status gauss_sum_grad_q_ex(const void* q, const void* k, const void* v, doubl
                               float* s_out, void* stream, const gs_options* opt) {
     Call c{q, k, v, tau, M, N, D, 1, dtype, true, grad, s_out,
            static_cast<cudaStream_t>(stream), opt ? *opt : defaults()};
+    if (M > 0 && D > 0 && !grad) return fail(GS_ERR_INVALID_ARGUMENT, "null output pointer");
     return run(c);
+}
+
+gs_status gauss_sum_vjp(const void* q, const void* k, const void* v, const float* g, double tau,
+                        int64_t M, int64_t N, int64_t D, int64_t C, gs_dtype dtype,
+                        float* grad_q, float* grad_k, float* grad_v, void* stream) {
+    const cudaStream_t st = static_cast<cudaStream_t>(stream);
+    // dL/dq: queries q, keys k weighted by v, contracted with g.
+    Call a{q, k, v, tau, M, N, D, C, dtype, true, grad_q, nullptr, st, defaults()};
+    a.u = g;
+    a.u_f32 = true;
+    // dL/dk and dL/dv: queries k, keys q weighted by g, contracted with v;
+    // the unweighted channel of each group is dL/dv.
+    Call b{k, q, g, tau, N, M, D, C, dtype, true, grad_k, grad_v, st, defaults()};
+    b.w_f32 = true;
+    b.u = v;
+    b.u_f32 = dtype == GS_FP32;
+    if (M > 0 && C > 0 && !g) return fail(GS_ERR_INVALID_ARGUMENT, "null g pointer");
+    gs_status status = validate(a);
+    if (status == GS_OK) status = validate(b);
+    if (status != GS_OK) return status;
+    if (grad_q) status = run(a);
+    if (status == GS_OK && (grad_k || grad_v)) status = run(b);
+    return status;
 }
 
 gs_status gauss_sum_grad_q(const void* q, const void* k, const void* v, double tau, int64_t M,

@@ -18,7 +18,8 @@ constexpr int kFmaMaxChannels = 4;
 // Workspace plan of the tensor-core path.  All offsets are bytes from the
 // workspace base and are 1024-byte aligned.
 struct TcPlan {
-    int64_t M, N, D, Cv;     // Cv: value channels (C, or D + 1 for the gradient)
+    int64_t M, N, D, Cv;     // Cv: value channels of one launch (C, or a chunk of the
+                             // C (D + 1) gradient channels)
     int64_t Mpad, Npad;      // rows padded to the row tile / key tile
     int Dp, Cp;              // D and Cv rounded up to 16
     int BN;                  // key tile width (128, or 64 when Cp > 128)
@@ -69,12 +70,29 @@ cudaError_t launch_mean(InType t, const void* q, const void* k, int64_t M, int64
 cudaError_t launch_center_cast_norm(InType t, const void* x, int64_t rows, int64_t rows_pad,
                                     int D, int Dp, const float* mu, float half_c, void* xh,
                                     float* nrm, float pad_value, cudaStream_t s, int batch = 1);
-cudaError_t launch_value_prep(InType t, bool grad, const void* v, const void* k,
-                              const float* mu, int64_t N, int64_t Npad, int D, int Cv, int Cp,
-                              unsigned* vmax_bits, void* vt, float* inv_scale, cudaStream_t s);
-// mode 0: forward (out M x Cv, scaled by inv_scale when given)
-// mode 1: gradient from augmented values (tensor path): needs q, mu, tau
-// mode 2: gradient from direct partials (SIMT path): Cv = D + 1
+// Transposed fp16 value operand of the two-MMA kernel for the channels
+// ch0 .. ch0 + Cc - 1 (Cp >= Cc rows of Npad keys), with per-channel
+// power-of-two scales.  Forward: channel ch of key n is w[n, ch] (w has the
+// input dtype, Cw = channels).  grad: channel c (D + 1) + d is
+// w[n, c] (x[n, d] - mu_d) for d < D and w[n, c] for d = D (w is N x Cw,
+// float32 when w_f32, else the input dtype; x is N x D).
+cudaError_t launch_value_prep(InType t, bool grad, bool w_f32, const void* w, const void* x,
+                              const float* mu, int64_t N, int64_t Npad, int D, int Cw, int ch0,
+                              int Cc, int Cp, unsigned* vmax_bits, void* vt, float* inv_scale,
+                              cudaStream_t s);
+// Forward: out (M x Cv) = inv_scale (when given) x the split partials summed
+// in split order.
+cudaError_t launch_finalize(const float* part, int splits, int64_t split_stride_rows,
+                            int64_t M, int Cv, int part_ld, const float* inv_scale, float* out,
+                            cudaStream_t s);
+// Gradient contraction of one launch's channels ch0 .. ch0 + Cc - 1 (see
+// prep.cu): out[m, d] (+)= tau sum_c u[m, c] (S_{c,d} - x^_{m,d} S_{c,D}),
+// s_out[m, c] = S_{c,D}.  direct: fp32 kernel partials (difference form).
+cudaError_t launch_finalize_points(bool direct, InType t, bool u_f32, const float* part,
+                                   int splits, int64_t split_stride_rows, int64_t M, int part_ld,
+                                   const float* inv_scale, const void* x, const float* mu,
+                                   float tau, int D, int Cw, int ch0, int Cc, const void* u,
+                                   int accumulate, float* out, float* s_out, cudaStream_t s);
 // MMD^2 of Sec. 3 per problem of a batch: out[b] = sum_n v[b, n] s[b, n]
 // (float64 accumulation, fixed order).
 cudaError_t launch_mmd2_reduce(InType t, const float* s, const void* v, int64_t B, int64_t N,
@@ -86,14 +104,13 @@ cudaError_t launch_mmd2_reduce(InType t, const float* s, const void* v, int64_t 
 cudaError_t launch_finalize_slots(const float* part, int64_t Mpad, int64_t M, int C,
                                   int rows_per_unit, int64_t key_tiles, int64_t unit_len,
                                   float* out, cudaStream_t s, int batch = 1);
-cudaError_t launch_finalize(int mode, InType t, const float* part, int splits,
-                            int64_t split_stride_rows, int64_t M, int Cv, int part_ld,
-                            const float* inv_scale, const void* q, const float* mu, float tau,
-                            int D, float* out, float* s_out, cudaStream_t s);
 
 // simt_fp32.cu ---------------------------------------------------------
+// grad: keys weighted by channel wch of v (N x Cw); partials have D + 1
+// channels (sum Phi w (k - q), sum Phi w).
 cudaError_t launch_simt(const SimtPlan& p, bool grad, const float* q, const float* k,
-                        const float* v, float half_c, float* part, cudaStream_t s);
+                        const float* v, int Cw, int wch, float half_c, float* part,
+                        cudaStream_t s);
 
 // Key records of the FMA kernel: per key pair (2t, 2t+1) the floats
 // B_2t, B_2t+1 (omitted when B is null), v_2t[0], v_2t+1[0], ...,

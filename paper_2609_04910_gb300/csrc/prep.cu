@@ -508,37 +508,42 @@ cudaError_t operand_typed(const void* x, int64_t rows, int64_t rows_pad, int D, 
 }
 
 // ---------------------------------------------------------------- values
-// Value of channel c of key n: v[n, c] (forward) or, for the gradient of
-// Sec. 3, v_n (k[n, c] - mu_c) for c < D and v_n for c = D.
-template <typename T, bool GRAD>
-__device__ __forceinline__ float value_at(const T* __restrict__ v, const T* __restrict__ k,
-                                          const float* __restrict__ mu, int64_t n, int c, int D,
-                                          int Cv) {
+// Value of channel ch of key n.  Forward (Eq. 1): w[n, ch] (Cw = channels).
+// Gradients (Sec. 3, and the vector-Jacobian product of Eq. 1): channel
+// ch = c (D + 1) + d holds w[n, c] (x[n, d] - mu_d) for d < D and w[n, c]
+// for d = D, one group of D + 1 channels per weight channel c < Cw.
+template <typename T, typename W, bool GRAD>
+__device__ __forceinline__ float value_at(const W* __restrict__ w, const T* __restrict__ x,
+                                          const float* __restrict__ mu, int64_t n, int ch, int D,
+                                          int Cw) {
     if (GRAD) {
-        const float vn = to_f(v[n]);
-        if (c < D) return vn * (to_f(k[n * D + c]) - (mu ? mu[c] : 0.f));
-        return vn;
+        const int c = ch / (D + 1);
+        const int d = ch - c * (D + 1);
+        const float wn = to_f(w[n * Cw + c]);
+        if (d < D) return wn * (to_f(x[n * D + d]) - (mu ? mu[d] : 0.f));
+        return wn;
     }
-    return to_f(v[n * Cv + c]);
+    return to_f(w[n * Cw + ch]);
 }
 
-// Per-channel max |value| over the keys; block (32, 8) as in the mean.
-template <typename T, bool GRAD>
-__global__ void value_max_kernel(const T* __restrict__ v, const T* __restrict__ k,
-                                 const float* __restrict__ mu, int64_t N, int D, int Cv,
-                                 int64_t rows_per_block, unsigned* __restrict__ vmax_bits) {
+// Per-channel max |value| over the keys for channels ch0 .. ch0 + Cc - 1;
+// block (32, 8) as in the mean.
+template <typename T, typename W, bool GRAD>
+__global__ void value_max_kernel(const W* __restrict__ w, const T* __restrict__ x,
+                                 const float* __restrict__ mu, int64_t N, int D, int Cw, int ch0,
+                                 int Cc, int64_t rows_per_block, unsigned* __restrict__ vmax_bits) {
     __shared__ float red[8][33];
     const int64_t r0 = static_cast<int64_t>(blockIdx.x) * rows_per_block;
     const int64_t r1 = min(r0 + rows_per_block, N);
-    for (int c0 = 0; c0 < Cv; c0 += 32) {
+    for (int c0 = 0; c0 < Cc; c0 += 32) {
         const int c = c0 + threadIdx.x;
         float mx = 0.f;
-        if (c < Cv)
+        if (c < Cc)
             for (int64_t n = r0 + threadIdx.y; n < r1; n += 8)
-                mx = fmaxf(mx, fabsf(value_at<T, GRAD>(v, k, mu, n, c, D, Cv)));
+                mx = fmaxf(mx, fabsf(value_at<T, W, GRAD>(w, x, mu, n, ch0 + c, D, Cw)));
         red[threadIdx.y][threadIdx.x] = mx;
         __syncthreads();
-        if (threadIdx.y == 0 && c < Cv) {
+        if (threadIdx.y == 0 && c < Cc) {
             float m = 0.f;
 #pragma unroll
             for (int y = 0; y < 8; ++y) m = fmaxf(m, red[y][threadIdx.x]);
@@ -563,13 +568,15 @@ __device__ __forceinline__ int channel_exponent(unsigned max_bits) {
 
 __device__ __forceinline__ float pow2f(int e) { return __uint_as_float(static_cast<unsigned>(e + 127) << 23); }
 
-// Transposed, scaled fp16 value operand vt[c][n] (Cp x Npad, zero padded),
-// through a 32 x 32 shared-memory tile; block (32, 8).
-template <typename T, bool GRAD>
-__global__ void value_prep_kernel(const T* __restrict__ v, const T* __restrict__ k,
+// Transposed, scaled fp16 value operand vt[j][n] = value of channel ch0 + j
+// (Cp x Npad, zero padded), through a 32 x 32 shared-memory tile; block
+// (32, 8).
+template <typename T, typename W, bool GRAD>
+__global__ void value_prep_kernel(const W* __restrict__ w, const T* __restrict__ x,
                                   const float* __restrict__ mu, int64_t N, int64_t Npad, int D,
-                                  int Cv, int Cp, const unsigned* __restrict__ vmax_bits,
-                                  __half* __restrict__ vt, float* __restrict__ inv_scale) {
+                                  int Cw, int ch0, int Cc, int Cp,
+                                  const unsigned* __restrict__ vmax_bits, __half* __restrict__ vt,
+                                  float* __restrict__ inv_scale) {
     __shared__ float tile[32][33];
     const int64_t n0 = static_cast<int64_t>(blockIdx.x) * 32;
     const int c0 = blockIdx.y * 32;
@@ -578,7 +585,7 @@ __global__ void value_prep_kernel(const T* __restrict__ v, const T* __restrict__
         const int64_t n = n0 + threadIdx.y + 8 * i;
         const int c = c0 + threadIdx.x;
         float val = 0.f;
-        if (n < N && c < Cv) val = value_at<T, GRAD>(v, k, mu, n, c, D, Cv);
+        if (n < N && c < Cc) val = value_at<T, W, GRAD>(w, x, mu, n, ch0 + c, D, Cw);
         tile[threadIdx.y + 8 * i][threadIdx.x] = val;
     }
     __syncthreads();
@@ -587,13 +594,13 @@ __global__ void value_prep_kernel(const T* __restrict__ v, const T* __restrict__
         const int c = c0 + threadIdx.y + 8 * i;
         const int64_t n = n0 + threadIdx.x;
         if (c < Cp && n < Npad) {
-            const float sc = c < Cv ? pow2f(channel_exponent(vmax_bits[c])) : 0.f;
+            const float sc = c < Cc ? pow2f(channel_exponent(vmax_bits[c])) : 0.f;
             vt[static_cast<int64_t>(c) * Npad + n] = __float2half_rn(tile[threadIdx.x][threadIdx.y + 8 * i] * sc);
         }
     }
     if (blockIdx.x == 0 && threadIdx.y == 0) {
         const int c = c0 + threadIdx.x;
-        if (c < Cp) inv_scale[c] = c < Cv ? pow2f(-channel_exponent(vmax_bits[c])) : 0.f;
+        if (c < Cp) inv_scale[c] = c < Cc ? pow2f(-channel_exponent(vmax_bits[c])) : 0.f;
     }
 }
 
@@ -623,75 +630,108 @@ __global__ void key_record_kernel(const T* __restrict__ v, const float* __restri
 }
 
 // ---------------------------------------------------------------- finalise
-// part: splits blocks of split_stride_rows rows x part_ld floats.
-template <int MODE, typename T>
+// Forward: out[m, c] = inv_scale[c] sum_s part[s][m][c] (splits added in
+// order).  part: splits blocks of split_stride_rows rows x part_ld floats.
 __global__ void finalize_kernel(const float* __restrict__ part, int splits,
                                 int64_t split_stride_rows, int64_t M, int Cv, int part_ld,
-                                const float* __restrict__ inv_scale, const T* __restrict__ q,
-                                const float* __restrict__ mu, float tau, int D,
-                                float* __restrict__ out, float* __restrict__ s_out) {
-    const int64_t width = MODE == 0 ? Cv : D;
+                                const float* __restrict__ inv_scale, float* __restrict__ out) {
+    const int64_t idx = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
+    if (idx >= M * Cv) return;
+    const int64_t m = idx / Cv;
+    const int c = static_cast<int>(idx - m * Cv);
+    float acc = 0.f;
+    for (int s = 0; s < splits; ++s)
+        acc += part[(static_cast<int64_t>(s) * split_stride_rows + m) * part_ld + c];
+    out[idx] = acc * (inv_scale ? inv_scale[c] : 1.f);
+}
+
+// Gradient contraction for the channels ch0 .. ch0 + Cc - 1 of one launch
+// (channel ch = c (D + 1) + d, as in value_at).  With S_j the sum over
+// splits of partial channel j (times inv_scale[j] when given):
+//   out[m, d] (+)= tau sum_c u[m, c] (S_{c,d} - x^_{m,d} S_{c,D})
+//   s_out[m, c]   = S_{c,D}
+// where x^ = x - mu is the row's centred point.  DIRECT: the partials
+// already hold sum Phi w (k - x) (the fp32 kernel's difference form), so the
+// x^ S_{c,D} term is left out.  Terms whose channel lies outside this launch
+// are added by the launch that holds it (accumulate = 1 adds to out).  u
+// null means u = 1; out may be null when only s_out is wanted.  One thread
+// per (m, d) for d < max(D, 1).
+template <bool DIRECT, typename T, typename U>
+__global__ void finalize_points_kernel(const float* __restrict__ part, int splits,
+                                       int64_t split_stride_rows, int64_t M, int part_ld,
+                                       const float* __restrict__ inv_scale,
+                                       const T* __restrict__ x, const float* __restrict__ mu,
+                                       float tau, int D, int Cw, int ch0, int Cc,
+                                       const U* __restrict__ u, int accumulate,
+                                       float* __restrict__ out, float* __restrict__ s_out) {
+    const int width = D > 0 ? D : 1;
     const int64_t idx = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
     if (idx >= M * width) return;
     const int64_t m = idx / width;
-    const int c = static_cast<int>(idx - m * width);
-    auto sum_channel = [&](int ch) {
+    const int d = static_cast<int>(idx - m * width);
+    auto S = [&](int j) {
         float acc = 0.f;
         for (int s = 0; s < splits; ++s)
-            acc += part[(static_cast<int64_t>(s) * split_stride_rows + m) * part_ld + ch];
-        return acc;
+            acc += part[(static_cast<int64_t>(s) * split_stride_rows + m) * part_ld + j];
+        return inv_scale ? acc * inv_scale[j] : acc;
     };
-    if (MODE == 0) {
-        const float sc = inv_scale ? inv_scale[c] : 1.f;
-        out[idx] = sum_channel(c) * sc;
-    } else if (MODE == 1) {
-        const float sd = sum_channel(c) * inv_scale[c];
-        const float s0 = sum_channel(D) * inv_scale[D];
-        const float qc = to_f(q[m * D + c]) - (mu ? mu[c] : 0.f);
-        out[idx] = tau * (sd - qc * s0);
-        if (c == 0 && s_out) s_out[m] = s0;
-    } else {
-        out[idx] = tau * sum_channel(c);
-        if (c == 0 && s_out) s_out[m] = sum_channel(D);
+    const int G = D + 1;
+    const int c_lo = ch0 / G, c_hi = (ch0 + Cc - 1) / G;
+    const float xd = (DIRECT || d >= D) ? 0.f : to_f(x[m * D + d]) - (mu ? mu[d] : 0.f);
+    float acc = 0.f;
+    for (int c = c_lo; c <= c_hi; ++c) {
+        const int jd = c * G + d - ch0;
+        const int js = c * G + D - ch0;
+        const bool has_d = d < D && jd >= 0 && jd < Cc;
+        const bool has_s = js >= 0 && js < Cc;
+        if (!has_d && !(has_s && (d == 0 || !DIRECT))) continue;
+        const float ss = has_s ? S(js) : 0.f;
+        if (d == 0 && has_s && s_out) s_out[m * Cw + c] = ss;
+        if (d >= D) continue;
+        float t = has_d ? S(jd) : 0.f;
+        if (!DIRECT && has_s) t -= xd * ss;
+        acc += (u ? to_f(u[m * Cw + c]) : 1.f) * t;
     }
+    if (out && d < D) out[m * D + d] = (accumulate ? out[m * D + d] : 0.f) + tau * acc;
 }
 
-template <typename T, bool GRAD>
-cudaError_t value_prep_typed(const void* v, const void* k, const float* mu, int64_t N,
-                             int64_t Npad, int D, int Cv, int Cp, unsigned* vmax_bits, void* vt,
-                             float* inv_scale, cudaStream_t s) {
+template <typename T, typename W, bool GRAD>
+cudaError_t value_prep_typed(const void* w, const void* x, const float* mu, int64_t N,
+                             int64_t Npad, int D, int Cw, int ch0, int Cc, int Cp,
+                             unsigned* vmax_bits, void* vt, float* inv_scale, cudaStream_t s) {
     cudaError_t e = cudaMemsetAsync(vmax_bits, 0, sizeof(unsigned) * Cp, s);
     if (e != cudaSuccess) return e;
     const int64_t rows_per_block = 512;
     const int64_t blocks = N > 0 ? (N + rows_per_block - 1) / rows_per_block : 0;
     if (blocks > 0) {
-        value_max_kernel<T, GRAD><<<static_cast<unsigned>(blocks), dim3(32, 8), 0, s>>>(
-            static_cast<const T*>(v), static_cast<const T*>(k), mu, N, D, Cv, rows_per_block,
-            vmax_bits);
+        value_max_kernel<T, W, GRAD><<<static_cast<unsigned>(blocks), dim3(32, 8), 0, s>>>(
+            static_cast<const W*>(w), static_cast<const T*>(x), mu, N, D, Cw, ch0, Cc,
+            rows_per_block, vmax_bits);
         note_launches(1);
         e = cudaGetLastError();
         if (e != cudaSuccess) return e;
     }
     dim3 grid(static_cast<unsigned>((Npad + 31) / 32), static_cast<unsigned>((Cp + 31) / 32));
-    value_prep_kernel<T, GRAD><<<grid, dim3(32, 8), 0, s>>>(
-        static_cast<const T*>(v), static_cast<const T*>(k), mu, N, Npad, D, Cv, Cp, vmax_bits,
-        static_cast<__half*>(vt), inv_scale);
+    value_prep_kernel<T, W, GRAD><<<grid, dim3(32, 8), 0, s>>>(
+        static_cast<const W*>(w), static_cast<const T*>(x), mu, N, Npad, D, Cw, ch0, Cc, Cp,
+        vmax_bits, static_cast<__half*>(vt), inv_scale);
     note_launches(1);
     return cudaGetLastError();
 }
 
-template <int MODE, typename T>
-cudaError_t finalize_typed(const float* part, int splits, int64_t stride_rows, int64_t M, int Cv,
-                           int part_ld, const float* inv_scale, const void* q, const float* mu,
-                           float tau, int D, float* out, float* s_out, cudaStream_t s) {
-    const int64_t width = MODE == 0 ? Cv : D;
-    const int64_t total = M * width;
+template <bool DIRECT, typename T, typename U>
+cudaError_t finalize_points_typed(const float* part, int splits, int64_t stride_rows, int64_t M,
+                                  int part_ld, const float* inv_scale, const void* x,
+                                  const float* mu, float tau, int D, int Cw, int ch0, int Cc,
+                                  const void* u, int accumulate, float* out, float* s_out,
+                                  cudaStream_t s) {
+    const int64_t total = M * (D > 0 ? D : 1);
     if (total == 0) return cudaSuccess;
     const int threads = 256;
     const int64_t blocks = (total + threads - 1) / threads;
-    finalize_kernel<MODE, T><<<static_cast<unsigned>(blocks), threads, 0, s>>>(
-        part, splits, stride_rows, M, Cv, part_ld, inv_scale, static_cast<const T*>(q), mu, tau,
-        D, out, s_out);
+    finalize_points_kernel<DIRECT, T, U><<<static_cast<unsigned>(blocks), threads, 0, s>>>(
+        part, splits, stride_rows, M, part_ld, inv_scale, static_cast<const T*>(x), mu, tau, D,
+        Cw, ch0, Cc, static_cast<const U*>(u), accumulate, out, s_out);
     note_launches(1);
     return cudaGetLastError();
 }
@@ -821,19 +861,20 @@ cudaError_t launch_center_cast_norm(InType t, const void* x, int64_t rows, int64
                                         xh, nullptr, nrm, s, batch);
 }
 
-cudaError_t launch_value_prep(InType t, bool grad, const void* v, const void* k,
-                              const float* mu, int64_t N, int64_t Npad, int D, int Cv, int Cp,
-                              unsigned* vmax_bits, void* vt, float* inv_scale, cudaStream_t s) {
+cudaError_t launch_value_prep(InType t, bool grad, bool w_f32, const void* w, const void* x,
+                              const float* mu, int64_t N, int64_t Npad, int D, int Cw, int ch0,
+                              int Cc, int Cp, unsigned* vmax_bits, void* vt, float* inv_scale,
+                              cudaStream_t s) {
+#define GS_VALUE_PREP(T, W, G) \
+    value_prep_typed<T, W, G>(w, x, mu, N, Npad, D, Cw, ch0, Cc, Cp, vmax_bits, vt, inv_scale, s)
     if (t == InType::BF16) {
-        return grad ? value_prep_typed<__nv_bfloat16, true>(v, k, mu, N, Npad, D, Cv, Cp,
-                                                            vmax_bits, vt, inv_scale, s)
-                    : value_prep_typed<__nv_bfloat16, false>(v, k, mu, N, Npad, D, Cv, Cp,
-                                                             vmax_bits, vt, inv_scale, s);
+        if (!grad) return GS_VALUE_PREP(__nv_bfloat16, __nv_bfloat16, false);
+        return w_f32 ? GS_VALUE_PREP(__nv_bfloat16, float, true)
+                     : GS_VALUE_PREP(__nv_bfloat16, __nv_bfloat16, true);
     }
-    return grad ? value_prep_typed<__half, true>(v, k, mu, N, Npad, D, Cv, Cp, vmax_bits, vt,
-                                                 inv_scale, s)
-                : value_prep_typed<__half, false>(v, k, mu, N, Npad, D, Cv, Cp, vmax_bits, vt,
-                                                  inv_scale, s);
+    if (!grad) return GS_VALUE_PREP(__half, __half, false);
+    return w_f32 ? GS_VALUE_PREP(__half, float, true) : GS_VALUE_PREP(__half, __half, true);
+#undef GS_VALUE_PREP
 }
 
 cudaError_t launch_aug_prep(InType t, const void* x, int64_t rows, int64_t rows_pad, int D,
@@ -863,21 +904,33 @@ cudaError_t launch_key_records(InType t, const void* v, const float* B, int64_t 
     return cudaGetLastError();
 }
 
-cudaError_t launch_finalize(int mode, InType t, const float* part, int splits,
-                            int64_t split_stride_rows, int64_t M, int Cv, int part_ld,
-                            const float* inv_scale, const void* q, const float* mu, float tau,
-                            int D, float* out, float* s_out, cudaStream_t s) {
-    if (mode == 0)
-        return finalize_typed<0, float>(part, splits, split_stride_rows, M, Cv, part_ld,
-                                        inv_scale, nullptr, nullptr, tau, D, out, s_out, s);
-    if (mode == 2)
-        return finalize_typed<2, float>(part, splits, split_stride_rows, M, Cv, part_ld,
-                                        inv_scale, nullptr, nullptr, tau, D, out, s_out, s);
+cudaError_t launch_finalize(const float* part, int splits, int64_t split_stride_rows,
+                            int64_t M, int Cv, int part_ld, const float* inv_scale, float* out,
+                            cudaStream_t s) {
+    const int64_t total = M * Cv;
+    if (total == 0) return cudaSuccess;
+    const int threads = 256;
+    const int64_t blocks = (total + threads - 1) / threads;
+    finalize_kernel<<<static_cast<unsigned>(blocks), threads, 0, s>>>(
+        part, splits, split_stride_rows, M, Cv, part_ld, inv_scale, out);
+    note_launches(1);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_finalize_points(bool direct, InType t, bool u_f32, const float* part,
+                                   int splits, int64_t split_stride_rows, int64_t M, int part_ld,
+                                   const float* inv_scale, const void* x, const float* mu,
+                                   float tau, int D, int Cw, int ch0, int Cc, const void* u,
+                                   int accumulate, float* out, float* s_out, cudaStream_t s) {
+#define GS_FIN(DIR, T, U)                                                                     \
+    finalize_points_typed<DIR, T, U>(part, splits, split_stride_rows, M, part_ld, inv_scale, x, \
+                                     mu, tau, D, Cw, ch0, Cc, u, accumulate, out, s_out, s)
+    if (direct) return GS_FIN(true, float, float);
     if (t == InType::BF16)
-        return finalize_typed<1, __nv_bfloat16>(part, splits, split_stride_rows, M, Cv, part_ld,
-                                                inv_scale, q, mu, tau, D, out, s_out, s);
-    return finalize_typed<1, __half>(part, splits, split_stride_rows, M, Cv, part_ld, inv_scale,
-                                     q, mu, tau, D, out, s_out, s);
+        return u_f32 ? GS_FIN(false, __nv_bfloat16, float)
+                     : GS_FIN(false, __nv_bfloat16, __nv_bfloat16);
+    return u_f32 ? GS_FIN(false, __half, float) : GS_FIN(false, __half, __half);
+#undef GS_FIN
 }
 
 }  // namespace gs

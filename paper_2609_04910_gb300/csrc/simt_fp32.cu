@@ -9,7 +9,8 @@
 // value is 2^(-(c/2) d^2) with c = tau log2 e, and the values are
 // accumulated with fp32 FMAs:
 //   forward (Eq. 1):     acc[j] += Phi v[n, c0 + j]       for CBLK channels
-//   gradient (Sec. 3):   acc[d] += Phi v_n (k_d - q_d),   acc[D] += Phi v_n
+//   gradient (Sec. 3):   acc[d] += Phi w_n (k_d - q_d),   acc[D] += Phi w_n
+//                        with w_n = v[n, c] for one weight channel c
 // The key range is split over gridDim.y; partial sums go to a workspace and
 // are added in a fixed order by the finalise kernel.
 #include <algorithm>
@@ -27,7 +28,7 @@ template <int DMAX, int CBLK, bool GRAD>
 __global__ void __launch_bounds__(THREADS)
 simt_gauss_kernel(const float* __restrict__ q, const float* __restrict__ k,
                   const float* __restrict__ v, int64_t M, int64_t N, int D, int Cv,
-                  float half_c, int64_t keys_per_split, float* __restrict__ part) {
+                  int wch, float half_c, int64_t keys_per_split, float* __restrict__ part) {
     constexpr int NACC = GRAD ? DMAX + 1 : CBLK;
     __shared__ __align__(16) float ks[KT][DMAX];
     __shared__ float vs[KT][GRAD ? 1 : CBLK];
@@ -53,7 +54,9 @@ simt_gauss_kernel(const float* __restrict__ q, const float* __restrict__ k,
             ks[kk][d] = (kk < cnt && d < D) ? k[(t0 + kk) * D + d] : 0.f;
         }
         if (GRAD) {
-            for (int i = threadIdx.x; i < KT; i += THREADS) vs[i][0] = i < cnt ? v[t0 + i] : 0.f;
+            // v is N x Cv here; the weight is its channel wch.
+            for (int i = threadIdx.x; i < KT; i += THREADS)
+                vs[i][0] = i < cnt ? v[(t0 + i) * Cv + wch] : 0.f;
         } else {
             for (int i = threadIdx.x; i < KT * CBLK; i += THREADS) {
                 const int kk = i / CBLK, j = i - kk * CBLK;
@@ -107,13 +110,13 @@ simt_gauss_kernel(const float* __restrict__ q, const float* __restrict__ k,
 
 template <int DMAX, bool GRAD>
 cudaError_t launch_dmax(const SimtPlan& p, const float* q, const float* k, const float* v,
-                        float half_c, float* part, cudaStream_t s) {
+                        int Cw, int wch, float half_c, float* part, cudaStream_t s) {
     constexpr int CBLK = 4;
     dim3 grid(static_cast<unsigned>((p.M + THREADS - 1) / THREADS), p.splits,
               GRAD ? 1u : static_cast<unsigned>((p.Cv + CBLK - 1) / CBLK));
     simt_gauss_kernel<DMAX, CBLK, GRAD><<<grid, THREADS, 0, s>>>(
-        q, k, v, p.M, p.N, static_cast<int>(p.D), static_cast<int>(p.Cv), half_c,
-        p.keys_per_split, part);
+        q, k, v, p.M, p.N, static_cast<int>(p.D), GRAD ? Cw : static_cast<int>(p.Cv), wch,
+        half_c, p.keys_per_split, part);
     note_launches(1);
     return cudaGetLastError();
 }
@@ -151,19 +154,20 @@ bool plan_simt(int64_t M, int64_t N, int64_t D, int64_t C, bool grad, int split_
 }
 
 cudaError_t launch_simt(const SimtPlan& p, bool grad, const float* q, const float* k,
-                        const float* v, float half_c, float* part, cudaStream_t s) {
+                        const float* v, int Cw, int wch, float half_c, float* part,
+                        cudaStream_t s) {
     if (grad) {
         switch (p.dmax) {
-            case 16: return launch_dmax<16, true>(p, q, k, v, half_c, part, s);
-            case 32: return launch_dmax<32, true>(p, q, k, v, half_c, part, s);
-            default: return launch_dmax<64, true>(p, q, k, v, half_c, part, s);
+            case 16: return launch_dmax<16, true>(p, q, k, v, Cw, wch, half_c, part, s);
+            case 32: return launch_dmax<32, true>(p, q, k, v, Cw, wch, half_c, part, s);
+            default: return launch_dmax<64, true>(p, q, k, v, Cw, wch, half_c, part, s);
         }
     }
     switch (p.dmax) {
-        case 16: return launch_dmax<16, false>(p, q, k, v, half_c, part, s);
-        case 32: return launch_dmax<32, false>(p, q, k, v, half_c, part, s);
-        case 64: return launch_dmax<64, false>(p, q, k, v, half_c, part, s);
-        default: return launch_dmax<128, false>(p, q, k, v, half_c, part, s);
+        case 16: return launch_dmax<16, false>(p, q, k, v, 0, 0, half_c, part, s);
+        case 32: return launch_dmax<32, false>(p, q, k, v, 0, 0, half_c, part, s);
+        case 64: return launch_dmax<64, false>(p, q, k, v, 0, 0, half_c, part, s);
+        default: return launch_dmax<128, false>(p, q, k, v, 0, 0, half_c, part, s);
     }
 }
 

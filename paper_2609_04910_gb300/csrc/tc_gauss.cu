@@ -421,11 +421,12 @@ bool plan_tensor(InType t, int64_t M, int64_t N, int64_t D, int64_t C, bool grad
     p->M = M;
     p->N = N;
     p->D = D;
-    p->Cv = grad ? D + 1 : C;
+    // grad: C is the channel count of one launch (a chunk of C_w (D + 1)).
+    p->Cv = C;
     p->Dp = static_cast<int>(std::max<int64_t>(16, (D + 15) / 16 * 16));
     p->Cp = static_cast<int>((p->Cv + 15) / 16 * 16);
     if (D > 256) { *why = "tensor-core path supports D <= 256"; return false; }
-    if (p->Cp > 256) { *why = grad ? "gradient needs D + 1 <= 256" : "tensor-core path supports C <= 256"; return false; }
+    if (p->Cp > 256) { *why = "tensor-core path supports C <= 256"; return false; }
     p->alias = alias;
     p->center = center;
     const int nkb = (p->Dp + KB - 1) / KB;

@@ -201,3 +201,11 @@ def sample_rows(M: int, count: int, seed: int = 1) -> np.ndarray:
         return np.arange(M, dtype=np.int64)
     rng = np.random.default_rng(seed)
     return np.sort(rng.choice(M, size=count, replace=False)).astype(np.int64)
+
+
+def upstream(M: int, C: int, seed: int = 0) -> np.ndarray:
+    """Seeded float32 upstream gradient g (M x C) of a vector-Jacobian
+    product: standard normal entries, drawn from a stream separate from the
+    points' (seed offset 7919)."""
+    rng = np.random.default_rng(seed + 7919)
+    return np.ascontiguousarray(rng.standard_normal((M, C)).astype(np.float32))

@@ -11,7 +11,7 @@ import os
 import numpy as np
 import pytest
 
-from oracle import build_oracle, oracle_grad_q, oracle_sum
+from oracle import build_oracle, oracle_grad_q, oracle_sum, oracle_vjp
 from tests.paper_forms import prescale
 
 SRC = os.path.join(os.path.dirname(os.path.dirname(os.path.abspath(__file__))), "oracle",
@@ -23,13 +23,19 @@ MUTANTS = {
     "dropped_coordinate": ("for (int64_t d = 0; d < D; ++d) {\n        double t",
                            "for (int64_t d = 0; d < D - 1; ++d) {\n        double t"),
     "channel_index": ("sr[c] += phi * vn[c];", "sr[c] += phi * vn[0];"),
-    "value_stride": ("const double* vn = v + n * C;", "const double* vn = v + n;"),
+    "value_stride": ("D, tau);\n            const double* vn = v + n * C;",
+                     "D, tau);\n            const double* vn = v + n;"),
     "row_index": ("const double* qm = q + m * D;\n        double* sr",
                   "const double* qm = q + r * D;\n        double* sr"),
     "grad_sign": ("gr[d] += w * (kn[d] - qm[d]);", "gr[d] += w * (qm[d] - kn[d]);"),
     "grad_factor": ("gr[d] *= tau;", "gr[d] *= 0.5 * tau;"),
     "transposed_key": ("double phi = gauss_kernel(qm, k + n * D, D, tau);",
                        "double phi = gauss_kernel(qm, k + n, D, tau);"),
+    "vjp_k_sign": ("outk[d] += phi * w * (qm[d] - kn[d]);", "outk[d] += phi * w * (kn[d] - qm[d]);"),
+    "vjp_v_upstream": ("if (outv) outv[c] += phi * gm[c];", "if (outv) outv[c] += phi * vn[c];"),
+    "vjp_q_contraction": ("w += gm[c] * vn[c];", "w += gm[0] * vn[c];"),
+    "vjp_k_contraction": ("w += vn[c] * gm[c];", "w += vn[c] * gm[c] * (c == 0);"),
+    "vjp_q_factor": ("if (out) out[d] *= tau;", "if (out) out[d] *= 0.5 * tau;"),
 }
 
 
@@ -72,6 +78,26 @@ def _pin_failures(lib):
         if abs(fd - g[0, d]) > 1e-6 * (1 + abs(fd)):
             fails.append("grad_fd")
             break
+    # vector-Jacobian product vs finite differences of sum_m g_m . s_m
+    q = rng.standard_normal((3, 2))
+    k = rng.standard_normal((4, 2))
+    v = rng.standard_normal((4, 2))
+    up = rng.standard_normal((3, 2))
+    r = oracle_vjp(q, k, v, up, 0.8, lib_path=lib)
+
+    def loss(qq, kk, vv):
+        return float(np.sum(up * oracle_sum(qq, kk, vv, 0.8, lib_path=lib)[0]))
+
+    for arr, got, which in ((q, r["gq"], 0), (k, r["gk"], 1), (v, r["gv"], 2)):
+        for idx in np.ndindex(arr.shape):
+            args_p = [q.copy(), k.copy(), v.copy()]
+            args_m = [q.copy(), k.copy(), v.copy()]
+            args_p[which][idx] += h
+            args_m[which][idx] -= h
+            fd = (loss(*args_p) - loss(*args_m)) / (2 * h)
+            if abs(fd - got[idx]) > 1e-6 * (1 + abs(fd)):
+                fails.append(f"vjp_fd_{which}")
+                break
     return fails
 
 
