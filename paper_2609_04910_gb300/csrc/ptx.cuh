@@ -405,4 +405,45 @@ __device__ __forceinline__ uint64_t f32x2_add(uint64_t a, uint64_t b) {
     return d;
 }
 
+__device__ __forceinline__ uint64_t f32x2_sub(uint64_t a, uint64_t b) {
+    uint64_t d;
+    asm("sub.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+    return d;
+}
+
+__device__ __forceinline__ uint64_t f32x2_mul_ftz(uint64_t a, uint64_t b) {
+    uint64_t d;
+    asm("mul.rn.ftz.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+    return d;
+}
+
+// 2^(c s) for a pair (s0, s1) on the FMA pipe, without the MUFU unit.
+// Cody-Waite reduction by an integer: j = round(c s) comes from adding
+// 1.5 * 2^23 (the sum's low mantissa bits are j), f = c s - j lies in
+// [-1/2, 1/2] and is exact (one fma); 2^f is a degree-4 polynomial of
+// minimax relative error 2.7e-6 on that interval (fitted by the Remez
+// exchange in fit_exp2_poly.py, coefficients rounded to float32); 2^j is
+// built in the exponent field and applied by one flush-to-zero multiply.
+// s_min = -127 / c keeps j >= -127: results below 2^-126 flush to 0, as
+// those of ex2.approx.ftz do.  Eleven issue slots for the pair, none on the
+// MIO path that MUFU instructions share with shared-memory traffic.
+__device__ __forceinline__ uint64_t exp2_fma_x2(float s0, float s1, uint64_t c2, float s_min) {
+    const uint64_t s2 = f32x2_pack(fmaxf(s0, s_min), fmaxf(s1, s_min));
+    const float kMagic = 12582912.0f;   // 1.5 * 2^23
+    const uint64_t magic = f32x2_pack(kMagic, kMagic);
+    const uint64_t t = f32x2_fma(s2, c2, magic);   // magic + j
+    const uint64_t f = f32x2_fma(s2, c2, f32x2_sub(magic, t));
+    uint64_t p = f32x2_fma(f, f32x2_pack(9.570102207e-03f, 9.570102207e-03f),
+                           f32x2_pack(5.591785908e-02f, 5.591785908e-02f));
+    p = f32x2_fma(p, f, f32x2_pack(2.402474433e-01f, 2.402474433e-01f));
+    p = f32x2_fma(p, f, f32x2_pack(6.931217909e-01f, 6.931217909e-01f));
+    p = f32x2_fma(p, f, f32x2_pack(9.999992847e-01f, 9.999992847e-01f));
+    float t0, t1;
+    f32x2_unpack(t, t0, t1);
+    // (magic + j) << 23 leaves j << 23 (mod 2^32); + 127 << 23 gives 2^j.
+    const float e0 = __uint_as_float(__float_as_uint(t0) * (1u << 23) + 0x3f800000u);
+    const float e1 = __uint_as_float(__float_as_uint(t1) * (1u << 23) + 0x3f800000u);
+    return f32x2_mul_ftz(p, f32x2_pack(e0, e1));
+}
+
 }  // namespace gs

@@ -60,6 +60,12 @@ constexpr int NQ = 2;              // query tiles per CTA
 constexpr int BN = 128;            // keys per key tile (MMA N)
 constexpr int KB = 64;             // 16-bit elements per 128-byte swizzled row
 constexpr int NEXP = 16;
+// Exponentials on the FMA pipe (exp2_fma_x2) instead of MUFU, augmented
+// path: the pair of row 0 (kSoftExpX) or row 1 (kSoftExpY) of key pair t
+// takes the FMA route when (t & mask) == 0; -1: never.  Each mask m moves
+// 1 / (4 (m + 1)) of the exponentials.
+constexpr int kSoftExpX = -1;
+constexpr int kSoftExpY = -1;
 constexpr int CTRL_WARP0 = 16;     // control warps 16..19, one per SMSP
 constexpr int NCTRL_MAX = 4;
 constexpr int THREADS = (NEXP + NCTRL_MAX) * 32;
@@ -376,6 +382,7 @@ tc_gauss_fma_kernel(const __grid_constant__ CUtensorMap tm_q,
             const uint64_t a2_0 = f32x2_pack(am0, am0);
             const uint64_t a2_1 = f32x2_pack(am1, am1);
             const uint64_t c2 = f32x2_pack(p.c, p.c);
+            const float s_min = -127.0f / p.c;   // exp2_fma_x2 range limit
             uint64_t acc0[C], acc1[C];
     #pragma unroll
             for (int cc = 0; cc < C; ++cc) acc0[cc] = acc1[cc] = 0ull;
@@ -423,11 +430,21 @@ tc_gauss_fma_kernel(const __grid_constant__ CUtensorMap tm_q,
     #pragma unroll
                     for (int t = 0; t < 16; ++t) {
                         const float* pr = rec + t * REC_PAIR;
-                        float x0, x1, y0, y1;
-                        f32x2_unpack(f32x2_mul(f32x2_pack(__uint_as_float(r0[2 * t]), __uint_as_float(r0[2 * t + 1])), c2), x0, x1);
-                        f32x2_unpack(f32x2_mul(f32x2_pack(__uint_as_float(r1[2 * t]), __uint_as_float(r1[2 * t + 1])), c2), y0, y1);
-                        const uint64_t px = f32x2_pack(ex2_approx(x0), ex2_approx(x1));
-                        const uint64_t py = f32x2_pack(ex2_approx(y0), ex2_approx(y1));
+                        uint64_t px, py;
+                        if (kSoftExpX >= 0 && (t & kSoftExpX) == 0) {
+                            px = exp2_fma_x2(__uint_as_float(r0[2 * t]), __uint_as_float(r0[2 * t + 1]), c2, s_min);
+                        } else {
+                            float x0, x1;
+                            f32x2_unpack(f32x2_mul(f32x2_pack(__uint_as_float(r0[2 * t]), __uint_as_float(r0[2 * t + 1])), c2), x0, x1);
+                            px = f32x2_pack(ex2_approx(x0), ex2_approx(x1));
+                        }
+                        if (kSoftExpY >= 0 && (t & kSoftExpY) == 0) {
+                            py = exp2_fma_x2(__uint_as_float(r1[2 * t]), __uint_as_float(r1[2 * t + 1]), c2, s_min);
+                        } else {
+                            float y0, y1;
+                            f32x2_unpack(f32x2_mul(f32x2_pack(__uint_as_float(r1[2 * t]), __uint_as_float(r1[2 * t + 1])), c2), y0, y1);
+                            py = f32x2_pack(ex2_approx(y0), ex2_approx(y1));
+                        }
     #pragma unroll
                         for (int cc = 0; cc < C; ++cc) {
                             const float2 vc = *reinterpret_cast<const float2*>(pr + 2 * cc);
