@@ -31,10 +31,14 @@
  *    cudaMallocAsync on `stream` and frees it with cudaFreeAsync on the same
  *    stream.
  *  - M = 0 is a no-op; N = 0 writes zeros.
- *  - fp16/bf16 inputs run on the tensor-core kernel (tcgen05, sm_103a) and
+ *  - fp16/bf16 inputs run on the tensor-core kernels (tcgen05, sm_103a) and
  *    need D <= 256 and C <= 256 (gradients: D <= 256, any C).  fp32 inputs
  *    run on the fp32 SIMT kernel (D <= 128 forward, D <= 64 gradients, any
- *    C).
+ *    C) or, for forward sums with C <= 4 and D <= 32, on the tensor cores
+ *    with three tf32 MMAs per product (q^ k^T ~ hi.hi + hi.lo + lo.hi of the
+ *    tf32 splits x = hi + lo, fp32-level accuracy): chosen automatically
+ *    from 2^25 pairs (per call, summed over a batch), or forced with
+ *    GS_PATH_TENSOR / GS_PATH_SIMT.
  *  - On a non-OK return gauss_sum_last_error() describes the failure.
  */
 #ifndef GAUSS_SUM_H
@@ -75,9 +79,12 @@ typedef enum { GS_PATH_AUTO = 0, GS_PATH_TENSOR = 1, GS_PATH_SIMT = 2 } gs_path;
  *  workspace       caller-owned device buffer of workspace_bytes bytes
  *                  (256-byte aligned) used instead of an allocation; its
  *                  required size is gauss_sum_workspace_size().
- *  path            GS_PATH_AUTO picks the tensor-core kernel for fp16/bf16
- *                  and the SIMT kernel for fp32; GS_PATH_TENSOR rejects fp32,
- *                  GS_PATH_SIMT rejects fp16/bf16.
+ *  path            GS_PATH_AUTO picks the tensor-core kernels for fp16/bf16
+ *                  and, for fp32, the 3xTF32 tensor-core variant for large
+ *                  forward sums with C <= 4 and D <= 32, else the SIMT
+ *                  kernel; GS_PATH_TENSOR takes fp32 only within that
+ *                  range (GS_ERR_UNSUPPORTED otherwise); GS_PATH_SIMT
+ *                  rejects fp16/bf16.
  *  main_events     measurement hook: two cudaEvent_t handles (or NULL) that
  *                  the call records on `stream` immediately before and after
  *                  the launch of its main kernel (the fused tensor-core

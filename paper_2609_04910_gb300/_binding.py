@@ -163,7 +163,7 @@ def _check_tensor(t, name):
 
 
 def gauss_sum(q, k, v, tau, out=None, stream=None, center=True, split_n=0, workspace=None,
-              main_events=None):
+              main_events=None, path=GS_PATH_AUTO):
     """Eq. 1: s[m] = sum_n exp(-tau/2 ||q_m - k_n||^2) v[n] as an (M, C) fp32 tensor.
 
     q: (M, D), k: (N, D), v: (N, C) or (N,) CUDA tensors of one dtype
@@ -181,7 +181,7 @@ def gauss_sum(q, k, v, tau, out=None, stream=None, center=True, split_n=0, works
     opt = options(center=center, split_n=split_n,
                   workspace=None if workspace is None else workspace.data_ptr(),
                   workspace_bytes=0 if workspace is None else workspace.numel() * workspace.element_size(),
-                  main_events=main_events)
+                  main_events=main_events, path=path)
     st = lib.gauss_sum_ex(_ptr(q), _ptr(k), _ptr(v), float(tau), M, N, D, C, _dtype_code(q),
                           _ptr(out), _stream_ptr(stream), ctypes.byref(opt))
     _check(lib, st)
@@ -300,9 +300,10 @@ def gauss_sum_grad_q(q, k, v, tau, grad=None, s_out=None, want_s=True, stream=No
     return grad, s_out
 
 
-def gauss_sum_workspace_size(M, N, D, C, dtype_code, grad=False, center=True, split_n=0):
+def gauss_sum_workspace_size(M, N, D, C, dtype_code, grad=False, center=True, split_n=0,
+                             path=GS_PATH_AUTO):
     lib = load_library()
-    opt = options(center=center, split_n=split_n)
+    opt = options(center=center, split_n=split_n, path=path)
     return int(lib.gauss_sum_workspace_size(M, N, D, C, dtype_code, 1 if grad else 0,
                                             ctypes.byref(opt)))
 

@@ -105,10 +105,12 @@ gs_status validate(const Call& c) {
     if (!aligned16(c.q) || !aligned16(c.k) || !aligned16(c.v) || !aligned16(c.out) ||
         !aligned16(c.s_out) || !aligned16(c.u))
         return fail(GS_ERR_INVALID_ARGUMENT, "base pointers must be 16-byte aligned");
-    if (c.opt.path == GS_PATH_TENSOR && c.dtype == GS_FP32)
-        return fail(GS_ERR_UNSUPPORTED, "the tensor-core path takes fp16/bf16 inputs");
     if (c.opt.path == GS_PATH_SIMT && c.dtype != GS_FP32)
         return fail(GS_ERR_UNSUPPORTED, "the SIMT path takes fp32 inputs");
+    if (c.opt.path == GS_PATH_TENSOR && c.dtype == GS_FP32 &&
+        (c.grad || c.C > gs::kFmaMaxChannels || c.D > gs::kTf32MaxDp))
+        return fail(GS_ERR_UNSUPPORTED,
+                    "the fp32 tensor-core path takes the forward sum with C <= 4 and D <= 32");
     if (c.opt.path < 0 || c.opt.path > 2) return fail(GS_ERR_INVALID_ARGUMENT, "unknown path");
     if (c.opt.split_n < 0) return fail(GS_ERR_INVALID_ARGUMENT, "split_n must be >= 0");
     if (c.opt.workspace && (reinterpret_cast<uintptr_t>(c.opt.workspace) & 255u))
@@ -129,11 +131,26 @@ gs::InType in_type(gs_dtype d) {
     return d == GS_FP16 ? gs::InType::F16 : d == GS_BF16 ? gs::InType::BF16 : gs::InType::F32;
 }
 
+// fp32 inputs go to the tensor cores (3xTF32) when the path is chosen
+// explicitly, or automatically for forward sums that the variant covers
+// and that are large enough to repay its extra operand kernels (measured
+// on a GB300 at D = 16, C = 1: 4096^2 pairs take 0.157 ms through the
+// tensor-core path and 0.136 ms through the SIMT kernel; 16384^2 pairs
+// 0.197 ms and 0.571 ms).
+constexpr int64_t kFp32TensorMinPairs = int64_t(1) << 25;
+
+bool fp32_on_tensor_cores(const Call& c) {
+    if (c.opt.path == GS_PATH_TENSOR) return true;
+    if (c.opt.path != GS_PATH_AUTO) return false;
+    return !c.grad && c.C <= gs::kFmaMaxChannels && c.D <= gs::kTf32MaxDp &&
+           c.B * c.M * c.N >= kFp32TensorMinPairs;
+}
+
 // Plans the call; returns GS_OK and the workspace size, or an error.
 gs_status plan(const Call& c, int sms, bool* tensor, gs::TcPlan* tp, gs::SimtPlan* sp,
                size_t* bytes) {
     const char* why = "unsupported shape";
-    *tensor = c.dtype != GS_FP32;
+    *tensor = c.dtype != GS_FP32 || fp32_on_tensor_cores(c);
     if (*tensor) {
         const bool alias = c.q == c.k && c.M == c.N && c.q != nullptr;
         int64_t nch = 1;
@@ -182,16 +199,14 @@ gs_status run(Call c) {
     unsigned* status = nullptr;
     cudaError_t e = device_info(&dev, &status);
     if (e != cudaSuccess) return cuda_fail(e, "device query");
-    const bool tensor_path = c.dtype != GS_FP32;
-    if (tensor_path && g_is_sm103[dev] != 1)
-        return fail(GS_ERR_UNSUPPORTED, "the tensor-core kernel needs an sm_103 (GB300) GPU");
-
     bool tensor = false;
     gs::TcPlan tp{};
     gs::SimtPlan sp{};
     size_t bytes = 0;
     st = plan(c, g_sm_count[dev], &tensor, &tp, &sp, &bytes);
     if (st != GS_OK) return st;
+    if (tensor && g_is_sm103[dev] != 1)
+        return fail(GS_ERR_UNSUPPORTED, "the tensor-core kernel needs an sm_103 (GB300) GPU");
     if (c.B > 1 && !(tensor && tp.fma)) {
         // Only the FMA kernel takes a batch in one launch: the problems of a
         // batch run one after another on the stream.
@@ -242,7 +257,23 @@ gs_status run(Call c) {
             where = "mean kernel";
         }
         const float ninf = -INFINITY;
-        if (e == cudaSuccess && tp.aug) {
+        if (e == cudaSuccess && tp.tf) {
+            // 3xTF32 operands: hi / lo tf32 halves and the norm terms.
+            e = gs::launch_tf32_split(static_cast<const float*>(c.q), c.M, tp.Mpad,
+                                      static_cast<int>(c.D), tp.Dp, mu, half_c,
+                                      reinterpret_cast<float*>(ws + tp.off_qh),
+                                      reinterpret_cast<float*>(ws + tp.off_A), ninf, c.stream,
+                                      batch);
+            where = "tf32 split kernel (q)";
+            if (e == cudaSuccess && !tp.alias) {
+                e = gs::launch_tf32_split(static_cast<const float*>(c.k), c.N, tp.Npad,
+                                          static_cast<int>(c.D), tp.Dp, mu, half_c,
+                                          reinterpret_cast<float*>(ws + tp.off_kh),
+                                          reinterpret_cast<float*>(ws + tp.off_B), ninf,
+                                          c.stream, batch);
+                where = "tf32 split kernel (k)";
+            }
+        } else if (e == cudaSuccess && tp.aug) {
             // Augmented operands: centred points with the norms folded in.
             e = gs::launch_aug_prep(t, c.q, c.M, tp.Mpad, static_cast<int>(c.D), tp.Dp, mu,
                                     ws + tp.off_qh, tp.alias ? ws + tp.off_kh : nullptr, c.stream,

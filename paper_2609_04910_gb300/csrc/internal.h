@@ -32,6 +32,8 @@ struct TcPlan {
     bool fma;                // kernel of tc_gauss_fma.cu (C <= kFmaMaxChannels, forward)
     bool aug;                // FMA kernel with augmented operands (Dp = D + 2 aug_norm_terms
                              // rounded to 16)
+    bool tf;                 // fp32 inputs on the FMA kernel with 3xTF32 MMAs: q^ and k^
+                             // rows are [hi | lo] of Dp (a multiple of 32) floats each
     int nq;                  // query tiles of 128 rows per CTA (FMA kernel)
     // FMA kernel work split: units = (pairs of query tiles) x key tiles, in
     // row-major order; CTA i takes units [i unit_len, (i + 1) unit_len); the
@@ -117,6 +119,11 @@ cudaError_t launch_simt(const SimtPlan& p, bool grad, const float* q, const floa
 // v_2t[C-1], v_2t+1[C-1].
 cudaError_t launch_key_records(InType t, const void* v, const float* B, int64_t N, int64_t Npad,
                                int C, float* rec, cudaStream_t s, int batch = 1);
+// 3xTF32 operands of fp32 inputs (see prep.cu): rows of 2 Dp floats
+// [hi | lo] into out, nrm = -(c/2)||x - mu||^2 (pad_value for padded rows).
+cudaError_t launch_tf32_split(const float* x, int64_t rows, int64_t rows_pad, int D, int Dp,
+                              const float* mu, float half_c, float* out, float* nrm,
+                              float pad_value, cudaStream_t s, int batch = 1);
 // Augmented MMA operands (see prep.cu): query layout into out_q, key layout
 // into out_k (either may be null), Dpa >= D + 2 aug_norm_terms(t) columns
 // per row.
@@ -133,7 +140,10 @@ cudaError_t launch_tc(const TcPlan& p, InType t, float c, char* ws, unsigned* st
 // Largest (augmented) Dp for which the FMA kernel keeps q^ in shared memory
 // and folds the norms into the MMA.
 constexpr int kAugMaxDp = 128;
-bool plan_fma_kernel(int Dp, int C, bool aug, int* nq, int* stages, size_t* smem);
+// Largest D of the 3xTF32 (fp32) variant: q^ hi and lo tiles of two query
+// tiles stay in shared memory next to the key stages.
+constexpr int kTf32MaxDp = 32;
+bool plan_fma_kernel(int Dp, int C, bool aug, bool tf, int* nq, int* stages, size_t* smem);
 cudaError_t launch_tc_fma(const TcPlan& p, InType t, float c, char* ws, unsigned* status,
                           cudaStream_t s, const char** why);
 

@@ -21,6 +21,7 @@
 #include <math_constants.h>
 
 #include "internal.h"
+#include "ptx.cuh"
 
 namespace gs {
 namespace {
@@ -332,6 +333,39 @@ operand_kernel(const T* __restrict__ x, int64_t rows, int64_t rows_pad, int D, i
         uint4* dst = reinterpret_cast<uint4*>(out_k + r0 * Dp);
         for (int i = tid; i < nvec; i += kOperandThreads) dst[i] = reinterpret_cast<const uint4*>(sk)[i];
     }
+}
+
+// 3xTF32 operands (fp32 inputs on the tensor cores).  Row r of problem b
+// becomes 2 Dp floats [hi_0 .. hi_Dp-1, lo_0 .. lo_Dp-1] with
+// x^ = x - mu (fp32), hi = x^ rounded to tf32 and lo = (x^ - hi) rounded to
+// tf32, zero padded; q^.k^ is then hi.hi + hi.lo + lo.hi up to the dropped
+// lo.lo term (2^-22 relative).  nrm = -(c/2) ||x^||^2 from the fp32 x^;
+// rows in [rows, rows_pad) are zero with norm pad_value.  One warp per row,
+// over all problems of a batch.
+__global__ void tf32_split_kernel(const float* __restrict__ x, int64_t rows, int64_t rows_pad,
+                                  int64_t total_rows, int D, int Dp,
+                                  const float* __restrict__ mu, float half_c, float pad_value,
+                                  float* __restrict__ out, float* __restrict__ nrm) {
+    const int64_t w = (static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
+    const int lane = threadIdx.x & 31;
+    if (w >= total_rows) return;
+    const int64_t b = w / rows_pad;
+    const int64_t r = w - b * rows_pad;
+    const bool valid = r < rows;
+    const float* xr = x + (b * rows + r) * D;
+    const float* mb = mu ? mu + b * D : nullptr;
+    float* o = out + w * 2 * Dp;
+    float acc = 0.f;
+    for (int d = lane; d < Dp; d += 32) {
+        const float xv = (valid && d < D) ? xr[d] - (mb ? mb[d] : 0.f) : 0.f;
+        const float hi = round_tf32(xv);
+        o[d] = hi;
+        o[Dp + d] = round_tf32(xv - hi);
+        acc = fmaf(xv, xv, acc);
+    }
+#pragma unroll
+    for (int s = 16; s > 0; s >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, s);
+    if (lane == 0) nrm[w] = valid ? -half_c * acc : pad_value;
 }
 
 __global__ void finalize_slots_kernel(const float* __restrict__ part, int64_t Mpad, int64_t M,
@@ -861,6 +895,19 @@ cudaError_t launch_center_cast_norm(InType t, const void* x, int64_t rows, int64
                                         xh, nullptr, nrm, s, batch);
 }
 
+cudaError_t launch_tf32_split(const float* x, int64_t rows, int64_t rows_pad, int D, int Dp,
+                              const float* mu, float half_c, float* out, float* nrm,
+                              float pad_value, cudaStream_t s, int batch) {
+    const int64_t total = rows_pad * batch;
+    if (total == 0) return cudaSuccess;
+    const int threads = 256;
+    const int64_t blocks = (total * 32 + threads - 1) / threads;
+    tf32_split_kernel<<<static_cast<unsigned>(blocks), threads, 0, s>>>(
+        x, rows, rows_pad, total, D, Dp, mu, half_c, pad_value, out, nrm);
+    note_launches(1);
+    return cudaGetLastError();
+}
+
 cudaError_t launch_value_prep(InType t, bool grad, bool w_f32, const void* w, const void* x,
                               const float* mu, int64_t N, int64_t Npad, int D, int Cw, int ch0,
                               int Cc, int Cp, unsigned* vmax_bits, void* vt, float* inv_scale,
@@ -897,6 +944,9 @@ cudaError_t launch_key_records(InType t, const void* v, const float* B, int64_t 
     if (t == InType::BF16)
         key_record_kernel<__nv_bfloat16><<<dim3(blocks, batch), threads, 0, s>>>(
             static_cast<const __nv_bfloat16*>(v), B, N, pairs, C, rec);
+    else if (t == InType::F32)
+        key_record_kernel<float><<<dim3(blocks, batch), threads, 0, s>>>(
+            static_cast<const float*>(v), B, N, pairs, C, rec);
     else
         key_record_kernel<__half><<<dim3(blocks, batch), threads, 0, s>>>(static_cast<const __half*>(v), B, N,
                                                              pairs, C, rec);

@@ -306,6 +306,8 @@ tc_gauss_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant_
             for (int ch = 0; ch < NCH; ++ch)
                 tmem_ld_32x32b_x32(tmem + lane_base + S_col0 + b * BN + col0 + ch * 32, r[ch]);
             tmem_wait_ld();
+#pragma unroll
+            for (int ch = 0; ch < NCH; ++ch) tmem_regs_ready(r[ch]);
             const float* Bs = b_smem(s) + col0;
 #pragma unroll
             for (int ch = 0; ch < NCH; ++ch) {
@@ -347,6 +349,7 @@ tc_gauss_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant_
                 uint32_t r[8];
                 tmem_ld_32x32b_x8(tmem + lane_base + O_col + c8, r);
                 tmem_wait_ld();
+                tmem_regs_ready(r);
                 float4 lo = make_float4(__uint_as_float(r[0]) * P_UNSHIFT, __uint_as_float(r[1]) * P_UNSHIFT,
                                         __uint_as_float(r[2]) * P_UNSHIFT, __uint_as_float(r[3]) * P_UNSHIFT);
                 float4 hi = make_float4(__uint_as_float(r[4]) * P_UNSHIFT, __uint_as_float(r[5]) * P_UNSHIFT,
@@ -429,20 +432,42 @@ bool plan_tensor(InType t, int64_t M, int64_t N, int64_t D, int64_t C, bool grad
     if (p->Cp > 256) { *why = "tensor-core path supports C <= 256"; return false; }
     p->alias = alias;
     p->center = center;
+    p->tf = false;
     const int nkb = (p->Dp + KB - 1) / KB;
     size_t fma_smem = 0;
     int fma_stages = 0, nq = 1;
+    if (t == InType::F32) {
+        // fp32 inputs on the tensor cores: the FMA kernel with 3xTF32 MMAs
+        // (forward sum, few channels, small D).
+        if (grad || p->Cv > kFmaMaxChannels || D > kTf32MaxDp) {
+            *why = "the fp32 tensor-core path takes the forward sum with C <= 4 and D <= 32";
+            return false;
+        }
+        p->tf = true;
+        p->aug = false;
+        p->Dp = 32;
+        if (!plan_fma_kernel(p->Dp, static_cast<int>(p->Cv), false, true, &nq, &fma_stages,
+                             &fma_smem)) {
+            *why = "shared-memory budget exceeded";
+            return false;
+        }
+    }
     // Few channels: FMA-pipe kernel.  When the augmented rows fit in 128
     // columns it takes the augmented operands (q^ in shared memory, norms
     // folded into the MMA).
     const int dp_aug = static_cast<int>((D + 2 * aug_norm_terms(t) + 15) / 16 * 16);
-    p->aug = !grad && p->Cv <= kFmaMaxChannels && dp_aug <= kAugMaxDp;
-    const int dp_fma = p->aug ? dp_aug : p->Dp;
-    p->fma = !grad && p->Cv <= kFmaMaxChannels &&
-             plan_fma_kernel(dp_fma, static_cast<int>(p->Cv), p->aug, &nq, &fma_stages, &fma_smem);
-    if (!p->fma) p->aug = false;
+    if (p->tf) {
+        p->fma = true;
+    } else {
+        p->aug = !grad && p->Cv <= kFmaMaxChannels && dp_aug <= kAugMaxDp;
+        const int dp_fma = p->aug ? dp_aug : p->Dp;
+        p->fma = !grad && p->Cv <= kFmaMaxChannels &&
+                 plan_fma_kernel(dp_fma, static_cast<int>(p->Cv), p->aug, false, &nq, &fma_stages,
+                                 &fma_smem);
+        if (!p->fma) p->aug = false;
+    }
     if (p->fma) {
-        p->Dp = dp_fma;
+        if (!p->tf) p->Dp = p->aug ? dp_aug : p->Dp;
         p->BN = 128;
         p->nq = nq;
         p->stages = fma_stages;
@@ -529,11 +554,13 @@ bool plan_tensor(InType t, int64_t M, int64_t N, int64_t D, int64_t C, bool grad
     auto take = [&](size_t bytes) { size_t o = off; off = align1k(off + bytes); return o; };
     p->off_mean_part = take(static_cast<size_t>(B) * p->mean_blocks * D * 2 * 4);
     p->off_mu = take(static_cast<size_t>(B) * D * 4);
-    p->off_qh = take(static_cast<size_t>(B) * p->Mpad * p->Dp * 2);
+    // Operand rows: Dp 16-bit values, or (3xTF32) hi and lo halves of Dp floats.
+    const size_t row_bytes = p->tf ? static_cast<size_t>(p->Dp) * 8 : static_cast<size_t>(p->Dp) * 2;
+    p->off_qh = take(static_cast<size_t>(B) * p->Mpad * row_bytes);
     // Augmented query and key operands differ in their extra columns, so
     // they are separate arrays even when q and k are the same points.
     p->off_kh = (alias && !p->aug) ? p->off_qh
-                                   : take(static_cast<size_t>(B) * p->Npad * p->Dp * 2);
+                                   : take(static_cast<size_t>(B) * p->Npad * row_bytes);
     if (p->aug) {
         p->off_A = p->off_B = 0;   // the norms live in the augmented columns
     } else {

@@ -17,9 +17,9 @@
 //     record serves two kernel values.
 //   * One barrier handshake per key tile: the 2 x (Dp / 16) MMAs of a key
 //     tile are issued back to back and committed once; the exponent warps
-//     release both S buffers of the key tile with one arrival per warp, as
-//     soon as they are in registers, and query the next key tile's
-//     barriers before exponentiating the current one.
+//     release both S buffers and the stage of the key tile with one
+//     arrival per warp on each barrier once the tile is done, and query the
+//     next key tile's barriers before exponentiating the current one.
 //   * TMEM holds SL slots of two 128-column S buffers (one per query
 //     tile); key tile j uses slot j % SL, so the MMAs of key tile j only
 //     wait for the release of key tile j - SL.  With Dp <= 128 the query
@@ -94,7 +94,9 @@ struct FmaParams {
     int pairs_per_batch; // pairs of query tiles per problem of a batch
     int npad;            // k^ rows per problem of a batch
     int Dp;
-    int nkb;             // 64-element K blocks of q^ / k^
+    int nkb;             // 128-byte K blocks of a q^ / k^ row (TF: hi blocks, then lo)
+    int kb_elems;        // elements per K block (64 16-bit, 32 fp32)
+    int ksteps;          // MMA K steps over the coordinates (16 fp16/bf16, 8 tf32 each)
     int stages;
     uint32_t q_bytes;    // shared-memory q^ tiles (0 when q^ is in TMEM)
     uint32_t stage_bytes;
@@ -128,10 +130,12 @@ __device__ __forceinline__ void exp_warps_sync() {
 // AUG: augmented operands (S = -||q^ - k^||^2 / 2; no norm terms in the
 // key records).  QSM: q^ tiles in shared memory (A operand from shared
 // memory, SL = 2); otherwise q^ in TMEM (A operand from TMEM, SL = 1).
-template <int C, bool AUG, bool QSM>
+template <int C, bool AUG, bool QSM, bool TF>
 __global__ void __launch_bounds__(THREADS, 1)
 tc_gauss_fma_kernel(const __grid_constant__ CUtensorMap tm_q,
                     const __grid_constant__ CUtensorMap tm_k, const FmaParams p) {
+    // TF (3xTF32): q^ in shared memory, norm terms from A and the records.
+    static_assert(!TF || (QSM && !AUG), "3xTF32 runs with q^ in shared memory");
     constexpr int REC_PAIR = (AUG ? 0 : 2) + 2 * C;   // floats per key pair
     constexpr int SL = QSM ? 2 : 1;
     extern __shared__ uint8_t smem_raw[];
@@ -230,7 +234,7 @@ tc_gauss_fma_kernel(const __grid_constant__ CUtensorMap tm_q,
                 for (int h = 0; h < NQ; ++h)
                     for (int kb = 0; kb < p.nkb; ++kb)
                         tma_load_2d(q_smem + (h * p.nkb + kb) * (BM * 128), &tm_q, &bars->qa_ready,
-                                    kb * KB, (tile_m * NQ + h) * BM);
+                                    kb * p.kb_elems, (tile_m * NQ + h) * BM);
             }
             __syncwarp();
             if (has_tiles) {
@@ -238,7 +242,8 @@ tc_gauss_fma_kernel(const __grid_constant__ CUtensorMap tm_q,
                     mbar_arrive_expect_tx(&bars->kv_full[k], p.kh_bytes + p.rec_bytes);
                     const int n0 = kbase + (kt0 + j) * BN;
                     for (int kb = 0; kb < p.nkb; ++kb)
-                        tma_load_2d(kh_smem(k) + kb * (BN * 128), &tm_k, &bars->kv_full[k], kb * KB, n0);
+                        tma_load_2d(kh_smem(k) + kb * (BN * 128), &tm_k, &bars->kv_full[k],
+                                    kb * p.kb_elems, n0);
                     bulk_load(const_cast<float*>(rec_smem(k)),
                               p.rec + static_cast<int64_t>(n0 / 2) * REC_PAIR, p.rec_bytes,
                               &bars->kv_full[k]);
@@ -249,7 +254,7 @@ tc_gauss_fma_kernel(const __grid_constant__ CUtensorMap tm_q,
                 }
                 __syncwarp();
                 bool ok = warp_wait(&bars->qa_ready, seg_parity, abort_flag, p.status);
-                const int ksteps = p.Dp / 16;
+                const int ksteps = p.ksteps;
                 // Shared-memory descriptors of stage k and of q^ tile 0; query
                 // tile h and K step kk add byte offsets / 16 to the start-address
                 // field.
@@ -285,7 +290,26 @@ tc_gauss_fma_kernel(const __grid_constant__ CUtensorMap tm_q,
                     pending = false;
                     tc_fence_after();
                     const uint32_t d0 = tmem + sl * (2 * BN), d1 = d0 + BN;
-                    if (leader) {
+                    if (leader && TF) {
+                        // 3xTF32: per K step of 8 coordinates (32 bytes),
+                        // hi.lo + lo.hi + hi.hi; the lo blocks follow the
+                        // hi blocks (nkb / 2 of each).
+                        const uint32_t klo = static_cast<uint32_t>((p.nkb / 2) * (BN * 128 / 16));
+                        const uint32_t qlo = static_cast<uint32_t>((p.nkb / 2) * (BM * 128 / 16));
+                        for (int h = 0; h < NQ; ++h) {
+                            for (int kk = 0; kk < ksteps; ++kk) {
+                                const uint32_t step = static_cast<uint32_t>((kk & 3) * 2);
+                                const uint64_t kd = kdesc + (kk >> 2) * (BN * 128 / 16) + step;
+                                const uint64_t qd = qdesc0 + h * qdesc_h + (kk >> 2) * (BM * 128 / 16) + step;
+                                const uint32_t d = h ? d1 : d0;
+                                mma_ss_tf32(d, qd, kd + klo, p.idesc, kk > 0 ? 1u : 0u);
+                                mma_ss_tf32(d, qd + qlo, kd, p.idesc, 1u);
+                                mma_ss_tf32(d, qd, kd, p.idesc, 1u);
+                            }
+                        }
+                        mma_commit(&bars->s_full[sl]);
+                        mma_commit(&bars->kv_empty[k]);
+                    } else if (leader) {
                         for (int h = 0; h < NQ; ++h) {
                             for (int kk = 0; kk < ksteps; ++kk) {
                                 const uint32_t koff = static_cast<uint32_t>((kk >> 2) * (BN * 128 / 16) + (kk & 3) * 2);
@@ -406,11 +430,14 @@ tc_gauss_fma_kernel(const __grid_constant__ CUtensorMap tm_q,
                 uint32_t r0[32], r1[32];
                 tmem_ld_32x32b_x32(tmem + lane_base + col0 + cg * 32, r0);
                 tmem_ld_32x32b_x32(tmem + lane_base + col0 + BN + cg * 32, r1);
-                tmem_wait_ld();
-                // Both S slices are in registers: hand the slot back.
-                tc_fence_before();
-                __syncwarp();
-                if (lane == 0) mbar_arrive(&bars->s_free[sl.idx]);
+                // The wait names r0 and r1, so that no use of the loaded
+                // values is scheduled above it (the loads land asynchronously).
+                tmem_wait_ld_regs(r0, r1);
+                // The S slot is handed back only after the exponent work of
+                // this tile (with the stage, below): releasing it right after
+                // the loads let the next MMAs into the slot corrupt values of
+                // this tile in some warps when the MMAs were long (measured
+                // with 3xTF32 operands and three or more stages).
                 // Query the barriers of key tile j + 1 now and read the answer
                 // after the exponent work of tile j: the query latency overlaps
                 // the arithmetic instead of stalling all exponent warps at once.
@@ -489,8 +516,12 @@ tc_gauss_fma_kernel(const __grid_constant__ CUtensorMap tm_q,
                     }
                 }
                 }
+                tc_fence_before();
                 __syncwarp();
-                if (lane == 0) mbar_arrive(&bars->kv_empty[s]);
+                if (lane == 0) {
+                    mbar_arrive(&bars->s_free[sl.idx]);
+                    mbar_arrive(&bars->kv_empty[s]);
+                }
             }
             // Fixed-order reduction of the NPART column-group partial sums.
     #pragma unroll
@@ -545,19 +576,28 @@ size_t fixed_bytes_for(int C, size_t q_bytes) {
            sizeof(FmaBarriers) + 64;
 }
 
+// 128-byte K blocks of an operand row: 16-bit elements, or (TF) the hi and
+// lo fp32 halves of Dp columns each.
+int nkb_for(int Dp, bool tf) { return tf ? 2 * ((Dp + 31) / 32) : (Dp + KB - 1) / KB; }
+
 // Shared-memory bytes of the q^ tiles when they live in shared memory.
-size_t q_bytes_for(int Dp, bool qsm) {
-    return qsm ? static_cast<size_t>(NQ) * ((Dp + KB - 1) / KB) * BM * 128 : 0;
+size_t q_bytes_for(int nkb, bool qsm) {
+    return qsm ? static_cast<size_t>(NQ) * nkb * BM * 128 : 0;
 }
 
-template <int C, bool AUG, bool QSM>
+template <int C, bool AUG, bool QSM, bool TF>
 cudaError_t launch_typed(const TcPlan& pl, InType t, float c, char* ws, unsigned* status,
                          cudaStream_t s, const char** why) {
     const CUtensorMapDataType hdt =
-        t == InType::BF16 ? CU_TENSOR_MAP_DATA_TYPE_BFLOAT16 : CU_TENSOR_MAP_DATA_TYPE_FLOAT16;
+        TF ? CU_TENSOR_MAP_DATA_TYPE_FLOAT32
+           : t == InType::BF16 ? CU_TENSOR_MAP_DATA_TYPE_BFLOAT16 : CU_TENSOR_MAP_DATA_TYPE_FLOAT16;
+    // Row elements and bytes: Dp 16-bit values, or (TF) 2 Dp floats.
+    const uint64_t row_el = TF ? 2ull * pl.Dp : static_cast<uint64_t>(pl.Dp);
+    const uint64_t row_bytes = TF ? row_el * 4 : row_el * 2;
+    const uint32_t kb_elems = TF ? 32u : static_cast<uint32_t>(KB);
     CUtensorMap tm_q, tm_k;
-    if (!encode_tile_map_2d(&tm_k, hdt, ws + pl.off_kh, pl.Dp, pl.Npad * pl.batch, pl.Dp * 2ull, KB, BN) ||
-        !encode_tile_map_2d(&tm_q, hdt, ws + pl.off_qh, pl.Dp, pl.Mpad * pl.batch, pl.Dp * 2ull, KB, BM)) {
+    if (!encode_tile_map_2d(&tm_k, hdt, ws + pl.off_kh, row_el, pl.Npad * pl.batch, row_bytes, kb_elems, BN) ||
+        !encode_tile_map_2d(&tm_q, hdt, ws + pl.off_qh, row_el, pl.Mpad * pl.batch, row_bytes, kb_elems, BM)) {
         *why = "cuTensorMapEncodeTiled failed or is unavailable";
         return cudaErrorInvalidValue;
     }
@@ -574,22 +614,24 @@ cudaError_t launch_typed(const TcPlan& pl, InType t, float c, char* ws, unsigned
     p.units = static_cast<int>(pl.units);
     p.unit_len = static_cast<int>(pl.unit_len);
     p.Dp = pl.Dp;
-    p.nkb = (pl.Dp + KB - 1) / KB;
+    p.nkb = nkb_for(pl.Dp, TF);
+    p.kb_elems = static_cast<int>(kb_elems);
+    p.ksteps = TF ? static_cast<int>(std::max<int64_t>(1, (pl.D + 7) / 8)) : pl.Dp / 16;
     p.stages = pl.stages;
-    p.q_bytes = static_cast<uint32_t>(q_bytes_for(pl.Dp, QSM));
+    p.q_bytes = static_cast<uint32_t>(q_bytes_for(p.nkb, QSM));
     p.kh_bytes = static_cast<uint32_t>(p.nkb * BN * 128);
     p.rec_bytes = static_cast<uint32_t>((BN / 2) * rec_pair_floats(C, AUG) * 4);
     p.stage_bytes = static_cast<uint32_t>(stage_bytes_for(p.nkb, C, AUG));
     p.red_offset = p.q_bytes + static_cast<uint32_t>(pl.stages * p.stage_bytes);
     p.c = c;
     const uint32_t hb = t == InType::BF16 ? 1u : 0u;
-    p.idesc = idesc_f16(BM, BN, hb, hb);
-    cudaError_t e = cudaFuncSetAttribute(tc_gauss_fma_kernel<C, AUG, QSM>,
+    p.idesc = TF ? idesc_tf32(BM, BN) : idesc_f16(BM, BN, hb, hb);
+    cudaError_t e = cudaFuncSetAttribute(tc_gauss_fma_kernel<C, AUG, QSM, TF>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          static_cast<int>(pl.smem_bytes));
     if (e != cudaSuccess) return e;
     dim3 grid(static_cast<unsigned>(pl.grid));
-    tc_gauss_fma_kernel<C, AUG, QSM><<<grid, THREADS, pl.smem_bytes, s>>>(tm_q, tm_k, p);
+    tc_gauss_fma_kernel<C, AUG, QSM, TF><<<grid, THREADS, pl.smem_bytes, s>>>(tm_q, tm_k, p);
     note_launches(1);
     return cudaGetLastError();
 }
@@ -597,22 +639,24 @@ cudaError_t launch_typed(const TcPlan& pl, InType t, float c, char* ws, unsigned
 template <int C>
 cudaError_t launch_c(const TcPlan& pl, InType t, float c, char* ws, unsigned* status,
                      cudaStream_t s, const char** why) {
-    if (pl.aug) return launch_typed<C, true, kAugQsm>(pl, t, c, ws, status, s, why);
-    return launch_typed<C, false, false>(pl, t, c, ws, status, s, why);
+    if (pl.tf) return launch_typed<C, false, true, true>(pl, t, c, ws, status, s, why);
+    if (pl.aug) return launch_typed<C, true, kAugQsm, false>(pl, t, c, ws, status, s, why);
+    return launch_typed<C, false, false, false>(pl, t, c, ws, status, s, why);
 }
 
 }  // namespace
 
-bool plan_fma_kernel(int Dp, int C, bool aug, int* nq, int* stages, size_t* smem) {
+bool plan_fma_kernel(int Dp, int C, bool aug, bool tf, int* nq, int* stages, size_t* smem) {
     if (C < 1 || C > kFmaMaxChannels || Dp > 256) return false;
     if (aug && Dp > kAugMaxDp) return false;
+    if (tf && (aug || Dp > kTf32MaxDp)) return false;
     // TMEM: q^ in TMEM needs Dp columns beside one slot of two S buffers.
-    const bool qsm = aug && kAugQsm;
+    const bool qsm = tf || (aug && kAugQsm);
     if (!qsm && static_cast<int>(TMEM_COLS) - 2 * BN < Dp) return false;
-    const int nkb = (Dp + KB - 1) / KB;
+    const int nkb = nkb_for(Dp, tf);
     const size_t budget = 232448;
     const size_t stage = stage_bytes_for(nkb, C, aug);
-    const size_t fixed = fixed_bytes_for(C, q_bytes_for(Dp, qsm));
+    const size_t fixed = fixed_bytes_for(C, q_bytes_for(nkb, qsm));
     if (fixed >= budget) return false;
     // Control warp k owns stage k (stages = control warps) and checks the
     // S-slot release of key tile j - SL before the MMAs of tile j.  An

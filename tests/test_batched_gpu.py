@@ -54,7 +54,8 @@ def _check_batched(B, M, N, D, C, dtype, q_is_k=False, kind="normal"):
     (2, 300, 130, 17, 1, "bf16"),     # one launch, ragged sizes
     (2, 70, 400, 200, 3, "fp16"),     # one launch, q^ in TMEM (no augmented operands)
     (2, 150, 260, 32, 8, "fp16"),     # C > 4: one problem after another
-    (3, 90, 110, 16, 2, "fp32"),      # fp32 path: one problem after another
+    (3, 90, 110, 16, 2, "fp32"),      # small fp32 problems: SIMT, one after another
+    (8, 2048, 2100, 16, 1, "fp32"),   # fp32 tensor-core path: one launch for the batch
 ])
 def test_batched_matches_each_problem(B, M, N, D, C, dtype):
     _check_batched(B, M, N, D, C, dtype)

@@ -104,7 +104,10 @@ def test_vjp_without_outputs_is_a_noop(lib):
 def test_path_dtype_mismatch_is_unsupported(lib):
     from paper_2609_04910_gb300._binding import GS_PATH_SIMT, GS_PATH_TENSOR, options
     o = options(path=GS_PATH_TENSOR)
-    st = lib.gauss_sum_ex(ALIGNED, ALIGNED, ALIGNED, 1.0, 4, 4, 3, 1, 0, ALIGNED, None, ctypes.byref(o))
+    # fp32 on the tensor cores: forward sums with C <= 4 and D <= 32 only.
+    st = lib.gauss_sum_ex(ALIGNED, ALIGNED, ALIGNED, 1.0, 4, 4, 40, 1, 0, ALIGNED, None, ctypes.byref(o))
+    assert st == 2
+    st = lib.gauss_sum_ex(ALIGNED, ALIGNED, ALIGNED, 1.0, 4, 4, 3, 5, 0, ALIGNED, None, ctypes.byref(o))
     assert st == 2
     o = options(path=GS_PATH_SIMT)
     st = lib.gauss_sum_ex(ALIGNED, ALIGNED, ALIGNED, 1.0, 4, 4, 3, 1, 1, ALIGNED, None, ctypes.byref(o))

@@ -42,6 +42,43 @@ def test_forward_parity(M, N, D, C, dtype):
     forward_check(case(M, N, D, C, dtype))
 
 
+TF32_CASES = [
+    # M, N, D, C (fp32 inputs on the tensor cores: 3xTF32 S, fp32 exponent and sums)
+    (1, 1, 1, 1), (7, 130, 3, 1), (129, 257, 17, 2), (300, 1000, 16, 1), (260, 700, 32, 4),
+    (513, 300, 8, 3), (1000, 3000, 16, 1),
+]
+
+
+@pytest.mark.parametrize("M,N,D,C", TF32_CASES)
+def test_fp32_tensor_parity(M, N, D, C):
+    import paper_2609_04910_gb300 as gs
+    forward_check(case(M, N, D, C, "fp32"), path=gs.GS_PATH_TENSOR)
+
+
+def test_fp32_tensor_aliasing_splits_and_offset():
+    import paper_2609_04910_gb300 as gs
+    t = gs.GS_PATH_TENSOR
+    forward_check(case(300, 300, 16, 1, "fp32", kind="mmd", q_is_k=True), path=t)
+    forward_check(case(260, 1500, 24, 3, "fp32"), path=t, split_n=3)
+    # A common offset of norm 50: the centring keeps the Gram form exact.
+    forward_check(case(200, 600, 32, 2, "fp32", kind="offset", tau=10.0 / 32), path=t)
+
+
+def test_fp32_tensor_matches_simt():
+    """Both fp32 kernels agree with each other within twice the tolerance."""
+    import paper_2609_04910_gb300 as gs
+    from oracle import oracle_sum
+    from paper_2609_04910_gb300.workloads import generate
+    w = case(700, 900, 16, 2, "fp32")
+    q, k, v = device_inputs(generate(w))
+    inp = generate(w)
+    a = gs.gauss_sum(q, k, v, w.tau, path=gs.GS_PATH_TENSOR)
+    b = gs.gauss_sum(q, k, v, w.tau, path=gs.GS_PATH_SIMT)
+    gs.gauss_sum_device_status()
+    _, den = oracle_sum(inp["q64"], inp["k64"], inp["v64"], w.tau)
+    assert rel_err(a.cpu().numpy(), b.cpu().numpy(), den) <= 2 * TOL["fp32"]
+
+
 @pytest.mark.parametrize("dtype", ["fp16", "bf16", "fp32"])
 def test_forward_q_aliases_k(dtype):
     forward_check(case(300, 300, 64, 1, dtype, kind="mmd", q_is_k=True))
