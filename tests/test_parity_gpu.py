@@ -280,3 +280,25 @@ def test_stream_ordering_on_side_stream():
         out = gs.gauss_sum(q, k, v, w.tau)
     s.synchronize()
     assert torch.equal(out, ref)
+
+
+@pytest.mark.parametrize("D,dtype", [(32, "fp32"), (24, "fp32"), (120, "fp16"), (122, "bf16")])
+def test_long_mma_sequences_repeat_bitwise(D, dtype):
+    """Long MMA sequences per key tile (3xTF32 at D = 24-32, augmented fp16 /
+    bf16 rows of 128 columns) with four pipeline stages: repeated calls
+    agree bit for bit and sampled rows match the oracle.  (An early release
+    of the TMEM S slots once made single warps read overwritten S values
+    here, nondeterministically.)"""
+    import paper_2609_04910_gb300 as gs
+    from oracle import oracle_sum
+    from paper_2609_04910_gb300.workloads import generate, sample_rows
+    w = case(16384, 16384, D, 1, dtype)
+    inp = generate(w)
+    q, k, v = device_inputs(inp)
+    path = gs.GS_PATH_TENSOR
+    outs = [gs.gauss_sum(q, k, v, w.tau, path=path) for _ in range(3)]
+    gs.gauss_sum_device_status()
+    assert all(torch.equal(outs[0], o) for o in outs[1:])
+    rows = sample_rows(16384, 96)
+    ref, den = oracle_sum(inp["q64"], inp["k64"], inp["v64"], w.tau, rows=rows)
+    assert rel_err(outs[0].cpu().numpy()[rows], ref, den) <= TOL[dtype]
