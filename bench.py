@@ -62,6 +62,24 @@ def dist_env():
     return rank, world, local
 
 
+def reduce_max(value, device):
+    """Largest `value` over the ranks of the default process group (the
+    value itself when no group of more than one rank is initialised)."""
+    import torch
+    import torch.distributed as dist
+    if not (dist.is_available() and dist.is_initialized()) or dist.get_world_size() == 1:
+        return float(value)
+    t = torch.tensor([float(value)], device=device, dtype=torch.float64)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def replica_value(world, pairs_per_rank, ms):
+    """Whole-job rate of `world` replicas that each process `pairs_per_rank`
+    pairs per step, from the slowest rank's step time in ms."""
+    return world * pairs_per_rank / (ms * 1e-3)
+
+
 def workload_config(w):
     return {
         "workload": f"{w.name}: M={w.M}, N={w.N}, D={w.D}, C={w.C}, {w.dtype}, tau={w.tau:g}"
@@ -317,11 +335,7 @@ def run_own(args):
     main_ms = [a.elapsed_time(b) for a, b in mev]
     ms = statistics.mean(step_ms)
     main_mean = statistics.mean(main_ms)
-    if world > 1:
-        import torch.distributed as dist
-        t = torch.tensor([ms], device=dev, dtype=torch.float64)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms = float(t.item())
+    ms = reduce_max(ms, dev)
 
     # End to end through the public API with host buffers: H2D of the
     # inputs, the call, D2H of the result, every step.
@@ -362,12 +376,8 @@ def run_own(args):
                 e_ev[i - W][1].record(stream)
         torch.cuda.synchronize()
         e_ms = statistics.mean(a.elapsed_time(b) for a, b in e_ev)
-        if world > 1:
-            import torch.distributed as dist
-            t = torch.tensor([e_ms], device=dev, dtype=torch.float64)
-            dist.all_reduce(t, op=dist.ReduceOp.MAX)
-            e_ms = float(t.item())
-        e2e = {"value": world * w.pairs / (e_ms * 1e-3), "unit": UNIT, "ms_per_step": e_ms,
+        e_ms = reduce_max(e_ms, dev)
+        e2e = {"value": replica_value(world, w.pairs, e_ms), "unit": UNIT, "ms_per_step": e_ms,
                "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h),
                "steps": len(e_ev)}
     clocks = sampler.stop() if sampler is not None else None
@@ -421,7 +431,7 @@ def run_own(args):
 
     if rank == 0:
         line = {
-            "metric": METRIC, "value": world * w.pairs / (ms * 1e-3), "unit": UNIT,
+            "metric": METRIC, "value": replica_value(world, w.pairs, ms), "unit": UNIT,
             "n_gpus": world, "steps": K, "warmup": W, "ms_per_step": ms,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
             "dtype": "fp16" if w.dtype == "fp16" else w.dtype, "data": "synthetic",
