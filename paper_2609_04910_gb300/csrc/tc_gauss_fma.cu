@@ -211,8 +211,6 @@ tc_gauss_fma_kernel(const __grid_constant__ CUtensorMap tm_q,
         const int kt0 = u - tile_m * p.key_tiles;
         const int T = min(p.key_tiles - kt0, u_end - u);
         const int g0 = u - u_begin;           // running index of the segment's first tile
-        const int slot = static_cast<int>(blockIdx.x) -
-                         static_cast<int>(static_cast<int64_t>(tile_m) * p.key_tiles / p.unit_len);
 
             // ------------------------------------------------ control warps
             // Control warp k (on SMSP k) owns shared-memory stage k and the key
@@ -433,11 +431,21 @@ tc_gauss_fma_kernel(const __grid_constant__ CUtensorMap tm_q,
                 // The wait names r0 and r1, so that no use of the loaded
                 // values is scheduled above it (the loads land asynchronously).
                 tmem_wait_ld_regs(r0, r1);
-                // The S slot is handed back only after the exponent work of
-                // this tile (with the stage, below): releasing it right after
-                // the loads let the next MMAs into the slot corrupt values of
-                // this tile in some warps when the MMAs were long (measured
-                // with 3xTF32 operands and three or more stages).
+                // When and where the S slot is handed back: with two slots
+                // (q^ in shared memory) only after the exponent work of this
+                // tile (with the stage, below), because releasing it right
+                // after the loads let the next MMAs into the slot corrupt S
+                // values of this tile in some warps when the MMAs were long
+                // (measured with 3xTF32 operands and three or more stages).
+                // With one slot (q^ in TMEM) a late release would serialise
+                // the MMAs and the exponent work, so it is released here; no
+                // corruption was seen there in repeated runs (regression
+                // test: repeated calls agree bit for bit).
+                if (!QSM) {
+                    tc_fence_before();
+                    __syncwarp();
+                    if (lane == 0) mbar_arrive(&bars->s_free[sl.idx]);
+                }
                 // Query the barriers of key tile j + 1 now and read the answer
                 // after the exponent work of tile j: the query latency overlaps
                 // the arithmetic instead of stalling all exponent warps at once.
@@ -519,7 +527,7 @@ tc_gauss_fma_kernel(const __grid_constant__ CUtensorMap tm_q,
                 tc_fence_before();
                 __syncwarp();
                 if (lane == 0) {
-                    mbar_arrive(&bars->s_free[sl.idx]);
+                    if (QSM) mbar_arrive(&bars->s_free[sl.idx]);
                     mbar_arrive(&bars->kv_empty[s]);
                 }
             }

@@ -282,13 +282,15 @@ def test_stream_ordering_on_side_stream():
     assert torch.equal(out, ref)
 
 
-@pytest.mark.parametrize("D,dtype", [(32, "fp32"), (24, "fp32"), (120, "fp16"), (122, "bf16")])
+@pytest.mark.parametrize("D,dtype", [(32, "fp32"), (24, "fp32"), (120, "fp16"), (122, "bf16"),
+                                     (256, "fp16"), (200, "bf16")])
 def test_long_mma_sequences_repeat_bitwise(D, dtype):
     """Long MMA sequences per key tile (3xTF32 at D = 24-32, augmented fp16 /
-    bf16 rows of 128 columns) with four pipeline stages: repeated calls
-    agree bit for bit and sampled rows match the oracle.  (An early release
-    of the TMEM S slots once made single warps read overwritten S values
-    here, nondeterministically.)"""
+    bf16 rows of 128 columns with four pipeline stages, q^ in TMEM with one
+    S slot at D = 200-256): repeated calls agree bit for bit and sampled rows
+    match the oracle.  (An early release of the TMEM S slots once made
+    single warps read overwritten S values on the two-slot path,
+    nondeterministically.)"""
     import paper_2609_04910_gb300 as gs
     from oracle import oracle_sum
     from paper_2609_04910_gb300.workloads import generate, sample_rows
@@ -296,7 +298,7 @@ def test_long_mma_sequences_repeat_bitwise(D, dtype):
     inp = generate(w)
     q, k, v = device_inputs(inp)
     path = gs.GS_PATH_TENSOR
-    outs = [gs.gauss_sum(q, k, v, w.tau, path=path) for _ in range(3)]
+    outs = [gs.gauss_sum(q, k, v, w.tau, path=path) for _ in range(4)]
     gs.gauss_sum_device_status()
     assert all(torch.equal(outs[0], o) for o in outs[1:])
     rows = sample_rows(16384, 96)
