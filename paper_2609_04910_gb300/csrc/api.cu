@@ -316,7 +316,7 @@ gs_status run(Call c) {
                 e = gs::launch_finalize_slots(reinterpret_cast<float*>(ws + tp.off_part), tp.Mpad,
                                               c.M, static_cast<int>(tp.Cv), 128 * tp.nq,
                                               tp.Npad / tp.BN, tp.unit_len, c.out, c.stream,
-                                              batch);
+                                              batch, tp.band_len > 0 ? tp.splits : 0);
                 where = "finalise kernel";
             }
         } else if (e == cudaSuccess) {

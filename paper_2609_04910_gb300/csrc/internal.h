@@ -41,6 +41,12 @@ struct TcPlan {
     // CTA (`splits` = the largest number of contributors).
     int64_t units, unit_len;
     int grid;
+    // Banded order of the FMA kernel for keys larger than L2 (band_len > 0):
+    // runs of band_len key tiles of one pair of query tiles, band-major, so
+    // that the CTAs read the same bands at the same time; `splits` is then
+    // the number of bands (one partial-sum slot per band).
+    int band_len;
+    int64_t nruns;
     // Problems of a batch handled by one launch (the FMA kernel stacks them:
     // q^ batch x Mpad rows, k^ batch x Npad rows); 1 for the other paths.
     int64_t batch;
@@ -99,13 +105,15 @@ cudaError_t launch_finalize_points(bool direct, InType t, bool u_f32, const floa
 // (float64 accumulation, fixed order).
 cudaError_t launch_mmd2_reduce(InType t, const float* s, const void* v, int64_t B, int64_t N,
                                float* out, cudaStream_t st);
-// Forward sum of the FMA kernel's contributor slots: rows of the pair of
-// query tiles r = m / rows_per_unit have slots 0 .. last(r) - first(r), with
-// first(r) = r key_tiles / unit_len and last(r) = ((r + 1) key_tiles - 1) /
-// unit_len, added in slot order.
+// Forward sum of the FMA kernel's contributor slots, added in slot order:
+// every row has slots 0 .. fixed_slots - 1 when fixed_slots > 0 (banded
+// order); otherwise rows of the pair of query tiles r = m / rows_per_unit
+// have slots 0 .. last(r) - first(r), with first(r) = r key_tiles /
+// unit_len and last(r) = ((r + 1) key_tiles - 1) / unit_len.
 cudaError_t launch_finalize_slots(const float* part, int64_t Mpad, int64_t M, int C,
                                   int rows_per_unit, int64_t key_tiles, int64_t unit_len,
-                                  float* out, cudaStream_t s, int batch = 1);
+                                  float* out, cudaStream_t s, int batch = 1,
+                                  int fixed_slots = 0);
 
 // simt_fp32.cu ---------------------------------------------------------
 // grad: keys weighted by channel wch of v (N x Cw); partials have D + 1

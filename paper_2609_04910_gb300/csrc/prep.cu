@@ -370,7 +370,8 @@ __global__ void tf32_split_kernel(const float* __restrict__ x, int64_t rows, int
 
 __global__ void finalize_slots_kernel(const float* __restrict__ part, int64_t Mpad, int64_t M,
                                       int C, int rows_per_unit, int64_t key_tiles,
-                                      int64_t unit_len, int64_t batch, float* __restrict__ out) {
+                                      int64_t unit_len, int64_t batch, int fixed_slots,
+                                      float* __restrict__ out) {
     // out: batch x M x C; partial rows are batch-stacked with Mpad rows per
     // problem and batch Mpad rows per slot.
     const int64_t idx = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
@@ -379,11 +380,15 @@ __global__ void finalize_slots_kernel(const float* __restrict__ part, int64_t Mp
     const int c = static_cast<int>(idx - bm * C);
     const int64_t b = bm / M;
     const int64_t m = (bm - b * M) + b * Mpad;
-    const int64_t r = m / rows_per_unit;
-    const int64_t first = r * key_tiles / unit_len;
-    const int64_t last = ((r + 1) * key_tiles - 1) / unit_len;
+    int64_t nslots = fixed_slots;
+    if (nslots == 0) {
+        const int64_t r = m / rows_per_unit;
+        const int64_t first = r * key_tiles / unit_len;
+        const int64_t last = ((r + 1) * key_tiles - 1) / unit_len;
+        nslots = last - first + 1;
+    }
     float acc = 0.f;
-    for (int64_t sl = 0; sl <= last - first; ++sl) acc += part[(sl * batch * Mpad + m) * C + c];
+    for (int64_t sl = 0; sl < nslots; ++sl) acc += part[(sl * batch * Mpad + m) * C + c];
     out[idx] = acc;
 }
 
@@ -875,12 +880,13 @@ cudaError_t launch_mmd2_reduce(InType t, const float* s, const void* v, int64_t 
 
 cudaError_t launch_finalize_slots(const float* part, int64_t Mpad, int64_t M, int C,
                                   int rows_per_unit, int64_t key_tiles, int64_t unit_len,
-                                  float* out, cudaStream_t s, int batch) {
+                                  float* out, cudaStream_t s, int batch, int fixed_slots) {
     const int64_t total = static_cast<int64_t>(batch) * M * C;
     if (total == 0) return cudaSuccess;
     const int threads = 256;
     finalize_slots_kernel<<<static_cast<unsigned>((total + threads - 1) / threads), threads, 0, s>>>(
-        part, Mpad, M, C, rows_per_unit, key_tiles, unit_len, static_cast<int64_t>(batch), out);
+        part, Mpad, M, C, rows_per_unit, key_tiles, unit_len, static_cast<int64_t>(batch),
+        fixed_slots, out);
     note_launches(1);
     return cudaGetLastError();
 }

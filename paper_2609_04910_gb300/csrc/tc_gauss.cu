@@ -418,6 +418,11 @@ cudaError_t launch_bn(const TcPlan& pl, InType t, float c, char* ws, unsigned* s
 
 }  // namespace
 
+// Banded order of the FMA kernel (see plan_tensor).
+constexpr double kBandMinKeyBytes = 64.0 * 1024 * 1024;
+constexpr int64_t kBandTiles = 64;
+constexpr int64_t kMaxBands = 256;
+
 bool plan_tensor(InType t, int64_t M, int64_t N, int64_t D, int64_t C, bool grad, bool center,
                  bool alias, int split_override, int sms, TcPlan* p, const char** why,
                  int64_t batch) {
@@ -525,6 +530,8 @@ bool plan_tensor(InType t, int64_t M, int64_t N, int64_t D, int64_t C, bool grad
     p->splits = std::max(1, best_s);
     p->units = p->unit_len = 0;
     p->grid = 0;
+    p->band_len = 0;
+    p->nruns = 0;
     if (p->fma) {
         // Persistent split: one CTA per SM, each taking an equal run of
         // (pair of query tiles, key tile) units; with a forced split count
@@ -546,6 +553,26 @@ bool plan_tensor(InType t, int64_t M, int64_t N, int64_t D, int64_t C, bool grad
         for (int64_t r = 0; r < tiles; ++r)
             most = std::max(most, ((r + 1) * key_tiles - 1) / len - r * key_tiles / len + 1);
         p->splits = static_cast<int>(most);
+        // Keys (operand rows and records) larger than half the L2: in the
+        // contiguous order the CTAs stand at evenly spread key tiles, so
+        // every pair of query tiles reads all keys from DRAM again.  The
+        // banded order keeps all CTAs within a few bands of 64 key tiles,
+        // which stay in L2 while the pairs of query tiles pass over them.
+        const double key_bytes =
+            static_cast<double>(B) * p->Npad *
+            ((p->tf ? 8.0 : 2.0) * p->Dp + 2.0 * ((p->aug ? 0 : 1) + p->Cv));
+        if (split_override == 0 && key_bytes > kBandMinKeyBytes && key_tiles > kBandTiles) {
+            const int64_t blen = std::max<int64_t>(kBandTiles, (key_tiles + kMaxBands - 1) / kMaxBands);
+            const int64_t nbands = (key_tiles + blen - 1) / blen;
+            const int64_t nruns = tiles * nbands;
+            if (nruns < (int64_t(1) << 31)) {
+                p->band_len = static_cast<int>(blen);
+                p->nruns = nruns;
+                p->grid = static_cast<int>(std::min<int64_t>(sms, nruns));
+                p->splits = static_cast<int>(nbands);
+                p->units = p->unit_len = 0;
+            }
+        }
     }
     // ~256 rows per block of the mean kernel, so that every SM has work.
     p->mean_blocks = static_cast<int>(std::max<int64_t>(1, std::min<int64_t>(4096, (M + N + 255) / 256)));

@@ -90,6 +90,12 @@ struct FmaParams {
     int64_t Mpad;
     int units;           // work units: (pair of query tiles, key tile), row major
     int unit_len;        // units per CTA (CTA i: units [i unit_len, (i + 1) unit_len))
+    // Banded order (band_len > 0, for keys larger than L2): run r = (band
+    // r / pairs_total, pair of query tiles r % pairs_total) covers band_len
+    // key tiles; CTA i takes runs i, i + grid, ...; the slot is the band.
+    int band_len;
+    int nruns;
+    int pairs_total;
     int key_tiles;       // key tiles per problem
     int pairs_per_batch; // pairs of query tiles per problem of a batch
     int npad;            // k^ rows per problem of a batch
@@ -121,6 +127,39 @@ __device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity, volati
                                           unsigned* status) {
     const bool ok = mbar_wait_bounded(bar, parity, abort_flag, status);
     return __all_sync(0xffffffffu, ok);
+}
+
+// One segment of a CTA's work: the pair of query tiles tile_m and T
+// consecutive key tiles from kt0, and the partial-sum slot it writes.
+struct Segment {
+    int tile_m, kt0, T, slot;
+};
+
+// Next segment of this CTA, or false after its last one.  Contiguous order:
+// the CTA's run of units [u, u_end) split at query-pair boundaries, slot =
+// rank of this CTA among the CTAs of that pair.  Banded order: runs
+// blockIdx.x, blockIdx.x + gridDim.x, ..., slot = band.
+__device__ __forceinline__ bool next_segment(const FmaParams& p, int u_end, int& u, int& run,
+                                             Segment& sg) {
+    if (p.band_len == 0) {
+        if (u >= u_end) return false;
+        sg.tile_m = u / p.key_tiles;
+        sg.kt0 = u - sg.tile_m * p.key_tiles;
+        sg.T = min(p.key_tiles - sg.kt0, u_end - u);
+        sg.slot = static_cast<int>(blockIdx.x) -
+                  static_cast<int>(static_cast<int64_t>(sg.tile_m) * p.key_tiles / p.unit_len);
+        u += sg.T;
+        return true;
+    }
+    const int r = static_cast<int>(blockIdx.x) + run * static_cast<int>(gridDim.x);
+    if (r >= p.nruns) return false;
+    const int band = r / p.pairs_total;
+    sg.tile_m = r - band * p.pairs_total;
+    sg.kt0 = band * p.band_len;
+    sg.T = min(p.band_len, p.key_tiles - sg.kt0);
+    sg.slot = band;
+    ++run;
+    return true;
 }
 
 __device__ __forceinline__ void exp_warps_sync() {
@@ -167,12 +206,12 @@ tc_gauss_fma_kernel(const __grid_constant__ CUtensorMap tm_q,
         return reinterpret_cast<const float*>(stage0 + s * p.stage_bytes + p.kh_bytes);
     };
 
-    // The CTA's units form segments of consecutive key tiles of one pair of
-    // query tiles.  The barriers are initialised once and keep running
-    // across segments: every stage, slot and phase follows the CTA-local
-    // running tile index g = u - u_begin, and qa_ready completes once per
-    // segment.  Each segment writes its partial sums to the slot of this
-    // CTA among the CTAs that contribute to that pair of query tiles.
+    // The CTA's work is a sequence of segments (next_segment): consecutive
+    // key tiles of one pair of query tiles.  The barriers are initialised
+    // once and keep running across segments: every stage, slot and phase
+    // follows the CTA-local running tile index g (tiles of all earlier
+    // segments plus the index within the segment), and qa_ready completes
+    // once per segment.  Each segment writes its partial sums to its slot.
     if (tid == 0) {
         mbar_init(&bars->qa_ready, QSM ? 1 : NEXP);
         for (int sl = 0; sl < SL; ++sl) {
@@ -201,16 +240,16 @@ tc_gauss_fma_kernel(const __grid_constant__ CUtensorMap tm_q,
         // (16 x 32 x kExpRegs + 4 x 32 x kCtrlRegs <= 640 x 96 at launch).
         reg_dealloc<kCtrlRegs>();
         uint32_t seg_parity = 0;   // parity of the qa_ready phase of this segment
-        for (int u = u_begin; u < u_end; seg_parity ^= 1u) {
+        int u = u_begin, run = 0, g0 = 0;   // g0: running index of the segment's first tile
+        Segment sg;
+        for (; next_segment(p, u_end, u, run, sg); seg_parity ^= 1u, g0 += sg.T) {
         // Read by every thread after a CTA barrier: uniform.
         if (*abort_flag) break;
-        const int tile_m = u / p.key_tiles;   // query tiles 2 tile_m, 2 tile_m + 1
+        const int tile_m = sg.tile_m;         // query tiles 2 tile_m, 2 tile_m + 1
         // First k^ row of this pair's problem (batch-stacked operands).
         const int kbase = (tile_m / p.pairs_per_batch) * p.npad;
-        (void)kbase;
-        const int kt0 = u - tile_m * p.key_tiles;
-        const int T = min(p.key_tiles - kt0, u_end - u);
-        const int g0 = u - u_begin;           // running index of the segment's first tile
+        const int kt0 = sg.kt0;
+        const int T = sg.T;
 
             // ------------------------------------------------ control warps
             // Control warp k (on SMSP k) owns shared-memory stage k and the key
@@ -355,23 +394,18 @@ tc_gauss_fma_kernel(const __grid_constant__ CUtensorMap tm_q,
         // Segment end: every MMA, copy and TMEM read of this segment is done
         // (control warps waited for their last stage release and copies).
         segment_sync();
-        u += T;
         }
     } else {
         reg_alloc<kExpRegs>();
         uint32_t seg_parity = 0;
-        for (int u = u_begin; u < u_end; seg_parity ^= 1u) {
+        int u = u_begin, run = 0, g0 = 0;
+        Segment sg;
+        for (; next_segment(p, u_end, u, run, sg); seg_parity ^= 1u, g0 += sg.T) {
         // Read by every thread after a CTA barrier: uniform.
         if (*abort_flag) break;
-        const int tile_m = u / p.key_tiles;   // query tiles 2 tile_m, 2 tile_m + 1
-        // First k^ row of this pair's problem (batch-stacked operands).
-        const int kbase = (tile_m / p.pairs_per_batch) * p.npad;
-        (void)kbase;
-        const int kt0 = u - tile_m * p.key_tiles;
-        const int T = min(p.key_tiles - kt0, u_end - u);
-        const int g0 = u - u_begin;           // running index of the segment's first tile
-        const int slot = static_cast<int>(blockIdx.x) -
-                         static_cast<int>(static_cast<int64_t>(tile_m) * p.key_tiles / p.unit_len);
+        const int tile_m = sg.tile_m;         // query tiles 2 tile_m, 2 tile_m + 1
+        const int T = sg.T;
+        const int slot = sg.slot;
 
             // ------------------------------------------------ exponent warps
             const int quarter = warp & 3;
@@ -556,7 +590,6 @@ tc_gauss_fma_kernel(const __grid_constant__ CUtensorMap tm_q,
         // Segment end: every MMA, copy and TMEM read of this segment is done
         // (control warps waited for their last stage release and copies).
         segment_sync();
-        u += T;
         }
     }
 
@@ -621,6 +654,9 @@ cudaError_t launch_typed(const TcPlan& pl, InType t, float c, char* ws, unsigned
     p.npad = static_cast<int>(pl.Npad);
     p.units = static_cast<int>(pl.units);
     p.unit_len = static_cast<int>(pl.unit_len);
+    p.band_len = pl.band_len;
+    p.nruns = static_cast<int>(pl.nruns);
+    p.pairs_total = static_cast<int>((pl.Mpad / (NQ * BM)) * pl.batch);
     p.Dp = pl.Dp;
     p.nkb = nkb_for(pl.Dp, TF);
     p.kb_elems = static_cast<int>(kb_elems);

@@ -304,3 +304,11 @@ def test_long_mma_sequences_repeat_bitwise(D, dtype):
     rows = sample_rows(16384, 96)
     ref, den = oracle_sum(inp["q64"], inp["k64"], inp["v64"], w.tau, rows=rows)
     assert rel_err(outs[0].cpu().numpy()[rows], ref, den) <= TOL[dtype]
+
+
+@pytest.mark.parametrize("M,N,D,C,dtype", [(700, 140000, 256, 3, "fp16"), (300, 200000, 200, 1, "bf16")])
+def test_keys_larger_than_l2_banded_order(M, N, D, C, dtype):
+    """Key operands above 64 MB take the banded work order of the FMA kernel
+    (all CTAs inside a few bands of 64 key tiles, one partial-sum slot per
+    band): ragged rows and key tail, every row against the oracle."""
+    forward_check(case(M, N, D, C, dtype))
