@@ -35,6 +35,8 @@ struct TcPlan {
     bool tf;                 // fp32 inputs on the FMA kernel with 3xTF32 MMAs: q^ and k^
                              // rows are [hi | lo] of Dp (a multiple of 32) floats each
     int nq;                  // query tiles of 128 rows per CTA (FMA kernel)
+    bool early_s;            // two-MMA kernel: S buffers handed back as soon as they are
+                             // in registers (exponent-bound shapes), else with P
     // FMA kernel work split: units = (pairs of query tiles) x key tiles, in
     // row-major order; CTA i takes units [i unit_len, (i + 1) unit_len); the
     // partial sums of a pair of query tiles have one slot per contributing

@@ -16,7 +16,7 @@
 //   MMA2  O  += P v~            tcgen05.mma kind::f16, A = P from TMEM,
 //                               B = value tile from shared memory, fp32 TMEM
 //
-// Warp roles ((NEXP + 2) x 32 threads; NEXP = 16 for BN = 128, 8 for BN = 64):
+// Warp roles ((NEXP + 4) x 32 threads; NEXP = 16 for BN = 128, 8 for BN = 64):
 //   warps 0 .. NEXP-1  exponent warps in two groups of NEXP/2; group g
 //              handles the key tiles j = g (mod 2).  Warp w owns TMEM lanes
 //              32 (w % 4) .. +31 (its hardware lane quarter) and a share of
@@ -24,12 +24,22 @@
 //              partial sums).
 //   warp NEXP  TMA producer: q^ tile once, then k^ / v~ / B tiles into a
 //              ring of `stages` shared-memory stages.
-//   warp NEXP+1  TMEM allocator and single-thread MMA issuer.
+//   warp NEXP+1  TMEM allocator and MMA1 issuer (one elected thread).
+//   warp NEXP+2  MMA2 issuer (EARLY; one elected thread); warp NEXP+3 idle.
 // TMEM columns: S double buffer [0, 2 BN), P double buffer [2 BN, 3 BN)
-// (fp16 pairs packed in 32-bit columns), O accumulator [3 BN, 3 BN + Cp).
-// MMA1 of tile j + 1 and the exponent work of tile j (one group) overlap the
-// exponent work of tile j - 1 (the other group); MMA2 of tile j - 1 is
-// issued after MMA1 of tile j.
+// (fp16 pairs packed in 32-bit columns), O accumulator [3 BN, 3 BN + Cp);
+// buffer g of S and of P belongs to exponent group g.
+//
+// Schedule (EARLY, exponent-bound shapes).  A group hands its S buffer
+// back (s_free) as soon as the tile is in registers, so MMA1 of the group's
+// next tile but one runs under the exponent work of the current tile; its P
+// buffer comes back (p_free) when MMA2 of that tile has read it.  MMA1 and
+// MMA2 are issued by two warps, each in key-tile order: the MMA1 stream
+// waits for the keys and the S buffer, the MMA2 stream for P, so that a
+// stage reload that MMA1 waits for never holds back an MMA2 that a group
+// needs.  Tensor-bound shapes keep one MMA warp issuing MMA1 of tile j + 1
+// after MMA2 of tile j - 1 (S handed back with P), which measured faster
+// there.
 #include <cuda.h>
 #include <cuda_runtime.h>
 
@@ -77,9 +87,12 @@ struct TcParams {
 struct __align__(8) Barriers {
     uint64_t q_full;
     uint64_t o_full;
-    uint64_t drain;
-    uint64_t s_full[2];
-    uint64_t p_full[2];
+    uint64_t drain;       // MMA1 warp: its MMAs are complete
+    uint64_t drain2;      // MMA2 warp: its MMAs are complete
+    uint64_t s_full[2];   // S buffer g computed (MMA1 commit)
+    uint64_t s_free[2];   // S buffer g in the registers of group g
+    uint64_t p_full[2];   // P buffer g written by group g
+    uint64_t p_free[2];   // P buffer g read by MMA2 (MMA2 commit)
     uint64_t kv_full[8];
     uint64_t kv_empty[8];
     uint32_t tmem_base;
@@ -104,13 +117,17 @@ constexpr uint32_t kCtrlRegs2 = 32;
 static_assert(16 * 32 * kExpRegs2 + 4 * 32 * kCtrlRegs2 <= 640 * 96, "register split");
 
 // AUG: augmented operands (S = -||q^ - k^||^2 / 2, no B records).
-template <int BN, int NEXP, bool AUG>
+// EARLY: S buffers handed back right after the TMEM loads, MMA1 and MMA2
+// issued by two warps (exponent-bound shapes); otherwise one MMA warp in
+// P-then-S order (tensor-bound shapes).
+template <int BN, int NEXP, bool AUG, bool EARLY>
 __global__ void __launch_bounds__(cta_threads<NEXP>(), 1)
 tc_gauss_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
                 const __grid_constant__ CUtensorMap tm_v, const TcParams p) {
     static_assert(NEXP % 4 == 0, "exponent warps cover the four TMEM lane quarters");
     constexpr int PRODUCER_WARP = NEXP;
-    constexpr int MMA_WARP = NEXP + 1;
+    constexpr int MMA_WARP = NEXP + 1;     // MMA1 issuer, TMEM allocator
+    constexpr int MMA2_WARP = NEXP + 2;    // MMA2 issuer
     // The exponent warps form two groups; group g handles the key tiles
     // j = g (mod 2), i.e. S/P buffer g, so that one group's TMEM and MMA
     // latency overlaps the other group's exp2 work.
@@ -142,9 +159,12 @@ tc_gauss_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant_
         mbar_init(&bars->q_full, 1);
         mbar_init(&bars->o_full, 1);
         mbar_init(&bars->drain, 1);
+        mbar_init(&bars->drain2, 1);
         for (int b = 0; b < 2; ++b) {
             mbar_init(&bars->s_full[b], 1);
+            mbar_init(&bars->s_free[b], GROUP_WARPS);  // one arrival per warp
             mbar_init(&bars->p_full[b], GROUP_WARPS);  // one arrival per warp
+            mbar_init(&bars->p_free[b], 1);
         }
         for (int s = 0; s < p.stages; ++s) {
             mbar_init(&bars->kv_full[s], 1);
@@ -208,10 +228,91 @@ tc_gauss_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant_
                                   static_cast<uint32_t>(j / p.stages) & 1u, nullptr, p.status);
             __syncwarp();
         }
-    } else if (warp == MMA_WARP) {
+    } else if (EARLY && warp == MMA_WARP) {
         if (NEXP == 16) reg_dealloc<kCtrlRegs2>();
-        // The whole warp runs the loop (warp-uniform descriptors); the
-        // elected lane issues the MMAs and commits.
+        // MMA1 stream: S of key tile j into buffer j % 2, as soon as the
+        // keys are loaded and group j % 2 holds tile j - 2 in registers.  The
+        // whole warp runs the loop (warp-uniform descriptors); the elected
+        // lane issues the MMAs and commits.
+        if (T > 0) {
+            const bool leader = elect_one();
+            const uint32_t q_base = smem_u32(q_smem);
+            bool ok = warp_wait(&bars->q_full, 0, abort_flag, p.status);
+            RingPos st;
+            for (int j = 0; ok && j < T; ++j, st.advance(p.stages)) {
+                const int b = j & 1;
+                ok = warp_wait(&bars->kv_full[st.idx], st.phase, abort_flag, p.status);
+                if (ok && j >= 2)
+                    ok = warp_wait(&bars->s_free[b], static_cast<uint32_t>((j - 2) >> 1) & 1u, abort_flag,
+                                   p.status);
+                if (!ok) break;
+                tc_fence_after();
+                const uint32_t kh_base = smem_u32(kh_smem(st.idx));
+                if (leader) {
+                    for (int kk = 0; kk < p.ksteps1; ++kk) {
+                        const uint32_t koff = static_cast<uint32_t>(kk & 3) * 32;
+                        const uint64_t ad = smem_desc_kmajor_sw128(q_base + (kk >> 2) * (BM * 128) + koff);
+                        const uint64_t bd = smem_desc_kmajor_sw128(kh_base + (kk >> 2) * (BN * 128) + koff);
+                        mma_ss_f16(tmem + S_col0 + b * BN, ad, bd, p.idesc1, kk > 0 ? 1u : 0u);
+                    }
+                    mma_commit(&bars->s_full[b]);
+                }
+                __syncwarp();
+            }
+            // No MMA of this warp may still be running when TMEM is released.
+            if (leader) mma_commit(&bars->drain);
+            __syncwarp();
+            mbar_wait_bounded(&bars->drain, 0, nullptr, p.status);
+            __syncwarp();
+        }
+    } else if (EARLY && warp == MMA2_WARP) {
+        if (NEXP == 16) reg_dealloc<kCtrlRegs2>();
+        // MMA2 stream: O += P v~ for key tile j once group j % 2 has written
+        // P; its commits hand back the P buffer and the stage.  (MMA1 of
+        // tile j completed before the group could write P of tile j, so the
+        // stage is released after both MMAs that read it.)
+        if (T > 0) {
+            const bool leader = elect_one();
+            bool ok = true;
+            RingPos st;
+            for (int j = 0; ok && j < T; ++j, st.advance(p.stages)) {
+                const int b = j & 1;
+                ok = warp_wait(&bars->p_full[b], static_cast<uint32_t>(j >> 1) & 1u, abort_flag, p.status);
+                // The values of tile j landed before MMA1 of tile j was issued;
+                // this wait (already complete) also orders them for this warp.
+                if (ok) ok = warp_wait(&bars->kv_full[st.idx], st.phase, abort_flag, p.status);
+                if (!ok) break;
+                tc_fence_after();
+                const uint32_t vt_base = smem_u32(vt_smem(st.idx));
+                if (leader) {
+                    for (int kk = 0; kk < BN / 16; ++kk) {
+                        const uint64_t bd = smem_desc_kmajor_sw128(vt_base + (kk >> 2) * (p.Cp * 128) + (kk & 3) * 32);
+                        mma_ts_f16(tmem + O_col, tmem + P_col0 + b * (BN / 2) + kk * 8, bd, p.idesc2,
+                                   (j > 0 || kk > 0) ? 1u : 0u);
+                    }
+                    mma_commit(&bars->p_free[b]);
+                    mma_commit(&bars->kv_empty[st.idx]);
+                }
+                __syncwarp();
+            }
+            if (leader) {
+                if (ok) mma_commit(&bars->o_full);
+                mma_commit(&bars->drain2);
+            }
+            __syncwarp();
+            mbar_wait_bounded(&bars->drain2, 0, nullptr, p.status);
+            __syncwarp();
+        }
+    } else if (!EARLY && warp == MMA_WARP) {
+        if (NEXP == 16) reg_dealloc<kCtrlRegs2>();
+        // Both streams in one warp, P-then-S order: MMA1 of tile j, then
+        // (once P of tile j - 1 is written) MMA2 of tile j - 1.  MMA1 of tile
+        // j + 1 thus enters the tensor queue behind MMA2 of tile j - 1, S
+        // buffer (j + 1) % 2 is free then (P of tile j - 1 is written), and
+        // the completion of S of a tile implies that MMA2 of the tile two
+        // before it has read its P buffer.  The whole warp runs the loop
+        // (warp-uniform descriptors); the elected lane issues the MMAs and
+        // commits.
         if (T > 0) {
             const bool leader = elect_one();
             const uint32_t q_base = smem_u32(q_smem);
@@ -267,7 +368,7 @@ tc_gauss_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant_
             mbar_wait_bounded(&bars->drain, 0, nullptr, p.status);
             __syncwarp();
         }
-    } else if (warp > MMA_WARP) {
+    } else if (warp >= MMA_WARP) {
         // Idle warps completing the control warpgroup.
         if (NEXP == 16) reg_dealloc<kCtrlRegs2>();
     } else {
@@ -308,6 +409,13 @@ tc_gauss_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant_
             tmem_wait_ld();
 #pragma unroll
             for (int ch = 0; ch < NCH; ++ch) tmem_regs_ready(r[ch]);
+            // S buffer b is in registers: MMA1 of tile j + 2 may overwrite it
+            // (EARLY; otherwise MMA1 of tile j + 2 follows P of tile j).
+            if (EARLY) {
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0) mbar_arrive(&bars->s_free[b]);
+            }
             const float* Bs = b_smem(s) + col0;
 #pragma unroll
             for (int ch = 0; ch < NCH; ++ch) {
@@ -333,8 +441,17 @@ tc_gauss_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant_
                     pk[2 * i + 0] = pack_half2_satfinite(ex2_approx(x0), ex2_approx(x1));
                     pk[2 * i + 1] = pack_half2_satfinite(ex2_approx(x2), ex2_approx(x3));
                 }
+                if (EARLY && ch == 0 && j >= 2) {
+                    // P buffer b: MMA2 of tile j - 2 has read it.  (With one
+                    // MMA warp the completion of S of tile j implies it.)
+                    ok = warp_wait(&bars->p_free[b], static_cast<uint32_t>((j - 2) >> 1) & 1u, abort_flag,
+                                   p.status);
+                    if (!ok) break;
+                    tc_fence_after();
+                }
                 tmem_st_32x32b_x16(tmem + lane_base + P_col0 + b * (BN / 2) + (col0 + ch * 32) / 2, pk);
             }
+            if (!ok) break;
             tmem_wait_st();
             tc_fence_before();
             __syncwarp();
@@ -371,7 +488,7 @@ tc_gauss_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant_
 // ---------------------------------------------------------------- host side
 size_t align1k(size_t x) { return (x + 1023) & ~static_cast<size_t>(1023); }
 
-template <int BN, int NEXP, bool AUG>
+template <int BN, int NEXP, bool AUG, bool EARLY>
 cudaError_t launch_bn(const TcPlan& pl, InType t, float c, char* ws, unsigned* status,
                       cudaStream_t s, const char** why) {
     const CUtensorMapDataType hdt =
@@ -406,12 +523,12 @@ cudaError_t launch_bn(const TcPlan& pl, InType t, float c, char* ws, unsigned* s
     p.idesc2 = idesc_f16(BM, static_cast<uint32_t>(pl.Cp), 0u, 0u);
 
     // Per-device function attribute; cheap enough to set on every launch.
-    cudaError_t e = cudaFuncSetAttribute(tc_gauss_kernel<BN, NEXP, AUG>,
+    cudaError_t e = cudaFuncSetAttribute(tc_gauss_kernel<BN, NEXP, AUG, EARLY>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          static_cast<int>(pl.smem_bytes));
     if (e != cudaSuccess) return e;
     dim3 grid(static_cast<unsigned>(pl.Mpad / BM), static_cast<unsigned>(pl.splits));
-    tc_gauss_kernel<BN, NEXP, AUG><<<grid, cta_threads<NEXP>(), pl.smem_bytes, s>>>(tm_q, tm_k, tm_v, p);
+    tc_gauss_kernel<BN, NEXP, AUG, EARLY><<<grid, cta_threads<NEXP>(), pl.smem_bytes, s>>>(tm_q, tm_k, tm_v, p);
     note_launches(1);
     return cudaGetLastError();
 }
@@ -438,6 +555,7 @@ bool plan_tensor(InType t, int64_t M, int64_t N, int64_t D, int64_t C, bool grad
     p->alias = alias;
     p->center = center;
     p->tf = false;
+    p->early_s = false;
     const int nkb = (p->Dp + KB - 1) / KB;
     size_t fma_smem = 0;
     int fma_stages = 0, nq = 1;
@@ -488,6 +606,7 @@ bool plan_tensor(InType t, int64_t M, int64_t N, int64_t D, int64_t C, bool grad
         const int nkb = (p->Dp + KB - 1) / KB;
         p->BN = p->Cp <= 128 ? 128 : 64;
         p->nq = 1;
+
         const size_t stage = align1k(static_cast<size_t>(nkb) * p->BN * 128 +
                                      static_cast<size_t>(p->BN / KB) * p->Cp * 128 + p->BN * 4);
         const size_t qbytes = static_cast<size_t>(nkb) * BM * 128;
@@ -496,6 +615,13 @@ bool plan_tensor(InType t, int64_t M, int64_t N, int64_t D, int64_t C, bool grad
         int stages = static_cast<int>(std::min<size_t>(6, (budget - fixed) / stage));
         if (stages < 2) { *why = "shared-memory budget exceeded"; return false; }
         p->stages = stages;
+        // Early S release with two MMA warps lets MMA1 run up to two key
+        // tiles ahead of the exponent work, which needs stages to load them
+        // into: with four or more stages it measured faster on every shape
+        // tried (fp16 forward C = 8..128, gradients, VJP: 3-16 %), with three
+        // (bf16 D = 128, C = 64) the P-then-S order of one MMA warp is 8 %
+        // faster.
+        p->early_s = stages >= 4;
         // At least ~116 KB so that one CTA (which owns all 512 TMEM columns)
         // runs per SM.
         p->smem_bytes = std::max<size_t>(fixed + stages * stage, 118 * 1024);
@@ -612,11 +738,17 @@ bool plan_tensor(InType t, int64_t M, int64_t N, int64_t D, int64_t C, bool grad
 cudaError_t launch_tc(const TcPlan& p, InType t, float c, char* ws, unsigned* status,
                       cudaStream_t s, const char** why) {
     if (p.aug) {
-        if (p.BN == 128) return launch_bn<128, 16, true>(p, t, c, ws, status, s, why);
-        return launch_bn<64, 8, true>(p, t, c, ws, status, s, why);
+        if (p.BN == 128)
+            return p.early_s ? launch_bn<128, 16, true, true>(p, t, c, ws, status, s, why)
+                             : launch_bn<128, 16, true, false>(p, t, c, ws, status, s, why);
+        return p.early_s ? launch_bn<64, 8, true, true>(p, t, c, ws, status, s, why)
+                         : launch_bn<64, 8, true, false>(p, t, c, ws, status, s, why);
     }
-    if (p.BN == 128) return launch_bn<128, 16, false>(p, t, c, ws, status, s, why);
-    return launch_bn<64, 8, false>(p, t, c, ws, status, s, why);
+    if (p.BN == 128)
+        return p.early_s ? launch_bn<128, 16, false, true>(p, t, c, ws, status, s, why)
+                         : launch_bn<128, 16, false, false>(p, t, c, ws, status, s, why);
+    return p.early_s ? launch_bn<64, 8, false, true>(p, t, c, ws, status, s, why)
+                     : launch_bn<64, 8, false, false>(p, t, c, ws, status, s, why);
 }
 
 }  // namespace gs

@@ -8,6 +8,8 @@ and key tiles with ragged tails; all calls go through the C ABI.
 import numpy as np
 import pytest
 
+from oracle import oracle_grad_q, oracle_sum
+from paper_2609_04910_gb300.workloads import generate
 from tests.gpu_helpers import TOL, case, device_inputs, forward_check, grad_check, rel_err
 
 pytestmark = pytest.mark.gpu
@@ -95,6 +97,40 @@ def test_long_key_range_one_split(D, dtype):
     # cycle through their stages and S slots many times (q^ in shared
     # memory for D + 4 <= 128, in TMEM otherwise).
     forward_check(case(256, 8192, D, 3, dtype), split_n=1)
+
+
+@pytest.mark.parametrize("M,N,D,C,dtype,grad", [
+    (300, 5000, 64, 16, "fp16", False),   # BN 128, augmented, early S release (six stages)
+    (200, 5000, 64, 100, "fp16", False),  # BN 128, plain operands, early S release (four stages)
+    (200, 5000, 128, 64, "bf16", False),  # BN 128, three stages: one MMA warp, P-then-S order
+    (150, 3000, 32, 200, "fp16", False),  # BN 64, early S release
+    (100, 3000, 256, 200, "fp16", False), # BN 64, two stages: one MMA warp
+    (256, 5000, 32, 1, "fp16", True),     # gradient (33 channels), early S release
+    (128, 3000, 100, 1, "bf16", True),    # gradient (101 channels), three stages
+])
+def test_two_mma_long_key_range(M, N, D, C, dtype, grad):
+    """Two-MMA kernel over long key ranges in one split (tens of key tiles
+    per CTA, so both S/P buffers and all stages cycle many times) on both
+    schedules: the early S release with MMA1 and MMA2 issued by two warps,
+    and one MMA warp in P-then-S order.  Repeated calls agree bit for bit
+    and match the oracle."""
+    import paper_2609_04910_gb300 as gs
+    w = case(M, N, D, C, dtype, kind="mmd" if grad else "normal")
+    inp = generate(w)
+    q, k, v = device_inputs(inp)
+    path = gs.GS_PATH_TENSOR
+    if grad:
+        outs = [gs.gauss_sum_grad_q(q, k, v, w.tau, split_n=1)[0] for _ in range(3)]
+    else:
+        outs = [gs.gauss_sum(q, k, v, w.tau, split_n=1, path=path) for _ in range(3)]
+    gs.gauss_sum_device_status()
+    assert all(torch.equal(outs[0], o) for o in outs[1:])
+    got = outs[0].cpu().numpy()
+    if grad:
+        ref, _, den, _ = oracle_grad_q(inp["q64"], inp["k64"], inp["v64"], w.tau)
+    else:
+        ref, den = oracle_sum(inp["q64"], inp["k64"], inp["v64"], w.tau)
+    assert rel_err(got, ref, den) <= TOL[dtype]
 
 
 @pytest.mark.parametrize("dtype", ["fp16", "bf16"])
