@@ -556,7 +556,6 @@ bool plan_tensor(InType t, int64_t M, int64_t N, int64_t D, int64_t C, bool grad
     p->center = center;
     p->tf = false;
     p->early_s = false;
-    const int nkb = (p->Dp + KB - 1) / KB;
     size_t fma_smem = 0;
     int fma_stages = 0, nq = 1;
     if (t == InType::F32) {

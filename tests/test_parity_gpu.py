@@ -133,6 +133,19 @@ def test_two_mma_long_key_range(M, N, D, C, dtype, grad):
     assert rel_err(got, ref, den) <= TOL[dtype]
 
 
+@pytest.mark.parametrize("N", [100, 256, 300, 500, 640])
+@pytest.mark.parametrize("D,C,grad", [(64, 16, False), (32, 200, False), (32, 1, True)])
+def test_two_mma_few_key_tiles(N, D, C, grad):
+    """One to five key tiles in one split on the early-release schedule
+    (BN 128 and BN 64 forward, gradient): the MMA1 warp's first tiles need no
+    S release, the second group may have no tile at all, and the MMA2 warp
+    ends on either group."""
+    if grad:
+        grad_check(case(150, N, D, 1, "fp16"), split_n=1)
+    else:
+        forward_check(case(150, N, D, C, "fp16"), split_n=1)
+
+
 @pytest.mark.parametrize("dtype", ["fp16", "bf16"])
 def test_centering_off(dtype):
     forward_check(case(200, 400, 32, 2, dtype), center=False)
