@@ -69,6 +69,28 @@ __device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
     asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
 }
 
+// Arrive on `bar` when sel == 0 (e.g. sel = lane: one arrival per warp),
+// as a predicated instruction instead of a branch.
+__device__ __forceinline__ void mbar_arrive_if_zero(uint64_t* bar, uint32_t sel) {
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "setp.eq.u32 p, %1, 0;\n\t"
+        "@p mbarrier.arrive.shared::cta.b64 _, [%0];\n\t}" ::"r"(smem_u32(bar)),
+        "r"(sel)
+        : "memory");
+}
+
+// Arrive on bar1 and on bar2 when sel == 0, predicated.
+__device__ __forceinline__ void mbar_arrive2_if_zero(uint64_t* bar1, uint64_t* bar2, uint32_t sel) {
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "setp.eq.u32 p, %2, 0;\n\t"
+        "@p mbarrier.arrive.shared::cta.b64 _, [%0];\n\t"
+        "@p mbarrier.arrive.shared::cta.b64 _, [%1];\n\t}" ::"r"(smem_u32(bar1)),
+        "r"(smem_u32(bar2)), "r"(sel)
+        : "memory");
+}
+
 __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
     uint32_t ok;
     asm volatile(

