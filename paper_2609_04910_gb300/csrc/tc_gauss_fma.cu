@@ -487,8 +487,11 @@ tc_gauss_fma_kernel(const __grid_constant__ CUtensorMap tm_q,
                 // that stage and slot.  Two slots only: with one, tile j + 1
                 // needs the slot this warp has just handed back, so the query
                 // would always fail (and skipping it measured 4 % faster on
-                // the D = 256, 1M-key workload).
-                if (QSM) {
+                // the D = 256, 1M-key workload).  Not with 3xTF32 operands
+                // either: their three MMAs per K step make the next tile rarely
+                // ready this early (skipping the query: fp32 65536^2 sums 4-5 %
+                // faster).
+                if (QSM && !TF) {
                     RingPos st2 = st, sl2 = sl;
                     st2.advance(p.stages);
                     sl2.advance(SL);
