@@ -181,10 +181,14 @@ gs_status gauss_sum_batched(const void* q, const void* k, const void* v, double 
  * x (B x N x D) carrying the signed weights v (B x N) of the difference of
  * two discrete measures,
  *     mmd2[b] = sum_{m,n} v[b,m] Phi(x[b,m], x[b,n]) v[b,n] = v_b^T s_b,
- * with s_b the Gauss sum of Eq. 1 for q = k = x_b and C = 1.  mmd2 is a
- * device array of B floats (16-byte aligned); the final sum over m runs in
- * float64 in a fixed order.  Allocates B x N floats on `stream`
- * (cudaMallocAsync) besides the Gauss sum's workspace.
+ * with s_b the Gauss sum of Eq. 1 for q = k = x_b and C = 1.  Since the
+ * kernel matrix is symmetric, fp16 / bf16 points with D + 4 (fp16) or
+ * D + 6 (bf16) <= 128 are evaluated over the upper triangle of 128 x 128
+ * tile pairs only, off-diagonal tiles counted twice (half the
+ * exponentials); other inputs use the full sum.  mmd2 is a device array of
+ * B floats (16-byte aligned); the final sum over m runs in float64 in a
+ * fixed order.  Allocates B x N floats and a few float64 partial sums on
+ * `stream` (cudaMallocAsync) besides the Gauss sum's workspace.
  */
 gs_status gauss_sum_mmd2(const void* x, const void* v, double tau, int64_t B, int64_t N,
                          int64_t D, gs_dtype dtype, float* mmd2, void* stream);

@@ -87,6 +87,10 @@ struct Call {
     bool w_f32 = false;
     const void* u = nullptr;
     bool u_f32 = false;
+    // Only v^T out is wanted (q = k, C = 1): the FMA kernel may evaluate the
+    // upper triangle of tile pairs, and out then holds row sums s' with
+    // sum_m v_m s'_m = v^T K v instead of K v.
+    bool tri = false;
 };
 
 gs_status validate(const Call& c) {
@@ -156,7 +160,7 @@ gs_status plan(const Call& c, int sms, bool* tensor, gs::TcPlan* tp, gs::SimtPla
         int64_t nch = 1;
         const int64_t width = c.grad ? grad_chunk(c.D, c.C, &nch) : c.C;
         if (!gs::plan_tensor(in_type(c.dtype), c.M, c.N, c.D, width, c.grad, c.opt.center != 0,
-                             alias, c.opt.split_n, sms, tp, &why, c.B))
+                             alias, c.opt.split_n, sms, tp, &why, c.B, c.tri && !c.grad))
             return fail(GS_ERR_UNSUPPORTED, "%s", why);
         *bytes = tp->total;
     } else {
@@ -316,7 +320,8 @@ gs_status run(Call c) {
                 e = gs::launch_finalize_slots(reinterpret_cast<float*>(ws + tp.off_part), tp.Mpad,
                                               c.M, static_cast<int>(tp.Cv), 128 * tp.nq,
                                               tp.Npad / tp.BN, tp.unit_len, c.out, c.stream,
-                                              batch, tp.band_len > 0 ? tp.splits : 0);
+                                              batch, tp.band_len > 0 ? tp.splits : 0,
+                                              tp.tri ? tp.Npad / tp.BN : 0);
                 where = "finalise kernel";
             }
         } else if (e == cudaSuccess) {
@@ -525,19 +530,28 @@ gs_status gauss_sum_mmd2(const void* x, const void* v, double tau, int64_t B, in
         return e == cudaSuccess ? GS_OK : cuda_fail(e, "cudaMemsetAsync");
     }
     // s = K v for every problem (q = k = x), then v^T s.  The arguments are
-    // validated with mmd2 standing in for the s buffer allocated below.
+    // validated with mmd2 standing in for the s buffer allocated below.  The
+    // FMA kernel (fp16 / bf16, augmented operands) evaluates only the upper
+    // triangle of tile pairs (K is symmetric): s then holds row sums s' with
+    // v^T s' = v^T K v, at half the exponentials.
     Call c{x, x, v, tau, N, N, D, 1, dtype, false, mmd2, nullptr, st, defaults()};
     c.B = B;
+    c.tri = true;
     gs_status status = validate(c);
     if (status != GS_OK) return status;
     if (forced_alloc_failure()) return fail(GS_ERR_OUT_OF_MEMORY, "workspace allocation failed (test hook)");
     float* s_buf = nullptr;
-    cudaError_t e = cudaMallocAsync(reinterpret_cast<void**>(&s_buf), sizeof(float) * B * N, st);
+    // s (B x N float32), then the float64 chunk partials of the reduction.
+    const size_t s_bytes = (sizeof(float) * B * N + 255) & ~static_cast<size_t>(255);
+    cudaError_t e = cudaMallocAsync(reinterpret_cast<void**>(&s_buf),
+                                    s_bytes + gs::mmd2_partial_bytes(B, N), st);
     if (e != cudaSuccess) return cuda_fail(e, "cudaMallocAsync");
     c.out = s_buf;
     status = run(c);
     if (status == GS_OK) {
-        e = gs::launch_mmd2_reduce(in_type(dtype), s_buf, v, B, N, mmd2, st);
+        e = gs::launch_mmd2_reduce(in_type(dtype), s_buf, v, B, N,
+                                   reinterpret_cast<double*>(reinterpret_cast<char*>(s_buf) + s_bytes),
+                                   mmd2, st);
         if (e != cudaSuccess) status = cuda_fail(e, "MMD reduction kernel");
     }
     cudaError_t ef = cudaFreeAsync(s_buf, st);

@@ -37,6 +37,13 @@ struct TcPlan {
     int nq;                  // query tiles of 128 rows per CTA (FMA kernel)
     bool early_s;            // two-MMA kernel: S buffers handed back as soon as they are
                              // in registers (exponent-bound shapes), else with P
+    // FMA kernel over the upper triangle of tile pairs (q = k, one value
+    // channel; for v^T K v only): pair P of query tiles takes the key tiles
+    // from 2P on, those past its own two with kernel values doubled, so the
+    // row sums s'_m satisfy sum_m v_m s'_m = v^T K v.  tri_units: units per
+    // problem, sum over pairs P of (key tiles - 2P).
+    bool tri;
+    int64_t tri_units;
     // FMA kernel work split: units = (pairs of query tiles) x key tiles, in
     // row-major order; CTA i takes units [i unit_len, (i + 1) unit_len); the
     // partial sums of a pair of query tiles have one slot per contributing
@@ -70,7 +77,7 @@ bool device_is_sm103(int device);
 
 bool plan_tensor(InType t, int64_t M, int64_t N, int64_t D, int64_t C, bool grad, bool center,
                  bool alias, int split_override, int sms, TcPlan* p, const char** why,
-                 int64_t batch = 1);
+                 int64_t batch = 1, bool tri = false);
 bool plan_simt(int64_t M, int64_t N, int64_t D, int64_t C, bool grad, int split_override,
                int sms, SimtPlan* p, const char** why);
 
@@ -104,18 +111,22 @@ cudaError_t launch_finalize_points(bool direct, InType t, bool u_f32, const floa
                                    float tau, int D, int Cw, int ch0, int Cc, const void* u,
                                    int accumulate, float* out, float* s_out, cudaStream_t s);
 // MMD^2 of Sec. 3 per problem of a batch: out[b] = sum_n v[b, n] s[b, n]
-// (float64 accumulation, fixed order).
+// (float64 accumulation, fixed order), through float64 chunk partials in
+// `partial` (mmd2_partial_bytes(B, N) bytes).
+size_t mmd2_partial_bytes(int64_t B, int64_t N);
 cudaError_t launch_mmd2_reduce(InType t, const float* s, const void* v, int64_t B, int64_t N,
-                               float* out, cudaStream_t st);
+                               double* partial, float* out, cudaStream_t st);
 // Forward sum of the FMA kernel's contributor slots, added in slot order:
 // every row has slots 0 .. fixed_slots - 1 when fixed_slots > 0 (banded
 // order); otherwise rows of the pair of query tiles r = m / rows_per_unit
 // have slots 0 .. last(r) - first(r), with first(r) = r key_tiles /
-// unit_len and last(r) = ((r + 1) key_tiles - 1) / unit_len.
+// unit_len and last(r) = ((r + 1) key_tiles - 1) / unit_len; with
+// tri_key_tiles = T > 0 (upper-triangle order, rows of T + 2 units: pair s,
+// then pair T / 2 - 1 - s) pair r = b (T / 2) + P holds T - 2P units.
 cudaError_t launch_finalize_slots(const float* part, int64_t Mpad, int64_t M, int C,
                                   int rows_per_unit, int64_t key_tiles, int64_t unit_len,
                                   float* out, cudaStream_t s, int batch = 1,
-                                  int fixed_slots = 0);
+                                  int fixed_slots = 0, int64_t tri_key_tiles = 0);
 
 // simt_fp32.cu ---------------------------------------------------------
 // grad: keys weighted by channel wch of v (N x Cw); partials have D + 1

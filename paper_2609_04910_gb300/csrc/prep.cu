@@ -371,7 +371,7 @@ __global__ void tf32_split_kernel(const float* __restrict__ x, int64_t rows, int
 __global__ void finalize_slots_kernel(const float* __restrict__ part, int64_t Mpad, int64_t M,
                                       int C, int rows_per_unit, int64_t key_tiles,
                                       int64_t unit_len, int64_t batch, int fixed_slots,
-                                      float* __restrict__ out) {
+                                      int64_t tri_kt, float* __restrict__ out) {
     // out: batch x M x C; partial rows are batch-stacked with Mpad rows per
     // problem and batch Mpad rows per slot.
     const int64_t idx = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
@@ -381,7 +381,19 @@ __global__ void finalize_slots_kernel(const float* __restrict__ part, int64_t Mp
     const int64_t b = bm / M;
     const int64_t m = (bm - b * M) + b * Mpad;
     int64_t nslots = fixed_slots;
-    if (nslots == 0) {
+    if (nslots == 0 && tri_kt > 0) {
+        // Upper-triangle order (folded rows of tri_kt + 2 units: pair s,
+        // then pair ppb - 1 - s): pair P of problem b holds tri_kt - 2P units.
+        const int64_t r = m / rows_per_unit;
+        const int64_t ppb = tri_kt / 2;
+        const int64_t bb = r / ppb, P = r - bb * ppb;
+        const int64_t U = ppb * tri_kt - ppb * (ppb - 1);
+        const int64_t s = 2 * P <= ppb - 1 ? P : ppb - 1 - P;
+        const int64_t start = bb * U + s * (tri_kt + 2) + (s == P ? 0 : tri_kt - 2 * s);
+        const int64_t first = start / unit_len;
+        const int64_t last = (start + tri_kt - 2 * P - 1) / unit_len;
+        nslots = last - first + 1;
+    } else if (nslots == 0) {
         const int64_t r = m / rows_per_unit;
         const int64_t first = r * key_tiles / unit_len;
         const int64_t last = ((r + 1) * key_tiles - 1) / unit_len;
@@ -834,18 +846,24 @@ cudaError_t launch_mean(InType t, const void* q, const void* k, int64_t M, int64
 
 namespace {
 
-// Sec. 3: MMD^2 = v^T s for s = K v (q = k).  One block per problem: each
-// thread folds the products v_n s_n of n = t, t + 256, ... in float64 and a
-// fixed tree adds the threads (deterministic).
+// Sec. 3: MMD^2 = v^T s for s = K v (q = k).  Block g of problem b folds
+// the products v_n s_n of its chunk of kMmdChunk points (n = chunk start + t,
+// + 256, ...) in float64, a fixed tree adds the threads, and
+// mmd2_final_kernel adds the chunks of each problem in order
+// (deterministic).
+constexpr int64_t kMmdChunk = 4096;
+
 template <typename T>
 __global__ void __launch_bounds__(256)
 mmd2_reduce_kernel(const float* __restrict__ s, const T* __restrict__ v, int64_t N,
-                   float* __restrict__ out) {
+                   double* __restrict__ partial) {
     __shared__ double red[256];
     const int t = threadIdx.x;
-    const int64_t b = blockIdx.x;
+    const int64_t b = blockIdx.y;
+    const int64_t n0 = static_cast<int64_t>(blockIdx.x) * kMmdChunk;
+    const int64_t n1 = min(N, n0 + kMmdChunk);
     double acc = 0.0;
-    for (int64_t n = t; n < N; n += 256)
+    for (int64_t n = n0 + t; n < n1; n += 256)
         acc += static_cast<double>(to_f(v[b * N + n])) * static_cast<double>(s[b * N + n]);
     red[t] = acc;
     __syncthreads();
@@ -853,40 +871,62 @@ mmd2_reduce_kernel(const float* __restrict__ s, const T* __restrict__ v, int64_t
         if (t < w) red[t] += red[t + w];
         __syncthreads();
     }
-    if (t == 0) out[b] = static_cast<float>(red[0]);
+    if (t == 0) partial[b * gridDim.x + blockIdx.x] = red[0];
+}
+
+__global__ void mmd2_final_kernel(const double* __restrict__ partial, int chunks, int64_t B,
+                                  float* __restrict__ out) {
+    const int64_t b = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
+    if (b >= B) return;
+    double acc = 0.0;
+    for (int g = 0; g < chunks; ++g) acc += partial[b * chunks + g];
+    out[b] = static_cast<float>(acc);
 }
 
 }  // namespace
 
+size_t mmd2_partial_bytes(int64_t B, int64_t N) {
+    const int64_t chunks = std::max<int64_t>(1, (N + kMmdChunk - 1) / kMmdChunk);
+    return static_cast<size_t>(B * chunks) * sizeof(double);
+}
+
 cudaError_t launch_mmd2_reduce(InType t, const float* s, const void* v, int64_t B, int64_t N,
-                               float* out, cudaStream_t st) {
+                               double* partial, float* out, cudaStream_t st) {
     if (B == 0) return cudaSuccess;
+    const int64_t chunks = std::max<int64_t>(1, (N + kMmdChunk - 1) / kMmdChunk);
+    const dim3 grid(static_cast<unsigned>(chunks), static_cast<unsigned>(B));
     switch (t) {
         case InType::F16:
-            mmd2_reduce_kernel<__half><<<static_cast<unsigned>(B), 256, 0, st>>>(
-                s, static_cast<const __half*>(v), N, out);
+            mmd2_reduce_kernel<__half><<<grid, 256, 0, st>>>(s, static_cast<const __half*>(v), N,
+                                                             partial);
             break;
         case InType::BF16:
-            mmd2_reduce_kernel<__nv_bfloat16><<<static_cast<unsigned>(B), 256, 0, st>>>(
-                s, static_cast<const __nv_bfloat16*>(v), N, out);
+            mmd2_reduce_kernel<__nv_bfloat16><<<grid, 256, 0, st>>>(
+                s, static_cast<const __nv_bfloat16*>(v), N, partial);
             break;
         default:
-            mmd2_reduce_kernel<float><<<static_cast<unsigned>(B), 256, 0, st>>>(
-                s, static_cast<const float*>(v), N, out);
+            mmd2_reduce_kernel<float><<<grid, 256, 0, st>>>(s, static_cast<const float*>(v), N,
+                                                            partial);
     }
+    note_launches(1);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    mmd2_final_kernel<<<static_cast<unsigned>((B + 127) / 128), 128, 0, st>>>(
+        partial, static_cast<int>(chunks), B, out);
     note_launches(1);
     return cudaGetLastError();
 }
 
 cudaError_t launch_finalize_slots(const float* part, int64_t Mpad, int64_t M, int C,
                                   int rows_per_unit, int64_t key_tiles, int64_t unit_len,
-                                  float* out, cudaStream_t s, int batch, int fixed_slots) {
+                                  float* out, cudaStream_t s, int batch, int fixed_slots,
+                                  int64_t tri_key_tiles) {
     const int64_t total = static_cast<int64_t>(batch) * M * C;
     if (total == 0) return cudaSuccess;
     const int threads = 256;
     finalize_slots_kernel<<<static_cast<unsigned>((total + threads - 1) / threads), threads, 0, s>>>(
         part, Mpad, M, C, rows_per_unit, key_tiles, unit_len, static_cast<int64_t>(batch),
-        fixed_slots, out);
+        fixed_slots, tri_key_tiles, out);
     note_launches(1);
     return cudaGetLastError();
 }

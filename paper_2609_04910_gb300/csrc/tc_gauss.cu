@@ -542,7 +542,7 @@ constexpr int64_t kMaxBands = 256;
 
 bool plan_tensor(InType t, int64_t M, int64_t N, int64_t D, int64_t C, bool grad, bool center,
                  bool alias, int split_override, int sms, TcPlan* p, const char** why,
-                 int64_t batch) {
+                 int64_t batch, bool tri) {
     p->M = M;
     p->N = N;
     p->D = D;
@@ -556,6 +556,8 @@ bool plan_tensor(InType t, int64_t M, int64_t N, int64_t D, int64_t C, bool grad
     p->center = center;
     p->tf = false;
     p->early_s = false;
+    p->tri = false;
+    p->tri_units = 0;
     size_t fma_smem = 0;
     int fma_stages = 0, nq = 1;
     if (t == InType::F32) {
@@ -678,6 +680,32 @@ bool plan_tensor(InType t, int64_t M, int64_t N, int64_t D, int64_t C, bool grad
         for (int64_t r = 0; r < tiles; ++r)
             most = std::max(most, ((r + 1) * key_tiles - 1) / len - r * key_tiles / len + 1);
         p->splits = static_cast<int>(most);
+        // v^T K v with q = k and one channel: the upper triangle of tile
+        // pairs only (pair P of query tiles takes key tiles 2P ..), half the
+        // exponentials.
+        if (tri && alias && p->aug && !p->tf && p->Cv == 1 && split_override == 0 &&
+            p->Mpad == p->Npad && key_tiles % 2 == 0 && key_tiles / 2 == p->Mpad / (BM * 2)) {
+            const int64_t ppb = key_tiles / 2;
+            const int64_t U = ppb * key_tiles - ppb * (ppb - 1);
+            const int64_t tunits = B * U;
+            if (tunits < (int64_t(1) << 31)) {
+                const int64_t tlen = std::max<int64_t>(1, (tunits + sms - 1) / sms);
+                int64_t tmost = 1;
+                for (int64_t r = 0; r < B * ppb; ++r) {
+                    // Folded rows of key_tiles + 2 units: pair s, then pair ppb - 1 - s.
+                    const int64_t b = r / ppb, P = r - b * ppb;
+                    const int64_t s = 2 * P <= ppb - 1 ? P : ppb - 1 - P;
+                    const int64_t start = b * U + s * (key_tiles + 2) + (s == P ? 0 : key_tiles - 2 * s);
+                    tmost = std::max(tmost, (start + key_tiles - 2 * P - 1) / tlen - start / tlen + 1);
+                }
+                p->tri = true;
+                p->tri_units = U;
+                p->units = tunits;
+                p->unit_len = tlen;
+                p->grid = static_cast<int>((tunits + tlen - 1) / tlen);
+                p->splits = static_cast<int>(tmost);
+            }
+        }
         // Keys (operand rows and records) larger than half the L2: in the
         // contiguous order the CTAs stand at evenly spread key tiles, so
         // every pair of query tiles reads all keys from DRAM again.  The
@@ -686,7 +714,7 @@ bool plan_tensor(InType t, int64_t M, int64_t N, int64_t D, int64_t C, bool grad
         const double key_bytes =
             static_cast<double>(B) * p->Npad *
             ((p->tf ? 8.0 : 2.0) * p->Dp + 2.0 * ((p->aug ? 0 : 1) + p->Cv));
-        if (split_override == 0 && key_bytes > kBandMinKeyBytes && key_tiles > kBandTiles) {
+        if (!p->tri && split_override == 0 && key_bytes > kBandMinKeyBytes && key_tiles > kBandTiles) {
             const int64_t blen = std::max<int64_t>(kBandTiles, (key_tiles + kMaxBands - 1) / kMaxBands);
             const int64_t nbands = (key_tiles + blen - 1) / blen;
             const int64_t nruns = tiles * nbands;

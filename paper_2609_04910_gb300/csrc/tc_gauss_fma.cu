@@ -94,7 +94,7 @@ struct FmaParams {
     // r / pairs_total, pair of query tiles r % pairs_total) covers band_len
     // key tiles; CTA i takes runs i, i + grid, ...; the slot is the band.
     int band_len;
-    int nruns;
+    int nruns;           // banded order: runs; upper-triangle order (TRI): units per problem
     int pairs_total;
     int key_tiles;       // key tiles per problem
     int pairs_per_batch; // pairs of query tiles per problem of a batch
@@ -139,8 +139,40 @@ struct Segment {
 // the CTA's run of units [u, u_end) split at query-pair boundaries, slot =
 // rank of this CTA among the CTAs of that pair.  Banded order: runs
 // blockIdx.x, blockIdx.x + gridDim.x, ..., slot = band.
+template <bool TRI>
 __device__ __forceinline__ bool next_segment(const FmaParams& p, int u_end, int& u, int& run,
                                              Segment& sg) {
+    if (TRI) {
+        // Upper-triangle order: pair P of query tiles takes the key tiles
+        // 2P .. KT - 1 (KT - 2P units).  Pairs are folded into rows of equal
+        // length KT + 2: row s holds pair s, then pair PPB - 1 - s (2s + 2
+        // units); with PPB odd the middle pair forms a last, shorter row.
+        // Every CTA thus walks about the same number of pairs.
+        if (u >= u_end) return false;
+        const int64_t U = p.nruns;
+        const int64_t KT = p.key_tiles;
+        const int64_t PPB = p.pairs_per_batch;
+        const int64_t b = u / U;
+        const int64_t r = u - b * U;
+        const int64_t s = r / (KT + 2);
+        const int64_t o = r - s * (KT + 2);
+        int64_t P, start, j0;
+        if (o < KT - 2 * s) {
+            P = s;                                   // first pair of the row
+            start = s * (KT + 2);
+            j0 = o;
+        } else {
+            P = PPB - 1 - s;                         // second pair of the row
+            start = s * (KT + 2) + (KT - 2 * s);
+            j0 = o - (KT - 2 * s);
+        }
+        sg.tile_m = static_cast<int>(b * PPB + P);
+        sg.kt0 = static_cast<int>(2 * P + j0);
+        sg.T = min(p.key_tiles - sg.kt0, u_end - u);
+        sg.slot = static_cast<int>(blockIdx.x) - static_cast<int>((b * U + start) / p.unit_len);
+        u += sg.T;
+        return true;
+    }
     if (p.band_len == 0) {
         if (u >= u_end) return false;
         sg.tile_m = u / p.key_tiles;
@@ -169,7 +201,10 @@ __device__ __forceinline__ void exp_warps_sync() {
 // AUG: augmented operands (S = -||q^ - k^||^2 / 2; no norm terms in the
 // key records).  QSM: q^ tiles in shared memory (A operand from shared
 // memory, SL = 2); otherwise q^ in TMEM (A operand from TMEM, SL = 1).
-template <int C, bool AUG, bool QSM, bool TF>
+// TRI: upper-triangle order for v^T K v (q = k, C = 1, augmented
+// operands): key tiles past the pair's own two get the weight 2, applied as
+// +1 in the exponent.
+template <int C, bool AUG, bool QSM, bool TF, bool TRI>
 __global__ void __launch_bounds__(THREADS, 1)
 tc_gauss_fma_kernel(const __grid_constant__ CUtensorMap tm_q,
                     const __grid_constant__ CUtensorMap tm_k, const FmaParams p) {
@@ -242,7 +277,7 @@ tc_gauss_fma_kernel(const __grid_constant__ CUtensorMap tm_q,
         uint32_t seg_parity = 0;   // parity of the qa_ready phase of this segment
         int u = u_begin, run = 0, g0 = 0;   // g0: running index of the segment's first tile
         Segment sg;
-        for (; next_segment(p, u_end, u, run, sg); seg_parity ^= 1u, g0 += sg.T) {
+        for (; next_segment<TRI>(p, u_end, u, run, sg); seg_parity ^= 1u, g0 += sg.T) {
         // Read by every thread after a CTA barrier: uniform.
         if (*abort_flag) break;
         const int tile_m = sg.tile_m;         // query tiles 2 tile_m, 2 tile_m + 1
@@ -400,11 +435,14 @@ tc_gauss_fma_kernel(const __grid_constant__ CUtensorMap tm_q,
         uint32_t seg_parity = 0;
         int u = u_begin, run = 0, g0 = 0;
         Segment sg;
-        for (; next_segment(p, u_end, u, run, sg); seg_parity ^= 1u, g0 += sg.T) {
+        for (; next_segment<TRI>(p, u_end, u, run, sg); seg_parity ^= 1u, g0 += sg.T) {
         // Read by every thread after a CTA barrier: uniform.
         if (*abort_flag) break;
         const int tile_m = sg.tile_m;         // query tiles 2 tile_m, 2 tile_m + 1
         const int T = sg.T;
+        // TRI: tiles j >= w_from of this segment lie past the pair's own two
+        // key tiles; their kernel values count twice.
+        const int w_from = TRI ? 2 * (tile_m % p.pairs_per_batch) + 2 - sg.kt0 : 0;
         const int slot = sg.slot;
 
             // ------------------------------------------------ exponent warps
@@ -499,6 +537,7 @@ tc_gauss_fma_kernel(const __grid_constant__ CUtensorMap tm_q,
                                                          &bars->s_full[sl2.idx], sl2.phase);
                 }
                 const float* rec = rec_smem(s) + (cg * 16) * REC_PAIR;
+                const uint64_t w2 = (TRI && j >= w_from) ? f32x2_pack(1.f, 1.f) : 0ull;
                 if (AUG) {
                     // Augmented operands: S = -||q^ - k^||^2 / 2, so Phi = 2^(c S).
                     // Keys 32 cg + 2t and + 1, rows row0 (S0) and row1 (S1).
@@ -510,14 +549,16 @@ tc_gauss_fma_kernel(const __grid_constant__ CUtensorMap tm_q,
                             px = exp2_fma_x2(__uint_as_float(r0[2 * t]), __uint_as_float(r0[2 * t + 1]), c2, s_min);
                         } else {
                             float x0, x1;
-                            f32x2_unpack(f32x2_mul(f32x2_pack(__uint_as_float(r0[2 * t]), __uint_as_float(r0[2 * t + 1])), c2), x0, x1);
+                            const uint64_t sx = f32x2_pack(__uint_as_float(r0[2 * t]), __uint_as_float(r0[2 * t + 1]));
+                            f32x2_unpack(TRI ? f32x2_fma(sx, c2, w2) : f32x2_mul(sx, c2), x0, x1);
                             px = f32x2_pack(ex2_approx(x0), ex2_approx(x1));
                         }
                         if (kSoftExpY >= 0 && (t & kSoftExpY) == 0) {
                             py = exp2_fma_x2(__uint_as_float(r1[2 * t]), __uint_as_float(r1[2 * t + 1]), c2, s_min);
                         } else {
                             float y0, y1;
-                            f32x2_unpack(f32x2_mul(f32x2_pack(__uint_as_float(r1[2 * t]), __uint_as_float(r1[2 * t + 1])), c2), y0, y1);
+                            const uint64_t sy = f32x2_pack(__uint_as_float(r1[2 * t]), __uint_as_float(r1[2 * t + 1]));
+                            f32x2_unpack(TRI ? f32x2_fma(sy, c2, w2) : f32x2_mul(sy, c2), y0, y1);
                             py = f32x2_pack(ex2_approx(y0), ex2_approx(y1));
                         }
     #pragma unroll
@@ -633,7 +674,7 @@ size_t q_bytes_for(int nkb, bool qsm) {
     return qsm ? static_cast<size_t>(NQ) * nkb * BM * 128 : 0;
 }
 
-template <int C, bool AUG, bool QSM, bool TF>
+template <int C, bool AUG, bool QSM, bool TF, bool TRI = false>
 cudaError_t launch_typed(const TcPlan& pl, InType t, float c, char* ws, unsigned* status,
                          cudaStream_t s, const char** why) {
     const CUtensorMapDataType hdt =
@@ -662,7 +703,7 @@ cudaError_t launch_typed(const TcPlan& pl, InType t, float c, char* ws, unsigned
     p.units = static_cast<int>(pl.units);
     p.unit_len = static_cast<int>(pl.unit_len);
     p.band_len = pl.band_len;
-    p.nruns = static_cast<int>(pl.nruns);
+    p.nruns = static_cast<int>(pl.tri ? pl.tri_units : pl.nruns);
     p.pairs_total = static_cast<int>((pl.Mpad / (NQ * BM)) * pl.batch);
     p.Dp = pl.Dp;
     p.nkb = nkb_for(pl.Dp, TF);
@@ -677,12 +718,12 @@ cudaError_t launch_typed(const TcPlan& pl, InType t, float c, char* ws, unsigned
     p.c = c;
     const uint32_t hb = t == InType::BF16 ? 1u : 0u;
     p.idesc = TF ? idesc_tf32(BM, BN) : idesc_f16(BM, BN, hb, hb);
-    cudaError_t e = cudaFuncSetAttribute(tc_gauss_fma_kernel<C, AUG, QSM, TF>,
+    cudaError_t e = cudaFuncSetAttribute(tc_gauss_fma_kernel<C, AUG, QSM, TF, TRI>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          static_cast<int>(pl.smem_bytes));
     if (e != cudaSuccess) return e;
     dim3 grid(static_cast<unsigned>(pl.grid));
-    tc_gauss_fma_kernel<C, AUG, QSM, TF><<<grid, THREADS, pl.smem_bytes, s>>>(tm_q, tm_k, p);
+    tc_gauss_fma_kernel<C, AUG, QSM, TF, TRI><<<grid, THREADS, pl.smem_bytes, s>>>(tm_q, tm_k, p);
     note_launches(1);
     return cudaGetLastError();
 }
@@ -691,6 +732,9 @@ template <int C>
 cudaError_t launch_c(const TcPlan& pl, InType t, float c, char* ws, unsigned* status,
                      cudaStream_t s, const char** why) {
     if (pl.tf) return launch_typed<C, false, true, true>(pl, t, c, ws, status, s, why);
+    if constexpr (C == 1 && kAugQsm) {
+        if (pl.tri && pl.aug) return launch_typed<1, true, true, false, true>(pl, t, c, ws, status, s, why);
+    }
     if (pl.aug) return launch_typed<C, true, kAugQsm, false>(pl, t, c, ws, status, s, why);
     return launch_typed<C, false, false, false>(pl, t, c, ws, status, s, why);
 }

@@ -107,3 +107,27 @@ def test_mmd2_of_equal_samples_vanishes():
     gs.gauss_sum_device_status()
     _, den = oracle_mmd2(x.astype(np.float64), v.astype(np.float64), 1 / 24)
     assert abs(float(got[0])) <= TOL["fp16"] * den
+
+
+@pytest.mark.parametrize("B,N,D,dtype", [
+    (1, 20000, 64, "fp16"),   # one problem, many CTAs per pair of query tiles
+    (5, 3000, 32, "fp16"),    # CTA runs crossing pairs and problems, ragged N
+    (4, 2100, 100, "bf16"),   # bf16 augmented operands (three norm terms)
+    (2, 1000, 125, "fp16"),   # no augmented operands: the full sum K v is used
+])
+def test_mmd2_upper_triangle(B, N, D, dtype):
+    """MMD^2 over the upper triangle of tile pairs (K symmetric, off-diagonal
+    tiles counted twice) against the oracle and against v^T (K v) from the
+    full Gauss sum."""
+    import paper_2609_04910_gb300 as gs
+    from oracle import oracle_mmd2
+    w, inps, x, _, v = _stacked(B, N, N, D, 1, dtype, q_is_k=True, kind="mmd")
+    v1 = v[..., 0].contiguous()
+    got = gs.gauss_sum_mmd2(x, v1, w.tau).cpu().numpy().astype(np.float64)
+    full = gs.gauss_sum_batched(x, x, v, w.tau)
+    gs.gauss_sum_device_status()
+    vt_s = (v1.double() * full[..., 0].double()).sum(dim=1).cpu().numpy()
+    for b, inp in enumerate(inps):
+        ref, den = oracle_mmd2(inp["q64"], inp["v64"][:, 0], w.tau)
+        assert abs(got[b] - ref) <= TOL[dtype] * den + 1e-30, (b, got[b], ref, den)
+        assert abs(got[b] - vt_s[b]) <= 2 * TOL[dtype] * den + 1e-30, (b, got[b], vt_s[b], den)
