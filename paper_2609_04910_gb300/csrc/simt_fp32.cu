@@ -12,7 +12,10 @@
 //   gradient (Sec. 3):   acc[d] += Phi w_n (k_d - q_d),   acc[D] += Phi w_n
 //                        with w_n = v[n, c] for one weight channel c
 // The key range is split over gridDim.y; partial sums go to a workspace and
-// are added in a fixed order by the finalise kernel.
+// are added in a fixed order by the finalise kernel.  Coordinates are
+// handled in pairs with the packed f32x2 subtract / FMA of sm_100+ (the
+// squared distance accumulates even and odd coordinates separately and
+// adds the two at the end).
 #include <algorithm>
 
 #include "internal.h"
@@ -29,7 +32,6 @@ __global__ void __launch_bounds__(THREADS)
 simt_gauss_kernel(const float* __restrict__ q, const float* __restrict__ k,
                   const float* __restrict__ v, int64_t M, int64_t N, int D, int Cv,
                   int wch, float half_c, int64_t keys_per_split, float* __restrict__ part) {
-    constexpr int NACC = GRAD ? DMAX + 1 : CBLK;
     __shared__ __align__(16) float ks[KT][DMAX];
     __shared__ float vs[KT][GRAD ? 1 : CBLK];
 
@@ -39,12 +41,17 @@ simt_gauss_kernel(const float* __restrict__ q, const float* __restrict__ k,
     const int64_t n_begin = static_cast<int64_t>(split) * keys_per_split;
     const int64_t n_end = min(N, n_begin + keys_per_split);
 
-    float qr[DMAX];
+    uint64_t qr[DMAX / 2];   // coordinate pairs of the query row
 #pragma unroll
-    for (int d = 0; d < DMAX; ++d) qr[d] = (m < M && d < D) ? q[m * D + d] : 0.f;
-    float acc[NACC];
+    for (int d = 0; d < DMAX; d += 2)
+        qr[d / 2] = f32x2_pack((m < M && d < D) ? q[m * D + d] : 0.f,
+                               (m < M && d + 1 < D) ? q[m * D + d + 1] : 0.f);
+    float acc[GRAD ? 1 : CBLK];      // forward channels; gradient: sum of w
+    uint64_t acc2[GRAD ? DMAX / 2 : 1];   // gradient coordinates, in pairs
 #pragma unroll
-    for (int j = 0; j < NACC; ++j) acc[j] = 0.f;
+    for (int j = 0; j < (GRAD ? 1 : CBLK); ++j) acc[j] = 0.f;
+#pragma unroll
+    for (int j = 0; j < (GRAD ? DMAX / 2 : 1); ++j) acc2[j] = 0ull;
 
     for (int64_t t0 = n_begin; t0 < n_end; t0 += KT) {
         const int cnt = static_cast<int>(min(static_cast<int64_t>(KT), n_end - t0));
@@ -65,28 +72,29 @@ simt_gauss_kernel(const float* __restrict__ q, const float* __restrict__ k,
         }
         __syncthreads();
         for (int kk = 0; kk < cnt; ++kk) {
-            float d2 = 0.f;
+            uint64_t d2p = 0ull;   // (even, odd) partial squared distances
 #pragma unroll
             for (int d = 0; d < DMAX; d += 4) {
                 const float4 kv = *reinterpret_cast<const float4*>(&ks[kk][d]);
-                float t;
-                t = qr[d + 0] - kv.x; d2 = fmaf(t, t, d2);
-                t = qr[d + 1] - kv.y; d2 = fmaf(t, t, d2);
-                t = qr[d + 2] - kv.z; d2 = fmaf(t, t, d2);
-                t = qr[d + 3] - kv.w; d2 = fmaf(t, t, d2);
+                const uint64_t t0 = f32x2_sub(qr[d / 2], f32x2_pack(kv.x, kv.y));
+                const uint64_t t1 = f32x2_sub(qr[d / 2 + 1], f32x2_pack(kv.z, kv.w));
+                d2p = f32x2_fma(t0, t0, d2p);
+                d2p = f32x2_fma(t1, t1, d2p);
             }
-            const float phi = ex2_approx(-half_c * d2);
+            float d2e, d2o;
+            f32x2_unpack(d2p, d2e, d2o);
+            const float phi = ex2_approx(-half_c * (d2e + d2o));
             if (GRAD) {
                 const float w = phi * vs[kk][0];
+                const uint64_t w2 = f32x2_pack(w, w);
 #pragma unroll
                 for (int d = 0; d < DMAX; d += 4) {
                     const float4 kv = *reinterpret_cast<const float4*>(&ks[kk][d]);
-                    acc[d + 0] = fmaf(w, kv.x - qr[d + 0], acc[d + 0]);
-                    acc[d + 1] = fmaf(w, kv.y - qr[d + 1], acc[d + 1]);
-                    acc[d + 2] = fmaf(w, kv.z - qr[d + 2], acc[d + 2]);
-                    acc[d + 3] = fmaf(w, kv.w - qr[d + 3], acc[d + 3]);
+                    acc2[d / 2] = f32x2_fma(w2, f32x2_sub(f32x2_pack(kv.x, kv.y), qr[d / 2]), acc2[d / 2]);
+                    acc2[d / 2 + 1] =
+                        f32x2_fma(w2, f32x2_sub(f32x2_pack(kv.z, kv.w), qr[d / 2 + 1]), acc2[d / 2 + 1]);
                 }
-                acc[DMAX] += w;
+                acc[0] += w;
             } else {
 #pragma unroll
                 for (int j = 0; j < CBLK; ++j) acc[j] = fmaf(phi, vs[kk][j], acc[j]);
@@ -97,9 +105,13 @@ simt_gauss_kernel(const float* __restrict__ q, const float* __restrict__ k,
     if (GRAD) {
         float* out = part + (static_cast<int64_t>(split) * M + m) * (D + 1);
 #pragma unroll
-        for (int d = 0; d < DMAX; ++d)
-            if (d < D) out[d] = acc[d];
-        out[D] = acc[DMAX];
+        for (int d = 0; d < DMAX; d += 2) {
+            float lo, hi;
+            f32x2_unpack(acc2[d / 2], lo, hi);
+            if (d < D) out[d] = lo;
+            if (d + 1 < D) out[d + 1] = hi;
+        }
+        out[D] = acc[0];
     } else {
         float* out = part + (static_cast<int64_t>(split) * M + m) * Cv + c0;
 #pragma unroll
@@ -108,10 +120,9 @@ simt_gauss_kernel(const float* __restrict__ q, const float* __restrict__ k,
     }
 }
 
-template <int DMAX, bool GRAD>
-cudaError_t launch_dmax(const SimtPlan& p, const float* q, const float* k, const float* v,
+template <int DMAX, int CBLK, bool GRAD>
+cudaError_t launch_cblk(const SimtPlan& p, const float* q, const float* k, const float* v,
                         int Cw, int wch, float half_c, float* part, cudaStream_t s) {
-    constexpr int CBLK = 4;
     dim3 grid(static_cast<unsigned>((p.M + THREADS - 1) / THREADS), p.splits,
               GRAD ? 1u : static_cast<unsigned>((p.Cv + CBLK - 1) / CBLK));
     simt_gauss_kernel<DMAX, CBLK, GRAD><<<grid, THREADS, 0, s>>>(
@@ -119,6 +130,14 @@ cudaError_t launch_dmax(const SimtPlan& p, const float* q, const float* k, const
         half_c, p.keys_per_split, part);
     note_launches(1);
     return cudaGetLastError();
+}
+
+// Channel blocks of 4, or of 1 for a single channel (no idle FMAs).
+template <int DMAX, bool GRAD>
+cudaError_t launch_dmax(const SimtPlan& p, const float* q, const float* k, const float* v,
+                        int Cw, int wch, float half_c, float* part, cudaStream_t s) {
+    if (!GRAD && p.Cv == 1) return launch_cblk<DMAX, 1, GRAD>(p, q, k, v, Cw, wch, half_c, part, s);
+    return launch_cblk<DMAX, 4, GRAD>(p, q, k, v, Cw, wch, half_c, part, s);
 }
 
 }  // namespace
