@@ -628,11 +628,13 @@ __global__ void value_prep_kernel(const W* __restrict__ w, const T* __restrict__
                                   int Cw, int ch0, int Cc, int Cp,
                                   const unsigned* __restrict__ vmax_bits, __half* __restrict__ vt,
                                   float* __restrict__ inv_scale) {
-    __shared__ float tile[32][33];
-    const int64_t n0 = static_cast<int64_t>(blockIdx.x) * 32;
+    // A block transposes 64 keys x 32 channels; each thread stores two
+    // adjacent keys of one channel as a half2 (Npad is a multiple of 128).
+    __shared__ float tile[64][33];
+    const int64_t n0 = static_cast<int64_t>(blockIdx.x) * 64;
     const int c0 = blockIdx.y * 32;
 #pragma unroll
-    for (int i = 0; i < 4; ++i) {
+    for (int i = 0; i < 8; ++i) {
         const int64_t n = n0 + threadIdx.y + 8 * i;
         const int c = c0 + threadIdx.x;
         float val = 0.f;
@@ -643,10 +645,12 @@ __global__ void value_prep_kernel(const W* __restrict__ w, const T* __restrict__
 #pragma unroll
     for (int i = 0; i < 4; ++i) {
         const int c = c0 + threadIdx.y + 8 * i;
-        const int64_t n = n0 + threadIdx.x;
+        const int64_t n = n0 + 2 * threadIdx.x;
         if (c < Cp && n < Npad) {
             const float sc = c < Cc ? pow2f(channel_exponent(vmax_bits[c])) : 0.f;
-            vt[static_cast<int64_t>(c) * Npad + n] = __float2half_rn(tile[threadIdx.x][threadIdx.y + 8 * i] * sc);
+            const int cl = threadIdx.y + 8 * i;
+            *reinterpret_cast<__half2*>(vt + static_cast<int64_t>(c) * Npad + n) =
+                __floats2half2_rn(tile[2 * threadIdx.x][cl] * sc, tile[2 * threadIdx.x + 1][cl] * sc);
         }
     }
     if (blockIdx.x == 0 && threadIdx.y == 0) {
@@ -756,7 +760,8 @@ cudaError_t value_prep_typed(const void* w, const void* x, const float* mu, int6
                              unsigned* vmax_bits, void* vt, float* inv_scale, cudaStream_t s) {
     cudaError_t e = cudaMemsetAsync(vmax_bits, 0, sizeof(unsigned) * Cp, s);
     if (e != cudaSuccess) return e;
-    const int64_t rows_per_block = 512;
+    // 64 rows per block: several blocks per SM even for N of a few 10^4.
+    const int64_t rows_per_block = 64;
     const int64_t blocks = N > 0 ? (N + rows_per_block - 1) / rows_per_block : 0;
     if (blocks > 0) {
         value_max_kernel<T, W, GRAD><<<static_cast<unsigned>(blocks), dim3(32, 8), 0, s>>>(
@@ -766,7 +771,7 @@ cudaError_t value_prep_typed(const void* w, const void* x, const float* mu, int6
         e = cudaGetLastError();
         if (e != cudaSuccess) return e;
     }
-    dim3 grid(static_cast<unsigned>((Npad + 31) / 32), static_cast<unsigned>((Cp + 31) / 32));
+    dim3 grid(static_cast<unsigned>((Npad + 63) / 64), static_cast<unsigned>((Cp + 31) / 32));
     value_prep_kernel<T, W, GRAD><<<grid, dim3(32, 8), 0, s>>>(
         static_cast<const W*>(w), static_cast<const T*>(x), mu, N, Npad, D, Cw, ch0, Cc, Cp,
         vmax_bits, static_cast<__half*>(vt), inv_scale);

@@ -18,8 +18,13 @@
 //   * One barrier handshake per key tile: the 2 x (Dp / 16) MMAs of a key
 //     tile are issued back to back and committed once; the exponent warps
 //     release both S buffers and the stage of the key tile with one
-//     arrival per warp on each barrier once the tile is done, and query the
-//     next key tile's barriers before exponentiating the current one.
+//     (predicated) arrival per warp on each barrier once the tile is done,
+//     and, on the two-slot fp16/bf16 path, query the next key tile's
+//     barriers before exponentiating the current one.
+//   * Work order: persistent CTAs over (pair of query tiles, key tile)
+//     units, contiguous runs or (keys beyond half the L2) bands of key
+//     tiles; for v^T K v with q = k (TRI) only the upper triangle of tile
+//     pairs, folded into rows of equal length.
 //   * TMEM holds SL slots of two 128-column S buffers (one per query
 //     tile); key tile j uses slot j % SL, so the MMAs of key tile j only
 //     wait for the release of key tile j - SL.  With Dp <= 128 the query
