@@ -181,6 +181,17 @@ bool forced_alloc_failure() {
     return s && s[0] == '1';
 }
 
+// Test hook: GS_TEST_STALL=1 makes one bounded wait of the next FMA-kernel
+// launch run out (2 s), so that the timeout path and its report through
+// gauss_sum_device_status can be tested without faulting the GPU.  The
+// request lives in the device status words and is cleared with them.
+cudaError_t request_stall_if_asked(unsigned* status, cudaStream_t s) {
+    const char* v = std::getenv("GS_TEST_STALL");
+    if (!(v && v[0] == '1')) return cudaSuccess;
+    static const unsigned one = 1u;
+    return cudaMemcpyAsync(status + gs::kDevStallRequest, &one, sizeof(one), cudaMemcpyHostToDevice, s);
+}
+
 gs_status run(Call c) {
     gs_status st = validate(c);
     if (st != GS_OK) return st;
@@ -311,6 +322,7 @@ gs_status run(Call c) {
                 c.stream, batch);
             where = "key-record kernel";
             if (e == cudaSuccess) e = record_event(c.opt.main_events[0], c.stream);
+            if (e == cudaSuccess) e = request_stall_if_asked(status, c.stream);
             if (e == cudaSuccess) {
                 e = gs::launch_tc_fma(tp, t, cexp, ws, status, c.stream, &why);
                 where = "fused tensor-core kernel";

@@ -20,6 +20,9 @@ namespace gs {
 
 // Device status codes written into the caller-visible status word.
 enum : unsigned { kDevOk = 0u, kDevTimeout = 1u };
+// Index in the device status words of the test-hook request that makes one
+// bounded wait of the FMA kernel run out (words 1-5 record a timeout).
+constexpr int kDevStallRequest = 6;
 
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
     return static_cast<uint32_t>(__cvta_generic_to_shared(p));

@@ -124,6 +124,7 @@ struct __align__(8) FmaBarriers {
     uint64_t s_free[MAX_SL];    // slot phase: both S tiles of a key tile in registers
     uint64_t kv_full[MAX_STAGES];
     uint64_t kv_empty[MAX_STAGES];
+    uint64_t stall;             // test hook: a barrier nothing arrives on
     uint32_t tmem_base;
     int abort_flag;
 };
@@ -254,6 +255,7 @@ tc_gauss_fma_kernel(const __grid_constant__ CUtensorMap tm_q,
     // once per segment.  Each segment writes its partial sums to its slot.
     if (tid == 0) {
         mbar_init(&bars->qa_ready, QSM ? 1 : NEXP);
+        mbar_init(&bars->stall, 1);
         for (int sl = 0; sl < SL; ++sl) {
             mbar_init(&bars->s_full[sl], 1);
             mbar_init(&bars->s_free[sl], NEXP);        // one arrival per exponent warp
@@ -331,6 +333,12 @@ tc_gauss_fma_kernel(const __grid_constant__ CUtensorMap tm_q,
                 }
                 __syncwarp();
                 bool ok = warp_wait(&bars->qa_ready, seg_parity, abort_flag, p.status);
+                // Test hook (status word 6 set by the host): control warp 0 of
+                // CTA 0 waits on a barrier that nothing arrives on, so its
+                // bounded wait runs out and every role takes the abort path.
+                if (ok && k == 0 && blockIdx.x == 0 && g0 == 0 &&
+                    *reinterpret_cast<volatile unsigned*>(p.status + kDevStallRequest) != 0u)
+                    ok = warp_wait(&bars->stall, 0, abort_flag, p.status);
                 const int ksteps = p.ksteps;
                 // Shared-memory descriptors of stage k and of q^ tile 0; query
                 // tile h and K step kk add byte offsets / 16 to the start-address
