@@ -44,6 +44,9 @@ struct TcPlan {
     // problem, sum over pairs P of (key tiles - 2P).
     bool tri;
     int64_t tri_units;
+    // Two-MMA kernel: q^ in tensor memory (MMA1 reads A from TMEM), so that
+    // its shared memory goes to a fourth key stage.
+    bool qtm;
     // FMA kernel work split: units = (pairs of query tiles) x key tiles, in
     // row-major order; CTA i takes units [i unit_len, (i + 1) unit_len); the
     // partial sums of a pair of query tiles have one slot per contributing

@@ -82,6 +82,7 @@ struct TcParams {
     uint32_t tx_bytes;   // bytes a stage's TMA copies deliver
     float c;
     uint32_t idesc1, idesc2;
+    const uint32_t* qh;  // QTM: q^ rows (packed 16-bit pairs, Dp / 2 per row)
 };
 
 struct __align__(8) Barriers {
@@ -119,8 +120,10 @@ static_assert(16 * 32 * kExpRegs2 + 4 * 32 * kCtrlRegs2 <= 640 * 96, "register s
 // AUG: augmented operands (S = -||q^ - k^||^2 / 2, no B records).
 // EARLY: S buffers handed back right after the TMEM loads, MMA1 and MMA2
 // issued by two warps (exponent-bound shapes); otherwise one MMA warp in
-// P-then-S order (tensor-bound shapes).
-template <int BN, int NEXP, bool AUG, bool EARLY>
+// P-then-S order (tensor-bound shapes).  QTM: q^ in TMEM (columns
+// [3 BN + Cp, 3 BN + Cp + Dp / 2), copied there by the exponent warps; MMA1
+// reads A from TMEM), which leaves its shared memory to the key stages.
+template <int BN, int NEXP, bool AUG, bool EARLY, bool QTM = false>
 __global__ void __launch_bounds__(cta_threads<NEXP>(), 1)
 tc_gauss_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
                 const __grid_constant__ CUtensorMap tm_v, const TcParams p) {
@@ -142,7 +145,7 @@ tc_gauss_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant_
     const uint32_t raw_addr = smem_u32(smem_raw);
     uint8_t* smem = smem_raw + (((raw_addr + 1023u) & ~1023u) - raw_addr);
     uint8_t* q_smem = smem;
-    uint8_t* stage0 = smem + p.nkb * (BM * 128);
+    uint8_t* stage0 = smem + (QTM ? 0 : p.nkb * (BM * 128));
     Barriers* bars = reinterpret_cast<Barriers*>(stage0 + p.stages * p.stage_bytes);
 
     const int tid = threadIdx.x;
@@ -156,7 +159,7 @@ tc_gauss_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant_
     volatile int* abort_flag = &bars->abort_flag;
 
     if (tid == 0) {
-        mbar_init(&bars->q_full, 1);
+        mbar_init(&bars->q_full, QTM ? NEXP : 1);   // TMA copy, or one arrival per exponent warp
         mbar_init(&bars->o_full, 1);
         mbar_init(&bars->drain, 1);
         mbar_init(&bars->drain2, 1);
@@ -182,6 +185,7 @@ tc_gauss_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant_
     tc_fence_after();
     const uint32_t tmem = bars->tmem_base;
     const uint32_t S_col0 = 0, P_col0 = 2 * BN, O_col = 3 * BN;
+    const uint32_t Q_col = 3 * BN + static_cast<uint32_t>(p.Cp);   // QTM
 
     auto kh_smem = [&](int s) { return stage0 + s * p.stage_bytes; };
     auto vt_smem = [&](int s) { return stage0 + s * p.stage_bytes + p.kh_bytes; };
@@ -196,12 +200,14 @@ tc_gauss_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant_
         if (T > 0) {
             const bool leader = elect_one();
             if (leader) {
-                tma_prefetch_desc(&tm_q);
                 tma_prefetch_desc(&tm_k);
                 tma_prefetch_desc(&tm_v);
-                mbar_arrive_expect_tx(&bars->q_full, static_cast<uint32_t>(p.nkb * BM * 128));
-                for (int kb = 0; kb < p.nkb; ++kb)
-                    tma_load_2d(q_smem + kb * (BM * 128), &tm_q, &bars->q_full, kb * KB, tile_m * BM);
+                if (!QTM) {
+                    tma_prefetch_desc(&tm_q);
+                    mbar_arrive_expect_tx(&bars->q_full, static_cast<uint32_t>(p.nkb * BM * 128));
+                    for (int kb = 0; kb < p.nkb; ++kb)
+                        tma_load_2d(q_smem + kb * (BM * 128), &tm_q, &bars->q_full, kb * KB, tile_m * BM);
+                }
             }
             __syncwarp();
             int issued = 0;
@@ -251,9 +257,14 @@ tc_gauss_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant_
                 if (leader) {
                     for (int kk = 0; kk < p.ksteps1; ++kk) {
                         const uint32_t koff = static_cast<uint32_t>(kk & 3) * 32;
-                        const uint64_t ad = smem_desc_kmajor_sw128(q_base + (kk >> 2) * (BM * 128) + koff);
                         const uint64_t bd = smem_desc_kmajor_sw128(kh_base + (kk >> 2) * (BN * 128) + koff);
-                        mma_ss_f16(tmem + S_col0 + b * BN, ad, bd, p.idesc1, kk > 0 ? 1u : 0u);
+                        if (QTM) {
+                            mma_ts_f16(tmem + S_col0 + b * BN, tmem + Q_col + kk * 8, bd, p.idesc1,
+                                       kk > 0 ? 1u : 0u);
+                        } else {
+                            const uint64_t ad = smem_desc_kmajor_sw128(q_base + (kk >> 2) * (BM * 128) + koff);
+                            mma_ss_f16(tmem + S_col0 + b * BN, ad, bd, p.idesc1, kk > 0 ? 1u : 0u);
+                        }
                     }
                     mma_commit(&bars->s_full[b]);
                 }
@@ -329,9 +340,14 @@ tc_gauss_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant_
                     if (leader) {
                         for (int kk = 0; kk < p.ksteps1; ++kk) {
                             const uint32_t koff = static_cast<uint32_t>(kk & 3) * 32;
-                            const uint64_t ad = smem_desc_kmajor_sw128(q_base + (kk >> 2) * (BM * 128) + koff);
                             const uint64_t bd = smem_desc_kmajor_sw128(kh_base + (kk >> 2) * (BN * 128) + koff);
-                            mma_ss_f16(tmem + S_col0 + b * BN, ad, bd, p.idesc1, kk > 0 ? 1u : 0u);
+                            if (QTM) {
+                                mma_ts_f16(tmem + S_col0 + b * BN, tmem + Q_col + kk * 8, bd, p.idesc1,
+                                           kk > 0 ? 1u : 0u);
+                            } else {
+                                const uint64_t ad = smem_desc_kmajor_sw128(q_base + (kk >> 2) * (BM * 128) + koff);
+                                mma_ss_f16(tmem + S_col0 + b * BN, ad, bd, p.idesc1, kk > 0 ? 1u : 0u);
+                            }
                         }
                         mma_commit(&bars->s_full[b]);
                     }
@@ -387,6 +403,22 @@ tc_gauss_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant_
         const uint64_t a2 = f32x2_pack(a_m, a_m);
         const uint64_t c2 = f32x2_pack(p.c, p.c);
         const uint32_t lane_base = static_cast<uint32_t>(quarter * 32) << 16;
+        if (QTM) {
+            // q^ rows of this lane quarter -> TMEM (MMA1's A operand): the
+            // NEXP / 4 warps of a quarter take every (NEXP / 4)-th chunk of 8
+            // columns (16 coordinates).
+            const uint32_t* src = p.qh + row * (p.ksteps1 * 8);
+            for (int ck = warp >> 2; ck < p.ksteps1; ck += NEXP / 4) {
+                const uint4 lo = *reinterpret_cast<const uint4*>(src + ck * 8);
+                const uint4 hi = *reinterpret_cast<const uint4*>(src + ck * 8 + 4);
+                const uint32_t r8[8] = {lo.x, lo.y, lo.z, lo.w, hi.x, hi.y, hi.z, hi.w};
+                tmem_st_32x32b_x8(tmem + lane_base + Q_col + ck * 8, r8);
+            }
+            tmem_wait_st();
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&bars->q_full);
+        }
         bool ok = true;
         RingPos st;   // stage of key tile j
         if (group) st.advance(p.stages);
@@ -488,7 +520,7 @@ tc_gauss_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant_
 // ---------------------------------------------------------------- host side
 size_t align1k(size_t x) { return (x + 1023) & ~static_cast<size_t>(1023); }
 
-template <int BN, int NEXP, bool AUG, bool EARLY>
+template <int BN, int NEXP, bool AUG, bool EARLY, bool QTM = false>
 cudaError_t launch_bn(const TcPlan& pl, InType t, float c, char* ws, unsigned* status,
                       cudaStream_t s, const char** why) {
     const CUtensorMapDataType hdt =
@@ -523,12 +555,13 @@ cudaError_t launch_bn(const TcPlan& pl, InType t, float c, char* ws, unsigned* s
     p.idesc2 = idesc_f16(BM, static_cast<uint32_t>(pl.Cp), 0u, 0u);
 
     // Per-device function attribute; cheap enough to set on every launch.
-    cudaError_t e = cudaFuncSetAttribute(tc_gauss_kernel<BN, NEXP, AUG, EARLY>,
+    p.qh = reinterpret_cast<const uint32_t*>(ws + pl.off_qh);
+    cudaError_t e = cudaFuncSetAttribute(tc_gauss_kernel<BN, NEXP, AUG, EARLY, QTM>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          static_cast<int>(pl.smem_bytes));
     if (e != cudaSuccess) return e;
     dim3 grid(static_cast<unsigned>(pl.Mpad / BM), static_cast<unsigned>(pl.splits));
-    tc_gauss_kernel<BN, NEXP, AUG, EARLY><<<grid, cta_threads<NEXP>(), pl.smem_bytes, s>>>(tm_q, tm_k, tm_v, p);
+    tc_gauss_kernel<BN, NEXP, AUG, EARLY, QTM><<<grid, cta_threads<NEXP>(), pl.smem_bytes, s>>>(tm_q, tm_k, tm_v, p);
     note_launches(1);
     return cudaGetLastError();
 }
@@ -558,6 +591,7 @@ bool plan_tensor(InType t, int64_t M, int64_t N, int64_t D, int64_t C, bool grad
     p->early_s = false;
     p->tri = false;
     p->tri_units = 0;
+    p->qtm = false;
     size_t fma_smem = 0;
     int fma_stages = 0, nq = 1;
     if (t == InType::F32) {
@@ -611,9 +645,20 @@ bool plan_tensor(InType t, int64_t M, int64_t N, int64_t D, int64_t C, bool grad
         const size_t stage = align1k(static_cast<size_t>(nkb) * p->BN * 128 +
                                      static_cast<size_t>(p->BN / KB) * p->Cp * 128 + p->BN * 4);
         const size_t qbytes = static_cast<size_t>(nkb) * BM * 128;
-        const size_t fixed = 1024 /*alignment slack*/ + qbytes + sizeof(Barriers) + 64;
+        size_t fixed = 1024 /*alignment slack*/ + qbytes + sizeof(Barriers) + 64;
         const size_t budget = 232448;
         int stages = static_cast<int>(std::min<size_t>(6, (budget - fixed) / stage));
+        // Fewer than four stages: q^ moves to tensor memory when its Dp / 2
+        // columns fit beside S, P and O (3 BN + Cp + Dp / 2 <= 512), and its
+        // shared memory buys another stage.
+        if (stages < 4 && !p->aug && p->BN == 128 && 3 * 128 + p->Cp + p->Dp / 2 <= static_cast<int>(TMEM_COLS)) {
+            const int st_t = static_cast<int>(std::min<size_t>(6, (budget - (fixed - qbytes)) / stage));
+            if (st_t > stages) {
+                p->qtm = true;
+                fixed -= qbytes;
+                stages = st_t;
+            }
+        }
         if (stages < 2) { *why = "shared-memory budget exceeded"; return false; }
         p->stages = stages;
         // Early S release with two MMA warps lets MMA1 run up to two key
@@ -771,6 +816,9 @@ cudaError_t launch_tc(const TcPlan& p, InType t, float c, char* ws, unsigned* st
         return p.early_s ? launch_bn<64, 8, true, true>(p, t, c, ws, status, s, why)
                          : launch_bn<64, 8, true, false>(p, t, c, ws, status, s, why);
     }
+    if (p.BN == 128 && p.qtm)
+        return p.early_s ? launch_bn<128, 16, false, true, true>(p, t, c, ws, status, s, why)
+                         : launch_bn<128, 16, false, false, true>(p, t, c, ws, status, s, why);
     if (p.BN == 128)
         return p.early_s ? launch_bn<128, 16, false, true>(p, t, c, ws, status, s, why)
                          : launch_bn<128, 16, false, false>(p, t, c, ws, status, s, why);
