@@ -36,6 +36,24 @@ MUTANTS = {
     "vjp_q_contraction": ("w += gm[c] * vn[c];", "w += gm[0] * vn[c];"),
     "vjp_k_contraction": ("w += vn[c] * gm[c];", "w += vn[c] * gm[c] * (c == 0);"),
     "vjp_q_factor": ("if (out) out[d] *= tau;", "if (out) out[d] *= 0.5 * tau;"),
+    # The error scales of the VJP (the denominators of its parity bar).
+    "vjp_dq_signed_upstream": (
+        "e += fabs(gm[c]) * (a[c * Dm + d] + fabs(qm[d] - mu[d]) * b[c]);",
+        "e += gm[c] * (a[c * Dm + d] + fabs(qm[d] - mu[d]) * b[c]);"),
+    "vjp_dq_first_channel": (
+        "e += fabs(gm[c]) * (a[c * Dm + d] + fabs(qm[d] - mu[d]) * b[c]);",
+        "e += fabs(gm[0]) * (a[c * Dm + d] + fabs(qm[d] - mu[d]) * b[c]);"),
+    "vjp_dk_dropped_shift_term": (
+        "e += fabs(vn[c]) * (a[c * Dm + d] + fabs(kn[d] - mu[d]) * b[c]);",
+        "e += fabs(vn[c]) * a[c * Dm + d];"),
+    "vjp_dk_unweighted_abs": (
+        "a[c * Dm + d] += pg * fabs(qm[d] - mu[d]);",
+        "a[c * Dm + d] += pg * (qm[d] - mu[d]);"),
+    "vjp_dv_signed_accumulation": ("const double pg = phi * fabs(gm[c]);",
+                                   "const double pg = phi * gm[c];"),
+    "vjp_dv_channel": ("dv[r * C + c] = b[c];", "dv[r * C + c] = b[0];"),
+    "vjp_dq_value_magnitude": ("const double pv = phi * fabs(vn[c]);",
+                               "const double pv = phi * vn[c];"),
 }
 
 
@@ -98,6 +116,21 @@ def _pin_failures(lib):
             if abs(fd - got[idx]) > 1e-6 * (1 + abs(fd)):
                 fails.append(f"vjp_fd_{which}")
                 break
+    # VJP error scales (C = 2, signed non-unit upstream g) against the
+    # scales of the q-gradient and forward oracles, contracted per channel.
+    q = rng.standard_normal((3, 2)) + 1.0
+    k = rng.standard_normal((4, 2)) - 0.5
+    v = rng.standard_normal((4, 2)) * np.array([1.0, -2.0])
+    up = rng.standard_normal((3, 2)) * np.array([-1.5, 0.5])
+    r = oracle_vjp(q, k, v, up, 0.8, lib_path=lib)
+    dq = sum(np.abs(up[:, c:c + 1]) * oracle_grad_q(q, k, v[:, c], 0.8, lib_path=lib)[2]
+             for c in range(2))
+    dk = sum(np.abs(v[:, c:c + 1]) * oracle_grad_q(k, q, up[:, c], 0.8, lib_path=lib)[2]
+             for c in range(2))
+    dv = oracle_sum(k, q, up, 0.8, lib_path=lib)[1]
+    for name, got, want in (("dq", r["dq"], dq), ("dk", r["dk"], dk), ("dv", r["dv"], dv)):
+        if not np.allclose(got, want, rtol=1e-12, atol=0):
+            fails.append(f"vjp_scale_{name}")
     return fails
 
 

@@ -453,3 +453,71 @@ def test_vjp_row_subsets_and_scales():
         assert np.all(np.abs(full[key]) <= full[den] * (1 + 1e-12))
     with pytest.raises(ValueError):
         oracle_vjp(q, k, v, g, 0.6, rows_q=[M])
+
+
+def test_vjp_error_scales_brute_force_signed_upstream():
+    """The three error scales of the vector-Jacobian product for C = 2 and a
+    signed, non-unit upstream g, recomputed by a pure-Python double loop
+    (math.fsum) from their definitions: the terms of the per-channel Gauss
+    sums with values (w x^, w) in coordinates shifted by the common mean mu,
+    contracted with the magnitudes of the other side's weights (chain rule on
+    Eq. 1, the gradient flows of Sec. 3)."""
+    from oracle import oracle_vjp
+    rng = np.random.default_rng(25)
+    M, N, D, C, tau = 4, 5, 3, 2, 0.7
+    q = rng.standard_normal((M, D)) + 1.5
+    k = rng.standard_normal((N, D)) - 0.5
+    v = rng.standard_normal((N, C)) * np.array([1.0, -3.0])
+    g = rng.standard_normal((M, C)) * np.array([-2.5, 0.4])
+    r = oracle_vjp(q, k, v, g, tau)
+    mu = np.concatenate([q, k]).mean(0)
+    phi = [[math.exp(-tau / 2 * math.fsum((q[m] - k[n]) ** 2)) for n in range(N)]
+           for m in range(M)]
+    for m in range(M):
+        for d in range(D):
+            want = tau * math.fsum(
+                abs(g[m, c]) * (math.fsum(phi[m][n] * abs(v[n, c]) * abs(k[n, d] - mu[d])
+                                          for n in range(N))
+                                + abs(q[m, d] - mu[d]) * math.fsum(phi[m][n] * abs(v[n, c])
+                                                                    for n in range(N)))
+                for c in range(C))
+            assert r["dq"][m, d] == pytest.approx(want, rel=1e-13)
+    for n in range(N):
+        for d in range(D):
+            want = tau * math.fsum(
+                abs(v[n, c]) * (math.fsum(phi[m][n] * abs(g[m, c]) * abs(q[m, d] - mu[d])
+                                          for m in range(M))
+                                + abs(k[n, d] - mu[d]) * math.fsum(phi[m][n] * abs(g[m, c])
+                                                                    for m in range(M)))
+                for c in range(C))
+            assert r["dk"][n, d] == pytest.approx(want, rel=1e-13)
+        for c in range(C):
+            want = math.fsum(phi[m][n] * abs(g[m, c]) for m in range(M))
+            assert r["dv"][n, c] == pytest.approx(want, rel=1e-13)
+
+
+def test_vjp_error_scales_from_the_other_oracle_functions():
+    """Each VJP scale is a contraction of scales that the separately written
+    (and separately pinned) oracle functions return: dq = sum_c |g_c| times
+    the q-gradient scale of channel c, dk = sum_c |v_c| times the q-gradient
+    scale with queries and keys exchanged and weights g_c, dv = the forward
+    denominator sum_m Phi |g_mc| with queries and keys exchanged."""
+    from oracle import oracle_vjp
+    rng = np.random.default_rng(26)
+    M, N, D, C, tau = 7, 6, 4, 3, 0.45
+    q = rng.standard_normal((M, D)) * 0.8 + 0.3
+    k = rng.standard_normal((N, D)) * 1.2
+    v = rng.standard_normal((N, C))
+    g = rng.standard_normal((M, C)) * 2.0
+    r = oracle_vjp(q, k, v, g, tau)
+    dq = np.zeros((M, D))
+    dk = np.zeros((N, D))
+    for c in range(C):
+        _, _, den_q, _ = oracle_grad_q(q, k, v[:, c], tau)
+        dq += np.abs(g[:, c:c + 1]) * den_q
+        _, _, den_k, _ = oracle_grad_q(k, q, g[:, c], tau)
+        dk += np.abs(v[:, c:c + 1]) * den_k
+    _, dv = oracle_sum(k, q, g, tau)
+    np.testing.assert_allclose(r["dq"], dq, rtol=1e-12)
+    np.testing.assert_allclose(r["dk"], dk, rtol=1e-12)
+    np.testing.assert_allclose(r["dv"], dv, rtol=1e-12)
