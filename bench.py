@@ -3,11 +3,13 @@
 
 A step is one full pass of the path -- centring mean, centre/cast/norm
 prep, value prep, fused tcgen05 kernel, finalise -- over one batch of the
-MMD-style workload: M = N = 65536 points in D = 64 (fp16, q = k), C = 1,
-v = +-1/N, tau = 1/64, i.e. 4.29e9 pair interactions per step.  The metric
-is pair interactions per second; the roofline of the fused kernel is the
-slower of dense fp16 tensor work 2 M N (D + C) and M N exponentials on the
-MUFU unit.
+MMD-style workload: M = N = 65536 points in D = 64 (fp16; q and k drawn
+independently from N(0, 1)), C = 1, v = +-1/N, tau = 1/64, i.e. 4.29e9 pair
+interactions per step.  The metric is pair interactions per second; the
+roofline of the fused kernel is the slower of dense fp16 tensor work
+2 M N (D + C) and M N exponentials on the MUFU unit.  The same run also
+times the other configurations (fewer steps) and reports them under
+"other_workloads".
 
 Usage:
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl own|reference]
@@ -52,6 +54,9 @@ def parse_args(argv=None):
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-clocks", action="store_true")
+    ap.add_argument("--no-other-workloads", action="store_true",
+                    help="skip timing the other four configurations")
+    ap.add_argument("--no-peak-probe", action="store_true")
     return ap.parse_args(argv)
 
 
@@ -150,6 +155,7 @@ def run_reference(args):
         "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
         "config": workload_config(w),
         "cpu_baseline": {"value": value, "unit": UNIT, "cores": threads, "kind": "oracle",
+                         "cpu_model": cpu_model(),
                          "sample": f"{rows} seeded query rows x all {w.N} keys per step"},
         "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
         "note": "float64 CPU oracle (plain double loop over Eq. 1) on the host cores; "
@@ -249,7 +255,7 @@ def profiled_traffic(w):
     """DRAM bytes per launch of the fused kernel from the committed ncu
     summary, if it was taken on the current library sources."""
     src = kernel_source_hash()
-    for path in glob.glob(os.path.join(ROOT, "profiles", f"{main_kernel_name(w)}_{w.name}*.md")):
+    for path in glob.glob(os.path.join(ROOT, "profiles", f"{main_kernel_name(w)}_{w.name}.md")):
         text = open(path).read()
         m_h = re.search(r"source_sha256_16:\s*([0-9a-f]+)", text)
         m_t = re.search(r"dram_bytes_per_launch:\s*([0-9.eE+]+)", text)
@@ -259,106 +265,184 @@ def profiled_traffic(w):
 
 
 # ---------------------------------------------------------------- own arm
-def run_own(args):
+def cpu_model():
+    """Host CPU model name (lscpu, else /proc/cpuinfo), or None."""
+    try:
+        out = subprocess.run(["lscpu"], capture_output=True, text=True, timeout=10).stdout
+        for line in out.splitlines():
+            if line.lower().startswith("model name"):
+                return line.split(":", 1)[1].strip()
+    except (OSError, subprocess.SubprocessError):
+        pass
+    try:
+        for line in open("/proc/cpuinfo"):
+            if line.lower().startswith("model name"):
+                return line.split(":", 1)[1].strip()
+    except OSError:
+        pass
+    return None
+
+
+def probe_fp16_tflops(dev):
+    """Dense fp16 matmul throughput (torch, 8192^3, best of 10): context for
+    the tensor peak, measured the way the bf16 peak in MEASURED_PEAKS.json
+    is.  Not a library kernel."""
     import torch
-    rank, world, local = dist_env()
-    torch.cuda.set_device(local)
-    dev = torch.device("cuda", local)
-    if world > 1:
-        import torch.distributed as dist
-        dist.init_process_group("nccl", device_id=dev)
+    n = 8192
+    a = torch.randn(n, n, device=dev, dtype=torch.float16)
+    b = torch.randn(n, n, device=dev, dtype=torch.float16)
+    for _ in range(3):
+        torch.matmul(a, b)
+    best = 0.0
+    for _ in range(10):
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        torch.matmul(a, b)
+        e1.record()
+        e1.synchronize()
+        best = max(best, 2.0 * n ** 3 / (e0.elapsed_time(e1) * 1e-3) / 1e12)
+    del a, b
+    torch.cuda.empty_cache()
+    return best
 
-    from paper_2609_04910_gb300.build import build_library
-    build_library()
-    import paper_2609_04910_gb300 as gs
-    from paper_2609_04910_gb300.workloads import WORKLOADS, device_inputs, generate
 
-    w = WORKLOADS[args.workload]
-    inp = generate(w, seed=0)
-    q, k, v = device_inputs(inp, dev)
+def roofline_of(w, main_ms, peaks, peak_src, sms, r_x, traffic=None, traffic_src=None):
+    """Roofline of the fused kernel (algorithmic work, unpadded D and C; the
+    gradient evaluates C' = D + 1 value channels): the slower of dense tensor
+    work 2 M N (D + C) at the measured bf16 peak (fp16 runs at the bf16
+    rate) and M N exponentials at the MUFU rate (32 ex2 per clock per SM at
+    the maximum SM clock)."""
     M, N, D, C = w.M, w.N, w.D, w.C
-    out = torch.empty((M, D if w.grad else C), dtype=torch.float32, device=dev)
-    s_out = torch.empty((M,), dtype=torch.float32, device=dev) if w.grad else None
-    flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=dev)
-    stream = torch.cuda.current_stream()
-
-    def step(main_events=None):
-        if w.grad:
-            gs.gauss_sum_grad_q(q, k, v, w.tau, grad=out, s_out=s_out, main_events=main_events)
-        else:
-            gs.gauss_sum(q, k, v, w.tau, out=out, main_events=main_events)
-
-    def barrier():
-        if world > 1:
-            import torch.distributed as dist
-            dist.barrier()
-
-    # Roofline denominators.
-    peaks, peak_src = measured_peaks()
-    r_x = gs.gauss_sum_probe_ex2_rate()
-    props = torch.cuda.get_device_properties(dev)
-    sms = props.multi_processor_count
+    Ceff = D + 1 if w.grad else C
+    flops = 2.0 * M * N * (D + Ceff)
+    exps = float(M) * N
+    r_t = float(peaks.get("bf16_tflops", FALLBACK_PEAKS["bf16_tflops"])) * 1e12
     sm_max_mhz = float(peaks.get("sm_max_mhz", 2070.0))
     r_x_nominal = 32.0 * sms * sm_max_mhz * 1e6
+    t_tensor = flops / r_t
+    t_sfu = exps / r_x_nominal
+    t_main = main_ms * 1e-3
+    if w.dtype == "fp32":
+        return None            # fp32_d16 runs on the SIMT kernel: launch and latency bound
+    if t_sfu >= t_tensor:
+        roof = {"bound": "alu", "achieved": exps / t_main / 1e12, "peak": r_x_nominal / 1e12,
+                "unit": "Texp/s", "frac": t_sfu / t_main}
+    else:
+        roof = {"bound": "tensor", "achieved": flops / t_main / 1e12, "peak": r_t / 1e12,
+                "unit": "TFLOP/s", "frac": t_tensor / t_main}
+    roof.update({
+        "traffic": traffic, "traffic_source": traffic_src,
+        "kernel": main_kernel_name(w), "kernel_ms": main_ms,
+        "t_roof_ms": max(t_tensor, t_sfu) * 1e3,
+        "peak_note": ("alu = MUFU ex2.approx: 32/clk/SM x "
+                      f"{sms} SMs x {sm_max_mhz:.0f} MHz = {r_x_nominal:.4g}/s "
+                      f"(the library's probe measured {r_x:.4g}/s live); tensor peak = "
+                      f"{peak_src} bf16 dense {r_t/1e12:.1f} TFLOP/s (fp16 at the bf16 rate, "
+                      "the nominal ratio 1)"),
+        "tensor": {"achieved": flops / t_main / 1e12, "peak": r_t / 1e12, "unit": "TFLOP/s",
+                   "frac": t_tensor / t_main},
+        "sfu": {"achieved": exps / t_main / 1e12, "peak": r_x_nominal / 1e12,
+                "unit": "Texp/s", "frac": t_sfu / t_main, "probe_ex2_per_s": r_x},
+    })
+    return roof
 
-    K, W = max(1, args.steps), max(3, args.warmup)
-    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
-          for _ in range(K)]
-    mev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
-           for _ in range(K)]
-    for a, b in ev + mev:  # create the CUDA events before handing them to the library
-        a.record(stream)
-        b.record(stream)
-    for _ in range(W):
-        flush.zero_()
-        step()
-    gs.gauss_sum_device_status()
-    torch.cuda.synchronize()
 
-    sampler = ClockSampler(local, enabled=not args.no_clocks)
-    time.sleep(0.3 if not args.no_clocks else 0.0)
-    barrier()
-    torch.cuda.synchronize()
-    wall0 = time.perf_counter()
-    launches0 = gs.gauss_sum_kernel_launches()
-    for i in range(K):
-        flush.zero_()
-        ev[i][0].record(stream)
-        step(main_events=mev[i])
-        ev[i][1].record(stream)
-    launches = gs.gauss_sum_kernel_launches() - launches0
-    torch.cuda.synchronize()
-    barrier()
-    wall = time.perf_counter() - wall0
-    gs.gauss_sum_device_status()
-    step_ms = [a.elapsed_time(b) for a, b in ev]
-    main_ms = [a.elapsed_time(b) for a, b in mev]
-    ms = statistics.mean(step_ms)
-    main_mean = statistics.mean(main_ms)
-    ms = reduce_max(ms, dev)
+class Runner:
+    """One workload's inputs on the device and its timed steps."""
 
-    # End to end through the public API with host buffers: H2D of the
-    # inputs, the call, D2H of the result, every step.
-    e2e = None
-    if not args.no_e2e:
+    def __init__(self, w, dev, flush):
+        import torch
+        from paper_2609_04910_gb300.workloads import device_inputs, generate
+        self.w = w
+        self.dev = dev
+        self.flush = flush
+        self.inp = generate(w, seed=0)
+        self.q, self.k, self.v = device_inputs(self.inp, dev)
+        M, D, C = w.M, w.D, w.C
+        self.out = torch.empty((M, D if w.grad else C), dtype=torch.float32, device=dev)
+        self.s_out = torch.empty((M,), dtype=torch.float32, device=dev) if w.grad else None
+
+    def step(self, main_events=None):
+        import paper_2609_04910_gb300 as gs
+        w = self.w
+        if w.grad:
+            gs.gauss_sum_grad_q(self.q, self.k, self.v, w.tau, grad=self.out, s_out=self.s_out,
+                                main_events=main_events)
+        else:
+            gs.gauss_sum(self.q, self.k, self.v, w.tau, out=self.out, main_events=main_events)
+
+    def timed(self, K, W, before=None, after=None):
+        """W warm-up steps, then K timed steps, each after an L2 flush, with
+        CUDA events around the step; then up to 50 more steps with events
+        that the library records around its main kernel (kept out of the
+        timed steps: an event between two kernels of a call makes the later
+        one launch without overlapping the earlier one's tail).  Returns
+        (step ms list, main-kernel ms list, launches in the timed steps)."""
+        import torch
+        import paper_2609_04910_gb300 as gs
+        stream = torch.cuda.current_stream()
+        Km = min(K, 50)
+        ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+              for _ in range(K)]
+        mev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+               for _ in range(Km)]
+        for a, b in ev + mev:  # create the CUDA events before handing them to the library
+            a.record(stream)
+            b.record(stream)
+        for _ in range(W):
+            self.flush.zero_()
+            self.step()
+        gs.gauss_sum_device_status()
+        torch.cuda.synchronize()
+        if before is not None:
+            before()
+        launches0 = gs.gauss_sum_kernel_launches()
+        for i in range(K):
+            self.flush.zero_()
+            ev[i][0].record(stream)
+            self.step()
+            ev[i][1].record(stream)
+        launches = gs.gauss_sum_kernel_launches() - launches0
+        torch.cuda.synchronize()
+        if after is not None:
+            after()
+        for i in range(Km):
+            self.flush.zero_()
+            self.step(main_events=mev[i])
+        torch.cuda.synchronize()
+        gs.gauss_sum_device_status()
+        return ([a.elapsed_time(b) for a, b in ev], [a.elapsed_time(b) for a, b in mev],
+                launches)
+
+    def e2e(self, K, W, world):
+        """The same step from pinned host buffers through the public API:
+        H2D of the step's inputs and D2H of its result inside the timed
+        region, every step."""
         import numpy as np
-        kh = torch.from_numpy(np.ascontiguousarray(inp["k"]).view(np.int16 if w.dtype == "bf16" else inp["k"].dtype)).pin_memory()
-        vh = torch.from_numpy(np.ascontiguousarray(inp["v"]).view(np.int16 if w.dtype == "bf16" else inp["v"].dtype)).pin_memory()
-        qh = kh if w.q_is_k else torch.from_numpy(
-            np.ascontiguousarray(inp["q"]).view(np.int16 if w.dtype == "bf16" else inp["q"].dtype)).pin_memory()
+        import torch
+        import paper_2609_04910_gb300 as gs
+        w, inp, dev = self.w, self.inp, self.dev
+        stream = torch.cuda.current_stream()
+
+        def host(a):
+            a = np.ascontiguousarray(a)
+            return torch.from_numpy(a.view(np.int16) if w.dtype == "bf16" else a).pin_memory()
+
+        kh, vh = host(inp["k"]), host(inp["v"])
+        qh = kh if w.q_is_k else host(inp["q"])
         kd = torch.empty_like(kh, device=dev)
         vd = torch.empty_like(vh, device=dev)
         qd = kd if w.q_is_k else torch.empty_like(qh, device=dev)
-        outh = torch.empty(tuple(out.shape), dtype=torch.float32).pin_memory()
-        sh = torch.empty((M,), dtype=torch.float32).pin_memory() if w.grad else None
+        outh = torch.empty(tuple(self.out.shape), dtype=torch.float32).pin_memory()
+        sh = torch.empty((w.M,), dtype=torch.float32).pin_memory() if w.grad else None
         conv = (lambda t: t.view(torch.bfloat16)) if w.dtype == "bf16" else (lambda t: t)
         e_ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
-                for _ in range(min(K, 200))]
+                for _ in range(K)]
         h2d = kh.numel() * kh.element_size() + vh.numel() * vh.element_size() + \
             (0 if w.q_is_k else qh.numel() * qh.element_size())
-        d2h = outh.numel() * 4 + (M * 4 if w.grad else 0)
-        for i in range(len(e_ev) + W):
-            flush.zero_()
+        d2h = outh.numel() * 4 + (w.M * 4 if w.grad else 0)
+        for i in range(K + W):
+            self.flush.zero_()
             if i >= W:
                 e_ev[i - W][0].record(stream)
             kd.copy_(kh, non_blocking=True)
@@ -377,55 +461,108 @@ def run_own(args):
         torch.cuda.synchronize()
         e_ms = statistics.mean(a.elapsed_time(b) for a, b in e_ev)
         e_ms = reduce_max(e_ms, dev)
-        e2e = {"value": replica_value(world, w.pairs, e_ms), "unit": UNIT, "ms_per_step": e_ms,
-               "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h),
-               "steps": len(e_ev)}
+        return {"value": replica_value(world, w.pairs, e_ms), "unit": UNIT, "ms_per_step": e_ms,
+                "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h),
+                "steps": K}
+
+
+OTHER_WORKLOADS = ("svgd_d32", "multi_c64", "offset_d256", "fp32_d16", "mmd_d64_qk")
+
+
+def run_own(args):
+    import torch
+    rank, world, local = dist_env()
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=dev)
+
+    from paper_2609_04910_gb300.build import build_library
+    build_library()
+    import paper_2609_04910_gb300 as gs
+    from paper_2609_04910_gb300.workloads import WORKLOADS
+
+    w = WORKLOADS[args.workload]
+    flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=dev)
+    run = Runner(w, dev, flush)
+
+    def barrier():
+        if world > 1:
+            import torch.distributed as dist
+            dist.barrier()
+
+    # Roofline denominators.
+    peaks, peak_src = measured_peaks()
+    r_x = gs.gauss_sum_probe_ex2_rate()
+    props = torch.cuda.get_device_properties(dev)
+    sms = props.multi_processor_count
+
+    K, W = max(1, args.steps), max(3, args.warmup)
+    sampler = ClockSampler(local, enabled=not args.no_clocks)
+
+    def start():
+        time.sleep(0.3 if not args.no_clocks else 0.0)
+        barrier()
+        torch.cuda.synchronize()
+
+    wall = {}
+
+    def t0():
+        start()
+        wall["t0"] = time.perf_counter()
+
+    def t1():
+        barrier()
+        wall["t"] = time.perf_counter() - wall["t0"]
+
+    step_ms, main_ms, launches = run.timed(K, W, before=t0, after=t1)
+    wall = wall["t"]
+    ms = reduce_max(statistics.mean(step_ms), dev)
+    main_mean = statistics.mean(main_ms)
+    e2e = None if args.no_e2e else run.e2e(min(K, 200), W, world)
     clocks = sampler.stop() if sampler is not None else None
 
-    # Roofline of the fused kernel (algorithmic work, unpadded D and C;
-    # the gradient evaluates C' = D + 1 value channels).
-    Ceff = D + 1 if w.grad else C
-    flops = 2.0 * M * N * (D + Ceff)
-    exps = float(M) * N
-    r_t = float(peaks.get("bf16_tflops", FALLBACK_PEAKS["bf16_tflops"])) * 1e12  # fp16 = bf16 rate
-    t_tensor = flops / r_t
-    t_sfu = exps / r_x
-    t_main = main_mean * 1e-3
     traffic, traffic_src = profiled_traffic(w)
-    if w.dtype == "fp32":
-        roof = None
-    elif t_sfu >= t_tensor:
-        # Bound by the MUFU exp2 issue rate: peak from unit count x SMs x
-        # maximum SM clock (32 ex2 per clock per SM, the rate the probe
-        # reaches at the maximum clock).
-        roof = {"bound": "alu", "achieved": exps / t_main / 1e12, "peak": r_x_nominal / 1e12,
-                "unit": "Texp/s", "frac": exps / r_x_nominal / t_main}
-    else:
-        roof = {"bound": "tensor", "achieved": flops / t_main / 1e12, "peak": r_t / 1e12,
-                "unit": "TFLOP/s", "frac": (t_tensor / t_main)}
-    if roof is not None:
-        roof.update({
-            "traffic": traffic, "traffic_source": traffic_src,
-            "kernel": main_kernel_name(w), "kernel_ms": main_mean,
-            "t_roof_ms": max(t_tensor, exps / r_x_nominal) * 1e3,
-            "peak_note": ("alu = MUFU ex2.approx: 32/clk/SM x "
-                          f"{sms} SMs x {sm_max_mhz:.0f} MHz = {r_x_nominal:.4g}/s "
-                          f"(the library's probe measured {r_x:.4g}/s live); tensor peak = "
-                          f"{peak_src} bf16 dense {r_t/1e12:.1f} TFLOP/s (fp16 runs at the bf16 "
-                          "rate)"),
-            "tensor": {"achieved": flops / t_main / 1e12, "peak": r_t / 1e12, "unit": "TFLOP/s",
-                       "frac": t_tensor / t_main},
-            "sfu": {"achieved": exps / t_main / 1e12, "peak": r_x_nominal / 1e12,
-                    "unit": "Texp/s", "frac": exps / r_x_nominal / t_main,
-                    "probe_ex2_per_s": r_x},
-        })
+    roof = roofline_of(w, main_mean, peaks, peak_src, sms, r_x, traffic, traffic_src)
+
+    # The other configurations, measured the same way (fewer steps) so that
+    # every configuration has a number from this run.
+    others = None
+    if rank == 0 and world == 1 and not args.no_other_workloads:
+        others = {}
+        del run
+        torch.cuda.empty_cache()
+        for name in OTHER_WORKLOADS:
+            wo = WORKLOADS[name]
+            try:
+                ro = Runner(wo, dev, flush)
+                s_ms, m_ms, n_l = ro.timed(min(K, 20), W)
+                tr, tr_src = profiled_traffic(wo)
+                rf = roofline_of(wo, statistics.mean(m_ms), peaks, peak_src, sms, r_x, tr,
+                                 tr_src)
+                others[name] = {
+                    "config": workload_config(wo), "steps": len(s_ms),
+                    "ms_per_step": statistics.mean(s_ms), "value": wo.pairs / (statistics.mean(s_ms) * 1e-3),
+                    "unit": UNIT, "main_kernel_ms": statistics.mean(m_ms),
+                    "main_kernel_ms_min": min(m_ms), "gpu_launches": n_l, "roofline": rf}
+                del ro
+                torch.cuda.empty_cache()
+            except Exception as exc:  # report, keep the headline line
+                others[name] = {"error": f"{type(exc).__name__}: {exc}"}
+
+    fp16_tf = None
+    if rank == 0 and not args.no_peak_probe:
+        fp16_tf = probe_fp16_tflops(dev)
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         from oracle import build_oracle
+        from paper_2609_04910_gb300.workloads import generate
         build_oracle()
-        rate, rows, el, threads = time_oracle(inp, args.cpu_seconds)
+        rate, rows, el, threads = time_oracle(generate(w, seed=0), args.cpu_seconds)
         cpu = {"value": rate, "unit": UNIT, "cores": threads, "kind": "oracle",
+               "cpu_model": cpu_model(),
                "sample": f"{rows} seeded query rows x all {w.N} keys ({el:.1f} s, float64, "
                          f"{threads} threads)"}
 
@@ -442,6 +579,8 @@ def run_own(args):
             "main_kernel_ms": main_mean,
             "main_kernel_ms_min": min(main_ms),
             "step_ms_min": min(step_ms),
+            "fp16_matmul_tflops_probe": fp16_tf,
+            "other_workloads": others,
         }
         print(json.dumps(line), flush=True)
     if world > 1:

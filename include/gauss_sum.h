@@ -90,6 +90,14 @@ typedef enum { GS_PATH_AUTO = 0, GS_PATH_TENSOR = 1, GS_PATH_SIMT = 2 } gs_path;
  *                  the launch of its main kernel (the fused tensor-core
  *                  kernel, or the fp32 SIMT kernel), so a caller can time
  *                  that kernel alone.  The caller owns the events.
+ *  exp2_fma        0 (default): every kernel value 2^x is computed by the
+ *                  MUFU ex2 unit.  1..4: a fixed share of them (1/32, 1/16,
+ *                  1/8, 1/4) is computed on the FMA pipe instead (Cody-Waite
+ *                  range reduction and a degree-4 minimax polynomial for
+ *                  2^f, relative error < 3e-6), the exponential-throughput
+ *                  variant for SFU-bound shapes.  Only forward fp16/bf16
+ *                  sums with C = 1 and D + 4 (fp16) or D + 6 (bf16) <= 128
+ *                  take it (GS_ERR_UNSUPPORTED otherwise).
  */
 typedef struct gs_options {
     int center;
@@ -98,9 +106,11 @@ typedef struct gs_options {
     size_t workspace_bytes;
     int path;
     void* main_events[2];
+    int exp2_fma;
 } gs_options;
 
-/* Fill *opt with the defaults (center = 1, split_n = 0, no workspace, auto path). */
+/* Fill *opt with the defaults (center = 1, split_n = 0, no workspace, auto
+ * path, no events, exp2_fma = 0). */
 void gauss_sum_default_options(gs_options* opt);
 
 /*
@@ -208,8 +218,8 @@ const char* gauss_sum_last_error(void);
 /* Static name of a status code. */
 const char* gauss_sum_status_string(gs_status status);
 
-/* Size of the static scratch array used by gauss_sum_noalloc: 16 MiB. */
-#define GS_NOALLOC_SCRATCH_BYTES (16u * 1024u * 1024u)
+/* Size of the static scratch array used by gauss_sum_noalloc: 32 MiB. */
+#define GS_NOALLOC_SCRATCH_BYTES (32u * 1024u * 1024u)
 
 /*
  * Eq. 1 like gauss_sum (default options), but without allocating device
@@ -222,15 +232,21 @@ const char* gauss_sum_status_string(gs_status status);
  *  - Arguments, layouts and ownership are those of gauss_sum.
  *  - Calls that need more scratch than the array holds return
  *    GS_ERR_UNSUPPORTED (see gauss_sum_last_error) without any GPU work;
- *    the M = N = 65536, D = 64, C = 1 fp16 MMD workload fits.
+ *    the M = N = 65536, D = 64, C = 1 fp16 MMD workload fits (it needs
+ *    21 MiB).
  *  - The first call on a device looks up the array's device address
- *    (cudaGetSymbolAddress with that device current); make that first call
- *    before any stream capture.
+ *    (cudaGetSymbolAddress with that device current) and keeps it for the
+ *    life of the process; make that first call before any stream capture.
+ *    The kept address assumes the device's primary context is never reset:
+ *    after cudaDeviceReset on that device the library's cached addresses
+ *    (this array and the device status word) are stale, and calls on that
+ *    device fail or misbehave.
  *  - All calls on a device share the array and leave their data in it:
  *    calls whose GPU work can overlap (unordered streams, several host
  *    threads) race and must be ordered by the caller.
  *  - No cudaMalloc, cudaMallocAsync, cudaFree or allocating library call is
- *    made.
+ *    made; each call clears the few scratch words it accumulates into
+ *    (cudaMemsetAsync) before using them.
  */
 gs_status gauss_sum_noalloc(const void* q, const void* k, const void* v, double tau, int64_t M,
                             int64_t N, int64_t D, int64_t C, gs_dtype dtype, float* out,

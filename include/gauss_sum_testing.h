@@ -1,0 +1,42 @@
+/*
+ * gauss_sum_testing.h -- test hooks of libgauss_sum.so.  Not part of the
+ * Gauss-sum computation (the paper has no counterpart); they exist so that
+ * the library's failure paths can be exercised without faulting a GPU or
+ * exhausting its memory.  Production code never needs them: with neither
+ * hook called, the library behaves as documented in gauss_sum.h.
+ */
+#ifndef GAUSS_SUM_TESTING_H
+#define GAUSS_SUM_TESTING_H
+
+#include "gauss_sum.h"
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/*
+ * on != 0: every workspace allocation the library would make from now on
+ * (cudaMallocAsync of gauss_sum_ex and friends, and of gauss_sum_mmd2)
+ * fails with GS_ERR_OUT_OF_MEMORY before any GPU work; on = 0 restores
+ * normal behaviour.  Process-wide.  Calls that allocate nothing (a caller
+ * workspace, gauss_sum_noalloc) are unaffected.
+ */
+void gauss_sum_testing_fail_allocations(int on);
+
+/*
+ * Makes one bounded device-side wait of every launch of the fused FMA
+ * kernel (C <= 4 forward) on the current device run out until the request
+ * is cleared: control warp 0 of block 0 waits on a barrier that nothing
+ * arrives on, gives up after the kernel's 2 s limit, raises the block's
+ * abort flag and records GS_ERR_DEVICE_TIMEOUT, which
+ * gauss_sum_device_status then reports.  The request is written on
+ * `stream` (a cudaStream_t as void*; the call synchronises it) into the
+ * device status words and cleared with them by gauss_sum_device_status.
+ */
+gs_status gauss_sum_testing_request_stall(void* stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* GAUSS_SUM_TESTING_H */

@@ -28,10 +28,12 @@ EXPORTS = (
     "gauss_sum_noalloc", "gauss_sum_kernel_launches", "gauss_sum_batched", "gauss_sum_mmd2",
     "gauss_sum_vjp",
 )
+# Test hooks declared in include/gauss_sum_testing.h.
+TESTING_EXPORTS = ("gauss_sum_testing_fail_allocations", "gauss_sum_testing_request_stall")
 
 # Bytes of the static scratch array behind gauss_sum_noalloc
 # (GS_NOALLOC_SCRATCH_BYTES in include/gauss_sum.h).
-NOALLOC_SCRATCH_BYTES = 16 * 1024 * 1024
+NOALLOC_SCRATCH_BYTES = 32 * 1024 * 1024
 
 
 class GaussSumError(RuntimeError):
@@ -44,7 +46,8 @@ class GaussSumError(RuntimeError):
 class GsOptions(ctypes.Structure):
     _fields_ = [("center", ctypes.c_int), ("split_n", ctypes.c_int),
                 ("workspace", ctypes.c_void_p), ("workspace_bytes", ctypes.c_size_t),
-                ("path", ctypes.c_int), ("main_events", ctypes.c_void_p * 2)]
+                ("path", ctypes.c_int), ("main_events", ctypes.c_void_p * 2),
+                ("exp2_fma", ctypes.c_int)]
 
 
 _lock = threading.Lock()
@@ -108,6 +111,10 @@ def _declare(lib):
     lib.gauss_sum_mmd2.restype = f
     lib.gauss_sum_vjp.argtypes = [vp, vp, vp, vp, d, i64, i64, i64, i64, f, vp, vp, vp, vp]
     lib.gauss_sum_vjp.restype = f
+    lib.gauss_sum_testing_fail_allocations.argtypes = [f]
+    lib.gauss_sum_testing_fail_allocations.restype = None
+    lib.gauss_sum_testing_request_stall.argtypes = [vp]
+    lib.gauss_sum_testing_request_stall.restype = f
 
 
 def _check(lib, status: int):
@@ -116,7 +123,7 @@ def _check(lib, status: int):
 
 
 def options(center=True, split_n=0, workspace=None, workspace_bytes=0, path=GS_PATH_AUTO,
-            main_events=None):
+            main_events=None, exp2_fma=0):
     """gs_options; ``main_events`` is an optional pair of torch.cuda.Event
     (already recorded once, so that their CUDA events exist) that the call
     records around its main kernel."""
@@ -127,6 +134,7 @@ def options(center=True, split_n=0, workspace=None, workspace_bytes=0, path=GS_P
     o.workspace = workspace
     o.workspace_bytes = int(workspace_bytes)
     o.path = int(path)
+    o.exp2_fma = int(exp2_fma)
     if main_events is not None:
         o.main_events[0] = main_events[0].cuda_event
         o.main_events[1] = main_events[1].cuda_event
@@ -163,11 +171,13 @@ def _check_tensor(t, name):
 
 
 def gauss_sum(q, k, v, tau, out=None, stream=None, center=True, split_n=0, workspace=None,
-              main_events=None, path=GS_PATH_AUTO):
+              main_events=None, path=GS_PATH_AUTO, exp2_fma=0):
     """Eq. 1: s[m] = sum_n exp(-tau/2 ||q_m - k_n||^2) v[n] as an (M, C) fp32 tensor.
 
     q: (M, D), k: (N, D), v: (N, C) or (N,) CUDA tensors of one dtype
     (fp32, fp16 or bf16).  ``q`` may be the same tensor as ``k``.
+    ``exp2_fma`` (0..4) moves a share of the exponentials to the FMA pipe
+    (gs_options.exp2_fma).
     """
     import torch
     lib = load_library()
@@ -181,7 +191,7 @@ def gauss_sum(q, k, v, tau, out=None, stream=None, center=True, split_n=0, works
     opt = options(center=center, split_n=split_n,
                   workspace=None if workspace is None else workspace.data_ptr(),
                   workspace_bytes=0 if workspace is None else workspace.numel() * workspace.element_size(),
-                  main_events=main_events, path=path)
+                  main_events=main_events, path=path, exp2_fma=exp2_fma)
     st = lib.gauss_sum_ex(_ptr(q), _ptr(k), _ptr(v), float(tau), M, N, D, C, _dtype_code(q),
                           _ptr(out), _stream_ptr(stream), ctypes.byref(opt))
     _check(lib, st)
@@ -259,7 +269,7 @@ def gauss_sum_vjp(q, k, v, g, tau, want=("q", "k", "v"), grad_q=None, grad_k=Non
 
 def gauss_sum_noalloc(q, k, v, tau, out=None, stream=None):
     """Eq. 1 like ``gauss_sum`` but without any device allocation by the
-    library: its scratch lives in a static 16 MiB device array (see
+    library: its scratch lives in a static 32 MiB device array (see
     ``gauss_sum_noalloc`` in include/gauss_sum.h for the rules of use).
     ``out`` should be passed by callers that must not allocate at all."""
     import torch
@@ -326,3 +336,14 @@ def gauss_sum_probe_ex2_rate(stream=None) -> float:
 def gauss_sum_kernel_launches() -> int:
     """Kernels the library has launched in this process (all devices)."""
     return int(load_library().gauss_sum_kernel_launches())
+
+
+def testing_fail_allocations(on: bool) -> None:
+    """Test hook: make the library's workspace allocations fail (or not)."""
+    load_library().gauss_sum_testing_fail_allocations(1 if on else 0)
+
+
+def testing_request_stall(stream=None) -> None:
+    """Test hook: the next FMA-kernel launch gives up one bounded wait."""
+    lib = load_library()
+    _check(lib, lib.gauss_sum_testing_request_stall(_stream_ptr(stream)))

@@ -11,6 +11,7 @@
 #include <mutex>
 
 #include "gauss_sum.h"
+#include "gauss_sum_testing.h"
 #include "internal.h"
 #include "ptx.cuh"
 
@@ -119,6 +120,8 @@ gs_status validate(const Call& c) {
     if (c.opt.split_n < 0) return fail(GS_ERR_INVALID_ARGUMENT, "split_n must be >= 0");
     if (c.opt.workspace && (reinterpret_cast<uintptr_t>(c.opt.workspace) & 255u))
         return fail(GS_ERR_INVALID_ARGUMENT, "caller workspace must be 256-byte aligned");
+    if (c.opt.exp2_fma < 0 || c.opt.exp2_fma > 4)
+        return fail(GS_ERR_INVALID_ARGUMENT, "exp2_fma must be 0..4");
     return GS_OK;
 }
 
@@ -162,8 +165,15 @@ gs_status plan(const Call& c, int sms, bool* tensor, gs::TcPlan* tp, gs::SimtPla
         if (!gs::plan_tensor(in_type(c.dtype), c.M, c.N, c.D, width, c.grad, c.opt.center != 0,
                              alias, c.opt.split_n, sms, tp, &why, c.B, c.tri && !c.grad))
             return fail(GS_ERR_UNSUPPORTED, "%s", why);
+        tp->exp2_fma = c.opt.exp2_fma;
+        if (tp->exp2_fma > 0 && !(tp->fma && tp->aug && !tp->tri && tp->Cv == 1))
+            return fail(GS_ERR_UNSUPPORTED,
+                        "exp2_fma needs a forward fp16/bf16 sum with C = 1 on augmented operands");
         *bytes = tp->total;
     } else {
+        if (c.opt.exp2_fma > 0)
+            return fail(GS_ERR_UNSUPPORTED,
+                        "exp2_fma needs a forward fp16/bf16 sum with C = 1 on augmented operands");
         if (!gs::plan_simt(c.M, c.N, c.D, c.C, c.grad, c.opt.split_n, sms, sp, &why))
             return fail(GS_ERR_UNSUPPORTED, "%s", why);
         *bytes = sp->total;
@@ -171,28 +181,23 @@ gs_status plan(const Call& c, int sms, bool* tensor, gs::TcPlan* tp, gs::SimtPla
     return GS_OK;
 }
 
+// Records a measurement event; the next kernel then launches without the
+// programmatic-serialization attribute (it follows an event, not a kernel).
 cudaError_t record_event(void* ev, cudaStream_t s) {
-    return ev ? cudaEventRecord(static_cast<cudaEvent_t>(ev), s) : cudaSuccess;
+    if (!ev) return cudaSuccess;
+    gs::pdl_reset();
+    return cudaEventRecord(static_cast<cudaEvent_t>(ev), s);
 }
 
-// Test hook: GS_TEST_FAIL_ALLOC=1 makes the workspace allocation fail.
-bool forced_alloc_failure() {
-    const char* s = std::getenv("GS_TEST_FAIL_ALLOC");
-    return s && s[0] == '1';
-}
+// Test hook (gauss_sum_testing_fail_allocations): workspace allocations
+// fail.  A relaxed atomic load per allocating call; nothing else reads it.
+std::atomic<int> g_fail_allocations{0};
 
-// Test hook: GS_TEST_STALL=1 makes one bounded wait of the next FMA-kernel
-// launch run out (2 s), so that the timeout path and its report through
-// gauss_sum_device_status can be tested without faulting the GPU.  The
-// request lives in the device status words and is cleared with them.
-cudaError_t request_stall_if_asked(unsigned* status, cudaStream_t s) {
-    const char* v = std::getenv("GS_TEST_STALL");
-    if (!(v && v[0] == '1')) return cudaSuccess;
-    static const unsigned one = 1u;
-    return cudaMemcpyAsync(status + gs::kDevStallRequest, &one, sizeof(one), cudaMemcpyHostToDevice, s);
-}
+bool forced_alloc_failure() { return g_fail_allocations.load(std::memory_order_relaxed) != 0; }
 
 gs_status run(Call c) {
+    // The first kernel of a call follows whatever the caller queued before.
+    gs::pdl_reset();
     gs_status st = validate(c);
     if (st != GS_OK) return st;
     if (c.M == 0 || c.B == 0) return GS_OK;
@@ -263,16 +268,30 @@ gs_status run(Call c) {
     const char* where = "kernel launch";
     if (tensor) {
         const gs::InType t = in_type(c.dtype);
-        float* mu = nullptr;
-        if (tp.center && c.D > 0) {
-            mu = reinterpret_cast<float*>(ws + tp.off_mu);
+        float* mu = (tp.center && c.D > 0) ? reinterpret_cast<float*>(ws + tp.off_mu) : nullptr;
+        // 16-bit inputs with D a multiple of 8: mean, operands and (FMA
+        // kernel) key records in one cooperative launch.
+        const bool fused = !tp.tf && gs::fused_prep_supported(t, c.D);
+        if (fused) {
+            e = gs::launch_fused_prep(
+                t, tp.aug, c.q, c.k, tp.fma ? c.v : nullptr, c.M, c.N, tp.Mpad, tp.Npad,
+                static_cast<int>(c.D), tp.Dp, static_cast<int>(tp.Cv), tp.alias, half_c,
+                tp.mean_blocks, reinterpret_cast<float*>(ws + tp.off_mean_part), mu,
+                ws + tp.off_qh, ws + tp.off_kh,
+                tp.aug ? nullptr : reinterpret_cast<float*>(ws + tp.off_A),
+                tp.aug ? nullptr : reinterpret_cast<float*>(ws + tp.off_B),
+                tp.fma ? reinterpret_cast<float*>(ws + tp.off_rec) : nullptr, c.stream, batch);
+            where = "fused preparation kernel";
+        } else if (mu) {
             e = gs::launch_mean(t, c.q, c.k, c.M, c.N, static_cast<int>(c.D), tp.mean_blocks,
                                 reinterpret_cast<float*>(ws + tp.off_mean_part), mu, c.stream,
                                 batch);
             where = "mean kernel";
         }
         const float ninf = -INFINITY;
-        if (e == cudaSuccess && tp.tf) {
+        if (fused || e != cudaSuccess) {
+            // Operands (and key records) written by the fused kernel, or an error.
+        } else if (tp.tf) {
             // 3xTF32 operands: hi / lo tf32 halves and the norm terms.
             e = gs::launch_tf32_split(static_cast<const float*>(c.q), c.M, tp.Mpad,
                                       static_cast<int>(c.D), tp.Dp, mu, half_c,
@@ -288,7 +307,7 @@ gs_status run(Call c) {
                                           c.stream, batch);
                 where = "tf32 split kernel (k)";
             }
-        } else if (e == cudaSuccess && tp.aug) {
+        } else if (tp.aug) {
             // Augmented operands: centred points with the norms folded in.
             e = gs::launch_aug_prep(t, c.q, c.M, tp.Mpad, static_cast<int>(c.D), tp.Dp, mu,
                                     ws + tp.off_qh, tp.alias ? ws + tp.off_kh : nullptr, c.stream,
@@ -300,7 +319,7 @@ gs_status run(Call c) {
                 where = "augmented-operand kernel (k)";
             }
         } else {
-            if (e == cudaSuccess) {
+            {
                 e = gs::launch_center_cast_norm(t, c.q, c.M, tp.Mpad, static_cast<int>(c.D), tp.Dp,
                                                 mu, half_c, ws + tp.off_qh,
                                                 reinterpret_cast<float*>(ws + tp.off_A), ninf,
@@ -316,13 +335,14 @@ gs_status run(Call c) {
             }
         }
         if (e == cudaSuccess && tp.fma) {
-            e = gs::launch_key_records(
-                t, c.v, tp.aug ? nullptr : reinterpret_cast<const float*>(ws + tp.off_B), c.N,
-                tp.Npad, static_cast<int>(tp.Cv), reinterpret_cast<float*>(ws + tp.off_rec),
-                c.stream, batch);
-            where = "key-record kernel";
+            if (!fused) {
+                e = gs::launch_key_records(
+                    t, c.v, tp.aug ? nullptr : reinterpret_cast<const float*>(ws + tp.off_B), c.N,
+                    tp.Npad, static_cast<int>(tp.Cv), reinterpret_cast<float*>(ws + tp.off_rec),
+                    c.stream, batch);
+                where = "key-record kernel";
+            }
             if (e == cudaSuccess) e = record_event(c.opt.main_events[0], c.stream);
-            if (e == cudaSuccess) e = request_stall_if_asked(status, c.stream);
             if (e == cudaSuccess) {
                 e = gs::launch_tc_fma(tp, t, cexp, ws, status, c.stream, &why);
                 where = "fused tensor-core kernel";
@@ -422,6 +442,7 @@ gs_options defaults() {
     o.path = GS_PATH_AUTO;
     o.main_events[0] = nullptr;
     o.main_events[1] = nullptr;
+    o.exp2_fma = 0;
     return o;
 }
 
@@ -674,6 +695,23 @@ const char* gauss_sum_status_string(gs_status s) {
 }
 
 uint64_t gauss_sum_kernel_launches(void) { return g_launches.load(std::memory_order_relaxed); }
+
+void gauss_sum_testing_fail_allocations(int on) {
+    g_fail_allocations.store(on ? 1 : 0, std::memory_order_relaxed);
+}
+
+gs_status gauss_sum_testing_request_stall(void* stream) {
+    int dev = 0;
+    unsigned* status = nullptr;
+    cudaError_t e = device_info(&dev, &status);
+    if (e != cudaSuccess) return cuda_fail(e, "device query");
+    static const unsigned one = 1u;
+    e = cudaMemcpyAsync(status + gs::kDevStallRequest, &one, sizeof(one), cudaMemcpyHostToDevice,
+                        static_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_fail(e, "stall request");
+    e = cudaStreamSynchronize(static_cast<cudaStream_t>(stream));
+    return e == cudaSuccess ? GS_OK : cuda_fail(e, "stall request");
+}
 
 gs_status gauss_sum_probe_ex2_rate(void* stream, double* exp2_per_second) {
     if (!exp2_per_second) return fail(GS_ERR_INVALID_ARGUMENT, "null output pointer");

@@ -11,6 +11,35 @@ namespace gs {
 
 enum class InType { F32 = 0, F16 = 1, BF16 = 2 };
 
+// Kernel launches of one library call, back to back on the caller's stream.
+// A kernel launched right after another kernel of the same call carries the
+// programmatic-stream-serialization attribute: it may be scheduled while its
+// predecessor drains, and every library kernel waits (pdl_wait, ptx.cuh)
+// for the previous kernel's completion before it reads that kernel's
+// outputs.  The first kernel of a call, and a kernel after any other stream
+// operation (memset, event record), is launched without it: t_pdl_next is
+// cleared by pdl_reset() at those points and set by every kernel launch.
+inline thread_local bool t_pdl_next = false;
+inline void pdl_reset() { t_pdl_next = false; }
+
+template <typename... K, typename... A>
+cudaError_t launch_kernel(void (*kern)(K...), dim3 grid, dim3 block, size_t smem, cudaStream_t s,
+                          A... args) {
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = s;
+    cfg.attrs = attr;
+    cfg.numAttrs = t_pdl_next ? 1u : 0u;
+    const cudaError_t e = cudaLaunchKernelEx(&cfg, kern, static_cast<K>(args)...);
+    t_pdl_next = e == cudaSuccess;
+    return e;
+}
+
 // Largest value-channel count evaluated on the FMA pipe (the P.v product of
 // tc_gauss_fma.cu); more channels use the two-MMA kernel of tc_gauss.cu.
 constexpr int kFmaMaxChannels = 4;
@@ -62,6 +91,9 @@ struct TcPlan {
     // Problems of a batch handled by one launch (the FMA kernel stacks them:
     // q^ batch x Mpad rows, k^ batch x Npad rows); 1 for the other paths.
     int64_t batch;
+    // FMA kernel: share of the exponentials computed on the FMA pipe
+    // (gs_options.exp2_fma: 0 none, 1..4 = 1/32 .. 1/4).
+    int exp2_fma;
     size_t off_mean_part, off_mu, off_qh, off_kh, off_A, off_B, off_vt, off_vmax, off_inv,
         off_rec, off_part, total;
 };
@@ -90,6 +122,18 @@ cudaError_t launch_mean(InType t, const void* q, const void* k, int64_t M, int64
 cudaError_t launch_center_cast_norm(InType t, const void* x, int64_t rows, int64_t rows_pad,
                                     int D, int Dp, const float* mu, float half_c, void* xh,
                                     float* nrm, float pad_value, cudaStream_t s, int batch = 1);
+// All of the operand preparation in one cooperative launch (16-bit inputs,
+// D a multiple of 8, D <= 256): the common mean (when mu is given; partial
+// holds batch x mean_blocks x 2 D floats), q^ and k^ in the augmented (aug)
+// or plain layout (plain: norm terms into nrm_q / nrm_k, which alias when
+// q is k), and, when rec is given, the FMA kernel's key records of v
+// (N x C per problem).  kh == qh for the plain layout with alias.
+bool fused_prep_supported(InType t, int64_t D);
+cudaError_t launch_fused_prep(InType t, bool aug, const void* q, const void* k, const void* v,
+                              int64_t M, int64_t N, int64_t Mpad, int64_t Npad, int D, int Dp,
+                              int C, bool alias, float half_c, int mean_blocks, float* partial,
+                              float* mu, void* qh, void* kh, float* nrm_q, float* nrm_k,
+                              float* rec, cudaStream_t s, int batch = 1);
 // Transposed fp16 value operand of the two-MMA kernel for the channels
 // ch0 .. ch0 + Cc - 1 (Cp >= Cc rows of Npad keys), with per-channel
 // power-of-two scales.  Forward: channel ch of key n is w[n, ch] (w has the

@@ -16,8 +16,12 @@
 //  * Calls whose workspace would exceed the static array are rejected with
 //    GS_ERR_UNSUPPORTED before any GPU work is issued.
 //  * The first call on a device looks up the device address of the array
-//    (cudaGetSymbolAddress, with that device current); make that first call
-//    before any stream capture begins.
+//    (cudaGetSymbolAddress, with that device current) and keeps it for the
+//    life of the process; make that first call before any stream capture
+//    begins.  The kept address assumes the device's primary context is never
+//    reset: after cudaDeviceReset it is stale (as is the device status word's
+//    address that api.cu keeps), so a process that resets a device must not
+//    call the library on it again.
 //  * All calls on a device share the one array and leave their data in it.
 //    Calls whose GPU work overlaps (different streams without ordering, or
 //    several host threads) race on it and give wrong results; order them.

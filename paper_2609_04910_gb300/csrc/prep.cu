@@ -16,6 +16,7 @@
 //    the gradient tau (S[:D] - q_m S[D]) of Sec. 3.
 #include <algorithm>
 
+#include <cooperative_groups.h>
 #include <cuda_bf16.h>
 #include <cuda_fp16.h>
 #include <math_constants.h>
@@ -48,6 +49,8 @@ template <typename T>
 __global__ void mean_partial_kernel(const T* __restrict__ q, const T* __restrict__ k, int64_t M,
                                     int64_t N, int D, int64_t rows_per_block,
                                     float* __restrict__ partial) {
+    pdl_trigger();
+    pdl_wait();
     __shared__ float red[8][33];
     __shared__ float big[8][33];
     // Problem blockIdx.y of a batch: its own points and partial rows.
@@ -95,6 +98,8 @@ template <typename T>
 __global__ void __launch_bounds__(kMeanVecThreads)
 mean_partial_vec_kernel(const T* __restrict__ q, const T* __restrict__ k, int64_t M, int64_t N,
                         int D, int64_t rows_per_block, int Gq, float* __restrict__ partial) {
+    pdl_trigger();
+    pdl_wait();
     __shared__ float s_sum[kMeanVecThreads][9];
     __shared__ float s_max[kMeanVecThreads][9];
     const int t = threadIdx.x;
@@ -156,6 +161,8 @@ constexpr int kMeanFinalThreads = 256;
 __global__ void __launch_bounds__(kMeanFinalThreads)
 mean_final_kernel(const float* __restrict__ partial, int G, int D, double total, int mant_bits,
                   int min_exp, float* __restrict__ mu) {
+    pdl_trigger();
+    pdl_wait();
     // Block d: thread t folds partials t, t + 256, ... in order, then a
     // fixed tree combines the threads (deterministic).
     __shared__ double red_s[kMeanFinalThreads];
@@ -230,6 +237,8 @@ __global__ void __launch_bounds__(kOperandThreads)
 operand_kernel(const T* __restrict__ x, int64_t rows, int64_t rows_pad, int D, int Dp, int nt, float F,
                const float* __restrict__ mu, float half_c, float pad_value,
                T* __restrict__ out_q, T* __restrict__ out_k, float* __restrict__ nrm) {
+    pdl_trigger();
+    pdl_wait();
     constexpr int R = kRowsPerBlock;
     // Dynamic shared memory sized to this call: s_out holds R x Dp
     // elements per written layout (AUG: q rows, then k rows), s_in the R x D
@@ -346,6 +355,8 @@ __global__ void tf32_split_kernel(const float* __restrict__ x, int64_t rows, int
                                   int64_t total_rows, int D, int Dp,
                                   const float* __restrict__ mu, float half_c, float pad_value,
                                   float* __restrict__ out, float* __restrict__ nrm) {
+    pdl_trigger();
+    pdl_wait();
     const int64_t w = (static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
     const int lane = threadIdx.x & 31;
     if (w >= total_rows) return;
@@ -372,6 +383,8 @@ __global__ void finalize_slots_kernel(const float* __restrict__ part, int64_t Mp
                                       int C, int rows_per_unit, int64_t key_tiles,
                                       int64_t unit_len, int64_t batch, int fixed_slots,
                                       int64_t tri_kt, float* __restrict__ out) {
+    pdl_trigger();
+    pdl_wait();
     // out: batch x M x C; partial rows are batch-stacked with Mpad rows per
     // problem and batch Mpad rows per slot.
     const int64_t idx = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
@@ -427,29 +440,25 @@ template <> __device__ __forceinline__ unsigned short to_bits<__nv_bfloat16>(__n
     return __bfloat16_as_ushort(h);
 }
 
+// One output row of the operand layouts, converted by the G lanes of a
+// row group (lane vi: coordinates 8 vi .. 8 vi + 7, one 16-byte vector).
+// in: lane vi's input vector of the row (used only when `valid` and
+// vi < D / 8); mu: the row problem's mean (or null); out_q / out_k: the row
+// in either layout (either
+// may be null; AUG only).  Every lane of the warp must call this together
+// (the squared norm is reduced with shuffles over the G lanes); rows outside
+// the output (in_pad false) write nothing.  Returns the norm term written
+// for the row (plain layout: -(c/2)||x^||^2, or pad_value) in every lane.
 template <typename T, bool AUG, int G>
-__global__ void __launch_bounds__(kOperandVecThreads)
-operand_vec_kernel(const T* __restrict__ x, int64_t rows, int64_t rows_pad, int64_t batch, int D,
-                   int Dp, int nt, float F, const float* __restrict__ mu, float half_c,
-                   float pad_value, T* __restrict__ out_q, T* __restrict__ out_k,
-                   float* __restrict__ nrm) {
-    const int vi = threadIdx.x % G;                              // vector within the row
-    // Output row of the batch-stacked operand (batch rows_pad rows per
-    // problem); problem b reads rows b rows .. of x and its own mean.
-    const int64_t row = (static_cast<int64_t>(blockIdx.x) * kOperandVecThreads + threadIdx.x) / G;
-    const int64_t b = row / rows_pad;
-    const int64_t i = row - b * rows_pad;
-    const bool in_pad = b < batch;
-    const bool valid = in_pad && i < rows;
-    if (mu && in_pad) mu += b * D;
+__device__ __forceinline__ float operand_row(const uint4 in, const float* __restrict__ mu, int vi,
+                                             bool in_pad, bool valid, int D, int Dp, int nt,
+                                             float F, float half_c, float pad_value,
+                                             T* __restrict__ out_q, T* __restrict__ out_k) {
     const int V = D / 8;
-    const bool wq = AUG ? out_q != nullptr : true;
-    const bool wk = AUG && out_k != nullptr;
     float acc = 0.f;
     if (in_pad && vi < V) {
         uint4 u = make_uint4(0u, 0u, 0u, 0u);
         if (valid) {
-            const uint4 in = *reinterpret_cast<const uint4*>(x + (b * rows + i) * D + 8 * vi);
             const unsigned short* hb = reinterpret_cast<const unsigned short*>(&in);
             float m[8];
             if (mu) {
@@ -471,17 +480,17 @@ operand_vec_kernel(const T* __restrict__ x, int64_t rows, int64_t rows_pad, int6
             }
             u = *reinterpret_cast<const uint4*>(ob);
         }
-        if (wq) *reinterpret_cast<uint4*>(out_q + row * Dp + 8 * vi) = u;
-        if (wk) *reinterpret_cast<uint4*>(out_k + row * Dp + 8 * vi) = u;
+        if (out_q) *reinterpret_cast<uint4*>(out_q + 8 * vi) = u;
+        if (out_k) *reinterpret_cast<uint4*>(out_k + 8 * vi) = u;
     }
 #pragma unroll
     for (int o = G / 2; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o, G);
-    if (!in_pad || vi != 0) return;
+    const float nrm = valid ? -half_c * acc : pad_value;
+    if (!in_pad || vi != 0) return nrm;
     if (!AUG) {
-        nrm[row] = valid ? -half_c * acc : pad_value;
         for (int c = D; c < Dp; c += 8)
-            *reinterpret_cast<uint4*>(out_q + row * Dp + c) = make_uint4(0u, 0u, 0u, 0u);
-        return;
+            *reinterpret_cast<uint4*>(out_q + c) = make_uint4(0u, 0u, 0u, 0u);
+        return nrm;
     }
     // Norm terms: a (or b) = -||x^||^2 / 2 = F t_0 + t_1 + ... (rounded
     // remainders), partners F, 1, 1 on the other side.
@@ -509,8 +518,234 @@ operand_vec_kernel(const T* __restrict__ x, int64_t rows, int64_t rows_pad, int6
             uq = *reinterpret_cast<const uint4*>(tq + e0);
             uk = *reinterpret_cast<const uint4*>(tk + e0);
         }
-        if (wq) *reinterpret_cast<uint4*>(out_q + row * Dp + c) = uq;
-        if (wk) *reinterpret_cast<uint4*>(out_k + row * Dp + c) = uk;
+        if (out_q) *reinterpret_cast<uint4*>(out_q + c) = uq;
+        if (out_k) *reinterpret_cast<uint4*>(out_k + c) = uk;
+    }
+    return nrm;
+}
+
+template <typename T, bool AUG, int G>
+__global__ void __launch_bounds__(kOperandVecThreads)
+operand_vec_kernel(const T* __restrict__ x, int64_t rows, int64_t rows_pad, int64_t batch, int D,
+                   int Dp, int nt, float F, const float* __restrict__ mu, float half_c,
+                   float pad_value, T* __restrict__ out_q, T* __restrict__ out_k,
+                   float* __restrict__ nrm) {
+    pdl_trigger();
+    pdl_wait();
+    const int vi = threadIdx.x % G;                              // vector within the row
+    // Output row of the batch-stacked operand (batch rows_pad rows per
+    // problem); problem b reads rows b rows .. of x and its own mean.
+    const int64_t row = (static_cast<int64_t>(blockIdx.x) * kOperandVecThreads + threadIdx.x) / G;
+    const int64_t b = row / rows_pad;
+    const int64_t i = row - b * rows_pad;
+    const bool in_pad = b < batch;
+    const bool valid = in_pad && i < rows;
+    const bool wq = AUG ? out_q != nullptr : true;
+    const bool wk = AUG && out_k != nullptr;
+    const uint4 in = (valid && vi < D / 8)
+                         ? *reinterpret_cast<const uint4*>(x + (b * rows + i) * D + 8 * vi)
+                         : make_uint4(0u, 0u, 0u, 0u);
+    const float n = operand_row<T, AUG, G>(in, (mu && in_pad) ? mu + b * D : nullptr, vi, in_pad,
+                                           valid, D, Dp, nt, F, half_c, pad_value,
+                                           wq ? out_q + row * Dp : nullptr,
+                                           wk ? out_k + row * Dp : nullptr);
+    if (!AUG && in_pad && vi == 0) nrm[row] = n;
+}
+
+// ---------------------------------------------------------------- fused prep
+// The whole preparation of the FMA kernel's operands in one cooperative
+// launch (16-bit inputs, D a multiple of 8), instead of the mean, mean-final,
+// operand (q, k) and key-record kernels:
+//   phase 1  per chunk of rows of one problem (q rows, then k rows unless
+//            q is k): coordinate sums and largest magnitudes (as
+//            mean_partial_kernel);            -- grid barrier --
+//   phase 2  per (problem, coordinate): the grid-rounded common mean from
+//            the chunk partials in chunk order (as mean_final_kernel);
+//                                             -- grid barrier --
+//   phase 3  every output row of q^ and k^ (operand_row) and, from the key
+//            rows, the key records [B_2t, B_2t+1,] v_2t[c], v_2t+1[c] ....
+// Without centring phases 1 and 2 and both barriers are skipped.  The
+// barriers are those of a cooperative launch (all blocks co-resident).
+constexpr int kRowsInFlight = 4;   // rows per thread with loads in flight (fused prep)
+
+struct FusedPrepArgs {
+    const void* q;
+    const void* k;
+    const void* v;          // N x C key values (records), batch-stacked
+    int64_t M, N, Mpad, Npad, batch;
+    int D, Dp, nt, C;
+    float F, half_c;
+    bool alias;             // q and k are the same points: rows written once to both layouts
+    int64_t rows_per_chunk;
+    int chunks_q, chunks_k; // chunks per problem (chunks_k = 0 when alias)
+    float* partial;         // chunks x 2 D (sums, then maxima); null: no centring
+    float* mu;              // batch x D
+    int mant_bits, min_exp;
+    void* qh;
+    void* kh;               // == qh for the plain layout with alias
+    float* nrm_q;           // plain layout: A (batch x Mpad)
+    float* nrm_k;           // plain layout: B (batch x Npad; == nrm_q with alias)
+    float* rec;             // key records (batch x Npad / 2 pairs)
+};
+
+template <typename T, bool AUG, int G>
+__global__ void __launch_bounds__(kOperandVecThreads)
+fused_prep_kernel(const FusedPrepArgs a) {
+    namespace cg = cooperative_groups;
+    pdl_trigger();
+    pdl_wait();
+    const int tid = threadIdx.x;
+    const int vi = tid % G;
+    constexpr int SLOTS = kOperandVecThreads / G;   // rows in flight per block
+    const int slot = tid / G;
+    const int D = a.D;
+    const T* q = static_cast<const T*>(a.q);
+    const T* k = static_cast<const T*>(a.k);
+    if (a.partial) {
+        __shared__ float s_sum[kOperandVecThreads][8];
+        __shared__ float s_max[kOperandVecThreads][8];
+        const int per_problem = a.chunks_q + a.chunks_k;
+        const int64_t chunks = a.batch * per_problem;
+        const int V = D / 8;
+        for (int64_t ch = blockIdx.x; ch < chunks; ch += gridDim.x) {
+            const int64_t b = ch / per_problem;
+            const int cb = static_cast<int>(ch - b * per_problem);
+            const bool on_q = cb < a.chunks_q;
+            const int64_t rows = on_q ? a.M : a.N;
+            const T* x = on_q ? q + b * a.M * D : k + b * a.N * D;
+            const int64_t r0 = static_cast<int64_t>(on_q ? cb : cb - a.chunks_q) * a.rows_per_chunk;
+            const int64_t r1 = min(rows, r0 + a.rows_per_chunk);
+            float sum[8], mx[8];
+#pragma unroll
+            for (int e = 0; e < 8; ++e) sum[e] = mx[e] = 0.f;
+            if (vi < V) {
+#pragma unroll 4
+                for (int64_t r = r0 + slot; r < r1; r += SLOTS) {
+                    const uint4 u = *reinterpret_cast<const uint4*>(x + r * D + 8 * vi);
+                    const T* h = reinterpret_cast<const T*>(&u);
+#pragma unroll
+                    for (int e = 0; e < 8; ++e) {
+                        const float f = to_f(h[e]);
+                        sum[e] += f;
+                        mx[e] = fmaxf(mx[e], fabsf(f));
+                    }
+                }
+            }
+#pragma unroll
+            for (int e = 0; e < 8; ++e) {
+                s_sum[tid][e] = sum[e];
+                s_max[tid][e] = mx[e];
+            }
+            __syncthreads();
+            // Coordinate d = 8 g + e: the slots' values of lane g, in slot order.
+            for (int d = tid; d < D; d += kOperandVecThreads) {
+                const int g = d >> 3, e = d & 7;
+                float s = 0.f, m = 0.f;
+                for (int sl = 0; sl < SLOTS; ++sl) {
+                    s += s_sum[sl * G + g][e];
+                    m = fmaxf(m, s_max[sl * G + g][e]);
+                }
+                a.partial[ch * 2 * D + d] = s;
+                a.partial[ch * 2 * D + D + d] = m;
+            }
+            __syncthreads();
+        }
+        cg::this_grid().sync();
+        // Phase 2: mean of coordinate d of problem b, rounded to the grid of
+        // the input format at the coordinate's largest magnitude; one warp
+        // per (problem, coordinate): lane l folds chunks l, l + 32, ... in
+        // order, then a fixed butterfly adds the lanes (deterministic).
+        const int64_t items = a.batch * D;
+        const int lane = tid & 31;
+        const int64_t warps = static_cast<int64_t>(gridDim.x) * (kOperandVecThreads / 32);
+        for (int64_t it = static_cast<int64_t>(blockIdx.x) * (kOperandVecThreads / 32) + (tid >> 5);
+             it < items; it += warps) {
+            const int64_t b = it / D;
+            const int d = static_cast<int>(it - b * D);
+            const float* pp = a.partial + b * per_problem * 2 * D;
+            double s = 0.0;
+            float m = 0.f;
+            for (int c = lane; c < per_problem; c += 32) {
+                s += static_cast<double>(pp[static_cast<int64_t>(c) * 2 * D + d]);
+                m = fmaxf(m, pp[static_cast<int64_t>(c) * 2 * D + D + d]);
+            }
+#pragma unroll
+            for (int o = 16; o > 0; o >>= 1) {
+                s += __shfl_xor_sync(0xffffffffu, s, o);
+                m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, o));
+            }
+            if (lane == 0) {
+                double mean = s / static_cast<double>(a.M + (a.alias ? 0 : a.N));
+                if (m > 0.f) {
+                    int e;
+                    frexp(static_cast<double>(m), &e);
+                    const double gstep = ldexp(1.0, max(e - 1 - a.mant_bits, a.min_exp));
+                    mean = rint(mean / gstep) * gstep;
+                }
+                a.mu[it] = static_cast<float>(mean);
+            }
+        }
+        cg::this_grid().sync();
+    }
+    // Phase 3: q rows (batch x Mpad), then k rows (batch x Npad) unless q is
+    // k.  A block takes SLOTS consecutive rows per slice; each thread handles
+    // kRowsInFlight slices one grid stride apart, with all their input
+    // vectors loaded before any is converted (several loads in flight per
+    // thread: the pass is bound by memory latency otherwise).
+    constexpr int U = kRowsInFlight;
+    const int64_t rows_q = a.batch * a.Mpad;
+    const int64_t rows_all = rows_q + (a.alias ? 0 : a.batch * a.Npad);
+    const int64_t step = static_cast<int64_t>(gridDim.x) * SLOTS;
+    const int head = AUG ? 0 : 2;
+    const int rec_pair = head + 2 * a.C;
+    const int V = D / 8;
+    for (int64_t base = static_cast<int64_t>(blockIdx.x) * SLOTS; base < rows_all; base += U * step) {
+        uint4 in[U];
+        int64_t rr[U], bb[U], ii[U];
+        bool onq[U], inr[U], val[U];
+#pragma unroll
+        for (int u = 0; u < U; ++u) {
+            const int64_t row = base + u * step + slot;
+            inr[u] = row < rows_all;
+            onq[u] = row < rows_q;
+            rr[u] = onq[u] ? row : row - rows_q;               // row of the stacked layout
+            const int64_t rpad = onq[u] ? a.Mpad : a.Npad;
+            bb[u] = rr[u] / rpad;
+            ii[u] = rr[u] - bb[u] * rpad;
+            val[u] = inr[u] && ii[u] < (onq[u] ? a.M : a.N);
+            const T* x = onq[u] ? q + (bb[u] * a.M + ii[u]) * D : k + (bb[u] * a.N + ii[u]) * D;
+            in[u] = (val[u] && vi < V) ? *reinterpret_cast<const uint4*>(x + 8 * vi)
+                                       : make_uint4(0u, 0u, 0u, 0u);
+        }
+#pragma unroll
+        for (int u = 0; u < U; ++u) {
+            const int64_t r = rr[u], b = bb[u], i = ii[u];
+            const bool on_q = onq[u], in_range = inr[u], valid = val[u];
+            const float* mu = (a.partial && in_range) ? a.mu + b * D : nullptr;
+            T* oq = nullptr;
+            T* ok = nullptr;
+            if (AUG) {
+                if (on_q) oq = static_cast<T*>(a.qh) + r * a.Dp;
+                if (!on_q || a.alias) ok = static_cast<T*>(a.kh) + r * a.Dp;
+            } else {
+                oq = static_cast<T*>(on_q ? a.qh : a.kh) + r * a.Dp;
+            }
+            // Plain layout: padded rows get the norm term -inf (kernel value 0).
+            const float nrm = operand_row<T, AUG, G>(in[u], mu, vi, in_range, valid, D, a.Dp, a.nt,
+                                                     a.F, a.half_c, -INFINITY,
+                                                     in_range ? oq : nullptr,
+                                                     in_range ? ok : nullptr);
+            if (!in_range) continue;
+            if (!AUG && vi == 0) (on_q ? a.nrm_q : a.nrm_k)[r] = nrm;
+            // Key records from the key rows (the q rows when q is k).
+            if (a.rec && (!on_q || a.alias)) {
+                float* rp = a.rec + (b * (a.Npad / 2) + (i >> 1)) * rec_pair;
+                const int par = static_cast<int>(i & 1);
+                if (!AUG && vi == 0) rp[par] = nrm;
+                const T* vb = static_cast<const T*>(a.v) + (b * a.N + i) * a.C;
+                for (int c = vi; c < a.C; c += G) rp[head + 2 * c + par] = valid ? to_f(vb[c]) : 0.f;
+            }
+        }
     }
 }
 
@@ -528,7 +763,7 @@ cudaError_t operand_typed(const void* x, int64_t rows, int64_t rows_pad, int D, 
         const int64_t threads = rows_pad * batch * G;
         const unsigned blocks = static_cast<unsigned>((threads + kOperandVecThreads - 1) / kOperandVecThreads);
         auto go = [&](auto kern) {
-            kern<<<blocks, kOperandVecThreads, 0, s>>>(static_cast<const T*>(x), rows, rows_pad,
+            launch_kernel(kern, blocks, kOperandVecThreads, 0, s, static_cast<const T*>(x), rows, rows_pad,
                                                      static_cast<int64_t>(batch), D,
                                                      Dp, nt, F, mu, half_c, pad_value,
                                                      static_cast<T*>(out_q), static_cast<T*>(out_k),
@@ -551,7 +786,7 @@ cudaError_t operand_typed(const void* x, int64_t rows, int64_t rows_pad, int D, 
     const size_t smem = static_cast<size_t>(nout) * kRowsPerBlock * Dp * sizeof(T) +
                         ((static_cast<size_t>(kRowsPerBlock) * D * sizeof(T) + 15) & ~size_t(15)) +
                         static_cast<size_t>(D) * sizeof(float);
-    operand_kernel<T, AUG><<<dim3(static_cast<unsigned>(blocks), batch), kOperandThreads, smem, s>>>(
+    launch_kernel(operand_kernel<T, AUG>, dim3(static_cast<unsigned>(blocks), batch), kOperandThreads, smem, s, 
         static_cast<const T*>(x), rows, rows_pad, D, Dp, nt, F, mu, half_c, pad_value,
         static_cast<T*>(out_q), static_cast<T*>(out_k), nrm);
     note_launches(1);
@@ -583,6 +818,8 @@ template <typename T, typename W, bool GRAD>
 __global__ void value_max_kernel(const W* __restrict__ w, const T* __restrict__ x,
                                  const float* __restrict__ mu, int64_t N, int D, int Cw, int ch0,
                                  int Cc, int64_t rows_per_block, unsigned* __restrict__ vmax_bits) {
+    pdl_trigger();
+    pdl_wait();
     __shared__ float red[8][33];
     const int64_t r0 = static_cast<int64_t>(blockIdx.x) * rows_per_block;
     const int64_t r1 = min(r0 + rows_per_block, N);
@@ -628,6 +865,8 @@ __global__ void value_prep_kernel(const W* __restrict__ w, const T* __restrict__
                                   int Cw, int ch0, int Cc, int Cp,
                                   const unsigned* __restrict__ vmax_bits, __half* __restrict__ vt,
                                   float* __restrict__ inv_scale) {
+    pdl_trigger();
+    pdl_wait();
     // A block transposes 64 keys x 32 channels; each thread stores two
     // adjacent keys of one channel as a half2 (Npad is a multiple of 128).
     __shared__ float tile[64][33];
@@ -665,6 +904,8 @@ __global__ void value_prep_kernel(const W* __restrict__ w, const T* __restrict__
 template <typename T>
 __global__ void key_record_kernel(const T* __restrict__ v, const float* __restrict__ B, int64_t N,
                                   int64_t pairs, int C, float* __restrict__ rec) {
+    pdl_trigger();
+    pdl_wait();
     const int64_t t = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
     if (t >= pairs) return;
     const int64_t n0 = 2 * t, n1 = 2 * t + 1;
@@ -690,6 +931,8 @@ __global__ void key_record_kernel(const T* __restrict__ v, const float* __restri
 __global__ void finalize_kernel(const float* __restrict__ part, int splits,
                                 int64_t split_stride_rows, int64_t M, int Cv, int part_ld,
                                 const float* __restrict__ inv_scale, float* __restrict__ out) {
+    pdl_trigger();
+    pdl_wait();
     const int64_t idx = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
     if (idx >= M * Cv) return;
     const int64_t m = idx / Cv;
@@ -719,6 +962,8 @@ __global__ void finalize_points_kernel(const float* __restrict__ part, int split
                                        float tau, int D, int Cw, int ch0, int Cc,
                                        const U* __restrict__ u, int accumulate,
                                        float* __restrict__ out, float* __restrict__ s_out) {
+    pdl_trigger();
+    pdl_wait();
     const int width = D > 0 ? D : 1;
     const int64_t idx = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
     if (idx >= M * width) return;
@@ -760,11 +1005,12 @@ cudaError_t value_prep_typed(const void* w, const void* x, const float* mu, int6
                              unsigned* vmax_bits, void* vt, float* inv_scale, cudaStream_t s) {
     cudaError_t e = cudaMemsetAsync(vmax_bits, 0, sizeof(unsigned) * Cp, s);
     if (e != cudaSuccess) return e;
+    pdl_reset();   // the next kernel follows a memset
     // 64 rows per block: several blocks per SM even for N of a few 10^4.
     const int64_t rows_per_block = 64;
     const int64_t blocks = N > 0 ? (N + rows_per_block - 1) / rows_per_block : 0;
     if (blocks > 0) {
-        value_max_kernel<T, W, GRAD><<<static_cast<unsigned>(blocks), dim3(32, 8), 0, s>>>(
+        launch_kernel(value_max_kernel<T, W, GRAD>, static_cast<unsigned>(blocks), dim3(32, 8), 0, s, 
             static_cast<const W*>(w), static_cast<const T*>(x), mu, N, D, Cw, ch0, Cc,
             rows_per_block, vmax_bits);
         note_launches(1);
@@ -772,7 +1018,7 @@ cudaError_t value_prep_typed(const void* w, const void* x, const float* mu, int6
         if (e != cudaSuccess) return e;
     }
     dim3 grid(static_cast<unsigned>((Npad + 63) / 64), static_cast<unsigned>((Cp + 31) / 32));
-    value_prep_kernel<T, W, GRAD><<<grid, dim3(32, 8), 0, s>>>(
+    launch_kernel(value_prep_kernel<T, W, GRAD>, grid, dim3(32, 8), 0, s, 
         static_cast<const W*>(w), static_cast<const T*>(x), mu, N, Npad, D, Cw, ch0, Cc, Cp,
         vmax_bits, static_cast<__half*>(vt), inv_scale);
     note_launches(1);
@@ -789,7 +1035,7 @@ cudaError_t finalize_points_typed(const float* part, int splits, int64_t stride_
     if (total == 0) return cudaSuccess;
     const int threads = 256;
     const int64_t blocks = (total + threads - 1) / threads;
-    finalize_points_kernel<DIRECT, T, U><<<static_cast<unsigned>(blocks), threads, 0, s>>>(
+    launch_kernel(finalize_points_kernel<DIRECT, T, U>, static_cast<unsigned>(blocks), threads, 0, s, 
         part, splits, stride_rows, M, part_ld, inv_scale, static_cast<const T*>(x), mu, tau, D,
         Cw, ch0, Cc, static_cast<const U*>(u), accumulate, out, s_out);
     note_launches(1);
@@ -814,11 +1060,11 @@ cudaError_t launch_mean(InType t, const void* q, const void* k, int64_t M, int64
         const int Gk = static_cast<int>((N + rpb - 1) / rpb);
         G = Gq + Gk;
         if (t == InType::F16)
-            mean_partial_vec_kernel<__half><<<dim3(G, batch), kMeanVecThreads, 0, s>>>(
+            launch_kernel(mean_partial_vec_kernel<__half>, dim3(G, batch), kMeanVecThreads, 0, s, 
                 static_cast<const __half*>(q), static_cast<const __half*>(k), M, N, D, rpb, Gq,
                 partial);
         else
-            mean_partial_vec_kernel<__nv_bfloat16><<<dim3(G, batch), kMeanVecThreads, 0, s>>>(
+            launch_kernel(mean_partial_vec_kernel<__nv_bfloat16>, dim3(G, batch), kMeanVecThreads, 0, s, 
                 static_cast<const __nv_bfloat16*>(q), static_cast<const __nv_bfloat16*>(k), M, N, D,
                 rpb, Gq, partial);
         note_launches(1);
@@ -827,17 +1073,17 @@ cudaError_t launch_mean(InType t, const void* q, const void* k, int64_t M, int64
         G = static_cast<int>((total + rpb - 1) / rpb);
         switch (t) {
             case InType::F16:
-                mean_partial_kernel<__half><<<dim3(G, batch), dim3(32, 8), 0, s>>>(
+                launch_kernel(mean_partial_kernel<__half>, dim3(G, batch), dim3(32, 8), 0, s, 
                     static_cast<const __half*>(q), static_cast<const __half*>(k), M, N, D, rpb,
                     partial);
                 break;
             case InType::BF16:
-                mean_partial_kernel<__nv_bfloat16><<<dim3(G, batch), dim3(32, 8), 0, s>>>(
+                launch_kernel(mean_partial_kernel<__nv_bfloat16>, dim3(G, batch), dim3(32, 8), 0, s, 
                     static_cast<const __nv_bfloat16*>(q), static_cast<const __nv_bfloat16*>(k), M, N,
                     D, rpb, partial);
                 break;
             default:
-                mean_partial_kernel<float><<<dim3(G, batch), dim3(32, 8), 0, s>>>(
+                launch_kernel(mean_partial_kernel<float>, dim3(G, batch), dim3(32, 8), 0, s, 
                     static_cast<const float*>(q), static_cast<const float*>(k), M, N, D, rpb,
                     partial);
         }
@@ -847,7 +1093,7 @@ cudaError_t launch_mean(InType t, const void* q, const void* k, int64_t M, int64
     if (e != cudaSuccess) return e;
     const int mant_bits = t == InType::F16 ? 10 : t == InType::BF16 ? 7 : 23;
     const int min_exp = t == InType::F16 ? -24 : t == InType::BF16 ? -133 : -149;
-    mean_final_kernel<<<dim3(D, batch), kMeanFinalThreads, 0, s>>>(partial, G, D, static_cast<double>(total),
+    launch_kernel(mean_final_kernel, dim3(D, batch), kMeanFinalThreads, 0, s, partial, G, D, static_cast<double>(total),
                                                      mant_bits, min_exp, mu);
     note_launches(1);
     return cudaGetLastError();
@@ -866,6 +1112,8 @@ template <typename T>
 __global__ void __launch_bounds__(256)
 mmd2_reduce_kernel(const float* __restrict__ s, const T* __restrict__ v, int64_t N,
                    double* __restrict__ partial) {
+    pdl_trigger();
+    pdl_wait();
     __shared__ double red[256];
     const int t = threadIdx.x;
     const int64_t b = blockIdx.y;
@@ -885,6 +1133,8 @@ mmd2_reduce_kernel(const float* __restrict__ s, const T* __restrict__ v, int64_t
 
 __global__ void mmd2_final_kernel(const double* __restrict__ partial, int chunks, int64_t B,
                                   float* __restrict__ out) {
+    pdl_trigger();
+    pdl_wait();
     const int64_t b = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
     if (b >= B) return;
     double acc = 0.0;
@@ -906,21 +1156,21 @@ cudaError_t launch_mmd2_reduce(InType t, const float* s, const void* v, int64_t 
     const dim3 grid(static_cast<unsigned>(chunks), static_cast<unsigned>(B));
     switch (t) {
         case InType::F16:
-            mmd2_reduce_kernel<__half><<<grid, 256, 0, st>>>(s, static_cast<const __half*>(v), N,
+            launch_kernel(mmd2_reduce_kernel<__half>, grid, 256, 0, st, s, static_cast<const __half*>(v), N,
                                                              partial);
             break;
         case InType::BF16:
-            mmd2_reduce_kernel<__nv_bfloat16><<<grid, 256, 0, st>>>(
+            launch_kernel(mmd2_reduce_kernel<__nv_bfloat16>, grid, 256, 0, st, 
                 s, static_cast<const __nv_bfloat16*>(v), N, partial);
             break;
         default:
-            mmd2_reduce_kernel<float><<<grid, 256, 0, st>>>(s, static_cast<const float*>(v), N,
+            launch_kernel(mmd2_reduce_kernel<float>, grid, 256, 0, st, s, static_cast<const float*>(v), N,
                                                             partial);
     }
     note_launches(1);
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
-    mmd2_final_kernel<<<static_cast<unsigned>((B + 127) / 128), 128, 0, st>>>(
+    launch_kernel(mmd2_final_kernel, static_cast<unsigned>((B + 127) / 128), 128, 0, st, 
         partial, static_cast<int>(chunks), B, out);
     note_launches(1);
     return cudaGetLastError();
@@ -933,11 +1183,109 @@ cudaError_t launch_finalize_slots(const float* part, int64_t Mpad, int64_t M, in
     const int64_t total = static_cast<int64_t>(batch) * M * C;
     if (total == 0) return cudaSuccess;
     const int threads = 256;
-    finalize_slots_kernel<<<static_cast<unsigned>((total + threads - 1) / threads), threads, 0, s>>>(
+    launch_kernel(finalize_slots_kernel, static_cast<unsigned>((total + threads - 1) / threads), threads, 0, s, 
         part, Mpad, M, C, rows_per_unit, key_tiles, unit_len, static_cast<int64_t>(batch),
         fixed_slots, tri_key_tiles, out);
     note_launches(1);
     return cudaGetLastError();
+}
+
+bool fused_prep_supported(InType t, int64_t D) {
+    return t != InType::F32 && D >= 8 && D % 8 == 0 && D <= kOperandMaxCols;
+}
+
+namespace {
+
+template <typename T, bool AUG, int G>
+cudaError_t fused_prep_go(FusedPrepArgs a, cudaStream_t s) {
+    auto kern = fused_prep_kernel<T, AUG, G>;
+    // Blocks that fit on the device at once (the grid barriers need all of
+    // them resident), per device.
+    static int per_sm[64] = {};
+    static int sms[64] = {};
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
+    if (per_sm[dev] == 0) {
+        int nb = 0, n = 0;
+        e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&nb, kern, kOperandVecThreads, 0);
+        if (e != cudaSuccess) return e;
+        e = cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
+        if (e != cudaSuccess) return e;
+        sms[dev] = n;
+        per_sm[dev] = nb > 0 ? nb : 1;
+    }
+    constexpr int SLOTS = kOperandVecThreads / G;
+    const int64_t rows = a.batch * (a.Mpad + (a.alias ? 0 : a.Npad));
+    const int64_t want = std::max<int64_t>((rows + SLOTS * kRowsInFlight - 1) / (SLOTS * kRowsInFlight),
+                                           a.partial ? a.batch * (a.chunks_q + a.chunks_k) : 1);
+    const int grid = static_cast<int>(std::max<int64_t>(
+        1, std::min<int64_t>(want, static_cast<int64_t>(per_sm[dev]) * sms[dev])));
+    void* args[] = {&a};
+    e = cudaLaunchCooperativeKernel(reinterpret_cast<const void*>(kern), dim3(grid),
+                                    dim3(kOperandVecThreads), args, 0, s);
+    t_pdl_next = e == cudaSuccess;
+    note_launches(1);
+    return e;
+}
+
+template <typename T, bool AUG>
+cudaError_t fused_prep_g(const FusedPrepArgs& a, cudaStream_t s) {
+    const int V = a.D / 8;
+    const int G = V <= 1 ? 1 : V <= 2 ? 2 : V <= 4 ? 4 : V <= 8 ? 8 : V <= 16 ? 16 : 32;
+    switch (G) {
+        case 1: return fused_prep_go<T, AUG, 1>(a, s);
+        case 2: return fused_prep_go<T, AUG, 2>(a, s);
+        case 4: return fused_prep_go<T, AUG, 4>(a, s);
+        case 8: return fused_prep_go<T, AUG, 8>(a, s);
+        case 16: return fused_prep_go<T, AUG, 16>(a, s);
+        default: return fused_prep_go<T, AUG, 32>(a, s);
+    }
+}
+
+}  // namespace
+
+cudaError_t launch_fused_prep(InType t, bool aug, const void* q, const void* k, const void* v,
+                              int64_t M, int64_t N, int64_t Mpad, int64_t Npad, int D, int Dp,
+                              int C, bool alias, float half_c, int mean_blocks, float* partial,
+                              float* mu, void* qh, void* kh, float* nrm_q, float* nrm_k,
+                              float* rec, cudaStream_t s, int batch) {
+    FusedPrepArgs a;
+    a.q = q;
+    a.k = k;
+    a.v = v;
+    a.M = M;
+    a.N = N;
+    a.Mpad = Mpad;
+    a.Npad = Npad;
+    a.batch = batch;
+    a.D = D;
+    a.Dp = Dp;
+    a.nt = aug ? aug_norm_terms(t) : 0;
+    a.C = C;
+    a.F = (aug && t == InType::F16) ? 1024.f : 1.f;
+    a.half_c = half_c;
+    a.alias = alias;
+    // Chunks of rows per problem for the mean partials: at most mean_blocks
+    // per problem (the partial buffer holds batch x mean_blocks x 2 D floats).
+    const int64_t rows = M + (alias ? 0 : N);
+    a.rows_per_chunk = std::max<int64_t>(1, (rows + std::max(1, mean_blocks - 2) - 1) /
+                                                std::max(1, mean_blocks - 2));
+    a.chunks_q = static_cast<int>((M + a.rows_per_chunk - 1) / a.rows_per_chunk);
+    a.chunks_k = alias ? 0 : static_cast<int>((N + a.rows_per_chunk - 1) / a.rows_per_chunk);
+    a.partial = mu ? partial : nullptr;
+    a.mu = mu;
+    a.mant_bits = t == InType::F16 ? 10 : 7;
+    a.min_exp = t == InType::F16 ? -24 : -133;
+    a.qh = qh;
+    a.kh = kh;
+    a.nrm_q = nrm_q;
+    a.nrm_k = nrm_k;
+    a.rec = rec;
+    if (t == InType::BF16)
+        return aug ? fused_prep_g<__nv_bfloat16, true>(a, s) : fused_prep_g<__nv_bfloat16, false>(a, s);
+    return aug ? fused_prep_g<__half, true>(a, s) : fused_prep_g<__half, false>(a, s);
 }
 
 cudaError_t launch_center_cast_norm(InType t, const void* x, int64_t rows, int64_t rows_pad,
@@ -957,7 +1305,7 @@ cudaError_t launch_tf32_split(const float* x, int64_t rows, int64_t rows_pad, in
     if (total == 0) return cudaSuccess;
     const int threads = 256;
     const int64_t blocks = (total * 32 + threads - 1) / threads;
-    tf32_split_kernel<<<static_cast<unsigned>(blocks), threads, 0, s>>>(
+    launch_kernel(tf32_split_kernel, static_cast<unsigned>(blocks), threads, 0, s, 
         x, rows, rows_pad, total, D, Dp, mu, half_c, pad_value, out, nrm);
     note_launches(1);
     return cudaGetLastError();
@@ -997,13 +1345,13 @@ cudaError_t launch_key_records(InType t, const void* v, const float* B, int64_t 
     const int threads = 256;
     const unsigned blocks = static_cast<unsigned>((pairs + threads - 1) / threads);
     if (t == InType::BF16)
-        key_record_kernel<__nv_bfloat16><<<dim3(blocks, batch), threads, 0, s>>>(
+        launch_kernel(key_record_kernel<__nv_bfloat16>, dim3(blocks, batch), threads, 0, s, 
             static_cast<const __nv_bfloat16*>(v), B, N, pairs, C, rec);
     else if (t == InType::F32)
-        key_record_kernel<float><<<dim3(blocks, batch), threads, 0, s>>>(
+        launch_kernel(key_record_kernel<float>, dim3(blocks, batch), threads, 0, s, 
             static_cast<const float*>(v), B, N, pairs, C, rec);
     else
-        key_record_kernel<__half><<<dim3(blocks, batch), threads, 0, s>>>(static_cast<const __half*>(v), B, N,
+        launch_kernel(key_record_kernel<__half>, dim3(blocks, batch), threads, 0, s, static_cast<const __half*>(v), B, N,
                                                              pairs, C, rec);
     note_launches(1);
     return cudaGetLastError();
@@ -1016,7 +1364,7 @@ cudaError_t launch_finalize(const float* part, int splits, int64_t split_stride_
     if (total == 0) return cudaSuccess;
     const int threads = 256;
     const int64_t blocks = (total + threads - 1) / threads;
-    finalize_kernel<<<static_cast<unsigned>(blocks), threads, 0, s>>>(
+    launch_kernel(finalize_kernel, static_cast<unsigned>(blocks), threads, 0, s, 
         part, splits, split_stride_rows, M, Cv, part_ld, inv_scale, out);
     note_launches(1);
     return cudaGetLastError();

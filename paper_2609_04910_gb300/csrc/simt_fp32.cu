@@ -32,6 +32,8 @@ __global__ void __launch_bounds__(THREADS)
 simt_gauss_kernel(const float* __restrict__ q, const float* __restrict__ k,
                   const float* __restrict__ v, int64_t M, int64_t N, int D, int Cv,
                   int wch, float half_c, int64_t keys_per_split, float* __restrict__ part) {
+    pdl_trigger();
+    pdl_wait();
     __shared__ __align__(16) float ks[KT][DMAX];
     __shared__ float vs[KT][GRAD ? 1 : CBLK];
 
@@ -125,7 +127,7 @@ cudaError_t launch_cblk(const SimtPlan& p, const float* q, const float* k, const
                         int Cw, int wch, float half_c, float* part, cudaStream_t s) {
     dim3 grid(static_cast<unsigned>((p.M + THREADS - 1) / THREADS), p.splits,
               GRAD ? 1u : static_cast<unsigned>((p.Cv + CBLK - 1) / CBLK));
-    simt_gauss_kernel<DMAX, CBLK, GRAD><<<grid, THREADS, 0, s>>>(
+    launch_kernel(simt_gauss_kernel<DMAX, CBLK, GRAD>, grid, THREADS, 0, s, 
         q, k, v, p.M, p.N, static_cast<int>(p.D), GRAD ? Cw : static_cast<int>(p.Cv), wch,
         half_c, p.keys_per_split, part);
     note_launches(1);

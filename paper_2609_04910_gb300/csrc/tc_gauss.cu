@@ -58,11 +58,22 @@ constexpr uint32_t TMEM_COLS = 512;
 // P is stored as fp16(2^(x + P_SHIFT)): since x <= 0 the stored value is at
 // most 2^15 < 65504, and kernel values down to 2^-29 stay normal fp16
 // numbers (instead of 2^-14).  The epilogue multiplies O by 2^-P_SHIFT.
-// x is not clamped: a rounding-positive exponent (x slightly above 0) is
-// kept as is, and the saturating fp16 conversion bounds P by 65504, i.e.
-// the kernel value by 65504 / 2^15 < 2, so that no inf can reach the MMA.
+// The exponent is <= 0 in exact arithmetic; a rounding-positive x is
+// clamped to 0 on the packed fp16 pair (P <= 2^15, i.e. Phi <= 1): one
+// min.f16x2 per pair (the shifted exponent x + 15 leaves no room for the
+// sign-free 2^-|x| form of ex2_nonpos).
 constexpr float P_SHIFT = 15.f;
 constexpr float P_UNSHIFT = 1.f / 32768.f;
+constexpr uint32_t kP2Max = 0x78007800u;   // fp16 pair (2^15, 2^15)
+
+// Element-wise minimum of two packed fp16 pairs.
+__device__ __forceinline__ uint32_t hmin2(uint32_t a, uint32_t b) {
+    uint32_t d;
+    asm("min.f16x2 %0, %1, %2;" : "=r"(d) : "r"(a), "r"(b));
+    return d;
+}
+
+__device__ __forceinline__ uint32_t bound_p2(uint32_t p2) { return hmin2(p2, kP2Max); }
 
 struct TcParams {
     const float* A;      // Mpad: -(c/2)||q^_m||^2
@@ -139,6 +150,7 @@ tc_gauss_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant_
     constexpr int NCH = COLS / 32;              // 32-column TMEM loads per warp and tile
     static_assert(GROUP_WARPS % 4 == 0, "each group covers the four TMEM lane quarters");
     static_assert(COLS % 32 == 0, "exponent warps load whole 32-column chunks");
+    static_assert(NCH == 2, "two 32-column TMEM loads per warp and tile");
 
     extern __shared__ uint8_t smem_raw[];
     // 1024-byte aligned base for the 128-byte swizzle atoms.
@@ -158,6 +170,7 @@ tc_gauss_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant_
     const int T = kt1 - kt0;
     volatile int* abort_flag = &bars->abort_flag;
 
+    pdl_trigger();
     if (tid == 0) {
         mbar_init(&bars->q_full, QTM ? NEXP : 1);   // TMA copy, or one arrival per exponent warp
         mbar_init(&bars->o_full, 1);
@@ -183,6 +196,9 @@ tc_gauss_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant_
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
+    // The prologue above may overlap the previous kernel of the call; its
+    // outputs (operands, values, norms) are read only from here on.
+    pdl_wait();
     const uint32_t tmem = bars->tmem_base;
     const uint32_t S_col0 = 0, P_col0 = 2 * BN, O_col = 3 * BN;
     const uint32_t Q_col = 3 * BN + static_cast<uint32_t>(p.Cp);   // QTM
@@ -438,9 +454,9 @@ tc_gauss_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant_
 #pragma unroll
             for (int ch = 0; ch < NCH; ++ch)
                 tmem_ld_32x32b_x32(tmem + lane_base + S_col0 + b * BN + col0 + ch * 32, r[ch]);
-            tmem_wait_ld();
-#pragma unroll
-            for (int ch = 0; ch < NCH; ++ch) tmem_regs_ready(r[ch]);
+            // The wait names the loaded registers, so that no use of them is
+            // scheduled above it (the loads land asynchronously).
+            tmem_wait_ld_regs(r[0], r[1]);
             // S buffer b is in registers: MMA1 of tile j + 2 may overwrite it
             // (EARLY; otherwise MMA1 of tile j + 2 follows P of tile j).
             if (EARLY) {
@@ -470,8 +486,8 @@ tc_gauss_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant_
                     float x0, x1, x2, x3;
                     f32x2_unpack(f32x2_fma(s01, c2, t01), x0, x1);
                     f32x2_unpack(f32x2_fma(s23, c2, t23), x2, x3);
-                    pk[2 * i + 0] = pack_half2_satfinite(ex2_approx(x0), ex2_approx(x1));
-                    pk[2 * i + 1] = pack_half2_satfinite(ex2_approx(x2), ex2_approx(x3));
+                    pk[2 * i + 0] = bound_p2(pack_half2_satfinite(ex2_approx(x0), ex2_approx(x1)));
+                    pk[2 * i + 1] = bound_p2(pack_half2_satfinite(ex2_approx(x2), ex2_approx(x3)));
                 }
                 if (EARLY && ch == 0 && j >= 2) {
                     // P buffer b: MMA2 of tile j - 2 has read it.  (With one
@@ -497,8 +513,7 @@ tc_gauss_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant_
             for (int c8 = epart * 8; c8 < p.Cp; c8 += 8 * PARTS) {
                 uint32_t r[8];
                 tmem_ld_32x32b_x8(tmem + lane_base + O_col + c8, r);
-                tmem_wait_ld();
-                tmem_regs_ready(r);
+                tmem_wait_ld_regs(r);
                 float4 lo = make_float4(__uint_as_float(r[0]) * P_UNSHIFT, __uint_as_float(r[1]) * P_UNSHIFT,
                                         __uint_as_float(r[2]) * P_UNSHIFT, __uint_as_float(r[3]) * P_UNSHIFT);
                 float4 hi = make_float4(__uint_as_float(r[4]) * P_UNSHIFT, __uint_as_float(r[5]) * P_UNSHIFT,
@@ -561,7 +576,7 @@ cudaError_t launch_bn(const TcPlan& pl, InType t, float c, char* ws, unsigned* s
                                          static_cast<int>(pl.smem_bytes));
     if (e != cudaSuccess) return e;
     dim3 grid(static_cast<unsigned>(pl.Mpad / BM), static_cast<unsigned>(pl.splits));
-    tc_gauss_kernel<BN, NEXP, AUG, EARLY, QTM><<<grid, cta_threads<NEXP>(), pl.smem_bytes, s>>>(tm_q, tm_k, tm_v, p);
+    launch_kernel(tc_gauss_kernel<BN, NEXP, AUG, EARLY, QTM>, grid, cta_threads<NEXP>(), pl.smem_bytes, s, tm_q, tm_k, tm_v, p);
     note_launches(1);
     return cudaGetLastError();
 }

@@ -65,12 +65,13 @@ constexpr int NQ = 2;              // query tiles per CTA
 constexpr int BN = 128;            // keys per key tile (MMA N)
 constexpr int KB = 64;             // 16-bit elements per 128-byte swizzled row
 constexpr int NEXP = 16;
-// Exponentials on the FMA pipe (exp2_fma_x2) instead of MUFU, augmented
-// path: the pair of row 0 (kSoftExpX) or row 1 (kSoftExpY) of key pair t
-// takes the FMA route when (t & mask) == 0; -1: never.  Each mask m moves
-// 1 / (4 (m + 1)) of the exponentials.
-constexpr int kSoftExpX = -1;
-constexpr int kSoftExpY = -1;
+// Exponentials on the FMA pipe (exp2_fma_x2) instead of MUFU (augmented
+// operands, template parameter SOFT = 1..4): the kernel values of row 0 of
+// key pair t take the FMA route when (t & soft_mask(SOFT)) == 0, which moves
+// 1/32, 1/16, 1/8 or 1/4 of the exponentials; SOFT = 0: none.
+__host__ __device__ constexpr int soft_mask(int soft) {
+    return soft == 1 ? 15 : soft == 2 ? 7 : soft == 3 ? 3 : 1;
+}
 constexpr int CTRL_WARP0 = 16;     // control warps 16..19, one per SMSP
 constexpr int NCTRL_MAX = 4;
 constexpr int THREADS = (NEXP + NCTRL_MAX) * 32;
@@ -125,6 +126,7 @@ struct __align__(8) FmaBarriers {
     uint64_t kv_full[MAX_STAGES];
     uint64_t kv_empty[MAX_STAGES];
     uint64_t stall;             // test hook: a barrier nothing arrives on
+    uint64_t drain[NCTRL_MAX];  // control warp k: its MMAs are complete
     uint32_t tmem_base;
     int abort_flag;
 };
@@ -210,12 +212,14 @@ __device__ __forceinline__ void exp_warps_sync() {
 // TRI: upper-triangle order for v^T K v (q = k, C = 1, augmented
 // operands): key tiles past the pair's own two get the weight 2, applied as
 // +1 in the exponent.
-template <int C, bool AUG, bool QSM, bool TF, bool TRI>
+template <int C, bool AUG, bool QSM, bool TF, bool TRI, int SOFT>
 __global__ void __launch_bounds__(THREADS, 1)
 tc_gauss_fma_kernel(const __grid_constant__ CUtensorMap tm_q,
                     const __grid_constant__ CUtensorMap tm_k, const FmaParams p) {
     // TF (3xTF32): q^ in shared memory, norm terms from A and the records.
     static_assert(!TF || (QSM && !AUG), "3xTF32 runs with q^ in shared memory");
+    static_assert(SOFT == 0 || (AUG && !TRI), "FMA-pipe exponentials: augmented operands");
+    constexpr int kSoftMask = soft_mask(SOFT);
     constexpr int REC_PAIR = (AUG ? 0 : 2) + 2 * C;   // floats per key pair
     constexpr int SL = QSM ? 2 : 1;
     extern __shared__ uint8_t smem_raw[];
@@ -231,6 +235,7 @@ tc_gauss_fma_kernel(const __grid_constant__ CUtensorMap tm_q,
     const int lane = tid & 31;
     volatile int* abort_flag = &bars->abort_flag;
 
+    pdl_trigger();
     if (tid == 0) bars->abort_flag = 0;
     if (warp == CTRL_WARP0) {
         tmem_alloc(&bars->tmem_base, TMEM_COLS);
@@ -256,9 +261,10 @@ tc_gauss_fma_kernel(const __grid_constant__ CUtensorMap tm_q,
     if (tid == 0) {
         mbar_init(&bars->qa_ready, QSM ? 1 : NEXP);
         mbar_init(&bars->stall, 1);
+        for (int k = 0; k < NCTRL_MAX; ++k) mbar_init(&bars->drain[k], 1);
         for (int sl = 0; sl < SL; ++sl) {
             mbar_init(&bars->s_full[sl], 1);
-            mbar_init(&bars->s_free[sl], NEXP);        // one arrival per exponent warp
+            mbar_init(&bars->s_free[sl], NEXP);        // one arrival per exponent warp (one slot)
         }
         for (int s = 0; s < p.stages; ++s) {
             mbar_init(&bars->kv_full[s], 1);
@@ -267,6 +273,9 @@ tc_gauss_fma_kernel(const __grid_constant__ CUtensorMap tm_q,
         fence_mbar_init();
     }
     __syncthreads();
+    // The prologue above may overlap the previous kernel of the call; its
+    // outputs (operands, key records) are read only from here on.
+    pdl_wait();
     // Unit indices fit in 32 bits (the plan checks units < 2^31).
     const int u_begin = static_cast<int>(blockIdx.x) * p.unit_len;
     const int u_end = p.units < u_begin + p.unit_len ? p.units : u_begin + p.unit_len;
@@ -281,6 +290,10 @@ tc_gauss_fma_kernel(const __grid_constant__ CUtensorMap tm_q,
         // Control warps need few registers; the exponent warps take them
         // (16 x 32 x kExpRegs + 4 x 32 x kCtrlRegs <= 640 x 96 at launch).
         reg_dealloc<kCtrlRegs>();
+        // The lane that issues this warp's copies, MMAs and commits (the
+        // warp is converged here; the same lane for the whole kernel).
+        const bool leader = elect_one();
+        bool issued = false;       // this warp has issued MMAs (warp-uniform)
         uint32_t seg_parity = 0;   // parity of the qa_ready phase of this segment
         int u = u_begin, run = 0, g0 = 0;   // g0: running index of the segment's first tile
         Segment sg;
@@ -305,7 +318,6 @@ tc_gauss_fma_kernel(const __grid_constant__ CUtensorMap tm_q,
             // This warp's tiles: running index g = g0 + j with g = k (mod nctrl).
             const int j_first = (k - g0 % nctrl + nctrl) % nctrl;
             const bool has_tiles = k < nctrl && j_first < T;
-            const bool leader = elect_one();
             if (QSM && k == 0 && leader) {
                 // q^ of this segment; the MMAs of earlier segments are complete.
                 tma_prefetch_desc(&tm_q);
@@ -358,15 +370,22 @@ tc_gauss_fma_kernel(const __grid_constant__ CUtensorMap tm_q,
                     // slot that tile g - SL released.
                     const int g = g0 + j;
                     const int sl = SL == 2 ? (g & 1) : 0;
-                    const uint32_t full_parity = static_cast<uint32_t>(SL == 2 ? (g >> 1) : g) & 1u;
-                    const uint32_t free_parity = full_parity ^ 1u;
+                    // The barrier that reports the slot free again: with two
+                    // slots (q^ in shared memory, four stages) the stage
+                    // release of tile g - 2, on stage (k + 2) mod 4 (the
+                    // exponent warps release a tile's stage and slot with one
+                    // arrival, after its MMAs have completed); with one slot,
+                    // s_free of tile g - 1.
+                    uint64_t* free_bar = QSM ? &bars->kv_empty[(k + 2) & 3] : &bars->s_free[0];
+                    const uint32_t free_parity =
+                        static_cast<uint32_t>(QSM ? ((g - 2) >> 2) : (g - 1)) & 1u;
                     const bool ready = __all_sync(
                         0xffffffffu, g < SL ? mbar_test_wait(&bars->kv_full[k], ph)
-                                            : mbar_test_wait2(&bars->s_free[sl], free_parity,
+                                            : mbar_test_wait2(free_bar, free_parity,
                                                               &bars->kv_full[k], ph));
                     if (!ready) {
                         if (g >= SL) {
-                            ok = warp_wait(&bars->s_free[sl], free_parity, abort_flag, p.status);
+                            ok = warp_wait(free_bar, free_parity, abort_flag, p.status);
                             if (!ok) break;
                         }
                         ok = warp_wait(&bars->kv_full[k], ph, abort_flag, p.status);
@@ -411,6 +430,7 @@ tc_gauss_fma_kernel(const __grid_constant__ CUtensorMap tm_q,
                         mma_commit(&bars->kv_empty[k]);
                     }
                     __syncwarp();
+                    issued = true;
                     // Stage k is free again once these MMAs and the exponent
                     // warps are done with tile j; after the last tile this also
                     // makes sure every arrival on the stage has landed before the
@@ -423,13 +443,11 @@ tc_gauss_fma_kernel(const __grid_constant__ CUtensorMap tm_q,
                         pending = true;
                     }
                 }
-                // Every copy and MMA this warp started must be complete before
-                // the barriers are initialised again or the CTA exits.  The
-                // stage-release wait after the last tile already covers the MMAs
-                // (the commit on kv_empty arrives once all MMAs this thread
-                // issued are complete); copies still in flight after an abort
-                // are waited for here.  These waits poll per lane, so the warp
-                // reconverges after them.
+                // Every copy this warp started must be complete before the
+                // CTA moves on: copies still in flight after an abort are
+                // waited for here (MMAs in flight after an abort are drained
+                // once, before TMEM is freed).  These waits poll per lane, so
+                // the warp reconverges after them.
                 if (pending) mbar_wait_bounded(&bars->kv_full[k], ph, nullptr, p.status);
                 __syncwarp();
             }
@@ -442,6 +460,18 @@ tc_gauss_fma_kernel(const __grid_constant__ CUtensorMap tm_q,
         // Segment end: every MMA, copy and TMEM read of this segment is done
         // (control warps waited for their last stage release and copies).
         segment_sync();
+        }
+        // No MMA of this warp may still run when TMEM is freed.  Without an
+        // abort the last stage-release wait has already seen them complete;
+        // after an abort a tile's MMAs may still be in flight.  The commit
+        // arrives on this warp's own drain barrier once every tcgen05
+        // operation the leader issued is done, so the wait ends by itself.
+        if (issued) {
+            const int k = warp - CTRL_WARP0;
+            if (leader) mma_commit(&bars->drain[k]);
+            __syncwarp();
+            mbar_wait_bounded(&bars->drain[k], 0, nullptr, p.status);
+            __syncwarp();
         }
     } else {
         reg_alloc<kExpRegs>();
@@ -495,41 +525,52 @@ tc_gauss_fma_kernel(const __grid_constant__ CUtensorMap tm_q,
             for (int cc = 0; cc < C; ++cc) acc0[cc] = acc1[cc] = 0ull;
             bool ok = true;
             bool ready = false;   // both barriers of key tile j already seen complete
-            RingPos st, sl;       // stage and TMEM slot of key tile j (running index g0 + j)
+            // Stage and TMEM slot of key tile j (running index g = g0 + j):
+            // with q^ in shared memory four stages and two slots, so stage
+            // g mod 4 with phase parity (g / 4) mod 2 and slot g mod 2 with
+            // parity (g / 2) mod 2 come from bits of g; otherwise a ring.
+            RingPos st, sl;
             st.idx = g0 % p.stages;
             st.phase = static_cast<uint32_t>(g0 / p.stages) & 1u;
-            sl.idx = g0 % SL;
-            sl.phase = static_cast<uint32_t>(g0 / SL) & 1u;
-            for (int j = 0; j < T; ++j, st.advance(p.stages), sl.advance(SL)) {
-                const int s = st.idx;
-                const uint32_t col0 = static_cast<uint32_t>(sl.idx * 2 * BN);
-                if (!__all_sync(0xffffffffu, ready || mbar_test_wait2(&bars->kv_full[s], st.phase,
-                                                                      &bars->s_full[sl.idx], sl.phase))) {
-                    ok = warp_wait(&bars->kv_full[s], st.phase, abort_flag, p.status);
-                    if (ok) ok = warp_wait(&bars->s_full[sl.idx], sl.phase, abort_flag, p.status);
+            sl.idx = 0;
+            sl.phase = static_cast<uint32_t>(g0) & 1u;
+            const uint32_t tcol = tmem + lane_base + static_cast<uint32_t>(cg * 32);
+            for (int j = 0; j < T; ++j) {
+                const int g = g0 + j;
+                const int s = QSM ? (g & 3) : st.idx;
+                const uint32_t st_ph = QSM ? (static_cast<uint32_t>(g >> 2) & 1u) : st.phase;
+                const int sli = QSM ? (g & 1) : 0;
+                const uint32_t sl_ph = QSM ? (static_cast<uint32_t>(g >> 1) & 1u) : sl.phase;
+                const uint32_t col0 = static_cast<uint32_t>(sli * 2 * BN);
+                if (!__all_sync(0xffffffffu, ready || mbar_test_wait2(&bars->kv_full[s], st_ph,
+                                                                      &bars->s_full[sli], sl_ph))) {
+                    ok = warp_wait(&bars->kv_full[s], st_ph, abort_flag, p.status);
+                    if (ok) ok = warp_wait(&bars->s_full[sli], sl_ph, abort_flag, p.status);
                     if (!ok) break;
                 }
                 tc_fence_after();
                 uint32_t r0[32], r1[32];
-                tmem_ld_32x32b_x32(tmem + lane_base + col0 + cg * 32, r0);
-                tmem_ld_32x32b_x32(tmem + lane_base + col0 + BN + cg * 32, r1);
+                tmem_ld_32x32b_x32(tcol + col0, r0);
+                tmem_ld_32x32b_x32(tcol + col0 + BN, r1);
                 // The wait names r0 and r1, so that no use of the loaded
                 // values is scheduled above it (the loads land asynchronously).
                 tmem_wait_ld_regs(r0, r1);
                 // When and where the S slot is handed back: with two slots
                 // (q^ in shared memory) only after the exponent work of this
-                // tile (with the stage, below), because releasing it right
-                // after the loads let the next MMAs into the slot corrupt S
-                // values of this tile in some warps when the MMAs were long
-                // (measured with 3xTF32 operands and three or more stages).
-                // With one slot (q^ in TMEM) a late release would serialise
-                // the MMAs and the exponent work, so it is released here; no
-                // corruption was seen there in repeated runs (regression
-                // test: repeated calls agree bit for bit).
+                // tile, together with the stage (one arrival), because
+                // releasing it right after the loads let the next MMAs into
+                // the slot corrupt S values of this tile in some warps when
+                // the MMAs were long (3xTF32 operands, three or more stages;
+                // still seen with the loads' registers named in the wait, and
+                // no faster on the 65536^2, D = 64 sum: 0.6428 against
+                // 0.6418 ms).  With one slot (q^ in TMEM) a late release
+                // would serialise the MMAs and the exponent work, so it is
+                // released here; no corruption was seen there in repeated
+                // runs (regression test: repeated calls agree bit for bit).
                 if (!QSM) {
                     tc_fence_before();
                     __syncwarp();
-                    mbar_arrive_if_zero(&bars->s_free[sl.idx], lane);
+                    mbar_arrive_if_zero(&bars->s_free[0], lane);
                 }
                 // Query the barriers of key tile j + 1 now and read the answer
                 // after the exponent work of tile j: the query latency overlaps
@@ -543,11 +584,10 @@ tc_gauss_fma_kernel(const __grid_constant__ CUtensorMap tm_q,
                 // ready this early (skipping the query: fp32 65536^2 sums 4-5 %
                 // faster).
                 if (QSM && !TF) {
-                    RingPos st2 = st, sl2 = sl;
-                    st2.advance(p.stages);
-                    sl2.advance(SL);
-                    ready = j + 1 < T && mbar_test_wait2(&bars->kv_full[st2.idx], st2.phase,
-                                                         &bars->s_full[sl2.idx], sl2.phase);
+                    const int g1 = g + 1;
+                    ready = j + 1 < T &&
+                            mbar_test_wait2(&bars->kv_full[g1 & 3], static_cast<uint32_t>(g1 >> 2) & 1u,
+                                            &bars->s_full[g1 & 1], static_cast<uint32_t>(g1 >> 1) & 1u);
                 }
                 const float* rec = rec_smem(s) + (cg * 16) * REC_PAIR;
                 const uint64_t w2 = (TRI && j >= w_from) ? f32x2_pack(1.f, 1.f) : 0ull;
@@ -558,21 +598,21 @@ tc_gauss_fma_kernel(const __grid_constant__ CUtensorMap tm_q,
                     for (int t = 0; t < 16; ++t) {
                         const float* pr = rec + t * REC_PAIR;
                         uint64_t px, py;
-                        if (kSoftExpX >= 0 && (t & kSoftExpX) == 0) {
+                        if (SOFT > 0 && (t & kSoftMask) == 0) {
                             px = exp2_fma_x2(__uint_as_float(r0[2 * t]), __uint_as_float(r0[2 * t + 1]), c2, s_min);
                         } else {
                             float x0, x1;
                             const uint64_t sx = f32x2_pack(__uint_as_float(r0[2 * t]), __uint_as_float(r0[2 * t + 1]));
                             f32x2_unpack(TRI ? f32x2_fma(sx, c2, w2) : f32x2_mul(sx, c2), x0, x1);
-                            px = f32x2_pack(ex2_approx(x0), ex2_approx(x1));
+                            px = f32x2_pack(TRI ? ex2_approx(x0) : ex2_nonpos(x0),
+                                            TRI ? ex2_approx(x1) : ex2_nonpos(x1));
                         }
-                        if (kSoftExpY >= 0 && (t & kSoftExpY) == 0) {
-                            py = exp2_fma_x2(__uint_as_float(r1[2 * t]), __uint_as_float(r1[2 * t + 1]), c2, s_min);
-                        } else {
+                        {
                             float y0, y1;
                             const uint64_t sy = f32x2_pack(__uint_as_float(r1[2 * t]), __uint_as_float(r1[2 * t + 1]));
                             f32x2_unpack(TRI ? f32x2_fma(sy, c2, w2) : f32x2_mul(sy, c2), y0, y1);
-                            py = f32x2_pack(ex2_approx(y0), ex2_approx(y1));
+                            py = f32x2_pack(TRI ? ex2_approx(y0) : ex2_nonpos(y0),
+                                            TRI ? ex2_approx(y1) : ex2_nonpos(y1));
                         }
     #pragma unroll
                         for (int cc = 0; cc < C; ++cc) {
@@ -604,8 +644,8 @@ tc_gauss_fma_kernel(const __grid_constant__ CUtensorMap tm_q,
                     float x0, x1, y0, y1;
                     f32x2_unpack(x01, x0, x1);
                     f32x2_unpack(y01, y0, y1);
-                    const uint64_t px = f32x2_pack(ex2_approx(x0), ex2_approx(x1));
-                    const uint64_t py = f32x2_pack(ex2_approx(y0), ex2_approx(y1));
+                    const uint64_t px = f32x2_pack(ex2_nonpos(x0), ex2_nonpos(x1));
+                    const uint64_t py = f32x2_pack(ex2_nonpos(y0), ex2_nonpos(y1));
                     const uint64_t vv0 = f32x2_pack(v0.x, v0.y);
                     acc0[0] = f32x2_fma(px, vv0, acc0[0]);
                     acc1[0] = f32x2_fma(py, vv0, acc1[0]);
@@ -623,8 +663,11 @@ tc_gauss_fma_kernel(const __grid_constant__ CUtensorMap tm_q,
                 // Lane 0 hands back the slot (two-slot path) and the stage,
                 // predicated rather than branched: a divergent branch here
                 // cost 0.7 % of the kernel time.
-                if (QSM) mbar_arrive2_if_zero(&bars->s_free[sl.idx], &bars->kv_empty[s], lane);
-                else mbar_arrive_if_zero(&bars->kv_empty[s], lane);
+                mbar_arrive_if_zero(&bars->kv_empty[s], lane);
+                if (!QSM) {
+                    st.advance(p.stages);
+                    sl.advance(1);
+                }
             }
             // Fixed-order reduction of the NPART column-group partial sums.
     #pragma unroll
@@ -687,7 +730,7 @@ size_t q_bytes_for(int nkb, bool qsm) {
     return qsm ? static_cast<size_t>(NQ) * nkb * BM * 128 : 0;
 }
 
-template <int C, bool AUG, bool QSM, bool TF, bool TRI = false>
+template <int C, bool AUG, bool QSM, bool TF, bool TRI = false, int SOFT = 0>
 cudaError_t launch_typed(const TcPlan& pl, InType t, float c, char* ws, unsigned* status,
                          cudaStream_t s, const char** why) {
     const CUtensorMapDataType hdt =
@@ -731,12 +774,12 @@ cudaError_t launch_typed(const TcPlan& pl, InType t, float c, char* ws, unsigned
     p.c = c;
     const uint32_t hb = t == InType::BF16 ? 1u : 0u;
     p.idesc = TF ? idesc_tf32(BM, BN) : idesc_f16(BM, BN, hb, hb);
-    cudaError_t e = cudaFuncSetAttribute(tc_gauss_fma_kernel<C, AUG, QSM, TF, TRI>,
+    cudaError_t e = cudaFuncSetAttribute(tc_gauss_fma_kernel<C, AUG, QSM, TF, TRI, SOFT>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          static_cast<int>(pl.smem_bytes));
     if (e != cudaSuccess) return e;
     dim3 grid(static_cast<unsigned>(pl.grid));
-    tc_gauss_fma_kernel<C, AUG, QSM, TF, TRI><<<grid, THREADS, pl.smem_bytes, s>>>(tm_q, tm_k, p);
+    launch_kernel(tc_gauss_fma_kernel<C, AUG, QSM, TF, TRI, SOFT>, grid, THREADS, pl.smem_bytes, s, tm_q, tm_k, p);
     note_launches(1);
     return cudaGetLastError();
 }
@@ -747,6 +790,14 @@ cudaError_t launch_c(const TcPlan& pl, InType t, float c, char* ws, unsigned* st
     if (pl.tf) return launch_typed<C, false, true, true>(pl, t, c, ws, status, s, why);
     if constexpr (C == 1 && kAugQsm) {
         if (pl.tri && pl.aug) return launch_typed<1, true, true, false, true>(pl, t, c, ws, status, s, why);
+        if (pl.aug && pl.exp2_fma > 0) {
+            switch (pl.exp2_fma) {
+                case 1: return launch_typed<1, true, true, false, false, 1>(pl, t, c, ws, status, s, why);
+                case 2: return launch_typed<1, true, true, false, false, 2>(pl, t, c, ws, status, s, why);
+                case 3: return launch_typed<1, true, true, false, false, 3>(pl, t, c, ws, status, s, why);
+                default: return launch_typed<1, true, true, false, false, 4>(pl, t, c, ws, status, s, why);
+            }
+        }
     }
     if (pl.aug) return launch_typed<C, true, kAugQsm, false>(pl, t, c, ws, status, s, why);
     return launch_typed<C, false, false, false>(pl, t, c, ws, status, s, why);
@@ -776,6 +827,9 @@ bool plan_fma_kernel(int Dp, int C, bool aug, bool tf, int* nq, int* stages, siz
     const int st = static_cast<int>(
         std::min<size_t>(std::min(MAX_STAGES, 2 * sl), (budget - fixed) / stage));
     if (st < 2) return false;
+    // With q^ in shared memory the kernel derives stage and slot from the
+    // running tile index for exactly four stages (two per slot).
+    if (qsm && st != MAX_STAGES) return false;
     *nq = NQ;
     *stages = st;
     *smem = std::max<size_t>(fixed + st * stage, 118 * 1024);

@@ -13,9 +13,11 @@ nearest even).  The clouds follow the benchmark of Sec. 4 of the paper
 tau = 1, which is the same kernel as unscaled points at tau = 1/D).
 
   fp32_d16     M=N=4096,   D=16,  C=1,  fp32: q, k, v ~ N(0,1); tau = 1/16
-  mmd_d64      M=N=65536,  D=64,  C=1,  fp16: X ~ N(0,1), q = k = X (the MMD
-               form q = k of Sec. 3); v = +1/N for the first N/2 points,
+  mmd_d64      M=N=65536,  D=64,  C=1,  fp16: q ~ N(0,1) and k ~ N(0,1) drawn
+               independently (q first); v = +1/N for the first N/2 keys,
                -1/N for the rest; tau = 1/64
+  mmd_d64_qk   the same sizes in the MMD form q = k = X of Sec. 3 (one cloud
+               X ~ N(0,1) carrying both signed halves)
   multi_c64    M=N=262144, D=128, C=64, bf16: q, k ~ 0.5 N(0,1); v ~ N(0,1);
                tau = 2/128
   svgd_d32     M=N=131072, D=32,  C=1,  fp16: 4-component Gaussian mixture
@@ -67,8 +69,10 @@ class Workload:
 WORKLOADS = {
     "fp32_d16": Workload("fp32_d16", 4096, 4096, 16, 1, "fp32", 1.0 / 16, "normal",
                          note="forward Gauss sum in fp32"),
-    "mmd_d64": Workload("mmd_d64", 65536, 65536, 64, 1, "fp16", 1.0 / 64, "mmd", q_is_k=True,
+    "mmd_d64": Workload("mmd_d64", 65536, 65536, 64, 1, "fp16", 1.0 / 64, "independent_mmd",
                         note="MMD-style forward in fp16, fp32 accumulation"),
+    "mmd_d64_qk": Workload("mmd_d64_qk", 65536, 65536, 64, 1, "fp16", 1.0 / 64, "mmd",
+                           q_is_k=True, note="MMD-style forward, q = k form"),
     "multi_c64": Workload("multi_c64", 262144, 262144, 128, 64, "bf16", 2.0 / 128, "half_normal",
                           note="multi-channel forward in bf16"),
     "svgd_d32": Workload("svgd_d32", 131072, 131072, 32, 1, "fp16", 1.0 / 32, "gmm", grad=True,

@@ -1,10 +1,12 @@
 """The five workloads at full size, in the launch configuration bench.py
 times (default options), checked against the float64 oracle on all rows
-(fp32 workload) or on seeded row samples the oracle computes one by one."""
+(fp32_d16, mmd_d64) or on seeded row samples the oracle computes one by one
+(multi_c64: 256 rows, svgd_d32: 4096, offset_d256: 1024 with centring on
+and off, the q = k reading of mmd_d64: 1024)."""
 import numpy as np
 import pytest
 
-from paper_2609_04910_gb300.workloads import WORKLOADS, Workload, sample_rows
+from paper_2609_04910_gb300.workloads import WORKLOADS, sample_rows
 from tests.gpu_helpers import forward_check, grad_check
 
 pytestmark = pytest.mark.gpu
@@ -27,19 +29,20 @@ def test_fp32_d16_all_rows():
     print(f"fp32_d16 max rel {rel:.3e}")
 
 
-def test_mmd_d64_sampled_rows():
+def test_mmd_d64_all_rows():
+    """The bench workload (independent q and k draws) on every one of its
+    65536 rows."""
     w = WORKLOADS["mmd_d64"]
-    rel, got, ref, den = forward_check(w, rows=sample_rows(w.M, 512))
-    print(f"mmd_d64 max rel {rel:.3e}")
+    rel, got, ref, den = forward_check(w)
+    print(f"mmd_d64 all rows max rel {rel:.3e}")
 
 
-def test_mmd_d64_independent_draws():
-    """Alternative reading of the MMD workload: independent q and k draws."""
-    base = WORKLOADS["mmd_d64"]
-    w = Workload("mmd_d64_indep", base.M, base.N, base.D, base.C, base.dtype, base.tau,
-                 "independent_mmd")
-    rel, *_ = forward_check(w, rows=sample_rows(w.M, 256))
-    print(f"mmd_d64 (independent q, k) max rel {rel:.3e}")
+def test_mmd_d64_q_is_k_sampled_rows():
+    """The other reading of the MMD workload: q = k = X (one cloud carrying
+    the two signed halves), 1024 seeded rows."""
+    w = WORKLOADS["mmd_d64_qk"]
+    rel, *_ = forward_check(w, rows=sample_rows(w.M, 1024))
+    print(f"mmd_d64 (q = k) max rel {rel:.3e}")
 
 
 def test_multi_c64_256_rows():
@@ -50,12 +53,12 @@ def test_multi_c64_256_rows():
 
 def test_svgd_d32_grad_and_sum():
     w = WORKLOADS["svgd_d32"]
-    relg, rels = grad_check(w, rows=sample_rows(w.M, 384))
+    relg, rels = grad_check(w, rows=sample_rows(w.M, 4096))
     print(f"svgd_d32 grad max rel {relg:.3e}, s max rel {rels:.3e}")
 
 
 @pytest.mark.parametrize("center", [True, False])
 def test_offset_d256(center):
     w = WORKLOADS["offset_d256"]
-    rel, got, ref, den = forward_check(w, rows=sample_rows(w.M, 128), center=center)
+    rel, got, ref, den = forward_check(w, rows=sample_rows(w.M, 1024), center=center)
     print(f"offset_d256 center={center} max rel {rel:.3e}")

@@ -4,7 +4,7 @@ Every mbarrier wait of the fused kernels is bounded (2 s of globaltimer);
 when one runs out, the kernel writes GS_ERR_DEVICE_TIMEOUT and where it
 happened into the device status words, raises an abort flag that every
 other role of the CTA polls, frees its tensor memory and returns.  The test
-hook GS_TEST_STALL=1 makes one control warp of CTA 0 wait on a barrier
+hook gauss_sum_testing_request_stall makes one control warp of CTA 0 wait on a barrier
 that nothing arrives on; the test checks that gauss_sum_device_status
 reports the timeout and that the next call on the same context runs
 normally (its result matches the oracle).
@@ -28,7 +28,7 @@ def _gpu():
     torch.cuda.set_device(0)
 
 
-def test_bounded_wait_runs_out_and_context_stays_usable(monkeypatch):
+def test_bounded_wait_runs_out_and_context_stays_usable():
     import paper_2609_04910_gb300 as gs
     from oracle import oracle_sum
     from paper_2609_04910_gb300.workloads import generate
@@ -37,9 +37,9 @@ def test_bounded_wait_runs_out_and_context_stays_usable(monkeypatch):
     q, k, v = device_inputs(inp)
     gs.gauss_sum_device_status()               # start from a clear status
 
-    monkeypatch.setenv("GS_TEST_STALL", "1")
+    from paper_2609_04910_gb300._binding import testing_request_stall
+    testing_request_stall()
     gs.gauss_sum(q, k, v, w.tau)               # the launch itself succeeds
-    monkeypatch.delenv("GS_TEST_STALL")
     with pytest.raises(gs.GaussSumError) as ei:
         gs.gauss_sum_device_status()
     assert ei.value.status == 5                # GS_ERR_DEVICE_TIMEOUT

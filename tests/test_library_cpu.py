@@ -18,19 +18,23 @@ def lib():
     return load_library()
 
 
-def _declared_functions():
-    src = open(os.path.join(ROOT, "include", "gauss_sum.h")).read()
+def _declared_functions(header="gauss_sum.h"):
+    src = open(os.path.join(ROOT, "include", header)).read()
     src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
     names = re.findall(r"\b(gauss_sum\w*)\s*\(", src)
     return sorted(set(names))
 
 
 def test_every_declared_symbol_is_exported(lib):
-    from paper_2609_04910_gb300._binding import EXPORTS
+    from paper_2609_04910_gb300._binding import EXPORTS, TESTING_EXPORTS
     declared = _declared_functions()
     assert len(declared) == 15
     assert sorted(EXPORTS) == declared
-    for name in declared:
+    testing = _declared_functions("gauss_sum_testing.h")
+    assert sorted(TESTING_EXPORTS) == testing
+    headers = sorted(f for f in os.listdir(os.path.join(ROOT, "include")) if f.endswith(".h"))
+    assert headers == ["gauss_sum.h", "gauss_sum_testing.h"]
+    for name in declared + testing:
         assert hasattr(lib, name), name
 
 
@@ -54,6 +58,19 @@ def test_default_options(lib):
     lib.gauss_sum_default_options(ctypes.byref(o))
     assert (o.center, o.split_n, o.workspace, o.workspace_bytes, o.path) == (1, 0, None, 0, 0)
     assert list(o.main_events) == [None, None]
+    assert o.exp2_fma == 0
+
+
+@pytest.mark.parametrize("bad", [-1, 5])
+def test_exp2_fma_range_checked(lib, bad):
+    from paper_2609_04910_gb300._binding import GsOptions
+    o = GsOptions()
+    lib.gauss_sum_default_options(ctypes.byref(o))
+    o.exp2_fma = bad
+    st = lib.gauss_sum_ex(ALIGNED, ALIGNED, ALIGNED, 1.0, 4, 4, 3, 1, 1, ALIGNED, None,
+                          ctypes.byref(o))
+    assert st == 1
+    assert b"exp2_fma" in lib.gauss_sum_last_error()
 
 
 ALIGNED = 4096  # a fake 16-byte-aligned address; never dereferenced

@@ -102,7 +102,11 @@ def test_long_key_range_one_split(D, dtype):
 @pytest.mark.parametrize("M,N,D,C,dtype,grad", [
     (300, 5000, 64, 16, "fp16", False),   # BN 128, augmented, early S release (six stages)
     (200, 5000, 64, 100, "fp16", False),  # BN 128, plain operands, early S release (four stages)
-    (200, 5000, 128, 64, "bf16", False),  # BN 128, three stages: one MMA warp, P-then-S order
+    (200, 5000, 128, 64, "bf16", False),  # BN 128, q^ in TMEM buys a fourth stage: early release
+    (200, 5000, 128, 96, "fp16", False),  # BN 128, q^ in shared memory (TMEM full), three
+                                          # stages: one MMA warp, P-then-S order
+    (150, 3000, 160, 48, "fp16", False),  # BN 128, q^ in TMEM buys a third stage: one MMA
+                                          # warp, P-then-S order, A operand from TMEM
     (150, 3000, 32, 200, "fp16", False),  # BN 64, early S release
     (100, 3000, 256, 200, "fp16", False), # BN 64, two stages: one MMA warp
     (256, 5000, 32, 1, "fp16", True),     # gradient (33 channels), early S release
@@ -304,15 +308,18 @@ def test_unsupported_shapes_raise():
     assert ei.value.status == 2
 
 
-def test_forced_allocation_failure(monkeypatch):
+def test_forced_allocation_failure():
     import paper_2609_04910_gb300 as gs
+    from paper_2609_04910_gb300._binding import testing_fail_allocations
     q = torch.randn(4, 8, device="cuda", dtype=torch.float16)
     v = torch.ones(4, 1, device="cuda", dtype=torch.float16)
-    monkeypatch.setenv("GS_TEST_FAIL_ALLOC", "1")
-    with pytest.raises(gs.GaussSumError) as ei:
-        gs.gauss_sum(q, q, v, 1.0)
+    testing_fail_allocations(True)
+    try:
+        with pytest.raises(gs.GaussSumError) as ei:
+            gs.gauss_sum(q, q, v, 1.0)
+    finally:
+        testing_fail_allocations(False)
     assert ei.value.status == 3
-    monkeypatch.delenv("GS_TEST_FAIL_ALLOC")
     gs.gauss_sum(q, q, v, 1.0)
     torch.cuda.synchronize()
 
@@ -361,3 +368,81 @@ def test_keys_larger_than_l2_banded_order(M, N, D, C, dtype):
     (all CTAs inside a few bands of 64 key tiles, one partial-sum slot per
     band): ragged rows and key tail, every row against the oracle."""
     forward_check(case(M, N, D, C, dtype))
+
+
+# ---------------------------------------------------------------- exponent bound
+@pytest.mark.parametrize("D,C,dtype,path", [
+    (64, 1, "fp16", None),      # FMA kernel, augmented operands
+    (128, 2, "fp16", None),     # FMA kernel, q^ in TMEM, norms from A and B
+    (64, 8, "fp16", None),      # two-MMA kernel (P in fp16 with the 2^15 shift)
+    (48, 40, "bf16", None),     # two-MMA kernel, plain operands
+    (16, 1, "fp32", "tensor"),  # 3xTF32 variant of the FMA kernel
+])
+def test_self_pairs_never_exceed_one(D, C, dtype, path):
+    """The exponent is <= 0 in exact arithmetic (Phi <= 1, proof of Prop. 1);
+    for q = k the computed self-pair exponent is only rounding, which can
+    be slightly positive.  With tau large enough that every other pair
+    underflows to 0, s_m = Phi(x_m, x_m) for unit values: it must lie in
+    [1 - tol, 1] (the kernels clamp the exponent at 0), never above 1."""
+    import paper_2609_04910_gb300 as gs
+    w = case(300, 300, D, C, dtype, tau=200.0 / D)
+    inp = generate(w)
+    q, k, _ = device_inputs(inp)
+    v = torch.ones((300, C), dtype=q.dtype, device="cuda")
+    kw = {"path": gs.GS_PATH_TENSOR} if path == "tensor" else {}
+    # Centring off: the operands keep the points' full norms, so the
+    # rounding of the self-pair exponent is as large as it gets.
+    s = gs.gauss_sum(q, q, v, w.tau, center=False, **kw).cpu().numpy()
+    gs.gauss_sum_device_status()
+    ones = np.ones((300, C))
+    ref, den = oracle_sum(inp["q64"], inp["q64"], ones, w.tau)
+    assert np.max(np.abs(ref - 1.0)) < 1e-10      # other pairs vanish in float64 too
+    assert np.all(s <= 1.0), f"max {s.max()!r}"
+    tol = TOL[dtype]
+    if path == "tensor":
+        # 3xTF32: the exponent carries the tf32 split error, about
+        # c |x^|^2 2^-21 (c = tau log2 e); at tau = 200 / D that is above
+        # the fp32 tolerance, which holds while c |x^|^2 stays below ~20.
+        c = w.tau * np.log2(np.e)
+        tol = c * float(np.max(np.sum(inp["q64"] ** 2, axis=1))) * 2.0 ** -20
+    assert rel_err(s, ref, den) <= tol
+
+
+# ---------------------------------------------------------------- FMA-pipe exp2
+@pytest.mark.parametrize("share", [1, 2, 3, 4])
+@pytest.mark.parametrize("M,N,D,dtype,q_is_k", [
+    (300, 1000, 64, "fp16", False), (513, 700, 60, "bf16", False),
+    (700, 700, 64, "fp16", True),
+])
+def test_exp2_on_fma_pipe_parity(share, M, N, D, dtype, q_is_k):
+    """exp2_fma = 1..4 computes 1/32 .. 1/4 of the kernel values with the
+    Cody-Waite + minimax-polynomial exp2 on the FMA pipe; the sums still
+    match the oracle at the fp16/bf16 tolerance."""
+    w = case(M, N, D, 1, dtype, kind="mmd" if q_is_k else "normal", q_is_k=q_is_k)
+    forward_check(w, exp2_fma=share)
+
+
+def test_exp2_on_fma_pipe_matches_mufu_closely():
+    """The polynomial's relative error (< 3e-6) is far below the fp16
+    tolerance: the variant agrees with the MUFU-only sums to 1e-5 of the
+    oracle's scale, and far values flush to zero as with ex2.approx.ftz."""
+    import paper_2609_04910_gb300 as gs
+    w = case(600, 2000, 64, 1, "fp16")
+    inp = generate(w)
+    q, k, v = device_inputs(inp)
+    a = gs.gauss_sum(q, k, v, w.tau)
+    b = gs.gauss_sum(q, k, v, w.tau, exp2_fma=4)
+    gs.gauss_sum_device_status()
+    _, den = oracle_sum(inp["q64"], inp["k64"], inp["v64"], w.tau)
+    assert rel_err(b.cpu().numpy(), a.cpu().numpy(), den) <= 1e-5
+
+
+def test_exp2_on_fma_pipe_rejected_outside_its_range():
+    import paper_2609_04910_gb300 as gs
+    q = torch.randn(200, 64, device="cuda", dtype=torch.float16)
+    v2 = torch.randn(200, 2, device="cuda", dtype=torch.float16)
+    for args in ((q, q, v2), (q.float(), q.float(), v2[:, :1].float())):
+        with pytest.raises(gs.GaussSumError) as ei:
+            gs.gauss_sum(*args, 0.1, exp2_fma=2)
+        assert ei.value.status == 2
+        assert "exp2_fma" in ei.value.message

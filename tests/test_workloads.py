@@ -29,7 +29,7 @@ def test_roundings_are_exact_and_nearest():
 
 
 def test_mmd_weights_and_offset_norm():
-    w = WORKLOADS["mmd_d64"].resized(N=100)
+    w = WORKLOADS["mmd_d64"].resized(M=100, N=100)
     g = generate(w)
     assert np.sum(g["v64"] > 0) == 50 and np.sum(g["v64"] < 0) == 50
     w5 = WORKLOADS["offset_d256"].resized(M=8, N=8)
