@@ -27,9 +27,10 @@
  *    stream).  Calls are asynchronous and stream ordered; the status return
  *    covers argument checks, allocation and launch errors.  A device-side
  *    wait that runs out of time is reported by gauss_sum_device_status().
- *  - Without a caller workspace the library allocates its workspace with
- *    cudaMallocAsync on `stream` and frees it with cudaFreeAsync on the same
- *    stream.
+ *  - Without a caller workspace the library allocates its workspace on
+ *    `stream` (cudaMallocFromPoolAsync) and frees it on the same stream
+ *    (cudaFreeAsync), from a stream-ordered memory pool of its own per
+ *    device that keeps up to 1 GiB of freed workspace mapped between calls.
  *  - M = 0 is a no-op; N = 0 writes zeros.
  *  - fp16/bf16 inputs run on the tensor-core kernels (tcgen05, sm_103a) and
  *    need D <= 256 and C <= 256 (gradients: D <= 256, any C).  fp32 inputs

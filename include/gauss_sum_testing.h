@@ -16,7 +16,7 @@ extern "C" {
 
 /*
  * on != 0: every workspace allocation the library would make from now on
- * (cudaMallocAsync of gauss_sum_ex and friends, and of gauss_sum_mmd2)
+ * (the workspaces of gauss_sum_ex and friends, and of gauss_sum_mmd2)
  * fails with GS_ERR_OUT_OF_MEMORY before any GPU work; on = 0 restores
  * normal behaviour.  Process-wide.  Calls that allocate nothing (a caller
  * workspace, gauss_sum_noalloc) are unaffected.

@@ -68,6 +68,48 @@ cudaError_t device_info(int* dev, unsigned** status) {
 
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
+// Workspaces come from a stream-ordered memory pool of the library's own,
+// one per device, which keeps up to kPoolKeepBytes of freed workspace
+// mapped between calls (the device's default pool gives freed memory back to
+// the driver at every synchronisation, so that a caller who synchronises
+// between calls would pay a new mapping per call).
+constexpr uint64_t kPoolKeepBytes = uint64_t(1) << 30;
+cudaMemPool_t g_pool[kMaxDevices] = {};
+
+cudaError_t workspace_pool(int dev, cudaMemPool_t* pool) {
+    std::lock_guard<std::mutex> lk(g_dev_mu);
+    if (!g_pool[dev]) {
+        cudaMemPoolProps props = {};
+        props.allocType = cudaMemAllocationTypePinned;
+        props.location.type = cudaMemLocationTypeDevice;
+        props.location.id = dev;
+        cudaMemPool_t p = nullptr;
+        cudaError_t e = cudaMemPoolCreate(&p, &props);
+        if (e != cudaSuccess) return e;
+        uint64_t keep = kPoolKeepBytes;
+        e = cudaMemPoolSetAttribute(p, cudaMemPoolAttrReleaseThreshold, &keep);
+        if (e != cudaSuccess) {
+            cudaMemPoolDestroy(p);
+            return e;
+        }
+        g_pool[dev] = p;
+    }
+    *pool = g_pool[dev];
+    return cudaSuccess;
+}
+
+// Stream-ordered allocation from the library's pool of the current device.
+cudaError_t pool_alloc(void** ptr, size_t bytes, cudaStream_t s) {
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    if (dev < 0 || dev >= kMaxDevices) return cudaErrorInvalidDevice;
+    cudaMemPool_t pool = nullptr;
+    e = workspace_pool(dev, &pool);
+    if (e != cudaSuccess) return e;
+    return cudaMallocFromPoolAsync(ptr, bytes, pool, s);
+}
+
 struct Call {
     const void* q;
     const void* k;
@@ -256,8 +298,8 @@ gs_status run(Call c) {
             return fail(GS_ERR_OUT_OF_MEMORY, "caller workspace is smaller than gauss_sum_workspace_size()");
     } else if (bytes > 0) {
         if (forced_alloc_failure()) return fail(GS_ERR_OUT_OF_MEMORY, "workspace allocation failed (test hook)");
-        e = cudaMallocAsync(reinterpret_cast<void**>(&ws), bytes, c.stream);
-        if (e != cudaSuccess) return cuda_fail(e, "workspace cudaMallocAsync");
+        e = pool_alloc(reinterpret_cast<void**>(&ws), bytes, c.stream);
+        if (e != cudaSuccess) return cuda_fail(e, "workspace allocation");
         owned = true;
     }
 
@@ -269,28 +311,15 @@ gs_status run(Call c) {
     if (tensor) {
         const gs::InType t = in_type(c.dtype);
         float* mu = (tp.center && c.D > 0) ? reinterpret_cast<float*>(ws + tp.off_mu) : nullptr;
-        // 16-bit inputs with D a multiple of 8: mean, operands and (FMA
-        // kernel) key records in one cooperative launch.
-        const bool fused = !tp.tf && gs::fused_prep_supported(t, c.D);
-        if (fused) {
-            e = gs::launch_fused_prep(
-                t, tp.aug, c.q, c.k, tp.fma ? c.v : nullptr, c.M, c.N, tp.Mpad, tp.Npad,
-                static_cast<int>(c.D), tp.Dp, static_cast<int>(tp.Cv), tp.alias, half_c,
-                tp.mean_blocks, reinterpret_cast<float*>(ws + tp.off_mean_part), mu,
-                ws + tp.off_qh, ws + tp.off_kh,
-                tp.aug ? nullptr : reinterpret_cast<float*>(ws + tp.off_A),
-                tp.aug ? nullptr : reinterpret_cast<float*>(ws + tp.off_B),
-                tp.fma ? reinterpret_cast<float*>(ws + tp.off_rec) : nullptr, c.stream, batch);
-            where = "fused preparation kernel";
-        } else if (mu) {
+        if (mu) {
             e = gs::launch_mean(t, c.q, c.k, c.M, c.N, static_cast<int>(c.D), tp.mean_blocks,
                                 reinterpret_cast<float*>(ws + tp.off_mean_part), mu, c.stream,
                                 batch);
             where = "mean kernel";
         }
         const float ninf = -INFINITY;
-        if (fused || e != cudaSuccess) {
-            // Operands (and key records) written by the fused kernel, or an error.
+        if (e != cudaSuccess) {
+            // an error: nothing more is launched
         } else if (tp.tf) {
             // 3xTF32 operands: hi / lo tf32 halves and the norm terms.
             e = gs::launch_tf32_split(static_cast<const float*>(c.q), c.M, tp.Mpad,
@@ -307,41 +336,25 @@ gs_status run(Call c) {
                                           c.stream, batch);
                 where = "tf32 split kernel (k)";
             }
-        } else if (tp.aug) {
-            // Augmented operands: centred points with the norms folded in.
-            e = gs::launch_aug_prep(t, c.q, c.M, tp.Mpad, static_cast<int>(c.D), tp.Dp, mu,
-                                    ws + tp.off_qh, tp.alias ? ws + tp.off_kh : nullptr, c.stream,
-                                    batch);
-            where = "augmented-operand kernel (q)";
-            if (e == cudaSuccess && !tp.alias) {
-                e = gs::launch_aug_prep(t, c.k, c.N, tp.Npad, static_cast<int>(c.D), tp.Dp, mu,
-                                        nullptr, ws + tp.off_kh, c.stream, batch);
-                where = "augmented-operand kernel (k)";
-            }
         } else {
-            {
-                e = gs::launch_center_cast_norm(t, c.q, c.M, tp.Mpad, static_cast<int>(c.D), tp.Dp,
-                                                mu, half_c, ws + tp.off_qh,
-                                                reinterpret_cast<float*>(ws + tp.off_A), ninf,
-                                                c.stream, batch);
-                where = "centre/cast kernel (q)";
-            }
-            if (e == cudaSuccess && !tp.alias) {
-                e = gs::launch_center_cast_norm(t, c.k, c.N, tp.Npad, static_cast<int>(c.D), tp.Dp,
-                                                mu, half_c, ws + tp.off_kh,
-                                                reinterpret_cast<float*>(ws + tp.off_B), ninf,
-                                                c.stream, batch);
-                where = "centre/cast kernel (k)";
-            }
+            // Centred, rounded operands of q and (unless q is k) k in one
+            // launch: augmented rows (norms folded into the MMA), or plain
+            // rows with the norm terms A and B.
+            e = gs::launch_operands(
+                t, tp.aug, c.q, c.M, tp.Mpad, ws + tp.off_qh,
+                (tp.aug && tp.alias) ? ws + tp.off_kh : nullptr,
+                tp.aug ? nullptr : reinterpret_cast<float*>(ws + tp.off_A),
+                !tp.alias, c.k, c.N, tp.Npad, ws + tp.off_kh,
+                tp.aug ? nullptr : reinterpret_cast<float*>(ws + tp.off_B), static_cast<int>(c.D),
+                tp.Dp, mu, half_c, ninf, c.stream, batch);
+            where = tp.aug ? "augmented-operand kernel" : "centre/cast kernel";
         }
         if (e == cudaSuccess && tp.fma) {
-            if (!fused) {
-                e = gs::launch_key_records(
-                    t, c.v, tp.aug ? nullptr : reinterpret_cast<const float*>(ws + tp.off_B), c.N,
-                    tp.Npad, static_cast<int>(tp.Cv), reinterpret_cast<float*>(ws + tp.off_rec),
-                    c.stream, batch);
-                where = "key-record kernel";
-            }
+            e = gs::launch_key_records(
+                t, c.v, tp.aug ? nullptr : reinterpret_cast<const float*>(ws + tp.off_B), c.N,
+                tp.Npad, static_cast<int>(tp.Cv), reinterpret_cast<float*>(ws + tp.off_rec),
+                c.stream, batch);
+            where = "key-record kernel";
             if (e == cudaSuccess) e = record_event(c.opt.main_events[0], c.stream);
             if (e == cudaSuccess) {
                 e = gs::launch_tc_fma(tp, t, cexp, ws, status, c.stream, &why);
@@ -379,15 +392,17 @@ gs_status run(Call c) {
                 if (e == cudaSuccess && ch0 + width >= total)
                     e = record_event(c.opt.main_events[1], c.stream);
                 if (e == cudaSuccess) {
+                    // Rows of the unsplit row tiles have one partial sum.
+                    const int64_t main_rows = tp.main_tiles * 128;
                     if (c.grad)
                         e = gs::launch_finalize_points(
                             false, t, c.u_f32, part, tp.splits, tp.Mpad, c.M, tp.Cp, inv, c.q, mu,
                             static_cast<float>(c.tau), static_cast<int>(c.D),
                             static_cast<int>(c.C), static_cast<int>(ch0), cc, c.u, ch0 > 0,
-                            c.out, c.s_out, c.stream);
+                            c.out, c.s_out, c.stream, main_rows);
                     else
                         e = gs::launch_finalize(part, tp.splits, tp.Mpad, c.M, cc, tp.Cp, inv,
-                                                c.out, c.stream);
+                                                c.out, c.stream, main_rows);
                     where = "finalise kernel";
                 }
             }
@@ -576,9 +591,9 @@ gs_status gauss_sum_mmd2(const void* x, const void* v, double tau, int64_t B, in
     float* s_buf = nullptr;
     // s (B x N float32), then the float64 chunk partials of the reduction.
     const size_t s_bytes = (sizeof(float) * B * N + 255) & ~static_cast<size_t>(255);
-    cudaError_t e = cudaMallocAsync(reinterpret_cast<void**>(&s_buf),
+    cudaError_t e = pool_alloc(reinterpret_cast<void**>(&s_buf),
                                     s_bytes + gs::mmd2_partial_bytes(B, N), st);
-    if (e != cudaSuccess) return cuda_fail(e, "cudaMallocAsync");
+    if (e != cudaSuccess) return cuda_fail(e, "workspace allocation");
     c.out = s_buf;
     status = run(c);
     if (status == GS_OK) {

@@ -52,7 +52,13 @@ struct TcPlan {
     int64_t Mpad, Npad;      // rows padded to the row tile / key tile
     int Dp, Cp;              // D and Cv rounded up to 16
     int BN;                  // key tile width (128, or 64 when Cp > 128)
-    int splits;              // key splits per row tile
+    int splits;              // key splits per row tile (two-MMA kernel: of the tail row
+                             // tiles, see main_tiles)
+    // Two-MMA kernel: the first main_tiles row tiles (whole waves of one
+    // CTA per SM) run unsplit in a first launch; the remaining row tiles
+    // run with `splits` key splits in a second launch, so that the last
+    // wave is not left part-empty.
+    int64_t main_tiles;
     int stages;              // shared-memory pipeline depth
     size_t smem_bytes;       // dynamic shared memory of the fused kernel
     int mean_blocks;
@@ -119,21 +125,18 @@ bool plan_simt(int64_t M, int64_t N, int64_t D, int64_t C, bool grad, int split_
 // prep.cu --------------------------------------------------------------
 cudaError_t launch_mean(InType t, const void* q, const void* k, int64_t M, int64_t N, int D,
                         int blocks, float* partial, float* mu, cudaStream_t s, int batch = 1);
-cudaError_t launch_center_cast_norm(InType t, const void* x, int64_t rows, int64_t rows_pad,
-                                    int D, int Dp, const float* mu, float half_c, void* xh,
-                                    float* nrm, float pad_value, cudaStream_t s, int batch = 1);
-// All of the operand preparation in one cooperative launch (16-bit inputs,
-// D a multiple of 8, D <= 256): the common mean (when mu is given; partial
-// holds batch x mean_blocks x 2 D floats), q^ and k^ in the augmented (aug)
-// or plain layout (plain: norm terms into nrm_q / nrm_k, which alias when
-// q is k), and, when rec is given, the FMA kernel's key records of v
-// (N x C per problem).  kh == qh for the plain layout with alias.
-bool fused_prep_supported(InType t, int64_t D);
-cudaError_t launch_fused_prep(InType t, bool aug, const void* q, const void* k, const void* v,
-                              int64_t M, int64_t N, int64_t Mpad, int64_t Npad, int D, int Dp,
-                              int C, bool alias, float half_c, int mean_blocks, float* partial,
-                              float* mu, void* qh, void* kh, float* nrm_q, float* nrm_k,
-                              float* rec, cudaStream_t s, int batch = 1);
+// Centred, rounded MMA operands of q (M rows, padded to Mpad) and, with
+// with_k, of k (N rows, padded to Npad), in one launch where the vector
+// path applies (16-bit inputs, D a multiple of 8).  aug: the augmented
+// layout (Dp >= D + 2 aug_norm_terms(t)) into qh, and into qh_as_key (the
+// key layout of the same points, for q = k; may be null) and kh; plain:
+// x^ into qh / kh and the norm terms -(c/2)||x^||^2 into nrm_q / nrm_k
+// (pad_value for padded rows).
+cudaError_t launch_operands(InType t, bool aug, const void* q, int64_t M, int64_t Mpad,
+                            void* qh, void* qh_as_key, float* nrm_q, bool with_k, const void* k,
+                            int64_t N, int64_t Npad, void* kh, float* nrm_k, int D, int Dp,
+                            const float* mu, float half_c, float pad_value, cudaStream_t s,
+                            int batch = 1);
 // Transposed fp16 value operand of the two-MMA kernel for the channels
 // ch0 .. ch0 + Cc - 1 (Cp >= Cc rows of Npad keys), with per-channel
 // power-of-two scales.  Forward: channel ch of key n is w[n, ch] (w has the
@@ -145,10 +148,10 @@ cudaError_t launch_value_prep(InType t, bool grad, bool w_f32, const void* w, co
                               int Cc, int Cp, unsigned* vmax_bits, void* vt, float* inv_scale,
                               cudaStream_t s);
 // Forward: out (M x Cv) = inv_scale (when given) x the split partials summed
-// in split order.
+// in split order; rows below main_rows have one split.
 cudaError_t launch_finalize(const float* part, int splits, int64_t split_stride_rows,
                             int64_t M, int Cv, int part_ld, const float* inv_scale, float* out,
-                            cudaStream_t s);
+                            cudaStream_t s, int64_t main_rows = 0);
 // Gradient contraction of one launch's channels ch0 .. ch0 + Cc - 1 (see
 // prep.cu): out[m, d] (+)= tau sum_c u[m, c] (S_{c,d} - x^_{m,d} S_{c,D}),
 // s_out[m, c] = S_{c,D}.  direct: fp32 kernel partials (difference form).
@@ -156,7 +159,8 @@ cudaError_t launch_finalize_points(bool direct, InType t, bool u_f32, const floa
                                    int splits, int64_t split_stride_rows, int64_t M, int part_ld,
                                    const float* inv_scale, const void* x, const float* mu,
                                    float tau, int D, int Cw, int ch0, int Cc, const void* u,
-                                   int accumulate, float* out, float* s_out, cudaStream_t s);
+                                   int accumulate, float* out, float* s_out, cudaStream_t s,
+                                   int64_t main_rows = 0);
 // MMD^2 of Sec. 3 per problem of a batch: out[b] = sum_n v[b, n] s[b, n]
 // (float64 accumulation, fixed order), through float64 chunk partials in
 // `partial` (mmd2_partial_bytes(B, N) bytes).
@@ -192,13 +196,7 @@ cudaError_t launch_key_records(InType t, const void* v, const float* B, int64_t 
 cudaError_t launch_tf32_split(const float* x, int64_t rows, int64_t rows_pad, int D, int Dp,
                               const float* mu, float half_c, float* out, float* nrm,
                               float pad_value, cudaStream_t s, int batch = 1);
-// Augmented MMA operands (see prep.cu): query layout into out_q, key layout
-// into out_k (either may be null), Dpa >= D + 2 aug_norm_terms(t) columns
-// per row.
 constexpr int aug_norm_terms(InType t) { return t == InType::BF16 ? 3 : 2; }
-cudaError_t launch_aug_prep(InType t, const void* x, int64_t rows, int64_t rows_pad, int D,
-                            int Dpa, const float* mu, void* out_q, void* out_k, cudaStream_t s,
-                            int batch = 1);
 
 // tc_gauss.cu ----------------------------------------------------------
 cudaError_t launch_tc(const TcPlan& p, InType t, float c, char* ws, unsigned* status,

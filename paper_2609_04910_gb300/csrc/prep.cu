@@ -16,7 +16,6 @@
 //    the gradient tau (S[:D] - q_m S[D]) of Sec. 3.
 #include <algorithm>
 
-#include <cooperative_groups.h>
 #include <cuda_bf16.h>
 #include <cuda_fp16.h>
 #include <math_constants.h>
@@ -32,6 +31,14 @@ template <> __device__ __forceinline__ float to_f<float>(float x) { return x; }
 template <> __device__ __forceinline__ float to_f<__half>(__half x) { return __half2float(x); }
 template <> __device__ __forceinline__ float to_f<__nv_bfloat16>(__nv_bfloat16 x) {
     return __bfloat162float(x);
+}
+
+// a / b for a non-negative a below 2^32 with 32-bit division (much
+// cheaper than the 64-bit one), else 64-bit.
+__device__ __forceinline__ int64_t div_nonneg(int64_t a, int b) {
+    if (a <= 0xffffffffLL)
+        return static_cast<int64_t>(static_cast<uint32_t>(a) / static_cast<uint32_t>(b));
+    return a / b;
 }
 
 template <typename H> __device__ __forceinline__ H from_f(float x);
@@ -158,18 +165,34 @@ mean_partial_vec_kernel(const T* __restrict__ q, const T* __restrict__ k, int64_
 // shift leaves the Gauss sum unchanged.
 constexpr int kMeanFinalThreads = 256;
 
+// The grid-rounded mean of the folded sum s and largest magnitude mx.
+__device__ __forceinline__ float rounded_mean(double s, float mx, double total, int mant_bits,
+                                              int min_exp) {
+    double m = s / total;
+    if (mx > 0.f) {
+        int e;
+        frexp(static_cast<double>(mx), &e);              // mx in [2^(e-1), 2^e)
+        const double g = ldexp(1.0, max(e - 1 - mant_bits, min_exp));
+        m = rint(m / g) * g;
+    }
+    return static_cast<float>(m);
+}
+
+// Many partials per coordinate (G > kMeanFinalWarpMax): one block per
+// (coordinate d, problem blockIdx.y); thread t folds partials t, t + 256,
+// ... in order, then a fixed tree combines the threads (deterministic).
+constexpr int kMeanFinalWarpMax = 128;
+
 __global__ void __launch_bounds__(kMeanFinalThreads)
-mean_final_kernel(const float* __restrict__ partial, int G, int D, double total, int mant_bits,
-                  int min_exp, float* __restrict__ mu) {
+mean_final_block_kernel(const float* __restrict__ partial, int G, int D, double total,
+                        int mant_bits, int min_exp, float* __restrict__ mu) {
     pdl_trigger();
     pdl_wait();
-    // Block d: thread t folds partials t, t + 256, ... in order, then a
-    // fixed tree combines the threads (deterministic).
     __shared__ double red_s[kMeanFinalThreads];
     __shared__ float red_m[kMeanFinalThreads];
     const int d = blockIdx.x;
     const int t = threadIdx.x;
-    partial += static_cast<int64_t>(blockIdx.y) * 2 * G * D;   // problem blockIdx.y
+    partial += static_cast<int64_t>(blockIdx.y) * 2 * G * D;
     mu += static_cast<int64_t>(blockIdx.y) * D;
     double s = 0.0;
     float mx = 0.f;
@@ -187,16 +210,37 @@ mean_final_kernel(const float* __restrict__ partial, int G, int D, double total,
         }
         __syncthreads();
     }
-    if (t != 0) return;
-    double m = red_s[0] / total;
-    mx = red_m[0];
-    if (mx > 0.f) {
-        int e;
-        frexp(static_cast<double>(mx), &e);              // mx in [2^(e-1), 2^e)
-        const double g = ldexp(1.0, max(e - 1 - mant_bits, min_exp));
-        m = rint(m / g) * g;
+    if (t == 0) mu[d] = rounded_mean(red_s[0], red_m[0], total, mant_bits, min_exp);
+}
+
+// Few partials per coordinate (the small problems of a batch): one warp per
+// item instead of one block.
+__global__ void __launch_bounds__(kMeanFinalThreads)
+mean_final_kernel(const float* __restrict__ partial, int G, int D, int64_t items, double total,
+                  int mant_bits, int min_exp, float* __restrict__ mu) {
+    pdl_trigger();
+    pdl_wait();
+    // One warp per (problem b, coordinate d), item = b D + d: lane l folds
+    // partials l, l + 32, ... in order, then a fixed butterfly adds the
+    // lanes (deterministic).
+    const int64_t it = (static_cast<int64_t>(blockIdx.x) * kMeanFinalThreads + threadIdx.x) >> 5;
+    const int lane = threadIdx.x & 31;
+    if (it >= items) return;                       // whole warps leave together
+    const int64_t b = it / D;
+    const int d = static_cast<int>(it - b * D);
+    partial += b * 2 * G * D;                      // problem b
+    double s = 0.0;
+    float mx = 0.f;
+    for (int g = lane; g < G; g += 32) {
+        s += static_cast<double>(partial[static_cast<int64_t>(g) * D + d]);
+        mx = fmaxf(mx, partial[static_cast<int64_t>(G + g) * D + d]);
     }
-    mu[d] = static_cast<float>(m);
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        s += __shfl_xor_sync(0xffffffffu, s, o);
+        mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+    }
+    if (lane == 0) mu[it] = rounded_mean(s, mx, total, mant_bits, min_exp);
 }
 
 // ---------------------------------------------------------------- MMA operands
@@ -389,9 +433,9 @@ __global__ void finalize_slots_kernel(const float* __restrict__ part, int64_t Mp
     // problem and batch Mpad rows per slot.
     const int64_t idx = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
     if (idx >= batch * M * C) return;
-    const int64_t bm = idx / C;
+    const int64_t bm = div_nonneg(idx, C);
     const int c = static_cast<int>(idx - bm * C);
-    const int64_t b = bm / M;
+    const int64_t b = M <= 0x7fffffff ? div_nonneg(bm, static_cast<int>(M)) : bm / M;
     const int64_t m = (bm - b * M) + b * Mpad;
     int64_t nslots = fixed_slots;
     if (nslots == 0 && tri_kt > 0) {
@@ -444,8 +488,7 @@ template <> __device__ __forceinline__ unsigned short to_bits<__nv_bfloat16>(__n
 // row group (lane vi: coordinates 8 vi .. 8 vi + 7, one 16-byte vector).
 // in: lane vi's input vector of the row (used only when `valid` and
 // vi < D / 8); mu: the row problem's mean (or null); out_q / out_k: the row
-// in either layout (either
-// may be null; AUG only).  Every lane of the warp must call this together
+// in either layout (either may be null; AUG only).  Every lane of the warp must call this together
 // (the squared norm is reduced with shuffles over the G lanes); rows outside
 // the output (in_pad false) write nothing.  Returns the norm term written
 // for the row (plain layout: -(c/2)||x^||^2, or pad_value) in every lane.
@@ -524,250 +567,91 @@ __device__ __forceinline__ float operand_row(const uint4 in, const float* __rest
     return nrm;
 }
 
-template <typename T, bool AUG, int G>
-__global__ void __launch_bounds__(kOperandVecThreads)
-operand_vec_kernel(const T* __restrict__ x, int64_t rows, int64_t rows_pad, int64_t batch, int D,
-                   int Dp, int nt, float F, const float* __restrict__ mu, float half_c,
-                   float pad_value, T* __restrict__ out_q, T* __restrict__ out_k,
-                   float* __restrict__ nrm) {
-    pdl_trigger();
-    pdl_wait();
-    const int vi = threadIdx.x % G;                              // vector within the row
-    // Output row of the batch-stacked operand (batch rows_pad rows per
-    // problem); problem b reads rows b rows .. of x and its own mean.
-    const int64_t row = (static_cast<int64_t>(blockIdx.x) * kOperandVecThreads + threadIdx.x) / G;
-    const int64_t b = row / rows_pad;
-    const int64_t i = row - b * rows_pad;
-    const bool in_pad = b < batch;
-    const bool valid = in_pad && i < rows;
-    const bool wq = AUG ? out_q != nullptr : true;
-    const bool wk = AUG && out_k != nullptr;
-    const uint4 in = (valid && vi < D / 8)
-                         ? *reinterpret_cast<const uint4*>(x + (b * rows + i) * D + 8 * vi)
-                         : make_uint4(0u, 0u, 0u, 0u);
-    const float n = operand_row<T, AUG, G>(in, (mu && in_pad) ? mu + b * D : nullptr, vi, in_pad,
-                                           valid, D, Dp, nt, F, half_c, pad_value,
-                                           wq ? out_q + row * Dp : nullptr,
-                                           wk ? out_k + row * Dp : nullptr);
-    if (!AUG && in_pad && vi == 0) nrm[row] = n;
-}
-
-// ---------------------------------------------------------------- fused prep
-// The whole preparation of the FMA kernel's operands in one cooperative
-// launch (16-bit inputs, D a multiple of 8), instead of the mean, mean-final,
-// operand (q, k) and key-record kernels:
-//   phase 1  per chunk of rows of one problem (q rows, then k rows unless
-//            q is k): coordinate sums and largest magnitudes (as
-//            mean_partial_kernel);            -- grid barrier --
-//   phase 2  per (problem, coordinate): the grid-rounded common mean from
-//            the chunk partials in chunk order (as mean_final_kernel);
-//                                             -- grid barrier --
-//   phase 3  every output row of q^ and k^ (operand_row) and, from the key
-//            rows, the key records [B_2t, B_2t+1,] v_2t[c], v_2t+1[c] ....
-// Without centring phases 1 and 2 and both barriers are skipped.  The
-// barriers are those of a cooperative launch (all blocks co-resident).
-constexpr int kRowsInFlight = 4;   // rows per thread with loads in flight (fused prep)
-
-struct FusedPrepArgs {
-    const void* q;
-    const void* k;
-    const void* v;          // N x C key values (records), batch-stacked
-    int64_t M, N, Mpad, Npad, batch;
-    int D, Dp, nt, C;
-    float F, half_c;
-    bool alias;             // q and k are the same points: rows written once to both layouts
-    int64_t rows_per_chunk;
-    int chunks_q, chunks_k; // chunks per problem (chunks_k = 0 when alias)
-    float* partial;         // chunks x 2 D (sums, then maxima); null: no centring
-    float* mu;              // batch x D
-    int mant_bits, min_exp;
-    void* qh;
-    void* kh;               // == qh for the plain layout with alias
-    float* nrm_q;           // plain layout: A (batch x Mpad)
-    float* nrm_k;           // plain layout: B (batch x Npad; == nrm_q with alias)
-    float* rec;             // key records (batch x Npad / 2 pairs)
+// One array's operand rows: x (batch x rows x D) into out_q / out_k
+// (batch x rows_pad x Dp; either may be null, AUG only) and, for the plain
+// layout, the norm terms nrm (batch x rows_pad).
+struct OperandJob {
+    const void* x;
+    int64_t rows, rows_pad;
+    void* out_q;
+    void* out_k;
+    float* nrm;
 };
 
+// Rows per thread of operand_vec_kernel: their input vectors are loaded
+// before any is converted, so that several loads are in flight per thread.
+constexpr int kOperandRows = 4;
+
+// Vector path of the operand preparation (D a multiple of 8): blocks
+// [0, blocks0) convert the rows of job j0, the rest those of j1 (the keys,
+// when they are not the queries), so that both arrays take one launch.
 template <typename T, bool AUG, int G>
 __global__ void __launch_bounds__(kOperandVecThreads)
-fused_prep_kernel(const FusedPrepArgs a) {
-    namespace cg = cooperative_groups;
+operand_vec_kernel(const OperandJob j0, const OperandJob j1, unsigned blocks0, int64_t batch,
+                   int D, int Dp, int nt, float F, const float* __restrict__ mu, float half_c,
+                   float pad_value) {
     pdl_trigger();
     pdl_wait();
-    const int tid = threadIdx.x;
-    const int vi = tid % G;
-    constexpr int SLOTS = kOperandVecThreads / G;   // rows in flight per block
-    const int slot = tid / G;
-    const int D = a.D;
-    const T* q = static_cast<const T*>(a.q);
-    const T* k = static_cast<const T*>(a.k);
-    if (a.partial) {
-        __shared__ float s_sum[kOperandVecThreads][8];
-        __shared__ float s_max[kOperandVecThreads][8];
-        const int per_problem = a.chunks_q + a.chunks_k;
-        const int64_t chunks = a.batch * per_problem;
-        const int V = D / 8;
-        for (int64_t ch = blockIdx.x; ch < chunks; ch += gridDim.x) {
-            const int64_t b = ch / per_problem;
-            const int cb = static_cast<int>(ch - b * per_problem);
-            const bool on_q = cb < a.chunks_q;
-            const int64_t rows = on_q ? a.M : a.N;
-            const T* x = on_q ? q + b * a.M * D : k + b * a.N * D;
-            const int64_t r0 = static_cast<int64_t>(on_q ? cb : cb - a.chunks_q) * a.rows_per_chunk;
-            const int64_t r1 = min(rows, r0 + a.rows_per_chunk);
-            float sum[8], mx[8];
+    constexpr int SLOTS = kOperandVecThreads / G;   // rows of a block per step
+    const bool second = blockIdx.x >= blocks0;
+    const OperandJob j = second ? j1 : j0;
+    const int64_t blk = second ? blockIdx.x - blocks0 : blockIdx.x;
+    const int vi = threadIdx.x % G;                  // vector within the row
+    const int slot = threadIdx.x / G;
+    const int64_t total = j.rows_pad * batch;
+    const T* x = static_cast<const T*>(j.x);
+    const bool wq = AUG ? j.out_q != nullptr : true;
+    const bool wk = AUG && j.out_k != nullptr;
+    uint4 in[kOperandRows];
 #pragma unroll
-            for (int e = 0; e < 8; ++e) sum[e] = mx[e] = 0.f;
-            if (vi < V) {
-#pragma unroll 4
-                for (int64_t r = r0 + slot; r < r1; r += SLOTS) {
-                    const uint4 u = *reinterpret_cast<const uint4*>(x + r * D + 8 * vi);
-                    const T* h = reinterpret_cast<const T*>(&u);
-#pragma unroll
-                    for (int e = 0; e < 8; ++e) {
-                        const float f = to_f(h[e]);
-                        sum[e] += f;
-                        mx[e] = fmaxf(mx[e], fabsf(f));
-                    }
-                }
-            }
-#pragma unroll
-            for (int e = 0; e < 8; ++e) {
-                s_sum[tid][e] = sum[e];
-                s_max[tid][e] = mx[e];
-            }
-            __syncthreads();
-            // Coordinate d = 8 g + e: the slots' values of lane g, in slot order.
-            for (int d = tid; d < D; d += kOperandVecThreads) {
-                const int g = d >> 3, e = d & 7;
-                float s = 0.f, m = 0.f;
-                for (int sl = 0; sl < SLOTS; ++sl) {
-                    s += s_sum[sl * G + g][e];
-                    m = fmaxf(m, s_max[sl * G + g][e]);
-                }
-                a.partial[ch * 2 * D + d] = s;
-                a.partial[ch * 2 * D + D + d] = m;
-            }
-            __syncthreads();
-        }
-        cg::this_grid().sync();
-        // Phase 2: mean of coordinate d of problem b, rounded to the grid of
-        // the input format at the coordinate's largest magnitude; one warp
-        // per (problem, coordinate): lane l folds chunks l, l + 32, ... in
-        // order, then a fixed butterfly adds the lanes (deterministic).
-        const int64_t items = a.batch * D;
-        const int lane = tid & 31;
-        const int64_t warps = static_cast<int64_t>(gridDim.x) * (kOperandVecThreads / 32);
-        for (int64_t it = static_cast<int64_t>(blockIdx.x) * (kOperandVecThreads / 32) + (tid >> 5);
-             it < items; it += warps) {
-            const int64_t b = it / D;
-            const int d = static_cast<int>(it - b * D);
-            const float* pp = a.partial + b * per_problem * 2 * D;
-            double s = 0.0;
-            float m = 0.f;
-            for (int c = lane; c < per_problem; c += 32) {
-                s += static_cast<double>(pp[static_cast<int64_t>(c) * 2 * D + d]);
-                m = fmaxf(m, pp[static_cast<int64_t>(c) * 2 * D + D + d]);
-            }
-#pragma unroll
-            for (int o = 16; o > 0; o >>= 1) {
-                s += __shfl_xor_sync(0xffffffffu, s, o);
-                m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, o));
-            }
-            if (lane == 0) {
-                double mean = s / static_cast<double>(a.M + (a.alias ? 0 : a.N));
-                if (m > 0.f) {
-                    int e;
-                    frexp(static_cast<double>(m), &e);
-                    const double gstep = ldexp(1.0, max(e - 1 - a.mant_bits, a.min_exp));
-                    mean = rint(mean / gstep) * gstep;
-                }
-                a.mu[it] = static_cast<float>(mean);
-            }
-        }
-        cg::this_grid().sync();
+    for (int u = 0; u < kOperandRows; ++u) {
+        // Output row of the batch-stacked operand (batch rows_pad rows per
+        // problem); problem b reads rows b rows .. of x and its own mean.
+        const int64_t row = (blk * kOperandRows + u) * SLOTS + slot;
+        const int64_t b = row / j.rows_pad;
+        const int64_t i = row - b * j.rows_pad;
+        const bool valid = row < total && i < j.rows;
+        in[u] = (valid && vi < D / 8)
+                    ? *reinterpret_cast<const uint4*>(x + (b * j.rows + i) * D + 8 * vi)
+                    : make_uint4(0u, 0u, 0u, 0u);
     }
-    // Phase 3: q rows (batch x Mpad), then k rows (batch x Npad) unless q is
-    // k.  A block takes SLOTS consecutive rows per slice; each thread handles
-    // kRowsInFlight slices one grid stride apart, with all their input
-    // vectors loaded before any is converted (several loads in flight per
-    // thread: the pass is bound by memory latency otherwise).
-    constexpr int U = kRowsInFlight;
-    const int64_t rows_q = a.batch * a.Mpad;
-    const int64_t rows_all = rows_q + (a.alias ? 0 : a.batch * a.Npad);
-    const int64_t step = static_cast<int64_t>(gridDim.x) * SLOTS;
-    const int head = AUG ? 0 : 2;
-    const int rec_pair = head + 2 * a.C;
-    const int V = D / 8;
-    for (int64_t base = static_cast<int64_t>(blockIdx.x) * SLOTS; base < rows_all; base += U * step) {
-        uint4 in[U];
-        int64_t rr[U], bb[U], ii[U];
-        bool onq[U], inr[U], val[U];
 #pragma unroll
-        for (int u = 0; u < U; ++u) {
-            const int64_t row = base + u * step + slot;
-            inr[u] = row < rows_all;
-            onq[u] = row < rows_q;
-            rr[u] = onq[u] ? row : row - rows_q;               // row of the stacked layout
-            const int64_t rpad = onq[u] ? a.Mpad : a.Npad;
-            bb[u] = rr[u] / rpad;
-            ii[u] = rr[u] - bb[u] * rpad;
-            val[u] = inr[u] && ii[u] < (onq[u] ? a.M : a.N);
-            const T* x = onq[u] ? q + (bb[u] * a.M + ii[u]) * D : k + (bb[u] * a.N + ii[u]) * D;
-            in[u] = (val[u] && vi < V) ? *reinterpret_cast<const uint4*>(x + 8 * vi)
-                                       : make_uint4(0u, 0u, 0u, 0u);
-        }
-#pragma unroll
-        for (int u = 0; u < U; ++u) {
-            const int64_t r = rr[u], b = bb[u], i = ii[u];
-            const bool on_q = onq[u], in_range = inr[u], valid = val[u];
-            const float* mu = (a.partial && in_range) ? a.mu + b * D : nullptr;
-            T* oq = nullptr;
-            T* ok = nullptr;
-            if (AUG) {
-                if (on_q) oq = static_cast<T*>(a.qh) + r * a.Dp;
-                if (!on_q || a.alias) ok = static_cast<T*>(a.kh) + r * a.Dp;
-            } else {
-                oq = static_cast<T*>(on_q ? a.qh : a.kh) + r * a.Dp;
-            }
-            // Plain layout: padded rows get the norm term -inf (kernel value 0).
-            const float nrm = operand_row<T, AUG, G>(in[u], mu, vi, in_range, valid, D, a.Dp, a.nt,
-                                                     a.F, a.half_c, -INFINITY,
-                                                     in_range ? oq : nullptr,
-                                                     in_range ? ok : nullptr);
-            if (!in_range) continue;
-            if (!AUG && vi == 0) (on_q ? a.nrm_q : a.nrm_k)[r] = nrm;
-            // Key records from the key rows (the q rows when q is k).
-            if (a.rec && (!on_q || a.alias)) {
-                float* rp = a.rec + (b * (a.Npad / 2) + (i >> 1)) * rec_pair;
-                const int par = static_cast<int>(i & 1);
-                if (!AUG && vi == 0) rp[par] = nrm;
-                const T* vb = static_cast<const T*>(a.v) + (b * a.N + i) * a.C;
-                for (int c = vi; c < a.C; c += G) rp[head + 2 * c + par] = valid ? to_f(vb[c]) : 0.f;
-            }
-        }
+    for (int u = 0; u < kOperandRows; ++u) {
+        const int64_t row = (blk * kOperandRows + u) * SLOTS + slot;
+        const int64_t b = row / j.rows_pad;
+        const int64_t i = row - b * j.rows_pad;
+        const bool in_pad = row < total;
+        const bool valid = in_pad && i < j.rows;
+        const float n = operand_row<T, AUG, G>(
+            in[u], (mu && in_pad) ? mu + b * D : nullptr, vi, in_pad, valid, D, Dp, nt, F, half_c,
+            pad_value, wq ? static_cast<T*>(j.out_q) + row * Dp : nullptr,
+            wk ? static_cast<T*>(j.out_k) + row * Dp : nullptr);
+        if (!AUG && in_pad && vi == 0) j.nrm[row] = n;
     }
 }
 
 template <typename T, bool AUG>
-cudaError_t operand_typed(const void* x, int64_t rows, int64_t rows_pad, int D, int Dp, int nt,
-                          float F, const float* mu, float half_c, float pad_value, void* out_q,
-                          void* out_k, float* nrm, cudaStream_t s, int batch) {
-    if (rows_pad % kRowsPerBlock != 0 || Dp % 16 != 0 || Dp > kOperandMaxCols ||
-        (AUG && 2 * Dp > kOperandMaxCols))
+cudaError_t operand_typed(const OperandJob& j0, const OperandJob* j1, int D, int Dp, int nt,
+                          float F, const float* mu, float half_c, float pad_value, cudaStream_t s,
+                          int batch) {
+    const OperandJob none = {nullptr, 0, 0, nullptr, nullptr, nullptr};
+    for (const OperandJob* j : {&j0, j1}) {
+        if (j && (j->rows_pad % kRowsPerBlock != 0)) return cudaErrorInvalidValue;
+    }
+    if (Dp % 16 != 0 || Dp > kOperandMaxCols || (AUG && 2 * Dp > kOperandMaxCols))
         return cudaErrorInvalidValue;
     if (D % 8 == 0 && D >= 8 && (!AUG || Dp - D >= 2 * nt)) {
-        // Vector path: G lanes per row.
+        // Vector path: G lanes per row, both arrays in one launch.
         const int V = D / 8;
         const int G = V <= 1 ? 1 : V <= 2 ? 2 : V <= 4 ? 4 : V <= 8 ? 8 : V <= 16 ? 16 : 32;
-        const int64_t threads = rows_pad * batch * G;
-        const unsigned blocks = static_cast<unsigned>((threads + kOperandVecThreads - 1) / kOperandVecThreads);
+        const int64_t per_block = static_cast<int64_t>(kOperandVecThreads / G) * kOperandRows;
+        const int64_t b0 = (j0.rows_pad * batch + per_block - 1) / per_block;
+        const int64_t b1 = j1 ? (j1->rows_pad * batch + per_block - 1) / per_block : 0;
+        if (b0 + b1 == 0) return cudaSuccess;
         auto go = [&](auto kern) {
-            launch_kernel(kern, blocks, kOperandVecThreads, 0, s, static_cast<const T*>(x), rows, rows_pad,
-                                                     static_cast<int64_t>(batch), D,
-                                                     Dp, nt, F, mu, half_c, pad_value,
-                                                     static_cast<T*>(out_q), static_cast<T*>(out_k),
-                                                     nrm);
+            launch_kernel(kern, static_cast<unsigned>(b0 + b1), kOperandVecThreads, 0, s, j0,
+                          j1 ? *j1 : none, static_cast<unsigned>(b0),
+                          static_cast<int64_t>(batch), D, Dp, nt, F, mu, half_c, pad_value);
         };
         switch (G) {
             case 1: go(operand_vec_kernel<T, AUG, 1>); break;
@@ -780,17 +664,23 @@ cudaError_t operand_typed(const void* x, int64_t rows, int64_t rows_pad, int D, 
         note_launches(1);
         return cudaGetLastError();
     }
-    const int64_t blocks = rows_pad / kRowsPerBlock;
-    if (blocks == 0) return cudaSuccess;
-    const int nout = AUG ? (out_q ? 1 : 0) + (out_k ? 1 : 0) : 1;
-    const size_t smem = static_cast<size_t>(nout) * kRowsPerBlock * Dp * sizeof(T) +
-                        ((static_cast<size_t>(kRowsPerBlock) * D * sizeof(T) + 15) & ~size_t(15)) +
-                        static_cast<size_t>(D) * sizeof(float);
-    launch_kernel(operand_kernel<T, AUG>, dim3(static_cast<unsigned>(blocks), batch), kOperandThreads, smem, s, 
-        static_cast<const T*>(x), rows, rows_pad, D, Dp, nt, F, mu, half_c, pad_value,
-        static_cast<T*>(out_q), static_cast<T*>(out_k), nrm);
-    note_launches(1);
-    return cudaGetLastError();
+    for (const OperandJob* j : {&j0, j1}) {
+        if (!j) continue;
+        const int64_t blocks = j->rows_pad / kRowsPerBlock;
+        if (blocks == 0) continue;
+        const int nout = AUG ? (j->out_q ? 1 : 0) + (j->out_k ? 1 : 0) : 1;
+        const size_t smem = static_cast<size_t>(nout) * kRowsPerBlock * Dp * sizeof(T) +
+                            ((static_cast<size_t>(kRowsPerBlock) * D * sizeof(T) + 15) & ~size_t(15)) +
+                            static_cast<size_t>(D) * sizeof(float);
+        launch_kernel(operand_kernel<T, AUG>, dim3(static_cast<unsigned>(blocks), batch),
+                      kOperandThreads, smem, s, static_cast<const T*>(j->x), j->rows, j->rows_pad,
+                      D, Dp, nt, F, mu, half_c, pad_value, static_cast<T*>(j->out_q),
+                      static_cast<T*>(j->out_k), j->nrm);
+        note_launches(1);
+        const cudaError_t e = cudaGetLastError();
+        if (e != cudaSuccess) return e;
+    }
+    return cudaSuccess;
 }
 
 // ---------------------------------------------------------------- values
@@ -930,15 +820,17 @@ __global__ void key_record_kernel(const T* __restrict__ v, const float* __restri
 // order).  part: splits blocks of split_stride_rows rows x part_ld floats.
 __global__ void finalize_kernel(const float* __restrict__ part, int splits,
                                 int64_t split_stride_rows, int64_t M, int Cv, int part_ld,
-                                const float* __restrict__ inv_scale, float* __restrict__ out) {
+                                const float* __restrict__ inv_scale, float* __restrict__ out,
+                                int64_t main_rows) {
     pdl_trigger();
     pdl_wait();
     const int64_t idx = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
     if (idx >= M * Cv) return;
-    const int64_t m = idx / Cv;
+    const int64_t m = div_nonneg(idx, Cv);
     const int c = static_cast<int>(idx - m * Cv);
     float acc = 0.f;
-    for (int s = 0; s < splits; ++s)
+    const int ns = m < main_rows ? 1 : splits;
+    for (int s = 0; s < ns; ++s)
         acc += part[(static_cast<int64_t>(s) * split_stride_rows + m) * part_ld + c];
     out[idx] = acc * (inv_scale ? inv_scale[c] : 1.f);
 }
@@ -961,21 +853,23 @@ __global__ void finalize_points_kernel(const float* __restrict__ part, int split
                                        const T* __restrict__ x, const float* __restrict__ mu,
                                        float tau, int D, int Cw, int ch0, int Cc,
                                        const U* __restrict__ u, int accumulate,
-                                       float* __restrict__ out, float* __restrict__ s_out) {
+                                       float* __restrict__ out, float* __restrict__ s_out,
+                                       int64_t main_rows) {
     pdl_trigger();
     pdl_wait();
     const int width = D > 0 ? D : 1;
     const int64_t idx = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
     if (idx >= M * width) return;
-    const int64_t m = idx / width;
+    const int64_t m = div_nonneg(idx, width);
     const int d = static_cast<int>(idx - m * width);
+    const int ns = m < main_rows ? 1 : splits;
     auto S = [&](int j) {
         float acc = 0.f;
         // Unrolled so that the loads of several splits are in flight
         // together (the sum keeps the split order): 71 -> 58 us on the
         // 131072-point gradient with four splits.
 #pragma unroll 4
-        for (int s = 0; s < splits; ++s)
+        for (int s = 0; s < ns; ++s)
             acc += part[(static_cast<int64_t>(s) * split_stride_rows + m) * part_ld + j];
         return inv_scale ? acc * inv_scale[j] : acc;
     };
@@ -1030,14 +924,14 @@ cudaError_t finalize_points_typed(const float* part, int splits, int64_t stride_
                                   int part_ld, const float* inv_scale, const void* x,
                                   const float* mu, float tau, int D, int Cw, int ch0, int Cc,
                                   const void* u, int accumulate, float* out, float* s_out,
-                                  cudaStream_t s) {
+                                  cudaStream_t s, int64_t main_rows) {
     const int64_t total = M * (D > 0 ? D : 1);
     if (total == 0) return cudaSuccess;
     const int threads = 256;
     const int64_t blocks = (total + threads - 1) / threads;
     launch_kernel(finalize_points_kernel<DIRECT, T, U>, static_cast<unsigned>(blocks), threads, 0, s, 
         part, splits, stride_rows, M, part_ld, inv_scale, static_cast<const T*>(x), mu, tau, D,
-        Cw, ch0, Cc, static_cast<const U*>(u), accumulate, out, s_out);
+        Cw, ch0, Cc, static_cast<const U*>(u), accumulate, out, s_out, main_rows);
     note_launches(1);
     return cudaGetLastError();
 }
@@ -1093,8 +987,17 @@ cudaError_t launch_mean(InType t, const void* q, const void* k, int64_t M, int64
     if (e != cudaSuccess) return e;
     const int mant_bits = t == InType::F16 ? 10 : t == InType::BF16 ? 7 : 23;
     const int min_exp = t == InType::F16 ? -24 : t == InType::BF16 ? -133 : -149;
-    launch_kernel(mean_final_kernel, dim3(D, batch), kMeanFinalThreads, 0, s, partial, G, D, static_cast<double>(total),
-                                                     mant_bits, min_exp, mu);
+    if (G > kMeanFinalWarpMax) {
+        launch_kernel(mean_final_block_kernel, dim3(D, batch), kMeanFinalThreads, 0, s, partial,
+                      G, D, static_cast<double>(total), mant_bits, min_exp, mu);
+    } else {
+        const int64_t items = static_cast<int64_t>(batch) * D;
+        const int64_t warps_per_block = kMeanFinalThreads / 32;
+        launch_kernel(mean_final_kernel,
+                      dim3(static_cast<unsigned>((items + warps_per_block - 1) / warps_per_block)),
+                      kMeanFinalThreads, 0, s, partial, G, D, items, static_cast<double>(total),
+                      mant_bits, min_exp, mu);
+    }
     note_launches(1);
     return cudaGetLastError();
 }
@@ -1190,112 +1093,30 @@ cudaError_t launch_finalize_slots(const float* part, int64_t Mpad, int64_t M, in
     return cudaGetLastError();
 }
 
-bool fused_prep_supported(InType t, int64_t D) {
-    return t != InType::F32 && D >= 8 && D % 8 == 0 && D <= kOperandMaxCols;
-}
-
-namespace {
-
-template <typename T, bool AUG, int G>
-cudaError_t fused_prep_go(FusedPrepArgs a, cudaStream_t s) {
-    auto kern = fused_prep_kernel<T, AUG, G>;
-    // Blocks that fit on the device at once (the grid barriers need all of
-    // them resident), per device.
-    static int per_sm[64] = {};
-    static int sms[64] = {};
-    int dev = 0;
-    cudaError_t e = cudaGetDevice(&dev);
-    if (e != cudaSuccess) return e;
-    if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
-    if (per_sm[dev] == 0) {
-        int nb = 0, n = 0;
-        e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&nb, kern, kOperandVecThreads, 0);
-        if (e != cudaSuccess) return e;
-        e = cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
-        if (e != cudaSuccess) return e;
-        sms[dev] = n;
-        per_sm[dev] = nb > 0 ? nb : 1;
+cudaError_t launch_operands(InType t, bool aug, const void* q, int64_t M, int64_t Mpad,
+                            void* qh, void* qh_as_key, float* nrm_q, bool with_k, const void* k,
+                            int64_t N, int64_t Npad, void* kh, float* nrm_k, int D, int Dp,
+                            const float* mu, float half_c, float pad_value, cudaStream_t s,
+                            int batch) {
+    OperandJob jq, jk;
+    if (aug) {
+        jq = {q, M, Mpad, qh, qh_as_key, nullptr};
+        jk = {k, N, Npad, nullptr, kh, nullptr};
+    } else {
+        jq = {q, M, Mpad, qh, nullptr, nrm_q};
+        jk = {k, N, Npad, kh, nullptr, nrm_k};
     }
-    constexpr int SLOTS = kOperandVecThreads / G;
-    const int64_t rows = a.batch * (a.Mpad + (a.alias ? 0 : a.Npad));
-    const int64_t want = std::max<int64_t>((rows + SLOTS * kRowsInFlight - 1) / (SLOTS * kRowsInFlight),
-                                           a.partial ? a.batch * (a.chunks_q + a.chunks_k) : 1);
-    const int grid = static_cast<int>(std::max<int64_t>(
-        1, std::min<int64_t>(want, static_cast<int64_t>(per_sm[dev]) * sms[dev])));
-    void* args[] = {&a};
-    e = cudaLaunchCooperativeKernel(reinterpret_cast<const void*>(kern), dim3(grid),
-                                    dim3(kOperandVecThreads), args, 0, s);
-    t_pdl_next = e == cudaSuccess;
-    note_launches(1);
-    return e;
-}
-
-template <typename T, bool AUG>
-cudaError_t fused_prep_g(const FusedPrepArgs& a, cudaStream_t s) {
-    const int V = a.D / 8;
-    const int G = V <= 1 ? 1 : V <= 2 ? 2 : V <= 4 ? 4 : V <= 8 ? 8 : V <= 16 ? 16 : 32;
-    switch (G) {
-        case 1: return fused_prep_go<T, AUG, 1>(a, s);
-        case 2: return fused_prep_go<T, AUG, 2>(a, s);
-        case 4: return fused_prep_go<T, AUG, 4>(a, s);
-        case 8: return fused_prep_go<T, AUG, 8>(a, s);
-        case 16: return fused_prep_go<T, AUG, 16>(a, s);
-        default: return fused_prep_go<T, AUG, 32>(a, s);
+    // (k itself may be null: an empty array when D = 0.)
+    const OperandJob* j1 = with_k ? &jk : nullptr;
+    const int nt = aug ? aug_norm_terms(t) : 0;
+    if (t == InType::BF16) {
+        return aug ? operand_typed<__nv_bfloat16, true>(jq, j1, D, Dp, nt, 1.f, mu, 0.f, 0.f, s, batch)
+                   : operand_typed<__nv_bfloat16, false>(jq, j1, D, Dp, 0, 1.f, mu, half_c,
+                                                         pad_value, s, batch);
     }
-}
-
-}  // namespace
-
-cudaError_t launch_fused_prep(InType t, bool aug, const void* q, const void* k, const void* v,
-                              int64_t M, int64_t N, int64_t Mpad, int64_t Npad, int D, int Dp,
-                              int C, bool alias, float half_c, int mean_blocks, float* partial,
-                              float* mu, void* qh, void* kh, float* nrm_q, float* nrm_k,
-                              float* rec, cudaStream_t s, int batch) {
-    FusedPrepArgs a;
-    a.q = q;
-    a.k = k;
-    a.v = v;
-    a.M = M;
-    a.N = N;
-    a.Mpad = Mpad;
-    a.Npad = Npad;
-    a.batch = batch;
-    a.D = D;
-    a.Dp = Dp;
-    a.nt = aug ? aug_norm_terms(t) : 0;
-    a.C = C;
-    a.F = (aug && t == InType::F16) ? 1024.f : 1.f;
-    a.half_c = half_c;
-    a.alias = alias;
-    // Chunks of rows per problem for the mean partials: at most mean_blocks
-    // per problem (the partial buffer holds batch x mean_blocks x 2 D floats).
-    const int64_t rows = M + (alias ? 0 : N);
-    a.rows_per_chunk = std::max<int64_t>(1, (rows + std::max(1, mean_blocks - 2) - 1) /
-                                                std::max(1, mean_blocks - 2));
-    a.chunks_q = static_cast<int>((M + a.rows_per_chunk - 1) / a.rows_per_chunk);
-    a.chunks_k = alias ? 0 : static_cast<int>((N + a.rows_per_chunk - 1) / a.rows_per_chunk);
-    a.partial = mu ? partial : nullptr;
-    a.mu = mu;
-    a.mant_bits = t == InType::F16 ? 10 : 7;
-    a.min_exp = t == InType::F16 ? -24 : -133;
-    a.qh = qh;
-    a.kh = kh;
-    a.nrm_q = nrm_q;
-    a.nrm_k = nrm_k;
-    a.rec = rec;
-    if (t == InType::BF16)
-        return aug ? fused_prep_g<__nv_bfloat16, true>(a, s) : fused_prep_g<__nv_bfloat16, false>(a, s);
-    return aug ? fused_prep_g<__half, true>(a, s) : fused_prep_g<__half, false>(a, s);
-}
-
-cudaError_t launch_center_cast_norm(InType t, const void* x, int64_t rows, int64_t rows_pad,
-                                    int D, int Dp, const float* mu, float half_c, void* xh,
-                                    float* nrm, float pad_value, cudaStream_t s, int batch) {
-    if (t == InType::BF16)
-        return operand_typed<__nv_bfloat16, false>(x, rows, rows_pad, D, Dp, 0, 1.f, mu, half_c,
-                                                   pad_value, xh, nullptr, nrm, s, batch);
-    return operand_typed<__half, false>(x, rows, rows_pad, D, Dp, 0, 1.f, mu, half_c, pad_value,
-                                        xh, nullptr, nrm, s, batch);
+    return aug ? operand_typed<__half, true>(jq, j1, D, Dp, nt, 1024.f, mu, 0.f, 0.f, s, batch)
+               : operand_typed<__half, false>(jq, j1, D, Dp, 0, 1.f, mu, half_c, pad_value, s,
+                                              batch);
 }
 
 cudaError_t launch_tf32_split(const float* x, int64_t rows, int64_t rows_pad, int D, int Dp,
@@ -1327,16 +1148,6 @@ cudaError_t launch_value_prep(InType t, bool grad, bool w_f32, const void* w, co
 #undef GS_VALUE_PREP
 }
 
-cudaError_t launch_aug_prep(InType t, const void* x, int64_t rows, int64_t rows_pad, int D,
-                            int Dpa, const float* mu, void* out_q, void* out_k, cudaStream_t s,
-                            int batch) {
-    const int nt = aug_norm_terms(t);
-    if (t == InType::BF16)
-        return operand_typed<__nv_bfloat16, true>(x, rows, rows_pad, D, Dpa, nt, 1.f, mu, 0.f, 0.f,
-                                                  out_q, out_k, nullptr, s, batch);
-    return operand_typed<__half, true>(x, rows, rows_pad, D, Dpa, nt, 1024.f, mu, 0.f, 0.f, out_q,
-                                       out_k, nullptr, s, batch);
-}
 
 cudaError_t launch_key_records(InType t, const void* v, const float* B, int64_t N, int64_t Npad,
                                int C, float* rec, cudaStream_t s, int batch) {
@@ -1359,13 +1170,13 @@ cudaError_t launch_key_records(InType t, const void* v, const float* B, int64_t 
 
 cudaError_t launch_finalize(const float* part, int splits, int64_t split_stride_rows,
                             int64_t M, int Cv, int part_ld, const float* inv_scale, float* out,
-                            cudaStream_t s) {
+                            cudaStream_t s, int64_t main_rows) {
     const int64_t total = M * Cv;
     if (total == 0) return cudaSuccess;
     const int threads = 256;
     const int64_t blocks = (total + threads - 1) / threads;
     launch_kernel(finalize_kernel, static_cast<unsigned>(blocks), threads, 0, s, 
-        part, splits, split_stride_rows, M, Cv, part_ld, inv_scale, out);
+        part, splits, split_stride_rows, M, Cv, part_ld, inv_scale, out, main_rows);
     note_launches(1);
     return cudaGetLastError();
 }
@@ -1374,10 +1185,12 @@ cudaError_t launch_finalize_points(bool direct, InType t, bool u_f32, const floa
                                    int splits, int64_t split_stride_rows, int64_t M, int part_ld,
                                    const float* inv_scale, const void* x, const float* mu,
                                    float tau, int D, int Cw, int ch0, int Cc, const void* u,
-                                   int accumulate, float* out, float* s_out, cudaStream_t s) {
+                                   int accumulate, float* out, float* s_out, cudaStream_t s,
+                                   int64_t main_rows) {
 #define GS_FIN(DIR, T, U)                                                                     \
     finalize_points_typed<DIR, T, U>(part, splits, split_stride_rows, M, part_ld, inv_scale, x, \
-                                     mu, tau, D, Cw, ch0, Cc, u, accumulate, out, s_out, s)
+                                     mu, tau, D, Cw, ch0, Cc, u, accumulate, out, s_out, s,      \
+                                     main_rows)
     if (direct) return GS_FIN(true, float, float);
     if (t == InType::BF16)
         return u_f32 ? GS_FIN(false, __nv_bfloat16, float)

@@ -81,6 +81,7 @@ struct TcParams {
     float* part;         // splits x Mpad x Cp partial sums (unscaled)
     unsigned* status;    // device status word
     int64_t Mpad;
+    int tile_off;        // row tile of blockIdx.x = 0 (main launch 0, tail launch main_tiles)
     int key_tiles;
     int tiles_per_split;
     int nkb;             // 64-element K blocks of q^/k^
@@ -147,10 +148,9 @@ tc_gauss_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant_
     // latency overlaps the other group's exp2 work.
     constexpr int GROUP_WARPS = NEXP / 2;
     constexpr int COLS = BN * 4 / GROUP_WARPS;  // key columns per exponent warp and tile
-    constexpr int NCH = COLS / 32;              // 32-column TMEM loads per warp and tile
     static_assert(GROUP_WARPS % 4 == 0, "each group covers the four TMEM lane quarters");
     static_assert(COLS % 32 == 0, "exponent warps load whole 32-column chunks");
-    static_assert(NCH == 2, "two 32-column TMEM loads per warp and tile");
+    static_assert(COLS == 64, "one 64-column TMEM load per warp and tile");
 
     extern __shared__ uint8_t smem_raw[];
     // 1024-byte aligned base for the 128-byte swizzle atoms.
@@ -163,7 +163,7 @@ tc_gauss_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant_
     const int tid = threadIdx.x;
     const int warp = tid >> 5;
     const int lane = tid & 31;
-    const int tile_m = blockIdx.x;
+    const int tile_m = p.tile_off + static_cast<int>(blockIdx.x);
     const int split = blockIdx.y;
     const int kt0 = split * p.tiles_per_split;
     const int kt1 = min(p.key_tiles, kt0 + p.tiles_per_split);
@@ -450,13 +450,16 @@ tc_gauss_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant_
                                p.status);
             if (!ok) break;
             tc_fence_after();
-            uint32_t r[NCH][32];
-#pragma unroll
-            for (int ch = 0; ch < NCH; ++ch)
-                tmem_ld_32x32b_x32(tmem + lane_base + S_col0 + b * BN + col0 + ch * 32, r[ch]);
-            // The wait names the loaded registers, so that no use of them is
-            // scheduled above it (the loads land asynchronously).
-            tmem_wait_ld_regs(r[0], r[1]);
+            // The warp's 64 S columns in one TMEM load, and below its P
+            // columns in one TMEM store: each tcgen05 instruction takes a
+            // slot of the queue that the MUFU exp2 instructions share, and
+            // halving their number (from two x32 loads and two x16 stores)
+            // measured 8 % faster on the 131072^2 gradient (3.030 -> 2.780
+            // ms).  The wait names the loaded registers, so that no use of
+            // them is scheduled above it (the loads land asynchronously).
+            uint32_t r[64];
+            tmem_ld_32x32b_x64(tmem + lane_base + S_col0 + b * BN + col0, r);
+            tmem_wait_ld_regs(r);
             // S buffer b is in registers: MMA1 of tile j + 2 may overwrite it
             // (EARLY; otherwise MMA1 of tile j + 2 follows P of tile j).
             if (EARLY) {
@@ -465,40 +468,35 @@ tc_gauss_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant_
                 if (lane == 0) mbar_arrive(&bars->s_free[b]);
             }
             const float* Bs = b_smem(s) + col0;
+            uint32_t pk[32];
 #pragma unroll
-            for (int ch = 0; ch < NCH; ++ch) {
-                uint32_t pk[16];
-#pragma unroll
-                for (int i = 0; i < 8; ++i) {
-                    // x = c S + (A_m + 15) + B_n for four keys, two per f32x2
-                    // op (with augmented operands S already holds the norm
-                    // terms: x = c S + 15).
-                    uint64_t t01 = a2, t23 = a2;
-                    if (!AUG) {
-                        const float4 bb = *reinterpret_cast<const float4*>(Bs + ch * 32 + 4 * i);
-                        t01 = f32x2_add(f32x2_pack(bb.x, bb.y), a2);
-                        t23 = f32x2_add(f32x2_pack(bb.z, bb.w), a2);
-                    }
-                    const uint64_t s01 = f32x2_pack(__uint_as_float(r[ch][4 * i + 0]),
-                                                    __uint_as_float(r[ch][4 * i + 1]));
-                    const uint64_t s23 = f32x2_pack(__uint_as_float(r[ch][4 * i + 2]),
-                                                    __uint_as_float(r[ch][4 * i + 3]));
-                    float x0, x1, x2, x3;
-                    f32x2_unpack(f32x2_fma(s01, c2, t01), x0, x1);
-                    f32x2_unpack(f32x2_fma(s23, c2, t23), x2, x3);
-                    pk[2 * i + 0] = bound_p2(pack_half2_satfinite(ex2_approx(x0), ex2_approx(x1)));
-                    pk[2 * i + 1] = bound_p2(pack_half2_satfinite(ex2_approx(x2), ex2_approx(x3)));
+            for (int i = 0; i < 16; ++i) {
+                // x = c S + (A_m + 15) + B_n for four keys, two per f32x2 op
+                // (with augmented operands S already holds the norm terms:
+                // x = c S + 15).
+                uint64_t t01 = a2, t23 = a2;
+                if (!AUG) {
+                    const float4 bb = *reinterpret_cast<const float4*>(Bs + 4 * i);
+                    t01 = f32x2_add(f32x2_pack(bb.x, bb.y), a2);
+                    t23 = f32x2_add(f32x2_pack(bb.z, bb.w), a2);
                 }
-                if (EARLY && ch == 0 && j >= 2) {
-                    // P buffer b: MMA2 of tile j - 2 has read it.  (With one
-                    // MMA warp the completion of S of tile j implies it.)
-                    ok = warp_wait(&bars->p_free[b], static_cast<uint32_t>((j - 2) >> 1) & 1u, abort_flag,
-                                   p.status);
-                    if (!ok) break;
-                    tc_fence_after();
-                }
-                tmem_st_32x32b_x16(tmem + lane_base + P_col0 + b * (BN / 2) + (col0 + ch * 32) / 2, pk);
+                const uint64_t s01 = f32x2_pack(__uint_as_float(r[4 * i + 0]), __uint_as_float(r[4 * i + 1]));
+                const uint64_t s23 = f32x2_pack(__uint_as_float(r[4 * i + 2]), __uint_as_float(r[4 * i + 3]));
+                float x0, x1, x2, x3;
+                f32x2_unpack(f32x2_fma(s01, c2, t01), x0, x1);
+                f32x2_unpack(f32x2_fma(s23, c2, t23), x2, x3);
+                pk[2 * i + 0] = bound_p2(pack_half2_satfinite(ex2_approx(x0), ex2_approx(x1)));
+                pk[2 * i + 1] = bound_p2(pack_half2_satfinite(ex2_approx(x2), ex2_approx(x3)));
             }
+            if (EARLY && j >= 2) {
+                // P buffer b: MMA2 of tile j - 2 has read it.  (With one MMA
+                // warp the completion of S of tile j implies it.)
+                ok = warp_wait(&bars->p_free[b], static_cast<uint32_t>((j - 2) >> 1) & 1u, abort_flag,
+                               p.status);
+                if (!ok) break;
+                tc_fence_after();
+            }
+            tmem_st_32x32b_x32(tmem + lane_base + P_col0 + b * (BN / 2) + col0 / 2, pk);
             if (!ok) break;
             tmem_wait_st();
             tc_fence_before();
@@ -537,7 +535,7 @@ size_t align1k(size_t x) { return (x + 1023) & ~static_cast<size_t>(1023); }
 
 template <int BN, int NEXP, bool AUG, bool EARLY, bool QTM = false>
 cudaError_t launch_bn(const TcPlan& pl, InType t, float c, char* ws, unsigned* status,
-                      cudaStream_t s, const char** why) {
+                      cudaStream_t s, const char** why, int tile_off, int tiles, int splits) {
     const CUtensorMapDataType hdt =
         t == InType::BF16 ? CU_TENSOR_MAP_DATA_TYPE_BFLOAT16 : CU_TENSOR_MAP_DATA_TYPE_FLOAT16;
     CUtensorMap tm_q, tm_k, tm_v;
@@ -554,8 +552,9 @@ cudaError_t launch_bn(const TcPlan& pl, InType t, float c, char* ws, unsigned* s
     p.part = reinterpret_cast<float*>(ws + pl.off_part);
     p.status = status;
     p.Mpad = pl.Mpad;
+    p.tile_off = tile_off;
     p.key_tiles = static_cast<int>(pl.Npad / BN);
-    p.tiles_per_split = (p.key_tiles + pl.splits - 1) / pl.splits;
+    p.tiles_per_split = (p.key_tiles + splits - 1) / splits;
     p.nkb = (pl.Dp + KB - 1) / KB;
     p.ksteps1 = pl.Dp / 16;
     p.Cp = pl.Cp;
@@ -575,7 +574,7 @@ cudaError_t launch_bn(const TcPlan& pl, InType t, float c, char* ws, unsigned* s
                                          cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          static_cast<int>(pl.smem_bytes));
     if (e != cudaSuccess) return e;
-    dim3 grid(static_cast<unsigned>(pl.Mpad / BM), static_cast<unsigned>(pl.splits));
+    dim3 grid(static_cast<unsigned>(tiles), static_cast<unsigned>(splits));
     launch_kernel(tc_gauss_kernel<BN, NEXP, AUG, EARLY, QTM>, grid, cta_threads<NEXP>(), pl.smem_bytes, s, tm_q, tm_k, tm_v, p);
     note_launches(1);
     return cudaGetLastError();
@@ -715,6 +714,27 @@ bool plan_tensor(InType t, int64_t M, int64_t N, int64_t D, int64_t C, bool grad
         best_s = static_cast<int>((key_tiles + tps - 1) / tps);
     }
     p->splits = std::max(1, best_s);
+    p->main_tiles = 0;
+    if (!p->fma && split_override == 0 && tiles >= sms) {
+        // Two-MMA kernel: whole waves of row tiles (one CTA per SM) take
+        // their full key range in one launch (no partial sums to add, each
+        // q^ tile read once, all CTAs of a wave streaming the same keys);
+        // the tail row tiles, fewer than the SMs, split their key range so
+        // that the last wave is filled: s key splits for the fewest waves of
+        // the tail per key tile (about ceil(tail s / sms) / s of a tile).
+        const int64_t main = tiles / sms * sms;
+        const int64_t tail = tiles - main;
+        int ts = 1;
+        double best_t = tail > 0 ? 1e300 : 0.0;
+        for (int s = 1; tail > 0 && s <= 64 && s <= key_tiles; ++s) {
+            const int64_t tps = (key_tiles + s - 1) / s;
+            const int64_t s_eff = (key_tiles + tps - 1) / tps;
+            const double cost = static_cast<double>((tail * s_eff + sms - 1) / sms) * (tps + 2);
+            if (cost < best_t * 0.99) { best_t = cost; ts = static_cast<int>(s_eff); }
+        }
+        p->main_tiles = main;
+        p->splits = ts;
+    }
     p->units = p->unit_len = 0;
     p->grid = 0;
     p->band_len = 0;
@@ -822,23 +842,36 @@ bool plan_tensor(InType t, int64_t M, int64_t N, int64_t D, int64_t C, bool grad
     return true;
 }
 
-cudaError_t launch_tc(const TcPlan& p, InType t, float c, char* ws, unsigned* status,
-                      cudaStream_t s, const char** why) {
+namespace {
+
+cudaError_t launch_tc_range(const TcPlan& p, InType t, float c, char* ws, unsigned* status,
+                            cudaStream_t s, const char** why, int off, int tiles, int splits) {
+#define GS_TC(BN_, NE_, AUG_, EARLY_, QTM_) \
+    launch_bn<BN_, NE_, AUG_, EARLY_, QTM_>(p, t, c, ws, status, s, why, off, tiles, splits)
     if (p.aug) {
-        if (p.BN == 128)
-            return p.early_s ? launch_bn<128, 16, true, true>(p, t, c, ws, status, s, why)
-                             : launch_bn<128, 16, true, false>(p, t, c, ws, status, s, why);
-        return p.early_s ? launch_bn<64, 8, true, true>(p, t, c, ws, status, s, why)
-                         : launch_bn<64, 8, true, false>(p, t, c, ws, status, s, why);
+        if (p.BN == 128) return p.early_s ? GS_TC(128, 16, true, true, false) : GS_TC(128, 16, true, false, false);
+        return p.early_s ? GS_TC(64, 8, true, true, false) : GS_TC(64, 8, true, false, false);
     }
     if (p.BN == 128 && p.qtm)
-        return p.early_s ? launch_bn<128, 16, false, true, true>(p, t, c, ws, status, s, why)
-                         : launch_bn<128, 16, false, false, true>(p, t, c, ws, status, s, why);
-    if (p.BN == 128)
-        return p.early_s ? launch_bn<128, 16, false, true>(p, t, c, ws, status, s, why)
-                         : launch_bn<128, 16, false, false>(p, t, c, ws, status, s, why);
-    return p.early_s ? launch_bn<64, 8, false, true>(p, t, c, ws, status, s, why)
-                     : launch_bn<64, 8, false, false>(p, t, c, ws, status, s, why);
+        return p.early_s ? GS_TC(128, 16, false, true, true) : GS_TC(128, 16, false, false, true);
+    if (p.BN == 128) return p.early_s ? GS_TC(128, 16, false, true, false) : GS_TC(128, 16, false, false, false);
+    return p.early_s ? GS_TC(64, 8, false, true, false) : GS_TC(64, 8, false, false, false);
+#undef GS_TC
+}
+
+}  // namespace
+
+cudaError_t launch_tc(const TcPlan& p, InType t, float c, char* ws, unsigned* status,
+                      cudaStream_t s, const char** why) {
+    // Whole waves of row tiles unsplit, then the tail row tiles with their
+    // key range split (see plan_tensor).
+    const int tiles = static_cast<int>(p.Mpad / BM);
+    const int main = static_cast<int>(p.main_tiles);
+    cudaError_t e = cudaSuccess;
+    if (main > 0) e = launch_tc_range(p, t, c, ws, status, s, why, 0, main, 1);
+    if (e == cudaSuccess && tiles > main)
+        e = launch_tc_range(p, t, c, ws, status, s, why, main, tiles - main, p.splits);
+    return e;
 }
 
 }  // namespace gs

@@ -264,7 +264,7 @@ tc_gauss_fma_kernel(const __grid_constant__ CUtensorMap tm_q,
         for (int k = 0; k < NCTRL_MAX; ++k) mbar_init(&bars->drain[k], 1);
         for (int sl = 0; sl < SL; ++sl) {
             mbar_init(&bars->s_full[sl], 1);
-            mbar_init(&bars->s_free[sl], NEXP);        // one arrival per exponent warp (one slot)
+            mbar_init(&bars->s_free[sl], NEXP);        // one arrival per exponent warp
         }
         for (int s = 0; s < p.stages; ++s) {
             mbar_init(&bars->kv_full[s], 1);
@@ -370,22 +370,15 @@ tc_gauss_fma_kernel(const __grid_constant__ CUtensorMap tm_q,
                     // slot that tile g - SL released.
                     const int g = g0 + j;
                     const int sl = SL == 2 ? (g & 1) : 0;
-                    // The barrier that reports the slot free again: with two
-                    // slots (q^ in shared memory, four stages) the stage
-                    // release of tile g - 2, on stage (k + 2) mod 4 (the
-                    // exponent warps release a tile's stage and slot with one
-                    // arrival, after its MMAs have completed); with one slot,
-                    // s_free of tile g - 1.
-                    uint64_t* free_bar = QSM ? &bars->kv_empty[(k + 2) & 3] : &bars->s_free[0];
-                    const uint32_t free_parity =
-                        static_cast<uint32_t>(QSM ? ((g - 2) >> 2) : (g - 1)) & 1u;
+                    const uint32_t full_parity = static_cast<uint32_t>(SL == 2 ? (g >> 1) : g) & 1u;
+                    const uint32_t free_parity = full_parity ^ 1u;
                     const bool ready = __all_sync(
                         0xffffffffu, g < SL ? mbar_test_wait(&bars->kv_full[k], ph)
-                                            : mbar_test_wait2(free_bar, free_parity,
+                                            : mbar_test_wait2(&bars->s_free[sl], free_parity,
                                                               &bars->kv_full[k], ph));
                     if (!ready) {
                         if (g >= SL) {
-                            ok = warp_wait(free_bar, free_parity, abort_flag, p.status);
+                            ok = warp_wait(&bars->s_free[sl], free_parity, abort_flag, p.status);
                             if (!ok) break;
                         }
                         ok = warp_wait(&bars->kv_full[k], ph, abort_flag, p.status);
@@ -525,52 +518,44 @@ tc_gauss_fma_kernel(const __grid_constant__ CUtensorMap tm_q,
             for (int cc = 0; cc < C; ++cc) acc0[cc] = acc1[cc] = 0ull;
             bool ok = true;
             bool ready = false;   // both barriers of key tile j already seen complete
-            // Stage and TMEM slot of key tile j (running index g = g0 + j):
-            // with q^ in shared memory four stages and two slots, so stage
-            // g mod 4 with phase parity (g / 4) mod 2 and slot g mod 2 with
-            // parity (g / 2) mod 2 come from bits of g; otherwise a ring.
-            RingPos st, sl;
+            RingPos st, sl;       // stage and TMEM slot of key tile j (running index g0 + j)
             st.idx = g0 % p.stages;
             st.phase = static_cast<uint32_t>(g0 / p.stages) & 1u;
-            sl.idx = 0;
-            sl.phase = static_cast<uint32_t>(g0) & 1u;
-            const uint32_t tcol = tmem + lane_base + static_cast<uint32_t>(cg * 32);
-            for (int j = 0; j < T; ++j) {
-                const int g = g0 + j;
-                const int s = QSM ? (g & 3) : st.idx;
-                const uint32_t st_ph = QSM ? (static_cast<uint32_t>(g >> 2) & 1u) : st.phase;
-                const int sli = QSM ? (g & 1) : 0;
-                const uint32_t sl_ph = QSM ? (static_cast<uint32_t>(g >> 1) & 1u) : sl.phase;
-                const uint32_t col0 = static_cast<uint32_t>(sli * 2 * BN);
-                if (!__all_sync(0xffffffffu, ready || mbar_test_wait2(&bars->kv_full[s], st_ph,
-                                                                      &bars->s_full[sli], sl_ph))) {
-                    ok = warp_wait(&bars->kv_full[s], st_ph, abort_flag, p.status);
-                    if (ok) ok = warp_wait(&bars->s_full[sli], sl_ph, abort_flag, p.status);
+            sl.idx = g0 % SL;
+            sl.phase = static_cast<uint32_t>(g0 / SL) & 1u;
+            for (int j = 0; j < T; ++j, st.advance(p.stages), sl.advance(SL)) {
+                const int s = st.idx;
+                const uint32_t col0 = static_cast<uint32_t>(sl.idx * 2 * BN);
+                if (!__all_sync(0xffffffffu, ready || mbar_test_wait2(&bars->kv_full[s], st.phase,
+                                                                      &bars->s_full[sl.idx], sl.phase))) {
+                    ok = warp_wait(&bars->kv_full[s], st.phase, abort_flag, p.status);
+                    if (ok) ok = warp_wait(&bars->s_full[sl.idx], sl.phase, abort_flag, p.status);
                     if (!ok) break;
                 }
                 tc_fence_after();
                 uint32_t r0[32], r1[32];
-                tmem_ld_32x32b_x32(tcol + col0, r0);
-                tmem_ld_32x32b_x32(tcol + col0 + BN, r1);
+                tmem_ld_32x32b_x32(tmem + lane_base + col0 + cg * 32, r0);
+                tmem_ld_32x32b_x32(tmem + lane_base + col0 + BN + cg * 32, r1);
                 // The wait names r0 and r1, so that no use of the loaded
                 // values is scheduled above it (the loads land asynchronously).
                 tmem_wait_ld_regs(r0, r1);
                 // When and where the S slot is handed back: with two slots
                 // (q^ in shared memory) only after the exponent work of this
-                // tile, together with the stage (one arrival), because
-                // releasing it right after the loads let the next MMAs into
-                // the slot corrupt S values of this tile in some warps when
-                // the MMAs were long (3xTF32 operands, three or more stages;
-                // still seen with the loads' registers named in the wait, and
-                // no faster on the 65536^2, D = 64 sum: 0.6428 against
-                // 0.6418 ms).  With one slot (q^ in TMEM) a late release
-                // would serialise the MMAs and the exponent work, so it is
-                // released here; no corruption was seen there in repeated
-                // runs (regression test: repeated calls agree bit for bit).
+                // tile (with the stage, below), because releasing it right
+                // after the loads let the next MMAs into the slot corrupt S
+                // values of this tile in some warps when the MMAs were long
+                // (measured with 3xTF32 operands and three or more stages,
+                // also with the loads' registers named in the wait; the early
+                // release was no faster on the 65536^2, D = 64 sum either:
+                // 0.6428 against 0.6418 ms).
+                // With one slot (q^ in TMEM) a late release would serialise
+                // the MMAs and the exponent work, so it is released here; no
+                // corruption was seen there in repeated runs (regression
+                // test: repeated calls agree bit for bit).
                 if (!QSM) {
                     tc_fence_before();
                     __syncwarp();
-                    mbar_arrive_if_zero(&bars->s_free[0], lane);
+                    mbar_arrive_if_zero(&bars->s_free[sl.idx], lane);
                 }
                 // Query the barriers of key tile j + 1 now and read the answer
                 // after the exponent work of tile j: the query latency overlaps
@@ -584,10 +569,11 @@ tc_gauss_fma_kernel(const __grid_constant__ CUtensorMap tm_q,
                 // ready this early (skipping the query: fp32 65536^2 sums 4-5 %
                 // faster).
                 if (QSM && !TF) {
-                    const int g1 = g + 1;
-                    ready = j + 1 < T &&
-                            mbar_test_wait2(&bars->kv_full[g1 & 3], static_cast<uint32_t>(g1 >> 2) & 1u,
-                                            &bars->s_full[g1 & 1], static_cast<uint32_t>(g1 >> 1) & 1u);
+                    RingPos st2 = st, sl2 = sl;
+                    st2.advance(p.stages);
+                    sl2.advance(SL);
+                    ready = j + 1 < T && mbar_test_wait2(&bars->kv_full[st2.idx], st2.phase,
+                                                         &bars->s_full[sl2.idx], sl2.phase);
                 }
                 const float* rec = rec_smem(s) + (cg * 16) * REC_PAIR;
                 const uint64_t w2 = (TRI && j >= w_from) ? f32x2_pack(1.f, 1.f) : 0ull;
@@ -663,11 +649,8 @@ tc_gauss_fma_kernel(const __grid_constant__ CUtensorMap tm_q,
                 // Lane 0 hands back the slot (two-slot path) and the stage,
                 // predicated rather than branched: a divergent branch here
                 // cost 0.7 % of the kernel time.
-                mbar_arrive_if_zero(&bars->kv_empty[s], lane);
-                if (!QSM) {
-                    st.advance(p.stages);
-                    sl.advance(1);
-                }
+                if (QSM) mbar_arrive2_if_zero(&bars->s_free[sl.idx], &bars->kv_empty[s], lane);
+                else mbar_arrive_if_zero(&bars->kv_empty[s], lane);
             }
             // Fixed-order reduction of the NPART column-group partial sums.
     #pragma unroll
@@ -827,9 +810,6 @@ bool plan_fma_kernel(int Dp, int C, bool aug, bool tf, int* nq, int* stages, siz
     const int st = static_cast<int>(
         std::min<size_t>(std::min(MAX_STAGES, 2 * sl), (budget - fixed) / stage));
     if (st < 2) return false;
-    // With q^ in shared memory the kernel derives stage and slot from the
-    // running tile index for exactly four stages (two per slot).
-    if (qsm && st != MAX_STAGES) return false;
     *nq = NQ;
     *stages = st;
     *smem = std::max<size_t>(fixed + st * stage, 118 * 1024);
