@@ -42,3 +42,23 @@ def test_sample_rows():
     r = sample_rows(1000, 10)
     assert len(r) == 10 and len(set(r.tolist())) == 10 and np.all(np.diff(r) > 0)
     assert np.array_equal(sample_rows(5, 10), np.arange(5))
+
+
+def test_fp16_kernel_value_floor_never_binds_on_the_two_mma_workloads():
+    """The two-MMA kernel stores each kernel value as fp16(2^(x + 15)), so
+    values below 2^-29 lose precision (2^-39 and below flush to zero).  A row
+    whose largest kernel value fell below that floor would have all of its
+    terms there; on the two workloads that take this kernel (multi_c64,
+    svgd_d32) the largest kernel value of every sampled row is far above it,
+    so a per-row exponent offset (a row maximum before the exponentials)
+    would change nothing there."""
+    floor = 2.0 ** -29
+    for name in ("multi_c64", "svgd_d32"):
+        w = WORKLOADS[name]
+        g = generate(w, seed=0)
+        rows = sample_rows(w.M, 48, seed=5)
+        q = g["q64"][rows]
+        k = g["k64"]
+        d2 = ((q * q).sum(1)[:, None] - 2.0 * q @ k.T + (k * k).sum(1)[None, :])
+        phi_max = np.exp(-0.5 * w.tau * np.maximum(d2.min(axis=1), 0.0))
+        assert phi_max.min() > 2.0 ** 10 * floor, (name, phi_max.min())
