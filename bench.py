@@ -57,6 +57,10 @@ def parse_args(argv=None):
     ap.add_argument("--no-other-workloads", action="store_true",
                     help="skip timing the other four configurations")
     ap.add_argument("--no-peak-probe", action="store_true")
+    ap.add_argument("--batched", action="store_true",
+                    help="time gauss_sum_batched on the paper's benchmark shapes "
+                         "(B = 64 clouds of 16384 points, D = 16..128) and smaller "
+                         "batches; one JSON line per case, instead of the step")
     return ap.parse_args(argv)
 
 
@@ -589,10 +593,72 @@ def run_own(args):
     return 0
 
 
+BATCHED_CASES = ((64, 16384, 16), (64, 16384, 32), (64, 16384, 64), (64, 16384, 128),
+                 (4, 65536, 64), (64, 4096, 64), (256, 1024, 64))
+
+
+def run_batched(args):
+    """gauss_sum_batched on the benchmark shape of Sec. 4 (B independent
+    Gaussian clouds, M = N = n points each, C = 1, fp16, tau = 1/D): 3
+    warm-up calls, then 8 timed calls (the paper's protocol), each after an
+    L2 flush, CUDA events around the whole call.  The roofline is the
+    slower of the dense tensor work 2 B n^2 (D + 1) at the measured bf16
+    peak and the B n^2 exponentials at the MUFU rate."""
+    import torch
+    from paper_2609_04910_gb300.build import build_library
+    build_library()
+    import paper_2609_04910_gb300 as gs
+    from paper_2609_04910_gb300.workloads import batched_clouds, to_device
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    peaks, peak_src = measured_peaks()
+    sms = torch.cuda.get_device_properties(dev).multi_processor_count
+    r_x = 32.0 * sms * float(peaks.get("sm_max_mhz", 2070.0)) * 1e6
+    r_t = float(peaks.get("bf16_tflops", FALLBACK_PEAKS["bf16_tflops"])) * 1e12
+    flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=dev)
+    stream = torch.cuda.current_stream()
+    sampler = ClockSampler(0, enabled=not args.no_clocks)
+    for B, n, D in BATCHED_CASES:
+        inp = batched_clouds(B, n, D)
+        q, k, v = (to_device(inp[x], "fp16", dev) for x in ("q", "k", "v"))
+        out = torch.empty((B, n, 1), dtype=torch.float32, device=dev)
+        for _ in range(3):
+            gs.gauss_sum_batched(q, k, v, inp["tau"], out=out)
+        torch.cuda.synchronize()
+        ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+              for _ in range(8)]
+        for a, b in ev:
+            flush.zero_()
+            a.record(stream)
+            gs.gauss_sum_batched(q, k, v, inp["tau"], out=out)
+            b.record(stream)
+        torch.cuda.synchronize()
+        gs.gauss_sum_device_status()
+        ms = [a.elapsed_time(b) for a, b in ev]
+        t = statistics.mean(ms) * 1e-3
+        pairs = float(B) * n * n
+        t_x, t_t = pairs / r_x, 2.0 * pairs * (D + 1) / r_t
+        print(json.dumps({
+            "case": f"batched B={B} M=N={n} D={D} C=1 fp16", "B": B, "n": n, "D": D,
+            "ms_mean": statistics.mean(ms), "ms_std": statistics.pstdev(ms), "ms_min": min(ms),
+            "pairs_per_s": pairs / t, "tflops": 2.0 * pairs * (D + 1) / t / 1e12,
+            "bound": "alu" if t_x >= t_t else "tensor", "roofline_frac": max(t_x, t_t) / t,
+            "ex2_frac": t_x / t, "tensor_frac": t_t / t,
+            "peaks": f"MUFU 32/clk/SM x {sms} SMs at max clock; {peak_src} bf16 {r_t / 1e12:.1f} TFLOP/s",
+            "l2": "flushed (512 MiB write) before every timed call", "timing": "whole call, CUDA events"}),
+            flush=True)
+        del q, k, v, out
+        torch.cuda.empty_cache()
+    clocks = sampler.stop() if sampler is not None else None
+    print(json.dumps({"batched_clocks": clocks}), flush=True)
+
+
 def main(argv=None):
     args = parse_args(argv)
     if args.impl == "reference":
         return run_reference(args)
+    if args.batched:
+        return run_batched(args)
     return run_own(args)
 
 

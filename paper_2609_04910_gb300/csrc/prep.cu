@@ -125,8 +125,9 @@ mean_partial_vec_kernel(const T* __restrict__ q, const T* __restrict__ k, int64_
     float sum[8], mx[8];
 #pragma unroll
     for (int e = 0; e < 8; ++e) sum[e] = mx[e] = 0.f;
-    for (int64_t v = v0 + t; v < v1; v += kMeanVecThreads) {
-        const uint4 u = xv[v];
+    // Four vectors in flight per thread, then the remainder one at a time
+    // (each thread's vectors are accumulated in index order either way).
+    auto add = [&](const uint4 u) {
         const T* h = reinterpret_cast<const T*>(&u);
 #pragma unroll
         for (int e = 0; e < 8; ++e) {
@@ -134,7 +135,16 @@ mean_partial_vec_kernel(const T* __restrict__ q, const T* __restrict__ k, int64_
             sum[e] += f;
             mx[e] = fmaxf(mx[e], fabsf(f));
         }
+    };
+    int64_t v = v0 + t;
+    for (; v + 3 * kMeanVecThreads < v1; v += 4 * kMeanVecThreads) {
+        uint4 u[4];
+#pragma unroll
+        for (int r = 0; r < 4; ++r) u[r] = xv[v + r * kMeanVecThreads];
+#pragma unroll
+        for (int r = 0; r < 4; ++r) add(u[r]);
     }
+    for (; v < v1; v += kMeanVecThreads) add(xv[v]);
 #pragma unroll
     for (int e = 0; e < 8; ++e) {
         s_sum[t][e] = sum[e];
@@ -484,44 +494,71 @@ template <> __device__ __forceinline__ unsigned short to_bits<__nv_bfloat16>(__n
     return __bfloat16_as_ushort(h);
 }
 
+// Packed 16-bit pair arithmetic of the operand conversion.  x - mu of two
+// 16-bit inputs and a mean on the input grid (see rounded_mean), rounded
+// once to the input format (the MMA operand type), and the pair as floats.
+template <typename T> struct Pair;
+template <> struct Pair<__half> {
+    using P = __half2;
+    static __device__ __forceinline__ P sub(P a, P b) { return __hsub2(a, b); }
+    static __device__ __forceinline__ float2 to_f2(P a) { return __half22float2(a); }
+    static __device__ __forceinline__ P from_f2(float lo, float hi) { return __floats2half2_rn(lo, hi); }
+};
+template <> struct Pair<__nv_bfloat16> {
+    using P = __nv_bfloat162;
+    static __device__ __forceinline__ P sub(P a, P b) { return __hsub2(a, b); }
+    static __device__ __forceinline__ float2 to_f2(P a) { return __bfloat1622float2(a); }
+    static __device__ __forceinline__ P from_f2(float lo, float hi) { return __floats2bfloat162_rn(lo, hi); }
+};
+
+// The mean of coordinates 8 vi .. 8 vi + 7 as four packed pairs of the input
+// format (exact: the mean lies on the input grid), or zeros.
+template <typename T>
+__device__ __forceinline__ uint4 mean_pairs(const float* __restrict__ mu, int vi) {
+    using PT = Pair<T>;
+    if (!mu) return make_uint4(0u, 0u, 0u, 0u);
+    const float4 m0 = *reinterpret_cast<const float4*>(mu + 8 * vi);
+    const float4 m1 = *reinterpret_cast<const float4*>(mu + 8 * vi + 4);
+    typename PT::P p[4] = {PT::from_f2(m0.x, m0.y), PT::from_f2(m0.z, m0.w),
+                           PT::from_f2(m1.x, m1.y), PT::from_f2(m1.z, m1.w)};
+    return *reinterpret_cast<const uint4*>(p);
+}
+
 // One output row of the operand layouts, converted by the G lanes of a
 // row group (lane vi: coordinates 8 vi .. 8 vi + 7, one 16-byte vector).
 // in: lane vi's input vector of the row (used only when `valid` and
-// vi < D / 8); mu: the row problem's mean (or null); out_q / out_k: the row
-// in either layout (either may be null; AUG only).  Every lane of the warp must call this together
-// (the squared norm is reduced with shuffles over the G lanes); rows outside
-// the output (in_pad false) write nothing.  Returns the norm term written
-// for the row (plain layout: -(c/2)||x^||^2, or pad_value) in every lane.
+// vi < D / 8); m2: the row problem's mean pairs (mean_pairs); out_q /
+// out_k: the row in either layout (either may be null; AUG only).  Every
+// lane of the warp must call this together (the squared norm is reduced
+// with shuffles over the G lanes); rows outside the output (in_pad false)
+// write nothing.  Returns the norm term written for the row (plain layout:
+// -(c/2)||x^||^2, or pad_value) in every lane.
 template <typename T, bool AUG, int G>
-__device__ __forceinline__ float operand_row(const uint4 in, const float* __restrict__ mu, int vi,
+__device__ __forceinline__ float operand_row(const uint4 in, const uint4 m2, int vi,
                                              bool in_pad, bool valid, int D, int Dp, int nt,
                                              float F, float half_c, float pad_value,
                                              T* __restrict__ out_q, T* __restrict__ out_k) {
+    using PT = Pair<T>;
     const int V = D / 8;
     float acc = 0.f;
     if (in_pad && vi < V) {
         uint4 u = make_uint4(0u, 0u, 0u, 0u);
         if (valid) {
-            const unsigned short* hb = reinterpret_cast<const unsigned short*>(&in);
-            float m[8];
-            if (mu) {
-                const float4 m0 = *reinterpret_cast<const float4*>(mu + 8 * vi);
-                const float4 m1 = *reinterpret_cast<const float4*>(mu + 8 * vi + 4);
-                m[0] = m0.x; m[1] = m0.y; m[2] = m0.z; m[3] = m0.w;
-                m[4] = m1.x; m[5] = m1.y; m[6] = m1.z; m[7] = m1.w;
-            } else {
+            const typename PT::P* x2 = reinterpret_cast<const typename PT::P*>(&in);
+            const typename PT::P* mm = reinterpret_cast<const typename PT::P*>(&m2);
+            typename PT::P h[4];
+            uint64_t acc2 = 0ull;
 #pragma unroll
-                for (int e = 0; e < 8; ++e) m[e] = 0.f;
+            for (int e = 0; e < 4; ++e) {
+                h[e] = PT::sub(x2[e], mm[e]);
+                const float2 f = PT::to_f2(h[e]);
+                const uint64_t f2 = f32x2_pack(f.x, f.y);
+                acc2 = f32x2_fma(f2, f2, acc2);
             }
-            __align__(16) unsigned short ob[8];
-#pragma unroll
-            for (int e = 0; e < 8; ++e) {
-                const T h = from_f<T>(to_f(bits_to<T>(hb[e])) - m[e]);
-                const float hf = to_f(h);
-                acc = fmaf(hf, hf, acc);
-                ob[e] = to_bits(h);
-            }
-            u = *reinterpret_cast<const uint4*>(ob);
+            float lo, hi;
+            f32x2_unpack(acc2, lo, hi);
+            acc = lo + hi;
+            u = *reinterpret_cast<const uint4*>(h);
         }
         if (out_q) *reinterpret_cast<uint4*>(out_q + 8 * vi) = u;
         if (out_k) *reinterpret_cast<uint4*>(out_k + 8 * vi) = u;
@@ -585,9 +622,11 @@ constexpr int kOperandRows = 4;
 // Vector path of the operand preparation (D a multiple of 8): blocks
 // [0, blocks0) convert the rows of job j0, the rest those of j1 (the keys,
 // when they are not the queries), so that both arrays take one launch.
+// Index arithmetic is 32-bit (the planner keeps batch x rows_pad below
+// 2^31); with one problem the lane's mean pairs are loaded once.
 template <typename T, bool AUG, int G>
 __global__ void __launch_bounds__(kOperandVecThreads)
-operand_vec_kernel(const OperandJob j0, const OperandJob j1, unsigned blocks0, int64_t batch,
+operand_vec_kernel(const OperandJob j0, const OperandJob j1, unsigned blocks0, int batch,
                    int D, int Dp, int nt, float F, const float* __restrict__ mu, float half_c,
                    float pad_value) {
     pdl_trigger();
@@ -595,37 +634,43 @@ operand_vec_kernel(const OperandJob j0, const OperandJob j1, unsigned blocks0, i
     constexpr int SLOTS = kOperandVecThreads / G;   // rows of a block per step
     const bool second = blockIdx.x >= blocks0;
     const OperandJob j = second ? j1 : j0;
-    const int64_t blk = second ? blockIdx.x - blocks0 : blockIdx.x;
+    const int blk = static_cast<int>(second ? blockIdx.x - blocks0 : blockIdx.x);
     const int vi = threadIdx.x % G;                  // vector within the row
     const int slot = threadIdx.x / G;
-    const int64_t total = j.rows_pad * batch;
+    const int rows_pad = static_cast<int>(j.rows_pad);
+    const int rows = static_cast<int>(j.rows);
+    const int total = rows_pad * batch;
     const T* x = static_cast<const T*>(j.x);
     const bool wq = AUG ? j.out_q != nullptr : true;
     const bool wk = AUG && j.out_k != nullptr;
+    const uint4 m_one = (batch == 1 && vi < D / 8) ? mean_pairs<T>(mu, vi) : make_uint4(0u, 0u, 0u, 0u);
     uint4 in[kOperandRows];
 #pragma unroll
     for (int u = 0; u < kOperandRows; ++u) {
         // Output row of the batch-stacked operand (batch rows_pad rows per
         // problem); problem b reads rows b rows .. of x and its own mean.
-        const int64_t row = (blk * kOperandRows + u) * SLOTS + slot;
-        const int64_t b = row / j.rows_pad;
-        const int64_t i = row - b * j.rows_pad;
-        const bool valid = row < total && i < j.rows;
+        const int row = (blk * kOperandRows + u) * SLOTS + slot;
+        const int b = batch == 1 ? 0 : row / rows_pad;
+        const int i = row - b * rows_pad;
+        const bool valid = row < total && i < rows;
         in[u] = (valid && vi < D / 8)
-                    ? *reinterpret_cast<const uint4*>(x + (b * j.rows + i) * D + 8 * vi)
+                    ? *reinterpret_cast<const uint4*>(x + (static_cast<int64_t>(b) * rows + i) * D + 8 * vi)
                     : make_uint4(0u, 0u, 0u, 0u);
     }
 #pragma unroll
     for (int u = 0; u < kOperandRows; ++u) {
-        const int64_t row = (blk * kOperandRows + u) * SLOTS + slot;
-        const int64_t b = row / j.rows_pad;
-        const int64_t i = row - b * j.rows_pad;
+        const int row = (blk * kOperandRows + u) * SLOTS + slot;
+        const int b = batch == 1 ? 0 : row / rows_pad;
+        const int i = row - b * rows_pad;
         const bool in_pad = row < total;
-        const bool valid = in_pad && i < j.rows;
+        const bool valid = in_pad && i < rows;
+        const uint4 m2 = (batch == 1 || !(in_pad && vi < D / 8))
+                             ? m_one
+                             : mean_pairs<T>(mu ? mu + static_cast<int64_t>(b) * D : nullptr, vi);
         const float n = operand_row<T, AUG, G>(
-            in[u], (mu && in_pad) ? mu + b * D : nullptr, vi, in_pad, valid, D, Dp, nt, F, half_c,
-            pad_value, wq ? static_cast<T*>(j.out_q) + row * Dp : nullptr,
-            wk ? static_cast<T*>(j.out_k) + row * Dp : nullptr);
+            in[u], m2, vi, in_pad, valid, D, Dp, nt, F, half_c, pad_value,
+            wq ? static_cast<T*>(j.out_q) + static_cast<int64_t>(row) * Dp : nullptr,
+            wk ? static_cast<T*>(j.out_k) + static_cast<int64_t>(row) * Dp : nullptr);
         if (!AUG && in_pad && vi == 0) j.nrm[row] = n;
     }
 }
@@ -640,7 +685,9 @@ cudaError_t operand_typed(const OperandJob& j0, const OperandJob* j1, int D, int
     }
     if (Dp % 16 != 0 || Dp > kOperandMaxCols || (AUG && 2 * Dp > kOperandMaxCols))
         return cudaErrorInvalidValue;
-    if (D % 8 == 0 && D >= 8 && (!AUG || Dp - D >= 2 * nt)) {
+    // The vector path indexes rows with 32-bit integers.
+    const int64_t most_rows = std::max(j0.rows_pad, j1 ? j1->rows_pad : int64_t(0)) * batch;
+    if (D % 8 == 0 && D >= 8 && (!AUG || Dp - D >= 2 * nt) && most_rows < (int64_t(1) << 30)) {
         // Vector path: G lanes per row, both arrays in one launch.
         const int V = D / 8;
         const int G = V <= 1 ? 1 : V <= 2 ? 2 : V <= 4 ? 4 : V <= 8 ? 8 : V <= 16 ? 16 : 32;
@@ -650,8 +697,8 @@ cudaError_t operand_typed(const OperandJob& j0, const OperandJob* j1, int D, int
         if (b0 + b1 == 0) return cudaSuccess;
         auto go = [&](auto kern) {
             launch_kernel(kern, static_cast<unsigned>(b0 + b1), kOperandVecThreads, 0, s, j0,
-                          j1 ? *j1 : none, static_cast<unsigned>(b0),
-                          static_cast<int64_t>(batch), D, Dp, nt, F, mu, half_c, pad_value);
+                          j1 ? *j1 : none, static_cast<unsigned>(b0), batch, D, Dp, nt, F, mu,
+                          half_c, pad_value);
         };
         switch (G) {
             case 1: go(operand_vec_kernel<T, AUG, 1>); break;

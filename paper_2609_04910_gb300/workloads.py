@@ -182,6 +182,19 @@ def generate(w: Workload, seed: int = 0) -> dict:
     }
 
 
+def batched_clouds(B: int, n: int, D: int, dtype: str = "fp16", seed: int = 0) -> dict:
+    """B independent problems of the Sec. 4 benchmark shape: per problem n
+    query and n key points ~ N(0, I_D) and weights v ~ N(0, 1) (C = 1),
+    tau = 1/D.  Drawn q (B n rows), then k, then v, as in ``generate``;
+    returns ``q`` and ``k`` of shape (B, n, D), ``v`` of shape (B, n, 1)
+    (rounded, see ``round_to``) and ``tau``."""
+    rng = np.random.default_rng(seed)
+    q = round_to(_normal_rows(rng, B * n, D), dtype).reshape(B, n, D)
+    k = round_to(_normal_rows(rng, B * n, D), dtype).reshape(B, n, D)
+    v = round_to(_normal_rows(rng, B * n, 1), dtype).reshape(B, n, 1)
+    return {"q": q, "k": k, "v": v, "tau": 1.0 / D, "dtype": dtype}
+
+
 def to_device(a: np.ndarray, dtype: str, dev="cuda:0"):
     """Copy a ``round_to`` array to a torch device tensor of the storage dtype."""
     import torch
