@@ -148,16 +148,25 @@ gs_status gauss_sum_grad_q_ex(const void* q, const void* k, const void* v, doubl
  *     grad_v[n] =     sum_m Phi(q_m, k_n) g_m                       N x C
  *
  * (all float32).  q, k, v as for gauss_sum (dtype); any of grad_q, grad_k,
- * grad_v may be NULL to skip it.  Evaluation: grad_q is a Gauss sum over
- * the keys with the C (D + 1) values (v_nc k^_n, v_nc) contracted with g_m;
- * grad_k and grad_v are one Gauss sum over the queries with the values
- * (g_mc q^_m, g_mc) contracted with v_n (its unweighted channels are
- * grad_v), k^ and q^ shifted by the common mean.  On the tensor-core path
- * the channels are evaluated in launches of at most 256 channels
- * (ceil(C (D + 1) / 256) launches per sum, each recomputing the kernel
- * values), with the values rounded to fp16 after a per-channel power-of-two
- * scale; the fp32 path makes C launches per sum.  g must be 16-byte
- * aligned.  Default options; the workspace is allocated on `stream`.
+ * grad_v may be NULL to skip it.  k^ and q^ below are shifted by the common
+ * mean.  Evaluation:
+ *  - fp16/bf16 with 2 <= C <= 8 and D + 1 <= 128 (weighted single pass):
+ *    with the pair weights w_mn = g_m . v_n multiplied into the kernel
+ *    values in float32 (before the rounding to fp16), grad_q is one Gauss
+ *    sum over the keys with the D + 1 values (k^_n, 1), grad_k one over the
+ *    queries with (q^_m, 1), and grad_v the forward sum over the queries
+ *    with the values g (three passes in all, each exponential computed once
+ *    per pass).
+ *  - otherwise: grad_q is a Gauss sum over the keys with the C (D + 1)
+ *    values (v_nc k^_n, v_nc) contracted with g_m; grad_k and grad_v are one
+ *    Gauss sum over the queries with the values (g_mc q^_m, g_mc)
+ *    contracted with v_n (its unweighted channels are grad_v).  On the
+ *    tensor-core path the channels are evaluated in launches of at most 256
+ *    channels (ceil(C (D + 1) / 256) launches per sum, each recomputing the
+ *    kernel values), with the values rounded to fp16 after a per-channel
+ *    power-of-two scale; the fp32 path makes C launches per sum.
+ * g must be 16-byte aligned.  Default options; the workspace is allocated
+ * on `stream`.
  */
 gs_status gauss_sum_vjp(const void* q, const void* k, const void* v, const float* g, double tau,
                         int64_t M, int64_t N, int64_t D, int64_t C, gs_dtype dtype,

@@ -134,7 +134,20 @@ struct Call {
     // upper triangle of tile pairs, and out then holds row sums s' with
     // sum_m v_m s'_m = v^T K v instead of K v.
     bool tri = false;
+    // Weighted vector-Jacobian pass (gradient mode with C = 1 and v null):
+    // the kernel values are multiplied by the pair weights
+    // w_mn = sum_c r[m, c] k[n, c] of wc channels, r = rw (M x wc, float32
+    // when rw_f32, else the input dtype) and k = kw (N x wc, likewise); the
+    // value channels are the unit-weight group (k^_n, 1).
+    int wc = 0;
+    const void* rw = nullptr;
+    bool rw_f32 = false;
+    const void* kw = nullptr;
+    bool kw_f32 = false;
 };
+
+// Padded weight channels of a weighted pass (the kernel's instances).
+int weight_channels(int64_t wc) { return wc <= 2 ? 2 : wc <= 4 ? 4 : 8; }
 
 gs_status validate(const Call& c) {
     if (c.dtype != GS_FP32 && c.dtype != GS_FP16 && c.dtype != GS_BF16)
@@ -148,7 +161,8 @@ gs_status validate(const Call& c) {
         return fail(GS_ERR_INVALID_ARGUMENT, "null output pointer");
     if (any && c.M > 0 && c.D > 0 && !c.q) return fail(GS_ERR_INVALID_ARGUMENT, "null q pointer");
     if (any && c.N > 0 && c.D > 0 && !c.k) return fail(GS_ERR_INVALID_ARGUMENT, "null k pointer");
-    if (any && c.N > 0 && c.C > 0 && !c.v) return fail(GS_ERR_INVALID_ARGUMENT, "null v pointer");
+    if (any && c.N > 0 && c.C > 0 && !c.v && c.wc == 0)
+        return fail(GS_ERR_INVALID_ARGUMENT, "null v pointer");
     if (!aligned16(c.q) || !aligned16(c.k) || !aligned16(c.v) || !aligned16(c.out) ||
         !aligned16(c.s_out) || !aligned16(c.u))
         return fail(GS_ERR_INVALID_ARGUMENT, "base pointers must be 16-byte aligned");
@@ -205,7 +219,8 @@ gs_status plan(const Call& c, int sms, bool* tensor, gs::TcPlan* tp, gs::SimtPla
         int64_t nch = 1;
         const int64_t width = c.grad ? grad_chunk(c.D, c.C, &nch) : c.C;
         if (!gs::plan_tensor(in_type(c.dtype), c.M, c.N, c.D, width, c.grad, c.opt.center != 0,
-                             alias, c.opt.split_n, sms, tp, &why, c.B, c.tri && !c.grad))
+                             alias, c.opt.split_n, sms, tp, &why, c.B, c.tri && !c.grad,
+                             c.wc > 0 ? weight_channels(c.wc) : 0))
             return fail(GS_ERR_UNSUPPORTED, "%s", why);
         tp->exp2_fma = c.opt.exp2_fma;
         if (tp->exp2_fma > 0 && !(tp->fma && tp->aug && !tp->tri && tp->Cv == 1))
@@ -351,7 +366,8 @@ gs_status run(Call c) {
         }
         if (e == cudaSuccess && tp.fma) {
             e = gs::launch_key_records(
-                t, c.v, tp.aug ? nullptr : reinterpret_cast<const float*>(ws + tp.off_B), c.N,
+                c.w_f32 ? gs::InType::F32 : t, c.v,
+                tp.aug ? nullptr : reinterpret_cast<const float*>(ws + tp.off_B), c.N,
                 tp.Npad, static_cast<int>(tp.Cv), reinterpret_cast<float*>(ws + tp.off_rec),
                 c.stream, batch);
             where = "key-record kernel";
@@ -384,6 +400,15 @@ gs_status run(Call c) {
                                           reinterpret_cast<unsigned*>(ws + tp.off_vmax),
                                           ws + tp.off_vt, inv, c.stream);
                 where = "value kernel";
+                if (e == cudaSuccess && tp.wt > 0) {
+                    e = gs::launch_weight_prep(t, c.rw, c.rw_f32, c.M, tp.Mpad, c.kw, c.kw_f32, c.N,
+                                               tp.Npad, static_cast<int>(c.wc), tp.wt, tp.BN,
+                                               reinterpret_cast<float*>(ws + tp.off_rowf),
+                                               reinterpret_cast<float*>(ws + tp.off_colT),
+                                               reinterpret_cast<unsigned*>(ws + tp.off_wmax),
+                                               c.stream);
+                    where = "pair-weight kernel";
+                }
                 if (e == cudaSuccess && ch0 == 0) e = record_event(c.opt.main_events[0], c.stream);
                 if (e == cudaSuccess) {
                     e = gs::launch_tc(tp, t, cexp, ws, status, c.stream, &why);
@@ -634,6 +659,34 @@ gs_status gauss_sum_vjp(const void* q, const void* k, const void* v, const float
     gs_status status = validate(a);
     if (status == GS_OK) status = validate(b);
     if (status != GS_OK) return status;
+    if (C >= 2 && C <= 8 && dtype != GS_FP32 && D >= 1 && D + 1 <= 128) {
+        // Weighted single pass per side: with the pair weights
+        // w_mn = g_m . v_n folded into the kernel values,
+        //   grad_q[m] = tau (sum_n Phi w k^_n - q^_m sum_n Phi w)
+        //   grad_k[n] = tau (sum_m Phi w q^_m - k^_n sum_m Phi w)
+        // are Gauss sums of the D + 1 unit-weight channels (x^, 1), and
+        // grad_v[n] = sum_m Phi_mn g_m is the forward sum with the values g.
+        Call wa{q, k, nullptr, tau, M, N, D, 1, dtype, true, grad_q, nullptr, st, defaults()};
+        wa.wc = static_cast<int>(C);
+        wa.rw = g;
+        wa.rw_f32 = true;
+        wa.kw = v;
+        Call wb{k, q, nullptr, tau, N, M, D, 1, dtype, true, grad_k, nullptr, st, defaults()};
+        wb.wc = static_cast<int>(C);
+        wb.rw = v;
+        wb.kw = g;
+        wb.kw_f32 = true;
+        Call wv{k, q, g, tau, N, M, D, C, dtype, false, grad_v, nullptr, st, defaults()};
+        wv.w_f32 = true;
+        status = validate(wa);
+        if (status == GS_OK) status = validate(wb);
+        if (status == GS_OK && grad_v) status = validate(wv);
+        if (status != GS_OK) return status;
+        if (grad_q) status = run(wa);
+        if (status == GS_OK && grad_k) status = run(wb);
+        if (status == GS_OK && grad_v) status = run(wv);
+        return status;
+    }
     if (grad_q) status = run(a);
     if (status == GS_OK && (grad_k || grad_v)) status = run(b);
     return status;

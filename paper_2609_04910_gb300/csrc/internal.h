@@ -100,6 +100,11 @@ struct TcPlan {
     // FMA kernel: share of the exponentials computed on the FMA pipe
     // (gs_options.exp2_fma: 0 none, 1..4 = 1/32 .. 1/4).
     int exp2_fma;
+    // Weighted vector-Jacobian pass (two-MMA kernel): the kernel values are
+    // multiplied by pair weights w_mn = sum_c r[m, c] k[n, c] of wt (padded)
+    // channels, computed from float32 factors in the exponent warps; 0: none.
+    int wt;
+    size_t off_rowf, off_colT, off_wmax;
     size_t off_mean_part, off_mu, off_qh, off_kh, off_A, off_B, off_vt, off_vmax, off_inv,
         off_rec, off_part, total;
 };
@@ -118,7 +123,7 @@ bool device_is_sm103(int device);
 
 bool plan_tensor(InType t, int64_t M, int64_t N, int64_t D, int64_t C, bool grad, bool center,
                  bool alias, int split_override, int sms, TcPlan* p, const char** why,
-                 int64_t batch = 1, bool tri = false);
+                 int64_t batch = 1, bool tri = false, int wt = 0);
 bool plan_simt(int64_t M, int64_t N, int64_t D, int64_t C, bool grad, int split_override,
                int sms, SimtPlan* p, const char** why);
 
@@ -147,6 +152,16 @@ cudaError_t launch_value_prep(InType t, bool grad, bool w_f32, const void* w, co
                               const float* mu, int64_t N, int64_t Npad, int D, int Cw, int ch0,
                               int Cc, int Cp, unsigned* vmax_bits, void* vt, float* inv_scale,
                               cudaStream_t s);
+// Factors of the pair weights w_mn = sum_c r[m, c] k[n, c] of the weighted
+// vector-Jacobian pass (see prep.cu): row factors rsrc (R x C) into rowf
+// (Rpad x WT float32), column factors csrc (Ncol x C) into colT (per key
+// tile of BN keys, channel-major), their per-channel maxima into wmax
+// (2 WT float bits).  One side is float32 (r_f32 / c_f32), the other has the
+// inputs' dtype t.
+cudaError_t launch_weight_prep(InType t, const void* rsrc, bool r_f32, int64_t R, int64_t Rpad,
+                               const void* csrc, bool c_f32, int64_t Ncol, int64_t Npad, int C,
+                               int WT, int BN, float* rowf, float* colT, unsigned* wmax,
+                               cudaStream_t s);
 // Forward: out (M x Cv) = inv_scale (when given) x the split partials summed
 // in split order; rows below main_rows have one split.
 cudaError_t launch_finalize(const float* part, int splits, int64_t split_stride_rows,

@@ -734,7 +734,9 @@ cudaError_t operand_typed(const OperandJob& j0, const OperandJob* j1, int D, int
 // Value of channel ch of key n.  Forward (Eq. 1): w[n, ch] (Cw = channels).
 // Gradients (Sec. 3, and the vector-Jacobian product of Eq. 1): channel
 // ch = c (D + 1) + d holds w[n, c] (x[n, d] - mu_d) for d < D and w[n, c]
-// for d = D, one group of D + 1 channels per weight channel c < Cw.
+// for d = D, one group of D + 1 channels per weight channel c < Cw; a null
+// w means unit weights (the weighted vector-Jacobian pass, whose weights
+// enter through the kernel values instead).
 template <typename T, typename W, bool GRAD>
 __device__ __forceinline__ float value_at(const W* __restrict__ w, const T* __restrict__ x,
                                           const float* __restrict__ mu, int64_t n, int ch, int D,
@@ -742,7 +744,7 @@ __device__ __forceinline__ float value_at(const W* __restrict__ w, const T* __re
     if (GRAD) {
         const int c = ch / (D + 1);
         const int d = ch - c * (D + 1);
-        const float wn = to_f(w[n * Cw + c]);
+        const float wn = w ? to_f(w[n * Cw + c]) : 1.f;
         if (d < D) return wn * (to_f(x[n * D + d]) - (mu ? mu[d] : 0.f));
         return wn;
     }
@@ -859,6 +861,55 @@ __global__ void key_record_kernel(const T* __restrict__ v, const float* __restri
     for (int c = 0; c < C; ++c) {
         out[head + 2 * c] = n0 < N ? to_f(v[n0 * C + c]) : 0.f;
         out[head + 1 + 2 * c] = n1 < N ? to_f(v[n1 * C + c]) : 0.f;
+    }
+}
+
+// ---------------------------------------------------------------- pair weights
+// Factors of the pair weights w_mn = sum_c r[m, c] k[n, c] of the weighted
+// vector-Jacobian pass (row factors r: the rows of the Gauss sum, column
+// factors k: its keys; C <= WT channels, zero padded to WT).  Blocks
+// [0, rblocks) write the row factors row-major in float32,
+// rowf[m WT + c] (Rpad rows, zero past R); the other blocks write the
+// column factors per key tile of BN keys, channel-major inside the tile,
+// colT[(n / BN) WT BN + c BN + n % BN] (Npad keys, zero past Ncol), so that
+// one bulk copy brings a key tile's factors into shared memory.  wmax[c]
+// and wmax[WT + c] receive the largest |r[., c]| and |k[., c]| (float bits,
+// atomicMax over blocks; the caller zeroes them).  One thread per (row or
+// key, channel), 256 threads per block.
+constexpr int kWeightThreads = 256;
+
+template <typename TR, typename TC>
+__global__ void __launch_bounds__(kWeightThreads)
+weight_prep_kernel(const TR* __restrict__ rsrc, int64_t R, int64_t Rpad,
+                   const TC* __restrict__ csrc, int64_t Ncol, int64_t Npad, int C, int WT, int BN,
+                   unsigned rblocks, float* __restrict__ rowf, float* __restrict__ colT,
+                   unsigned* __restrict__ wmax) {
+    pdl_trigger();
+    pdl_wait();
+    __shared__ float red[kWeightThreads];
+    const bool on_rows = blockIdx.x < rblocks;
+    const int64_t blk = on_rows ? blockIdx.x : blockIdx.x - rblocks;
+    const int64_t idx = blk * kWeightThreads + threadIdx.x;
+    const int64_t i = idx / WT;                 // row or key
+    const int c = static_cast<int>(idx - i * WT);
+    float val = 0.f;
+    if (on_rows) {
+        if (i < Rpad) {
+            if (i < R && c < C) val = to_f(rsrc[i * C + c]);
+            rowf[idx] = val;
+        }
+    } else if (i < Npad) {
+        if (i < Ncol && c < C) val = to_f(csrc[i * C + c]);
+        colT[(i / BN) * WT * BN + static_cast<int64_t>(c) * BN + i % BN] = val;
+    }
+    // Channel c of this block: threads t with t % WT == c (WT divides 256).
+    red[threadIdx.x] = fabsf(val);
+    __syncthreads();
+    if (threadIdx.x < WT) {
+        float m = 0.f;
+        for (int t = threadIdx.x; t < kWeightThreads; t += WT) m = fmaxf(m, red[t]);
+        // Non-negative floats order like their bit patterns.
+        atomicMax(&wmax[(on_rows ? 0 : WT) + threadIdx.x], __float_as_uint(m));
     }
 }
 
@@ -1186,11 +1237,13 @@ cudaError_t launch_value_prep(InType t, bool grad, bool w_f32, const void* w, co
 #define GS_VALUE_PREP(T, W, G) \
     value_prep_typed<T, W, G>(w, x, mu, N, Npad, D, Cw, ch0, Cc, Cp, vmax_bits, vt, inv_scale, s)
     if (t == InType::BF16) {
-        if (!grad) return GS_VALUE_PREP(__nv_bfloat16, __nv_bfloat16, false);
+        if (!grad)
+            return w_f32 ? GS_VALUE_PREP(__nv_bfloat16, float, false)
+                         : GS_VALUE_PREP(__nv_bfloat16, __nv_bfloat16, false);
         return w_f32 ? GS_VALUE_PREP(__nv_bfloat16, float, true)
                      : GS_VALUE_PREP(__nv_bfloat16, __nv_bfloat16, true);
     }
-    if (!grad) return GS_VALUE_PREP(__half, __half, false);
+    if (!grad) return w_f32 ? GS_VALUE_PREP(__half, float, false) : GS_VALUE_PREP(__half, __half, false);
     return w_f32 ? GS_VALUE_PREP(__half, float, true) : GS_VALUE_PREP(__half, __half, true);
 #undef GS_VALUE_PREP
 }
@@ -1211,6 +1264,40 @@ cudaError_t launch_key_records(InType t, const void* v, const float* B, int64_t 
     else
         launch_kernel(key_record_kernel<__half>, dim3(blocks, batch), threads, 0, s, static_cast<const __half*>(v), B, N,
                                                              pairs, C, rec);
+    note_launches(1);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_weight_prep(InType t, const void* rsrc, bool r_f32, int64_t R, int64_t Rpad,
+                               const void* csrc, bool c_f32, int64_t Ncol, int64_t Npad, int C,
+                               int WT, int BN, float* rowf, float* colT, unsigned* wmax,
+                               cudaStream_t s) {
+    if (WT <= 0 || kWeightThreads % WT != 0 || C > WT) return cudaErrorInvalidValue;
+    cudaError_t e = cudaMemsetAsync(wmax, 0, sizeof(unsigned) * 2 * WT, s);
+    if (e != cudaSuccess) return e;
+    pdl_reset();   // the next kernel follows a memset
+    const int64_t rb = (Rpad * WT + kWeightThreads - 1) / kWeightThreads;
+    const int64_t cb = (Npad * WT + kWeightThreads - 1) / kWeightThreads;
+    if (rb + cb == 0) return cudaSuccess;
+    const dim3 grid(static_cast<unsigned>(rb + cb));
+    const unsigned rbu = static_cast<unsigned>(rb);
+#define GS_WPREP(TR, TC)                                                                        \
+    launch_kernel(weight_prep_kernel<TR, TC>, grid, kWeightThreads, 0, s,                      \
+                  static_cast<const TR*>(rsrc), R, Rpad, static_cast<const TC*>(csrc), Ncol,   \
+                  Npad, C, WT, BN, rbu, rowf, colT, wmax)
+    // One side is the float32 upstream gradient, the other the inputs' dtype.
+    if (t == InType::BF16) {
+        if (r_f32 && !c_f32) GS_WPREP(float, __nv_bfloat16);
+        else if (!r_f32 && c_f32) GS_WPREP(__nv_bfloat16, float);
+        else return cudaErrorInvalidValue;
+    } else if (t == InType::F16) {
+        if (r_f32 && !c_f32) GS_WPREP(float, __half);
+        else if (!r_f32 && c_f32) GS_WPREP(__half, float);
+        else return cudaErrorInvalidValue;
+    } else {
+        return cudaErrorInvalidValue;
+    }
+#undef GS_WPREP
     note_launches(1);
     return cudaGetLastError();
 }

@@ -95,6 +95,12 @@ struct TcParams {
     float c;
     uint32_t idesc1, idesc2;
     const uint32_t* qh;  // QTM: q^ rows (packed 16-bit pairs, Dp / 2 per row)
+    // WT: factors of the pair weights (see launch_weight_prep): row factors
+    // (Mpad x WT), column factors per key tile (WT x BN), and their
+    // per-channel maxima (2 WT float bits).
+    const float* rowf;
+    const float* colT;
+    const unsigned* wmax;
 };
 
 struct __align__(8) Barriers {
@@ -135,7 +141,10 @@ static_assert(16 * 32 * kExpRegs2 + 4 * 32 * kCtrlRegs2 <= 640 * 96, "register s
 // P-then-S order (tensor-bound shapes).  QTM: q^ in TMEM (columns
 // [3 BN + Cp, 3 BN + Cp + Dp / 2), copied there by the exponent warps; MMA1
 // reads A from TMEM), which leaves its shared memory to the key stages.
-template <int BN, int NEXP, bool AUG, bool EARLY, bool QTM = false>
+// WT > 0: weighted vector-Jacobian pass: the kernel values are multiplied
+// by the pair weights w_mn = sum_c r[m, c] k[n, c] (WT channels) before the
+// rounding to fp16; see the exponent warps.
+template <int BN, int NEXP, bool AUG, bool EARLY, bool QTM = false, int WT = 0>
 __global__ void __launch_bounds__(cta_threads<NEXP>(), 1)
 tc_gauss_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
                 const __grid_constant__ CUtensorMap tm_v, const TcParams p) {
@@ -208,6 +217,11 @@ tc_gauss_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant_
     auto b_smem = [&](int s) {
         return reinterpret_cast<const float*>(stage0 + s * p.stage_bytes + p.kh_bytes + p.vt_bytes);
     };
+    // WT: the key tile's column factors, channel-major (WT x BN floats).
+    auto cw_smem = [&](int s) {
+        return reinterpret_cast<const float*>(stage0 + s * p.stage_bytes + p.kh_bytes + p.vt_bytes +
+                                              BN * 4);
+    };
 
     if (warp == PRODUCER_WARP) {
         if (NEXP == 16) reg_dealloc<kCtrlRegs2>();
@@ -239,6 +253,9 @@ tc_gauss_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant_
                     for (int h = 0; h < BN / KB; ++h)
                         tma_load_2d(vt_smem(s) + h * (p.Cp * 128), &tm_v, &bars->kv_full[s], n0 + h * KB, 0);
                     if (!AUG) bulk_load(const_cast<float*>(b_smem(s)), p.B + n0, BN * 4, &bars->kv_full[s]);
+                    if (WT > 0)
+                        bulk_load(const_cast<float*>(cw_smem(s)), p.colT + static_cast<int64_t>(n0) * WT,
+                                  BN * WT * 4, &bars->kv_full[s]);
                 }
                 __syncwarp();
                 issued = j + 1;
@@ -415,8 +432,31 @@ tc_gauss_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant_
         const int col0 = part * COLS;
         const int row_local = quarter * 32 + lane;
         const int64_t row = static_cast<int64_t>(tile_m) * BM + row_local;
-        const float a_m = (AUG ? 0.f : p.A[row]) + P_SHIFT;
+        const float a_m = (AUG ? 0.f : p.A[row]) + (WT > 0 ? 0.f : P_SHIFT);
         const uint64_t a2 = f32x2_pack(a_m, a_m);
+        // WT: this row's factors of the pair weights, times 2^sw, and the
+        // epilogue's inverse scale.  With Wb = sum_c max|r_c| max|k_c| >=
+        // |w_mn| and sw = 15 - ceil(log2 Wb), |2^sw w_mn| <= 2^15, so the
+        // products 2^x 2^sw w_mn (x <= 0) fit fp16 like the unweighted
+        // P = 2^(x + 15), and small weights keep their precision.
+        float unshift = P_UNSHIFT;
+        uint64_t rw2[WT > 0 ? WT : 1];
+        if (WT > 0) {
+            float wb = 0.f;
+#pragma unroll
+            for (int c = 0; c < WT; ++c)
+                wb = fmaf(__uint_as_float(p.wmax[c]), __uint_as_float(p.wmax[WT + c]), wb);
+            int e = 0;
+            if (wb > 0.f) frexpf(wb, &e);                // wb <= 2^e
+            const int sw = max(-100, min(100, 15 - e));
+            const float sc = ldexpf(1.f, sw);
+            unshift = ldexpf(1.f, -sw);
+#pragma unroll
+            for (int c = 0; c < WT; ++c) {
+                const float r = p.rowf[row * WT + c] * sc;
+                rw2[c] = f32x2_pack(r, r);
+            }
+        }
         const uint64_t c2 = f32x2_pack(p.c, p.c);
         const uint32_t lane_base = static_cast<uint32_t>(quarter * 32) << 16;
         if (QTM) {
@@ -441,9 +481,10 @@ tc_gauss_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant_
         for (int j = group; j < T; j += 2, st.advance(p.stages), st.advance(p.stages)) {
             const int b = group;
             const int s = st.idx;
-            // The B records of the stage are only read without augmented
-            // operands; S itself is ordered by s_full.
-            if (!AUG) ok = warp_wait(&bars->kv_full[s], st.phase, abort_flag, p.status);
+            // The B records and the column factors of the stage are read
+            // from shared memory (without augmented operands / with pair
+            // weights); S itself is ordered by s_full.
+            if (!AUG || WT > 0) ok = warp_wait(&bars->kv_full[s], st.phase, abort_flag, p.status);
             if (ok && !__all_sync(0xffffffffu, mbar_test_wait(&bars->s_full[b],
                                                                static_cast<uint32_t>(j >> 1) & 1u)))
                 ok = warp_wait(&bars->s_full[b], static_cast<uint32_t>(j >> 1) & 1u, abort_flag,
@@ -485,8 +526,28 @@ tc_gauss_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant_
                 float x0, x1, x2, x3;
                 f32x2_unpack(f32x2_fma(s01, c2, t01), x0, x1);
                 f32x2_unpack(f32x2_fma(s23, c2, t23), x2, x3);
-                pk[2 * i + 0] = bound_p2(pack_half2_satfinite(ex2_approx(x0), ex2_approx(x1)));
-                pk[2 * i + 1] = bound_p2(pack_half2_satfinite(ex2_approx(x2), ex2_approx(x3)));
+                if (WT > 0) {
+                    // P' = 2^min(x, 0) (2^sw w_mn) for the four keys: the
+                    // weights from the row factors (registers) and the key
+                    // tile's column factors (shared memory, one broadcast
+                    // 16-byte load per channel), in float32.
+                    const float* cws = cw_smem(s) + col0 + 4 * i;
+                    uint64_t w01 = 0ull, w23 = 0ull;
+#pragma unroll
+                    for (int c = 0; c < WT; ++c) {
+                        const float4 kc = *reinterpret_cast<const float4*>(cws + c * BN);
+                        w01 = f32x2_fma(rw2[c], f32x2_pack(kc.x, kc.y), w01);
+                        w23 = f32x2_fma(rw2[c], f32x2_pack(kc.z, kc.w), w23);
+                    }
+                    float p0, p1, p2, p3;
+                    f32x2_unpack(f32x2_mul(f32x2_pack(ex2_nonpos(x0), ex2_nonpos(x1)), w01), p0, p1);
+                    f32x2_unpack(f32x2_mul(f32x2_pack(ex2_nonpos(x2), ex2_nonpos(x3)), w23), p2, p3);
+                    pk[2 * i + 0] = pack_half2_satfinite(p0, p1);
+                    pk[2 * i + 1] = pack_half2_satfinite(p2, p3);
+                } else {
+                    pk[2 * i + 0] = bound_p2(pack_half2_satfinite(ex2_approx(x0), ex2_approx(x1)));
+                    pk[2 * i + 1] = bound_p2(pack_half2_satfinite(ex2_approx(x2), ex2_approx(x3)));
+                }
             }
             if (EARLY && j >= 2) {
                 // P buffer b: MMA2 of tile j - 2 has read it.  (With one MMA
@@ -512,10 +573,10 @@ tc_gauss_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant_
                 uint32_t r[8];
                 tmem_ld_32x32b_x8(tmem + lane_base + O_col + c8, r);
                 tmem_wait_ld_regs(r);
-                float4 lo = make_float4(__uint_as_float(r[0]) * P_UNSHIFT, __uint_as_float(r[1]) * P_UNSHIFT,
-                                        __uint_as_float(r[2]) * P_UNSHIFT, __uint_as_float(r[3]) * P_UNSHIFT);
-                float4 hi = make_float4(__uint_as_float(r[4]) * P_UNSHIFT, __uint_as_float(r[5]) * P_UNSHIFT,
-                                        __uint_as_float(r[6]) * P_UNSHIFT, __uint_as_float(r[7]) * P_UNSHIFT);
+                float4 lo = make_float4(__uint_as_float(r[0]) * unshift, __uint_as_float(r[1]) * unshift,
+                                        __uint_as_float(r[2]) * unshift, __uint_as_float(r[3]) * unshift);
+                float4 hi = make_float4(__uint_as_float(r[4]) * unshift, __uint_as_float(r[5]) * unshift,
+                                        __uint_as_float(r[6]) * unshift, __uint_as_float(r[7]) * unshift);
                 *reinterpret_cast<float4*>(out + c8) = lo;
                 *reinterpret_cast<float4*>(out + c8 + 4) = hi;
             }
@@ -533,7 +594,7 @@ tc_gauss_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant_
 // ---------------------------------------------------------------- host side
 size_t align1k(size_t x) { return (x + 1023) & ~static_cast<size_t>(1023); }
 
-template <int BN, int NEXP, bool AUG, bool EARLY, bool QTM = false>
+template <int BN, int NEXP, bool AUG, bool EARLY, bool QTM = false, int WT = 0>
 cudaError_t launch_bn(const TcPlan& pl, InType t, float c, char* ws, unsigned* status,
                       cudaStream_t s, const char** why, int tile_off, int tiles, int splits) {
     const CUtensorMapDataType hdt =
@@ -561,8 +622,8 @@ cudaError_t launch_bn(const TcPlan& pl, InType t, float c, char* ws, unsigned* s
     p.stages = pl.stages;
     p.kh_bytes = static_cast<uint32_t>(p.nkb * BN * 128);
     p.vt_bytes = static_cast<uint32_t>((BN / KB) * pl.Cp * 128);
-    p.tx_bytes = p.kh_bytes + p.vt_bytes + (AUG ? 0 : BN * 4);
-    p.stage_bytes = static_cast<uint32_t>(align1k(p.kh_bytes + p.vt_bytes + BN * 4));
+    p.tx_bytes = p.kh_bytes + p.vt_bytes + (AUG ? 0 : BN * 4) + BN * WT * 4;
+    p.stage_bytes = static_cast<uint32_t>(align1k(p.kh_bytes + p.vt_bytes + BN * 4 + BN * WT * 4));
     p.c = c;
     const uint32_t hb = t == InType::BF16 ? 1u : 0u;
     p.idesc1 = idesc_f16(BM, BN, hb, hb);
@@ -570,12 +631,15 @@ cudaError_t launch_bn(const TcPlan& pl, InType t, float c, char* ws, unsigned* s
 
     // Per-device function attribute; cheap enough to set on every launch.
     p.qh = reinterpret_cast<const uint32_t*>(ws + pl.off_qh);
-    cudaError_t e = cudaFuncSetAttribute(tc_gauss_kernel<BN, NEXP, AUG, EARLY, QTM>,
+    p.rowf = WT > 0 ? reinterpret_cast<const float*>(ws + pl.off_rowf) : nullptr;
+    p.colT = WT > 0 ? reinterpret_cast<const float*>(ws + pl.off_colT) : nullptr;
+    p.wmax = WT > 0 ? reinterpret_cast<const unsigned*>(ws + pl.off_wmax) : nullptr;
+    cudaError_t e = cudaFuncSetAttribute(tc_gauss_kernel<BN, NEXP, AUG, EARLY, QTM, WT>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          static_cast<int>(pl.smem_bytes));
     if (e != cudaSuccess) return e;
     dim3 grid(static_cast<unsigned>(tiles), static_cast<unsigned>(splits));
-    launch_kernel(tc_gauss_kernel<BN, NEXP, AUG, EARLY, QTM>, grid, cta_threads<NEXP>(), pl.smem_bytes, s, tm_q, tm_k, tm_v, p);
+    launch_kernel(tc_gauss_kernel<BN, NEXP, AUG, EARLY, QTM, WT>, grid, cta_threads<NEXP>(), pl.smem_bytes, s, tm_q, tm_k, tm_v, p);
     note_launches(1);
     return cudaGetLastError();
 }
@@ -589,7 +653,7 @@ constexpr int64_t kMaxBands = 256;
 
 bool plan_tensor(InType t, int64_t M, int64_t N, int64_t D, int64_t C, bool grad, bool center,
                  bool alias, int split_override, int sms, TcPlan* p, const char** why,
-                 int64_t batch, bool tri) {
+                 int64_t batch, bool tri, int wt) {
     p->M = M;
     p->N = N;
     p->D = D;
@@ -606,6 +670,11 @@ bool plan_tensor(InType t, int64_t M, int64_t N, int64_t D, int64_t C, bool grad
     p->tri = false;
     p->tri_units = 0;
     p->qtm = false;
+    p->wt = wt;
+    if (wt != 0 && !(grad && t != InType::F32 && (wt == 2 || wt == 4 || wt == 8))) {
+        *why = "pair weights need a 16-bit gradient pass with 2, 4 or 8 weight channels";
+        return false;
+    }
     size_t fma_smem = 0;
     int fma_stages = 0, nq = 1;
     if (t == InType::F32) {
@@ -655,9 +724,14 @@ bool plan_tensor(InType t, int64_t M, int64_t N, int64_t D, int64_t C, bool grad
         const int nkb = (p->Dp + KB - 1) / KB;
         p->BN = p->Cp <= 128 ? 128 : 64;
         p->nq = 1;
+        if (wt > 0 && p->BN != 128) {
+            *why = "pair weights need D + 1 <= 128 value channels";
+            return false;
+        }
 
         const size_t stage = align1k(static_cast<size_t>(nkb) * p->BN * 128 +
-                                     static_cast<size_t>(p->BN / KB) * p->Cp * 128 + p->BN * 4);
+                                     static_cast<size_t>(p->BN / KB) * p->Cp * 128 + p->BN * 4 +
+                                     static_cast<size_t>(p->BN) * wt * 4);
         const size_t qbytes = static_cast<size_t>(nkb) * BM * 128;
         size_t fixed = 1024 /*alignment slack*/ + qbytes + sizeof(Barriers) + 64;
         const size_t budget = 232448;
@@ -838,6 +912,12 @@ bool plan_tensor(InType t, int64_t M, int64_t N, int64_t D, int64_t C, bool grad
         p->off_inv = take(static_cast<size_t>(p->Cp) * 4);
         p->off_part = take(static_cast<size_t>(p->splits) * p->Mpad * p->Cp * 4);
     }
+    p->off_rowf = p->off_colT = p->off_wmax = 0;
+    if (wt > 0) {
+        p->off_rowf = take(static_cast<size_t>(p->Mpad) * wt * 4);
+        p->off_colT = take(static_cast<size_t>(p->Npad) * wt * 4);
+        p->off_wmax = take(static_cast<size_t>(2) * wt * 4);
+    }
     p->total = off;
     return true;
 }
@@ -848,6 +928,20 @@ cudaError_t launch_tc_range(const TcPlan& p, InType t, float c, char* ws, unsign
                             cudaStream_t s, const char** why, int off, int tiles, int splits) {
 #define GS_TC(BN_, NE_, AUG_, EARLY_, QTM_) \
     launch_bn<BN_, NE_, AUG_, EARLY_, QTM_>(p, t, c, ws, status, s, why, off, tiles, splits)
+#define GS_TCW(AUG_, EARLY_, QTM_)                                                               \
+    (p.wt == 2   ? launch_bn<128, 16, AUG_, EARLY_, QTM_, 2>(p, t, c, ws, status, s, why, off,   \
+                                                             tiles, splits)                      \
+     : p.wt == 4 ? launch_bn<128, 16, AUG_, EARLY_, QTM_, 4>(p, t, c, ws, status, s, why, off,   \
+                                                             tiles, splits)                      \
+                 : launch_bn<128, 16, AUG_, EARLY_, QTM_, 8>(p, t, c, ws, status, s, why, off,   \
+                                                             tiles, splits))
+    if (p.wt > 0) {
+        // Weighted vector-Jacobian pass (BN = 128 only, see plan_tensor).
+        if (p.BN != 128) return cudaErrorInvalidValue;
+        if (p.aug) return p.early_s ? GS_TCW(true, true, false) : GS_TCW(true, false, false);
+        if (p.qtm) return p.early_s ? GS_TCW(false, true, true) : GS_TCW(false, false, true);
+        return p.early_s ? GS_TCW(false, true, false) : GS_TCW(false, false, false);
+    }
     if (p.aug) {
         if (p.BN == 128) return p.early_s ? GS_TC(128, 16, true, true, false) : GS_TC(128, 16, true, false, false);
         return p.early_s ? GS_TC(64, 8, true, true, false) : GS_TC(64, 8, true, false, false);
@@ -856,6 +950,7 @@ cudaError_t launch_tc_range(const TcPlan& p, InType t, float c, char* ws, unsign
         return p.early_s ? GS_TC(128, 16, false, true, true) : GS_TC(128, 16, false, false, true);
     if (p.BN == 128) return p.early_s ? GS_TC(128, 16, false, true, false) : GS_TC(128, 16, false, false, false);
     return p.early_s ? GS_TC(64, 8, false, true, false) : GS_TC(64, 8, false, false, false);
+#undef GS_TCW
 #undef GS_TC
 }
 

@@ -4,9 +4,11 @@ L = sum_m g_m . s_m in q, k and v) against the float64 oracle.
 Tolerance per output: |x_gpu - x_oracle| / (its error scale + 1e-30) within
 the forward tolerance (2e-3 fp16/bf16, 1e-5 fp32), with the error scales of
 the oracle (the terms of the per-channel Gauss sums the library evaluates,
-shifted by the common mean).  Cases cover one and several channel chunks
-(C (D + 1) above 256), ragged row and key tails, q = k, and the degenerate
-sizes.
+shifted by the common mean).  Cases cover the weighted single pass
+(2 <= C <= 8 weight channels, D + 1 <= 128, fp16/bf16: pair weights g_m . v_n
+folded into the kernel values), its boundaries (C = 9, D = 128), one and
+several channel chunks of the per-channel path (C (D + 1) above 256),
+ragged row and key tails, q = k, and the degenerate sizes.
 """
 import numpy as np
 import pytest
@@ -66,6 +68,12 @@ VJP_CASES = [
     (64, 100, 100, 3, "bf16"),     # 303 channels: two chunks
     (100, 130, 16, 1, "fp32"),
     (70, 90, 33, 3, "fp32"),
+    # weighted single pass: several row and key tiles, ragged tails
+    (400, 700, 64, 4, "fp16"),     # four weight channels
+    (300, 520, 32, 8, "bf16"),     # eight
+    (260, 390, 127, 6, "fp16"),    # D + 1 = 128 value channels, six weights padded to eight
+    (333, 300, 40, 9, "fp16"),     # nine weights: per-channel path
+    (200, 300, 128, 2, "fp16"),    # D + 1 = 129: per-channel path
 ]
 
 
