@@ -198,8 +198,9 @@ mean_final_block_kernel(const float* __restrict__ partial, int G, int D, double 
                         int mant_bits, int min_exp, float* __restrict__ mu) {
     pdl_trigger();
     pdl_wait();
-    __shared__ double red_s[kMeanFinalThreads];
-    __shared__ float red_m[kMeanFinalThreads];
+    constexpr int W = kMeanFinalThreads / 32;
+    __shared__ double red_s[W];
+    __shared__ float red_m[W];
     const int d = blockIdx.x;
     const int t = threadIdx.x;
     partial += static_cast<int64_t>(blockIdx.y) * 2 * G * D;
@@ -210,17 +211,26 @@ mean_final_block_kernel(const float* __restrict__ partial, int G, int D, double 
         s += static_cast<double>(partial[static_cast<int64_t>(g) * D + d]);
         mx = fmaxf(mx, partial[static_cast<int64_t>(G + g) * D + d]);
     }
-    red_s[t] = s;
-    red_m[t] = mx;
-    __syncthreads();
-    for (int w = kMeanFinalThreads / 2; w > 0; w >>= 1) {
-        if (t < w) {
-            red_s[t] += red_s[t + w];
-            red_m[t] = fmaxf(red_m[t], red_m[t + w]);
-        }
-        __syncthreads();
+    // Fixed butterfly inside each warp, then warp 0 adds the warps in order.
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        s += __shfl_xor_sync(0xffffffffu, s, o);
+        mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
     }
-    if (t == 0) mu[d] = rounded_mean(red_s[0], red_m[0], total, mant_bits, min_exp);
+    if ((t & 31) == 0) {
+        red_s[t >> 5] = s;
+        red_m[t >> 5] = mx;
+    }
+    __syncthreads();
+    if (t == 0) {
+        double a = 0.0;
+        float m = 0.f;
+        for (int w = 0; w < W; ++w) {
+            a += red_s[w];
+            m = fmaxf(m, red_m[w]);
+        }
+        mu[d] = rounded_mean(a, m, total, mant_bits, min_exp);
+    }
 }
 
 // Few partials per coordinate (the small problems of a batch): one warp per
@@ -573,33 +583,49 @@ __device__ __forceinline__ float operand_row(const uint4 in, const uint4 m2, int
         return nrm;
     }
     // Norm terms: a (or b) = -||x^||^2 / 2 = F t_0 + t_1 + ... (rounded
-    // remainders), partners F, 1, 1 on the other side.
-    __align__(16) unsigned short tq[16];
-    __align__(16) unsigned short tk[16];
-#pragma unroll
-    for (int e = 0; e < 16; ++e) tq[e] = tk[e] = 0;
+    // remainders, nt <= 3 of them), partners F, 1, 1 on the other side.
+    // Built in registers: element e of the query tail is the partner
+    // (F, 1, 1) for e < nt and t_(e - nt) for nt <= e < 2 nt; the key tail
+    // the other way round; zeros after that.
+    unsigned short t0 = 0, t1 = 0, t2 = 0;
     if (valid) {
         float r = -0.5f * acc;
-        for (int i = 0; i < nt; ++i) {
-            const T t = from_f<T>(i == 0 ? r / F : r);
-            r -= (i == 0 ? F : 1.f) * to_f(t);
-            const unsigned short one = to_bits(from_f<T>(i == 0 ? F : 1.f));
-            tq[i] = one;
-            tq[nt + i] = to_bits(t);
-            tk[i] = to_bits(t);
-            tk[nt + i] = one;
-        }
-    } else {
-        tk[0] = to_bits(from_f<T>(-30000.f / F));
+        const T a0 = from_f<T>(r * (1.f / F));   // F is a power of two: exact
+        r -= F * to_f(a0);
+        const T a1 = from_f<T>(r);
+        r -= to_f(a1);
+        const T a2 = from_f<T>(r);
+        t0 = to_bits(a0);
+        t1 = to_bits(a1);
+        t2 = nt > 2 ? to_bits(a2) : 0;
     }
-    for (int c = D, e0 = 0; c < Dp; c += 8, e0 += 8) {
-        uint4 uq = make_uint4(0u, 0u, 0u, 0u), uk = make_uint4(0u, 0u, 0u, 0u);
-        if (e0 < 16) {
-            uq = *reinterpret_cast<const uint4*>(tq + e0);
-            uk = *reinterpret_cast<const uint4*>(tk + e0);
+    const unsigned short oneF = valid ? to_bits(from_f<T>(F)) : 0;
+    const unsigned short one1 = valid ? to_bits(from_f<T>(1.f)) : 0;
+    const unsigned short pad_b = valid ? t0 : to_bits(from_f<T>(-30000.f / F));
+    auto term = [&](int i) { return i == 0 ? pad_b : i == 1 ? t1 : t2; };
+    auto partner = [&](int i) { return i == 0 ? oneF : one1; };
+    auto tail_q = [&](int e) -> unsigned {
+        return e < nt ? partner(e) : e < 2 * nt ? (e == nt ? t0 : term(e - nt)) : 0u;
+    };
+    auto tail_k = [&](int e) -> unsigned {
+        return e < nt ? term(e) : e < 2 * nt ? partner(e - nt) : 0u;
+    };
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+        const int c = D + 8 * h;
+        if (c >= Dp) break;
+        uint32_t wq[4], wk[4];
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+            wq[e] = tail_q(8 * h + 2 * e) | (tail_q(8 * h + 2 * e + 1) << 16);
+            wk[e] = tail_k(8 * h + 2 * e) | (tail_k(8 * h + 2 * e + 1) << 16);
         }
-        if (out_q) *reinterpret_cast<uint4*>(out_q + c) = uq;
-        if (out_k) *reinterpret_cast<uint4*>(out_k + c) = uk;
+        if (out_q) *reinterpret_cast<uint4*>(out_q + c) = make_uint4(wq[0], wq[1], wq[2], wq[3]);
+        if (out_k) *reinterpret_cast<uint4*>(out_k + c) = make_uint4(wk[0], wk[1], wk[2], wk[3]);
+    }
+    for (int c = D + 16; c < Dp; c += 8) {
+        if (out_q) *reinterpret_cast<uint4*>(out_q + c) = make_uint4(0u, 0u, 0u, 0u);
+        if (out_k) *reinterpret_cast<uint4*>(out_k + c) = make_uint4(0u, 0u, 0u, 0u);
     }
     return nrm;
 }
