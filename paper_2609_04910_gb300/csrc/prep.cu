@@ -176,42 +176,44 @@ mean_partial_vec_kernel(const T* __restrict__ q, const T* __restrict__ k, int64_
 constexpr int kMeanFinalThreads = 256;
 
 // The grid-rounded mean of the folded sum s and largest magnitude mx.
-__device__ __forceinline__ float rounded_mean(double s, float mx, double total, int mant_bits,
+__device__ __forceinline__ float rounded_mean(float s, float mx, float total, int mant_bits,
                                               int min_exp) {
-    double m = s / total;
+    // float32 throughout: any shift is exact for the Gauss sum, so the mean
+    // needs no more precision than that, and float64 is slow on this GPU.
+    float m = s / total;
     if (mx > 0.f) {
         int e;
-        frexp(static_cast<double>(mx), &e);              // mx in [2^(e-1), 2^e)
-        const double g = ldexp(1.0, max(e - 1 - mant_bits, min_exp));
-        m = rint(m / g) * g;
+        frexpf(mx, &e);                                   // mx in [2^(e-1), 2^e)
+        const float g = ldexpf(1.f, max(e - 1 - mant_bits, min_exp));
+        m = rintf(m / g) * g;
     }
-    return static_cast<float>(m);
+    return m;
 }
 
-// Many partials per coordinate (G > kMeanFinalWarpMax): one block per
+// Many partials per coordinate (G > kMeanFinalThreadMax): one block per
 // (coordinate d, problem blockIdx.y); thread t folds partials t, t + 256,
-// ... in order, then a fixed tree combines the threads (deterministic).
-constexpr int kMeanFinalWarpMax = 128;
+// ... in order, a fixed butterfly adds the lanes of each warp and thread 0
+// the warps in order (deterministic).
+constexpr int kMeanFinalThreadMax = 32;
 
 __global__ void __launch_bounds__(kMeanFinalThreads)
-mean_final_block_kernel(const float* __restrict__ partial, int G, int D, double total,
+mean_final_block_kernel(const float* __restrict__ partial, int G, int D, float total,
                         int mant_bits, int min_exp, float* __restrict__ mu) {
     pdl_trigger();
     pdl_wait();
     constexpr int W = kMeanFinalThreads / 32;
-    __shared__ double red_s[W];
+    __shared__ float red_s[W];
     __shared__ float red_m[W];
     const int d = blockIdx.x;
     const int t = threadIdx.x;
     partial += static_cast<int64_t>(blockIdx.y) * 2 * G * D;
     mu += static_cast<int64_t>(blockIdx.y) * D;
-    double s = 0.0;
+    float s = 0.f;
     float mx = 0.f;
     for (int g = t; g < G; g += kMeanFinalThreads) {
-        s += static_cast<double>(partial[static_cast<int64_t>(g) * D + d]);
+        s += partial[static_cast<int64_t>(g) * D + d];
         mx = fmaxf(mx, partial[static_cast<int64_t>(G + g) * D + d]);
     }
-    // Fixed butterfly inside each warp, then warp 0 adds the warps in order.
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) {
         s += __shfl_xor_sync(0xffffffffu, s, o);
@@ -223,8 +225,7 @@ mean_final_block_kernel(const float* __restrict__ partial, int G, int D, double 
     }
     __syncthreads();
     if (t == 0) {
-        double a = 0.0;
-        float m = 0.f;
+        float a = 0.f, m = 0.f;
         for (int w = 0; w < W; ++w) {
             a += red_s[w];
             m = fmaxf(m, red_m[w]);
@@ -233,34 +234,25 @@ mean_final_block_kernel(const float* __restrict__ partial, int G, int D, double 
     }
 }
 
-// Few partials per coordinate (the small problems of a batch): one warp per
-// item instead of one block.
+// Few partials per coordinate (the small problems of a batch): one thread
+// per item = (problem b, coordinate d), folding the G partials in order.
 __global__ void __launch_bounds__(kMeanFinalThreads)
-mean_final_kernel(const float* __restrict__ partial, int G, int D, int64_t items, double total,
+mean_final_kernel(const float* __restrict__ partial, int G, int D, int64_t items, float total,
                   int mant_bits, int min_exp, float* __restrict__ mu) {
     pdl_trigger();
     pdl_wait();
-    // One warp per (problem b, coordinate d), item = b D + d: lane l folds
-    // partials l, l + 32, ... in order, then a fixed butterfly adds the
-    // lanes (deterministic).
-    const int64_t it = (static_cast<int64_t>(blockIdx.x) * kMeanFinalThreads + threadIdx.x) >> 5;
-    const int lane = threadIdx.x & 31;
-    if (it >= items) return;                       // whole warps leave together
+    const int64_t it = static_cast<int64_t>(blockIdx.x) * kMeanFinalThreads + threadIdx.x;
+    if (it >= items) return;
     const int64_t b = it / D;
     const int d = static_cast<int>(it - b * D);
     partial += b * 2 * G * D;                      // problem b
-    double s = 0.0;
+    float s = 0.f;
     float mx = 0.f;
-    for (int g = lane; g < G; g += 32) {
-        s += static_cast<double>(partial[static_cast<int64_t>(g) * D + d]);
+    for (int g = 0; g < G; ++g) {
+        s += partial[static_cast<int64_t>(g) * D + d];
         mx = fmaxf(mx, partial[static_cast<int64_t>(G + g) * D + d]);
     }
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) {
-        s += __shfl_xor_sync(0xffffffffu, s, o);
-        mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
-    }
-    if (lane == 0) mu[it] = rounded_mean(s, mx, total, mant_bits, min_exp);
+    mu[it] = rounded_mean(s, mx, total, mant_bits, min_exp);
 }
 
 // ---------------------------------------------------------------- MMA operands
@@ -646,18 +638,20 @@ struct OperandJob {
 constexpr int kOperandRows = 4;
 
 // Vector path of the operand preparation (D a multiple of 8): blocks
-// [0, blocks0) convert the rows of job j0, the rest those of j1 (the keys,
-// when they are not the queries), so that both arrays take one launch.
-// Index arithmetic is 32-bit (the planner keeps batch x rows_pad below
-// 2^31); with one problem the lane's mean pairs are loaded once.
+// [0, blocks0) of grid row b convert rows of job j0 of problem b, the rest
+// those of j1 (the keys, when they are not the queries), so that both
+// arrays of every problem take one launch.  A block never straddles two
+// problems, so the lane's mean pairs are loaded once and no row index is
+// divided; indices are 32-bit (the planner keeps batch x rows_pad below
+// 2^30).
 template <typename T, bool AUG, int G>
 __global__ void __launch_bounds__(kOperandVecThreads)
-operand_vec_kernel(const OperandJob j0, const OperandJob j1, unsigned blocks0, int batch,
-                   int D, int Dp, int nt, float F, const float* __restrict__ mu, float half_c,
-                   float pad_value) {
+operand_vec_kernel(const OperandJob j0, const OperandJob j1, unsigned blocks0, int D, int Dp,
+                   int nt, float F, const float* __restrict__ mu, float half_c, float pad_value) {
     pdl_trigger();
     pdl_wait();
     constexpr int SLOTS = kOperandVecThreads / G;   // rows of a block per step
+    const int b = blockIdx.y;                        // problem of the batch
     const bool second = blockIdx.x >= blocks0;
     const OperandJob j = second ? j1 : j0;
     const int blk = static_cast<int>(second ? blockIdx.x - blocks0 : blockIdx.x);
@@ -665,38 +659,29 @@ operand_vec_kernel(const OperandJob j0, const OperandJob j1, unsigned blocks0, i
     const int slot = threadIdx.x / G;
     const int rows_pad = static_cast<int>(j.rows_pad);
     const int rows = static_cast<int>(j.rows);
-    const int total = rows_pad * batch;
-    const T* x = static_cast<const T*>(j.x);
+    const T* x = static_cast<const T*>(j.x) + static_cast<int64_t>(b) * rows * D;
     const bool wq = AUG ? j.out_q != nullptr : true;
     const bool wk = AUG && j.out_k != nullptr;
-    const uint4 m_one = (batch == 1 && vi < D / 8) ? mean_pairs<T>(mu, vi) : make_uint4(0u, 0u, 0u, 0u);
+    const uint4 m2 = vi < D / 8 ? mean_pairs<T>(mu ? mu + static_cast<int64_t>(b) * D : nullptr, vi)
+                                : make_uint4(0u, 0u, 0u, 0u);
     uint4 in[kOperandRows];
 #pragma unroll
     for (int u = 0; u < kOperandRows; ++u) {
-        // Output row of the batch-stacked operand (batch rows_pad rows per
-        // problem); problem b reads rows b rows .. of x and its own mean.
-        const int row = (blk * kOperandRows + u) * SLOTS + slot;
-        const int b = batch == 1 ? 0 : row / rows_pad;
-        const int i = row - b * rows_pad;
-        const bool valid = row < total && i < rows;
-        in[u] = (valid && vi < D / 8)
-                    ? *reinterpret_cast<const uint4*>(x + (static_cast<int64_t>(b) * rows + i) * D + 8 * vi)
+        const int i = (blk * kOperandRows + u) * SLOTS + slot;   // row of problem b
+        in[u] = (i < rows && vi < D / 8)
+                    ? *reinterpret_cast<const uint4*>(x + static_cast<int64_t>(i) * D + 8 * vi)
                     : make_uint4(0u, 0u, 0u, 0u);
     }
 #pragma unroll
     for (int u = 0; u < kOperandRows; ++u) {
-        const int row = (blk * kOperandRows + u) * SLOTS + slot;
-        const int b = batch == 1 ? 0 : row / rows_pad;
-        const int i = row - b * rows_pad;
-        const bool in_pad = row < total;
-        const bool valid = in_pad && i < rows;
-        const uint4 m2 = (batch == 1 || !(in_pad && vi < D / 8))
-                             ? m_one
-                             : mean_pairs<T>(mu ? mu + static_cast<int64_t>(b) * D : nullptr, vi);
+        const int i = (blk * kOperandRows + u) * SLOTS + slot;
+        const bool in_pad = i < rows_pad;
+        const bool valid = i < rows;
+        const int64_t row = static_cast<int64_t>(b) * rows_pad + i;  // batch-stacked output row
         const float n = operand_row<T, AUG, G>(
             in[u], m2, vi, in_pad, valid, D, Dp, nt, F, half_c, pad_value,
-            wq ? static_cast<T*>(j.out_q) + static_cast<int64_t>(row) * Dp : nullptr,
-            wk ? static_cast<T*>(j.out_k) + static_cast<int64_t>(row) * Dp : nullptr);
+            wq ? static_cast<T*>(j.out_q) + row * Dp : nullptr,
+            wk ? static_cast<T*>(j.out_k) + row * Dp : nullptr);
         if (!AUG && in_pad && vi == 0) j.nrm[row] = n;
     }
 }
@@ -718,13 +703,13 @@ cudaError_t operand_typed(const OperandJob& j0, const OperandJob* j1, int D, int
         const int V = D / 8;
         const int G = V <= 1 ? 1 : V <= 2 ? 2 : V <= 4 ? 4 : V <= 8 ? 8 : V <= 16 ? 16 : 32;
         const int64_t per_block = static_cast<int64_t>(kOperandVecThreads / G) * kOperandRows;
-        const int64_t b0 = (j0.rows_pad * batch + per_block - 1) / per_block;
-        const int64_t b1 = j1 ? (j1->rows_pad * batch + per_block - 1) / per_block : 0;
-        if (b0 + b1 == 0) return cudaSuccess;
+        const int64_t b0 = (j0.rows_pad + per_block - 1) / per_block;
+        const int64_t b1 = j1 ? (j1->rows_pad + per_block - 1) / per_block : 0;
+        if (b0 + b1 == 0 || batch == 0) return cudaSuccess;
         auto go = [&](auto kern) {
-            launch_kernel(kern, static_cast<unsigned>(b0 + b1), kOperandVecThreads, 0, s, j0,
-                          j1 ? *j1 : none, static_cast<unsigned>(b0), batch, D, Dp, nt, F, mu,
-                          half_c, pad_value);
+            launch_kernel(kern, dim3(static_cast<unsigned>(b0 + b1), static_cast<unsigned>(batch)),
+                          kOperandVecThreads, 0, s, j0, j1 ? *j1 : none, static_cast<unsigned>(b0),
+                          D, Dp, nt, F, mu, half_c, pad_value);
         };
         switch (G) {
             case 1: go(operand_vec_kernel<T, AUG, 1>); break;
@@ -1111,15 +1096,14 @@ cudaError_t launch_mean(InType t, const void* q, const void* k, int64_t M, int64
     if (e != cudaSuccess) return e;
     const int mant_bits = t == InType::F16 ? 10 : t == InType::BF16 ? 7 : 23;
     const int min_exp = t == InType::F16 ? -24 : t == InType::BF16 ? -133 : -149;
-    if (G > kMeanFinalWarpMax) {
+    if (G > kMeanFinalThreadMax) {
         launch_kernel(mean_final_block_kernel, dim3(D, batch), kMeanFinalThreads, 0, s, partial,
-                      G, D, static_cast<double>(total), mant_bits, min_exp, mu);
+                      G, D, static_cast<float>(total), mant_bits, min_exp, mu);
     } else {
         const int64_t items = static_cast<int64_t>(batch) * D;
-        const int64_t warps_per_block = kMeanFinalThreads / 32;
         launch_kernel(mean_final_kernel,
-                      dim3(static_cast<unsigned>((items + warps_per_block - 1) / warps_per_block)),
-                      kMeanFinalThreads, 0, s, partial, G, D, items, static_cast<double>(total),
+                      dim3(static_cast<unsigned>((items + kMeanFinalThreads - 1) / kMeanFinalThreads)),
+                      kMeanFinalThreads, 0, s, partial, G, D, items, static_cast<float>(total),
                       mant_bits, min_exp, mu);
     }
     note_launches(1);
