@@ -513,57 +513,54 @@ template <> struct Pair<__nv_bfloat16> {
     static __device__ __forceinline__ P from_f2(float lo, float hi) { return __floats2bfloat162_rn(lo, hi); }
 };
 
-// The mean of coordinates 8 vi .. 8 vi + 7 as four packed pairs of the input
-// format (exact: the mean lies on the input grid), or zeros.
-template <typename T>
-__device__ __forceinline__ uint4 mean_pairs(const float* __restrict__ mu, int vi) {
-    using PT = Pair<T>;
-    if (!mu) return make_uint4(0u, 0u, 0u, 0u);
-    const float4 m0 = *reinterpret_cast<const float4*>(mu + 8 * vi);
-    const float4 m1 = *reinterpret_cast<const float4*>(mu + 8 * vi + 4);
-    typename PT::P p[4] = {PT::from_f2(m0.x, m0.y), PT::from_f2(m0.z, m0.w),
-                           PT::from_f2(m1.x, m1.y), PT::from_f2(m1.z, m1.w)};
-    return *reinterpret_cast<const uint4*>(p);
-}
-
 // One output row of the operand layouts, converted by the G lanes of a
-// row group (lane vi: coordinates 8 vi .. 8 vi + 7, one 16-byte vector).
-// in: lane vi's input vector of the row (used only when `valid` and
-// vi < D / 8); m2: the row problem's mean pairs (mean_pairs); out_q /
-// out_k: the row in either layout (either may be null; AUG only).  Every
-// lane of the warp must call this together (the squared norm is reduced
-// with shuffles over the G lanes); rows outside the output (in_pad false)
-// write nothing.  Returns the norm term written for the row (plain layout:
-// -(c/2)||x^||^2, or pad_value) in every lane.
+// row group: lane vi holds the row's 16-byte input vectors vi, vi + G, ...
+// (in[e] = vector vi + G e, 8 coordinates each, for vi + G e < D / 8; up to
+// kOperandVecs of them) and smean the problem's mean as packed pairs of the
+// input format in shared memory (exact: the mean lies on the input grid).
+// out_q / out_k: the row in either layout (either may be null; AUG only).
+// Every lane of the warp must call this together (the squared norm is
+// reduced with shuffles over the G lanes); rows outside the output (in_pad
+// false) write nothing.  Returns the norm term written for the row (plain
+// layout: -(c/2)||x^||^2, or pad_value) in every lane.
+constexpr int kOperandVecs = 8;
+
 template <typename T, bool AUG, int G>
-__device__ __forceinline__ float operand_row(const uint4 in, const uint4 m2, int vi,
+__device__ __forceinline__ float operand_row(const uint4 (&in)[kOperandVecs],
+                                             const uint4* __restrict__ smean, int vi,
                                              bool in_pad, bool valid, int D, int Dp, int nt,
                                              float F, float half_c, float pad_value,
                                              T* __restrict__ out_q, T* __restrict__ out_k) {
     using PT = Pair<T>;
     const int V = D / 8;
     float acc = 0.f;
-    if (in_pad && vi < V) {
-        uint4 u = make_uint4(0u, 0u, 0u, 0u);
-        if (valid) {
-            const typename PT::P* x2 = reinterpret_cast<const typename PT::P*>(&in);
-            const typename PT::P* mm = reinterpret_cast<const typename PT::P*>(&m2);
-            typename PT::P h[4];
-            uint64_t acc2 = 0ull;
+    if (in_pad) {
+        uint64_t acc2 = 0ull;
 #pragma unroll
-            for (int e = 0; e < 4; ++e) {
-                h[e] = PT::sub(x2[e], mm[e]);
-                const float2 f = PT::to_f2(h[e]);
-                const uint64_t f2 = f32x2_pack(f.x, f.y);
-                acc2 = f32x2_fma(f2, f2, acc2);
+        for (int e = 0; e < kOperandVecs; ++e) {
+            const int v = vi + G * e;
+            if (v >= V) break;
+            uint4 u = make_uint4(0u, 0u, 0u, 0u);
+            if (valid) {
+                const uint4 m2 = smean[v];
+                const typename PT::P* x2 = reinterpret_cast<const typename PT::P*>(&in[e]);
+                const typename PT::P* mm = reinterpret_cast<const typename PT::P*>(&m2);
+                typename PT::P h[4];
+#pragma unroll
+                for (int k = 0; k < 4; ++k) {
+                    h[k] = PT::sub(x2[k], mm[k]);
+                    const float2 f = PT::to_f2(h[k]);
+                    const uint64_t f2 = f32x2_pack(f.x, f.y);
+                    acc2 = f32x2_fma(f2, f2, acc2);
+                }
+                u = *reinterpret_cast<const uint4*>(h);
             }
-            float lo, hi;
-            f32x2_unpack(acc2, lo, hi);
-            acc = lo + hi;
-            u = *reinterpret_cast<const uint4*>(h);
+            if (out_q) *reinterpret_cast<uint4*>(out_q + 8 * v) = u;
+            if (out_k) *reinterpret_cast<uint4*>(out_k + 8 * v) = u;
         }
-        if (out_q) *reinterpret_cast<uint4*>(out_q + 8 * vi) = u;
-        if (out_k) *reinterpret_cast<uint4*>(out_k + 8 * vi) = u;
+        float lo, hi;
+        f32x2_unpack(acc2, lo, hi);
+        acc = lo + hi;
     }
 #pragma unroll
     for (int o = G / 2; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o, G);
@@ -633,57 +630,57 @@ struct OperandJob {
     float* nrm;
 };
 
-// Rows per thread of operand_vec_kernel: their input vectors are loaded
-// before any is converted, so that several loads are in flight per thread.
-constexpr int kOperandRows = 4;
-
-// Vector path of the operand preparation (D a multiple of 8): blocks
-// [0, blocks0) of grid row b convert rows of job j0 of problem b, the rest
-// those of j1 (the keys, when they are not the queries), so that both
-// arrays of every problem take one launch.  A block never straddles two
-// problems, so the lane's mean pairs are loaded once and no row index is
-// divided; indices are 32-bit (the planner keeps batch x rows_pad below
-// 2^30).
+// Vector path of the operand preparation (D a multiple of 8): G lanes per
+// row (G = 1 up to D = 64, 2 up to 128, 4 up to 256), each lane converting
+// up to eight 16-byte vectors of its row, all loaded before any is
+// converted; so every lane of a warp does its own row's work (no lanes idle
+// during the norm split) and has up to 128 bytes of loads in flight.
+// Blocks [0, blocks0) of grid row b convert rows of job j0 of problem b,
+// the rest those of j1 (the keys, when they are not the queries), so that
+// both arrays of every problem take one launch; a block never straddles
+// two problems.  The problem's mean is staged once per block in shared
+// memory as packed pairs of the input format.
 template <typename T, bool AUG, int G>
 __global__ void __launch_bounds__(kOperandVecThreads)
 operand_vec_kernel(const OperandJob j0, const OperandJob j1, unsigned blocks0, int D, int Dp,
                    int nt, float F, const float* __restrict__ mu, float half_c, float pad_value) {
+    using PT = Pair<T>;
     pdl_trigger();
     pdl_wait();
-    constexpr int SLOTS = kOperandVecThreads / G;   // rows of a block per step
+    constexpr int SLOTS = kOperandVecThreads / G;   // rows of a block
+    __shared__ uint4 smean[kOperandMaxCols / 8];
     const int b = blockIdx.y;                        // problem of the batch
     const bool second = blockIdx.x >= blocks0;
     const OperandJob j = second ? j1 : j0;
     const int blk = static_cast<int>(second ? blockIdx.x - blocks0 : blockIdx.x);
-    const int vi = threadIdx.x % G;                  // vector within the row
+    const int vi = threadIdx.x % G;                  // first vector of this lane
     const int slot = threadIdx.x / G;
+    const int V = D / 8;
     const int rows_pad = static_cast<int>(j.rows_pad);
     const int rows = static_cast<int>(j.rows);
-    const T* x = static_cast<const T*>(j.x) + static_cast<int64_t>(b) * rows * D;
+    const int i = blk * SLOTS + slot;                // row of problem b
+    const T* xr = static_cast<const T*>(j.x) + (static_cast<int64_t>(b) * rows + i) * D;
+    uint4 in[kOperandVecs];
+#pragma unroll
+    for (int e = 0; e < kOperandVecs; ++e) {
+        const int v = vi + G * e;
+        in[e] = (i < rows && v < V) ? *reinterpret_cast<const uint4*>(xr + 8 * v)
+                                    : make_uint4(0u, 0u, 0u, 0u);
+    }
+    const float* mb = mu ? mu + static_cast<int64_t>(b) * D : nullptr;
+    typename PT::P* sm = reinterpret_cast<typename PT::P*>(smean);
+    for (int c = threadIdx.x; c < D / 2; c += kOperandVecThreads)
+        sm[c] = mb ? PT::from_f2(mb[2 * c], mb[2 * c + 1]) : PT::from_f2(0.f, 0.f);
+    __syncthreads();
     const bool wq = AUG ? j.out_q != nullptr : true;
     const bool wk = AUG && j.out_k != nullptr;
-    const uint4 m2 = vi < D / 8 ? mean_pairs<T>(mu ? mu + static_cast<int64_t>(b) * D : nullptr, vi)
-                                : make_uint4(0u, 0u, 0u, 0u);
-    uint4 in[kOperandRows];
-#pragma unroll
-    for (int u = 0; u < kOperandRows; ++u) {
-        const int i = (blk * kOperandRows + u) * SLOTS + slot;   // row of problem b
-        in[u] = (i < rows && vi < D / 8)
-                    ? *reinterpret_cast<const uint4*>(x + static_cast<int64_t>(i) * D + 8 * vi)
-                    : make_uint4(0u, 0u, 0u, 0u);
-    }
-#pragma unroll
-    for (int u = 0; u < kOperandRows; ++u) {
-        const int i = (blk * kOperandRows + u) * SLOTS + slot;
-        const bool in_pad = i < rows_pad;
-        const bool valid = i < rows;
-        const int64_t row = static_cast<int64_t>(b) * rows_pad + i;  // batch-stacked output row
-        const float n = operand_row<T, AUG, G>(
-            in[u], m2, vi, in_pad, valid, D, Dp, nt, F, half_c, pad_value,
-            wq ? static_cast<T*>(j.out_q) + row * Dp : nullptr,
-            wk ? static_cast<T*>(j.out_k) + row * Dp : nullptr);
-        if (!AUG && in_pad && vi == 0) j.nrm[row] = n;
-    }
+    const bool in_pad = i < rows_pad;
+    const int64_t row = static_cast<int64_t>(b) * rows_pad + i;   // batch-stacked output row
+    const float n = operand_row<T, AUG, G>(
+        in, smean, vi, in_pad, i < rows, D, Dp, nt, F, half_c, pad_value,
+        wq ? static_cast<T*>(j.out_q) + row * Dp : nullptr,
+        wk ? static_cast<T*>(j.out_k) + row * Dp : nullptr);
+    if (!AUG && in_pad && vi == 0) j.nrm[row] = n;
 }
 
 template <typename T, bool AUG>
@@ -699,10 +696,11 @@ cudaError_t operand_typed(const OperandJob& j0, const OperandJob* j1, int D, int
     // The vector path indexes rows with 32-bit integers.
     const int64_t most_rows = std::max(j0.rows_pad, j1 ? j1->rows_pad : int64_t(0)) * batch;
     if (D % 8 == 0 && D >= 8 && (!AUG || Dp - D >= 2 * nt) && most_rows < (int64_t(1) << 30)) {
-        // Vector path: G lanes per row, both arrays in one launch.
+        // Vector path: G lanes per row (up to kOperandVecs vectors each),
+        // both arrays in one launch.
         const int V = D / 8;
-        const int G = V <= 1 ? 1 : V <= 2 ? 2 : V <= 4 ? 4 : V <= 8 ? 8 : V <= 16 ? 16 : 32;
-        const int64_t per_block = static_cast<int64_t>(kOperandVecThreads / G) * kOperandRows;
+        const int G = V <= kOperandVecs ? 1 : V <= 2 * kOperandVecs ? 2 : 4;
+        const int64_t per_block = kOperandVecThreads / G;
         const int64_t b0 = (j0.rows_pad + per_block - 1) / per_block;
         const int64_t b1 = j1 ? (j1->rows_pad + per_block - 1) / per_block : 0;
         if (b0 + b1 == 0 || batch == 0) return cudaSuccess;
@@ -714,10 +712,7 @@ cudaError_t operand_typed(const OperandJob& j0, const OperandJob* j1, int D, int
         switch (G) {
             case 1: go(operand_vec_kernel<T, AUG, 1>); break;
             case 2: go(operand_vec_kernel<T, AUG, 2>); break;
-            case 4: go(operand_vec_kernel<T, AUG, 4>); break;
-            case 8: go(operand_vec_kernel<T, AUG, 8>); break;
-            case 16: go(operand_vec_kernel<T, AUG, 16>); break;
-            default: go(operand_vec_kernel<T, AUG, 32>); break;
+            default: go(operand_vec_kernel<T, AUG, 4>); break;
         }
         note_launches(1);
         return cudaGetLastError();
