@@ -310,7 +310,8 @@ def probe_fp16_tflops(dev):
     return best
 
 
-def roofline_of(w, main_ms, peaks, peak_src, sms, r_x, traffic=None, traffic_src=None):
+def roofline_of(w, main_ms, peaks, peak_src, sms, r_x, traffic=None, traffic_src=None,
+                r_mix=None):
     """Roofline of the fused kernel (algorithmic work, unpadded D and C; the
     gradient evaluates C' = D + 1 value channels): the slower of dense tensor
     work 2 M N (D + C) at the measured bf16 peak (fp16 runs at the bf16
@@ -348,6 +349,12 @@ def roofline_of(w, main_ms, peaks, peak_src, sms, r_x, traffic=None, traffic_src
         "sfu": {"achieved": exps / t_main / 1e12, "peak": r_x_nominal / 1e12,
                 "unit": "Texp/s", "frac": t_sfu / t_main, "probe_ex2_per_s": r_x},
     })
+    if r_mix and main_kernel_name(w) == "tc_gauss_fma_kernel" and roof["bound"] == "alu":
+        # The exp2 rate that the FMA kernel's own exponent-loop instruction
+        # mix reaches without tiles, barriers or tensor-memory traffic
+        # (gauss_sum_probe_ex2_mix_rate): the practical ceiling of that loop.
+        roof["sfu"]["mix_ceiling_per_s"] = r_mix
+        roof["sfu"]["frac_of_mix_ceiling"] = exps / t_main / r_mix
     return roof
 
 
@@ -499,6 +506,7 @@ def run_own(args):
     # Roofline denominators.
     peaks, peak_src = measured_peaks()
     r_x = gs.gauss_sum_probe_ex2_rate()
+    r_mix = gs.gauss_sum_probe_ex2_mix_rate()
     props = torch.cuda.get_device_properties(dev)
     sms = props.multi_processor_count
 
@@ -528,7 +536,7 @@ def run_own(args):
     clocks = sampler.stop() if sampler is not None else None
 
     traffic, traffic_src = profiled_traffic(w)
-    roof = roofline_of(w, main_mean, peaks, peak_src, sms, r_x, traffic, traffic_src)
+    roof = roofline_of(w, main_mean, peaks, peak_src, sms, r_x, traffic, traffic_src, r_mix)
 
     # The other configurations, measured the same way (fewer steps) so that
     # every configuration has a number from this run.
@@ -544,7 +552,7 @@ def run_own(args):
                 s_ms, m_ms, n_l = ro.timed(min(K, 20), W)
                 tr, tr_src = profiled_traffic(wo)
                 rf = roofline_of(wo, statistics.mean(m_ms), peaks, peak_src, sms, r_x, tr,
-                                 tr_src)
+                                 tr_src, r_mix=r_mix)
                 others[name] = {
                     "config": workload_config(wo), "steps": len(s_ms),
                     "ms_per_step": statistics.mean(s_ms), "value": wo.pairs / (statistics.mean(s_ms) * 1e-3),

@@ -271,6 +271,17 @@ gs_status gauss_sum_noalloc(const void* q, const void* k, const void* v, double 
 gs_status gauss_sum_probe_ex2_rate(void* stream, double* exp2_per_second);
 
 /*
+ * Measurement helper (not part of Eq. 1): the exp2 rate that the instruction
+ * mix of the fused FMA kernel's exponent loop can reach, in exponentials
+ * per second: per key pair and two query rows two paired multiplies by c,
+ * four ex2.approx, one broadcast shared-memory load of the pair's values and
+ * two paired FMAs, on four warps per SMSP like the kernel's exponent warps,
+ * without its tensor-memory loads, barriers or MMAs.  Synchronises
+ * `stream`.  Reported beside the MUFU rate as the ceiling of that loop.
+ */
+gs_status gauss_sum_probe_ex2_mix_rate(void* stream, double* exp2_per_second);
+
+/*
  * Accounting helper (not part of Eq. 1): number of CUDA kernels this
  * library has launched in this process, over all devices and streams,
  * counted on the host at each launch.  Never fails.

@@ -9,7 +9,8 @@ raise instead of falling back to anything else.
 from ._binding import (GS_BF16, GS_FP16, GS_FP32, GS_PATH_AUTO, GS_PATH_SIMT, GS_PATH_TENSOR,
                        EXPORTS, GaussSumError, gauss_sum, gauss_sum_batched, gauss_sum_device_status,
                        gauss_sum_mmd2, gauss_sum_noalloc, gauss_sum_vjp,
-                       gauss_sum_grad_q, gauss_sum_kernel_launches, gauss_sum_probe_ex2_rate,
+                       gauss_sum_grad_q, gauss_sum_kernel_launches, gauss_sum_probe_ex2_mix_rate,
+                       gauss_sum_probe_ex2_rate,
                        gauss_sum_workspace_size,
                        library_path, load_library)
 
@@ -17,6 +18,6 @@ __all__ = [
     "GS_BF16", "GS_FP16", "GS_FP32", "GS_PATH_AUTO", "GS_PATH_SIMT", "GS_PATH_TENSOR",
     "EXPORTS", "GaussSumError", "gauss_sum", "gauss_sum_device_status", "gauss_sum_grad_q",
     "gauss_sum_batched", "gauss_sum_kernel_launches", "gauss_sum_mmd2", "gauss_sum_noalloc",
-    "gauss_sum_probe_ex2_rate", "gauss_sum_vjp", "gauss_sum_workspace_size", "library_path",
+    "gauss_sum_probe_ex2_mix_rate", "gauss_sum_probe_ex2_rate", "gauss_sum_vjp", "gauss_sum_workspace_size", "library_path",
     "load_library",
 ]

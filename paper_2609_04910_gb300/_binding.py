@@ -26,7 +26,7 @@ EXPORTS = (
     "gauss_sum_grad_q_ex", "gauss_sum_workspace_size", "gauss_sum_device_status",
     "gauss_sum_last_error", "gauss_sum_status_string", "gauss_sum_probe_ex2_rate",
     "gauss_sum_noalloc", "gauss_sum_kernel_launches", "gauss_sum_batched", "gauss_sum_mmd2",
-    "gauss_sum_vjp",
+    "gauss_sum_vjp", "gauss_sum_probe_ex2_mix_rate",
 )
 # Test hooks declared in include/gauss_sum_testing.h.
 TESTING_EXPORTS = ("gauss_sum_testing_fail_allocations", "gauss_sum_testing_request_stall")
@@ -101,6 +101,8 @@ def _declare(lib):
     lib.gauss_sum_status_string.restype = ctypes.c_char_p
     lib.gauss_sum_probe_ex2_rate.argtypes = [vp, ctypes.POINTER(ctypes.c_double)]
     lib.gauss_sum_probe_ex2_rate.restype = f
+    lib.gauss_sum_probe_ex2_mix_rate.argtypes = [vp, ctypes.POINTER(ctypes.c_double)]
+    lib.gauss_sum_probe_ex2_mix_rate.restype = f
     lib.gauss_sum_noalloc.argtypes = [vp, vp, vp, d, i64, i64, i64, i64, f, vp, vp]
     lib.gauss_sum_noalloc.restype = f
     lib.gauss_sum_kernel_launches.argtypes = []
@@ -330,6 +332,15 @@ def gauss_sum_probe_ex2_rate(stream=None) -> float:
     lib = load_library()
     r = ctypes.c_double(0.0)
     _check(lib, lib.gauss_sum_probe_ex2_rate(_stream_ptr(stream), ctypes.byref(r)))
+    return r.value
+
+
+def gauss_sum_probe_ex2_mix_rate(stream=None) -> float:
+    """exp2 rate reachable with the FMA kernel's exponent-loop instruction
+    mix (see include/gauss_sum.h), in exponentials per second."""
+    lib = load_library()
+    r = ctypes.c_double(0.0)
+    _check(lib, lib.gauss_sum_probe_ex2_mix_rate(_stream_ptr(stream), ctypes.byref(r)))
     return r.value
 
 

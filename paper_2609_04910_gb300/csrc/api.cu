@@ -502,6 +502,54 @@ __global__ void ex2_probe_kernel(float* out, int iters) {
     out[blockIdx.x * blockDim.x + threadIdx.x] = s;
 }
 
+// The FMA kernel's exponent loop without its tiles: per key pair and two
+// query rows two paired multiplies by c (here paired FMAs that also add a
+// per-iteration offset, so that no exponential is loop invariant and none
+// can be hoisted out of the loop), four ex2.approx (-|x| form), one
+// broadcast 8-byte shared-memory load of the pair's values and two paired
+// FMAs, on 16 warps per SM (the kernel's exponent warps: four per SMSP), no
+// tensor-memory traffic or barriers.  Measures the exp2 rate this
+// instruction mix can reach.
+
+constexpr int kMixProbeThreads = 512;
+
+__global__ void __launch_bounds__(kMixProbeThreads, 1) ex2_mix_probe_kernel(float* out, int iters,
+                                                                            float c) {
+    __shared__ float2 vals[64];
+    if (threadIdx.x < 64)
+        vals[threadIdx.x] = make_float2(1e-3f * threadIdx.x, -1e-3f * threadIdx.x);
+    __syncthreads();
+    float s0[16], s1[16];
+#pragma unroll
+    for (int i = 0; i < 16; ++i) {
+        s0[i] = -0.01f * static_cast<float>(threadIdx.x + i);
+        s1[i] = -0.02f * static_cast<float>(threadIdx.x + i);
+    }
+    const uint64_t c2 = gs::f32x2_pack(c, c);
+    uint64_t a0 = 0ull, a1 = 0ull;
+    float off = 0.f;
+    for (int it = 0; it < iters; ++it) {
+        off -= 1e-7f;
+        const uint64_t o2 = gs::f32x2_pack(off, off);
+#pragma unroll
+        for (int t = 0; t < 8; ++t) {
+            float x0, x1, y0, y1;
+            gs::f32x2_unpack(gs::f32x2_fma(gs::f32x2_pack(s0[2 * t], s0[2 * t + 1]), c2, o2), x0, x1);
+            gs::f32x2_unpack(gs::f32x2_fma(gs::f32x2_pack(s1[2 * t], s1[2 * t + 1]), c2, o2), y0, y1);
+            const uint64_t px = gs::f32x2_pack(gs::ex2_nonpos(x0), gs::ex2_nonpos(x1));
+            const uint64_t py = gs::f32x2_pack(gs::ex2_nonpos(y0), gs::ex2_nonpos(y1));
+            const float2 v = vals[(t + it) & 63];
+            const uint64_t vv = gs::f32x2_pack(v.x, v.y);
+            a0 = gs::f32x2_fma(px, vv, a0);
+            a1 = gs::f32x2_fma(py, vv, a1);
+        }
+    }
+    float u0, u1, w0, w1;
+    gs::f32x2_unpack(a0, u0, u1);
+    gs::f32x2_unpack(a1, w0, w1);
+    out[blockIdx.x * blockDim.x + threadIdx.x] = u0 + u1 + w0 + w1;
+}
+
 }  // namespace
 
 namespace gs {
@@ -528,13 +576,16 @@ gs_status set_last_error(gs_status st, const char* msg) { return fail(st, "%s", 
 
 void note_launches(int n) { g_launches.fetch_add(static_cast<uint64_t>(n), std::memory_order_relaxed); }
 
-cudaError_t run_ex2_probe(cudaStream_t s, double* rate) {
+cudaError_t run_ex2_probe(cudaStream_t s, double* rate, bool mix) {
     int dev = 0;
     cudaError_t e = cudaGetDevice(&dev);
     if (e != cudaSuccess) return e;
     int sms = 1;
     cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-    const int blocks = sms * 4, threads = 512, iters = 4096;
+    // Plain: independent ex2 chains on 64 warps per SM; mix: the FMA
+    // kernel's loop on one block of 16 warps per SM.
+    const int blocks = mix ? sms : sms * 4, threads = mix ? kMixProbeThreads : 512;
+    const int iters = mix ? 2048 : 4096;
     float* out = nullptr;
     e = cudaMallocAsync(reinterpret_cast<void**>(&out), sizeof(float) * blocks * threads, s);
     if (e != cudaSuccess) return e;
@@ -544,14 +595,17 @@ cudaError_t run_ex2_probe(cudaStream_t s, double* rate) {
     double best = 0.0;
     for (int rep = 0; rep < 4; ++rep) {
         cudaEventRecord(e0, s);
-        ex2_probe_kernel<8><<<blocks, threads, 0, s>>>(out, iters);
+        if (mix)
+            ex2_mix_probe_kernel<<<blocks, threads, 0, s>>>(out, iters, 0.0225f);
+        else
+            ex2_probe_kernel<8><<<blocks, threads, 0, s>>>(out, iters);
         note_launches(1);
         cudaEventRecord(e1, s);
         e = cudaEventSynchronize(e1);
         if (e != cudaSuccess) break;
         float ms = 0.f;
         cudaEventElapsedTime(&ms, e0, e1);
-        const double n = static_cast<double>(blocks) * threads * iters * 8;
+        const double n = static_cast<double>(blocks) * threads * iters * (mix ? 32 : 8);
         if (rep > 0 && ms > 0.f) best = std::max(best, n / (ms * 1e-3));
     }
     cudaEventDestroy(e0);
@@ -783,8 +837,15 @@ gs_status gauss_sum_testing_request_stall(void* stream) {
 
 gs_status gauss_sum_probe_ex2_rate(void* stream, double* exp2_per_second) {
     if (!exp2_per_second) return fail(GS_ERR_INVALID_ARGUMENT, "null output pointer");
-    cudaError_t e = gs::run_ex2_probe(static_cast<cudaStream_t>(stream), exp2_per_second);
+    cudaError_t e = gs::run_ex2_probe(static_cast<cudaStream_t>(stream), exp2_per_second, false);
     if (e != cudaSuccess) return cuda_fail(e, "ex2 probe");
+    return GS_OK;
+}
+
+gs_status gauss_sum_probe_ex2_mix_rate(void* stream, double* exp2_per_second) {
+    if (!exp2_per_second) return fail(GS_ERR_INVALID_ARGUMENT, "null output pointer");
+    cudaError_t e = gs::run_ex2_probe(static_cast<cudaStream_t>(stream), exp2_per_second, true);
+    if (e != cudaSuccess) return cuda_fail(e, "ex2 mix probe");
     return GS_OK;
 }
 

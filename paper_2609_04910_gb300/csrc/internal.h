@@ -229,7 +229,9 @@ cudaError_t launch_tc_fma(const TcPlan& p, InType t, float c, char* ws, unsigned
                           cudaStream_t s, const char** why);
 
 // probe
-cudaError_t run_ex2_probe(cudaStream_t s, double* rate);
+// Best of three timed runs of the ex2 probe kernel: independent ex2 chains
+// (mix false), or the FMA kernel's exponent-loop instruction mix (true).
+cudaError_t run_ex2_probe(cudaStream_t s, double* rate, bool mix);
 
 // api.cu: workspace bytes that a forward call with exactly these arguments
 // and default options needs (through *bytes), or the status the call

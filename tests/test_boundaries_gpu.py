@@ -78,3 +78,16 @@ def test_fp32_gradient_register_tiles(D):
 def test_fp32_tensor_variant_edges(D, C):
     import paper_2609_04910_gb300 as gs
     forward_check(case(130, 257, D, C, "fp32"), path=gs.GS_PATH_TENSOR)
+
+
+def test_ex2_rate_probes():
+    """The MUFU probe stays below 32 exp2 per clock per SM at a 2.2 GHz
+    bound, and the probe of the FMA kernel's exponent-loop instruction mix
+    (which adds multiplies, loads and FMAs to every exp2) does not exceed it."""
+    import torch
+    import paper_2609_04910_gb300 as gs
+    sms = torch.cuda.get_device_properties(0).multi_processor_count
+    plain = gs.gauss_sum_probe_ex2_rate()
+    mix = gs.gauss_sum_probe_ex2_mix_rate()
+    assert 0 < plain <= 32 * sms * 2.2e9
+    assert 0 < mix <= 1.05 * plain
