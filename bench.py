@@ -435,38 +435,48 @@ class Runner:
         w, inp, dev = self.w, self.inp, self.dev
         stream = torch.cuda.current_stream()
 
-        def host(a):
-            a = np.ascontiguousarray(a)
-            return torch.from_numpy(a.view(np.int16) if w.dtype == "bf16" else a).pin_memory()
+        # The step's inputs live in one pinned host buffer and travel in one
+        # copy (q, k and v at 256-byte aligned offsets); the result comes
+        # back into a pinned host buffer.
+        arrays = [np.ascontiguousarray(inp["k"]), np.ascontiguousarray(inp["v"])]
+        if not w.q_is_k:
+            arrays.append(np.ascontiguousarray(inp["q"]))
+        offs, total = [], 0
+        for a in arrays:
+            offs.append(total)
+            total += (a.nbytes + 255) // 256 * 256
+        host = torch.empty(total, dtype=torch.uint8).pin_memory()
+        for a, o in zip(arrays, offs):
+            host[o:o + a.nbytes].copy_(torch.from_numpy(a.view(np.uint8).reshape(-1)))
+        devbuf = torch.empty(total, dtype=torch.uint8, device=dev)
+        tdt = {"fp16": torch.float16, "bf16": torch.bfloat16, "fp32": torch.float32}[w.dtype]
 
-        kh, vh = host(inp["k"]), host(inp["v"])
-        qh = kh if w.q_is_k else host(inp["q"])
-        kd = torch.empty_like(kh, device=dev)
-        vd = torch.empty_like(vh, device=dev)
-        qd = kd if w.q_is_k else torch.empty_like(qh, device=dev)
+        def view(i):
+            a = arrays[i]
+            return devbuf[offs[i]:offs[i] + a.nbytes].view(tdt).view(a.shape)
+
+        kd, vd = view(0), view(1)
+        qd = kd if w.q_is_k else view(2)
         outh = torch.empty(tuple(self.out.shape), dtype=torch.float32).pin_memory()
         sh = torch.empty((w.M,), dtype=torch.float32).pin_memory() if w.grad else None
-        conv = (lambda t: t.view(torch.bfloat16)) if w.dtype == "bf16" else (lambda t: t)
+        outd = torch.empty(tuple(self.out.shape), dtype=torch.float32, device=dev)
+        sd = torch.empty((w.M,), dtype=torch.float32, device=dev) if w.grad else None
         e_ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
                 for _ in range(K)]
-        h2d = kh.numel() * kh.element_size() + vh.numel() * vh.element_size() + \
-            (0 if w.q_is_k else qh.numel() * qh.element_size())
+        h2d = sum(a.nbytes for a in arrays)
         d2h = outh.numel() * 4 + (w.M * 4 if w.grad else 0)
         for i in range(K + W):
             self.flush.zero_()
             if i >= W:
                 e_ev[i - W][0].record(stream)
-            kd.copy_(kh, non_blocking=True)
-            vd.copy_(vh, non_blocking=True)
-            if not w.q_is_k:
-                qd.copy_(qh, non_blocking=True)
+            devbuf.copy_(host, non_blocking=True)
             if w.grad:
-                g, s_ = gs.gauss_sum_grad_q(conv(qd), conv(kd), conv(vd), w.tau)
-                outh.copy_(g, non_blocking=True)
-                sh.copy_(s_, non_blocking=True)
+                gs.gauss_sum_grad_q(qd, kd, vd, w.tau, grad=outd, s_out=sd)
+                outh.copy_(outd, non_blocking=True)
+                sh.copy_(sd, non_blocking=True)
             else:
-                o = gs.gauss_sum(conv(qd), conv(kd), conv(vd), w.tau)
-                outh.copy_(o, non_blocking=True)
+                gs.gauss_sum(qd, kd, vd, w.tau, out=outd)
+                outh.copy_(outd, non_blocking=True)
             if i >= W:
                 e_ev[i - W][1].record(stream)
         torch.cuda.synchronize()
