@@ -35,6 +35,15 @@ void gauss_sum_testing_fail_allocations(int on);
  */
 gs_status gauss_sum_testing_request_stall(void* stream);
 
+/*
+ * Bit flags describing the fused FMA kernel (C <= 4 forward) that the last
+ * call of this process launched: bit 0 = overlapped segment transitions
+ * (short runs of key tiles per pair of query tiles), bit 1 = banded key
+ * order, bit 2 = q^ in TMEM; -1 before the first such launch.  Lets the
+ * parity tests check that each side of a planning switch is exercised.
+ */
+int gauss_sum_testing_last_fma_variant(void);
+
 #ifdef __cplusplus
 }
 #endif

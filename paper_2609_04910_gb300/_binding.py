@@ -29,7 +29,8 @@ EXPORTS = (
     "gauss_sum_vjp", "gauss_sum_probe_ex2_mix_rate",
 )
 # Test hooks declared in include/gauss_sum_testing.h.
-TESTING_EXPORTS = ("gauss_sum_testing_fail_allocations", "gauss_sum_testing_request_stall")
+TESTING_EXPORTS = ("gauss_sum_testing_fail_allocations", "gauss_sum_testing_request_stall",
+                   "gauss_sum_testing_last_fma_variant")
 
 # Bytes of the static scratch array behind gauss_sum_noalloc
 # (GS_NOALLOC_SCRATCH_BYTES in include/gauss_sum.h).
@@ -117,6 +118,8 @@ def _declare(lib):
     lib.gauss_sum_testing_fail_allocations.restype = None
     lib.gauss_sum_testing_request_stall.argtypes = [vp]
     lib.gauss_sum_testing_request_stall.restype = f
+    lib.gauss_sum_testing_last_fma_variant.argtypes = []
+    lib.gauss_sum_testing_last_fma_variant.restype = f
 
 
 def _check(lib, status: int):
@@ -352,6 +355,13 @@ def gauss_sum_kernel_launches() -> int:
 def testing_fail_allocations(on: bool) -> None:
     """Test hook: make the library's workspace allocations fail (or not)."""
     load_library().gauss_sum_testing_fail_allocations(1 if on else 0)
+
+
+def testing_last_fma_variant() -> int:
+    """Bit flags of the last fused FMA-kernel launch (test hook): 1 =
+    overlapped segment transitions, 2 = banded key order, 4 = q^ in TMEM;
+    -1 before the first launch."""
+    return int(load_library().gauss_sum_testing_last_fma_variant())
 
 
 def testing_request_stall(stream=None) -> None:

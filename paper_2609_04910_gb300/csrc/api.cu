@@ -19,6 +19,7 @@ namespace {
 
 thread_local char g_last_error[512] = "no error";
 std::atomic<uint64_t> g_launches{0};
+std::atomic<int> g_last_fma_variant{-1};
 
 gs_status fail(gs_status st, const char* fmt, const char* detail = nullptr) {
     if (detail)
@@ -575,6 +576,7 @@ gs_status forward_workspace_bytes(const void* q, const void* k, const void* v, d
 gs_status set_last_error(gs_status st, const char* msg) { return fail(st, "%s", msg); }
 
 void note_launches(int n) { g_launches.fetch_add(static_cast<uint64_t>(n), std::memory_order_relaxed); }
+void note_fma_variant(int flags) { g_last_fma_variant.store(flags, std::memory_order_relaxed); }
 
 cudaError_t run_ex2_probe(cudaStream_t s, double* rate, bool mix) {
     int dev = 0;
@@ -817,6 +819,8 @@ const char* gauss_sum_status_string(gs_status s) {
 }
 
 uint64_t gauss_sum_kernel_launches(void) { return g_launches.load(std::memory_order_relaxed); }
+
+int gauss_sum_testing_last_fma_variant(void) { return g_last_fma_variant.load(std::memory_order_relaxed); }
 
 void gauss_sum_testing_fail_allocations(int on) {
     g_fail_allocations.store(on ? 1 : 0, std::memory_order_relaxed);

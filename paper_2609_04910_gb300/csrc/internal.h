@@ -94,6 +94,11 @@ struct TcPlan {
     // the number of bands (one partial-sum slot per band).
     int band_len;
     int64_t nruns;
+    // FMA kernel with short segments (runs of at most kOverlapMaxTiles key
+    // tiles per pair of query tiles): the control warps start the next
+    // segment's copies and MMAs while the exponent warps finish the current
+    // one, instead of meeting them at a CTA barrier at every segment end.
+    bool overlap;
     // Problems of a batch handled by one launch (the FMA kernel stacks them:
     // q^ batch x Mpad rows, k^ batch x Npad rows); 1 for the other paths.
     int64_t batch;
@@ -243,5 +248,8 @@ gs_status set_last_error(gs_status st, const char* msg);
 // Adds n to the count behind gauss_sum_kernel_launches(); called right
 // after each kernel launch of the library.
 void note_launches(int n);
+// Records the variant of the last fused FMA-kernel launch (bit flags of
+// gauss_sum_testing_last_fma_variant).
+void note_fma_variant(int flags);
 
 }  // namespace gs

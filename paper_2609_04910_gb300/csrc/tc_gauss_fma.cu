@@ -24,7 +24,13 @@
 //   * Work order: persistent CTAs over (pair of query tiles, key tile)
 //     units, contiguous runs or (keys beyond half the L2) bands of key
 //     tiles; for v^T K v with q = k (TRI) only the upper triangle of tile
-//     pairs, folded into rows of equal length.
+//     pairs, folded into rows of equal length.  A CTA's work is a sequence
+//     of segments (one pair of query tiles, consecutive key tiles).  With
+//     short segments (OVL) the control warps move on to the next segment
+//     without a CTA barrier: they reload q^ once the last two S tiles of
+//     the segment are complete and release each stage when they next load
+//     it, so the next segment's copies and MMAs run while the exponent
+//     warps finish the current one.
 //   * TMEM holds SL slots of two 128-column S buffers (one per query
 //     tile); key tile j uses slot j % SL, so the MMAs of key tile j only
 //     wait for the release of key tile j - SL.  With Dp <= 128 the query
@@ -121,6 +127,7 @@ struct FmaParams {
 
 struct __align__(8) FmaBarriers {
     uint64_t qa_ready;          // q^ available to the MMAs
+    uint64_t q_free;            // OVL: every MMA of the segment has read q^ (one arrival per control warp)
     uint64_t s_full[MAX_SL];    // slot phase: both S tiles of a key tile computed
     uint64_t s_free[MAX_SL];    // slot phase: both S tiles of a key tile in registers
     uint64_t kv_full[MAX_STAGES];
@@ -212,12 +219,13 @@ __device__ __forceinline__ void exp_warps_sync() {
 // TRI: upper-triangle order for v^T K v (q = k, C = 1, augmented
 // operands): key tiles past the pair's own two get the weight 2, applied as
 // +1 in the exponent.
-template <int C, bool AUG, bool QSM, bool TF, bool TRI, int SOFT>
+template <int C, bool AUG, bool QSM, bool TF, bool TRI, int SOFT, bool OVL>
 __global__ void __launch_bounds__(THREADS, 1)
 tc_gauss_fma_kernel(const __grid_constant__ CUtensorMap tm_q,
                     const __grid_constant__ CUtensorMap tm_k, const FmaParams p) {
     // TF (3xTF32): q^ in shared memory, norm terms from A and the records.
     static_assert(!TF || (QSM && !AUG), "3xTF32 runs with q^ in shared memory");
+    static_assert(!OVL || QSM, "overlapped segments keep q^ in shared memory");
     static_assert(SOFT == 0 || (AUG && !TRI), "FMA-pipe exponentials: augmented operands");
     constexpr int kSoftMask = soft_mask(SOFT);
     constexpr int REC_PAIR = (AUG ? 0 : 2) + 2 * C;   // floats per key pair
@@ -260,6 +268,7 @@ tc_gauss_fma_kernel(const __grid_constant__ CUtensorMap tm_q,
     // once per segment.  Each segment writes its partial sums to its slot.
     if (tid == 0) {
         mbar_init(&bars->qa_ready, QSM ? 1 : NEXP);
+        mbar_init(&bars->q_free, NCTRL_MAX);
         mbar_init(&bars->stall, 1);
         for (int k = 0; k < NCTRL_MAX; ++k) mbar_init(&bars->drain[k], 1);
         for (int sl = 0; sl < SL; ++sl) {
@@ -298,8 +307,7 @@ tc_gauss_fma_kernel(const __grid_constant__ CUtensorMap tm_q,
         int u = u_begin, run = 0, g0 = 0;   // g0: running index of the segment's first tile
         Segment sg;
         for (; next_segment<TRI>(p, u_end, u, run, sg); seg_parity ^= 1u, g0 += sg.T) {
-        // Read by every thread after a CTA barrier: uniform.
-        if (*abort_flag) break;
+        if (__any_sync(0xffffffffu, *abort_flag != 0)) break;
         const int tile_m = sg.tile_m;         // query tiles 2 tile_m, 2 tile_m + 1
         // First k^ row of this pair's problem (batch-stacked operands).
         const int kbase = (tile_m / p.pairs_per_batch) * p.npad;
@@ -318,8 +326,17 @@ tc_gauss_fma_kernel(const __grid_constant__ CUtensorMap tm_q,
             // This warp's tiles: running index g = g0 + j with g = k (mod nctrl).
             const int j_first = (k - g0 % nctrl + nctrl) % nctrl;
             const bool has_tiles = k < nctrl && j_first < T;
-            if (QSM && k == 0 && leader) {
-                // q^ of this segment; the MMAs of earlier segments are complete.
+            bool ok = true;
+            if (OVL && k == 0 && g0 > 0) {
+                // q^ of this segment overwrites that of the previous one once
+                // every MMA that read it is complete (q_free of the previous
+                // segment), while the exponent warps may still be working on
+                // that segment's last tiles.
+                ok = warp_wait(&bars->q_free, seg_parity ^ 1u, abort_flag, p.status);
+            }
+            const bool q_issued = QSM && k == 0 && ok;   // warp-uniform
+            if (q_issued && leader) {
+                // q^ of this segment.
                 tma_prefetch_desc(&tm_q);
                 mbar_arrive_expect_tx(&bars->qa_ready, p.q_bytes);
                 for (int h = 0; h < NQ; ++h)
@@ -328,7 +345,7 @@ tc_gauss_fma_kernel(const __grid_constant__ CUtensorMap tm_q,
                                     kb * p.kb_elems, (tile_m * NQ + h) * BM);
             }
             __syncwarp();
-            if (has_tiles) {
+            if (has_tiles && ok) {
                 auto load_keys = [&](int j) {
                     mbar_arrive_expect_tx(&bars->kv_full[k], p.kh_bytes + p.rec_bytes);
                     const int n0 = kbase + (kt0 + j) * BN;
@@ -339,12 +356,21 @@ tc_gauss_fma_kernel(const __grid_constant__ CUtensorMap tm_q,
                               p.rec + static_cast<int64_t>(n0 / 2) * REC_PAIR, p.rec_bytes,
                               &bars->kv_full[k]);
                 };
-                if (leader) {
+                // Parity of stage k's barriers for tile j: stage k completes once
+                // per tile g = k (mod nctrl).
+                uint32_t ph = static_cast<uint32_t>((g0 + j_first) / nctrl) & 1u;
+                // OVL: the stage's previous tile (the last one of an earlier
+                // segment) is released here rather than waited for at the end
+                // of that segment, so that the next segment's loads and MMAs
+                // overlap the exponent work on the last tiles.
+                if (OVL && g0 + j_first >= nctrl)
+                    ok = warp_wait(&bars->kv_empty[k], ph ^ 1u, abort_flag, p.status);
+                if (leader && ok) {
                     tma_prefetch_desc(&tm_k);
                     load_keys(j_first);
                 }
                 __syncwarp();
-                bool ok = warp_wait(&bars->qa_ready, seg_parity, abort_flag, p.status);
+                if (ok) ok = warp_wait(&bars->qa_ready, seg_parity, abort_flag, p.status);
                 // Test hook (status word 6 set by the host): control warp 0 of
                 // CTA 0 waits on a barrier that nothing arrives on, so its
                 // bounded wait runs out and every role takes the abort path.
@@ -359,10 +385,7 @@ tc_gauss_fma_kernel(const __grid_constant__ CUtensorMap tm_q,
                 const uint64_t qdesc0 = smem_desc_kmajor_sw128(smem_u32(q_smem));
                 const uint32_t qdesc_h = static_cast<uint32_t>((p.nkb * BM * 128) >> 4);
                 const uint32_t a0 = tmem + qa_col, a1 = a0 + (p.Dp / 2);
-                bool pending = true;          // keys of tile j requested, not yet waited for
-                // Parity of stage k's barriers for tile j: stage k completes once
-                // per tile g = k (mod nctrl).
-                uint32_t ph = static_cast<uint32_t>((g0 + j_first) / nctrl) & 1u;
+                bool pending = ok;            // keys of tile j requested, not yet waited for
                 int j = j_first;
                 for (; ok && j < T; j += nctrl, ph ^= 1u) {
                     // S slot of tile j and the parities of its barriers: s_full
@@ -406,6 +429,7 @@ tc_gauss_fma_kernel(const __grid_constant__ CUtensorMap tm_q,
                         }
                         mma_commit(&bars->s_full[sl]);
                         mma_commit(&bars->kv_empty[k]);
+                        if (OVL && j + nctrl >= T) mma_commit(&bars->q_free);
                     } else if (leader) {
                         for (int h = 0; h < NQ; ++h) {
                             for (int kk = 0; kk < ksteps; ++kk) {
@@ -421,15 +445,22 @@ tc_gauss_fma_kernel(const __grid_constant__ CUtensorMap tm_q,
                         }
                         mma_commit(&bars->s_full[sl]);
                         mma_commit(&bars->kv_empty[k]);
+                        // OVL, the warp's last tile of the segment: q_free
+                        // arrives once these MMAs, and so all of this warp's
+                        // MMAs that read the segment's q^, are complete.
+                        if (OVL && j + nctrl >= T) mma_commit(&bars->q_free);
                     }
                     __syncwarp();
                     issued = true;
                     // Stage k is free again once these MMAs and the exponent
-                    // warps are done with tile j; after the last tile this also
-                    // makes sure every arrival on the stage has landed before the
-                    // barriers are initialised for the next segment.
-                    ok = warp_wait(&bars->kv_empty[k], ph, abort_flag, p.status);
-                    if (!ok) break;
+                    // warps are done with tile j.  OVL: the release of a
+                    // segment's last tile on this stage is waited for when the
+                    // stage is next loaded (above); otherwise the segment ends
+                    // with it.
+                    if (!OVL || j + nctrl < T) {
+                        ok = warp_wait(&bars->kv_empty[k], ph, abort_flag, p.status);
+                        if (!ok) break;
+                    }
                     if (j + nctrl < T) {
                         if (leader) load_keys(j + nctrl);
                         __syncwarp();
@@ -443,16 +474,28 @@ tc_gauss_fma_kernel(const __grid_constant__ CUtensorMap tm_q,
                 // the warp reconverges after them.
                 if (pending) mbar_wait_bounded(&bars->kv_full[k], ph, nullptr, p.status);
                 __syncwarp();
+            } else if (OVL && ok) {
+                // A control warp without tiles in this segment arrives on
+                // q_free once the segment's q^ has landed: that orders the
+                // arrival after the completion of the previous q_free phase,
+                // which the q^ copy waited for.
+                ok = warp_wait(&bars->qa_ready, seg_parity, abort_flag, p.status);
+                if (leader && ok) mbar_arrive(&bars->q_free);
+                __syncwarp();
             }
-            if (QSM && k == 0) {
-                // The q^ copy of this segment must have landed before the CTA
-                // moves on (the next segment overwrites q^).
+            if (q_issued) {
+                // The q^ copy of this segment must have landed before the
+                // CTA moves on (the next segment overwrites q^; after an
+                // abort the copy may still be in flight).
                 mbar_wait_bounded(&bars->qa_ready, seg_parity, nullptr, p.status);
                 __syncwarp();
             }
-        // Segment end: every MMA, copy and TMEM read of this segment is done
-        // (control warps waited for their last stage release and copies).
-        segment_sync();
+            if (!OVL) {
+                // Segment end: every MMA, copy and TMEM read of this segment
+                // is done (control warps waited for their last stage release
+                // and copies).
+                segment_sync();
+            }
         }
         // No MMA of this warp may still run when TMEM is freed.  Without an
         // abort the last stage-release wait has already seen them complete;
@@ -472,8 +515,7 @@ tc_gauss_fma_kernel(const __grid_constant__ CUtensorMap tm_q,
         int u = u_begin, run = 0, g0 = 0;
         Segment sg;
         for (; next_segment<TRI>(p, u_end, u, run, sg); seg_parity ^= 1u, g0 += sg.T) {
-        // Read by every thread after a CTA barrier: uniform.
-        if (*abort_flag) break;
+        if (__any_sync(0xffffffffu, *abort_flag != 0)) break;
         const int tile_m = sg.tile_m;         // query tiles 2 tile_m, 2 tile_m + 1
         const int T = sg.T;
         // TRI: tiles j >= w_from of this segment lie past the pair's own two
@@ -653,6 +695,10 @@ tc_gauss_fma_kernel(const __grid_constant__ CUtensorMap tm_q,
                 else mbar_arrive_if_zero(&bars->kv_empty[s], lane);
             }
             // Fixed-order reduction of the NPART column-group partial sums.
+            // (OVL: the warps do not meet at segment ends, so the reduction
+            // area of the previous segment must have been read by every warp
+            // before it is written again.)
+            if (OVL) exp_warps_sync();
     #pragma unroll
             for (int cc = 0; cc < C; ++cc) {
                 float lo, hi;
@@ -675,8 +721,8 @@ tc_gauss_fma_kernel(const __grid_constant__ CUtensorMap tm_q,
                 }
             }
         // Segment end: every MMA, copy and TMEM read of this segment is done
-        // (control warps waited for their last stage release and copies).
-        segment_sync();
+        // (not OVL; with q^ in TMEM, before the exponent warps copy the next q^).
+        if (!OVL) segment_sync();
         }
     }
 
@@ -713,7 +759,7 @@ size_t q_bytes_for(int nkb, bool qsm) {
     return qsm ? static_cast<size_t>(NQ) * nkb * BM * 128 : 0;
 }
 
-template <int C, bool AUG, bool QSM, bool TF, bool TRI = false, int SOFT = 0>
+template <int C, bool AUG, bool QSM, bool TF, bool TRI = false, int SOFT = 0, bool OVL = false>
 cudaError_t launch_typed(const TcPlan& pl, InType t, float c, char* ws, unsigned* status,
                          cudaStream_t s, const char** why) {
     const CUtensorMapDataType hdt =
@@ -757,12 +803,12 @@ cudaError_t launch_typed(const TcPlan& pl, InType t, float c, char* ws, unsigned
     p.c = c;
     const uint32_t hb = t == InType::BF16 ? 1u : 0u;
     p.idesc = TF ? idesc_tf32(BM, BN) : idesc_f16(BM, BN, hb, hb);
-    cudaError_t e = cudaFuncSetAttribute(tc_gauss_fma_kernel<C, AUG, QSM, TF, TRI, SOFT>,
+    cudaError_t e = cudaFuncSetAttribute(tc_gauss_fma_kernel<C, AUG, QSM, TF, TRI, SOFT, OVL>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          static_cast<int>(pl.smem_bytes));
     if (e != cudaSuccess) return e;
     dim3 grid(static_cast<unsigned>(pl.grid));
-    launch_kernel(tc_gauss_fma_kernel<C, AUG, QSM, TF, TRI, SOFT>, grid, THREADS, pl.smem_bytes, s, tm_q, tm_k, p);
+    launch_kernel(tc_gauss_fma_kernel<C, AUG, QSM, TF, TRI, SOFT, OVL>, grid, THREADS, pl.smem_bytes, s, tm_q, tm_k, p);
     note_launches(1);
     return cudaGetLastError();
 }
@@ -782,6 +828,8 @@ cudaError_t launch_c(const TcPlan& pl, InType t, float c, char* ws, unsigned* st
             }
         }
     }
+    if (pl.aug && kAugQsm && pl.overlap)
+        return launch_typed<C, true, true, false, false, 0, true>(pl, t, c, ws, status, s, why);
     if (pl.aug) return launch_typed<C, true, kAugQsm, false>(pl, t, c, ws, status, s, why);
     return launch_typed<C, false, false, false>(pl, t, c, ws, status, s, why);
 }
@@ -818,6 +866,9 @@ bool plan_fma_kernel(int Dp, int C, bool aug, bool tf, int* nq, int* stages, siz
 
 cudaError_t launch_tc_fma(const TcPlan& p, InType t, float c, char* ws, unsigned* status,
                           cudaStream_t s, const char** why) {
+    const bool qsm = p.tf || (p.aug && kAugQsm);
+    note_fma_variant((p.aug && kAugQsm && p.overlap && !p.tri && p.exp2_fma == 0 ? 1 : 0) |
+                     (p.band_len > 0 ? 2 : 0) | (qsm ? 0 : 4));
     switch (p.Cv) {
         case 1: return launch_c<1>(p, t, c, ws, status, s, why);
         case 2: return launch_c<2>(p, t, c, ws, status, s, why);

@@ -7,8 +7,9 @@ Switches (plan_tensor / plan_simt): augmented operands of the FMA kernel
 (Dp_aug + Cp <= 128); 128- versus 64-key tiles (Cp <= 128); early S
 release (four or more stages) versus one MMA warp; gradient channels in one
 launch (D + 1 <= 256) versus two; fp32 register tiles of 16 / 32 / 64 / 128
-coordinates; 3xTF32 tensor-core variant (D <= 32, C <= 4).  Key counts
-straddle one key tile (127, 128, 129).
+coordinates; 3xTF32 tensor-core variant (D <= 32, C <= 4); overlapped
+segment transitions of the FMA kernel (runs of at most 64 key tiles).  Key
+counts straddle one key tile (127, 128, 129).
 """
 import pytest
 
@@ -91,3 +92,23 @@ def test_ex2_rate_probes():
     mix = gs.gauss_sum_probe_ex2_mix_rate()
     assert 0 < plain <= 32 * sms * 2.2e9
     assert 0 < mix <= 1.05 * plain
+
+
+@pytest.mark.parametrize("M,N,overlap,banded", [
+    (65536, 8192, True, False),      # 64 key tiles per pair of query tiles: overlapped
+    (65536, 8320, False, False),     # 65 key tiles, 110 units per CTA: segment barrier
+    (2048, 8320, True, False),       # 65 key tiles but 4 units per CTA: overlapped
+    (1024, 524288, True, True),      # keys beyond half the L2: bands of 64 key tiles
+])
+def test_fma_segment_overlap_switch(M, N, overlap, banded):
+    """The FMA kernel overlaps segment transitions when a CTA's runs of key
+    tiles for one pair of query tiles are at most 64 tiles long (the
+    smaller of the key tiles per pair and the units per CTA, or the band
+    length); each side against the oracle on sampled rows."""
+    from paper_2609_04910_gb300._binding import testing_last_fma_variant
+    from paper_2609_04910_gb300.workloads import sample_rows
+    w = case(M, N, 64, 1, "fp16")
+    forward_check(w, rows=sample_rows(M, 256))
+    flags = testing_last_fma_variant()
+    assert bool(flags & 1) == overlap, flags
+    assert bool(flags & 2) == banded, flags
