@@ -12,7 +12,7 @@
 //
 //   MMA1  S   = q^ k^T          tcgen05.mma kind::f16, A,B from shared memory,
 //                               fp32 accumulator in TMEM (128 x BN)
-//   exp   P   = fp16(2^(c S + A_m + B_n + 15))   TMEM -> registers -> TMEM
+//   exp   P   = fp16(2^(c S + A_m + B_n + 16))   TMEM -> registers -> TMEM
 //   MMA2  O  += P v~            tcgen05.mma kind::f16, A = P from TMEM,
 //                               B = value tile from shared memory, fp32 TMEM
 //
@@ -55,25 +55,16 @@ namespace {
 constexpr int BM = 128;           // query rows per CTA (MMA M)
 constexpr int KB = 64;            // 16-bit elements per 128-byte swizzled row
 constexpr uint32_t TMEM_COLS = 512;
-// P is stored as fp16(2^(x + P_SHIFT)): since x <= 0 the stored value is at
-// most 2^15 < 65504, and kernel values down to 2^-29 stay normal fp16
-// numbers (instead of 2^-14).  The epilogue multiplies O by 2^-P_SHIFT.
-// The exponent is <= 0 in exact arithmetic; a rounding-positive x is
-// clamped to 0 on the packed fp16 pair (P <= 2^15, i.e. Phi <= 1): one
-// min.f16x2 per pair (the shifted exponent x + 15 leaves no room for the
-// sign-free 2^-|x| form of ex2_nonpos).
-constexpr float P_SHIFT = 15.f;
-constexpr float P_UNSHIFT = 1.f / 32768.f;
-constexpr uint32_t kP2Max = 0x78007800u;   // fp16 pair (2^15, 2^15)
-
-// Element-wise minimum of two packed fp16 pairs.
-__device__ __forceinline__ uint32_t hmin2(uint32_t a, uint32_t b) {
-    uint32_t d;
-    asm("min.f16x2 %0, %1, %2;" : "=r"(d) : "r"(a), "r"(b));
-    return d;
-}
-
-__device__ __forceinline__ uint32_t bound_p2(uint32_t p2) { return hmin2(p2, kP2Max); }
+// P is stored as fp16(2^(x + P_SHIFT)) with P_SHIFT = 16, and kernel
+// values down to 2^-30 stay normal fp16 numbers (instead of 2^-14).  The
+// epilogue multiplies O by 2^-P_SHIFT.  The exponent is <= 0 in exact
+// arithmetic; the conversion saturates at the largest finite fp16 value,
+// 65504 = 2^16 (1 - 2^-11), so a rounding-positive x gives P = 65504, i.e.
+// Phi <= 1 without a separate clamp.  The price: kernel values in
+// (1 - 2^-11, 1] are stored as 1 - 2^-11, an error of at most 2^-11
+// relative, the unit roundoff of the fp16 P itself.
+constexpr float P_SHIFT = 16.f;
+constexpr float P_UNSHIFT = 1.f / 65536.f;
 
 struct TcParams {
     const float* A;      // Mpad: -(c/2)||q^_m||^2
@@ -438,7 +429,8 @@ tc_gauss_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant_
         // epilogue's inverse scale.  With Wb = sum_c max|r_c| max|k_c| >=
         // |w_mn| and sw = 15 - ceil(log2 Wb), |2^sw w_mn| <= 2^15, so the
         // products 2^x 2^sw w_mn (x <= 0) fit fp16 like the unweighted
-        // P = 2^(x + 15), and small weights keep their precision.
+        // P = 2^(x + 16) (largest 65504), and small weights keep their
+        // precision.
         float unshift = P_UNSHIFT;
         uint64_t rw2[WT > 0 ? WT : 1];
         if (WT > 0) {
@@ -512,9 +504,9 @@ tc_gauss_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant_
             uint32_t pk[32];
 #pragma unroll
             for (int i = 0; i < 16; ++i) {
-                // x = c S + (A_m + 15) + B_n for four keys, two per f32x2 op
+                // x = c S + (A_m + 16) + B_n for four keys, two per f32x2 op
                 // (with augmented operands S already holds the norm terms:
-                // x = c S + 15).
+                // x = c S + 16).
                 uint64_t t01 = a2, t23 = a2;
                 if (!AUG) {
                     const float4 bb = *reinterpret_cast<const float4*>(Bs + 4 * i);
@@ -545,8 +537,8 @@ tc_gauss_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant_
                     pk[2 * i + 0] = pack_half2_satfinite(p0, p1);
                     pk[2 * i + 1] = pack_half2_satfinite(p2, p3);
                 } else {
-                    pk[2 * i + 0] = bound_p2(pack_half2_satfinite(ex2_approx(x0), ex2_approx(x1)));
-                    pk[2 * i + 1] = bound_p2(pack_half2_satfinite(ex2_approx(x2), ex2_approx(x3)));
+                    pk[2 * i + 0] = pack_half2_satfinite(ex2_approx(x0), ex2_approx(x1));
+                    pk[2 * i + 1] = pack_half2_satfinite(ex2_approx(x2), ex2_approx(x3));
                 }
             }
             if (EARLY && j >= 2) {
