@@ -349,6 +349,17 @@ def roofline_of(w, main_ms, peaks, peak_src, sms, r_x, traffic=None, traffic_src
         "sfu": {"achieved": exps / t_main / 1e12, "peak": r_x_nominal / 1e12,
                 "unit": "Texp/s", "frac": t_sfu / t_main, "probe_ex2_per_s": r_x},
     })
+    r_ts = peaks.get("bf16_tflops_sustained")
+    if r_ts:
+        # A tensor-bound kernel that runs for a whole timed loop meets the
+        # power cap like the sustained cuBLAS loop that measured this peak;
+        # its fraction of that peak is reported beside the burst fraction.
+        r_ts = float(r_ts) * 1e12
+        roof["tensor"]["peak_sustained"] = r_ts / 1e12
+        roof["tensor"]["frac_of_sustained"] = flops / r_ts / t_main
+        if roof["bound"] == "tensor":
+            roof["peak_sustained"] = r_ts / 1e12
+            roof["frac_of_sustained"] = flops / r_ts / t_main
     if r_mix and main_kernel_name(w) == "tc_gauss_fma_kernel" and roof["bound"] == "alu":
         # The exp2 rate that the FMA kernel's own exponent-loop instruction
         # mix reaches without tiles, barriers or tensor-memory traffic

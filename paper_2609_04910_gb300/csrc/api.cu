@@ -327,10 +327,15 @@ gs_status run(Call c) {
     if (tensor) {
         const gs::InType t = in_type(c.dtype);
         float* mu = (tp.center && c.D > 0) ? reinterpret_cast<float*>(ws + tp.off_mu) : nullptr;
+        // Key records of the FMA kernel with augmented operands depend on the
+        // values only: the mean launch writes them where it can.
+        bool records_done = false;
         if (mu) {
+            const gs::RecordArgs rec = {c.v, c.w_f32, c.N, tp.Npad, static_cast<int>(tp.Cv),
+                                        reinterpret_cast<float*>(ws + tp.off_rec)};
             e = gs::launch_mean(t, c.q, c.k, c.M, c.N, static_cast<int>(c.D), tp.mean_blocks,
                                 reinterpret_cast<float*>(ws + tp.off_mean_part), mu, c.stream,
-                                batch);
+                                batch, (tp.fma && tp.aug) ? &rec : nullptr, &records_done);
             where = "mean kernel";
         }
         const float ninf = -INFINITY;
@@ -366,12 +371,14 @@ gs_status run(Call c) {
             where = tp.aug ? "augmented-operand kernel" : "centre/cast kernel";
         }
         if (e == cudaSuccess && tp.fma) {
-            e = gs::launch_key_records(
-                c.w_f32 ? gs::InType::F32 : t, c.v,
-                tp.aug ? nullptr : reinterpret_cast<const float*>(ws + tp.off_B), c.N,
-                tp.Npad, static_cast<int>(tp.Cv), reinterpret_cast<float*>(ws + tp.off_rec),
-                c.stream, batch);
-            where = "key-record kernel";
+            if (!records_done) {
+                e = gs::launch_key_records(
+                    c.w_f32 ? gs::InType::F32 : t, c.v,
+                    tp.aug ? nullptr : reinterpret_cast<const float*>(ws + tp.off_B), c.N,
+                    tp.Npad, static_cast<int>(tp.Cv), reinterpret_cast<float*>(ws + tp.off_rec),
+                    c.stream, batch);
+                where = "key-record kernel";
+            }
             if (e == cudaSuccess) e = record_event(c.opt.main_events[0], c.stream);
             if (e == cudaSuccess) {
                 e = gs::launch_tc_fma(tp, t, cexp, ws, status, c.stream, &why);

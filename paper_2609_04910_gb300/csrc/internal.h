@@ -133,8 +133,21 @@ bool plan_simt(int64_t M, int64_t N, int64_t D, int64_t C, bool grad, int split_
                int sms, SimtPlan* p, const char** why);
 
 // prep.cu --------------------------------------------------------------
+// Key records of the FMA kernel that the mean launch may write alongside
+// (values only: augmented operands, no norm terms in the records).
+struct RecordArgs {
+    const void* v;       // N x C values per problem, 16-bit like q, or fp32 (v_f32)
+    bool v_f32;
+    int64_t N, Npad;
+    int C;
+    float* out;          // Npad / 2 pairs x 2C floats per problem
+};
+// Common mean of q and k per problem.  With `rec`, the launch also writes
+// those key records where it can (the vectorised path); *rec_done says
+// whether it did.
 cudaError_t launch_mean(InType t, const void* q, const void* k, int64_t M, int64_t N, int D,
-                        int blocks, float* partial, float* mu, cudaStream_t s, int batch = 1);
+                        int blocks, float* partial, float* mu, cudaStream_t s, int batch = 1,
+                        const RecordArgs* rec = nullptr, bool* rec_done = nullptr);
 // Centred, rounded MMA operands of q (M rows, padded to Mpad) and, with
 // with_k, of k (N rows, padded to Npad), in one launch where the vector
 // path applies (16-bit inputs, D a multiple of 8).  aug: the augmented

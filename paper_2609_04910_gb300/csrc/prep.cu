@@ -99,21 +99,50 @@ __global__ void mean_partial_kernel(const T* __restrict__ q, const T* __restrict
 // always sees the same 8 coordinates and keeps their sums and maxima in
 // registers.  Blocks [0, Gq) cover rows of q, blocks [Gq, G) rows of k
 // (none when q and k are the same points).  Same partial layout as above.
+// Blocks from G on, when given a record job, write the FMA kernel's key
+// records instead (see key_record_kernel): they depend on the values only,
+// so they ride along in this first launch of the call rather than taking
+// a launch of their own later in the chain.
 constexpr int kMeanVecThreads = 256;
 
-template <typename T>
+template <typename TV>
+struct RecordJob {
+    const TV* v;         // N x C values per problem (batch-stacked)
+    int64_t N, pairs;    // keys and key pairs (Npad / 2) per problem
+    int C;
+    float* rec;          // pairs x 2C floats per problem
+};
+
+template <typename TV>
+__device__ __forceinline__ void write_key_record(const RecordJob<TV>& j, int64_t t, int problem) {
+    const int64_t n0 = 2 * t, n1 = 2 * t + 1;
+    const TV* v = j.v + static_cast<int64_t>(problem) * j.N * j.C;
+    float* out = j.rec + (static_cast<int64_t>(problem) * j.pairs + t) * (2 * j.C);
+    for (int c = 0; c < j.C; ++c) {
+        out[2 * c] = n0 < j.N ? to_f(v[n0 * j.C + c]) : 0.f;
+        out[2 * c + 1] = n1 < j.N ? to_f(v[n1 * j.C + c]) : 0.f;
+    }
+}
+
+template <typename T, typename TV>
 __global__ void __launch_bounds__(kMeanVecThreads)
 mean_partial_vec_kernel(const T* __restrict__ q, const T* __restrict__ k, int64_t M, int64_t N,
-                        int D, int64_t rows_per_block, int Gq, float* __restrict__ partial) {
+                        int D, int64_t rows_per_block, int Gq, int G, float* __restrict__ partial,
+                        const RecordJob<TV> rj) {
     pdl_trigger();
     pdl_wait();
+    if (static_cast<int>(blockIdx.x) >= G) {
+        const int64_t t = static_cast<int64_t>(blockIdx.x - G) * kMeanVecThreads + threadIdx.x;
+        if (t < rj.pairs) write_key_record(rj, t, blockIdx.y);
+        return;
+    }
     __shared__ float s_sum[kMeanVecThreads][9];
     __shared__ float s_max[kMeanVecThreads][9];
     const int t = threadIdx.x;
     // Problem blockIdx.y of a batch: its own points and partial rows.
     q += static_cast<int64_t>(blockIdx.y) * M * D;
     k += static_cast<int64_t>(blockIdx.y) * N * D;
-    partial += static_cast<int64_t>(blockIdx.y) * 2 * gridDim.x * D;
+    partial += static_cast<int64_t>(blockIdx.y) * 2 * G * D;
     const bool on_q = static_cast<int>(blockIdx.x) < Gq;
     const int64_t b = on_q ? blockIdx.x : blockIdx.x - Gq;
     const int64_t rows = on_q ? M : N;
@@ -161,7 +190,7 @@ mean_partial_vec_kernel(const T* __restrict__ q, const T* __restrict__ k, int64_
             m = fmaxf(m, s_max[u][e]);
         }
         partial[static_cast<int64_t>(blockIdx.x) * D + d] = a;
-        partial[static_cast<int64_t>(gridDim.x + blockIdx.x) * D + d] = m;
+        partial[static_cast<int64_t>(G + blockIdx.x) * D + d] = m;
     }
 }
 
@@ -1043,7 +1072,9 @@ cudaError_t finalize_points_typed(const float* part, int splits, int64_t stride_
 }  // namespace
 
 cudaError_t launch_mean(InType t, const void* q, const void* k, int64_t M, int64_t N, int D,
-                        int blocks, float* partial, float* mu, cudaStream_t s, int batch) {
+                        int blocks, float* partial, float* mu, cudaStream_t s, int batch,
+                        const RecordArgs* rec, bool* rec_done) {
+    if (rec_done) *rec_done = false;
     // q and k the same points: the mean of [q; q] is the mean of q.
     if (q == k && M == N) N = 0;
     const int64_t total = M + N;
@@ -1057,14 +1088,25 @@ cudaError_t launch_mean(InType t, const void* q, const void* k, int64_t M, int64
         const int Gq = static_cast<int>((M + rpb - 1) / rpb);
         const int Gk = static_cast<int>((N + rpb - 1) / rpb);
         G = Gq + Gk;
-        if (t == InType::F16)
-            launch_kernel(mean_partial_vec_kernel<__half>, dim3(G, batch), kMeanVecThreads, 0, s, 
-                static_cast<const __half*>(q), static_cast<const __half*>(k), M, N, D, rpb, Gq,
-                partial);
-        else
-            launch_kernel(mean_partial_vec_kernel<__nv_bfloat16>, dim3(G, batch), kMeanVecThreads, 0, s, 
-                static_cast<const __nv_bfloat16*>(q), static_cast<const __nv_bfloat16*>(k), M, N, D,
-                rpb, Gq, partial);
+        // Key records (see RecordJob) in blocks G .. G + rblocks - 1.
+        const int64_t pairs = rec ? rec->Npad / 2 : 0;
+        const int rblocks = static_cast<int>((pairs + kMeanVecThreads - 1) / kMeanVecThreads);
+        auto go = [&](auto tag, auto vtag) {
+            using T = decltype(tag);
+            using TV = decltype(vtag);
+            const RecordJob<TV> rj = {rec ? static_cast<const TV*>(rec->v) : nullptr, rec ? rec->N : 0,
+                                      pairs, rec ? rec->C : 0, rec ? rec->out : nullptr};
+            launch_kernel(mean_partial_vec_kernel<T, TV>, dim3(G + rblocks, batch), kMeanVecThreads, 0,
+                          s, static_cast<const T*>(q), static_cast<const T*>(k), M, N, D, rpb, Gq, G,
+                          partial, rj);
+        };
+        const bool vf = rec && rec->v_f32;
+        if (t == InType::F16) {
+            if (vf) go(__half(), float()); else go(__half(), __half());
+        } else {
+            if (vf) go(__nv_bfloat16(), float()); else go(__nv_bfloat16(), __nv_bfloat16());
+        }
+        if (rec_done) *rec_done = rec != nullptr;
         note_launches(1);
     } else {
         const int64_t rpb = (total + blocks - 1) / blocks;
