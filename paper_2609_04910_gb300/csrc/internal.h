@@ -59,6 +59,10 @@ struct TcPlan {
     // run with `splits` key splits in a second launch, so that the last
     // wave is not left part-empty.
     int64_t main_tiles;
+    // Row tiles per wave of the main launch (the SM count): waves of odd
+    // index walk the keys in reverse order, so that the keys the previous
+    // wave read last are still in L2 when this wave starts.
+    int wave_tiles;
     int stages;              // shared-memory pipeline depth
     size_t smem_bytes;       // dynamic shared memory of the fused kernel
     int mean_blocks;

@@ -12,7 +12,7 @@
 //
 //   MMA1  S   = q^ k^T          tcgen05.mma kind::f16, A,B from shared memory,
 //                               fp32 accumulator in TMEM (128 x BN)
-//   exp   P   = fp16(2^(c S + A_m + B_n + 16))   TMEM -> registers -> TMEM
+//   exp   P   = fp16(2^(c S + A_m + B_n + 15))   TMEM -> registers -> TMEM
 //   MMA2  O  += P v~            tcgen05.mma kind::f16, A = P from TMEM,
 //                               B = value tile from shared memory, fp32 TMEM
 //
@@ -55,16 +55,16 @@ namespace {
 constexpr int BM = 128;           // query rows per CTA (MMA M)
 constexpr int KB = 64;            // 16-bit elements per 128-byte swizzled row
 constexpr uint32_t TMEM_COLS = 512;
-// P is stored as fp16(2^(x + P_SHIFT)) with P_SHIFT = 16, and kernel
-// values down to 2^-30 stay normal fp16 numbers (instead of 2^-14).  The
-// epilogue multiplies O by 2^-P_SHIFT.  The exponent is <= 0 in exact
-// arithmetic; the conversion saturates at the largest finite fp16 value,
-// 65504 = 2^16 (1 - 2^-11), so a rounding-positive x gives P = 65504, i.e.
-// Phi <= 1 without a separate clamp.  The price: kernel values in
-// (1 - 2^-11, 1] are stored as 1 - 2^-11, an error of at most 2^-11
-// relative, the unit roundoff of the fp16 P itself.
-constexpr float P_SHIFT = 16.f;
-constexpr float P_UNSHIFT = 1.f / 65536.f;
+// P is stored as fp16(2^(x + P_SHIFT)) with P_SHIFT = 15: kernel values
+// down to 2^-29 stay normal fp16 numbers (instead of 2^-14), a kernel value
+// of 1 is stored exactly (2^15), and the epilogue multiplies O by
+// 2^-P_SHIFT.  The exponent is <= 0 in exact arithmetic.  A rounding-
+// positive x is not clamped: 2^(15 + x) differs from the clamped 2^15 by
+// less than x ln 2 relative, no more than the rounding error of x itself
+// (and below 2^-12, half an fp16 ulp at 2^15, it rounds to 2^15 anyway);
+// the saturating conversion keeps P finite for any x.
+constexpr float P_SHIFT = 15.f;
+constexpr float P_UNSHIFT = 1.f / 32768.f;
 
 struct TcParams {
     const float* A;      // Mpad: -(c/2)||q^_m||^2
@@ -73,6 +73,8 @@ struct TcParams {
     unsigned* status;    // device status word
     int64_t Mpad;
     int tile_off;        // row tile of blockIdx.x = 0 (main launch 0, tail launch main_tiles)
+    int wave_tiles;      // > 0: blocks of odd waves (blockIdx.x / wave_tiles) take their key
+                         // tiles in reverse order
     int key_tiles;
     int tiles_per_split;
     int nkb;             // 64-element K blocks of q^/k^
@@ -232,13 +234,20 @@ tc_gauss_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant_
             }
             __syncwarp();
             int issued = 0;
+            // Waves of one block per SM stream the same keys at about the
+            // same time; every other wave streams them backwards, starting
+            // with the keys the previous wave read last (still in L2)
+            // instead of those it read first (evicted by then).  The sum of
+            // a row is then taken in the reverse key order, a fixed order
+            // all the same.
+            const bool reverse = p.wave_tiles > 0 && ((blockIdx.x / p.wave_tiles) & 1u);
             RingPos st;
             for (int j = 0; j < T; ++j, st.advance(p.stages)) {
                 const int s = st.idx;
                 if (!warp_wait(&bars->kv_empty[s], st.phase ^ 1u, abort_flag, p.status)) break;
                 if (leader) {
                     mbar_arrive_expect_tx(&bars->kv_full[s], p.tx_bytes);
-                    const int n0 = (kt0 + j) * BN;
+                    const int n0 = (reverse ? kt1 - 1 - j : kt0 + j) * BN;
                     for (int kb = 0; kb < p.nkb; ++kb)
                         tma_load_2d(kh_smem(s) + kb * (BN * 128), &tm_k, &bars->kv_full[s], kb * KB, n0);
                     for (int h = 0; h < BN / KB; ++h)
@@ -429,8 +438,7 @@ tc_gauss_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant_
         // epilogue's inverse scale.  With Wb = sum_c max|r_c| max|k_c| >=
         // |w_mn| and sw = 15 - ceil(log2 Wb), |2^sw w_mn| <= 2^15, so the
         // products 2^x 2^sw w_mn (x <= 0) fit fp16 like the unweighted
-        // P = 2^(x + 16) (largest 65504), and small weights keep their
-        // precision.
+        // P = 2^(x + 15), and small weights keep their precision.
         float unshift = P_UNSHIFT;
         uint64_t rw2[WT > 0 ? WT : 1];
         if (WT > 0) {
@@ -504,9 +512,9 @@ tc_gauss_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant_
             uint32_t pk[32];
 #pragma unroll
             for (int i = 0; i < 16; ++i) {
-                // x = c S + (A_m + 16) + B_n for four keys, two per f32x2 op
+                // x = c S + (A_m + 15) + B_n for four keys, two per f32x2 op
                 // (with augmented operands S already holds the norm terms:
-                // x = c S + 16).
+                // x = c S + 15).
                 uint64_t t01 = a2, t23 = a2;
                 if (!AUG) {
                     const float4 bb = *reinterpret_cast<const float4*>(Bs + 4 * i);
@@ -606,6 +614,7 @@ cudaError_t launch_bn(const TcPlan& pl, InType t, float c, char* ws, unsigned* s
     p.status = status;
     p.Mpad = pl.Mpad;
     p.tile_off = tile_off;
+    p.wave_tiles = splits == 1 ? pl.wave_tiles : 0;
     p.key_tiles = static_cast<int>(pl.Npad / BN);
     p.tiles_per_split = (p.key_tiles + splits - 1) / splits;
     p.nkb = (pl.Dp + KB - 1) / KB;
@@ -803,7 +812,9 @@ bool plan_tensor(InType t, int64_t M, int64_t N, int64_t D, int64_t C, bool grad
         }
         p->main_tiles = main;
         p->splits = ts;
+        p->wave_tiles = sms;
     }
+    if (p->fma || split_override != 0 || tiles < sms) p->wave_tiles = 0;
     p->units = p->unit_len = 0;
     p->grid = 0;
     p->band_len = 0;

@@ -204,7 +204,7 @@ def test_far_points_underflow_to_zero():
 
 
 def test_fp16_kernel_value_floor():
-    """Kernel values below 2^-30 may be flushed (fp16 P stored with a +16
+    """Kernel values below 2^-29 may be flushed (fp16 P stored with a +15
     exponent shift); the error stays below tol * den + sum of flushed terms."""
     from oracle import oracle_sum
     rng = np.random.default_rng(5)

@@ -45,14 +45,14 @@ def test_sample_rows():
 
 
 def test_fp16_kernel_value_floor_never_binds_on_the_two_mma_workloads():
-    """The two-MMA kernel stores each kernel value as fp16(2^(x + 16)), so
-    values below 2^-30 lose precision (2^-40 and below flush to zero).  A row
+    """The two-MMA kernel stores each kernel value as fp16(2^(x + 15)), so
+    values below 2^-29 lose precision (2^-39 and below flush to zero).  A row
     whose largest kernel value fell below that floor would have all of its
     terms there; on the two workloads that take this kernel (multi_c64,
     svgd_d32) the largest kernel value of every sampled row is far above it,
     so a per-row exponent offset (a row maximum before the exponentials)
     would change nothing there."""
-    floor = 2.0 ** -30
+    floor = 2.0 ** -29
     for name in ("multi_c64", "svgd_d32"):
         w = WORKLOADS[name]
         g = generate(w, seed=0)
