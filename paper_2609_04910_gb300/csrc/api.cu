@@ -227,6 +227,13 @@ gs_status plan(const Call& c, int sms, bool* tensor, gs::TcPlan* tp, gs::SimtPla
         if (tp->exp2_fma > 0 && !(tp->fma && tp->aug && !tp->tri && tp->Cv == 1))
             return fail(GS_ERR_UNSUPPORTED,
                         "exp2_fma needs a forward fp16/bf16 sum with C = 1 on augmented operands");
+        // One fp16 value channel on augmented operands: the value magnitudes
+        // go into the key operands and the key records keep the signs.  Not
+        // for short segments (small problems), where the flag kernel and the
+        // second pass of the fused kernel cost more than they save (B = 256
+        // problems of 1024 points: 0.135 -> 0.144 ms per call).
+        tp->vfold = tp->fma && tp->aug && !tp->tf && tp->Cv == 1 && c.dtype == GS_FP16 &&
+                    !c.w_f32 && tp->exp2_fma == 0 && c.C == 1 && !tp->overlap;
         *bytes = tp->total;
     } else {
         if (c.opt.exp2_fma > 0)
@@ -332,7 +339,7 @@ gs_status run(Call c) {
         bool records_done = false;
         if (mu) {
             const gs::RecordArgs rec = {c.v, c.w_f32, c.N, tp.Npad, static_cast<int>(tp.Cv),
-                                        reinterpret_cast<float*>(ws + tp.off_rec)};
+                                        reinterpret_cast<float*>(ws + tp.off_rec), tp.vfold};
             e = gs::launch_mean(t, c.q, c.k, c.M, c.N, static_cast<int>(c.D), tp.mean_blocks,
                                 reinterpret_cast<float*>(ws + tp.off_mean_part), mu, c.stream,
                                 batch, (tp.fma && tp.aug) ? &rec : nullptr, &records_done);
@@ -367,7 +374,7 @@ gs_status run(Call c) {
                 tp.aug ? nullptr : reinterpret_cast<float*>(ws + tp.off_A),
                 !tp.alias, c.k, c.N, tp.Npad, ws + tp.off_kh,
                 tp.aug ? nullptr : reinterpret_cast<float*>(ws + tp.off_B), static_cast<int>(c.D),
-                tp.Dp, mu, half_c, ninf, c.stream, batch);
+                tp.Dp, mu, half_c, ninf, c.stream, batch, tp.vfold ? c.v : nullptr);
             where = tp.aug ? "augmented-operand kernel" : "centre/cast kernel";
         }
         if (e == cudaSuccess && tp.fma) {
@@ -376,12 +383,23 @@ gs_status run(Call c) {
                     c.w_f32 ? gs::InType::F32 : t, c.v,
                     tp.aug ? nullptr : reinterpret_cast<const float*>(ws + tp.off_B), c.N,
                     tp.Npad, static_cast<int>(tp.Cv), reinterpret_cast<float*>(ws + tp.off_rec),
-                    c.stream, batch);
+                    c.stream, batch, tp.vfold);
                 where = "key-record kernel";
+            }
+            if (e == cudaSuccess && tp.vfold) {
+                e = gs::launch_vf_flags(reinterpret_cast<float*>(ws + tp.off_rec), tp.Npad, batch,
+                                        c.stream);
+                where = "folded-value flag kernel";
             }
             if (e == cudaSuccess) e = record_event(c.opt.main_events[0], c.stream);
             if (e == cudaSuccess) {
-                e = gs::launch_tc_fma(tp, t, cexp, ws, status, c.stream, &why);
+                // Folded values: two passes of the fused kernel, for the
+                // problems whose 32-key groups all have values of one sign
+                // (no record loads) and for the others; each pass skips the
+                // other's problems.
+                e = gs::launch_tc_fma(tp, t, cexp, ws, status, c.stream, &why, tp.vfold ? 1 : 0);
+                if (e == cudaSuccess && tp.vfold)
+                    e = gs::launch_tc_fma(tp, t, cexp, ws, status, c.stream, &why, 2);
                 where = "fused tensor-core kernel";
             }
             if (e == cudaSuccess) e = record_event(c.opt.main_events[1], c.stream);

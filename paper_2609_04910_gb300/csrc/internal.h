@@ -103,6 +103,10 @@ struct TcPlan {
     // segment's copies and MMAs while the exponent warps finish the current
     // one, instead of meeting them at a CTA barrier at every segment end.
     bool overlap;
+    // FMA kernel, C = 1 with fp16 values on augmented operands: the value
+    // magnitudes are folded into the key operands' norm terms
+    // (log2(|v| 2^-16) / c) and the key records hold only signs (VF).
+    bool vfold;
     // Problems of a batch handled by one launch (the FMA kernel stacks them:
     // q^ batch x Mpad rows, k^ batch x Npad rows); 1 for the other paths.
     int64_t batch;
@@ -145,6 +149,8 @@ struct RecordArgs {
     int64_t N, Npad;
     int C;
     float* out;          // Npad / 2 pairs x 2C floats per problem
+    bool signs;          // sign records of folded value magnitudes (fp16 values, C = 1;
+                         // per key tile of 128 keys: 128 signed 2^16 and 4 group words)
 };
 // Common mean of q and k per problem.  With `rec`, the launch also writes
 // those key records where it can (the vectorised path); *rec_done says
@@ -163,7 +169,7 @@ cudaError_t launch_operands(InType t, bool aug, const void* q, int64_t M, int64_
                             void* qh, void* qh_as_key, float* nrm_q, bool with_k, const void* k,
                             int64_t N, int64_t Npad, void* kh, float* nrm_k, int D, int Dp,
                             const float* mu, float half_c, float pad_value, cudaStream_t s,
-                            int batch = 1);
+                            int batch = 1, const void* vw = nullptr);
 // Transposed fp16 value operand of the two-MMA kernel for the channels
 // ch0 .. ch0 + Cc - 1 (Cp >= Cc rows of Npad keys), with per-channel
 // power-of-two scales.  Forward: channel ch of key n is w[n, ch] (w has the
@@ -227,7 +233,7 @@ cudaError_t launch_simt(const SimtPlan& p, bool grad, const float* q, const floa
 // B_2t, B_2t+1 (omitted when B is null), v_2t[0], v_2t+1[0], ...,
 // v_2t[C-1], v_2t+1[C-1].
 cudaError_t launch_key_records(InType t, const void* v, const float* B, int64_t N, int64_t Npad,
-                               int C, float* rec, cudaStream_t s, int batch = 1);
+                               int C, float* rec, cudaStream_t s, int batch = 1, bool signs = false);
 // 3xTF32 operands of fp32 inputs (see prep.cu): rows of 2 Dp floats
 // [hi | lo] into out, nrm = -(c/2)||x - mu||^2 (pad_value for padded rows).
 cudaError_t launch_tf32_split(const float* x, int64_t rows, int64_t rows_pad, int D, int Dp,
@@ -247,8 +253,14 @@ constexpr int kAugMaxDp = 128;
 // tiles stay in shared memory next to the key stages.
 constexpr int kTf32MaxDp = 32;
 bool plan_fma_kernel(int Dp, int C, bool aug, bool tf, int* nq, int* stages, size_t* smem);
+// vf_pass (plans with vfold): 1 = the problems whose 32-key groups all have
+// values of one sign, 2 = the others (launched after pass 1); 0 otherwise.
 cudaError_t launch_tc_fma(const TcPlan& p, InType t, float c, char* ws, unsigned* status,
-                          cudaStream_t s, const char** why);
+                          cudaStream_t s, const char** why, int vf_pass = 0);
+// Per-problem words after the sign records (rec: batch x (Npad / 128) tiles
+// of 132 floats): 1 where every 32-key group of the problem has values of
+// one sign, else 0.
+cudaError_t launch_vf_flags(float* rec, int64_t Npad, int batch, cudaStream_t s);
 
 // probe
 // Best of three timed runs of the ex2 probe kernel: independent ex2 chains

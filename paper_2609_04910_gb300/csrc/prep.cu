@@ -15,6 +15,7 @@
 //  * the fixed-order sum of key-split partials and the final scaling, or
 //    the gradient tau (S[:D] - q_m S[D]) of Sec. 3.
 #include <algorithm>
+#include <type_traits>
 
 #include <cuda_bf16.h>
 #include <cuda_fp16.h>
@@ -111,7 +112,57 @@ struct RecordJob {
     int64_t N, pairs;    // keys and key pairs (Npad / 2) per problem
     int C;
     float* rec;          // pairs x 2C floats per problem
+    bool signs;          // sign records (see sign_record) instead of values
 };
+
+// Sign records of the FMA kernel with folded value magnitudes (C = 1, the
+// magnitudes sit in the key operands): per key tile of kRecTile keys, the
+// floats s_n = sign(v_n) 2^16 in key order (0 for v_n = 0 and for padded
+// keys), then one word per group of 32 keys: -2^16 if the group's nonzero
+// values are all negative, 0 if it has values of both signs, else 2^16.
+// One thread per key n < Npad of problem `problem`, whole warps per group.
+constexpr int kRecTile = 128;
+constexpr int kRecTileFloats = kRecTile + kRecTile / 32;
+
+__device__ __forceinline__ void write_sign_record(const __half* v, int64_t N, float* rec, int64_t n,
+                                                  int problem, int64_t npad) {
+    const float x = n < N ? __half2float(v[static_cast<int64_t>(problem) * N + n]) : 0.f;
+    const float sg = x > 0.f ? 65536.f : x < 0.f ? -65536.f : 0.f;
+    float* r = rec + (static_cast<int64_t>(problem) * (npad / kRecTile) + n / kRecTile) * kRecTileFloats;
+    const int kn = static_cast<int>(n % kRecTile);
+    r[kn] = sg;
+    // Zero values and padded keys contribute nothing whatever the group's
+    // sign (their folded exponent flushes), so only the signs of the
+    // nonzero values decide.
+    const bool any_pos = __any_sync(0xffffffffu, x > 0.f);
+    const bool any_neg = __any_sync(0xffffffffu, x < 0.f);
+    if ((kn & 31) == 0) r[kRecTile + kn / 32] = any_pos && any_neg ? 0.f : any_neg ? -65536.f : 65536.f;
+}
+
+// One block per problem: the AND over its 32-key groups of "values of one
+// sign" (group word != 0), into the word after all problems' records.
+__global__ void __launch_bounds__(256)
+vf_flags_kernel(float* __restrict__ rec, int64_t tiles, int batch) {
+    pdl_trigger();
+    pdl_wait();
+    const int b = blockIdx.x;
+    const float* gw = rec + static_cast<int64_t>(b) * tiles * kRecTileFloats + kRecTile;
+    bool mixed = false;
+    for (int64_t i = threadIdx.x; i < tiles * (kRecTile / 32); i += blockDim.x)
+        mixed |= gw[(i / (kRecTile / 32)) * kRecTileFloats + i % (kRecTile / 32)] == 0.f;
+    const int any_mixed = __syncthreads_or(mixed ? 1 : 0);
+    if (threadIdx.x == 0)
+        reinterpret_cast<unsigned*>(rec + static_cast<int64_t>(batch) * tiles * kRecTileFloats)[b] =
+            any_mixed ? 0u : 1u;
+}
+
+__global__ void sign_record_kernel(const __half* __restrict__ v, int64_t N, int64_t npad,
+                                   float* __restrict__ rec) {
+    pdl_trigger();
+    pdl_wait();
+    const int64_t n = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
+    if (n < npad) write_sign_record(v, N, rec, n, blockIdx.y, npad);
+}
 
 template <typename TV>
 __device__ __forceinline__ void write_key_record(const RecordJob<TV>& j, int64_t t, int problem) {
@@ -133,7 +184,13 @@ mean_partial_vec_kernel(const T* __restrict__ q, const T* __restrict__ k, int64_
     pdl_wait();
     if (static_cast<int>(blockIdx.x) >= G) {
         const int64_t t = static_cast<int64_t>(blockIdx.x - G) * kMeanVecThreads + threadIdx.x;
-        if (t < rj.pairs) write_key_record(rj, t, blockIdx.y);
+        if (rj.signs) {
+            if constexpr (std::is_same<TV, __half>::value) {
+                if (t < 2 * rj.pairs) write_sign_record(rj.v, rj.N, rj.rec, t, blockIdx.y, 2 * rj.pairs);
+            }
+        } else if (t < rj.pairs) {
+            write_key_record(rj, t, blockIdx.y);
+        }
         return;
     }
     __shared__ float s_sum[kMeanVecThreads][9];
@@ -313,6 +370,26 @@ mean_final_kernel(const float* __restrict__ partial, int G, int D, int64_t items
 // range.  Padded key rows get b_0 = -30000 / F (their values are zero as
 // well); padded query rows are zero.  `out_q` and/or `out_k` may be given
 // (both for q = k).
+//
+// Folded value magnitudes (vw given, one fp16 value per key): the key-side
+// term becomes b + log2(|v_n| 2^-16) / c, so that 2^(c S) = Phi |v_n| 2^-16;
+// the FMA kernel then needs only the signs of the values (see
+// write_sign_record).  |v_n| < 2^16 for every finite fp16 value, so the
+// exponent stays <= 0.  Keys with v_n = 0, and padded keys, get -256 / c
+// (at least -30000 for padded keys): their 2^(c S) flushes to zero, so they
+// may sit in a group of either sign.  inv_c = 1 / c.
+constexpr float kZeroWeightLog2 = -256.f;
+
+__device__ __forceinline__ float log_weight(const __half* vw, float inv_c) {
+    if (!vw) return 0.f;
+    const float a = fabsf(__half2float(*vw));
+    return a > 0.f ? log2f(a * (1.f / 65536.f)) * inv_c : kZeroWeightLog2 * inv_c;
+}
+
+// Norm term of a padded key row (b_0 of the split, times F).
+__device__ __forceinline__ float pad_key_term(bool fold, float inv_c) {
+    return fold ? fminf(-30000.f, kZeroWeightLog2 * inv_c) : -30000.f;
+}
 constexpr int kRowsPerBlock = 32;
 constexpr int kOperandThreads = 128;
 constexpr int kOperandMaxCols = 256;
@@ -321,7 +398,8 @@ template <typename T, bool AUG>
 __global__ void __launch_bounds__(kOperandThreads)
 operand_kernel(const T* __restrict__ x, int64_t rows, int64_t rows_pad, int D, int Dp, int nt, float F,
                const float* __restrict__ mu, float half_c, float pad_value,
-               T* __restrict__ out_q, T* __restrict__ out_k, float* __restrict__ nrm) {
+               T* __restrict__ out_q, T* __restrict__ out_k, float* __restrict__ nrm,
+               const __half* __restrict__ vw, float inv_c) {
     pdl_trigger();
     pdl_wait();
     constexpr int R = kRowsPerBlock;
@@ -345,6 +423,7 @@ operand_kernel(const T* __restrict__ x, int64_t rows, int64_t rows_pad, int D, i
         if (out_q) out_q += b * rows_pad * Dp;
         if (out_k) out_k += b * rows_pad * Dp;
         if (nrm) nrm += b * rows_pad;
+        if (vw) vw += b * rows;
     }
     const int64_t r0 = static_cast<int64_t>(blockIdx.x) * R;
     for (int d = tid; d < D; d += kOperandThreads) s_mu[d] = mu ? mu[d] : 0.f;
@@ -392,26 +471,33 @@ operand_kernel(const T* __restrict__ x, int64_t rows, int64_t rows_pad, int D, i
             if (wk) ok[d] = zero;
         }
         if (lane < nt) {
-            // Lane i writes term i of the split and its partner column.
-            T t = zero, one = zero;
-            if (valid) {
-                float r = -0.5f * acc;
-                t = from_f<T>(r / F);
+            // Lane i writes term i of the split and its partner column (the
+            // key side with its log weight, when values are folded).
+            auto split_term = [&](float r) {
+                T t = from_f<T>(r / F);
                 r -= F * to_f(t);
                 for (int i = 1; i <= lane; ++i) {
                     t = from_f<T>(r);
                     r -= to_f(t);
                 }
+                return t;
+            };
+            T t = zero, tk = zero, one = zero;
+            if (valid) {
+                t = split_term(-0.5f * acc);
+                const float lw = log_weight(vw ? vw + r0 + row : nullptr, inv_c);
+                tk = lw != 0.f ? split_term(-0.5f * acc + lw) : t;
                 one = from_f<T>(lane == 0 ? F : 1.f);
             } else if (lane == 0) {
                 t = from_f<T>(-30000.f / F);
+                tk = from_f<T>(pad_key_term(vw != nullptr, inv_c) / F);
             }
             if (wq) {
                 oq[D + lane] = valid ? one : zero;
                 oq[D + nt + lane] = valid ? t : zero;
             }
             if (wk) {
-                ok[D + lane] = t;
+                ok[D + lane] = tk;
                 ok[D + nt + lane] = one;
             }
         }
@@ -559,7 +645,8 @@ __device__ __forceinline__ float operand_row(const uint4 (&in)[kOperandVecs],
                                              const uint4* __restrict__ smean, int vi,
                                              bool in_pad, bool valid, int D, int Dp, int nt,
                                              float F, float half_c, float pad_value,
-                                             T* __restrict__ out_q, T* __restrict__ out_k) {
+                                             T* __restrict__ out_q, T* __restrict__ out_k,
+                                             bool fold, const __half* vw, float inv_c) {
     using PT = Pair<T>;
     const int V = D / 8;
     float acc = 0.f;
@@ -605,25 +692,32 @@ __device__ __forceinline__ float operand_row(const uint4 (&in)[kOperandVecs],
     // Built in registers: element e of the query tail is the partner
     // (F, 1, 1) for e < nt and t_(e - nt) for nt <= e < 2 nt; the key tail
     // the other way round; zeros after that.
-    unsigned short t0 = 0, t1 = 0, t2 = 0;
-    if (valid) {
-        float r = -0.5f * acc;
+    unsigned short t0 = 0, t1 = 0, t2 = 0, k0 = 0, k1 = 0, k2 = 0;
+    auto split = [&](float r, unsigned short& z0, unsigned short& z1, unsigned short& z2) {
         const T a0 = from_f<T>(r * (1.f / F));   // F is a power of two: exact
         r -= F * to_f(a0);
         const T a1 = from_f<T>(r);
         r -= to_f(a1);
         const T a2 = from_f<T>(r);
-        t0 = to_bits(a0);
-        t1 = to_bits(a1);
-        t2 = nt > 2 ? to_bits(a2) : 0;
+        z0 = to_bits(a0);
+        z1 = to_bits(a1);
+        z2 = nt > 2 ? to_bits(a2) : 0;
+    };
+    if (valid) {
+        split(-0.5f * acc, t0, t1, t2);
+        // Key side: the log weight of the folded value magnitude, if any.
+        const float lw = fold ? log_weight(vw, inv_c) : 0.f;
+        if (lw != 0.f) split(-0.5f * acc + lw, k0, k1, k2);
+        else { k0 = t0; k1 = t1; k2 = t2; }
     }
     const unsigned short oneF = valid ? to_bits(from_f<T>(F)) : 0;
     const unsigned short one1 = valid ? to_bits(from_f<T>(1.f)) : 0;
-    const unsigned short pad_b = valid ? t0 : to_bits(from_f<T>(-30000.f / F));
-    auto term = [&](int i) { return i == 0 ? pad_b : i == 1 ? t1 : t2; };
+    const unsigned short pad_b = valid ? k0 : to_bits(from_f<T>(pad_key_term(fold, inv_c) / F));
+    auto term = [&](int i) { return i == 0 ? pad_b : i == 1 ? k1 : k2; };
+    auto qterm = [&](int i) { return i == 0 ? t0 : i == 1 ? t1 : t2; };
     auto partner = [&](int i) { return i == 0 ? oneF : one1; };
     auto tail_q = [&](int e) -> unsigned {
-        return e < nt ? partner(e) : e < 2 * nt ? (e == nt ? t0 : term(e - nt)) : 0u;
+        return e < nt ? partner(e) : e < 2 * nt ? qterm(e - nt) : 0u;
     };
     auto tail_k = [&](int e) -> unsigned {
         return e < nt ? term(e) : e < 2 * nt ? partner(e - nt) : 0u;
@@ -657,6 +751,7 @@ struct OperandJob {
     void* out_q;
     void* out_k;
     float* nrm;
+    const void* vw;      // fp16 values of the rows written to out_k (folded magnitudes), or null
 };
 
 // Vector path of the operand preparation (D a multiple of 8): G lanes per
@@ -672,7 +767,8 @@ struct OperandJob {
 template <typename T, bool AUG, int G>
 __global__ void __launch_bounds__(kOperandVecThreads)
 operand_vec_kernel(const OperandJob j0, const OperandJob j1, unsigned blocks0, int D, int Dp,
-                   int nt, float F, const float* __restrict__ mu, float half_c, float pad_value) {
+                   int nt, float F, const float* __restrict__ mu, float half_c, float pad_value,
+                   float inv_c) {
     using PT = Pair<T>;
     pdl_trigger();
     pdl_wait();
@@ -705,18 +801,22 @@ operand_vec_kernel(const OperandJob j0, const OperandJob j1, unsigned blocks0, i
     const bool wk = AUG && j.out_k != nullptr;
     const bool in_pad = i < rows_pad;
     const int64_t row = static_cast<int64_t>(b) * rows_pad + i;   // batch-stacked output row
+    const bool fold = wk && j.vw;
+    const __half* vw = (fold && i < rows)
+                           ? static_cast<const __half*>(j.vw) + static_cast<int64_t>(b) * rows + i
+                           : nullptr;
     const float n = operand_row<T, AUG, G>(
         in, smean, vi, in_pad, i < rows, D, Dp, nt, F, half_c, pad_value,
         wq ? static_cast<T*>(j.out_q) + row * Dp : nullptr,
-        wk ? static_cast<T*>(j.out_k) + row * Dp : nullptr);
+        wk ? static_cast<T*>(j.out_k) + row * Dp : nullptr, fold, vw, inv_c);
     if (!AUG && in_pad && vi == 0) j.nrm[row] = n;
 }
 
 template <typename T, bool AUG>
 cudaError_t operand_typed(const OperandJob& j0, const OperandJob* j1, int D, int Dp, int nt,
                           float F, const float* mu, float half_c, float pad_value, cudaStream_t s,
-                          int batch) {
-    const OperandJob none = {nullptr, 0, 0, nullptr, nullptr, nullptr};
+                          int batch, float inv_c) {
+    const OperandJob none = {nullptr, 0, 0, nullptr, nullptr, nullptr, nullptr};
     for (const OperandJob* j : {&j0, j1}) {
         if (j && (j->rows_pad % kRowsPerBlock != 0)) return cudaErrorInvalidValue;
     }
@@ -736,7 +836,7 @@ cudaError_t operand_typed(const OperandJob& j0, const OperandJob* j1, int D, int
         auto go = [&](auto kern) {
             launch_kernel(kern, dim3(static_cast<unsigned>(b0 + b1), static_cast<unsigned>(batch)),
                           kOperandVecThreads, 0, s, j0, j1 ? *j1 : none, static_cast<unsigned>(b0),
-                          D, Dp, nt, F, mu, half_c, pad_value);
+                          D, Dp, nt, F, mu, half_c, pad_value, inv_c);
         };
         switch (G) {
             case 1: go(operand_vec_kernel<T, AUG, 1>); break;
@@ -757,7 +857,7 @@ cudaError_t operand_typed(const OperandJob& j0, const OperandJob* j1, int D, int
         launch_kernel(operand_kernel<T, AUG>, dim3(static_cast<unsigned>(blocks), batch),
                       kOperandThreads, smem, s, static_cast<const T*>(j->x), j->rows, j->rows_pad,
                       D, Dp, nt, F, mu, half_c, pad_value, static_cast<T*>(j->out_q),
-                      static_cast<T*>(j->out_k), j->nrm);
+                      static_cast<T*>(j->out_k), j->nrm, static_cast<const __half*>(j->vw), inv_c);
         note_launches(1);
         const cudaError_t e = cudaGetLastError();
         if (e != cudaSuccess) return e;
@@ -1090,12 +1190,15 @@ cudaError_t launch_mean(InType t, const void* q, const void* k, int64_t M, int64
         G = Gq + Gk;
         // Key records (see RecordJob) in blocks G .. G + rblocks - 1.
         const int64_t pairs = rec ? rec->Npad / 2 : 0;
-        const int rblocks = static_cast<int>((pairs + kMeanVecThreads - 1) / kMeanVecThreads);
+        // One thread per key pair, or per key for sign records.
+        const int64_t rthreads = rec && rec->signs ? 2 * pairs : pairs;
+        const int rblocks = static_cast<int>((rthreads + kMeanVecThreads - 1) / kMeanVecThreads);
         auto go = [&](auto tag, auto vtag) {
             using T = decltype(tag);
             using TV = decltype(vtag);
             const RecordJob<TV> rj = {rec ? static_cast<const TV*>(rec->v) : nullptr, rec ? rec->N : 0,
-                                      pairs, rec ? rec->C : 0, rec ? rec->out : nullptr};
+                                      pairs, rec ? rec->C : 0, rec ? rec->out : nullptr,
+                                      rec && rec->signs};
             launch_kernel(mean_partial_vec_kernel<T, TV>, dim3(G + rblocks, batch), kMeanVecThreads, 0,
                           s, static_cast<const T*>(q), static_cast<const T*>(k), M, N, D, rpb, Gq, G,
                           partial, rj);
@@ -1242,26 +1345,30 @@ cudaError_t launch_operands(InType t, bool aug, const void* q, int64_t M, int64_
                             void* qh, void* qh_as_key, float* nrm_q, bool with_k, const void* k,
                             int64_t N, int64_t Npad, void* kh, float* nrm_k, int D, int Dp,
                             const float* mu, float half_c, float pad_value, cudaStream_t s,
-                            int batch) {
+                            int batch, const void* vw) {
     OperandJob jq, jk;
     if (aug) {
-        jq = {q, M, Mpad, qh, qh_as_key, nullptr};
-        jk = {k, N, Npad, nullptr, kh, nullptr};
+        // vw: folded value magnitudes on the key rows (the q job writes the
+        // key rows too when q is k).
+        jq = {q, M, Mpad, qh, qh_as_key, nullptr, qh_as_key ? vw : nullptr};
+        jk = {k, N, Npad, nullptr, kh, nullptr, vw};
     } else {
-        jq = {q, M, Mpad, qh, nullptr, nrm_q};
-        jk = {k, N, Npad, kh, nullptr, nrm_k};
+        jq = {q, M, Mpad, qh, nullptr, nrm_q, nullptr};
+        jk = {k, N, Npad, kh, nullptr, nrm_k, nullptr};
     }
+    const float inv_c = half_c > 0.f ? 0.5f / half_c : 0.f;
     // (k itself may be null: an empty array when D = 0.)
     const OperandJob* j1 = with_k ? &jk : nullptr;
     const int nt = aug ? aug_norm_terms(t) : 0;
     if (t == InType::BF16) {
-        return aug ? operand_typed<__nv_bfloat16, true>(jq, j1, D, Dp, nt, 1.f, mu, 0.f, 0.f, s, batch)
+        return aug ? operand_typed<__nv_bfloat16, true>(jq, j1, D, Dp, nt, 1.f, mu, 0.f, 0.f, s, batch,
+                                                        inv_c)
                    : operand_typed<__nv_bfloat16, false>(jq, j1, D, Dp, 0, 1.f, mu, half_c,
-                                                         pad_value, s, batch);
+                                                         pad_value, s, batch, inv_c);
     }
-    return aug ? operand_typed<__half, true>(jq, j1, D, Dp, nt, 1024.f, mu, 0.f, 0.f, s, batch)
+    return aug ? operand_typed<__half, true>(jq, j1, D, Dp, nt, 1024.f, mu, 0.f, 0.f, s, batch, inv_c)
                : operand_typed<__half, false>(jq, j1, D, Dp, 0, 1.f, mu, half_c, pad_value, s,
-                                              batch);
+                                              batch, inv_c);
 }
 
 cudaError_t launch_tf32_split(const float* x, int64_t rows, int64_t rows_pad, int D, int Dp,
@@ -1297,7 +1404,16 @@ cudaError_t launch_value_prep(InType t, bool grad, bool w_f32, const void* w, co
 
 
 cudaError_t launch_key_records(InType t, const void* v, const float* B, int64_t N, int64_t Npad,
-                               int C, float* rec, cudaStream_t s, int batch) {
+                               int C, float* rec, cudaStream_t s, int batch, bool signs) {
+    if (signs) {
+        // Sign records (fp16 values, C = 1): one thread per key, 256 per block.
+        if (t != InType::F16 || C != 1 || B || Npad % kRecTile != 0) return cudaErrorInvalidValue;
+        if (Npad == 0) return cudaSuccess;
+        launch_kernel(sign_record_kernel, dim3(static_cast<unsigned>((Npad + 255) / 256), batch), 256, 0,
+                      s, static_cast<const __half*>(v), N, Npad, rec);
+        note_launches(1);
+        return cudaGetLastError();
+    }
     const int64_t pairs = Npad / 2;
     if (pairs == 0) return cudaSuccess;
     const int threads = 256;
@@ -1311,6 +1427,14 @@ cudaError_t launch_key_records(InType t, const void* v, const float* B, int64_t 
     else
         launch_kernel(key_record_kernel<__half>, dim3(blocks, batch), threads, 0, s, static_cast<const __half*>(v), B, N,
                                                              pairs, C, rec);
+    note_launches(1);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_vf_flags(float* rec, int64_t Npad, int batch, cudaStream_t s) {
+    if (batch <= 0) return cudaSuccess;
+    launch_kernel(vf_flags_kernel, dim3(static_cast<unsigned>(batch)), 256, 0, s, rec, Npad / kRecTile,
+                  batch);
     note_launches(1);
     return cudaGetLastError();
 }

@@ -921,7 +921,12 @@ bool plan_tensor(InType t, int64_t M, int64_t N, int64_t D, int64_t C, bool grad
     }
     if (p->fma) {
         p->off_vt = p->off_vmax = p->off_inv = 0;
-        p->off_rec = take(static_cast<size_t>(B) * (p->Npad / 2) * ((p->aug ? 0 : 2) + 2 * p->Cv) * 4);
+        // Key records: value pairs, or (one channel on augmented operands,
+        // when the value magnitudes are folded) 132 floats per key tile.
+        size_t rec_floats = static_cast<size_t>(p->Npad / 2) * ((p->aug ? 0 : 2) + 2 * p->Cv);
+        if (p->aug && p->Cv == 1) rec_floats = std::max<size_t>(rec_floats, (p->Npad / 128) * 132);
+        // (+ one word per problem: the folded-value pass flags.)
+        p->off_rec = take(static_cast<size_t>(B) * (rec_floats + 1) * 4);
         p->off_part = take(static_cast<size_t>(p->splits) * B * p->Mpad * p->Cv * 4);
     } else {
         p->off_rec = 0;

@@ -53,11 +53,18 @@
 //                their MMAs.  Warp 16 also allocates TMEM and loads q^.
 // Key records: for each pair of keys (2t, 2t + 1) the floats
 //   [B_2t, B_2t+1,] v_2t[0], v_2t+1[0], ..., v_2t[C-1], v_2t+1[C-1]
-// (B only without augmented operands).
+// (B only without augmented operands).  With folded value magnitudes (VF:
+// C = 1, fp16 values, augmented operands whose key norm terms carry
+// log2(|v_n| 2^-16) / c, so that 2^(c S) = Phi |v_n| 2^-16), the records of
+// a key tile are the signs s_n = sign(v_n) 2^16 in key order and one word
+// per 32-key column group, +-2^16 where all the group's values share a
+// sign, else 0: such a group's exponent loop then reads no record at all
+// (the broadcast record load per key pair was a fifth of its MIO work).
 #include <cuda.h>
 #include <cuda_runtime.h>
 
 #include <algorithm>
+#include <type_traits>
 
 #include "internal.h"
 #include "ptx.cuh"
@@ -209,8 +216,36 @@ __device__ __forceinline__ bool next_segment(const FmaParams& p, int u_end, int&
     return true;
 }
 
+// Folded values (VF): per-problem words after the sign records of all
+// problems, 1 where every 32-key group of the problem has values of one
+// sign (written by vf_flags_kernel).  Pass VF = 1 takes those problems
+// (the exponent loop reads no records), pass VF = 2 the others.
+template <int VF>
+__device__ __forceinline__ bool vf_takes(const FmaParams& p, int tile_m) {
+    if (VF == 0) return true;
+    const int problem = tile_m / p.pairs_per_batch;
+    const int batch = p.pairs_total / p.pairs_per_batch;
+    const unsigned* flags = reinterpret_cast<const unsigned*>(
+        p.rec + static_cast<int64_t>(batch) * (p.npad / BN) * (BN + BN / 32));
+    return (flags[problem] != 0u) == (VF == 1);
+}
+
 __device__ __forceinline__ void exp_warps_sync() {
     asm volatile("bar.sync 1, %0;" ::"r"(NEXP * 32) : "memory");
+}
+
+// The OR of v over all exponent warps, and a barrier of theirs: every
+// exponent warp gets the same answer (so that they leave their segment
+// loop together and never leave one of them waiting at a named barrier).
+__device__ __forceinline__ bool exp_warps_any(bool v) {
+    unsigned r;
+    asm volatile(
+        "{\n\t.reg .pred p, q;\n\tsetp.ne.u32 p, %1, 0;\n\t"
+        "bar.red.or.pred q, 1, %2, p;\n\tselp.u32 %0, 1, 0, q;\n\t}"
+        : "=r"(r)
+        : "r"(v ? 1u : 0u), "r"(NEXP * 32)
+        : "memory");
+    return r != 0u;
 }
 
 // AUG: augmented operands (S = -||q^ - k^||^2 / 2; no norm terms in the
@@ -219,13 +254,14 @@ __device__ __forceinline__ void exp_warps_sync() {
 // TRI: upper-triangle order for v^T K v (q = k, C = 1, augmented
 // operands): key tiles past the pair's own two get the weight 2, applied as
 // +1 in the exponent.
-template <int C, bool AUG, bool QSM, bool TF, bool TRI, int SOFT, bool OVL>
+template <int C, bool AUG, bool QSM, bool TF, bool TRI, int SOFT, bool OVL, int VF>
 __global__ void __launch_bounds__(THREADS, 1)
 tc_gauss_fma_kernel(const __grid_constant__ CUtensorMap tm_q,
                     const __grid_constant__ CUtensorMap tm_k, const FmaParams p) {
     // TF (3xTF32): q^ in shared memory, norm terms from A and the records.
     static_assert(!TF || (QSM && !AUG), "3xTF32 runs with q^ in shared memory");
     static_assert(!OVL || QSM, "overlapped segments keep q^ in shared memory");
+    static_assert(VF == 0 || (C == 1 && AUG && SOFT == 0), "folded values: C = 1, augmented operands");
     static_assert(SOFT == 0 || (AUG && !TRI), "FMA-pipe exponentials: augmented operands");
     constexpr int kSoftMask = soft_mask(SOFT);
     constexpr int REC_PAIR = (AUG ? 0 : 2) + 2 * C;   // floats per key pair
@@ -290,10 +326,20 @@ tc_gauss_fma_kernel(const __grid_constant__ CUtensorMap tm_q,
     const int u_end = p.units < u_begin + p.unit_len ? p.units : u_begin + p.unit_len;
     // Segment barrier of both role loops (a non-aligned barrier, since the
     // two roles reach it from different loops).
-    auto segment_sync = [&]() {
+    // Segment end of both role loops (not OVL; a non-aligned barrier, since
+    // the two roles reach it from different loops), with the OR of the
+    // threads' abort observations: all roles leave the loop together.
+    auto segment_sync_any = [&](bool v) -> bool {
         tc_fence_before();
-        asm volatile("barrier.sync 2, %0;" ::"r"(THREADS) : "memory");
+        unsigned r;
+        asm volatile(
+            "{\n\t.reg .pred p, q;\n\tsetp.ne.u32 p, %1, 0;\n\t"
+            "barrier.red.or.pred q, 2, %2, p;\n\tselp.u32 %0, 1, 0, q;\n\t}"
+            : "=r"(r)
+            : "r"(v ? 1u : 0u), "r"(THREADS)
+            : "memory");
         tc_fence_after();
+        return r != 0u;
     };
     if (warp >= CTRL_WARP0) {
         // Control warps need few registers; the exponent warps take them
@@ -306,8 +352,12 @@ tc_gauss_fma_kernel(const __grid_constant__ CUtensorMap tm_q,
         uint32_t seg_parity = 0;   // parity of the qa_ready phase of this segment
         int u = u_begin, run = 0, g0 = 0;   // g0: running index of the segment's first tile
         Segment sg;
-        for (; next_segment<TRI>(p, u_end, u, run, sg); seg_parity ^= 1u, g0 += sg.T) {
-        if (__any_sync(0xffffffffu, *abort_flag != 0)) break;
+        for (; next_segment<TRI>(p, u_end, u, run, sg); ) {
+        // Segments of the other folded-value pass are skipped, and the
+        // running tile index and the q^ phase count only this pass's tiles.
+        if (!vf_takes<VF>(p, sg.tile_m)) continue;
+        // (Not OVL: the abort decision is taken at the segment-end barrier.)
+        if (OVL && __any_sync(0xffffffffu, *abort_flag != 0)) break;
         const int tile_m = sg.tile_m;         // query tiles 2 tile_m, 2 tile_m + 1
         // First k^ row of this pair's problem (batch-stacked operands).
         const int kbase = (tile_m / p.pairs_per_batch) * p.npad;
@@ -353,8 +403,9 @@ tc_gauss_fma_kernel(const __grid_constant__ CUtensorMap tm_q,
                         tma_load_2d(kh_smem(k) + kb * (BN * 128), &tm_k, &bars->kv_full[k],
                                     kb * p.kb_elems, n0);
                     bulk_load(const_cast<float*>(rec_smem(k)),
-                              p.rec + static_cast<int64_t>(n0 / 2) * REC_PAIR, p.rec_bytes,
-                              &bars->kv_full[k]);
+                              p.rec + (VF != 0 ? static_cast<int64_t>(n0 / BN) * (BN + BN / 32)
+                                          : static_cast<int64_t>(n0 / 2) * REC_PAIR),
+                              p.rec_bytes, &bars->kv_full[k]);
                 };
                 // Parity of stage k's barriers for tile j: stage k completes once
                 // per tile g = k (mod nctrl).
@@ -490,12 +541,12 @@ tc_gauss_fma_kernel(const __grid_constant__ CUtensorMap tm_q,
                 mbar_wait_bounded(&bars->qa_ready, seg_parity, nullptr, p.status);
                 __syncwarp();
             }
-            if (!OVL) {
-                // Segment end: every MMA, copy and TMEM read of this segment
-                // is done (control warps waited for their last stage release
-                // and copies).
-                segment_sync();
-            }
+            // Segment end (not OVL): every MMA, copy and TMEM read of this
+            // segment is done (control warps waited for their last stage
+            // release and copies).
+            if (!OVL && segment_sync_any(*abort_flag != 0)) break;
+            seg_parity ^= 1u;
+            g0 += sg.T;
         }
         // No MMA of this warp may still run when TMEM is freed.  Without an
         // abort the last stage-release wait has already seen them complete;
@@ -514,8 +565,10 @@ tc_gauss_fma_kernel(const __grid_constant__ CUtensorMap tm_q,
         uint32_t seg_parity = 0;
         int u = u_begin, run = 0, g0 = 0;
         Segment sg;
-        for (; next_segment<TRI>(p, u_end, u, run, sg); seg_parity ^= 1u, g0 += sg.T) {
-        if (__any_sync(0xffffffffu, *abort_flag != 0)) break;
+        for (; next_segment<TRI>(p, u_end, u, run, sg); ) {
+        if (!vf_takes<VF>(p, sg.tile_m)) continue;   // the other folded-value pass
+        // (The abort decision is taken at the end of each segment, at a
+        // barrier of all exponent warps.)
         const int tile_m = sg.tile_m;         // query tiles 2 tile_m, 2 tile_m + 1
         const int T = sg.T;
         // TRI: tiles j >= w_from of this segment lie past the pair's own two
@@ -565,140 +618,168 @@ tc_gauss_fma_kernel(const __grid_constant__ CUtensorMap tm_q,
             st.phase = static_cast<uint32_t>(g0 / p.stages) & 1u;
             sl.idx = g0 % SL;
             sl.phase = static_cast<uint32_t>(g0 / SL) & 1u;
-            for (int j = 0; j < T; ++j, st.advance(p.stages), sl.advance(SL)) {
-                const int s = st.idx;
-                const uint32_t col0 = static_cast<uint32_t>(sl.idx * 2 * BN);
-                if (!__all_sync(0xffffffffu, ready || mbar_test_wait2(&bars->kv_full[s], st.phase,
-                                                                      &bars->s_full[sl.idx], sl.phase))) {
-                    ok = warp_wait(&bars->kv_full[s], st.phase, abort_flag, p.status);
-                    if (ok) ok = warp_wait(&bars->s_full[sl.idx], sl.phase, abort_flag, p.status);
-                    if (!ok) break;
-                }
-                tc_fence_after();
-                uint32_t r0[32], r1[32];
-                tmem_ld_32x32b_x32(tmem + lane_base + col0 + cg * 32, r0);
-                tmem_ld_32x32b_x32(tmem + lane_base + col0 + BN + cg * 32, r1);
-                // The wait names r0 and r1, so that no use of the loaded
-                // values is scheduled above it (the loads land asynchronously).
-                tmem_wait_ld_regs(r0, r1);
-                // When and where the S slot is handed back: with two slots
-                // (q^ in shared memory) only after the exponent work of this
-                // tile (with the stage, below), because releasing it right
-                // after the loads let the next MMAs into the slot corrupt S
-                // values of this tile in some warps when the MMAs were long
-                // (measured with 3xTF32 operands and three or more stages,
-                // also with the loads' registers named in the wait; the early
-                // release was no faster on the 65536^2, D = 64 sum either:
-                // 0.6428 against 0.6418 ms).
-                // With one slot (q^ in TMEM) a late release would serialise
-                // the MMAs and the exponent work, so it is released here; no
-                // corruption was seen there in repeated runs (regression
-                // test: repeated calls agree bit for bit).
-                if (!QSM) {
-                    tc_fence_before();
-                    __syncwarp();
-                    mbar_arrive_if_zero(&bars->s_free[sl.idx], lane);
-                }
-                // Query the barriers of key tile j + 1 now and read the answer
-                // after the exponent work of tile j: the query latency overlaps
-                // the arithmetic instead of stalling all exponent warps at once.
-                // A phase seen complete stays complete until this warp releases
-                // that stage and slot.  Two slots only: with one, tile j + 1
-                // needs the slot this warp has just handed back, so the query
-                // would always fail (and skipping it measured 4 % faster on
-                // the D = 256, 1M-key workload).  Not with 3xTF32 operands
-                // either: their three MMAs per K step make the next tile rarely
-                // ready this early (skipping the query: fp32 65536^2 sums 4-5 %
-                // faster).
-                if (QSM && !TF) {
-                    RingPos st2 = st, sl2 = sl;
-                    st2.advance(p.stages);
-                    sl2.advance(SL);
-                    ready = j + 1 < T && mbar_test_wait2(&bars->kv_full[st2.idx], st2.phase,
-                                                         &bars->s_full[sl2.idx], sl2.phase);
-                }
-                const float* rec = rec_smem(s) + (cg * 16) * REC_PAIR;
-                const uint64_t w2 = (TRI && j >= w_from) ? f32x2_pack(1.f, 1.f) : 0ull;
-                if (AUG) {
-                    // Augmented operands: S = -||q^ - k^||^2 / 2, so Phi = 2^(c S).
-                    // Keys 32 cg + 2t and + 1, rows row0 (S0) and row1 (S1).
-    #pragma unroll
-                    for (int t = 0; t < 16; ++t) {
-                        const float* pr = rec + t * REC_PAIR;
-                        uint64_t px, py;
-                        if (SOFT > 0 && (t & kSoftMask) == 0) {
-                            px = exp2_fma_x2(__uint_as_float(r0[2 * t]), __uint_as_float(r0[2 * t + 1]), c2, s_min);
-                        } else {
-                            float x0, x1;
+            // The key-tile loop; FAST (folded values, pass 1): every 32-key
+            // group of the problem has values of one sign, and the exponent
+            // loop reads no records.  (One kernel holding both versions of the
+            // loop measured 3 % slower on the fast one than a kernel with the
+            // fast one alone.)
+            auto tile_loop = [&](auto fast_tag) {
+                constexpr bool FAST = decltype(fast_tag)::value;
+                for (int j = 0; j < T; ++j, st.advance(p.stages), sl.advance(SL)) {
+                    const int s = st.idx;
+                    const uint32_t col0 = static_cast<uint32_t>(sl.idx * 2 * BN);
+                    if (!__all_sync(0xffffffffu, ready || mbar_test_wait2(&bars->kv_full[s], st.phase,
+                                                                          &bars->s_full[sl.idx], sl.phase))) {
+                        ok = warp_wait(&bars->kv_full[s], st.phase, abort_flag, p.status);
+                        if (ok) ok = warp_wait(&bars->s_full[sl.idx], sl.phase, abort_flag, p.status);
+                        if (!ok) break;
+                    }
+                    tc_fence_after();
+                    uint32_t r0[32], r1[32];
+                    tmem_ld_32x32b_x32(tmem + lane_base + col0 + cg * 32, r0);
+                    tmem_ld_32x32b_x32(tmem + lane_base + col0 + BN + cg * 32, r1);
+                    // The wait names r0 and r1, so that no use of the loaded
+                    // values is scheduled above it (the loads land asynchronously).
+                    tmem_wait_ld_regs(r0, r1);
+                    // When and where the S slot is handed back: with two slots
+                    // (q^ in shared memory) only after the exponent work of this
+                    // tile (with the stage, below), because releasing it right
+                    // after the loads let the next MMAs into the slot corrupt S
+                    // values of this tile in some warps when the MMAs were long
+                    // (measured with 3xTF32 operands and three or more stages,
+                    // also with the loads' registers named in the wait; the early
+                    // release was no faster on the 65536^2, D = 64 sum either:
+                    // 0.6428 against 0.6418 ms).
+                    // With one slot (q^ in TMEM) a late release would serialise
+                    // the MMAs and the exponent work, so it is released here; no
+                    // corruption was seen there in repeated runs (regression
+                    // test: repeated calls agree bit for bit).
+                    if (!QSM) {
+                        tc_fence_before();
+                        __syncwarp();
+                        mbar_arrive_if_zero(&bars->s_free[sl.idx], lane);
+                    }
+                    // Query the barriers of key tile j + 1 now and read the answer
+                    // after the exponent work of tile j: the query latency overlaps
+                    // the arithmetic instead of stalling all exponent warps at once.
+                    // A phase seen complete stays complete until this warp releases
+                    // that stage and slot.  Two slots only: with one, tile j + 1
+                    // needs the slot this warp has just handed back, so the query
+                    // would always fail (and skipping it measured 4 % faster on
+                    // the D = 256, 1M-key workload).  Not with 3xTF32 operands
+                    // either: their three MMAs per K step make the next tile rarely
+                    // ready this early (skipping the query: fp32 65536^2 sums 4-5 %
+                    // faster).
+                    if (QSM && !TF) {
+                        RingPos st2 = st, sl2 = sl;
+                        st2.advance(p.stages);
+                        sl2.advance(SL);
+                        ready = j + 1 < T && mbar_test_wait2(&bars->kv_full[st2.idx], st2.phase,
+                                                             &bars->s_full[sl2.idx], sl2.phase);
+                    }
+                    const float* rec = rec_smem(s) + (cg * 16) * REC_PAIR;
+                    const uint64_t w2 = (TRI && j >= w_from) ? f32x2_pack(1.f, 1.f) : 0ull;
+                    if constexpr (FAST) {
+                        // Folded values, every group of this problem of one sign:
+                        // P = Phi |v| 2^-16 from the MMA's exponent, times this
+                        // column group's sign word +-2^16; no per-key records.
+                        const float uw = rec_smem(s)[BN + cg];
+                        const uint64_t u2 = f32x2_pack(uw, uw);
+        #pragma unroll
+                        for (int t = 0; t < 16; ++t) {
+                            float x0, x1, y0, y1;
                             const uint64_t sx = f32x2_pack(__uint_as_float(r0[2 * t]), __uint_as_float(r0[2 * t + 1]));
-                            f32x2_unpack(TRI ? f32x2_fma(sx, c2, w2) : f32x2_mul(sx, c2), x0, x1);
-                            px = f32x2_pack(TRI ? ex2_approx(x0) : ex2_nonpos(x0),
-                                            TRI ? ex2_approx(x1) : ex2_nonpos(x1));
-                        }
-                        {
-                            float y0, y1;
                             const uint64_t sy = f32x2_pack(__uint_as_float(r1[2 * t]), __uint_as_float(r1[2 * t + 1]));
+                            f32x2_unpack(TRI ? f32x2_fma(sx, c2, w2) : f32x2_mul(sx, c2), x0, x1);
                             f32x2_unpack(TRI ? f32x2_fma(sy, c2, w2) : f32x2_mul(sy, c2), y0, y1);
-                            py = f32x2_pack(TRI ? ex2_approx(y0) : ex2_nonpos(y0),
-                                            TRI ? ex2_approx(y1) : ex2_nonpos(y1));
+                            const uint64_t px = f32x2_pack(TRI ? ex2_approx(x0) : ex2_nonpos(x0),
+                                                           TRI ? ex2_approx(x1) : ex2_nonpos(x1));
+                            const uint64_t py = f32x2_pack(TRI ? ex2_approx(y0) : ex2_nonpos(y0),
+                                                           TRI ? ex2_approx(y1) : ex2_nonpos(y1));
+                            acc0[0] = f32x2_fma(px, u2, acc0[0]);
+                            acc1[0] = f32x2_fma(py, u2, acc1[0]);
                         }
-    #pragma unroll
-                        for (int cc = 0; cc < C; ++cc) {
-                            const float2 vc = *reinterpret_cast<const float2*>(pr + 2 * cc);
+                    } else if (AUG) {
+                        // Augmented operands: S = -||q^ - k^||^2 / 2, so Phi = 2^(c S)
+                        // (VF: Phi |v| 2^-16, the records holding the signs 2^16).
+                        // Keys 32 cg + 2t and + 1, rows row0 (S0) and row1 (S1).
+        #pragma unroll
+                        for (int t = 0; t < 16; ++t) {
+                            const float* pr = rec + t * REC_PAIR;
+                            uint64_t px, py;
+                            if (SOFT > 0 && (t & kSoftMask) == 0) {
+                                px = exp2_fma_x2(__uint_as_float(r0[2 * t]), __uint_as_float(r0[2 * t + 1]), c2, s_min);
+                            } else {
+                                float x0, x1;
+                                const uint64_t sx = f32x2_pack(__uint_as_float(r0[2 * t]), __uint_as_float(r0[2 * t + 1]));
+                                f32x2_unpack(TRI ? f32x2_fma(sx, c2, w2) : f32x2_mul(sx, c2), x0, x1);
+                                px = f32x2_pack(TRI ? ex2_approx(x0) : ex2_nonpos(x0),
+                                                TRI ? ex2_approx(x1) : ex2_nonpos(x1));
+                            }
+                            {
+                                float y0, y1;
+                                const uint64_t sy = f32x2_pack(__uint_as_float(r1[2 * t]), __uint_as_float(r1[2 * t + 1]));
+                                f32x2_unpack(TRI ? f32x2_fma(sy, c2, w2) : f32x2_mul(sy, c2), y0, y1);
+                                py = f32x2_pack(TRI ? ex2_approx(y0) : ex2_nonpos(y0),
+                                                TRI ? ex2_approx(y1) : ex2_nonpos(y1));
+                            }
+        #pragma unroll
+                            for (int cc = 0; cc < C; ++cc) {
+                                const float2 vc = *reinterpret_cast<const float2*>(pr + 2 * cc);
+                                const uint64_t vv = f32x2_pack(vc.x, vc.y);
+                                acc0[cc] = f32x2_fma(px, vv, acc0[cc]);
+                                acc1[cc] = f32x2_fma(py, vv, acc1[cc]);
+                            }
+                        }
+                    } else {
+        #pragma unroll
+                    for (int t = 0; t < 16; ++t) {
+                        // Keys 32 cg + 2t and + 1, rows row0 (S0) and row1 (S1).
+                        const float* pr = rec + t * REC_PAIR;
+                        float2 bb, v0;
+                        if (C == 1) {
+                            const float4 bv = *reinterpret_cast<const float4*>(pr);
+                            bb = make_float2(bv.x, bv.y);
+                            v0 = make_float2(bv.z, bv.w);
+                        } else {
+                            bb = *reinterpret_cast<const float2*>(pr);
+                            v0 = *reinterpret_cast<const float2*>(pr + 2);
+                        }
+                        const uint64_t b2 = f32x2_pack(bb.x, bb.y);
+                        const uint64_t x01 = f32x2_fma(f32x2_pack(__uint_as_float(r0[2 * t]), __uint_as_float(r0[2 * t + 1])),
+                                                       c2, f32x2_add(b2, a2_0));
+                        const uint64_t y01 = f32x2_fma(f32x2_pack(__uint_as_float(r1[2 * t]), __uint_as_float(r1[2 * t + 1])),
+                                                       c2, f32x2_add(b2, a2_1));
+                        float x0, x1, y0, y1;
+                        f32x2_unpack(x01, x0, x1);
+                        f32x2_unpack(y01, y0, y1);
+                        const uint64_t px = f32x2_pack(ex2_nonpos(x0), ex2_nonpos(x1));
+                        const uint64_t py = f32x2_pack(ex2_nonpos(y0), ex2_nonpos(y1));
+                        const uint64_t vv0 = f32x2_pack(v0.x, v0.y);
+                        acc0[0] = f32x2_fma(px, vv0, acc0[0]);
+                        acc1[0] = f32x2_fma(py, vv0, acc1[0]);
+        #pragma unroll
+                        for (int cc = 1; cc < C; ++cc) {
+                            const float2 vc = *reinterpret_cast<const float2*>(pr + 2 + 2 * cc);
                             const uint64_t vv = f32x2_pack(vc.x, vc.y);
                             acc0[cc] = f32x2_fma(px, vv, acc0[cc]);
                             acc1[cc] = f32x2_fma(py, vv, acc1[cc]);
                         }
                     }
-                } else {
-    #pragma unroll
-                for (int t = 0; t < 16; ++t) {
-                    // Keys 32 cg + 2t and + 1, rows row0 (S0) and row1 (S1).
-                    const float* pr = rec + t * REC_PAIR;
-                    float2 bb, v0;
-                    if (C == 1) {
-                        const float4 bv = *reinterpret_cast<const float4*>(pr);
-                        bb = make_float2(bv.x, bv.y);
-                        v0 = make_float2(bv.z, bv.w);
-                    } else {
-                        bb = *reinterpret_cast<const float2*>(pr);
-                        v0 = *reinterpret_cast<const float2*>(pr + 2);
                     }
-                    const uint64_t b2 = f32x2_pack(bb.x, bb.y);
-                    const uint64_t x01 = f32x2_fma(f32x2_pack(__uint_as_float(r0[2 * t]), __uint_as_float(r0[2 * t + 1])),
-                                                   c2, f32x2_add(b2, a2_0));
-                    const uint64_t y01 = f32x2_fma(f32x2_pack(__uint_as_float(r1[2 * t]), __uint_as_float(r1[2 * t + 1])),
-                                                   c2, f32x2_add(b2, a2_1));
-                    float x0, x1, y0, y1;
-                    f32x2_unpack(x01, x0, x1);
-                    f32x2_unpack(y01, y0, y1);
-                    const uint64_t px = f32x2_pack(ex2_nonpos(x0), ex2_nonpos(x1));
-                    const uint64_t py = f32x2_pack(ex2_nonpos(y0), ex2_nonpos(y1));
-                    const uint64_t vv0 = f32x2_pack(v0.x, v0.y);
-                    acc0[0] = f32x2_fma(px, vv0, acc0[0]);
-                    acc1[0] = f32x2_fma(py, vv0, acc1[0]);
-    #pragma unroll
-                    for (int cc = 1; cc < C; ++cc) {
-                        const float2 vc = *reinterpret_cast<const float2*>(pr + 2 + 2 * cc);
-                        const uint64_t vv = f32x2_pack(vc.x, vc.y);
-                        acc0[cc] = f32x2_fma(px, vv, acc0[cc]);
-                        acc1[cc] = f32x2_fma(py, vv, acc1[cc]);
-                    }
+                    tc_fence_before();
+                    __syncwarp();
+                    // Lane 0 hands back the slot (two-slot path) and the stage,
+                    // predicated rather than branched: a divergent branch here
+                    // cost 0.7 % of the kernel time.
+                    if (QSM) mbar_arrive2_if_zero(&bars->s_free[sl.idx], &bars->kv_empty[s], lane);
+                    else mbar_arrive_if_zero(&bars->kv_empty[s], lane);
                 }
-                }
-                tc_fence_before();
-                __syncwarp();
-                // Lane 0 hands back the slot (two-slot path) and the stage,
-                // predicated rather than branched: a divergent branch here
-                // cost 0.7 % of the kernel time.
-                if (QSM) mbar_arrive2_if_zero(&bars->s_free[sl.idx], &bars->kv_empty[s], lane);
-                else mbar_arrive_if_zero(&bars->kv_empty[s], lane);
-            }
+            };
+            tile_loop(std::integral_constant<bool, VF == 1>{});
             // Fixed-order reduction of the NPART column-group partial sums.
-            // (OVL: the warps do not meet at segment ends, so the reduction
-            // area of the previous segment must have been read by every warp
-            // before it is written again.)
-            if (OVL) exp_warps_sync();
+            // (The reduction area of the previous segment has been read by
+            // every warp: they met at its end.)
     #pragma unroll
             for (int cc = 0; cc < C; ++cc) {
                 float lo, hi;
@@ -720,9 +801,13 @@ tc_gauss_fma_kernel(const __grid_constant__ CUtensorMap tm_q,
                     out[cc] = sum;
                 }
             }
-        // Segment end: every MMA, copy and TMEM read of this segment is done
-        // (not OVL; with q^ in TMEM, before the exponent warps copy the next q^).
-        if (!OVL) segment_sync();
+        // Segment end: every exponent warp is done with the reduction area;
+        // not OVL also every MMA, copy and TMEM read of the segment (with q^
+        // in TMEM, before the exponent warps copy the next q^).  The abort
+        // decision is the same for all warps that meet here.
+        if (OVL ? exp_warps_any(*abort_flag != 0) : segment_sync_any(*abort_flag != 0)) break;
+        seg_parity ^= 1u;
+        g0 += sg.T;
         }
     }
 
@@ -740,9 +825,14 @@ size_t align1k(size_t x) { return (x + 1023) & ~static_cast<size_t>(1023); }
 // are folded into augmented operands) + both keys' values.
 int rec_pair_floats(int C, bool aug) { return (aug ? 0 : 2) + 2 * C; }
 
-size_t stage_bytes_for(int nkb, int C, bool aug) {
-    return align1k(static_cast<size_t>(nkb) * BN * 128 +
-                   static_cast<size_t>(BN / 2) * rec_pair_floats(C, aug) * 4);
+// Key-record bytes of one key tile (VF: the signs and four group words).
+size_t rec_bytes_for(int C, bool aug, bool vf) {
+    return vf ? static_cast<size_t>(BN + BN / 32) * 4
+              : static_cast<size_t>(BN / 2) * rec_pair_floats(C, aug) * 4;
+}
+
+size_t stage_bytes_for(int nkb, int C, bool aug, bool vf = false) {
+    return align1k(static_cast<size_t>(nkb) * BN * 128 + rec_bytes_for(C, aug, vf));
 }
 
 size_t fixed_bytes_for(int C, size_t q_bytes) {
@@ -759,7 +849,8 @@ size_t q_bytes_for(int nkb, bool qsm) {
     return qsm ? static_cast<size_t>(NQ) * nkb * BM * 128 : 0;
 }
 
-template <int C, bool AUG, bool QSM, bool TF, bool TRI = false, int SOFT = 0, bool OVL = false>
+template <int C, bool AUG, bool QSM, bool TF, bool TRI = false, int SOFT = 0, bool OVL = false,
+          int VF = 0>
 cudaError_t launch_typed(const TcPlan& pl, InType t, float c, char* ws, unsigned* status,
                          cudaStream_t s, const char** why) {
     const CUtensorMapDataType hdt =
@@ -797,28 +888,44 @@ cudaError_t launch_typed(const TcPlan& pl, InType t, float c, char* ws, unsigned
     p.stages = pl.stages;
     p.q_bytes = static_cast<uint32_t>(q_bytes_for(p.nkb, QSM));
     p.kh_bytes = static_cast<uint32_t>(p.nkb * BN * 128);
-    p.rec_bytes = static_cast<uint32_t>((BN / 2) * rec_pair_floats(C, AUG) * 4);
-    p.stage_bytes = static_cast<uint32_t>(stage_bytes_for(p.nkb, C, AUG));
+    p.rec_bytes = static_cast<uint32_t>(rec_bytes_for(C, AUG, VF != 0));
+    p.stage_bytes = static_cast<uint32_t>(stage_bytes_for(p.nkb, C, AUG, VF != 0));
     p.red_offset = p.q_bytes + static_cast<uint32_t>(pl.stages * p.stage_bytes);
     p.c = c;
     const uint32_t hb = t == InType::BF16 ? 1u : 0u;
     p.idesc = TF ? idesc_tf32(BM, BN) : idesc_f16(BM, BN, hb, hb);
-    cudaError_t e = cudaFuncSetAttribute(tc_gauss_fma_kernel<C, AUG, QSM, TF, TRI, SOFT, OVL>,
+    cudaError_t e = cudaFuncSetAttribute(tc_gauss_fma_kernel<C, AUG, QSM, TF, TRI, SOFT, OVL, VF>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          static_cast<int>(pl.smem_bytes));
     if (e != cudaSuccess) return e;
     dim3 grid(static_cast<unsigned>(pl.grid));
-    launch_kernel(tc_gauss_fma_kernel<C, AUG, QSM, TF, TRI, SOFT, OVL>, grid, THREADS, pl.smem_bytes, s, tm_q, tm_k, p);
+    launch_kernel(tc_gauss_fma_kernel<C, AUG, QSM, TF, TRI, SOFT, OVL, VF>, grid, THREADS, pl.smem_bytes, s, tm_q, tm_k, p);
     note_launches(1);
     return cudaGetLastError();
 }
 
 template <int C>
 cudaError_t launch_c(const TcPlan& pl, InType t, float c, char* ws, unsigned* status,
-                     cudaStream_t s, const char** why) {
+                     cudaStream_t s, const char** why, int vf_pass) {
     if (pl.tf) return launch_typed<C, false, true, true>(pl, t, c, ws, status, s, why);
     if constexpr (C == 1 && kAugQsm) {
+        // Folded values: pass 1 (problems whose groups are all of one sign)
+        // or pass 2 (the others).
+        if (pl.tri && pl.aug && vf_pass == 1)
+            return launch_typed<1, true, true, false, true, 0, false, 1>(pl, t, c, ws, status, s, why);
+        if (pl.tri && pl.aug && vf_pass == 2)
+            return launch_typed<1, true, true, false, true, 0, false, 2>(pl, t, c, ws, status, s, why);
         if (pl.tri && pl.aug) return launch_typed<1, true, true, false, true>(pl, t, c, ws, status, s, why);
+        if (pl.aug && vf_pass == 1) {
+            if (pl.overlap)
+                return launch_typed<1, true, true, false, false, 0, true, 1>(pl, t, c, ws, status, s, why);
+            return launch_typed<1, true, true, false, false, 0, false, 1>(pl, t, c, ws, status, s, why);
+        }
+        if (pl.aug && vf_pass == 2) {
+            if (pl.overlap)
+                return launch_typed<1, true, true, false, false, 0, true, 2>(pl, t, c, ws, status, s, why);
+            return launch_typed<1, true, true, false, false, 0, false, 2>(pl, t, c, ws, status, s, why);
+        }
         if (pl.aug && pl.exp2_fma > 0) {
             switch (pl.exp2_fma) {
                 case 1: return launch_typed<1, true, true, false, false, 1>(pl, t, c, ws, status, s, why);
@@ -865,15 +972,16 @@ bool plan_fma_kernel(int Dp, int C, bool aug, bool tf, int* nq, int* stages, siz
 }
 
 cudaError_t launch_tc_fma(const TcPlan& p, InType t, float c, char* ws, unsigned* status,
-                          cudaStream_t s, const char** why) {
+                          cudaStream_t s, const char** why, int vf_pass) {
     const bool qsm = p.tf || (p.aug && kAugQsm);
     note_fma_variant((p.aug && kAugQsm && p.overlap && !p.tri && p.exp2_fma == 0 ? 1 : 0) |
-                     (p.band_len > 0 ? 2 : 0) | (qsm ? 0 : 4));
+                     (p.band_len > 0 ? 2 : 0) | (qsm ? 0 : 4) |
+                     (p.vfold && p.aug && kAugQsm && p.Cv == 1 && p.exp2_fma == 0 ? 8 : 0));
     switch (p.Cv) {
-        case 1: return launch_c<1>(p, t, c, ws, status, s, why);
-        case 2: return launch_c<2>(p, t, c, ws, status, s, why);
-        case 3: return launch_c<3>(p, t, c, ws, status, s, why);
-        default: return launch_c<4>(p, t, c, ws, status, s, why);
+        case 1: return launch_c<1>(p, t, c, ws, status, s, why, vf_pass);
+        case 2: return launch_c<2>(p, t, c, ws, status, s, why, vf_pass);
+        case 3: return launch_c<3>(p, t, c, ws, status, s, why, vf_pass);
+        default: return launch_c<4>(p, t, c, ws, status, s, why, vf_pass);
     }
 }
 

@@ -112,3 +112,95 @@ def test_fma_segment_overlap_switch(M, N, overlap, banded):
     flags = testing_last_fma_variant()
     assert bool(flags & 1) == overlap, flags
     assert bool(flags & 2) == banded, flags
+
+
+def _value_pattern(N, pattern, rng):
+    """fp16 values with the sign structure the folded-value path
+    distinguishes: groups of 32 keys of one sign (no record loads), mixed
+    groups, zeros, and magnitudes across the fp16 range."""
+    import numpy as np
+    if pattern == "halves":          # MMD weights: every group of one sign
+        v = np.where(np.arange(N) < N // 2, 1.0, -1.0) / N
+    elif pattern == "random":        # mixed groups throughout
+        v = rng.standard_normal(N)
+    elif pattern == "blocks":        # runs of 32 or 96 keys of one sign, some groups with a zero
+        v = np.repeat(np.where(rng.random((N + 31) // 32) < 0.5, 1.0, -1.0), 32)[:N]
+        v = v * rng.uniform(0.5, 2.0, N)
+        v[rng.choice(N, size=max(1, N // 100), replace=False)] = 0.0
+    else:                            # "range": magnitudes from subnormal to near 65504
+        v = np.exp2(rng.uniform(-23.0, 15.9, N)) * np.where(rng.random(N) < 0.5, 1.0, -1.0)
+    return v.astype(np.float16).reshape(N, 1)
+
+
+@pytest.mark.parametrize("pattern", ["halves", "random", "blocks", "range"])
+@pytest.mark.parametrize("center", [True, False])
+def test_folded_value_magnitudes(pattern, center):
+    """One fp16 value channel: the value magnitudes are folded into the key
+    operands (log2(|v| 2^-16) / c in the key norm term) and the key records
+    hold only signs, with a per-32-key-group sign word that lets groups of
+    one sign skip the record loads.  Against the oracle for every sign
+    pattern, with and without centring (the sign records then come from
+    their own kernel rather than the mean launch).  The shape gives every
+    CTA long runs of key tiles (65 key tiles, 110 units per CTA), where the
+    folded path is used; sampled rows."""
+    import numpy as np
+    import paper_2609_04910_gb300 as gs
+    from oracle import oracle_sum
+    from paper_2609_04910_gb300._binding import testing_last_fma_variant
+    from paper_2609_04910_gb300.workloads import sample_rows
+    rng = np.random.default_rng(7)
+    M, N, D = 65536, 8320, 48
+    q = rng.standard_normal((M, D)).astype(np.float16)
+    k = rng.standard_normal((N, D)).astype(np.float16)
+    v = _value_pattern(N, pattern, rng)
+    tau = 1.0 / D
+    s = gs.gauss_sum(torch.from_numpy(q).cuda(), torch.from_numpy(k).cuda(), torch.from_numpy(v).cuda(),
+                     tau, center=center)
+    gs.gauss_sum_device_status()
+    assert testing_last_fma_variant() & 8, "folded-value path not taken"
+    rows = sample_rows(M, 256)
+    ref, den = oracle_sum(q, k, v, tau, rows=rows)
+    rel = float(np.max(np.abs(s.cpu().numpy()[rows] - ref) / (den + 1e-30)))
+    assert rel <= 2e-3, f"{pattern} center={center}: max rel {rel:.3e}"
+
+
+def test_folded_values_only_for_one_fp16_channel_and_long_runs():
+    """bf16 values (range beyond 2^16), C > 1 and short runs of key tiles
+    (small problems: the extra launches would cost more than they save)
+    keep the value records."""
+    import paper_2609_04910_gb300 as gs
+    from paper_2609_04910_gb300._binding import testing_last_fma_variant
+    for n, dtype, C in ((65536, torch.bfloat16, 1), (65536, torch.float16, 2), (300, torch.float16, 1)):
+        q = torch.randn(n, 32, device="cuda").to(dtype)
+        v = torch.randn(n, C, device="cuda").to(dtype)
+        gs.gauss_sum(q, q, v, 1.0 / 32)
+        gs.gauss_sum_device_status()
+        assert not testing_last_fma_variant() & 8, (n, dtype, C)
+
+
+def test_folded_values_both_passes_in_one_batch():
+    """A batch whose problems differ in sign structure: problems whose
+    32-key groups all have values of one sign go through the first pass
+    of the fused kernel, the others through the second; together they
+    give every problem's sum (against the oracle, problem by problem)."""
+    import numpy as np
+    import paper_2609_04910_gb300 as gs
+    from oracle import oracle_sum
+    from paper_2609_04910_gb300._binding import testing_last_fma_variant
+    from paper_2609_04910_gb300.workloads import sample_rows
+    rng = np.random.default_rng(11)
+    B, M, n, D = 4, 16384, 8320, 32
+    q = rng.standard_normal((B, M, D)).astype(np.float16)
+    k = rng.standard_normal((B, n, D)).astype(np.float16)
+    v = np.stack([_value_pattern(n, pat, rng) for pat in ("halves", "random", "blocks", "range")])
+    tau = 1.0 / D
+    s = gs.gauss_sum_batched(torch.from_numpy(q).cuda(), torch.from_numpy(k).cuda(),
+                             torch.from_numpy(v).cuda(), tau)
+    gs.gauss_sum_device_status()
+    assert testing_last_fma_variant() & 8, "folded-value path not taken"
+    s = s.cpu().numpy()
+    rows = sample_rows(M, 128)
+    for b in range(B):
+        ref, den = oracle_sum(q[b], k[b], v[b], tau, rows=rows)
+        rel = float(np.max(np.abs(s[b][rows] - ref) / (den + 1e-30)))
+        assert rel <= 2e-3, f"problem {b}: max rel {rel:.3e}"

@@ -372,7 +372,8 @@ def test_keys_larger_than_l2_banded_order(M, N, D, C, dtype):
 
 # ---------------------------------------------------------------- exponent bound
 @pytest.mark.parametrize("D,C,dtype,path", [
-    (64, 1, "fp16", None),      # FMA kernel, augmented operands
+    (64, 1, "fp16", None),      # FMA kernel, augmented operands, value magnitudes folded
+    (64, 1, "bf16", None),      # FMA kernel, augmented operands, value records
     (128, 2, "fp16", None),     # FMA kernel, q^ in TMEM, norms from A and B
     (64, 8, "fp16", None),      # two-MMA kernel (P in fp16 with the 2^15 shift)
     (48, 40, "bf16", None),     # two-MMA kernel, plain operands
@@ -383,7 +384,12 @@ def test_self_pairs_never_exceed_one(D, C, dtype, path):
     for q = k the computed self-pair exponent is only rounding, which can
     be slightly positive.  With tau large enough that every other pair
     underflows to 0, s_m = Phi(x_m, x_m) for unit values: it must lie in
-    [1 - tol, 1] (the kernels clamp the exponent at 0), never above 1."""
+    [1 - tol, 1] (the kernels clamp the exponent at 0), never above 1 --
+    except with folded value magnitudes (one fp16 channel on augmented
+    operands), where the exponent also carries log2(|v| 2^-16) and cannot
+    be clamped at the value's own log: there s_m may exceed 1 by the
+    rounding of the exponent, about c |x|^2 2^-22 relative (c = tau log2 e,
+    centring off), and no more."""
     import paper_2609_04910_gb300 as gs
     w = case(300, 300, D, C, dtype, tau=200.0 / D)
     inp = generate(w)
@@ -397,7 +403,12 @@ def test_self_pairs_never_exceed_one(D, C, dtype, path):
     ones = np.ones((300, C))
     ref, den = oracle_sum(inp["q64"], inp["q64"], ones, w.tau)
     assert np.max(np.abs(ref - 1.0)) < 1e-10      # other pairs vanish in float64 too
-    assert np.all(s <= 1.0), f"max {s.max()!r}"
+    if dtype == "fp16" and C == 1 and path is None:
+        c = w.tau * np.log2(np.e)
+        bound = 4.0 * c * float(np.max(np.sum(inp["q64"] ** 2, axis=1))) * 2.0 ** -22
+        assert np.all(s <= 1.0 + bound), f"max {s.max()!r}, bound 1 + {bound:.2e}"
+    else:
+        assert np.all(s <= 1.0), f"max {s.max()!r}"
     tol = TOL[dtype]
     if path == "tensor":
         # 3xTF32: the exponent carries the tf32 split error, about
