@@ -337,6 +337,7 @@ gs_status run(Call c) {
         // Key records of the FMA kernel with augmented operands depend on the
         // values only: the mean launch writes them where it can.
         bool records_done = false;
+        bool flags_done = false;   // folded values: per-problem flags written by the operand launch
         if (mu) {
             const gs::RecordArgs rec = {c.v, c.w_f32, c.N, tp.Npad, static_cast<int>(tp.Cv),
                                         reinterpret_cast<float*>(ws + tp.off_rec), tp.vfold};
@@ -374,7 +375,9 @@ gs_status run(Call c) {
                 tp.aug ? nullptr : reinterpret_cast<float*>(ws + tp.off_A),
                 !tp.alias, c.k, c.N, tp.Npad, ws + tp.off_kh,
                 tp.aug ? nullptr : reinterpret_cast<float*>(ws + tp.off_B), static_cast<int>(c.D),
-                tp.Dp, mu, half_c, ninf, c.stream, batch, tp.vfold ? c.v : nullptr);
+                tp.Dp, mu, half_c, ninf, c.stream, batch, tp.vfold ? c.v : nullptr,
+                (tp.vfold && records_done) ? reinterpret_cast<float*>(ws + tp.off_rec) : nullptr,
+                &flags_done);
             where = tp.aug ? "augmented-operand kernel" : "centre/cast kernel";
         }
         if (e == cudaSuccess && tp.fma) {
@@ -386,7 +389,7 @@ gs_status run(Call c) {
                     c.stream, batch, tp.vfold);
                 where = "key-record kernel";
             }
-            if (e == cudaSuccess && tp.vfold) {
+            if (e == cudaSuccess && tp.vfold && !flags_done) {
                 e = gs::launch_vf_flags(reinterpret_cast<float*>(ws + tp.off_rec), tp.Npad, batch,
                                         c.stream);
                 where = "folded-value flag kernel";

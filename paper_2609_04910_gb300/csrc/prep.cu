@@ -139,13 +139,10 @@ __device__ __forceinline__ void write_sign_record(const __half* v, int64_t N, fl
     if ((kn & 31) == 0) r[kRecTile + kn / 32] = any_pos && any_neg ? 0.f : any_neg ? -65536.f : 65536.f;
 }
 
-// One block per problem: the AND over its 32-key groups of "values of one
-// sign" (group word != 0), into the word after all problems' records.
-__global__ void __launch_bounds__(256)
-vf_flags_kernel(float* __restrict__ rec, int64_t tiles, int batch) {
-    pdl_trigger();
-    pdl_wait();
-    const int b = blockIdx.x;
+// One block per problem b: the AND over its 32-key groups of "values of
+// one sign" (group word != 0), into the word after all problems' records.
+// Every thread of the block calls this.
+__device__ __forceinline__ void write_vf_flag(float* __restrict__ rec, int64_t tiles, int batch, int b) {
     const float* gw = rec + static_cast<int64_t>(b) * tiles * kRecTileFloats + kRecTile;
     bool mixed = false;
     for (int64_t i = threadIdx.x; i < tiles * (kRecTile / 32); i += blockDim.x)
@@ -154,6 +151,13 @@ vf_flags_kernel(float* __restrict__ rec, int64_t tiles, int batch) {
     if (threadIdx.x == 0)
         reinterpret_cast<unsigned*>(rec + static_cast<int64_t>(batch) * tiles * kRecTileFloats)[b] =
             any_mixed ? 0u : 1u;
+}
+
+__global__ void __launch_bounds__(256)
+vf_flags_kernel(float* __restrict__ rec, int64_t tiles, int batch) {
+    pdl_trigger();
+    pdl_wait();
+    write_vf_flag(rec, tiles, batch, blockIdx.x);
 }
 
 __global__ void sign_record_kernel(const __half* __restrict__ v, int64_t N, int64_t npad,
@@ -768,10 +772,16 @@ template <typename T, bool AUG, int G>
 __global__ void __launch_bounds__(kOperandVecThreads)
 operand_vec_kernel(const OperandJob j0, const OperandJob j1, unsigned blocks0, int D, int Dp,
                    int nt, float F, const float* __restrict__ mu, float half_c, float pad_value,
-                   float inv_c) {
+                   float inv_c, unsigned op_blocks, float* __restrict__ vf_rec, int64_t vf_tiles) {
     using PT = Pair<T>;
     pdl_trigger();
     pdl_wait();
+    if (blockIdx.x >= op_blocks) {
+        // Folded values: the per-problem flag of the sign records (written
+        // by an earlier launch of the call), one extra block per problem.
+        write_vf_flag(vf_rec, vf_tiles, static_cast<int>(gridDim.y), blockIdx.y);
+        return;
+    }
     constexpr int SLOTS = kOperandVecThreads / G;   // rows of a block
     __shared__ uint4 smean[kOperandMaxCols / 8];
     const int b = blockIdx.y;                        // problem of the batch
@@ -815,7 +825,7 @@ operand_vec_kernel(const OperandJob j0, const OperandJob j1, unsigned blocks0, i
 template <typename T, bool AUG>
 cudaError_t operand_typed(const OperandJob& j0, const OperandJob* j1, int D, int Dp, int nt,
                           float F, const float* mu, float half_c, float pad_value, cudaStream_t s,
-                          int batch, float inv_c) {
+                          int batch, float inv_c, float* vf_rec, int64_t vf_tiles, bool* flags_done) {
     const OperandJob none = {nullptr, 0, 0, nullptr, nullptr, nullptr, nullptr};
     for (const OperandJob* j : {&j0, j1}) {
         if (j && (j->rows_pad % kRowsPerBlock != 0)) return cudaErrorInvalidValue;
@@ -833,11 +843,13 @@ cudaError_t operand_typed(const OperandJob& j0, const OperandJob* j1, int D, int
         const int64_t b0 = (j0.rows_pad + per_block - 1) / per_block;
         const int64_t b1 = j1 ? (j1->rows_pad + per_block - 1) / per_block : 0;
         if (b0 + b1 == 0 || batch == 0) return cudaSuccess;
+        const unsigned op_blocks = static_cast<unsigned>(b0 + b1);
         auto go = [&](auto kern) {
-            launch_kernel(kern, dim3(static_cast<unsigned>(b0 + b1), static_cast<unsigned>(batch)),
+            launch_kernel(kern, dim3(op_blocks + (vf_rec ? 1u : 0u), static_cast<unsigned>(batch)),
                           kOperandVecThreads, 0, s, j0, j1 ? *j1 : none, static_cast<unsigned>(b0),
-                          D, Dp, nt, F, mu, half_c, pad_value, inv_c);
+                          D, Dp, nt, F, mu, half_c, pad_value, inv_c, op_blocks, vf_rec, vf_tiles);
         };
+        if (flags_done) *flags_done = vf_rec != nullptr;
         switch (G) {
             case 1: go(operand_vec_kernel<T, AUG, 1>); break;
             case 2: go(operand_vec_kernel<T, AUG, 2>); break;
@@ -1345,7 +1357,9 @@ cudaError_t launch_operands(InType t, bool aug, const void* q, int64_t M, int64_
                             void* qh, void* qh_as_key, float* nrm_q, bool with_k, const void* k,
                             int64_t N, int64_t Npad, void* kh, float* nrm_k, int D, int Dp,
                             const float* mu, float half_c, float pad_value, cudaStream_t s,
-                            int batch, const void* vw) {
+                            int batch, const void* vw, float* vf_rec, bool* flags_done) {
+    if (flags_done) *flags_done = false;
+    const int64_t vf_tiles = Npad / kRecTile;
     OperandJob jq, jk;
     if (aug) {
         // vw: folded value magnitudes on the key rows (the q job writes the
@@ -1362,13 +1376,15 @@ cudaError_t launch_operands(InType t, bool aug, const void* q, int64_t M, int64_
     const int nt = aug ? aug_norm_terms(t) : 0;
     if (t == InType::BF16) {
         return aug ? operand_typed<__nv_bfloat16, true>(jq, j1, D, Dp, nt, 1.f, mu, 0.f, 0.f, s, batch,
-                                                        inv_c)
+                                                        inv_c, vf_rec, vf_tiles, flags_done)
                    : operand_typed<__nv_bfloat16, false>(jq, j1, D, Dp, 0, 1.f, mu, half_c,
-                                                         pad_value, s, batch, inv_c);
+                                                         pad_value, s, batch, inv_c, vf_rec,
+                                                         vf_tiles, flags_done);
     }
-    return aug ? operand_typed<__half, true>(jq, j1, D, Dp, nt, 1024.f, mu, 0.f, 0.f, s, batch, inv_c)
+    return aug ? operand_typed<__half, true>(jq, j1, D, Dp, nt, 1024.f, mu, 0.f, 0.f, s, batch,
+                                             inv_c, vf_rec, vf_tiles, flags_done)
                : operand_typed<__half, false>(jq, j1, D, Dp, 0, 1.f, mu, half_c, pad_value, s,
-                                              batch, inv_c);
+                                              batch, inv_c, vf_rec, vf_tiles, flags_done);
 }
 
 cudaError_t launch_tf32_split(const float* x, int64_t rows, int64_t rows_pad, int D, int Dp,
