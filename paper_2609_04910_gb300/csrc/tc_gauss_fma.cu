@@ -280,6 +280,20 @@ tc_gauss_fma_kernel(const __grid_constant__ CUtensorMap tm_q,
     volatile int* abort_flag = &bars->abort_flag;
 
     pdl_trigger();
+    if (VF == 2) {
+        // The second folded-value pass often has nothing to do (every problem
+        // of the call went to the first): a CTA none of whose segments is of
+        // this pass leaves before allocating tensor memory.  (The flags come
+        // from an earlier launch, hence the wait first.)
+        pdl_wait();
+        const int ub = static_cast<int>(blockIdx.x) * p.unit_len;
+        const int ue = p.units < ub + p.unit_len ? p.units : ub + p.unit_len;
+        int u = ub, run = 0;
+        Segment sg;
+        bool any = false;
+        while (!any && next_segment<TRI>(p, ue, u, run, sg)) any = vf_takes<VF>(p, sg.tile_m);
+        if (!any) return;   // uniform over the block: every thread reads the same flags
+    }
     if (tid == 0) bars->abort_flag = 0;
     if (warp == CTRL_WARP0) {
         tmem_alloc(&bars->tmem_base, TMEM_COLS);
