@@ -232,8 +232,13 @@ gs_status plan(const Call& c, int sms, bool* tensor, gs::TcPlan* tp, gs::SimtPla
         // for short segments (small problems), where the flag kernel and the
         // second pass of the fused kernel cost more than they save (B = 256
         // problems of 1024 points: 0.135 -> 0.144 ms per call).
+        // The exponent scale c folds into the query rows with them (rn(c q^)
+        // must stay a normal fp16 number for points of any spread: c <= 1/2,
+        // and not far below it: c >= 2^-14).
+        const double cx = c.tau * 1.4426950408889634;
         tp->vfold = tp->fma && tp->aug && !tp->tf && tp->Cv == 1 && c.dtype == GS_FP16 &&
-                    !c.w_f32 && tp->exp2_fma == 0 && c.C == 1 && !tp->overlap;
+                    !c.w_f32 && tp->exp2_fma == 0 && c.C == 1 && !tp->overlap &&
+                    cx <= 0.5 && cx >= 1.0 / 16384.0;
         *bytes = tp->total;
     } else {
         if (c.opt.exp2_fma > 0)
@@ -376,6 +381,7 @@ gs_status run(Call c) {
                 !tp.alias, c.k, c.N, tp.Npad, ws + tp.off_kh,
                 tp.aug ? nullptr : reinterpret_cast<float*>(ws + tp.off_B), static_cast<int>(c.D),
                 tp.Dp, mu, half_c, ninf, c.stream, batch, tp.vfold ? c.v : nullptr,
+                tp.vfold ? cexp : 0.f,
                 (tp.vfold && records_done) ? reinterpret_cast<float*>(ws + tp.off_rec) : nullptr,
                 &flags_done);
             where = tp.aug ? "augmented-operand kernel" : "centre/cast kernel";

@@ -158,7 +158,8 @@ struct RecordArgs {
 cudaError_t launch_mean(InType t, const void* q, const void* k, int64_t M, int64_t N, int D,
                         int blocks, float* partial, float* mu, cudaStream_t s, int batch = 1,
                         const RecordArgs* rec = nullptr, bool* rec_done = nullptr);
-// (vw: fp16 values whose magnitudes fold into the key rows' norm terms;
+// (cf > 0 with vw: the exponent scale c folds into the query rows and the
+// magnitudes of the fp16 values vw into the key rows' norm terms;
 // vf_rec: sign records already written, whose per-problem flags the launch
 // then also computes where it can, *flags_done saying whether it did.)
 // Centred, rounded MMA operands of q (M rows, padded to Mpad) and, with
@@ -172,8 +173,8 @@ cudaError_t launch_operands(InType t, bool aug, const void* q, int64_t M, int64_
                             void* qh, void* qh_as_key, float* nrm_q, bool with_k, const void* k,
                             int64_t N, int64_t Npad, void* kh, float* nrm_k, int D, int Dp,
                             const float* mu, float half_c, float pad_value, cudaStream_t s,
-                            int batch = 1, const void* vw = nullptr, float* vf_rec = nullptr,
-                            bool* flags_done = nullptr);
+                            int batch = 1, const void* vw = nullptr, float cf = 0.f,
+                            float* vf_rec = nullptr, bool* flags_done = nullptr);
 // Transposed fp16 value operand of the two-MMA kernel for the channels
 // ch0 .. ch0 + Cc - 1 (Cp >= Cc rows of Npad keys), with per-channel
 // power-of-two scales.  Forward: channel ch of key n is w[n, ch] (w has the

@@ -375,25 +375,25 @@ mean_final_kernel(const float* __restrict__ partial, int G, int D, int64_t items
 // well); padded query rows are zero.  `out_q` and/or `out_k` may be given
 // (both for q = k).
 //
-// Folded value magnitudes (vw given, one fp16 value per key): the key-side
-// term becomes b + log2(|v_n| 2^-16) / c, so that 2^(c S) = Phi |v_n| 2^-16;
-// the FMA kernel then needs only the signs of the values (see
-// write_sign_record).  |v_n| < 2^16 for every finite fp16 value, so the
-// exponent stays <= 0.  Keys with v_n = 0, and padded keys, get -256 / c
-// (at least -30000 for padded keys): their 2^(c S) flushes to zero, so they
-// may sit in a group of either sign.  inv_c = 1 / c.
+// Folded exponent scale and value magnitudes (cf = c > 0, one fp16 value
+// per key in vw): the query rows hold u = rn(c q^), with a = -||u||^2/(2c),
+// and the key rows b = -c ||k^||^2 / 2 + log2(|v_n| 2^-16), so that the MMA
+// yields S = u.k^ + a + b = -(1/(2c)) ||u - c k^||^2 + log2(|v_n| 2^-16):
+// the exponent of Phi |v_n| 2^-16 itself, at the query point u / c (within
+// 2^-12 of q^ per coordinate), and never above log2(|v_n| 2^-16) in exact
+// arithmetic.  The FMA kernel then needs no multiply by c and only the
+// signs of the values (see write_sign_record).  |v_n| < 2^16 for every
+// finite fp16 value.  Keys with v_n = 0 get -256: their 2^S flushes to
+// zero, so they may sit in a group of either sign (padded keys have
+// -30000 already).
 constexpr float kZeroWeightLog2 = -256.f;
 
-__device__ __forceinline__ float log_weight(const __half* vw, float inv_c) {
+__device__ __forceinline__ float log_weight(const __half* vw) {
     if (!vw) return 0.f;
     const float a = fabsf(__half2float(*vw));
-    return a > 0.f ? log2f(a * (1.f / 65536.f)) * inv_c : kZeroWeightLog2 * inv_c;
+    return a > 0.f ? log2f(a * (1.f / 65536.f)) : kZeroWeightLog2;
 }
 
-// Norm term of a padded key row (b_0 of the split, times F).
-__device__ __forceinline__ float pad_key_term(bool fold, float inv_c) {
-    return fold ? fminf(-30000.f, kZeroWeightLog2 * inv_c) : -30000.f;
-}
 constexpr int kRowsPerBlock = 32;
 constexpr int kOperandThreads = 128;
 constexpr int kOperandMaxCols = 256;
@@ -403,7 +403,7 @@ __global__ void __launch_bounds__(kOperandThreads)
 operand_kernel(const T* __restrict__ x, int64_t rows, int64_t rows_pad, int D, int Dp, int nt, float F,
                const float* __restrict__ mu, float half_c, float pad_value,
                T* __restrict__ out_q, T* __restrict__ out_k, float* __restrict__ nrm,
-               const __half* __restrict__ vw, float inv_c) {
+               const __half* __restrict__ vw, float cf) {
     pdl_trigger();
     pdl_wait();
     constexpr int R = kRowsPerBlock;
@@ -454,18 +454,28 @@ operand_kernel(const T* __restrict__ x, int64_t rows, int64_t rows_pad, int D, i
         const bool valid = row < rin;
         T* oq = sq + row * Dp;
         T* ok = sk + row * Dp;
-        float acc = 0.f;
+        float acc = 0.f, accu = 0.f;
+        const bool fold = AUG && cf > 0.f;
         const int dend = AUG ? D : Dp;
         for (int d = lane; d < dend; d += 32) {
             const float val = (valid && d < D) ? to_f(s_in[row * D + d]) - s_mu[d] : 0.f;
             const T h = from_f<T>(val);
-            if (wq) oq[d] = h;
-            if (wk) ok[d] = h;
             const float hf = to_f(h);
+            if (fold) {
+                const T hs = from_f<T>(cf * hf);   // folded scale: the query row holds rn(c x^)
+                if (wq) oq[d] = hs;
+                accu = fmaf(to_f(hs), to_f(hs), accu);
+            } else if (wq) {
+                oq[d] = h;
+            }
+            if (wk) ok[d] = h;
             acc = fmaf(hf, hf, acc);
         }
 #pragma unroll
-        for (int o = 16; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
+        for (int o = 16; o > 0; o >>= 1) {
+            acc += __shfl_xor_sync(0xffffffffu, acc, o);
+            accu += __shfl_xor_sync(0xffffffffu, accu, o);
+        }
         if (!AUG) {
             if (lane == 0) nrm[r0 + row] = valid ? -half_c * acc : pad_value;
             continue;
@@ -488,13 +498,15 @@ operand_kernel(const T* __restrict__ x, int64_t rows, int64_t rows_pad, int D, i
             };
             T t = zero, tk = zero, one = zero;
             if (valid) {
-                t = split_term(-0.5f * acc);
-                const float lw = log_weight(vw ? vw + r0 + row : nullptr, inv_c);
-                tk = lw != 0.f ? split_term(-0.5f * acc + lw) : t;
+                if (fold) {
+                    t = split_term(-0.5f * accu / cf);
+                    tk = split_term(-0.5f * cf * acc + log_weight(vw ? vw + r0 + row : nullptr));
+                } else {
+                    t = tk = split_term(-0.5f * acc);
+                }
                 one = from_f<T>(lane == 0 ? F : 1.f);
             } else if (lane == 0) {
-                t = from_f<T>(-30000.f / F);
-                tk = from_f<T>(pad_key_term(vw != nullptr, inv_c) / F);
+                t = tk = from_f<T>(-30000.f / F);
             }
             if (wq) {
                 oq[D + lane] = valid ? one : zero;
@@ -650,40 +662,54 @@ __device__ __forceinline__ float operand_row(const uint4 (&in)[kOperandVecs],
                                              bool in_pad, bool valid, int D, int Dp, int nt,
                                              float F, float half_c, float pad_value,
                                              T* __restrict__ out_q, T* __restrict__ out_k,
-                                             bool fold, const __half* vw, float inv_c) {
+                                             float cf, const __half* vw) {
     using PT = Pair<T>;
     const int V = D / 8;
-    float acc = 0.f;
+    const bool fold = AUG && cf > 0.f;
+    float acc = 0.f, accu = 0.f;
     if (in_pad) {
-        uint64_t acc2 = 0ull;
+        uint64_t acc2 = 0ull, accu2 = 0ull;
 #pragma unroll
         for (int e = 0; e < kOperandVecs; ++e) {
             const int v = vi + G * e;
             if (v >= V) break;
-            uint4 u = make_uint4(0u, 0u, 0u, 0u);
+            uint4 u = make_uint4(0u, 0u, 0u, 0u), us = u;
             if (valid) {
                 const uint4 m2 = smean[v];
                 const typename PT::P* x2 = reinterpret_cast<const typename PT::P*>(&in[e]);
                 const typename PT::P* mm = reinterpret_cast<const typename PT::P*>(&m2);
-                typename PT::P h[4];
+                typename PT::P h[4], hs[4];
 #pragma unroll
                 for (int k = 0; k < 4; ++k) {
                     h[k] = PT::sub(x2[k], mm[k]);
                     const float2 f = PT::to_f2(h[k]);
                     const uint64_t f2 = f32x2_pack(f.x, f.y);
                     acc2 = f32x2_fma(f2, f2, acc2);
+                    if (fold) {
+                        // Folded scale: the query row holds rn(c x^).
+                        hs[k] = PT::from_f2(cf * f.x, cf * f.y);
+                        const float2 g = PT::to_f2(hs[k]);
+                        const uint64_t g2 = f32x2_pack(g.x, g.y);
+                        accu2 = f32x2_fma(g2, g2, accu2);
+                    }
                 }
                 u = *reinterpret_cast<const uint4*>(h);
+                us = fold ? *reinterpret_cast<const uint4*>(hs) : u;
             }
-            if (out_q) *reinterpret_cast<uint4*>(out_q + 8 * v) = u;
+            if (out_q) *reinterpret_cast<uint4*>(out_q + 8 * v) = fold ? us : u;
             if (out_k) *reinterpret_cast<uint4*>(out_k + 8 * v) = u;
         }
         float lo, hi;
         f32x2_unpack(acc2, lo, hi);
         acc = lo + hi;
+        f32x2_unpack(accu2, lo, hi);
+        accu = lo + hi;
     }
 #pragma unroll
-    for (int o = G / 2; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o, G);
+    for (int o = G / 2; o > 0; o >>= 1) {
+        acc += __shfl_xor_sync(0xffffffffu, acc, o, G);
+        if (fold) accu += __shfl_xor_sync(0xffffffffu, accu, o, G);
+    }
     const float nrm = valid ? -half_c * acc : pad_value;
     if (!in_pad || vi != 0) return nrm;
     if (!AUG) {
@@ -708,15 +734,19 @@ __device__ __forceinline__ float operand_row(const uint4 (&in)[kOperandVecs],
         z2 = nt > 2 ? to_bits(a2) : 0;
     };
     if (valid) {
-        split(-0.5f * acc, t0, t1, t2);
-        // Key side: the log weight of the folded value magnitude, if any.
-        const float lw = fold ? log_weight(vw, inv_c) : 0.f;
-        if (lw != 0.f) split(-0.5f * acc + lw, k0, k1, k2);
-        else { k0 = t0; k1 = t1; k2 = t2; }
+        if (fold) {
+            // Folded: a = -||u||^2 / (2c) from the rounded scaled row, and
+            // b = -c ||k^||^2 / 2 + log2(|v| 2^-16) (see log_weight).
+            split(-0.5f * accu / cf, t0, t1, t2);
+            split(-0.5f * cf * acc + log_weight(vw), k0, k1, k2);
+        } else {
+            split(-0.5f * acc, t0, t1, t2);
+            k0 = t0; k1 = t1; k2 = t2;
+        }
     }
     const unsigned short oneF = valid ? to_bits(from_f<T>(F)) : 0;
     const unsigned short one1 = valid ? to_bits(from_f<T>(1.f)) : 0;
-    const unsigned short pad_b = valid ? k0 : to_bits(from_f<T>(pad_key_term(fold, inv_c) / F));
+    const unsigned short pad_b = valid ? k0 : to_bits(from_f<T>(-30000.f / F));
     auto term = [&](int i) { return i == 0 ? pad_b : i == 1 ? k1 : k2; };
     auto qterm = [&](int i) { return i == 0 ? t0 : i == 1 ? t1 : t2; };
     auto partner = [&](int i) { return i == 0 ? oneF : one1; };
@@ -772,7 +802,7 @@ template <typename T, bool AUG, int G>
 __global__ void __launch_bounds__(kOperandVecThreads)
 operand_vec_kernel(const OperandJob j0, const OperandJob j1, unsigned blocks0, int D, int Dp,
                    int nt, float F, const float* __restrict__ mu, float half_c, float pad_value,
-                   float inv_c, unsigned op_blocks, float* __restrict__ vf_rec, int64_t vf_tiles) {
+                   float cf, unsigned op_blocks, float* __restrict__ vf_rec, int64_t vf_tiles) {
     using PT = Pair<T>;
     pdl_trigger();
     pdl_wait();
@@ -811,21 +841,20 @@ operand_vec_kernel(const OperandJob j0, const OperandJob j1, unsigned blocks0, i
     const bool wk = AUG && j.out_k != nullptr;
     const bool in_pad = i < rows_pad;
     const int64_t row = static_cast<int64_t>(b) * rows_pad + i;   // batch-stacked output row
-    const bool fold = wk && j.vw;
-    const __half* vw = (fold && i < rows)
+    const __half* vw = (wk && j.vw && i < rows)
                            ? static_cast<const __half*>(j.vw) + static_cast<int64_t>(b) * rows + i
                            : nullptr;
     const float n = operand_row<T, AUG, G>(
         in, smean, vi, in_pad, i < rows, D, Dp, nt, F, half_c, pad_value,
         wq ? static_cast<T*>(j.out_q) + row * Dp : nullptr,
-        wk ? static_cast<T*>(j.out_k) + row * Dp : nullptr, fold, vw, inv_c);
+        wk ? static_cast<T*>(j.out_k) + row * Dp : nullptr, cf, vw);
     if (!AUG && in_pad && vi == 0) j.nrm[row] = n;
 }
 
 template <typename T, bool AUG>
 cudaError_t operand_typed(const OperandJob& j0, const OperandJob* j1, int D, int Dp, int nt,
                           float F, const float* mu, float half_c, float pad_value, cudaStream_t s,
-                          int batch, float inv_c, float* vf_rec, int64_t vf_tiles, bool* flags_done) {
+                          int batch, float cf, float* vf_rec, int64_t vf_tiles, bool* flags_done) {
     const OperandJob none = {nullptr, 0, 0, nullptr, nullptr, nullptr, nullptr};
     for (const OperandJob* j : {&j0, j1}) {
         if (j && (j->rows_pad % kRowsPerBlock != 0)) return cudaErrorInvalidValue;
@@ -847,7 +876,7 @@ cudaError_t operand_typed(const OperandJob& j0, const OperandJob* j1, int D, int
         auto go = [&](auto kern) {
             launch_kernel(kern, dim3(op_blocks + (vf_rec ? 1u : 0u), static_cast<unsigned>(batch)),
                           kOperandVecThreads, 0, s, j0, j1 ? *j1 : none, static_cast<unsigned>(b0),
-                          D, Dp, nt, F, mu, half_c, pad_value, inv_c, op_blocks, vf_rec, vf_tiles);
+                          D, Dp, nt, F, mu, half_c, pad_value, cf, op_blocks, vf_rec, vf_tiles);
         };
         if (flags_done) *flags_done = vf_rec != nullptr;
         switch (G) {
@@ -869,7 +898,7 @@ cudaError_t operand_typed(const OperandJob& j0, const OperandJob* j1, int D, int
         launch_kernel(operand_kernel<T, AUG>, dim3(static_cast<unsigned>(blocks), batch),
                       kOperandThreads, smem, s, static_cast<const T*>(j->x), j->rows, j->rows_pad,
                       D, Dp, nt, F, mu, half_c, pad_value, static_cast<T*>(j->out_q),
-                      static_cast<T*>(j->out_k), j->nrm, static_cast<const __half*>(j->vw), inv_c);
+                      static_cast<T*>(j->out_k), j->nrm, static_cast<const __half*>(j->vw), cf);
         note_launches(1);
         const cudaError_t e = cudaGetLastError();
         if (e != cudaSuccess) return e;
@@ -1357,7 +1386,7 @@ cudaError_t launch_operands(InType t, bool aug, const void* q, int64_t M, int64_
                             void* qh, void* qh_as_key, float* nrm_q, bool with_k, const void* k,
                             int64_t N, int64_t Npad, void* kh, float* nrm_k, int D, int Dp,
                             const float* mu, float half_c, float pad_value, cudaStream_t s,
-                            int batch, const void* vw, float* vf_rec, bool* flags_done) {
+                            int batch, const void* vw, float cf, float* vf_rec, bool* flags_done) {
     if (flags_done) *flags_done = false;
     const int64_t vf_tiles = Npad / kRecTile;
     OperandJob jq, jk;
@@ -1370,21 +1399,21 @@ cudaError_t launch_operands(InType t, bool aug, const void* q, int64_t M, int64_
         jq = {q, M, Mpad, qh, nullptr, nrm_q, nullptr};
         jk = {k, N, Npad, kh, nullptr, nrm_k, nullptr};
     }
-    const float inv_c = half_c > 0.f ? 0.5f / half_c : 0.f;
+    if (!aug) cf = 0.f;
     // (k itself may be null: an empty array when D = 0.)
     const OperandJob* j1 = with_k ? &jk : nullptr;
     const int nt = aug ? aug_norm_terms(t) : 0;
     if (t == InType::BF16) {
         return aug ? operand_typed<__nv_bfloat16, true>(jq, j1, D, Dp, nt, 1.f, mu, 0.f, 0.f, s, batch,
-                                                        inv_c, vf_rec, vf_tiles, flags_done)
+                                                        cf, vf_rec, vf_tiles, flags_done)
                    : operand_typed<__nv_bfloat16, false>(jq, j1, D, Dp, 0, 1.f, mu, half_c,
-                                                         pad_value, s, batch, inv_c, vf_rec,
+                                                         pad_value, s, batch, cf, vf_rec,
                                                          vf_tiles, flags_done);
     }
     return aug ? operand_typed<__half, true>(jq, j1, D, Dp, nt, 1024.f, mu, 0.f, 0.f, s, batch,
-                                             inv_c, vf_rec, vf_tiles, flags_done)
+                                             cf, vf_rec, vf_tiles, flags_done)
                : operand_typed<__half, false>(jq, j1, D, Dp, 0, 1.f, mu, half_c, pad_value, s,
-                                              batch, inv_c, vf_rec, vf_tiles, flags_done);
+                                              batch, cf, vf_rec, vf_tiles, flags_done);
 }
 
 cudaError_t launch_tf32_split(const float* x, int64_t rows, int64_t rows_pad, int D, int Dp,

@@ -53,13 +53,14 @@
 //                their MMAs.  Warp 16 also allocates TMEM and loads q^.
 // Key records: for each pair of keys (2t, 2t + 1) the floats
 //   [B_2t, B_2t+1,] v_2t[0], v_2t+1[0], ..., v_2t[C-1], v_2t+1[C-1]
-// (B only without augmented operands).  With folded value magnitudes (VF:
-// C = 1, fp16 values, augmented operands whose key norm terms carry
-// log2(|v_n| 2^-16) / c, so that 2^(c S) = Phi |v_n| 2^-16), the records of
-// a key tile are the signs s_n = sign(v_n) 2^16 in key order and one word
-// per 32-key column group, +-2^16 where all the group's values share a
-// sign, else 0: such a group's exponent loop then reads no record at all
-// (the broadcast record load per key pair was a fifth of its MIO work).
+// (B only without augmented operands).  With folded values (VF: C = 1,
+// fp16 values, augmented operands whose query rows carry the exponent
+// scale c and whose key norm terms carry log2(|v_n| 2^-16), so that
+// 2^S = Phi |v_n| 2^-16 with no multiply), the records of a key tile are
+// the signs s_n = sign(v_n) 2^16 in key order and one word per 32-key
+// column group, +-2^16 where all the group's values share a sign, else 0:
+// such a group's exponent loop then reads no record at all (the broadcast
+// record load per key pair was a fifth of its MIO work).
 #include <cuda.h>
 #include <cuda_runtime.h>
 
@@ -704,8 +705,8 @@ tc_gauss_fma_kernel(const __grid_constant__ CUtensorMap tm_q,
                             float x0, x1, y0, y1;
                             const uint64_t sx = f32x2_pack(__uint_as_float(r0[2 * t]), __uint_as_float(r0[2 * t + 1]));
                             const uint64_t sy = f32x2_pack(__uint_as_float(r1[2 * t]), __uint_as_float(r1[2 * t + 1]));
-                            f32x2_unpack(TRI ? f32x2_fma(sx, c2, w2) : f32x2_mul(sx, c2), x0, x1);
-                            f32x2_unpack(TRI ? f32x2_fma(sy, c2, w2) : f32x2_mul(sy, c2), y0, y1);
+                            f32x2_unpack(TRI ? f32x2_add(sx, w2) : sx, x0, x1);   // the operands carry c
+                            f32x2_unpack(TRI ? f32x2_add(sy, w2) : sy, y0, y1);
                             const uint64_t px = f32x2_pack(TRI ? ex2_approx(x0) : ex2_nonpos(x0),
                                                            TRI ? ex2_approx(x1) : ex2_nonpos(x1));
                             const uint64_t py = f32x2_pack(TRI ? ex2_approx(y0) : ex2_nonpos(y0),
@@ -726,14 +727,18 @@ tc_gauss_fma_kernel(const __grid_constant__ CUtensorMap tm_q,
                             } else {
                                 float x0, x1;
                                 const uint64_t sx = f32x2_pack(__uint_as_float(r0[2 * t]), __uint_as_float(r0[2 * t + 1]));
-                                f32x2_unpack(TRI ? f32x2_fma(sx, c2, w2) : f32x2_mul(sx, c2), x0, x1);
+                                f32x2_unpack(VF != 0 ? (TRI ? f32x2_add(sx, w2) : sx)
+                                                      : (TRI ? f32x2_fma(sx, c2, w2) : f32x2_mul(sx, c2)),
+                                             x0, x1);
                                 px = f32x2_pack(TRI ? ex2_approx(x0) : ex2_nonpos(x0),
                                                 TRI ? ex2_approx(x1) : ex2_nonpos(x1));
                             }
                             {
                                 float y0, y1;
                                 const uint64_t sy = f32x2_pack(__uint_as_float(r1[2 * t]), __uint_as_float(r1[2 * t + 1]));
-                                f32x2_unpack(TRI ? f32x2_fma(sy, c2, w2) : f32x2_mul(sy, c2), y0, y1);
+                                f32x2_unpack(VF != 0 ? (TRI ? f32x2_add(sy, w2) : sy)
+                                                      : (TRI ? f32x2_fma(sy, c2, w2) : f32x2_mul(sy, c2)),
+                                             y0, y1);
                                 py = f32x2_pack(TRI ? ex2_approx(y0) : ex2_nonpos(y0),
                                                 TRI ? ex2_approx(y1) : ex2_nonpos(y1));
                             }
