@@ -39,7 +39,9 @@ gs_status gauss_sum_testing_request_stall(void* stream);
  * Bit flags describing the fused FMA kernel (C <= 4 forward) that the last
  * call of this process launched: bit 0 = overlapped segment transitions
  * (short runs of key tiles per pair of query tiles), bit 1 = banded key
- * order, bit 2 = q^ in TMEM; -1 before the first such launch.  Lets the
+ * order, bit 2 = q^ in TMEM, bit 3 = value magnitudes folded into the key
+ * operands (two passes), bit 4 = exponent scale folded into the query
+ * operands; -1 before the first such launch.  Lets the
  * parity tests check that each side of a planning switch is exercised.
  */
 int gauss_sum_testing_last_fma_variant(void);

@@ -236,9 +236,9 @@ gs_status plan(const Call& c, int sms, bool* tensor, gs::TcPlan* tp, gs::SimtPla
         // must stay a normal fp16 number for points of any spread: c <= 1/2,
         // and not far below it: c >= 2^-14).
         const double cx = c.tau * 1.4426950408889634;
-        tp->vfold = tp->fma && tp->aug && !tp->tf && tp->Cv == 1 && c.dtype == GS_FP16 &&
-                    !c.w_f32 && tp->exp2_fma == 0 && c.C == 1 && !tp->overlap &&
+        tp->cfold = tp->fma && tp->aug && !tp->tf && c.dtype == GS_FP16 && tp->exp2_fma == 0 &&
                     cx <= 0.5 && cx >= 1.0 / 16384.0;
+        tp->vfold = tp->cfold && tp->Cv == 1 && !c.w_f32 && c.C == 1 && !tp->overlap;
         *bytes = tp->total;
     } else {
         if (c.opt.exp2_fma > 0)
@@ -381,7 +381,7 @@ gs_status run(Call c) {
                 !tp.alias, c.k, c.N, tp.Npad, ws + tp.off_kh,
                 tp.aug ? nullptr : reinterpret_cast<float*>(ws + tp.off_B), static_cast<int>(c.D),
                 tp.Dp, mu, half_c, ninf, c.stream, batch, tp.vfold ? c.v : nullptr,
-                tp.vfold ? cexp : 0.f,
+                (tp.vfold || tp.cfold) ? cexp : 0.f,
                 (tp.vfold && records_done) ? reinterpret_cast<float*>(ws + tp.off_rec) : nullptr,
                 &flags_done);
             where = tp.aug ? "augmented-operand kernel" : "centre/cast kernel";

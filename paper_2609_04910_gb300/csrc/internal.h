@@ -107,6 +107,10 @@ struct TcPlan {
     // magnitudes are folded into the key operands' norm terms
     // (log2(|v| 2^-16) / c) and the key records hold only signs (VF).
     bool vfold;
+    // FMA kernel with augmented fp16 operands: the exponent scale c is folded
+    // into the query rows (rn(c q^)), so the exponent loop has no multiply;
+    // implied by vfold.
+    bool cfold;
     // Problems of a batch handled by one launch (the FMA kernel stacks them:
     // q^ batch x Mpad rows, k^ batch x Npad rows); 1 for the other paths.
     int64_t batch;

@@ -223,7 +223,7 @@ __device__ __forceinline__ bool next_segment(const FmaParams& p, int u_end, int&
 // (the exponent loop reads no records), pass VF = 2 the others.
 template <int VF>
 __device__ __forceinline__ bool vf_takes(const FmaParams& p, int tile_m) {
-    if (VF == 0) return true;
+    if (VF == 0 || VF == 3) return true;
     const int problem = tile_m / p.pairs_per_batch;
     const int batch = p.pairs_total / p.pairs_per_batch;
     const unsigned* flags = reinterpret_cast<const unsigned*>(
@@ -262,7 +262,9 @@ tc_gauss_fma_kernel(const __grid_constant__ CUtensorMap tm_q,
     // TF (3xTF32): q^ in shared memory, norm terms from A and the records.
     static_assert(!TF || (QSM && !AUG), "3xTF32 runs with q^ in shared memory");
     static_assert(!OVL || QSM, "overlapped segments keep q^ in shared memory");
-    static_assert(VF == 0 || (C == 1 && AUG && SOFT == 0), "folded values: C = 1, augmented operands");
+    static_assert(VF == 0 || (AUG && SOFT == 0 && !TF), "folded operands: augmented fp16 rows");
+    static_assert(VF != 1 || C == 1, "folded values: one channel");
+    static_assert(VF != 2 || C == 1, "folded values: one channel");
     static_assert(SOFT == 0 || (AUG && !TRI), "FMA-pipe exponentials: augmented operands");
     constexpr int kSoftMask = soft_mask(SOFT);
     constexpr int REC_PAIR = (AUG ? 0 : 2) + 2 * C;   // floats per key pair
@@ -418,7 +420,7 @@ tc_gauss_fma_kernel(const __grid_constant__ CUtensorMap tm_q,
                         tma_load_2d(kh_smem(k) + kb * (BN * 128), &tm_k, &bars->kv_full[k],
                                     kb * p.kb_elems, n0);
                     bulk_load(const_cast<float*>(rec_smem(k)),
-                              p.rec + (VF != 0 ? static_cast<int64_t>(n0 / BN) * (BN + BN / 32)
+                              p.rec + ((VF == 1 || VF == 2) ? static_cast<int64_t>(n0 / BN) * (BN + BN / 32)
                                           : static_cast<int64_t>(n0 / 2) * REC_PAIR),
                               p.rec_bytes, &bars->kv_full[k]);
                 };
@@ -907,8 +909,8 @@ cudaError_t launch_typed(const TcPlan& pl, InType t, float c, char* ws, unsigned
     p.stages = pl.stages;
     p.q_bytes = static_cast<uint32_t>(q_bytes_for(p.nkb, QSM));
     p.kh_bytes = static_cast<uint32_t>(p.nkb * BN * 128);
-    p.rec_bytes = static_cast<uint32_t>(rec_bytes_for(C, AUG, VF != 0));
-    p.stage_bytes = static_cast<uint32_t>(stage_bytes_for(p.nkb, C, AUG, VF != 0));
+    p.rec_bytes = static_cast<uint32_t>(rec_bytes_for(C, AUG, VF == 1 || VF == 2));
+    p.stage_bytes = static_cast<uint32_t>(stage_bytes_for(p.nkb, C, AUG, VF == 1 || VF == 2));
     p.red_offset = p.q_bytes + static_cast<uint32_t>(pl.stages * p.stage_bytes);
     p.c = c;
     const uint32_t hb = t == InType::BF16 ? 1u : 0u;
@@ -927,24 +929,23 @@ template <int C>
 cudaError_t launch_c(const TcPlan& pl, InType t, float c, char* ws, unsigned* status,
                      cudaStream_t s, const char** why, int vf_pass) {
     if (pl.tf) return launch_typed<C, false, true, true>(pl, t, c, ws, status, s, why);
+    // Folded operands (template parameter VF): 1 / 2 = folded values, the
+    // pass of the problems whose groups all share a sign / of the others;
+    // 3 = only the exponent scale folded, value records as usual.
+    const int vf = pl.vfold ? vf_pass : pl.cfold ? 3 : 0;
     if constexpr (C == 1 && kAugQsm) {
-        // Folded values: pass 1 (problems whose groups are all of one sign)
-        // or pass 2 (the others).
-        if (pl.tri && pl.aug && vf_pass == 1)
-            return launch_typed<1, true, true, false, true, 0, false, 1>(pl, t, c, ws, status, s, why);
-        if (pl.tri && pl.aug && vf_pass == 2)
-            return launch_typed<1, true, true, false, true, 0, false, 2>(pl, t, c, ws, status, s, why);
-        if (pl.tri && pl.aug) return launch_typed<1, true, true, false, true>(pl, t, c, ws, status, s, why);
-        if (pl.aug && vf_pass == 1) {
-            if (pl.overlap)
-                return launch_typed<1, true, true, false, false, 0, true, 1>(pl, t, c, ws, status, s, why);
+        if (pl.tri && pl.aug) {
+            switch (vf) {
+                case 1: return launch_typed<1, true, true, false, true, 0, false, 1>(pl, t, c, ws, status, s, why);
+                case 2: return launch_typed<1, true, true, false, true, 0, false, 2>(pl, t, c, ws, status, s, why);
+                case 3: return launch_typed<1, true, true, false, true, 0, false, 3>(pl, t, c, ws, status, s, why);
+                default: return launch_typed<1, true, true, false, true>(pl, t, c, ws, status, s, why);
+            }
+        }
+        if (pl.aug && vf == 1)
             return launch_typed<1, true, true, false, false, 0, false, 1>(pl, t, c, ws, status, s, why);
-        }
-        if (pl.aug && vf_pass == 2) {
-            if (pl.overlap)
-                return launch_typed<1, true, true, false, false, 0, true, 2>(pl, t, c, ws, status, s, why);
+        if (pl.aug && vf == 2)
             return launch_typed<1, true, true, false, false, 0, false, 2>(pl, t, c, ws, status, s, why);
-        }
         if (pl.aug && pl.exp2_fma > 0) {
             switch (pl.exp2_fma) {
                 case 1: return launch_typed<1, true, true, false, false, 1>(pl, t, c, ws, status, s, why);
@@ -954,8 +955,12 @@ cudaError_t launch_c(const TcPlan& pl, InType t, float c, char* ws, unsigned* st
             }
         }
     }
-    if (pl.aug && kAugQsm && pl.overlap)
+    if (pl.aug && kAugQsm && pl.overlap) {
+        if (vf == 3) return launch_typed<C, true, true, false, false, 0, true, 3>(pl, t, c, ws, status, s, why);
         return launch_typed<C, true, true, false, false, 0, true>(pl, t, c, ws, status, s, why);
+    }
+    if (pl.aug && vf == 3)
+        return launch_typed<C, true, kAugQsm, false, false, 0, false, 3>(pl, t, c, ws, status, s, why);
     if (pl.aug) return launch_typed<C, true, kAugQsm, false>(pl, t, c, ws, status, s, why);
     return launch_typed<C, false, false, false>(pl, t, c, ws, status, s, why);
 }
@@ -995,7 +1000,7 @@ cudaError_t launch_tc_fma(const TcPlan& p, InType t, float c, char* ws, unsigned
     const bool qsm = p.tf || (p.aug && kAugQsm);
     note_fma_variant((p.aug && kAugQsm && p.overlap && !p.tri && p.exp2_fma == 0 ? 1 : 0) |
                      (p.band_len > 0 ? 2 : 0) | (qsm ? 0 : 4) |
-                     (p.vfold && p.aug && kAugQsm && p.Cv == 1 && p.exp2_fma == 0 ? 8 : 0));
+                     (p.vfold ? 8 : 0) | (p.cfold || p.vfold ? 16 : 0));
     switch (p.Cv) {
         case 1: return launch_c<1>(p, t, c, ws, status, s, why, vf_pass);
         case 2: return launch_c<2>(p, t, c, ws, status, s, why, vf_pass);

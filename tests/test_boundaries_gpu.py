@@ -204,3 +204,18 @@ def test_folded_values_both_passes_in_one_batch():
         ref, den = oracle_sum(q[b], k[b], v[b], tau, rows=rows)
         rel = float(np.max(np.abs(s[b][rows] - ref) / (den + 1e-30)))
         assert rel <= 2e-3, f"problem {b}: max rel {rel:.3e}"
+
+
+@pytest.mark.parametrize("dtype,C,tau,folded", [
+    ("fp16", 3, 1.0 / 40, True),     # exponent scale folded into the query rows
+    ("fp16", 1, 1.0 / 40, True),     # small problem: scale folded, value records kept
+    ("fp16", 2, 0.4, False),         # c = tau log2 e > 1/2: rn(c q^) could overflow
+    ("bf16", 2, 1.0 / 40, False),    # bf16 rows keep the multiply
+])
+def test_folded_exponent_scale_switch(dtype, C, tau, folded):
+    """fp16 augmented operands of the FMA kernel carry the exponent scale c
+    in the query rows (rn(c q^), norm term -||rn(c q^)||^2 / (2c)) when
+    2^-14 <= c <= 1/2; each side against the oracle."""
+    from paper_2609_04910_gb300._binding import testing_last_fma_variant
+    forward_check(case(300, 700, 40, C, dtype, tau=tau))
+    assert bool(testing_last_fma_variant() & 16) == folded, testing_last_fma_variant()
