@@ -792,7 +792,11 @@ struct OperandJob {
 // row (G = 1 up to D = 64, 2 up to 128, 4 up to 256), each lane converting
 // up to eight 16-byte vectors of its row, all loaded before any is
 // converted; so every lane of a warp does its own row's work (no lanes idle
-// during the norm split) and has up to 128 bytes of loads in flight.
+// during the norm split) and has up to 128 bytes of loads in flight.  The
+// block's output rows are staged in shared memory (a row stride of an odd
+// number of 16-byte vectors, so that the lanes' row stores do not share
+// banks) and then written as one contiguous run of 16-byte vectors, one per
+// thread and step, instead of one row per lane.
 // Blocks [0, blocks0) of grid row b convert rows of job j0 of problem b,
 // the rest those of j1 (the keys, when they are not the queries), so that
 // both arrays of every problem take one launch; a block never straddles
@@ -814,6 +818,7 @@ operand_vec_kernel(const OperandJob j0, const OperandJob j1, unsigned blocks0, i
     }
     constexpr int SLOTS = kOperandVecThreads / G;   // rows of a block
     __shared__ uint4 smean[kOperandMaxCols / 8];
+    extern __shared__ uint4 staged[];                // SLOTS rows of each output
     const int b = blockIdx.y;                        // problem of the batch
     const bool second = blockIdx.x >= blocks0;
     const OperandJob j = second ? j1 : j0;
@@ -844,11 +849,29 @@ operand_vec_kernel(const OperandJob j0, const OperandJob j1, unsigned blocks0, i
     const __half* vw = (wk && j.vw && i < rows)
                            ? static_cast<const __half*>(j.vw) + static_cast<int64_t>(b) * rows + i
                            : nullptr;
+    const int nv = Dp / 8;                           // 16-byte vectors per output row
+    const int sv = nv | 1;                           // staged row stride (odd)
+    uint4* stage_q = staged;
+    uint4* stage_k = staged + (wq ? SLOTS * sv : 0);
     const float n = operand_row<T, AUG, G>(
         in, smean, vi, in_pad, i < rows, D, Dp, nt, F, half_c, pad_value,
-        wq ? static_cast<T*>(j.out_q) + row * Dp : nullptr,
-        wk ? static_cast<T*>(j.out_k) + row * Dp : nullptr, cf, vw);
+        wq ? reinterpret_cast<T*>(stage_q + slot * sv) : nullptr,
+        wk ? reinterpret_cast<T*>(stage_k + slot * sv) : nullptr, cf, vw);
     if (!AUG && in_pad && vi == 0) j.nrm[row] = n;
+    __syncthreads();
+    // The block's rows [i0, i0 + nrows) are consecutive output rows.
+    const int i0 = blk * SLOTS;
+    const int nrows = min(SLOTS, rows_pad - i0);
+    const int total = nrows * nv;
+    const int64_t base = (static_cast<int64_t>(b) * rows_pad + i0) * Dp;
+    uint4* gq = wq ? reinterpret_cast<uint4*>(static_cast<T*>(j.out_q) + base) : nullptr;
+    uint4* gk = wk ? reinterpret_cast<uint4*>(static_cast<T*>(j.out_k) + base) : nullptr;
+    for (int u = threadIdx.x; u < total; u += kOperandVecThreads) {
+        const int r = u / nv;
+        const int s = r * sv + (u - r * nv);
+        if (wq) gq[u] = stage_q[s];
+        if (wk) gk[u] = stage_k[s];
+    }
 }
 
 template <typename T, bool AUG>
@@ -873,17 +896,30 @@ cudaError_t operand_typed(const OperandJob& j0, const OperandJob* j1, int D, int
         const int64_t b1 = j1 ? (j1->rows_pad + per_block - 1) / per_block : 0;
         if (b0 + b1 == 0 || batch == 0) return cudaSuccess;
         const unsigned op_blocks = static_cast<unsigned>(b0 + b1);
+        // Staged output rows: one or two outputs per job (AUG with q = k
+        // writes both layouts of the same rows).
+        auto nout = [](const OperandJob* j) {
+            return j ? (AUG ? (j->out_q ? 1 : 0) + (j->out_k ? 1 : 0) : 1) : 0;
+        };
+        const size_t smem = static_cast<size_t>(std::max(nout(&j0), nout(j1))) * per_block *
+                            ((Dp / 8) | 1) * 16;
         auto go = [&](auto kern) {
+            cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                                 static_cast<int>(smem));
+            if (e != cudaSuccess) return e;
             launch_kernel(kern, dim3(op_blocks + (vf_rec ? 1u : 0u), static_cast<unsigned>(batch)),
-                          kOperandVecThreads, 0, s, j0, j1 ? *j1 : none, static_cast<unsigned>(b0),
+                          kOperandVecThreads, smem, s, j0, j1 ? *j1 : none, static_cast<unsigned>(b0),
                           D, Dp, nt, F, mu, half_c, pad_value, cf, op_blocks, vf_rec, vf_tiles);
+            return cudaSuccess;
         };
         if (flags_done) *flags_done = vf_rec != nullptr;
+        cudaError_t e;
         switch (G) {
-            case 1: go(operand_vec_kernel<T, AUG, 1>); break;
-            case 2: go(operand_vec_kernel<T, AUG, 2>); break;
-            default: go(operand_vec_kernel<T, AUG, 4>); break;
+            case 1: e = go(operand_vec_kernel<T, AUG, 1>); break;
+            case 2: e = go(operand_vec_kernel<T, AUG, 2>); break;
+            default: e = go(operand_vec_kernel<T, AUG, 4>); break;
         }
+        if (e != cudaSuccess) return e;
         note_launches(1);
         return cudaGetLastError();
     }
