@@ -73,8 +73,10 @@ typedef enum { GS_PATH_AUTO = 0, GS_PATH_TENSOR = 1, GS_PATH_SIMT = 2 } gs_path;
  *                     the MMA type (the overflow/cancellation safeguard of
  *                     Remark 2, Sec. 2); 0: use the raw points.
  *  split_n         number of key splits per row tile (0: chosen from the
- *                  SM count; for C <= 4 one persistent block per SM takes an
- *                  equal run of (row tile, key tile) pairs); partial sums
+ *                  SM count; on the FMA-pipe kernel (C <= 2, or C <= 4
+ *                  below 2^28 pairs or with rows too wide for the augmented
+ *                  layout) one persistent block per SM takes an equal run
+ *                  of (row tile, key tile) pairs); partial sums
  *                  over splits are added in a fixed order, so results are
  *                  deterministic for a fixed split and GPU.
  *  workspace       caller-owned device buffer of workspace_bytes bytes

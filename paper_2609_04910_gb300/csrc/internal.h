@@ -43,6 +43,9 @@ cudaError_t launch_kernel(void (*kern)(K...), dim3 grid, dim3 block, size_t smem
 // Largest value-channel count evaluated on the FMA pipe (the P.v product of
 // tc_gauss_fma.cu); more channels use the two-MMA kernel of tc_gauss.cu.
 constexpr int kFmaMaxChannels = 4;
+// Calls of at least this many pairs take the two-MMA kernel for three or
+// four channels when the augmented rows fit (plan_tensor, tc_gauss.cu).
+constexpr int64_t kTwoMmaMinPairs = int64_t(1) << 28;
 
 // Workspace plan of the tensor-core path.  All offsets are bytes from the
 // workspace base and are 1024-byte aligned.

@@ -701,12 +701,23 @@ bool plan_tensor(InType t, int64_t M, int64_t N, int64_t D, int64_t C, bool grad
     // columns it takes the augmented operands (q^ in shared memory, norms
     // folded into the MMA).
     const int dp_aug = static_cast<int>((D + 2 * aug_norm_terms(t) + 15) / 16 * 16);
+    // Three or four channels: on the FMA pipe their P.v costs the exponent
+    // warps more than a second MMA costs the tensor cores, once a call is
+    // large enough to repay the two-MMA path's value preparation (one
+    // GB300, whole calls, 65536^2 pairs: D = 32, C = 4 1.16 ms on the FMA
+    // kernel against 0.70 ms for C = 5 on the two-MMA kernel; D = 64, C = 3
+    // and 4 0.94 and 1.16 against 0.87 ms).  Not with rows too wide for the
+    // augmented layout (q^ in tensor memory: at D = 256, C = 4 the FMA
+    // kernel took 6.4 ms against 12.8 ms for C = 5), nor for batches of
+    // problems (their one-launch path) or the MMD^2 upper triangle.
+    const bool channels_on_mma = p->Cv >= 3 && batch == 1 && !tri && dp_aug <= kAugMaxDp &&
+                                 M * N >= kTwoMmaMinPairs;
     if (p->tf) {
         p->fma = true;
     } else {
         p->aug = !grad && p->Cv <= kFmaMaxChannels && dp_aug <= kAugMaxDp;
         const int dp_fma = p->aug ? dp_aug : p->Dp;
-        p->fma = !grad && p->Cv <= kFmaMaxChannels &&
+        p->fma = !grad && p->Cv <= kFmaMaxChannels && !channels_on_mma &&
                  plan_fma_kernel(dp_fma, static_cast<int>(p->Cv), p->aug, false, &nq, &fma_stages,
                                  &fma_smem);
         if (!p->fma) p->aug = false;

@@ -3,7 +3,8 @@ layouts, each side of every switch against the float64 oracle.
 
 Switches (plan_tensor / plan_simt): augmented operands of the FMA kernel
 (fp16 D + 4 <= 128, bf16 D + 6 <= 128) versus q^ in TMEM; FMA kernel
-(C <= 4) versus two-MMA kernel; augmented two-MMA operands
+(C <= 4) versus two-MMA kernel, and for three or four channels on
+augmented rows the call size (2^28 pairs); augmented two-MMA operands
 (Dp_aug + Cp <= 128); 128- versus 64-key tiles (Cp <= 128); early S
 release (four or more stages) versus one MMA warp; gradient channels in one
 launch (D + 1 <= 256) versus two; fp32 register tiles of 16 / 32 / 64 / 128
@@ -40,6 +41,26 @@ def test_fma_augmented_switch(D, dtype, C):
 @pytest.mark.parametrize("N", [127, 128, 129])
 def test_fma_two_mma_switch(C, N):
     forward_check(case(140, N, 40, C, "fp16"))
+
+
+@pytest.mark.parametrize("C", [2, 3, 4])
+def test_three_and_four_channels_switch_kernels_at_2_28_pairs(C):
+    """From 2^28 pairs a single call with three or four channels on
+    augmented rows takes the two-MMA kernel (its value preparation adds
+    launches), below it and with two channels the FMA kernel: sampled rows
+    of both sides against the oracle."""
+    import numpy as np
+    import paper_2609_04910_gb300 as gs
+    rows = np.arange(0, 16384, 61)
+    launches = []
+    for N in (16383, 16384):
+        before = gs.gauss_sum_kernel_launches()
+        forward_check(case(16384, N, 64, C, "fp16"), rows=rows)
+        launches.append(gs.gauss_sum_kernel_launches() - before)
+    if C == 2:
+        assert launches[1] == launches[0]
+    else:
+        assert launches[1] > launches[0]
 
 
 @pytest.mark.parametrize("D,C", [(64, 48), (64, 49), (60, 64), (61, 64)])
