@@ -252,7 +252,12 @@ def main_kernel_name(w):
         # fp32 forward sums with C <= 4, D <= 32 from 2^25 pairs: 3xTF32 variant.
         tf32 = not w.grad and w.C <= 4 and w.D <= 32 and w.M * w.N >= 2 ** 25
         return "tc_gauss_fma_kernel" if tf32 else "simt_gauss_kernel"
-    return "tc_gauss_fma_kernel" if (not w.grad and w.C <= 4) else "tc_gauss_kernel"
+    if w.grad or w.C > 4:
+        return "tc_gauss_kernel"
+    # Three or four channels on augmented rows (D + 4 <= 128 for fp16, + 6
+    # for bf16) go to the two-MMA kernel from 2^28 pairs.
+    aug = w.D + (4 if w.dtype == "fp16" else 6) <= 128
+    return "tc_gauss_kernel" if (w.C >= 3 and aug and w.M * w.N >= 2 ** 28) else "tc_gauss_fma_kernel"
 
 
 def profiled_traffic(w):
