@@ -6,9 +6,13 @@
 // Phi(q_m, k_n) = 2^(c S + A_m + B_n) (the exponent is <= 0, so no running
 // maximum is needed; see tc_gauss.cu) and accumulate sum_n Phi v_n in fp32
 // on the FMA pipe.  With augmented operands (prep.cu) the MMA already adds
-// the norm terms, S = -||q^ - k^||^2 / 2, and Phi = 2^(c S).  For C <= 4
-// this costs fewer issue slots than a second MMA with N = 16, and it keeps
-// kernel values and values in fp32.
+// the norm terms, S = -||q^ - k^||^2 / 2, and Phi = 2^(c S).  For one or
+// two channels this costs fewer issue slots than a second MMA with N = 16,
+// and it keeps kernel values and values in fp32; three or four channels
+// come here for calls below 2^28 pairs and for rows too wide for the
+// augmented layout (larger calls of three or four channels on augmented
+// rows run faster on the two-MMA kernel, whose value preparation they
+// repay).
 //
 // Layout choices:
 //   * A CTA owns two query tiles (256 rows), which halves the L2 -> shared
