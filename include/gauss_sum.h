@@ -245,7 +245,12 @@ const char* gauss_sum_status_string(gs_status status);
  *  - Calls that need more scratch than the array holds return
  *    GS_ERR_UNSUPPORTED (see gauss_sum_last_error) without any GPU work;
  *    the M = N = 65536, D = 64, C = 1 fp16 MMD workload fits (it needs
- *    21 MiB).
+ *    21 MiB).  The scratch a call needs is that of the kernel gauss_sum
+ *    would run: calls of 2^28 or more pairs with three or four channels
+ *    on rows of D + 4 <= 128 (fp16; D + 6 for bf16) take the two-MMA
+ *    kernel, whose transposed values and per-split partial sums need more
+ *    than the FMA-pipe kernel that smaller calls use
+ *    (gauss_sum_workspace_size gives the figure).
  *  - The first call on a device looks up the array's device address
  *    (cudaGetSymbolAddress with that device current) and keeps it for the
  *    life of the process; make that first call before any stream capture.
